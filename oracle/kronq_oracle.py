@@ -1,0 +1,281 @@
+"""Plain float64 CPU oracle of the KronQ per-layer quantization path.
+
+TEST INFRASTRUCTURE ONLY. This module exists to check the CUDA library; only the tests,
+the smoke check and the benchmark's CPU-baseline leg may import it. The product path
+never calls it, and it shares no code with the CUDA kernels.
+
+It follows "KronQ: LLM Quantization via Kronecker-Factored Hessian":
+  * Kronecker factors          Sec. 2.1 Eq. (ptq_obj), Sec. 3.1 Eq. (kfac), Algorithm 1
+  * bidirectional rescaling    Sec. 3.2 Eq. (rescale), Algorithm 1
+  * randomized Hadamard (BiIP) Sec. 3.2 Eq. (biip), Algorithm 1
+  * damping, inverse Cholesky  Algorithm 2, Proposition 1
+  * column-wise OBS sweep      Sec. 2.1 Eq. (obs_update), Algorithm 2 (GPTQ mode, P = 0)
+  * revert and proxy loss      Algorithm 2, Sec. 3.1 Eq. (kron_obj), Theorem 1
+  * sensitivity traces         Sec. 3.3 Eq. (sensitivity)
+Tokens are stored as rows here (X is T x d_in), so the paper's X X^T is X^T X.
+
+Readings of points the paper leaves open (all listed in the design notes):
+  * factors are raw sums over tokens (no 1/T);
+  * the rotations are V = H_n diag(sigma_V) / sqrt(n) with H_n Sylvester for n = 2^k and
+    H_28 (Paley construction II, q = 13) Kronecker H_{2^k} for n = 28 * 2^k;
+  * damping adds damp * mean(diag) to the rescaled, rotated H_X;
+  * the update row of Algorithm 2 is row j of R = L^T, H^-1 = R^T R (R upper);
+  * the quantizer is the asymmetric min-max grid of GPTQ/GPTAQ with round-half-even;
+  * per-row grids come from the whole rotated row before the sweep; group grids
+    (group == block) from the current, compensated block at block start;
+  * the per-column loss is sum over rows of E_j^2 (no 1/2).
+"""
+from __future__ import annotations
+
+import numpy as np
+
+__all__ = [
+    "accum_factor", "sylvester", "paley28", "hadamard_matrix", "rht_matrix",
+    "biip_scales", "biip", "damp", "inverse_cholesky_upper", "lower_factor",
+    "quant_params", "quantize", "obs_sweep", "dequant", "revert", "proxy_loss",
+    "traces", "pipeline",
+]
+
+
+# ----------------------------------------------------------------------------------
+# Stage 1: Kronecker factors (Eq. ptq_obj: H_X = X X^T; Eq. kfac: H_G = E[g g^T];
+# Algorithm 1, "online statistics").
+# ----------------------------------------------------------------------------------
+def accum_factor(A: np.ndarray) -> np.ndarray:
+    """H = A^T A for A [T, d] with tokens as rows, in float64 (a library matmul)."""
+    A = np.asarray(A, dtype=np.float64)
+    return A.T @ A
+
+
+# ----------------------------------------------------------------------------------
+# Randomized Hadamard transforms (Eq. biip; Algorithm 1 "sample random Hadamard").
+# ----------------------------------------------------------------------------------
+def sylvester(n: int) -> np.ndarray:
+    """Sylvester Hadamard matrix of order n = 2^k (H_2 = [[1, 1], [1, -1]], H_2n = H_2 (x) H_n)."""
+    if n < 1 or n & (n - 1):
+        raise ValueError(f"{n} is not a power of two")
+    h = np.ones((1, 1), dtype=np.int64)
+    while h.shape[0] < n:
+        h = np.block([[h, h], [h, -h]])
+    return h
+
+
+def paley28() -> np.ndarray:
+    """Hadamard matrix of order 28 by Paley's second construction with q = 13.
+
+    chi is the quadratic character of GF(13); the Jacobsthal matrix Q[i, j] = chi(j - i)
+    is symmetric because 13 = 1 (mod 4). The conference matrix C = [[0, 1^T], [1, Q]] of
+    order 14 is expanded entry by entry: 0 -> [[1, -1], [-1, -1]], +-1 -> +-[[1, 1], [1, -1]].
+    """
+    q = 13
+    squares = {(x * x) % q for x in range(1, q)}
+
+    def chi(a: int) -> int:
+        a %= q
+        return 0 if a == 0 else (1 if a in squares else -1)
+
+    C = np.zeros((q + 1, q + 1), dtype=np.int64)
+    C[0, 1:] = 1
+    C[1:, 0] = 1
+    for i in range(q):
+        for j in range(q):
+            C[1 + i, 1 + j] = chi(j - i)
+    zero_blk = np.array([[1, -1], [-1, -1]], dtype=np.int64)
+    one_blk = np.array([[1, 1], [1, -1]], dtype=np.int64)
+    H = np.zeros((2 * (q + 1), 2 * (q + 1)), dtype=np.int64)
+    for i in range(q + 1):
+        for j in range(q + 1):
+            H[2 * i:2 * i + 2, 2 * j:2 * j + 2] = zero_blk if C[i, j] == 0 else C[i, j] * one_blk
+    return H
+
+
+def hadamard_matrix(n: int) -> np.ndarray:
+    """H_n for n = 2^k (Sylvester) or n = 28 * 2^k (H_28 (x) H_{2^k}, index a * 2^k + b)."""
+    if n >= 1 and n & (n - 1) == 0:
+        return sylvester(n)
+    if n % 28 == 0 and (n // 28) & (n // 28 - 1) == 0:
+        return np.kron(paley28(), sylvester(n // 28))
+    raise ValueError(f"no Hadamard construction for n = {n}")
+
+
+def rht_matrix(n: int, sign: np.ndarray) -> np.ndarray:
+    """Randomized Hadamard transform V = H_n diag(sigma) / sqrt(n) (orthogonal)."""
+    sign = np.asarray(sign, dtype=np.float64).reshape(-1)
+    assert sign.shape == (n,)
+    return hadamard_matrix(n).astype(np.float64) * sign[None, :] / np.sqrt(n)
+
+
+# ----------------------------------------------------------------------------------
+# Stage 2: bidirectional incoherence processing (Eq. rescale, Eq. biip, Algorithm 1).
+# ----------------------------------------------------------------------------------
+def biip_scales(W: np.ndarray, HX: np.ndarray, HG: np.ndarray):
+    """S_X = (diag(H_X) / diag(W^T W))^(1/4), S_G = (diag(H_G) / diag(W W^T))^(1/4).
+
+    A channel whose Hessian diagonal or weight norm is zero gets scale 1 (reading of a
+    case the paper does not discuss).
+    """
+    W = np.asarray(W, dtype=np.float64)
+    a = np.sum(W * W, axis=0)          # ||W_{:,j}||^2, j over d_in
+    r = np.sum(W * W, axis=1)          # ||W_{i,:}||^2, i over d_out
+    hx = np.diag(HX).astype(np.float64)
+    hg = np.diag(HG).astype(np.float64)
+    with np.errstate(divide="ignore", invalid="ignore"):
+        sx = np.where((hx > 0) & (a > 0), (hx / a) ** 0.25, 1.0)
+        sg = np.where((hg > 0) & (r > 0), (hg / r) ** 0.25, 1.0)
+    return sx, sg
+
+
+def biip(W, HX, HG, sign_u, sign_v):
+    """Algorithm 1 without the drift statistic (X-tilde = X):
+    W <- S_G W S_X; H_X <- S_X^-1 H_X S_X^-1; H_G <- S_G^-1 H_G S_G^-1;
+    W <- U W V^T; H_X <- V H_X V^T; H_G <- U H_G U^T (dense products)."""
+    W = np.asarray(W, dtype=np.float64)
+    HX = np.asarray(HX, dtype=np.float64)
+    HG = np.asarray(HG, dtype=np.float64)
+    d_out, d_in = W.shape
+    sx, sg = biip_scales(W, HX, HG)
+    Ws = sg[:, None] * W * sx[None, :]
+    HXs = HX / sx[:, None] / sx[None, :]
+    HGs = HG / sg[:, None] / sg[None, :]
+    U = rht_matrix(d_out, sign_u)
+    V = rht_matrix(d_in, sign_v)
+    return {"W": U @ Ws @ V.T, "HX": V @ HXs @ V.T, "HG": U @ HGs @ U.T,
+            "s_x": sx, "s_g": sg, "U": U, "V": V}
+
+
+# ----------------------------------------------------------------------------------
+# Stage 3: damping and inverse Cholesky (Algorithm 2; Proposition 1 names L with
+# H_X^-1 = L L^T).
+# ----------------------------------------------------------------------------------
+def damp(H: np.ndarray, lam: float) -> np.ndarray:
+    """H + lam * mean(diag(H)) * I."""
+    H = np.asarray(H, dtype=np.float64)
+    return H + lam * np.mean(np.diag(H)) * np.eye(H.shape[0])
+
+
+def inverse_cholesky_upper(Hd: np.ndarray) -> np.ndarray:
+    """R upper triangular with positive diagonal and Hd^-1 = R^T R, by the textbook
+    route: a library inverse followed by a library Cholesky."""
+    Hinv = np.linalg.inv(np.asarray(Hd, dtype=np.float64))
+    Hinv = 0.5 * (Hinv + Hinv.T)
+    return np.linalg.cholesky(Hinv).T
+
+
+def lower_factor(Hd: np.ndarray) -> np.ndarray:
+    """The paper's L = R^T (lower), H^-1 = L L^T; this is what kq_chol_inv returns."""
+    return inverse_cholesky_upper(Hd).T
+
+
+# ----------------------------------------------------------------------------------
+# Stage 4: quantizer and the blocked OBS sweep (Eq. obs_update, Algorithm 2 with P = 0).
+# ----------------------------------------------------------------------------------
+def quant_params(x: np.ndarray, bits: int):
+    """Asymmetric min-max grid per row of x: xmin = min(0, min x), xmax = max(0, max x),
+    (-1, 1) when both are 0; scale = (xmax - xmin) / (2^b - 1); zero = rint(-xmin/scale)."""
+    x = np.asarray(x, dtype=np.float64)
+    xmin = np.minimum(x.min(axis=-1), 0.0)
+    xmax = np.maximum(x.max(axis=-1), 0.0)
+    both = (xmin == 0) & (xmax == 0)
+    xmin = np.where(both, -1.0, xmin)
+    xmax = np.where(both, 1.0, xmax)
+    scale = (xmax - xmin) / (2 ** bits - 1)
+    zero = np.rint(-xmin / scale)
+    return scale, zero
+
+
+def quantize(w, scale, zero, bits):
+    """q = clamp(rint(w / scale) + zero, 0, 2^b - 1) (round half to even)."""
+    return np.clip(np.rint(np.asarray(w, np.float64) / scale) + zero, 0, 2 ** bits - 1)
+
+
+def obs_sweep(Wp: np.ndarray, R: np.ndarray, bits: int, group: int, block: int):
+    """Column-wise OBS sweep of Algorithm 2 in GPTQ mode (no P term).
+
+    For each block [i, e): for j in the block, quantize column j, E_j = (w_j - w^_j)/R_jj,
+    update the rest of the block by -E_j R[j, j+1:e]; then the lazy trailing update
+    W[:, e:] -= E_blk R[i:e, e:]. Returns codes, scale, zero (per row or per group)
+    and E for every column (the per-column loss is sum over rows of E^2), and pre_q,
+    the value of each column just before it is quantized.
+    """
+    W = np.array(Wp, dtype=np.float64, copy=True)
+    R = np.asarray(R, dtype=np.float64)
+    m, n = W.shape
+    if group not in (0, block):
+        raise ValueError("group must be 0 (per row) or equal to the block size")
+    ngroups = 1 if group == 0 else (n + group - 1) // group
+    codes = np.zeros((m, n), dtype=np.uint8)
+    scale = np.zeros((m, ngroups))
+    zero = np.zeros((m, ngroups))
+    E = np.zeros((m, n))
+    pre_q = np.zeros((m, n))
+    if group == 0:
+        s, z = quant_params(W, bits)
+        scale[:, 0], zero[:, 0] = s, z
+    for i in range(0, n, block):
+        e = min(i + block, n)
+        if group:
+            s, z = quant_params(W[:, i:e], bits)
+            scale[:, i // group], zero[:, i // group] = s, z
+        gidx = 0 if group == 0 else i // group
+        for j in range(i, e):
+            w = W[:, j]
+            pre_q[:, j] = w
+            q = quantize(w, scale[:, gidx], zero[:, gidx], bits)
+            codes[:, j] = q.astype(np.uint8)
+            what = scale[:, gidx] * (q - zero[:, gidx])
+            E[:, j] = (w - what) / R[j, j]
+            W[:, j + 1:e] -= np.outer(E[:, j], R[j, j + 1:e])
+        if e < n:
+            W[:, e:] -= E[:, i:e] @ R[i:e, e:]
+    return {"codes": codes, "scale": scale, "zero": zero, "E": E, "pre_q": pre_q}
+
+
+def dequant(codes, scale, zero, group: int) -> np.ndarray:
+    """Q' = scale * (q - zero) on the grid of each row or group."""
+    codes = np.asarray(codes, dtype=np.float64)
+    m, n = codes.shape
+    if group == 0:
+        return scale[:, :1] * (codes - zero[:, :1])
+    gi = np.arange(n) // group
+    return scale[:, gi] * (codes - zero[:, gi])
+
+
+def revert(Qp, s_x, s_g, U, V) -> np.ndarray:
+    """Algorithm 2's revert: Q <- U^T Q V, then Q <- S_G^-1 Q S_X^-1."""
+    Q = U.T @ np.asarray(Qp, dtype=np.float64) @ V
+    return Q / s_g[:, None] / s_x[None, :]
+
+
+def proxy_loss(W, What, HX, HG) -> float:
+    """tr(H_G dW H_X dW^T) with dW = W - W^ (Eq. kron_obj)."""
+    dW = np.asarray(W, np.float64) - np.asarray(What, np.float64)
+    return float(np.trace(np.asarray(HG, np.float64) @ dW @ np.asarray(HX, np.float64) @ dW.T))
+
+
+def traces(HX, HG, HXp, HGp) -> dict:
+    """Sensitivity s = tr(H_G) tr(H_X) (Eq. sensitivity), raw and after BiIP."""
+    tx, tg = float(np.trace(HX)), float(np.trace(HG))
+    txp, tgp = float(np.trace(HXp)), float(np.trace(HGp))
+    return {"trHX": tx, "trHG": tg, "s": tx * tg, "trHX_post": txp, "trHG_post": tgp,
+            "s_post": txp * tgp}
+
+
+def pipeline(X, G, W, sign_u, sign_v, bits: int, group: int, block: int = 128,
+             lam: float = 0.01) -> dict:
+    """Algorithms 1 and 2 end to end (GPTQ mode, X-tilde = X), all in float64."""
+    HX = accum_factor(X)
+    HG = accum_factor(G)
+    b = biip(W, HX, HG, sign_u, sign_v)
+    Hd = damp(b["HX"], lam)
+    R = inverse_cholesky_upper(Hd)
+    sw = obs_sweep(b["W"], R, bits, group, block)
+    Qp = dequant(sw["codes"], sw["scale"], sw["zero"], group)
+    What = revert(Qp, b["s_x"], b["s_g"], b["U"], b["V"])
+    out = {"HX": HX, "HG": HG, "Wp": b["W"], "HXp": b["HX"], "HGp": b["HG"],
+           "s_x": b["s_x"], "s_g": b["s_g"], "Hd": Hd, "R": R, "L": R.T,
+           "What": What, "loss": proxy_loss(W, What, HX, HG),
+           "loss_rot": proxy_loss(b["W"], Qp, b["HX"], b["HG"]),
+           "col_loss": np.sum(sw["E"] ** 2, axis=0)}
+    out.update(sw)
+    out.update(traces(HX, HG, b["HX"], b["HG"]))
+    return out

@@ -1,0 +1,385 @@
+"""Pins of the float64 oracle against facts the paper and mathematics fix.
+
+None of these compares the oracle with itself: each check is a brute-force sum, a
+closed form, an identity from the paper (Theorem 1, Proposition 1, Proposition 2's
+equality case, the LDL identity of Proposition 2's proof), a hand-derived worked example
+or a special case that reduces to plain rounding.
+"""
+import json
+import os
+
+import numpy as np
+import pytest
+
+import kqsynth
+from oracle import kronq_oracle as ref
+from oracle import obs_sweep_fp32
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _rng(seed):
+    return np.random.default_rng(seed)
+
+
+# ---------------------------------------------------------------- Kronecker factors
+def test_factor_brute_force_integers():
+    """H = sum_t x_t x_t^T (Eq. ptq_obj with tokens as rows), by Python integer loops."""
+    rng = _rng(1)
+    T, d = 37, 6
+    A = rng.integers(-9, 10, size=(T, d))
+    H = ref.accum_factor(A.astype(np.float64))
+    brute = [[0] * d for _ in range(d)]
+    for t in range(T):
+        for i in range(d):
+            for j in range(d):
+                brute[i][j] += int(A[t, i]) * int(A[t, j])
+    assert np.array_equal(H, np.array(brute, dtype=np.float64))
+
+
+def test_factor_bf16_exact_and_trace():
+    """bf16 products are exact in fp64; tr(A^T A) = ||A||_F^2 summed entry by entry."""
+    cfg = kqsynth.CONFIGS["tiny256"].replace(d_in=16, d_out=8, T=64)
+    X = kqsynth.activations(cfg).astype(np.float64)
+    H = ref.accum_factor(X)
+    tr = 0.0
+    for v in X.ravel():
+        tr += float(v) * float(v)
+    assert np.isclose(np.trace(H), tr, rtol=1e-14)
+    # additivity over token chunks (streamed accumulation)
+    parts = sum(ref.accum_factor(X[t:t + 16]) for t in range(0, 64, 16))
+    assert np.allclose(parts, H, rtol=1e-14, atol=0)
+
+
+# ---------------------------------------------------------------- Hadamard / RHT
+@pytest.mark.parametrize("n", [1, 2, 4, 8, 64, 256, 28, 56, 112, 896])
+def test_hadamard_orthogonal_symmetric(n):
+    H = ref.hadamard_matrix(n)
+    assert set(np.unique(H)) <= {-1, 1}
+    assert np.array_equal(H @ H.T, n * np.eye(n, dtype=np.int64))
+    assert np.array_equal(H, H.T)
+
+
+def test_sylvester_h2_and_recursion():
+    assert np.array_equal(ref.sylvester(2), np.array([[1, 1], [1, -1]]))
+    h4 = ref.sylvester(4)
+    for i in range(4):
+        for j in range(4):  # entry (i, j) of H_{2^k} is (-1)^{popcount(i & j)}
+            assert h4[i, j] == (-1) ** bin(i & j).count("1")
+
+
+def test_paley28_structure():
+    H = ref.paley28()
+    assert H.shape == (28, 28)
+    assert np.array_equal(H @ H.T, 28 * np.eye(28, dtype=np.int64))
+    # expanding the conference matrix's zero diagonal gives the block [[1,-1],[-1,-1]]
+    for i in range(14):
+        assert np.array_equal(H[2 * i:2 * i + 2, 2 * i:2 * i + 2], [[1, -1], [-1, -1]])
+
+
+def test_kron_index_layout():
+    """n = 28 * 2^k uses index a * 2^k + b: entry = H28[a, a'] * H_{2^k}[b, b']."""
+    H = ref.hadamard_matrix(28 * 4)
+    h28, h4 = ref.paley28(), ref.sylvester(4)
+    for (a, b, a2, b2) in [(0, 0, 0, 0), (3, 1, 5, 2), (27, 3, 1, 3), (13, 2, 13, 1)]:
+        assert H[a * 4 + b, a2 * 4 + b2] == h28[a, a2] * h4[b, b2]
+
+
+@pytest.mark.parametrize("n", [64, 112])
+def test_rht_rotate_unrotate(n):
+    rng = _rng(n)
+    sign = np.where(rng.random(n) < 0.5, -1, 1)
+    V = ref.rht_matrix(n, sign)
+    assert np.allclose(V @ V.T, np.eye(n), atol=1e-13)
+    W = rng.standard_normal((5, n))
+    assert np.allclose((W @ V.T) @ V, W, atol=1e-13)
+    assert np.allclose(np.linalg.norm(W @ V.T, axis=1), np.linalg.norm(W, axis=1))
+
+
+# ---------------------------------------------------------------- rescaling (Eq. rescale)
+def test_rescale_equalizes_norms_and_diagonals():
+    """With S_X = (h/a)^(1/4), the rescaled column energy a_j s_j^2 equals the rescaled
+    Hessian diagonal h_j / s_j^2 (= sqrt(h_j a_j)); any other exponent breaks this."""
+    cfg = kqsynth.CONFIGS["tiny256"].replace(d_in=32, d_out=24, T=256)
+    L = kqsynth.layer(cfg)
+    HX, HG = ref.accum_factor(L["X"]), ref.accum_factor(L["G"])
+    W = L["W"].astype(np.float64)
+    sx, sg = ref.biip_scales(W, HX, HG)
+    a, r = np.sum(W * W, 0), np.sum(W * W, 1)
+    assert np.allclose(a * sx ** 2, np.diag(HX) / sx ** 2, rtol=1e-12)
+    assert np.allclose(r * sg ** 2, np.diag(HG) / sg ** 2, rtol=1e-12)
+    assert np.allclose(a * sx ** 2, np.sqrt(np.diag(HX) * a), rtol=1e-12)
+
+
+def test_prop2_cauchy_schwarz_equality():
+    """Prop. 2: (sum h/s^2)(sum s^2 a) >= (sum sqrt(h a))^2 with equality at the S_G of
+    Eq. (rescale); the gain rho = (sum sqrt(h a))^2 / (sum h sum a) <= 1."""
+    rng = _rng(7)
+    h = np.exp(3 * rng.standard_normal(50))
+    W = rng.standard_normal((50, 40))
+    a = np.sum(W * W, 1)
+    HG = np.diag(h)
+    _, s = ref.biip_scales(W, np.eye(40), HG)
+    lhs = np.sum(h / s ** 2) * np.sum(s ** 2 * a)
+    assert np.isclose(lhs, np.sum(np.sqrt(h * a)) ** 2, rtol=1e-12)
+    s_half = (h / a) ** 0.5
+    assert np.sum(h / s_half ** 2) * np.sum(s_half ** 2 * a) > lhs * (1 + 1e-3)
+    rho = np.sum(np.sqrt(h * a)) ** 2 / (np.sum(h) * np.sum(a))
+    assert 0 < rho < 1
+
+
+def test_dead_channel_scale_is_one():
+    W = np.ones((4, 3))
+    W[:, 1] = 0.0
+    HX = np.diag([4.0, 2.0, 0.0])
+    sx, _ = ref.biip_scales(W, HX, np.eye(4))
+    assert sx[1] == 1.0 and sx[2] == 1.0 and np.isclose(sx[0], (4.0 / 4.0) ** 0.25)
+
+
+# ---------------------------------------------------------------- Theorem 1
+def test_theorem1_objective_invariance():
+    """tr(H_G dW H_X dW^T) is the same in the original and the BiIP space for any W^."""
+    cfg = kqsynth.CONFIGS["tiny256"].replace(d_in=56, d_out=32, T=512)
+    L = kqsynth.layer(cfg)
+    HX, HG = ref.accum_factor(L["X"]), ref.accum_factor(L["G"])
+    W = L["W"].astype(np.float64)
+    b = ref.biip(W, HX, HG, L["sign_u"], L["sign_v"])
+    rng = _rng(3)
+    Qp = b["W"] + 0.01 * rng.standard_normal(b["W"].shape)
+    What = ref.revert(Qp, b["s_x"], b["s_g"], b["U"], b["V"])
+    l_orig = ref.proxy_loss(W, What, HX, HG)
+    l_rot = ref.proxy_loss(b["W"], Qp, b["HX"], b["HG"])
+    assert np.isclose(l_orig, l_rot, rtol=1e-9)
+    # reverting the unquantized W' gives back W exactly
+    assert np.allclose(ref.revert(b["W"], b["s_x"], b["s_g"], b["U"], b["V"]), W, atol=1e-12)
+
+
+def test_proxy_loss_is_kronecker_quadratic():
+    """Eq. (kfac)/(kron_obj): vec(dW)^T (H_X kron H_G) vec(dW), vec stacking columns."""
+    rng = _rng(11)
+    m, n = 4, 5
+    A, B = rng.standard_normal((9, n)), rng.standard_normal((9, m))
+    HX, HG = A.T @ A, B.T @ B
+    W, What = rng.standard_normal((m, n)), rng.standard_normal((m, n))
+    v = (W - What).reshape(-1, order="F")
+    assert np.isclose(ref.proxy_loss(W, What, HX, HG), v @ np.kron(HX, HG) @ v, rtol=1e-12)
+
+
+def test_post_biip_traces():
+    """RHTs preserve the trace: tr(V S^-1 H S^-1 V^T) = sum_j h_j / s_j^2 = sum sqrt(h a)."""
+    cfg = kqsynth.CONFIGS["tiny256"].replace(d_in=64, d_out=28, T=300)
+    L = kqsynth.layer(cfg)
+    out = ref.pipeline(L["X"], L["G"], L["W"], L["sign_u"], L["sign_v"], 4, 0, 32)
+    W = L["W"].astype(np.float64)
+    a, r = np.sum(W * W, 0), np.sum(W * W, 1)
+    assert np.isclose(out["trHX_post"], np.sum(np.sqrt(np.diag(out["HX"]) * a)), rtol=1e-12)
+    assert np.isclose(out["trHG_post"], np.sum(np.sqrt(np.diag(out["HG"]) * r)), rtol=1e-12)
+    assert np.isclose(out["trHX"], np.sum(L["X"].astype(np.float64) ** 2), rtol=1e-12)
+    assert np.isclose(out["s_post"], out["trHX_post"] * out["trHG_post"])
+
+
+# ---------------------------------------------------------------- inverse Cholesky
+def _textbook_reverse_route(H):
+    """Pure-Python route independent of the library one: factor H = U U^T with U upper
+    (Cholesky from the bottom-right corner), then R = U^-1 by back substitution."""
+    n = len(H)
+    U = [[0.0] * n for _ in range(n)]
+    A = [list(map(float, row)) for row in H]
+    for k in range(n - 1, -1, -1):
+        U[k][k] = A[k][k] ** 0.5
+        for i in range(k):
+            U[i][k] = A[i][k] / U[k][k]
+        for i in range(k):
+            for j in range(k):
+                A[i][j] -= U[i][k] * U[j][k]
+    R = [[0.0] * n for _ in range(n)]
+    for j in range(n):           # solve U R = I column by column (R upper)
+        for i in range(j, -1, -1):
+            s = 1.0 if i == j else 0.0
+            for k in range(i + 1, j + 1):
+                s -= U[i][k] * R[k][j]
+            R[i][j] = s / U[i][i]
+    return np.array(R)
+
+
+def test_inverse_cholesky_routes_agree():
+    H = ref.damp(kqsynth.random_spd(12, seed=5), 0.01)
+    R = ref.inverse_cholesky_upper(H)
+    assert np.allclose(np.triu(R), R) and np.all(np.diag(R) > 0)
+    assert np.allclose(R.T @ R @ H, np.eye(12), atol=1e-9)
+    assert np.allclose(_textbook_reverse_route(H), R, rtol=1e-9, atol=1e-12)
+    assert np.array_equal(ref.lower_factor(H), R.T)
+
+
+def test_obs_row_is_inverse_of_remaining_block():
+    """Eq. (obs_update): R[p, p:]/R[p, p] = [H_F^-1]_{p, :}/[H_F^-1]_{pp}, F = {p, .., n-1}."""
+    H = ref.damp(kqsynth.random_spd(10, seed=9), 0.01)
+    R = ref.inverse_cholesky_upper(H)
+    for p in range(10):
+        HFi = np.linalg.inv(H[p:, p:])
+        assert np.allclose(R[p, p:] / R[p, p], HFi[0] / HFi[0, 0], rtol=1e-9, atol=1e-12)
+        assert np.isclose(R[p, p] ** 2, HFi[0, 0], rtol=1e-10)
+
+
+def test_damping_is_relative_to_mean_diagonal():
+    H = np.diag([1.0, 3.0])
+    assert np.allclose(ref.damp(H, 0.5), np.diag([2.0, 4.0]))
+
+
+# ---------------------------------------------------------------- quantizer
+def test_quantizer_grid_points_and_ties():
+    s, z = ref.quant_params(np.array([[-1.0, 0.5, 2.0]]), 2)  # scale = 3/3 = 1, zero = 1
+    assert s[0] == 1.0 and z[0] == 1.0
+    grid = s[0] * (np.arange(4) - z[0])
+    assert np.array_equal(ref.quantize(grid, s[0], z[0], 2), np.arange(4))
+    # ties to even: 0.5 -> 0, 1.5 -> 2, -0.5 -> -0; plus zero
+    assert np.array_equal(ref.quantize(np.array([0.5, 1.5, -0.5]), 1.0, 1.0, 2), [1, 3, 1])
+    # clamping and the all-zero row
+    assert ref.quantize(np.array([100.0]), 1.0, 1.0, 2)[0] == 3
+    s0, z0 = ref.quant_params(np.zeros((1, 4)), 3)
+    assert s0[0] == 2.0 / 7 and z0[0] == np.rint(7 / 2)
+    # min-max grid: dequantized error at most scale/2 inside the range
+    x = _rng(2).standard_normal((3, 50))
+    s, z = ref.quant_params(x, 4)
+    q = ref.quantize(x, s[:, None], z[:, None], 4)
+    assert np.all(np.abs(s[:, None] * (q - z[:, None]) - x) <= s[:, None] / 2 + 1e-12)
+
+
+# ---------------------------------------------------------------- OBS sweep
+def test_worked_example_golden():
+    g = json.load(open(os.path.join(GOLDEN, "obs_worked_2col.json")))
+    R = ref.inverse_cholesky_upper(np.array(g["H"]))
+    assert np.allclose(R, g["R"], rtol=1e-14)
+    sw = ref.obs_sweep(np.array(g["W"]), R, g["bits"], 0, 128)
+    assert sw["codes"].tolist() == g["codes"]
+    assert np.isclose(sw["scale"][0, 0], g["scale"]) and sw["zero"][0, 0] == g["zero"]
+    assert np.allclose(sw["pre_q"], g["pre_q"], rtol=1e-14)
+    assert np.allclose(sw["E"], g["E"], rtol=1e-13)
+    assert np.isclose(np.sum(sw["E"] ** 2), g["loss"], rtol=1e-13)
+    # the fp32-ordered C sweep gives the same codes on the same example
+    c = obs_sweep_fp32(np.array(g["W"], np.float32), R.T.astype(np.float32), g["bits"], 0, 128)
+    assert c["codes"].tolist() == g["codes"]
+
+
+@pytest.mark.parametrize("group,block", [(0, 16), (16, 16), (0, 128)])
+def test_identity_hessian_reduces_to_rtn(group, block):
+    """H = c I (R diagonal): no compensation, the sweep is round-to-nearest on the grid."""
+    rng = _rng(4)
+    W = rng.standard_normal((20, 48)) * 0.02
+    R = ref.inverse_cholesky_upper(2.5 * np.eye(48))
+    sw = ref.obs_sweep(W, R, 3, group, block)
+    if group == 0:
+        s, z = ref.quant_params(W, 3)
+        rtn = np.clip(np.rint(W / s[:, None]) + z[:, None], 0, 7)
+    else:
+        rtn = np.zeros_like(W)
+        for g0 in range(0, 48, group):
+            s, z = ref.quant_params(W[:, g0:g0 + group], 3)
+            rtn[:, g0:g0 + group] = np.clip(np.rint(W[:, g0:g0 + group] / s[:, None]) + z[:, None], 0, 7)
+    assert np.array_equal(sw["codes"], rtn.astype(np.uint8))
+    assert np.array_equal(sw["pre_q"], W)
+    c = obs_sweep_fp32(W.astype(np.float32), R.T.astype(np.float32), 3, group, block)
+    W32 = W.astype(np.float32)
+    if group == 0:
+        s32 = c["scale"][:, 0]
+        z32 = c["zero"][:, 0]
+        rtn32 = np.clip(np.rint(W32 / s32[:, None]) + z32[:, None], 0, 7)
+        assert np.array_equal(c["codes"], rtn32.astype(np.uint8))
+
+
+@pytest.mark.parametrize("group,block", [(0, 8), (8, 8), (0, 32)])
+def test_ldl_identity(group, block):
+    """Proof of Prop. 2 (e H e^T = eta D eta^T): sum_j sum_rows E_j^2 = tr(dW H dW^T)."""
+    cfg = kqsynth.CONFIGS["tiny256"].replace(d_in=32, d_out=16, T=200)
+    L = kqsynth.layer(cfg)
+    H = ref.damp(ref.accum_factor(L["X"]), 0.01)
+    R = ref.inverse_cholesky_upper(H)
+    W = L["W"].astype(np.float64)
+    sw = ref.obs_sweep(W, R, 2, group, block)
+    dW = W - ref.dequant(sw["codes"], sw["scale"], sw["zero"], group)
+    assert np.isclose(np.sum(sw["E"] ** 2), np.trace(dW @ H @ dW.T), rtol=1e-10)
+
+
+@pytest.mark.parametrize("block", [4, 32])
+def test_sequential_least_squares(block):
+    """Each compensated column equals the fp64 argmin of the quadratic with the earlier
+    columns fixed at their quantized values: w_F + (w_Q - q_Q) H_QF H_FF^-1."""
+    n = 20
+    H = ref.damp(kqsynth.random_spd(n, seed=13), 0.01)
+    R = ref.inverse_cholesky_upper(H)
+    W = _rng(5).standard_normal((6, n)) * 0.05
+    sw = ref.obs_sweep(W, R, 3, 0, block)
+    Q = ref.dequant(sw["codes"], sw["scale"], sw["zero"], 0)
+    for p in range(1, n):
+        Qi, F = slice(0, p), slice(p, n)
+        comp = W[:, F] + (W[:, Qi] - Q[:, Qi]) @ H[Qi, F] @ np.linalg.inv(H[F, F])
+        assert np.allclose(sw["pre_q"][:, p], comp[:, 0], rtol=1e-9, atol=1e-12)
+
+
+def test_prop1_hg_offdiagonal_does_not_change_codes():
+    """Prop. 1: H_G cancels in the update; only diag(H_G) reaches the sweep (through S_G)."""
+    cfg = kqsynth.CONFIGS["tiny256"].replace(d_in=32, d_out=28, T=400)
+    L = kqsynth.layer(cfg)
+    a = ref.pipeline(L["X"], L["G"], L["W"], L["sign_u"], L["sign_v"], 3, 0, 16)
+    HG = ref.accum_factor(L["G"])
+    HG2 = np.diag(np.diag(HG)) + 0.3 * (HG - np.diag(np.diag(HG)))
+    HX = ref.accum_factor(L["X"])
+    b = ref.biip(L["W"], HX, HG2, L["sign_u"], L["sign_v"])
+    sw = ref.obs_sweep(b["W"], ref.inverse_cholesky_upper(ref.damp(b["HX"], 0.01)), 3, 0, 16)
+    assert np.array_equal(sw["codes"], a["codes"])
+
+
+def test_greedy_sweep_bounded_by_brute_force():
+    """Tiny layers: the sweep is greedy, so its loss (which equals the quadratic of its
+    own codes) is bounded below by the optimum over all grid codes (brute force)."""
+    rng = _rng(21)
+    for trial in range(5):
+        n = 4
+        H = ref.damp(kqsynth.random_spd(n, seed=30 + trial), 0.01)
+        R = ref.inverse_cholesky_upper(H)
+        w = rng.standard_normal((1, n))
+        sw = ref.obs_sweep(w, R, 2, 0, 128)
+        s, z = sw["scale"][0, 0], sw["zero"][0, 0]
+        loss = np.sum(sw["E"] ** 2)
+        best = np.inf
+        for code in np.ndindex(*(4,) * n):
+            d = w[0] - s * (np.array(code) - z)
+            best = min(best, d @ H @ d)
+        d = w[0] - s * (sw["codes"][0] - z)
+        assert np.isclose(loss, d @ H @ d, rtol=1e-10)
+        assert best - 1e-12 <= loss
+
+
+# ---------------------------------------------------------------- fp32-ordered C sweep
+@pytest.mark.parametrize("group", [0, 32])
+def test_fp32_sweep_matches_fp64_off_ties(group):
+    """The fp32-ordered sweep agrees with the fp64 sweep wherever the decision is not
+    within fp32 noise of a rounding tie, and its losses agree to fp32 accuracy."""
+    n, m = 64, 40
+    H = ref.damp(kqsynth.random_spd(n, seed=17), 0.01)
+    R = ref.inverse_cholesky_upper(H)
+    R32 = R.astype(np.float32)
+    W32 = (_rng(8).standard_normal((m, n)) * 0.02).astype(np.float32)
+    s64 = ref.obs_sweep(W32.astype(np.float64), R32.astype(np.float64), 4, group, 32)
+    s32 = obs_sweep_fp32(W32, R32.T, 4, group, 32)
+    diff = s64["codes"] != s32["codes"]
+    # rows diverge after a flipped decision; the first flip in each row must be a near-tie
+    for r in np.nonzero(diff.any(1))[0]:
+        j = np.argmax(diff[r])
+        g = 0 if group == 0 else j // group
+        t = s64["pre_q"][r, j] / s64["scale"][r, g]
+        assert abs(abs(t - np.floor(t)) - 0.5) < 1e-3
+    assert diff.mean() < 0.02
+    assert np.isclose(np.sum(s32["E"].astype(np.float64) ** 2), np.sum(s64["E"] ** 2), rtol=1e-3)
+
+
+def test_fp32_sweep_row_subset():
+    n, m = 48, 12
+    H = ref.damp(kqsynth.random_spd(n, seed=3), 0.01)
+    Lt = ref.lower_factor(H).astype(np.float32)
+    W = (_rng(9).standard_normal((m, n)) * 0.02).astype(np.float32)
+    full = obs_sweep_fp32(W, Lt, 3, 16, 16)
+    rows = np.array([7, 0, 11])
+    part = obs_sweep_fp32(W, Lt, 3, 16, 16, rows=rows)
+    assert np.array_equal(part["codes"], full["codes"][rows])
+    assert np.array_equal(part["E"], full["E"][rows])
