@@ -1,0 +1,352 @@
+#!/usr/bin/env python
+"""Benchmark: one synthetic Llama-shaped linear layer through the KronQ per-layer path
+(factors -> BiIP rescale + RHT -> damped inverse Cholesky -> OBS sweep) per step.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--config q_proj_8b] [--impl ours|reference]
+
+Prints one JSON line. `value` is milliseconds per linear layer for the whole job (lower is
+better). Under torchrun each rank quantizes its own layer (the path has no cross-layer
+exchange: weak scaling, no collective on the data path); the timed region is bracketed by
+a barrier and a device synchronize on every rank and the slowest rank's time is used.
+`--impl reference` times the CPU oracle (float64 numpy + the fp32-ordered C sweep) on a
+bounded sample of the same workload and extrapolates to the same metric.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import kqsynth  # noqa: E402
+
+METRIC = "ms per linear layer (factors+rotate+chol+OBS sweep)"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--config", default="q_proj_8b", choices=sorted(kqsynth.CONFIGS))
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def workload_name(cfg) -> str:
+    return (f"{cfg.name}: W {cfg.d_out}x{cfg.d_in}, T={cfg.T} tokens, {cfg.bits}-bit "
+            f"{'per-row' if cfg.group == 0 else 'group ' + str(cfg.group)}, block {cfg.block}, "
+            f"damp {cfg.damp}")
+
+
+def config_dict(cfg) -> dict:
+    return {"workload": workload_name(cfg), "d_out": cfg.d_out, "d_in": cfg.d_in, "T": cfg.T,
+            "bits": cfg.bits, "group": cfg.group, "block": cfg.block, "damp": cfg.damp,
+            "l2": "inputs larger than L2 (X and G are T x d bf16, >= 1 GiB each); no flush"}
+
+
+def algorithmic_flops(cfg) -> dict:
+    return {"factor_x": cfg.T * cfg.d_in * (cfg.d_in + 1),
+            "factor_g": cfg.T * cfg.d_out * (cfg.d_out + 1),
+            "chol": 2 * cfg.d_in ** 3 / 3,
+            "sweep": cfg.d_out * cfg.d_in * max(cfg.d_in - cfg.block, 0)}
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    except (OSError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def syrk_traffic(cfg):
+    """DRAM bytes per SYRK launch from a committed ncu capture, if it was taken on the
+    current kernel source (else None)."""
+    src = os.path.join(ROOT, "paper_2607_07964_gb300", "csrc", "syrk.cu")
+    rec = os.path.join(ROOT, "profiles", "syrk_traffic.json")
+    try:
+        with open(rec) as f:
+            r = json.load(f)
+        h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        if r.get("syrk_cu_sha256_16") != h:
+            return None
+        per_token = r["dram_bytes_per_launch"] / r["T"]
+        if r.get("d") != cfg.d_in:
+            return None
+        return per_token * cfg.T
+    except (OSError, ValueError, KeyError):
+        return None
+
+
+# --------------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap,pci.bus_id")
+
+    def __init__(self, bus_id: str | None):
+        self.bus_id = (bus_id or "").lower()
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.out = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.out, stderr=subprocess.DEVNULL)
+        except (OSError, ValueError):
+            self.proc = None
+
+    def stop(self) -> dict | None:
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.out.close()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 8:
+                continue
+            if self.bus_id and not f[7].lower().endswith(self.bus_id[-12:]):
+                continue
+            try:
+                sm.append(float(f[0]))
+                mx.append(float(f[1]))
+            except ValueError:
+                continue
+            for k, n in enumerate(names):
+                if f[3 + k].lower() == "active":
+                    reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+# ---------------------------------------------------------------- CPU oracle timing
+def oracle_sample_ms(cfg, repeats: int = 1, T_s: int = 4096, f: int = 2, rows_s: int = 128) -> dict:
+    """Time the oracle on a bounded sample of the workload and extrapolate each stage to
+    the full layer by its cost model: the factors run on T_s of the T tokens at full width
+    (linear in tokens); BiIP, Cholesky and the fp32-ordered sweep run on a layer shrunk by
+    f in both dimensions (dense products and Cholesky cubic in the size; the sweep
+    proportional to rows x d_in^2, run on rows_s rows)."""
+    from oracle import kronq_oracle as ref
+    import oracle
+
+    T_s = min(cfg.T, T_s)
+    if min(cfg.d_in, cfg.d_out) < 256 * f:
+        f = 1
+    sub = cfg.replace(d_out=cfg.d_out // f, d_in=cfg.d_in // f, T=T_s)
+    rows_s = min(sub.d_out, rows_s)
+    L = kqsynth.layer(cfg.replace(T=T_s))
+    Ls = kqsynth.layer(sub)
+    stage = {"factors": [], "biip": [], "chol": [], "sweep": []}
+    for _ in range(repeats):
+        t0 = time.perf_counter()
+        HX = ref.accum_factor(L["X"])
+        HG = ref.accum_factor(L["G"])
+        t1 = time.perf_counter()
+        stage["factors"].append((t1 - t0) * cfg.T / T_s)
+        HXs, HGs = ref.accum_factor(Ls["X"]), ref.accum_factor(Ls["G"])
+        t1 = time.perf_counter()
+        b = ref.biip(Ls["W"], HXs, HGs, Ls["sign_u"], Ls["sign_v"])
+        t2 = time.perf_counter()
+        stage["biip"].append((t2 - t1) * f ** 3)
+        R = ref.inverse_cholesky_upper(ref.damp(b["HX"], cfg.damp))
+        t3 = time.perf_counter()
+        stage["chol"].append((t3 - t2) * f ** 3)
+        Wp = b["W"][:rows_s].astype("float32")
+        Lt = R.T.astype("float32")
+        t4 = time.perf_counter()
+        oracle.obs_sweep_fp32(Wp, Lt, cfg.bits, cfg.group, cfg.block)
+        t5 = time.perf_counter()
+        stage["sweep"].append((t5 - t4) * (cfg.d_out / rows_s) * f ** 2)
+        del HX, HG, HXs, HGs, b, R
+    per = {k: 1e3 * statistics.mean(v) for k, v in stage.items()}
+    return {"value": sum(per.values()), "unit": "ms", "cores": os.cpu_count(), "kind": "oracle",
+            "stages_ms": per,
+            "sample": (f"factors on {T_s} of {cfg.T} tokens at full width (x{cfg.T / T_s:g}); BiIP dense "
+                       f"products, Cholesky and fp32-ordered sweep ({rows_s} rows) on the "
+                       f"{sub.d_out}x{sub.d_in} layer (x{f}^3, x{f}^3, x{f}^2*{cfg.d_out / rows_s:g}); "
+                       f"{repeats} repeat(s), mean")}
+
+
+# --------------------------------------------------------------------- distributed
+def dist_setup(backend: str):
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if ws > 1:
+        import torch.distributed as dist
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group(backend=backend)
+    return ws, rank, local
+
+
+def run_reference(args):
+    ws, rank, _ = dist_setup("gloo")
+    cfg = kqsynth.CONFIGS[args.config]
+    if rank != 0:
+        return
+    small = dict(T_s=2048, f=4, rows_s=64)
+    for _ in range(args.warmup):
+        oracle_sample_ms(cfg, **small)
+    vals, last = [], None
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        last = oracle_sample_ms(cfg, **small)
+        vals.append(last["value"])
+    wall = time.perf_counter() - t0
+    v = statistics.mean(vals)
+    out = {"impl": "reference", "metric": METRIC, "value": v, "unit": "ms", "n_gpus": args.gpus,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": v, "higher_is_better": False,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": config_dict(cfg),
+           "cpu_baseline": {"value": v, "unit": "ms", "cores": last["cores"], "kind": "oracle",
+                            "sample": last["sample"], "stages_ms": last["stages_ms"]},
+           "e2e": {"value": v, "unit": "ms", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+           "wall_s": wall}
+    print(json.dumps(out), flush=True)
+
+
+def run_ours(args):
+    import torch
+
+    from paper_2607_07964_gb300 import build as kbuild
+    ws, rank, local = dist_setup("nccl")
+    kbuild.build()
+    from paper_2607_07964_gb300 import kronq as kq
+    from paper_2607_07964_gb300.pipeline import STAGES, LayerPipeline
+
+    torch.cuda.set_device(local)
+    dev = f"cuda:{local}"
+    cfg = kqsynth.CONFIGS[args.config].replace(seed=rank)
+    inp = kqsynth.device_layer(cfg, device=dev)
+    p = LayerPipeline(cfg.d_out, cfg.d_in, cfg.bits, cfg.group, cfg.block, cfg.damp, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def barrier():
+        if ws > 1:
+            torch.distributed.barrier()
+
+    for _ in range(args.warmup):
+        p.run(inp["X"], inp["G"], inp["W"], inp["sign_u"], inp["sign_v"], stream=stream)
+    p.check(stream)
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(len(STAGES) + 1)] for _ in range(args.steps)]
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(torch.cuda.get_device_properties(local).pci_bus_id if hasattr(
+        torch.cuda.get_device_properties(local), "pci_bus_id") else None)
+    barrier()
+    torch.cuda.synchronize()
+    sampler.start()
+    n0 = kq.launch_count()
+    t_start.record(stream)
+    for k in range(args.steps):
+        p.run(inp["X"], inp["G"], inp["W"], inp["sign_u"], inp["sign_v"], stream=stream, events=evs[k])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    launches = kq.launch_count() - n0
+    clocks = sampler.stop()
+    p.check(stream)
+    total_ms = t_start.elapsed_time(t_end)
+    if ws > 1:
+        t = torch.tensor([total_ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms = float(t.item())
+    stage_ms = {name: statistics.mean(evs[k][i].elapsed_time(evs[k][i + 1]) for k in range(args.steps))
+                for i, name in enumerate(STAGES)}
+    fl = algorithmic_flops(cfg)
+    tflops = {"factor_x": fl["factor_x"] / stage_ms["factor_x"] / 1e9,
+              "factor_g": fl["factor_g"] / stage_ms["factor_g"] / 1e9,
+              "chol": fl["chol"] / stage_ms["chol"] / 1e9,
+              "sweep_trailing": fl["sweep"] / stage_ms["sweep"] / 1e9}
+    peaks, peak_src = measured_peaks()
+    peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+    achieved = tflops["factor_x"]
+    traffic = syrk_traffic(cfg)
+    roofline = {"kernel": "syrk_tc_kernel (H_X = X^T X)", "bound": "tensor", "achieved": achieved,
+                "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak, "traffic": traffic,
+                "peak_source": f"{peak_src} bf16 dense burst",
+                "algorithmic_flops_per_launch": fl["factor_x"]}
+
+    e2e = None
+    if not args.no_e2e:
+        Xh = inp["X"].cpu().pin_memory()
+        Gh = inp["G"].cpu().pin_memory()
+        Wh = inp["W"].cpu().pin_memory()
+        suh, svh = inp["sign_u"].cpu().pin_memory(), inp["sign_v"].cpu().pin_memory()
+        ch = torch.empty(p.codes.shape, dtype=p.codes.dtype).pin_memory()
+        sh = torch.empty(p.scale.shape, dtype=p.scale.dtype).pin_memory()
+        zh = torch.empty(p.zero.shape, dtype=p.zero.dtype).pin_memory()
+        p.run_host(Xh, Gh, Wh, suh, svh, ch, sh, zh, stream=stream)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        barrier()
+        torch.cuda.synchronize()
+        e0.record(stream)
+        nin = nout = 0
+        for _ in range(args.steps):
+            nin, nout = p.run_host(Xh, Gh, Wh, suh, svh, ch, sh, zh, stream=stream)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        e_ms = e0.elapsed_time(e1)
+        if ws > 1:
+            t = torch.tensor([e_ms], device=dev)
+            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+            e_ms = float(t.item())
+        e2e = {"value": e_ms / (ws * args.steps), "unit": "ms", "h2d_bytes_per_step": nin,
+               "d2h_bytes_per_step": nout}
+
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        cpu = oracle_sample_ms(cfg, repeats=2)
+
+    if rank == 0:
+        out = {"metric": METRIC, "value": total_ms / (ws * args.steps), "unit": "ms", "n_gpus": ws,
+               "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
+               "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
+               "dtype": "bf16 products, f32 accumulate/arithmetic", "data": "synthetic",
+               "config": config_dict(cfg), "stages_ms": stage_ms, "tflops": tflops,
+               "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
+               "clocks": clocks}
+        print(json.dumps(out), flush=True)
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,210 @@
+/*
+ * libkronq -- the per-layer quantization path of KronQ ("KronQ: LLM Quantization via
+ * Kronecker-Factored Hessian") as a C ABI over hand-written CUDA kernels for sm_103a.
+ *
+ * One linear layer W [d_out x d_in] is processed in four stages:
+ *   1. Kronecker factors  H_X = X^T X, H_G = G^T G            (kq_accum_factor, kq_traces)
+ *   2. bidirectional incoherence processing (BiIP)            (kq_compute_scales,
+ *                                                              kq_rotate_in, kq_rotate_out)
+ *   3. damped inverse Cholesky                                (kq_chol_inv)
+ *   4. column-wise OBS sweep with b-bit asymmetric grids      (kq_obs_quantize)
+ * plus two check-only calls (kq_dequant_revert, kq_proxy_loss).
+ *
+ * Conventions shared by every call
+ *   - Tokens are rows: X is [T x d_in], G is [T x d_out]; the paper stacks tokens as
+ *     columns, so its X X^T is X^T X here.
+ *   - All pointers are DEVICE pointers owned by the caller unless stated otherwise. The
+ *     library allocates no memory; scratch space is passed in as `ws` with a size from
+ *     the matching *_workspace() query.
+ *   - Matrices are dense row-major. Only kq_accum_factor takes a leading dimension (for
+ *     its input); every other matrix is contiguous (leading dimension = row length).
+ *   - Every call is asynchronous on `stream` (NULL = the legacy default stream) and
+ *     returns a kq_status for errors detected on the host (bad arguments, launch
+ *     failures). Errors detected by kernels are written to the optional device word
+ *     `info` (first error wins) and read back with kq_check().
+ *   - bf16 inputs are passed as their 16-bit patterns (uint16_t).
+ *   - Supported rotation sizes are n = 2^k (0 <= k <= 15) and n = 28 * 2^k (2^k <= 1024).
+ */
+#ifndef KRONQ_H
+#define KRONQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define KQ_API __attribute__((visibility("default")))
+#else
+#define KQ_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t. */
+typedef struct CUstream_st* kq_stream_t;
+
+typedef enum kq_status {
+    KQ_OK = 0,
+    KQ_ERR_INVALID_ARG = 1,  /* null pointer, negative size, size mismatch, bad alignment */
+    KQ_ERR_UNSUPPORTED = 2,  /* dimension without a Hadamard construction, group not in {0, block} */
+    KQ_ERR_NOT_PD = 3,       /* non-positive pivot in kq_chol_inv (reported through `info`) */
+    KQ_ERR_CUDA = 4,         /* a CUDA runtime/driver call failed */
+    KQ_ERR_TIMEOUT = 5,      /* a kernel gave up a bounded wait (reported through `info`) */
+    KQ_ERR_WORKSPACE = 6     /* ws is NULL or smaller than the *_workspace() size */
+} kq_status;
+
+/* Text of the last host-side error of the calling thread ("" when none). */
+KQ_API const char* kq_last_error(void);
+/* Name of a status code. */
+KQ_API const char* kq_status_name(int status);
+/* Library version: major * 10000 + minor * 100 + patch. */
+KQ_API int kq_version(void);
+/* Number of kernels this library has launched in this process (all threads, all devices). */
+KQ_API uint64_t kq_launch_count(void);
+
+/*
+ * Synchronize `stream`, then read the device error word `info` (may be NULL) and map it:
+ * 0 -> KQ_OK, > 0 -> KQ_ERR_NOT_PD (the value is the 1-based index of the first
+ * non-positive pivot), < 0 -> the status -info. Resets *info to 0 when `reset` != 0.
+ * `pivot_out` (host, may be NULL) receives the raw word.
+ */
+KQ_API kq_status kq_check(int* info, int reset, int* pivot_out, kq_stream_t stream);
+
+/* ------------------------------------------------------------------------------------
+ * Stage 1: Kronecker factors.
+ * Paper: Sec. 2.1 Eq. (ptq_obj) defines H_X = X X^T; Sec. 3.1 Eq. (kfac) the factor pair
+ * H_X (x) H_G; Algorithm 1 computes H_X as an online statistic and loads a precomputed H_G.
+ *
+ * kq_accum_factor: H (+)= A^T A for A [T x d] bf16 (row t = token t, row stride `lda`
+ *   elements). The sum is raw (no 1/T). H is [d x d] fp32, full symmetric storage (both
+ *   triangles written). accumulate = 0 overwrites H, 1 adds to it (for token chunks
+ *   streamed through several calls). If `trace` (device double*) is non-NULL it receives
+ *   tr(H) of the resulting H, summed in fp64.
+ *   Products of bf16 values are exact in fp32; sums are fp32 with the tensor-core
+ *   accumulator drained into an fp32 running sum every `KQ_SYRK_CHUNK_TOKENS` tokens.
+ *   Requirements: A 16-byte aligned, lda % 8 == 0, lda >= d, T >= 0, 1 <= d <= 65536.
+ *   T == 0 gives H = 0 (accumulate = 0) or leaves H unchanged. `info` (nullable) receives
+ *   -KQ_ERR_TIMEOUT if a pipeline wait gave up.
+ * ---------------------------------------------------------------------------------- */
+#define KQ_SYRK_CHUNK_TOKENS 2048
+KQ_API kq_status kq_accum_factor(const uint16_t* A, int64_t T, int64_t d, int64_t lda, float* H,
+                          int accumulate, double* trace, int* info, kq_stream_t stream);
+
+/* ------------------------------------------------------------------------------------
+ * Stage 2: bidirectional incoherence processing.
+ * Paper: Sec. 3.2 Eq. (rescale) gives S_X = diag(H_X_jj / ||W_:,j||^2)^(1/4) and
+ * S_G = diag(H_G_ii / ||W_i,:||^2)^(1/4); Eq. (biip) the rotations W <- U W V^T,
+ * H_X <- V H_X V^T, H_G <- U H_G U^T with randomized Hadamard transforms; Algorithm 1
+ * applies the rescale first, then the rotations, then releases H_G.
+ *
+ * The randomized Hadamard transform of size n is V = H_n diag(sigma) / sqrt(n) with
+ * sigma in {-1, +1}^n (int8, caller-drawn) and H_n the Sylvester matrix for n = 2^k, or
+ * H_28 (x) H_{2^k} for n = 28 * 2^k, where H_28 is Paley's second construction over
+ * GF(13) and index j = a * 2^k + b (b fastest). H_n is symmetric, so V^-1 = V^T.
+ *
+ * kq_compute_scales: s_x [d_in] and s_g [d_out] (fp32) from the ORIGINAL W [d_out x d_in]
+ *   fp32 and the diagonals of the raw H_X [d_in x d_in] and H_G [d_out x d_out]. Norms are
+ *   summed in fp64; s = sqrt(sqrt(h / a)), and s = 1 when h == 0 or a == 0 (a dead
+ *   channel). Must run before either rotation. H_G may be NULL (then s_g = 1; the
+ *   one-sided variant).
+ *
+ * kq_traces: the sensitivity statistics of Sec. 3.3 Eq. (sensitivity), from the raw
+ *   factors' diagonals and the scales (call before the rotations overwrite H_X / H_G).
+ *   out [6] (device double): tr(H_X), tr(H_G), tr(H_X) tr(H_G), and the post-BiIP
+ *   tr(H_X'), tr(H_G'), tr(H_X') tr(H_G') with tr(H') = sum_j H_jj / s_j^2 (the rotations
+ *   preserve the trace).
+ *
+ * kq_rotate_in (input side, length d_in, sign_v = sigma_V):
+ *   dir = KQ_FWD: W <- (W S_X) V^T, and if H_X != NULL: H_X <- V S_X^-1 H_X S_X^-1 V^T.
+ *   dir = KQ_INV: W <- (W V) S_X^-1 (undoes the forward map; H_X untouched).
+ * kq_rotate_out (output side, length d_out, sign_u = sigma_U):
+ *   dir = KQ_FWD: W <- U (S_G W), and if H_G != NULL: H_G <- U S_G^-1 H_G S_G^-1 U^T.
+ *   dir = KQ_INV: W <- S_G^-1 (U^T W).
+ *   All in place, fp32. s_x / s_g may be NULL for a pure rotation (S = I).
+ *   Returns KQ_ERR_UNSUPPORTED if the length has no Hadamard construction.
+ * ---------------------------------------------------------------------------------- */
+#define KQ_FWD 0
+#define KQ_INV 1
+KQ_API kq_status kq_compute_scales(const float* W, int64_t d_out, int64_t d_in, const float* H_X,
+                            const float* H_G, float* s_x, float* s_g, kq_stream_t stream);
+KQ_API kq_status kq_traces(const float* H_X, const float* s_x, int64_t d_in, const float* H_G,
+                    const float* s_g, int64_t d_out, double* out, kq_stream_t stream);
+KQ_API kq_status kq_rotate_in(float* W, int64_t d_out, int64_t d_in, float* H_X, const float* s_x,
+                       const int8_t* sign_v, int dir, kq_stream_t stream);
+KQ_API kq_status kq_rotate_out(float* W, int64_t d_out, int64_t d_in, float* H_G, const float* s_g,
+                        const int8_t* sign_u, int dir, kq_stream_t stream);
+
+/* ------------------------------------------------------------------------------------
+ * Stage 3: damped inverse Cholesky.
+ * Paper: Algorithm 2 damps H_X <- H_X + lambda * mean(diag(H_X)) I and takes
+ * L = Inverse_Cholesky(H_X); Proposition 1 defines L by H_X^-1 = L L^T (L lower).
+ *
+ * kq_chol_inv: H [n x n] fp32 symmetric (read only; the lower triangle is used) ->
+ *   Lt [n x n] fp32, the lower-triangular L with (H + damp_rel * mean(diag H) I)^-1 = L L^T
+ *   and positive diagonal; the strict upper triangle of Lt is written with zeros. R = L^T
+ *   is the upper factor whose row j drives the OBS update of column j. Computed as the
+ *   Cholesky factorization of the index-reversed matrix followed by a triangular inverse
+ *   (2 n^3 / 3 flops), fp32.
+ *   On a non-positive pivot, *info (required for that report) receives the 1-based index
+ *   (in H's own indexing) of the failing pivot; Lt is then undefined. The caller may retry
+ *   with a larger damp_rel.
+ *   ws: kq_chol_inv_workspace(n) bytes.
+ * ---------------------------------------------------------------------------------- */
+KQ_API size_t kq_chol_inv_workspace(int64_t n);
+KQ_API kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, float* Lt, int* info, void* ws,
+                      size_t ws_bytes, kq_stream_t stream);
+
+/* ------------------------------------------------------------------------------------
+ * Stage 4: column-wise OBS sweep (GPTQ mode; the GPTAQ drift term P is zero).
+ * Paper: Sec. 2.1 Eq. (obs_update); Algorithm 2's inner column loop and lazy trailing
+ * update; Proposition 1 (H_G cancels, so the sweep reads only L).
+ *
+ * kq_obs_quantize: W [d_out x d_in] fp32 (the rotated, rescaled W'; destroyed), Lt from
+ *   kq_chol_inv. For each block of `block` columns and each column j of it:
+ *     q_j = clamp(rint(w_j / scale) + zero, 0, 2^bits - 1)        (round half to even)
+ *     E_j = (w_j - scale * (q_j - zero)) / R_jj,  w_k -= E_j R_jk for k in (j, block end)
+ *   then W[:, block end:] -= E_block R[block, block end:].
+ *   Grid (asymmetric min-max): xmin = min(0, min x), xmax = max(0, max x), (-1, 1) if both
+ *   are 0; scale = (xmax - xmin) / (2^bits - 1); zero = rint(-xmin / scale).
+ *   group = 0: one grid per row from the whole row before the sweep (scale/zero [d_out]).
+ *   group = block: one grid per row and block from the current, compensated block at
+ *   block start (scale/zero [d_out x ceil(d_in / block)]).
+ *   Outputs: codes [d_out x d_in] uint8; scale fp32 and zero int32 as above; col_loss
+ *   [d_in] (nullable) = sum over rows of E_j^2; pre_q [d_out x d_in] (nullable) = the value
+ *   w_j just before it was quantized.
+ *   Every fp32 operation and its order are fixed (IEEE division, rintf, one fmaf per
+ *   intra-block update; trailing update as acc = fmaf(E_k, R_kc, acc) over ascending k,
+ *   then w_c - acc), so results are reproducible bit for bit.
+ *   Requirements: 1 <= bits <= 8, block == 128, group in {0, block}.
+ *   ws: kq_obs_quantize_workspace(d_out, d_in, block) bytes.
+ * ---------------------------------------------------------------------------------- */
+KQ_API size_t kq_obs_quantize_workspace(int64_t d_out, int64_t d_in, int block);
+KQ_API kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, const float* Lt, int bits,
+                          int group, int block, uint8_t* codes, float* scale, int32_t* zero,
+                          float* col_loss, float* pre_q, void* ws, size_t ws_bytes,
+                          kq_stream_t stream);
+
+/* ------------------------------------------------------------------------------------
+ * Check-only calls (not part of the timed path).
+ *
+ * kq_dequant_revert: Algorithm 2's revert. Q' = scale * (codes - zero) on each row/group
+ *   grid, then W_hat = S_G^-1 U^T Q' V S_X^-1, written to W_hat [d_out x d_in] fp32.
+ * kq_proxy_loss: Sec. 3.1 Eq. (kron_obj), loss = tr(H_G dW H_X dW^T), dW = W - W_hat, with
+ *   H_G = NULL meaning the identity. Result in *loss (device double). ws:
+ *   kq_proxy_loss_workspace(d_out, d_in) bytes.
+ * ---------------------------------------------------------------------------------- */
+KQ_API kq_status kq_dequant_revert(const uint8_t* codes, const float* scale, const int32_t* zero,
+                            int64_t d_out, int64_t d_in, int group, const float* s_x,
+                            const float* s_g, const int8_t* sign_u, const int8_t* sign_v,
+                            float* W_hat, kq_stream_t stream);
+KQ_API size_t kq_proxy_loss_workspace(int64_t d_out, int64_t d_in);
+KQ_API kq_status kq_proxy_loss(const float* W, const float* W_hat, int64_t d_out, int64_t d_in,
+                        const float* H_X, const float* H_G, double* loss, void* ws,
+                        size_t ws_bytes, kq_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* KRONQ_H */

@@ -1,0 +1,483 @@
+// Stage 2: bidirectional incoherence processing (BiIP) and the sensitivity traces.
+//
+// Paper: Sec. 3.2 Eq. (rescale) (S_X, S_G from Hessian diagonals and weight norms),
+// Eq. (biip) (W <- U W V^T, H_X <- V H_X V^T, H_G <- U H_G U^T), Algorithm 1 (rescale,
+// then rotate, then release H_G); Sec. 3.3 Eq. (sensitivity) (s = tr(H_G) tr(H_X),
+// computed after BiIP).
+//
+// The rotations are randomized Hadamard transforms applied as fast transforms, never as
+// dense matrices (the paper's dense products cost O(n^3); these cost O(n^2 log n) and are
+// bound by HBM): a row transform (along the contiguous dimension, one row per CTA in
+// shared memory) and a column transform (along the strided dimension) done as one pass
+// per radix stage, each CTA holding R rows x CW columns. For n = 28 * 2^k the 2^k part is
+// a Walsh-Hadamard butterfly and the 28-point factor a dense +-1 mix at stride 2^k.
+#include <math.h>
+
+#include "kq_common.cuh"
+
+namespace kq {
+namespace {
+
+// ---------------------------------------------------------------------------------------
+// H_28 by Paley's second construction over GF(13): the symmetric conference matrix
+// C = [[0, 1^T], [1, Q]], Q[i][j] = chi(j - i) (chi = quadratic character mod 13), with
+// every entry replaced by a 2 x 2 block: 0 -> [[1,-1],[-1,-1]], c = +-1 -> c [[1,1],[1,-1]].
+// Stored as 28 row masks; bit a of row r is set when H_28[r][a] = -1.
+constexpr int chi13(int a) {
+    a %= 13;
+    if (a < 0) a += 13;
+    if (a == 0) return 0;
+    for (int x = 1; x < 13; ++x)
+        if ((x * x) % 13 == a) return 1;
+    return -1;
+}
+constexpr int conf14(int i, int j) {
+    if (i == 0 && j == 0) return 0;
+    if (i == 0 || j == 0) return 1;
+    return chi13((j - 1) - (i - 1));
+}
+constexpr int h28_entry(int r, int a) {
+    const int c = conf14(r / 2, a / 2);
+    const int u = r % 2, v = a % 2;
+    if (c == 0) return (u == 0 && v == 0) ? 1 : -1;   // [[1,-1],[-1,-1]]
+    const int blk = (u == 1 && v == 1) ? -1 : 1;     // [[1,1],[1,-1]]
+    return c * blk;
+}
+struct H28Masks {
+    uint32_t m[28];
+};
+constexpr H28Masks make_h28() {
+    H28Masks t{};
+    for (int r = 0; r < 28; ++r) {
+        uint32_t m = 0;
+        for (int a = 0; a < 28; ++a)
+            if (h28_entry(r, a) < 0) m |= 1u << a;
+        t.m[r] = m;
+    }
+    return t;
+}
+constexpr bool h28_is_hadamard() {
+    for (int r = 0; r < 28; ++r)
+        for (int q = 0; q < 28; ++q) {
+            int dot = 0;
+            for (int a = 0; a < 28; ++a) dot += h28_entry(r, a) * h28_entry(q, a);
+            if (dot != (r == q ? 28 : 0)) return false;
+            if (h28_entry(r, q) != h28_entry(q, r)) return false;
+        }
+    return true;
+}
+static_assert(h28_is_hadamard(), "H_28 must satisfy H H^T = 28 I and be symmetric");
+__constant__ H28Masks c_h28 = make_h28();
+
+// Factor applied to element index j before (pre) or after (post) a transform.
+enum FactorMode { F_NONE = 0, F_SMUL = 1, F_SDIV = 2, F_SIGN = 3 };
+
+__device__ __forceinline__ float factor(int mode, const int8_t* sign, const float* s, int64_t j) {
+    if (mode == F_NONE) return 1.0f;
+    const float sg = static_cast<float>(sign[j]);
+    if (mode == F_SIGN || s == nullptr) return sg;
+    return mode == F_SMUL ? sg * s[j] : sg / s[j];
+}
+
+// y = H_28 x for 28 values in registers.
+__device__ __forceinline__ void mix28(const float (&x)[28], float (&y)[28]) {
+#pragma unroll
+    for (int r = 0; r < 28; ++r) {
+        const uint32_t m = c_h28.m[r];
+        float acc = 0.0f;
+#pragma unroll
+        for (int a = 0; a < 28; ++a) acc += ((m >> a) & 1u) ? -x[a] : x[a];
+        y[r] = acc;
+    }
+}
+
+// ------------------------------------------------------------------ row transform
+// For each row of M [rows x n]: v <- pre (.) v; v <- (H_28 (x) H_P) v (or H_P); row <-
+// post (.) v / sqrt(n). One CTA per row (grid-stride); n floats of shared memory.
+__global__ void __launch_bounds__(512) rht_rows_kernel(float* __restrict__ M, int64_t rows, int n, int P, int has28,
+                                int pre_mode, int post_mode, const int8_t* __restrict__ sign,
+                                const float* __restrict__ s, float inv_sqrt_n) {
+    extern __shared__ float v[];
+    for (int64_t r = blockIdx.x; r < rows; r += gridDim.x) {
+        float* row = M + r * n;
+        for (int j = threadIdx.x; j < n; j += blockDim.x)
+            v[j] = row[j] * factor(pre_mode, sign, s, j);
+        __syncthreads();
+        // Butterflies with span h < P stay inside each P-aligned chunk: I_28 (x) H_P.
+        for (int h = 1; h < P; h <<= 1) {
+            for (int t = threadIdx.x; t < n / 2; t += blockDim.x) {
+                const int i = (t / h) * 2 * h + (t % h);
+                const float a = v[i], b = v[i + h];
+                v[i] = a + b;
+                v[i + h] = a - b;
+            }
+            __syncthreads();
+        }
+        if (has28) {   // H_28 (x) I_P
+            for (int b = threadIdx.x; b < P; b += blockDim.x) {
+                float x[28], y[28];
+#pragma unroll
+                for (int a = 0; a < 28; ++a) x[a] = v[a * P + b];
+                mix28(x, y);
+#pragma unroll
+                for (int a = 0; a < 28; ++a) v[a * P + b] = y[a];
+            }
+            __syncthreads();
+        }
+        for (int j = threadIdx.x; j < n; j += blockDim.x)
+            row[j] = v[j] * (factor(post_mode, sign, s, j) * inv_sqrt_n);
+        __syncthreads();
+    }
+}
+
+// --------------------------------------------------------------- column transform
+// One radix stage along the row index of M [n x ncols]: for every group base = hi*R*S + lo
+// (lo < S) and CW-column strip, rows base + i*S (i < R) are transformed along i by H_R
+// (R a power of two) or H_28 (R == 28). Shared memory [R][CW].
+__global__ void __launch_bounds__(256) rht_cols_kernel(float* __restrict__ M, int n, int64_t ncols, int R, int S, int CW,
+                                int pre_mode, int post_mode, const int8_t* __restrict__ sign,
+                                const float* __restrict__ s, float post_scale) {
+    extern __shared__ float v[];
+    const int64_t nstrips = (ncols + CW - 1) / CW;
+    const int64_t ngroups = n / R;
+    for (int64_t w = blockIdx.x; w < ngroups * nstrips; w += gridDim.x) {
+        const int64_t g = w / nstrips;
+        const int64_t c0 = (w % nstrips) * CW;
+        const int64_t base = (g / S) * static_cast<int64_t>(R) * S + (g % S);
+        const int cw = static_cast<int>(min(static_cast<int64_t>(CW), ncols - c0));
+        for (int e = threadIdx.x; e < R * CW; e += blockDim.x) {
+            const int i = e / CW, c = e % CW;
+            const int64_t r = base + static_cast<int64_t>(i) * S;
+            v[e] = c < cw ? M[r * ncols + c0 + c] * factor(pre_mode, sign, s, r) : 0.0f;
+        }
+        __syncthreads();
+        if (R == 28) {
+            for (int c = threadIdx.x; c < CW; c += blockDim.x) {
+                float x[28], y[28];
+#pragma unroll
+                for (int a = 0; a < 28; ++a) x[a] = v[a * CW + c];
+                mix28(x, y);
+#pragma unroll
+                for (int a = 0; a < 28; ++a) v[a * CW + c] = y[a];
+            }
+            __syncthreads();
+        } else {
+            for (int h = 1; h < R; h <<= 1) {
+                for (int e = threadIdx.x; e < (R / 2) * CW; e += blockDim.x) {
+                    const int t = e / CW, c = e % CW;
+                    const int i = (t / h) * 2 * h + (t % h);
+                    const float a = v[i * CW + c], b = v[(i + h) * CW + c];
+                    v[i * CW + c] = a + b;
+                    v[(i + h) * CW + c] = a - b;
+                }
+                __syncthreads();
+            }
+        }
+        for (int e = threadIdx.x; e < R * CW; e += blockDim.x) {
+            const int i = e / CW, c = e % CW;
+            if (c < cw) {
+                const int64_t r = base + static_cast<int64_t>(i) * S;
+                M[r * ncols + c0 + c] = v[e] * (factor(post_mode, sign, s, r) * post_scale);
+            }
+        }
+        __syncthreads();
+    }
+}
+
+// ------------------------------------------------------------------------ scales
+__device__ __forceinline__ float quarter_root_ratio(float h, double a) {
+    if (!(h > 0.0f) || !(a > 0.0)) return 1.0f;   // dead channel (or NaN): scale 1
+    return static_cast<float>(sqrt(sqrt(static_cast<double>(h) / a)));
+}
+
+// a_j = ||W[:, j]||^2 and s_x[j] = (H_X[j][j] / a_j)^(1/4). Block (32, 8).
+__global__ void colscale_kernel(const float* __restrict__ W, int64_t d_out, int64_t d_in,
+                                const float* __restrict__ HX, float* __restrict__ s_x) {
+    __shared__ double part[8][33];
+    const int64_t j = static_cast<int64_t>(blockIdx.x) * 32 + threadIdx.x;
+    double acc = 0.0;
+    if (j < d_in) {
+        float p = 0.0f;
+        int cnt = 0;
+        for (int64_t r = threadIdx.y; r < d_out; r += 8) {
+            const float w = W[r * d_in + j];
+            p = fmaf(w, w, p);
+            if (++cnt == 32) {
+                acc += p;
+                p = 0.0f;
+                cnt = 0;
+            }
+        }
+        acc += p;
+    }
+    part[threadIdx.y][threadIdx.x] = acc;
+    __syncthreads();
+    if (threadIdx.y == 0 && j < d_in) {
+        double a = 0.0;
+        for (int y = 0; y < 8; ++y) a += part[y][threadIdx.x];
+        s_x[j] = quarter_root_ratio(HX[j * d_in + j], a);
+    }
+}
+
+// r_i = ||W[i, :]||^2 and s_g[i] = (H_G[i][i] / r_i)^(1/4) (1 when H_G is NULL). Warp per row.
+__global__ void rowscale_kernel(const float* __restrict__ W, int64_t d_out, int64_t d_in,
+                                const float* __restrict__ HG, float* __restrict__ s_g) {
+    const int64_t i = static_cast<int64_t>(blockIdx.x) * (blockDim.x / 32) + threadIdx.x / 32;
+    const int lane = threadIdx.x & 31;
+    if (i >= d_out) return;
+    double acc = 0.0;
+    float p = 0.0f;
+    int cnt = 0;
+    for (int64_t j = lane; j < d_in; j += 32) {
+        const float w = W[i * d_in + j];
+        p = fmaf(w, w, p);
+        if (++cnt == 32) {
+            acc += p;
+            p = 0.0f;
+            cnt = 0;
+        }
+    }
+    acc += p;
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (lane == 0) s_g[i] = HG ? quarter_root_ratio(HG[i * d_out + i], acc) : 1.0f;
+}
+
+// out = [tr H_X, tr H_G, product, tr H_X', tr H_G', product'] with tr H' = sum h_j / s_j^2.
+__global__ void traces_kernel(const float* __restrict__ HX, const float* __restrict__ s_x,
+                              int64_t d_in, const float* __restrict__ HG,
+                              const float* __restrict__ s_g, int64_t d_out, double* out) {
+    __shared__ double part[4][32];
+    double v[4] = {0.0, 0.0, 0.0, 0.0};
+    for (int64_t j = threadIdx.x; j < d_in; j += blockDim.x) {
+        const double h = HX[j * d_in + j];
+        const double sc = s_x ? static_cast<double>(s_x[j]) : 1.0;
+        v[0] += h;
+        v[2] += h / (sc * sc);
+    }
+    for (int64_t i = threadIdx.x; i < d_out; i += blockDim.x) {
+        const double h = HG[i * d_out + i];
+        const double sc = s_g ? static_cast<double>(s_g[i]) : 1.0;
+        v[1] += h;
+        v[3] += h / (sc * sc);
+    }
+    for (int k = 0; k < 4; ++k) {
+        for (int o = 16; o > 0; o >>= 1) v[k] += __shfl_xor_sync(0xffffffffu, v[k], o);
+        if ((threadIdx.x & 31) == 0) part[k][threadIdx.x >> 5] = v[k];
+    }
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        for (int k = 0; k < 4; ++k) {
+            double x = threadIdx.x < blockDim.x / 32 ? part[k][threadIdx.x] : 0.0;
+            for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+            v[k] = x;
+        }
+        if (threadIdx.x == 0) {
+            out[0] = v[0];
+            out[1] = v[1];
+            out[2] = v[0] * v[1];
+            out[3] = v[2];
+            out[4] = v[3];
+            out[5] = v[2] * v[3];
+        }
+    }
+}
+
+// ------------------------------------------------------------------ host helpers
+struct HadamardPlan {
+    int P = 0;       // power-of-two factor
+    int has28 = 0;   // n = 28 * P
+};
+
+bool plan_of(int64_t n, HadamardPlan* p) {
+    if (n < 1 || n > 32768) return false;
+    if ((n & (n - 1)) == 0) {
+        p->P = static_cast<int>(n);
+        p->has28 = 0;
+        return true;
+    }
+    if (n % 28 == 0) {
+        const int64_t q = n / 28;
+        if ((q & (q - 1)) == 0 && q <= 1024) {
+            p->P = static_cast<int>(q);
+            p->has28 = 1;
+            return true;
+        }
+    }
+    return false;
+}
+
+int log2i(int64_t x) {
+    int k = 0;
+    while ((1ll << k) < x) ++k;
+    return k;
+}
+
+kq_status rows_transform(float* M, int64_t rows, int64_t n, int pre, int post, const int8_t* sign,
+                         const float* s, cudaStream_t stream) {
+    HadamardPlan p;
+    if (!plan_of(n, &p)) return KQ_ERR_UNSUPPORTED;
+    const size_t smem = static_cast<size_t>(n) * sizeof(float);
+    static bool attr = false;
+    if (!attr) {
+        KQ_CUDA(cudaFuncSetAttribute(rht_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     32768 * 4));
+        attr = true;
+    }
+    const int threads = n >= 2048 ? 512 : (n >= 512 ? 256 : 128);
+    const int64_t grid = std::min<int64_t>(rows, static_cast<int64_t>(num_sms()) * 16);
+    if (grid > 0) {
+        rht_rows_kernel<<<static_cast<unsigned>(grid), threads, smem, stream>>>(
+            M, rows, static_cast<int>(n), p.P, p.has28, pre, post, sign, s,
+            static_cast<float>(1.0 / sqrt(static_cast<double>(n))));
+        KQ_LAUNCH_CHECK("rht_rows_kernel");
+    }
+    return KQ_OK;
+}
+
+kq_status cols_transform(float* M, int64_t n, int64_t ncols, int pre, int post, const int8_t* sign,
+                         const float* s, cudaStream_t stream) {
+    HadamardPlan p;
+    if (!plan_of(n, &p)) return KQ_ERR_UNSUPPORTED;
+    // Radix stages: (R, S) pairs applied in order; S = product of earlier radices.
+    int R[3], S[3], ns = 0;
+    const int kp = log2i(p.P);
+    if (kp <= 10) {
+        if (p.P > 1) { R[ns] = p.P; S[ns] = 1; ++ns; }
+    } else {
+        const int k1 = kp - kp / 2, k2 = kp / 2;
+        R[ns] = 1 << k1; S[ns] = 1; ++ns;
+        R[ns] = 1 << k2; S[ns] = 1 << k1; ++ns;
+    }
+    if (p.has28) { R[ns] = 28; S[ns] = p.P; ++ns; }
+    static bool attr = false;
+    if (!attr) {
+        KQ_CUDA(cudaFuncSetAttribute(rht_cols_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     128 * 1024));
+        attr = true;
+    }
+    const float post_scale = static_cast<float>(1.0 / sqrt(static_cast<double>(n)));
+    if (ns == 0) {   // n == 1: only the factors apply
+        R[0] = 1; S[0] = 1; ns = 1;
+    }
+    for (int st = 0; st < ns; ++st) {
+        int CW = 32768 / R[st];
+        CW = CW < 32 ? 32 : (CW > 256 ? 256 : CW);
+        const size_t smem = static_cast<size_t>(R[st]) * CW * sizeof(float);
+        const int64_t items = (n / R[st]) * cdiv(ncols, CW);
+        const int64_t grid = std::min<int64_t>(items, static_cast<int64_t>(num_sms()) * 8);
+        rht_cols_kernel<<<static_cast<unsigned>(grid), 256, smem, stream>>>(
+            M, static_cast<int>(n), ncols, R[st], S[st], CW, st == 0 ? pre : F_NONE,
+            st == ns - 1 ? post : F_NONE, sign, s, st == ns - 1 ? post_scale : 1.0f);
+        KQ_LAUNCH_CHECK("rht_cols_kernel");
+    }
+    return KQ_OK;
+}
+
+}  // namespace
+}  // namespace kq
+
+using namespace kq;
+
+extern "C" kq_status kq_compute_scales(const float* W, int64_t d_out, int64_t d_in, const float* H_X,
+                                       const float* H_G, float* s_x, float* s_g,
+                                       kq_stream_t stream_) {
+    cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+    if (!W || !H_X || !s_x || !s_g || d_out < 1 || d_in < 1) {
+        set_error("kq_compute_scales: invalid arguments");
+        return KQ_ERR_INVALID_ARG;
+    }
+    colscale_kernel<<<static_cast<unsigned>(cdiv(d_in, 32)), dim3(32, 8), 0, stream>>>(W, d_out, d_in,
+                                                                                    H_X, s_x);
+    KQ_LAUNCH_CHECK("colscale_kernel");
+    rowscale_kernel<<<static_cast<unsigned>(cdiv(d_out, 8)), 256, 0, stream>>>(W, d_out, d_in, H_G,
+                                                                              s_g);
+    KQ_LAUNCH_CHECK("rowscale_kernel");
+    return KQ_OK;
+}
+
+extern "C" kq_status kq_traces(const float* H_X, const float* s_x, int64_t d_in, const float* H_G,
+                               const float* s_g, int64_t d_out, double* out, kq_stream_t stream_) {
+    cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+    if (!H_X || !H_G || !out || d_in < 1 || d_out < 1) {
+        set_error("kq_traces: invalid arguments");
+        return KQ_ERR_INVALID_ARG;
+    }
+    traces_kernel<<<1, 1024, 0, stream>>>(H_X, s_x, d_in, H_G, s_g, d_out, out);
+    KQ_LAUNCH_CHECK("traces_kernel");
+    return KQ_OK;
+}
+
+extern "C" kq_status kq_rotate_in(float* W, int64_t d_out, int64_t d_in, float* H_X, const float* s_x,
+                                  const int8_t* sign_v, int dir, kq_stream_t stream_) {
+    cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+    HadamardPlan p;
+    if (!W || !sign_v || d_out < 1 || d_in < 1 || (dir != KQ_FWD && dir != KQ_INV)) {
+        set_error("kq_rotate_in: invalid arguments");
+        return KQ_ERR_INVALID_ARG;
+    }
+    if (!plan_of(d_in, &p)) {
+        set_error("kq_rotate_in: d_in=%lld has no Hadamard construction", (long long)d_in);
+        return KQ_ERR_UNSUPPORTED;
+    }
+    kq_status st;
+    if (dir == KQ_FWD) {
+        // W <- (W S_X) V^T: each row times sigma_j s_j, then H_n, then 1/sqrt(n).
+        st = rows_transform(W, d_out, d_in, s_x ? F_SMUL : F_SIGN, F_NONE, sign_v, s_x, stream);
+        if (st != KQ_OK) return st;
+        if (H_X) {
+            // H_X <- V S_X^-1 H_X S_X^-1 V^T: both sides scaled by sigma / s, then H_n twice.
+            st = rows_transform(H_X, d_in, d_in, s_x ? F_SDIV : F_SIGN, F_NONE, sign_v, s_x, stream);
+            if (st != KQ_OK) return st;
+            st = cols_transform(H_X, d_in, d_in, s_x ? F_SDIV : F_SIGN, F_NONE, sign_v, s_x, stream);
+            if (st != KQ_OK) return st;
+        }
+    } else {
+        // W <- (W V) S_X^-1 = (W H_n) diag(sigma / s) / sqrt(n).
+        st = rows_transform(W, d_out, d_in, F_NONE, s_x ? F_SDIV : F_SIGN, sign_v, s_x, stream);
+        if (st != KQ_OK) return st;
+    }
+    return KQ_OK;
+}
+
+extern "C" kq_status kq_rotate_out(float* W, int64_t d_out, int64_t d_in, float* H_G, const float* s_g,
+                                   const int8_t* sign_u, int dir, kq_stream_t stream_) {
+    cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+    HadamardPlan p;
+    if (!W || !sign_u || d_out < 1 || d_in < 1 || (dir != KQ_FWD && dir != KQ_INV)) {
+        set_error("kq_rotate_out: invalid arguments");
+        return KQ_ERR_INVALID_ARG;
+    }
+    if (!plan_of(d_out, &p)) {
+        set_error("kq_rotate_out: d_out=%lld has no Hadamard construction", (long long)d_out);
+        return KQ_ERR_UNSUPPORTED;
+    }
+    kq_status st;
+    if (dir == KQ_FWD) {
+        // W <- U (S_G W): rows scaled by sigma_i s_i, then H_n along the row index.
+        st = cols_transform(W, d_out, d_in, s_g ? F_SMUL : F_SIGN, F_NONE, sign_u, s_g, stream);
+        if (st != KQ_OK) return st;
+        if (H_G) {
+            st = rows_transform(H_G, d_out, d_out, s_g ? F_SDIV : F_SIGN, F_NONE, sign_u, s_g, stream);
+            if (st != KQ_OK) return st;
+            st = cols_transform(H_G, d_out, d_out, s_g ? F_SDIV : F_SIGN, F_NONE, sign_u, s_g, stream);
+            if (st != KQ_OK) return st;
+        }
+    } else {
+        // W <- S_G^-1 U^T W = diag(sigma / s) H_n W / sqrt(n).
+        st = cols_transform(W, d_out, d_in, F_NONE, s_g ? F_SDIV : F_SIGN, sign_u, s_g, stream);
+        if (st != KQ_OK) return st;
+    }
+    return KQ_OK;
+}
+
+// Used by the check-only revert (check.cu).
+namespace kq {
+kq_status rotate_rows_inv(float* M, int64_t rows, int64_t n, const float* s, const int8_t* sign,
+                          cudaStream_t stream) {
+    return rows_transform(M, rows, n, F_NONE, s ? F_SDIV : F_SIGN, sign, s, stream);
+}
+kq_status rotate_cols_inv(float* M, int64_t n, int64_t ncols, const float* s, const int8_t* sign,
+                          cudaStream_t stream) {
+    return cols_transform(M, n, ncols, F_NONE, s ? F_SDIV : F_SIGN, sign, s, stream);
+}
+}  // namespace kq

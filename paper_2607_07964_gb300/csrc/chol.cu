@@ -1,0 +1,311 @@
+// Stage 3: damped inverse Cholesky.
+//
+// Paper: Algorithm 2 ("H_X <- H_X + lambda mean(diag(H_X)) I; L <- Inverse_Cholesky(H_X)")
+// and Proposition 1 (H_X^-1 = L L^T, L lower). The OBS sweep (Eq. obs_update) uses row j of
+// R = L^T.
+//
+// Route (2 n^3 / 3 flops instead of factor -> invert -> factor): with J the index
+// reversal, the lower Cholesky factor C of A = J H J gives H = (J C J)(J C J)^T, J C J
+// upper, hence H^-1 = (J C^-T J)(J C^-T J)^T and L = J C^-T J, i.e. L[i][j] = C^-1[n-1-j][n-1-i].
+// One right-looking blocked sweep (block nb = 128) computes C and Z = C^-1 together:
+//   step k: diag  -- factor A_kk = C_kk C_kk^T and invert C_kk in shared memory (1 CTA);
+//           panel -- C_ik = A_ik C_kk^-T (i > k) and Z_kj = C_kk^-1 B_kj (j < k);
+//           update-- A_ij -= C_ik C_jk^T (k < j <= i) and B_ij -= C_ik Z_kj (j <= k < i),
+// where B (stored in Z's blocks) is the right-hand side I of C Z = I after the earlier
+// steps' eliminations. The matrix is padded to a multiple of nb with an identity block.
+// All arithmetic is fp32 with fused multiply-add.
+#include <math.h>
+
+#include "kq_common.cuh"
+
+namespace kq {
+namespace {
+
+constexpr int NB = 128;
+constexpr int LD = NB + 1;                      // padded shared-memory row
+constexpr int TILE_FLOATS = NB * LD;
+constexpr int GEMM_THREADS = 256;               // 16 x 16 threads, 8 x 8 outputs each
+constexpr size_t GEMM_SMEM = 2 * TILE_FLOATS * sizeof(float);
+
+struct Work {
+    float* A;      // npad x npad, reversed damped H -> C (lower)
+    float* Z;      // npad x npad, B -> C^-1 (lower)
+    double* dsum;  // sum of diag(H)
+};
+
+inline size_t npad_of(int64_t n) { return static_cast<size_t>(cdiv(n, NB) * NB); }
+
+// --------------------------------------------------------------------- prep
+__global__ void diag_sum_kernel(const float* __restrict__ H, int64_t n, double* out) {
+    __shared__ double part[32];
+    double s = 0.0;
+    for (int64_t j = threadIdx.x; j < n; j += blockDim.x) s += static_cast<double>(H[j * n + j]);
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = s;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        s = threadIdx.x < blockDim.x / 32 ? part[threadIdx.x] : 0.0;
+        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        if (threadIdx.x == 0) *out = s;
+    }
+}
+
+// A[i][j] = H[n-1-i][n-1-j] + delta [i == j] inside n; identity in the padding; Z = 0.
+__global__ void prep_kernel(const float* __restrict__ H, int64_t n, int64_t npad, float damp_rel,
+                            const double* __restrict__ dsum, float* __restrict__ A,
+                            float* __restrict__ Z) {
+    const float delta = static_cast<float>(static_cast<double>(damp_rel) * (*dsum / static_cast<double>(n)));
+    const int64_t total = npad * npad;
+    for (int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < total;
+         e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t i = e / npad, j = e % npad;
+        float v;
+        if (i < n && j < n) {
+            v = H[(n - 1 - i) * n + (n - 1 - j)];
+            if (i == j) v += delta;
+        } else {
+            v = (i == j) ? 1.0f : 0.0f;
+        }
+        A[e] = v;
+        Z[e] = 0.0f;
+    }
+}
+
+// ---------------------------------------------------------------- diag block
+// Factor A_kk (lower) = C C^T in shared memory, write C to A_kk and C^-1 to Z_kk.
+// A non-positive (or NaN) pivot records its index in H's own numbering (1-based).
+__global__ void __launch_bounds__(512) chol_diag_kernel(Work w, int64_t n, int64_t npad, int k, int* info) {
+    extern __shared__ float sm[];
+    float* a = sm;                  // [NB][LD]
+    float* x = sm + TILE_FLOATS;    // [NB][LD] inverse
+    const int64_t off = static_cast<int64_t>(k) * NB;
+    for (int e = threadIdx.x; e < NB * NB; e += blockDim.x) {
+        const int r = e / NB, c = e % NB;
+        a[r * LD + c] = c <= r ? w.A[(off + r) * npad + off + c] : 0.0f;
+    }
+    __syncthreads();
+    __shared__ float dj;
+    for (int j = 0; j < NB; ++j) {
+        if (threadIdx.x == 0) {
+            const float p = a[j * LD + j];
+            if (!(p > 0.0f)) {
+                const int64_t rev = off + j;
+                if (rev < n) record_error(info, static_cast<int>(n - rev));
+            }
+            dj = sqrtf(p);
+            a[j * LD + j] = dj;
+        }
+        __syncthreads();
+        const float d = dj;
+        for (int r = j + 1 + threadIdx.x; r < NB; r += blockDim.x) a[r * LD + j] = a[r * LD + j] / d;
+        __syncthreads();
+        const int m = NB - 1 - j;   // trailing size
+        for (int e = threadIdx.x; e < m * m; e += blockDim.x) {
+            const int r = j + 1 + e / m, c = j + 1 + e % m;
+            if (c <= r) a[r * LD + c] = fmaf(-a[r * LD + j], a[c * LD + j], a[r * LD + c]);
+        }
+        __syncthreads();
+    }
+    // Inverse of the lower-triangular C: thread c solves C x = e_c (x lower: rows >= c).
+    for (int c = threadIdx.x; c < NB; c += blockDim.x) {
+        for (int r = 0; r < NB; ++r) {
+            if (r < c) {
+                x[r * LD + c] = 0.0f;
+                continue;
+            }
+            float s = (r == c) ? 1.0f : 0.0f;
+            for (int m2 = c; m2 < r; ++m2) s = fmaf(-a[r * LD + m2], x[m2 * LD + c], s);
+            x[r * LD + c] = s / a[r * LD + r];
+        }
+    }
+    __syncthreads();
+    for (int e = threadIdx.x; e < NB * NB; e += blockDim.x) {
+        const int r = e / NB, c = e % NB;
+        w.A[(off + r) * npad + off + c] = c <= r ? a[r * LD + c] : 0.0f;
+        w.Z[(off + r) * npad + off + c] = x[r * LD + c];
+    }
+}
+
+// ---------------------------------------------------------------- tile GEMM core
+// acc[a][b] += sum_m P[r_a][m] * Q(m, c_b), r_a = ty + 16 a, c_b = tx + 16 b, m ascending.
+// Q(m, c) = TRANSQ ? q[c][m] : q[m][c]. Both operands are [NB][LD] shared tiles.
+template <bool TRANSQ>
+__device__ __forceinline__ void tile_mac(const float* p, const float* q, float (&acc)[8][8], int ty,
+                                         int tx) {
+#pragma unroll 2
+    for (int m = 0; m < NB; ++m) {
+        float pa[8], qb[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) pa[i] = p[(ty + 16 * i) * LD + m];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) qb[j] = TRANSQ ? q[(tx + 16 * j) * LD + m] : q[m * LD + tx + 16 * j];
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+#pragma unroll
+            for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(pa[i], qb[j], acc[i][j]);
+    }
+}
+
+__device__ __forceinline__ void load_tile(float* dst, const float* src, int64_t ld_src) {
+    for (int e = threadIdx.x; e < NB * NB; e += blockDim.x) {
+        const int r = e / NB, c = e % NB;
+        dst[r * LD + c] = src[r * ld_src + c];
+    }
+}
+
+// --------------------------------------------------------------------- panel
+// CTA b < k: Z_kb <- C_kk^-1 Z_kb.  CTA b >= k: i = b + 1, A_ik <- A_ik C_kk^-T.
+__global__ void __launch_bounds__(GEMM_THREADS) chol_panel_kernel(Work w, int64_t npad, int k) {
+    extern __shared__ float sm[];
+    float* cinv = sm;
+    float* t = sm + TILE_FLOATS;
+    const int b = blockIdx.x;
+    const int64_t off = static_cast<int64_t>(k) * NB;
+    load_tile(cinv, w.Z + off * npad + off, npad);
+    const bool zpart = b < k;
+    float* blk = zpart ? w.Z + off * npad + static_cast<int64_t>(b) * NB
+                       : w.A + static_cast<int64_t>(b + 1) * NB * npad + off;
+    load_tile(t, blk, npad);
+    __syncthreads();
+    const int ty = threadIdx.x / 16, tx = threadIdx.x % 16;
+    float acc[8][8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[i][j] = 0.0f;
+    if (zpart)
+        tile_mac<false>(cinv, t, acc, ty, tx);   // C^-1 (rows) x B
+    else
+        tile_mac<true>(t, cinv, acc, ty, tx);    // A x (C^-1)^T
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) blk[static_cast<int64_t>(ty + 16 * i) * npad + tx + 16 * j] = acc[i][j];
+}
+
+// -------------------------------------------------------------------- update
+// Tiles (i, j), k < i < nbk, 0 <= j <= i:
+//   j > k : A_ij -= C_ik C_jk^T;     j <= k : Z_ij -= C_ik Z_kj.
+__global__ void __launch_bounds__(GEMM_THREADS) chol_update_kernel(Work w, int64_t npad, int k) {
+    extern __shared__ float sm[];
+    float* p = sm;
+    float* q = sm + TILE_FLOATS;
+    int bid = blockIdx.x;
+    int i = k + 1;
+    while (bid >= i + 1) {
+        bid -= i + 1;
+        ++i;
+    }
+    const int j = bid;
+    const int64_t ko = static_cast<int64_t>(k) * NB;
+    load_tile(p, w.A + static_cast<int64_t>(i) * NB * npad + ko, npad);   // C_ik
+    const bool apart = j > k;
+    if (apart)
+        load_tile(q, w.A + static_cast<int64_t>(j) * NB * npad + ko, npad);   // C_jk
+    else
+        load_tile(q, w.Z + ko * npad + static_cast<int64_t>(j) * NB, npad);   // Z_kj
+    __syncthreads();
+    const int ty = threadIdx.x / 16, tx = threadIdx.x % 16;
+    float acc[8][8];
+#pragma unroll
+    for (int a = 0; a < 8; ++a)
+#pragma unroll
+        for (int b = 0; b < 8; ++b) acc[a][b] = 0.0f;
+    if (apart)
+        tile_mac<true>(p, q, acc, ty, tx);
+    else
+        tile_mac<false>(p, q, acc, ty, tx);
+    float* out = (apart ? w.A : w.Z) + static_cast<int64_t>(i) * NB * npad + static_cast<int64_t>(j) * NB;
+#pragma unroll
+    for (int a = 0; a < 8; ++a)
+#pragma unroll
+        for (int b = 0; b < 8; ++b) {
+            float* o = out + static_cast<int64_t>(ty + 16 * a) * npad + tx + 16 * b;
+            *o = *o - acc[a][b];
+        }
+}
+
+// -------------------------------------------------------------------- finish
+// Lt[i][j] = Z[n-1-j][n-1-i] for j <= i < n, 0 above the diagonal (32 x 32 smem transpose).
+__global__ void finish_kernel(const float* __restrict__ Z, int64_t n, int64_t npad, float* __restrict__ Lt) {
+    __shared__ float t[32][33];
+    const int64_t i0 = static_cast<int64_t>(blockIdx.y) * 32, j0 = static_cast<int64_t>(blockIdx.x) * 32;
+    // Source block: rows a = n-1-j (j in [j0, j0+32)), cols b = n-1-i.
+    for (int r = threadIdx.y; r < 32; r += blockDim.y) {
+        const int64_t j = j0 + r;
+        const int64_t i = i0 + threadIdx.x;
+        float v = 0.0f;
+        if (i < n && j < n && j <= i) v = Z[(n - 1 - j) * npad + (n - 1 - i)];
+        t[r][threadIdx.x] = v;
+    }
+    __syncthreads();
+    for (int r = threadIdx.y; r < 32; r += blockDim.y) {
+        const int64_t i = i0 + r, j = j0 + threadIdx.x;
+        if (i < n && j < n) Lt[i * n + j] = t[threadIdx.x][r];
+    }
+}
+
+}  // namespace
+}  // namespace kq
+
+using namespace kq;
+
+extern "C" size_t kq_chol_inv_workspace(int64_t n) {
+    if (n < 1) return 0;
+    const size_t np = npad_of(n);
+    return 2 * np * np * sizeof(float) + 256;
+}
+
+extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, float* Lt, int* info, void* ws,
+                                 size_t ws_bytes, kq_stream_t stream_) {
+    cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+    if (!H || !Lt || n < 1 || n > 65536 || !(damp_rel >= 0.0f)) {
+        set_error("kq_chol_inv: invalid arguments (n=%lld)", (long long)n);
+        return KQ_ERR_INVALID_ARG;
+    }
+    if (!ws || ws_bytes < kq_chol_inv_workspace(n) || (reinterpret_cast<uintptr_t>(ws) & 15u)) {
+        set_error("kq_chol_inv: workspace must be 16-byte aligned and hold %zu bytes",
+                  kq_chol_inv_workspace(n));
+        return KQ_ERR_WORKSPACE;
+    }
+    const int64_t npad = static_cast<int64_t>(npad_of(n));
+    const int nbk = static_cast<int>(npad / NB);
+    Work w;
+    w.A = static_cast<float*>(ws);
+    w.Z = w.A + npad * npad;
+    w.dsum = reinterpret_cast<double*>(w.Z + npad * npad);
+    static bool attr = false;
+    if (!attr) {
+        KQ_CUDA(cudaFuncSetAttribute(chol_diag_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     static_cast<int>(GEMM_SMEM)));
+        KQ_CUDA(cudaFuncSetAttribute(chol_panel_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     static_cast<int>(GEMM_SMEM)));
+        KQ_CUDA(cudaFuncSetAttribute(chol_update_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     static_cast<int>(GEMM_SMEM)));
+        attr = true;
+    }
+    diag_sum_kernel<<<1, 1024, 0, stream>>>(H, n, w.dsum);
+    KQ_LAUNCH_CHECK("diag_sum_kernel");
+    const int64_t total = npad * npad;
+    const int64_t pgrid = std::min<int64_t>(cdiv(total, 256), static_cast<int64_t>(num_sms()) * 32);
+    prep_kernel<<<static_cast<unsigned>(pgrid), 256, 0, stream>>>(H, n, npad, damp_rel, w.dsum, w.A, w.Z);
+    KQ_LAUNCH_CHECK("prep_kernel");
+    for (int k = 0; k < nbk; ++k) {
+        chol_diag_kernel<<<1, 512, GEMM_SMEM, stream>>>(w, n, npad, k, info);
+        KQ_LAUNCH_CHECK("chol_diag_kernel");
+        if (nbk > 1) {
+            chol_panel_kernel<<<nbk - 1, GEMM_THREADS, GEMM_SMEM, stream>>>(w, npad, k);
+            KQ_LAUNCH_CHECK("chol_panel_kernel");
+        }
+        int64_t tiles = 0;
+        for (int i = k + 1; i < nbk; ++i) tiles += i + 1;
+        if (tiles > 0) {
+            chol_update_kernel<<<static_cast<unsigned>(tiles), GEMM_THREADS, GEMM_SMEM, stream>>>(w, npad, k);
+            KQ_LAUNCH_CHECK("chol_update_kernel");
+        }
+    }
+    finish_kernel<<<dim3(static_cast<unsigned>(cdiv(n, 32)), static_cast<unsigned>(cdiv(n, 32))),
+                    dim3(32, 8), 0, stream>>>(w.Z, n, npad, Lt);
+    KQ_LAUNCH_CHECK("finish_kernel");
+    return KQ_OK;
+}

@@ -1,0 +1,79 @@
+// Host-side plumbing of libkronq: error strings, status mapping, device queries, and
+// kq_check (reads the device error word written by kernels).
+#include <atomic>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+
+#include "kq_common.cuh"
+
+namespace kq {
+
+static thread_local char g_err[512] = "";
+static std::atomic<uint64_t> g_launches{0};
+
+void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+
+void set_error(const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    std::vsnprintf(g_err, sizeof(g_err), fmt, ap);
+    va_end(ap);
+}
+
+kq_status cuda_status(cudaError_t e, const char* where) {
+    set_error("%s: %s (%s)", where, cudaGetErrorName(e), cudaGetErrorString(e));
+    return KQ_ERR_CUDA;
+}
+
+int num_sms() {
+    static int cache[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+    if (!cache[dev]) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+            n = 148;
+        cache[dev] = n;
+    }
+    return cache[dev];
+}
+
+}  // namespace kq
+
+extern "C" const char* kq_last_error(void) { return kq::g_err; }
+
+extern "C" const char* kq_status_name(int s) {
+    switch (s) {
+        case KQ_OK: return "KQ_OK";
+        case KQ_ERR_INVALID_ARG: return "KQ_ERR_INVALID_ARG";
+        case KQ_ERR_UNSUPPORTED: return "KQ_ERR_UNSUPPORTED";
+        case KQ_ERR_NOT_PD: return "KQ_ERR_NOT_PD";
+        case KQ_ERR_CUDA: return "KQ_ERR_CUDA";
+        case KQ_ERR_TIMEOUT: return "KQ_ERR_TIMEOUT";
+        case KQ_ERR_WORKSPACE: return "KQ_ERR_WORKSPACE";
+        default: return "KQ_ERR_UNKNOWN";
+    }
+}
+
+extern "C" int kq_version(void) { return 100; }
+
+extern "C" uint64_t kq_launch_count(void) { return kq::g_launches.load(std::memory_order_relaxed); }
+
+extern "C" kq_status kq_check(int* info, int reset, int* pivot_out, kq_stream_t stream_) {
+    cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+    KQ_CUDA(cudaStreamSynchronize(stream));
+    int v = 0;
+    if (info) {
+        KQ_CUDA(cudaMemcpy(&v, info, sizeof(int), cudaMemcpyDeviceToHost));
+        if (reset && v != 0) KQ_CUDA(cudaMemset(info, 0, sizeof(int)));
+    }
+    if (pivot_out) *pivot_out = v;
+    if (v == 0) return KQ_OK;
+    if (v > 0) {
+        kq::set_error("non-positive pivot at index %d", v);
+        return KQ_ERR_NOT_PD;
+    }
+    kq::set_error("kernel reported %s", kq_status_name(-v));
+    return static_cast<kq_status>(-v);
+}

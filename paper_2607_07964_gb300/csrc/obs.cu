@@ -1,0 +1,305 @@
+// Stage 4: the column-wise OBS sweep with b-bit asymmetric grids (GPTQ mode).
+//
+// Paper: Sec. 2.1 Eq. (obs_update) (compensation -(w_p - q_p)/[H^-1]_pp [H^-1]_{p,p+1:}),
+// Algorithm 2 (inner column loop over a block of B columns with error E, then the lazy
+// trailing update W[:, i+B:] -= E R[i:i+B, i+B:]), Proposition 1 (H_G cancels, so only
+// L = R^T enters). The GPTAQ drift term P is zero here (one input set, X-tilde = X).
+//
+// Every fp32 operation is written with an explicit round-to-nearest intrinsic so the
+// compiler cannot contract or reorder it; the order is:
+//   grid      scale = (xmax - xmin) / (2^b - 1), zero = rint(-xmin / scale)
+//   column j  q = clamp(rint(w / scale) + zero, 0, 2^b - 1); what = scale * (q - zero)
+//             E = (w - what) / R_jj;  w_k = fma(-E, R_jk, w_k) for k in (j, block end)
+//   trailing  acc = fma(E_k, R_kc, acc) over ascending k; w_c = w_c - acc
+// Kernels:
+//   rowgrid_kernel   per-row grid (group = 0) from the whole row before the sweep
+//   obs_block_kernel one warp per row; the block's R (128 x 128) in shared memory
+//   trailing_kernel  128 x 128 output tiles, K = block, shared-memory operands
+//   colloss_kernel   col_loss[j] = sum over rows of E_j^2, fixed order, fp64
+#include <math.h>
+
+#include "kq_common.cuh"
+
+namespace kq {
+namespace {
+
+constexpr int BLK = 128;          // block size B (Algorithm 2); the only supported value
+constexpr int RLD = BLK + 1;
+constexpr int TT = 128;           // trailing tile
+constexpr int TLD = BLK + 1;
+
+struct Grid {
+    float scale, zero;
+};
+
+__device__ __forceinline__ Grid make_grid(float xmin, float xmax, float maxq) {
+    xmin = fminf(xmin, 0.0f);
+    xmax = fmaxf(xmax, 0.0f);
+    if (xmin == 0.0f && xmax == 0.0f) {
+        xmin = -1.0f;
+        xmax = 1.0f;
+    }
+    Grid g;
+    g.scale = __fdiv_rn(__fsub_rn(xmax, xmin), maxq);
+    g.zero = rintf(__fdiv_rn(-xmin, g.scale));
+    return g;
+}
+
+__device__ __forceinline__ float warp_min(float v) {
+    for (int o = 16; o > 0; o >>= 1) v = fminf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+
+// Per-row grid from the whole row (group = 0). Warp per row.
+__global__ void rowgrid_kernel(const float* __restrict__ W, int64_t d_out, int64_t d_in, int bits,
+                               float* __restrict__ scale, int32_t* __restrict__ zero,
+                               float* __restrict__ gscale, float* __restrict__ gzero) {
+    const int64_t r = static_cast<int64_t>(blockIdx.x) * (blockDim.x / 32) + threadIdx.x / 32;
+    const int lane = threadIdx.x & 31;
+    if (r >= d_out) return;
+    float mn = 0.0f, mx = 0.0f;
+    for (int64_t j = lane; j < d_in; j += 32) {
+        const float v = W[r * d_in + j];
+        mn = fminf(mn, v);
+        mx = fmaxf(mx, v);
+    }
+    mn = warp_min(mn);
+    mx = warp_max(mx);
+    const Grid g = make_grid(mn, mx, static_cast<float>((1 << bits) - 1));
+    if (lane == 0) {
+        scale[r] = g.scale;
+        zero[r] = static_cast<int32_t>(g.zero);
+        gscale[r] = g.scale;
+        gzero[r] = g.zero;
+    }
+}
+
+// One block [i0, e) of the sweep for all rows. Warp per row (grid-stride over rows); lane l
+// holds columns i0 + 32 s + l (s = 0..3) in registers.
+__global__ void __launch_bounds__(256) obs_block_kernel(
+    const float* __restrict__ W, int64_t d_out, int64_t d_in, const float* __restrict__ Lt, int64_t i0,
+    int bits, int group, const float* __restrict__ gscale, const float* __restrict__ gzero,
+    uint8_t* __restrict__ codes, float* __restrict__ scale, int32_t* __restrict__ zero,
+    float* __restrict__ E, float* __restrict__ pre_q) {
+    extern __shared__ float Rs[];   // [BLK][RLD], Rs[j][k] = R[i0 + j][i0 + k] = Lt[i0 + k][i0 + j]
+    const int nb = static_cast<int>(min(static_cast<int64_t>(BLK), d_in - i0));
+    for (int e = threadIdx.x; e < BLK * BLK; e += blockDim.x) {
+        const int k = e / BLK, j = e % BLK;   // coalesced over j along row i0 + k of Lt
+        float v = 0.0f;
+        if (j < nb && k < nb && k >= j) v = Lt[(i0 + k) * d_in + i0 + j];
+        Rs[j * RLD + k] = v;
+    }
+    __syncthreads();
+    const float maxq = static_cast<float>((1 << bits) - 1);
+    const int lane = threadIdx.x & 31;
+    const int64_t ngroups = group ? (d_in + group - 1) / group : 1;
+    const int warps = blockDim.x / 32;
+    for (int64_t r = static_cast<int64_t>(blockIdx.x) * warps + threadIdx.x / 32; r < d_out;
+         r += static_cast<int64_t>(gridDim.x) * warps) {
+        const float* wr = W + r * d_in + i0;
+        float w[4], e[4];
+        uint32_t qv[4];
+#pragma unroll
+        for (int s = 0; s < 4; ++s) {
+            const int c = 32 * s + lane;
+            w[s] = c < nb ? wr[c] : 0.0f;
+            e[s] = 0.0f;
+            qv[s] = 0;
+        }
+        Grid g;
+        if (group) {
+            float mn = 0.0f, mx = 0.0f;
+#pragma unroll
+            for (int s = 0; s < 4; ++s)
+                if (32 * s + lane < nb) {
+                    mn = fminf(mn, w[s]);
+                    mx = fmaxf(mx, w[s]);
+                }
+            g = make_grid(warp_min(mn), warp_max(mx), maxq);
+            if (lane == 0) {
+                const int64_t gi = r * ngroups + i0 / group;
+                scale[gi] = g.scale;
+                zero[gi] = static_cast<int32_t>(g.zero);
+            }
+        } else {
+            g.scale = gscale[r];
+            g.zero = gzero[r];
+        }
+        float pq[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
+        for (int s = 0; s < 4; ++s) {
+            for (int jl = 0; jl < 32; ++jl) {
+                const int j = 32 * s + jl;
+                if (j >= nb) break;
+                const float wj = __shfl_sync(0xffffffffu, w[s], jl);
+                float q = __fadd_rn(rintf(__fdiv_rn(wj, g.scale)), g.zero);
+                q = fminf(fmaxf(q, 0.0f), maxq);
+                const float what = __fmul_rn(g.scale, __fsub_rn(q, g.zero));
+                const float err = __fdiv_rn(__fsub_rn(wj, what), Rs[j * RLD + j]);
+                if (lane == jl) {
+                    e[s] = err;
+                    qv[s] = static_cast<uint32_t>(q);
+                    pq[s] = wj;
+                }
+#pragma unroll
+                for (int t = s; t < 4; ++t) {
+                    const int k = 32 * t + lane;
+                    if (k > j) w[t] = __fmaf_rn(-err, Rs[j * RLD + k], w[t]);
+                }
+            }
+        }
+#pragma unroll
+        for (int s = 0; s < 4; ++s) {
+            const int c = 32 * s + lane;
+            if (c < nb) {
+                codes[r * d_in + i0 + c] = static_cast<uint8_t>(qv[s]);
+                E[r * d_in + i0 + c] = e[s];
+                if (pre_q) pre_q[r * d_in + i0 + c] = pq[s];
+            }
+        }
+    }
+}
+
+// W[:, e0:] -= E[:, i0:e0] R[i0:e0, e0:], R[k][c] = Lt[c][k]. Tile: 128 rows x 128 columns.
+// acc = fma(E_k, R_kc, acc) over ascending k, then w = w - acc.
+__global__ void __launch_bounds__(256) trailing_kernel(float* __restrict__ W, const float* __restrict__ E,
+                                                       const float* __restrict__ Lt, int64_t d_out,
+                                                       int64_t d_in, int64_t i0, int kb) {
+    extern __shared__ float sm[];
+    float* es = sm;                 // [TT][TLD]  es[r][k] = E[r0 + r][i0 + k]
+    float* ls = sm + TT * TLD;      // [TT][TLD]  ls[c][k] = Lt[c0 + c][i0 + k]
+    const int64_t e0 = i0 + kb;
+    const int64_t r0 = static_cast<int64_t>(blockIdx.y) * TT;
+    const int64_t c0 = e0 + static_cast<int64_t>(blockIdx.x) * TT;
+    for (int idx = threadIdx.x; idx < TT * BLK; idx += blockDim.x) {
+        const int a = idx / BLK, k = idx % BLK;
+        const int64_t r = r0 + a, c = c0 + a;
+        es[a * TLD + k] = (k < kb && r < d_out) ? E[r * d_in + i0 + k] : 0.0f;
+        ls[a * TLD + k] = (k < kb && c < d_in) ? Lt[c * d_in + i0 + k] : 0.0f;
+    }
+    __syncthreads();
+    const int ty = threadIdx.x / 16, tx = threadIdx.x % 16;
+    float acc[8][8];
+#pragma unroll
+    for (int a = 0; a < 8; ++a)
+#pragma unroll
+        for (int b = 0; b < 8; ++b) acc[a][b] = 0.0f;
+    for (int k = 0; k < kb; ++k) {
+        float ea[8], lb[8];
+#pragma unroll
+        for (int a = 0; a < 8; ++a) ea[a] = es[(ty + 16 * a) * TLD + k];
+#pragma unroll
+        for (int b = 0; b < 8; ++b) lb[b] = ls[(tx + 16 * b) * TLD + k];
+#pragma unroll
+        for (int a = 0; a < 8; ++a)
+#pragma unroll
+            for (int b = 0; b < 8; ++b) acc[a][b] = __fmaf_rn(ea[a], lb[b], acc[a][b]);
+    }
+#pragma unroll
+    for (int a = 0; a < 8; ++a) {
+        const int64_t r = r0 + ty + 16 * a;
+        if (r >= d_out) continue;
+#pragma unroll
+        for (int b = 0; b < 8; ++b) {
+            const int64_t c = c0 + tx + 16 * b;
+            if (c < d_in) {
+                float* o = W + r * d_in + c;
+                *o = __fsub_rn(*o, acc[a][b]);
+            }
+        }
+    }
+}
+
+__global__ void colloss_kernel(const float* __restrict__ E, int64_t d_out, int64_t d_in,
+                               float* __restrict__ col_loss) {
+    const int64_t j = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (j >= d_in) return;
+    double s = 0.0;
+    for (int64_t r = 0; r < d_out; ++r) {
+        const double v = E[r * d_in + j];
+        s += v * v;
+    }
+    col_loss[j] = static_cast<float>(s);
+}
+
+struct ObsWs {
+    float* E;
+    float* gscale;
+    float* gzero;
+};
+
+ObsWs carve(void* ws, int64_t d_out, int64_t d_in) {
+    ObsWs o;
+    o.E = static_cast<float*>(ws);
+    o.gscale = o.E + d_out * d_in;
+    o.gzero = o.gscale + d_out;
+    return o;
+}
+
+}  // namespace
+}  // namespace kq
+
+using namespace kq;
+
+extern "C" size_t kq_obs_quantize_workspace(int64_t d_out, int64_t d_in, int block) {
+    (void)block;
+    if (d_out < 1 || d_in < 1) return 0;
+    return static_cast<size_t>(d_out) * d_in * sizeof(float) + 2 * static_cast<size_t>(d_out) * sizeof(float) + 256;
+}
+
+extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, const float* Lt, int bits,
+                                     int group, int block, uint8_t* codes, float* scale, int32_t* zero,
+                                     float* col_loss, float* pre_q, void* ws, size_t ws_bytes,
+                                     kq_stream_t stream_) {
+    cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+    if (!W || !Lt || !codes || !scale || !zero || d_out < 1 || d_in < 1 || bits < 1 || bits > 8) {
+        set_error("kq_obs_quantize: invalid arguments");
+        return KQ_ERR_INVALID_ARG;
+    }
+    if (block != BLK || (group != 0 && group != block)) {
+        set_error("kq_obs_quantize: block must be %d and group 0 or equal to block", BLK);
+        return KQ_ERR_UNSUPPORTED;
+    }
+    if (!ws || ws_bytes < kq_obs_quantize_workspace(d_out, d_in, block) ||
+        (reinterpret_cast<uintptr_t>(ws) & 15u)) {
+        set_error("kq_obs_quantize: workspace must be 16-byte aligned and hold %zu bytes",
+                  kq_obs_quantize_workspace(d_out, d_in, block));
+        return KQ_ERR_WORKSPACE;
+    }
+    static bool attr = false;
+    if (!attr) {
+        KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     BLK * RLD * 4));
+        KQ_CUDA(cudaFuncSetAttribute(trailing_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     2 * TT * TLD * 4));
+        attr = true;
+    }
+    ObsWs o = carve(ws, d_out, d_in);
+    if (group == 0) {
+        rowgrid_kernel<<<static_cast<unsigned>(cdiv(d_out, 8)), 256, 0, stream>>>(W, d_out, d_in, bits, scale,
+                                                                                zero, o.gscale, o.gzero);
+        KQ_LAUNCH_CHECK("rowgrid_kernel");
+    }
+    const int64_t row_ctas = std::min<int64_t>(cdiv(d_out, 8), static_cast<int64_t>(num_sms()) * 3);
+    for (int64_t i0 = 0; i0 < d_in; i0 += BLK) {
+        const int kb = static_cast<int>(std::min<int64_t>(BLK, d_in - i0));
+        obs_block_kernel<<<static_cast<unsigned>(row_ctas), 256, BLK * RLD * 4, stream>>>(
+            W, d_out, d_in, Lt, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q);
+        KQ_LAUNCH_CHECK("obs_block_kernel");
+        const int64_t rest = d_in - (i0 + kb);
+        if (rest > 0) {
+            dim3 grid(static_cast<unsigned>(cdiv(rest, TT)), static_cast<unsigned>(cdiv(d_out, TT)));
+            trailing_kernel<<<grid, 256, 2 * TT * TLD * 4, stream>>>(W, o.E, Lt, d_out, d_in, i0, kb);
+            KQ_LAUNCH_CHECK("trailing_kernel");
+        }
+    }
+    if (col_loss) {
+        colloss_kernel<<<static_cast<unsigned>(cdiv(d_in, 256)), 256, 0, stream>>>(o.E, d_out, d_in, col_loss);
+        KQ_LAUNCH_CHECK("colloss_kernel");
+    }
+    return KQ_OK;
+}

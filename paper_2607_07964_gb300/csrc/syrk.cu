@@ -1,0 +1,317 @@
+// Stage 1: Kronecker-factor accumulation H (+)= A^T A on the 5th-generation tensor cores.
+//
+// Paper: Sec. 2.1 Eq. (ptq_obj) (H_X = X X^T, tokens as columns there), Sec. 3.1 Eq. (kfac)
+// (H = H_X (x) H_G), Algorithm 1 ("online statistics"). Tokens are rows here, so the
+// factor is A^T A for A [T x d].
+//
+// Design (sm_103a):
+//   * one CTA per 128 x 256 output tile of the lower triangle (row tile i, column tile j,
+//     128 i + 127 >= 256 j); the tile is mirrored into the upper triangle on write-out;
+//   * warp 0 issues TMA loads of 64-token x 64-feature boxes (128-byte swizzle) into a
+//     4-stage ring; both operands are slices of the same A, read MN-major (features
+//     contiguous), so no transpose pass is needed;
+//   * warp 1 allocates 512 TMEM columns and issues tcgen05.mma kind::f16 (bf16 x bf16 ->
+//     fp32, M = 128, N = 256, K = 16) into one of two 256-column accumulators;
+//   * warps 2..9 drain an accumulator every KQ_SYRK_CHUNK_TOKENS tokens into an fp32
+//     running sum held in registers (each thread owns 128 columns of one row), while the
+//     MMAs continue into the other accumulator. This bounds how many tensor-core
+//     additions any fp32 partial sum sees;
+//   * every mbarrier wait is bounded (kq::mbar_wait); a timeout is reported as
+//     -KQ_ERR_TIMEOUT in *info and the CTA drains its own copies and MMAs before exit.
+#include <cstdio>
+#include <cstring>
+
+#include "kq_common.cuh"
+
+namespace kq {
+namespace {
+
+constexpr int BM = 128;   // output rows per tile (MMA M, TMEM lanes)
+constexpr int BN = 256;   // output columns per tile (MMA N)
+constexpr int BK = 64;    // tokens per pipeline stage
+constexpr int STAGES = 4;
+constexpr int BOX_BYTES = BK * 64 * 2;          // one 64-token x 64-feature bf16 box
+constexpr int A_BYTES = BK * BM * 2;            // 16 KB
+constexpr int B_BYTES = BK * BN * 2;            // 32 KB
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;  // 48 KB
+constexpr int NUM_THREADS = 320;                // 10 warps
+constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
+constexpr uint32_t TMEM_COLS = 512;
+// Canonical MN-major SW128 layout: atoms of 64 features x 8 tokens (1 KB). Along the MN
+// dimension atoms are one TMA box apart; along K they are 1 KB apart.
+constexpr uint32_t LBO = BOX_BYTES;   // next 64 features
+constexpr uint32_t SBO = 1024;        // next 8 tokens
+
+__device__ __forceinline__ void tile_of(int bid, int n_row_tiles, int* ti, int* tj) {
+    int j = 0;
+    for (;;) {
+        int cnt = n_row_tiles - 2 * j;
+        if (bid < cnt) break;
+        bid -= cnt;
+        ++j;
+    }
+    *tj = j;
+    *ti = 2 * j + bid;
+}
+
+__device__ __forceinline__ bool wait_noabort(uint64_t* bar, uint32_t parity) {
+    int dummy = 0;
+    return mbar_wait(bar, parity, &dummy);
+}
+
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+syrk_tc_kernel(const __grid_constant__ CUtensorMap tmap, float* __restrict__ H, int d, int T,
+               int n_row_tiles, int chunk_stages, int accumulate, int* info) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+    uint64_t* empty = full + STAGES;
+    uint64_t* tfull = empty + STAGES;
+    uint64_t* tempty = tfull + 2;
+    uint64_t* mma_done = tempty + 2;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    int ti, tj;
+    tile_of(blockIdx.x, n_row_tiles, &ti, &tj);
+    const int i0 = ti * BM;
+    const int j0 = tj * BN;
+    const int nk = (T + BK - 1) / BK;
+    const int nchunks = (nk + chunk_stages - 1) / chunk_stages;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&tfull[b], 1);
+            mbar_init(&tempty[b], 8);
+        }
+        mbar_init(mma_done, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(tmem_slot, TMEM_COLS);
+        tmem_relinquish();
+    }
+    if (warp == 0 && lane == 0) tma_prefetch_desc(&tmap);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            int issued = 0;
+            for (int k = 0; k < nk; ++k) {
+                const int s = k % STAGES;
+                const uint32_t u = static_cast<uint32_t>(k / STAGES);
+                if (!mbar_wait(&empty[s], (u & 1u) ^ 1u, abort_flag)) break;
+                mbar_arrive_expect_tx(&full[s], STAGE_BYTES);
+                uint8_t* a = smem + s * STAGE_BYTES;
+                uint8_t* b = a + A_BYTES;
+                const int y = k * BK;
+                tma_load_2d(a, &tmap, &full[s], i0, y);
+                tma_load_2d(a + BOX_BYTES, &tmap, &full[s], i0 + 64, y);
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    tma_load_2d(b + q * BOX_BYTES, &tmap, &full[s], j0 + 64 * q, y);
+                issued = k + 1;
+            }
+            // Drain: every issued load must have landed before the CTA may exit.
+            for (int k = (issued > STAGES ? issued - STAGES : 0); k < issued; ++k)
+                wait_noabort(&full[k % STAGES], static_cast<uint32_t>(k / STAGES) & 1u);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_bf16_mn_major(BM, BN);
+            int k = 0;
+            bool ok = true;
+            for (int c = 0; c < nchunks && ok; ++c) {
+                const int buf = c & 1;
+                const uint32_t u = static_cast<uint32_t>(c >> 1);
+                if (!mbar_wait(&tempty[buf], (u & 1u) ^ 1u, abort_flag)) break;
+                tc_fence_after();
+                const uint32_t dt = tmem + static_cast<uint32_t>(buf * BN);
+                const int kend = min(nk, (c + 1) * chunk_stages);
+                for (int kk = 0; k < kend; ++k, ++kk) {
+                    const int s = k % STAGES;
+                    if (!mbar_wait(&full[s], static_cast<uint32_t>(k / STAGES) & 1u, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a = smem_u32(smem + s * STAGE_BYTES);
+                    const uint32_t b = a + A_BYTES;
+#pragma unroll
+                    for (int k16 = 0; k16 < BK / 16; ++k16) {
+                        const uint64_t ad = smem_desc_sw128(a + k16 * 2048, LBO, SBO);
+                        const uint64_t bd = smem_desc_sw128(b + k16 * 2048, LBO, SBO);
+                        tc_mma_f16(dt, ad, bd, idesc, (kk > 0 || k16 > 0) ? 1u : 0u);
+                    }
+                    tc_commit(&empty[s]);
+                }
+                if (ok) tc_commit(&tfull[buf]);
+            }
+            // All MMAs must be complete before TMEM is released.
+            tc_commit(mma_done);
+            wait_noabort(mma_done, 0);
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue (8 warps)
+        const int q = warp & 3;                 // TMEM lane quadrant this warp may access
+        const int half = (warp - 2) >> 2;       // which 128 of the 256 columns
+        const int row = i0 + q * 32 + lane;
+        float acc[128];
+#pragma unroll
+        for (int i = 0; i < 128; ++i) acc[i] = 0.0f;
+        bool ok = true;
+        for (int c = 0; c < nchunks; ++c) {
+            const int buf = c & 1;
+            const uint32_t u = static_cast<uint32_t>(c >> 1);
+            ok = mbar_wait(&tfull[buf], u & 1u, abort_flag);
+            ok = __all_sync(0xffffffffu, ok);
+            if (!ok) break;
+            tc_fence_after();
+            const uint32_t base = tmem + (static_cast<uint32_t>(q * 32) << 16) +
+                                  static_cast<uint32_t>(buf * BN + half * 128);
+#pragma unroll
+            for (int p = 0; p < 4; ++p) {
+                float v[32];
+                tmem_ld32(base + p * 32, v);
+                tc_wait_ld();
+#pragma unroll
+                for (int i = 0; i < 32; ++i) acc[p * 32 + i] += v[i];
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty[buf]);
+        }
+        if (ok && !*abort_flag && row < d) {
+            const int cbase = j0 + half * 128;
+#pragma unroll
+            for (int i = 0; i < 128; ++i) {
+                const int col = cbase + i;
+                if (col < d && col <= row) {
+                    float v = acc[i];
+                    float* dst = H + static_cast<int64_t>(row) * d + col;
+                    if (accumulate) v += *dst;
+                    *dst = v;
+                    if (col < row) H[static_cast<int64_t>(col) * d + row] = v;
+                }
+            }
+        }
+    }
+
+    __syncthreads();
+    if (*abort_flag && threadIdx.x == 0) record_error(info, -KQ_ERR_TIMEOUT);
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, TMEM_COLS);
+    }
+}
+
+// tr(H) in fp64 from the diagonal (one CTA).
+__global__ void trace_kernel(const float* __restrict__ H, int64_t n, double* out) {
+    __shared__ double part[32];
+    double s = 0.0;
+    for (int64_t j = threadIdx.x; j < n; j += blockDim.x) s += static_cast<double>(H[j * n + j]);
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = s;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        s = threadIdx.x < blockDim.x / 32 ? part[threadIdx.x] : 0.0;
+        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        if (threadIdx.x == 0) *out = s;
+    }
+}
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    }
+    return fn;
+}
+
+}  // namespace
+
+kq_status launch_trace(const float* H, int64_t n, double* out, cudaStream_t stream) {
+    trace_kernel<<<1, 1024, 0, stream>>>(H, n, out);
+    KQ_LAUNCH_CHECK("trace_kernel");
+    return KQ_OK;
+}
+
+}  // namespace kq
+
+extern "C" kq_status kq_accum_factor(const uint16_t* A, int64_t T, int64_t d, int64_t lda,
+                                     float* H, int accumulate, double* trace, int* info,
+                                     kq_stream_t stream_) {
+    using namespace kq;
+    cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+    if (!H || d < 1 || d > 65536 || T < 0 || (T > 0 && !A) || lda < d) {
+        set_error("kq_accum_factor: invalid arguments (d=%lld T=%lld lda=%lld)", (long long)d,
+                  (long long)T, (long long)lda);
+        return KQ_ERR_INVALID_ARG;
+    }
+    if (T > 0 && ((reinterpret_cast<uintptr_t>(A) & 15u) != 0 || (lda % 8) != 0 || T > (1ll << 31) - 64)) {
+        set_error("kq_accum_factor: A must be 16-byte aligned with lda %% 8 == 0 and T < 2^31");
+        return KQ_ERR_INVALID_ARG;
+    }
+    if (T == 0) {
+        if (!accumulate) KQ_CUDA(cudaMemsetAsync(H, 0, sizeof(float) * d * d, stream));
+    } else {
+        EncodeTiledFn enc = encode_fn();
+        if (!enc) {
+            set_error("kq_accum_factor: cuTensorMapEncodeTiled is unavailable");
+            return KQ_ERR_CUDA;
+        }
+        CUtensorMap tmap;
+        std::memset(&tmap, 0, sizeof(tmap));
+        cuuint64_t gdim[2] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(T)};
+        cuuint64_t gstride[1] = {static_cast<cuuint64_t>(lda) * 2};
+        cuuint32_t box[2] = {64, static_cast<cuuint32_t>(BK)};
+        cuuint32_t estride[2] = {1, 1};
+        CUresult r = enc(&tmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<uint16_t*>(A), gdim,
+                         gstride, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                         CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS) {
+            set_error("kq_accum_factor: cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
+            return KQ_ERR_CUDA;
+        }
+        static bool attr_set = false;
+        if (!attr_set) {
+            KQ_CUDA(cudaFuncSetAttribute(syrk_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         SMEM_BYTES));
+            attr_set = true;
+        }
+        const int n_row = static_cast<int>(cdiv(d, BM));
+        const int n_col = static_cast<int>(cdiv(d, BN));
+        int64_t tiles = 0;
+        for (int j = 0; j < n_col; ++j) tiles += (n_row - 2 * j > 0) ? n_row - 2 * j : 0;
+        const int chunk_stages = KQ_SYRK_CHUNK_TOKENS / BK;
+        syrk_tc_kernel<<<static_cast<unsigned>(tiles), NUM_THREADS, SMEM_BYTES, stream>>>(
+            tmap, H, static_cast<int>(d), static_cast<int>(T), n_row, chunk_stages, accumulate, info);
+        KQ_LAUNCH_CHECK("syrk_tc_kernel");
+    }
+    if (trace) return launch_trace(H, d, trace, stream);
+    return KQ_OK;
+}

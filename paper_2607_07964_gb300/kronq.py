@@ -1,0 +1,231 @@
+"""Thin Python binding of libkronq (include/kronq.h): the same entry points, taking torch
+CUDA tensors. It only checks and marshals arguments (pointers, sizes, the current CUDA
+stream); every step of the computation runs in the library's kernels. There is no CPU
+or PyTorch fallback: if libkronq.so is missing or fails to load, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libkronq.so")
+
+KQ_OK, KQ_ERR_INVALID_ARG, KQ_ERR_UNSUPPORTED, KQ_ERR_NOT_PD = 0, 1, 2, 3
+KQ_ERR_CUDA, KQ_ERR_TIMEOUT, KQ_ERR_WORKSPACE = 4, 5, 6
+KQ_FWD, KQ_INV = 0, 1
+KQ_SYRK_CHUNK_TOKENS = 2048
+
+_lib = None
+
+
+class KronqError(RuntimeError):
+    def __init__(self, status: int, where: str, msg: str):
+        super().__init__(f"{where}: {status_name(status)} ({msg})")
+        self.status = status
+
+
+def lib() -> ctypes.CDLL:
+    """Load libkronq.so (built by paper_2607_07964_gb300.build); raises if it is missing."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is missing: build it with "
+                               "`python -m paper_2607_07964_gb300.build` (needs nvcc)")
+        L = ctypes.CDLL(LIB_PATH)
+        P, I64, I, F, SZ = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_float, ctypes.c_size_t
+        sig = {
+            "kq_last_error": ([], ctypes.c_char_p),
+            "kq_status_name": ([I], ctypes.c_char_p),
+            "kq_version": ([], I),
+            "kq_launch_count": ([], ctypes.c_uint64),
+            "kq_check": ([P, I, P, P], I),
+            "kq_accum_factor": ([P, I64, I64, I64, P, I, P, P, P], I),
+            "kq_compute_scales": ([P, I64, I64, P, P, P, P, P], I),
+            "kq_traces": ([P, P, I64, P, P, I64, P, P], I),
+            "kq_rotate_in": ([P, I64, I64, P, P, P, I, P], I),
+            "kq_rotate_out": ([P, I64, I64, P, P, P, I, P], I),
+            "kq_chol_inv_workspace": ([I64], SZ),
+            "kq_chol_inv": ([P, I64, F, P, P, P, SZ, P], I),
+            "kq_obs_quantize_workspace": ([I64, I64, I], SZ),
+            "kq_obs_quantize": ([P, I64, I64, P, I, I, I, P, P, P, P, P, P, SZ, P], I),
+            "kq_dequant_revert": ([P, P, P, I64, I64, I, P, P, P, P, P, P], I),
+            "kq_proxy_loss_workspace": ([I64, I64], SZ),
+            "kq_proxy_loss": ([P, P, I64, I64, P, P, P, P, SZ, P], I),
+        }
+        for name, (args, res) in sig.items():
+            f = getattr(L, name)
+            f.argtypes = args
+            f.restype = res
+        _lib = L
+    return _lib
+
+
+def status_name(s: int) -> str:
+    return lib().kq_status_name(int(s)).decode()
+
+
+def last_error() -> str:
+    return lib().kq_last_error().decode()
+
+
+def _ok(st: int, where: str) -> None:
+    if st != KQ_OK:
+        raise KronqError(st, where, last_error())
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _need(t, name, dtype, shape=None, contiguous=True):
+    if t is None:
+        return
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} must have shape {tuple(shape)}, got {tuple(t.shape)}")
+    if contiguous and not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+
+
+def version() -> int:
+    return lib().kq_version()
+
+
+def launch_count() -> int:
+    """Kernels launched by libkronq so far in this process."""
+    return int(lib().kq_launch_count())
+
+
+def kq_check(info=None, reset: bool = True, stream=None) -> tuple[int, int]:
+    """Synchronize the stream and read the device error word; returns (status, raw)."""
+    raw = ctypes.c_int(0)
+    st = lib().kq_check(_ptr(info), int(reset), ctypes.byref(raw), _stream(stream))
+    return st, raw.value
+
+
+def kq_accum_factor(A, H, accumulate: bool = False, trace=None, info=None, stream=None) -> None:
+    """H (+)= A^T A; A [T, d] bf16 (row stride may exceed d), H [d, d] fp32."""
+    if A.dim() != 2 or A.stride(1) != 1:
+        raise ValueError("A must be 2-D with unit column stride")
+    T, d = A.shape
+    _need(A, "A", torch.bfloat16, contiguous=False)
+    _need(H, "H", torch.float32, (d, d))
+    _need(trace, "trace", torch.float64)
+    _need(info, "info", torch.int32)
+    _ok(lib().kq_accum_factor(_ptr(A), T, d, A.stride(0), _ptr(H), int(accumulate), _ptr(trace),
+                              _ptr(info), _stream(stream)), "kq_accum_factor")
+
+
+def kq_compute_scales(W, H_X, H_G, s_x, s_g, stream=None) -> None:
+    d_out, d_in = W.shape
+    _need(W, "W", torch.float32)
+    _need(H_X, "H_X", torch.float32, (d_in, d_in))
+    _need(H_G, "H_G", torch.float32, (d_out, d_out))
+    _need(s_x, "s_x", torch.float32, (d_in,))
+    _need(s_g, "s_g", torch.float32, (d_out,))
+    _ok(lib().kq_compute_scales(_ptr(W), d_out, d_in, _ptr(H_X), _ptr(H_G), _ptr(s_x), _ptr(s_g),
+                                _stream(stream)), "kq_compute_scales")
+
+
+def kq_traces(H_X, s_x, H_G, s_g, out, stream=None) -> None:
+    d_in, d_out = H_X.shape[0], H_G.shape[0]
+    _need(H_X, "H_X", torch.float32, (d_in, d_in))
+    _need(H_G, "H_G", torch.float32, (d_out, d_out))
+    _need(s_x, "s_x", torch.float32, (d_in,))
+    _need(s_g, "s_g", torch.float32, (d_out,))
+    _need(out, "out", torch.float64, (6,))
+    _ok(lib().kq_traces(_ptr(H_X), _ptr(s_x), d_in, _ptr(H_G), _ptr(s_g), d_out, _ptr(out),
+                        _stream(stream)), "kq_traces")
+
+
+def kq_rotate_in(W, H_X, s_x, sign_v, direction: int = KQ_FWD, stream=None) -> None:
+    d_out, d_in = W.shape
+    _need(W, "W", torch.float32)
+    _need(H_X, "H_X", torch.float32, (d_in, d_in))
+    _need(s_x, "s_x", torch.float32, (d_in,))
+    _need(sign_v, "sign_v", torch.int8, (d_in,))
+    _ok(lib().kq_rotate_in(_ptr(W), d_out, d_in, _ptr(H_X), _ptr(s_x), _ptr(sign_v), int(direction),
+                           _stream(stream)), "kq_rotate_in")
+
+
+def kq_rotate_out(W, H_G, s_g, sign_u, direction: int = KQ_FWD, stream=None) -> None:
+    d_out, d_in = W.shape
+    _need(W, "W", torch.float32)
+    _need(H_G, "H_G", torch.float32, (d_out, d_out))
+    _need(s_g, "s_g", torch.float32, (d_out,))
+    _need(sign_u, "sign_u", torch.int8, (d_out,))
+    _ok(lib().kq_rotate_out(_ptr(W), d_out, d_in, _ptr(H_G), _ptr(s_g), _ptr(sign_u), int(direction),
+                            _stream(stream)), "kq_rotate_out")
+
+
+def kq_chol_inv_workspace(n: int) -> int:
+    return int(lib().kq_chol_inv_workspace(n))
+
+
+def kq_chol_inv(H, damp_rel: float, Lt, info, ws, stream=None) -> None:
+    n = H.shape[0]
+    _need(H, "H", torch.float32, (n, n))
+    _need(Lt, "Lt", torch.float32, (n, n))
+    _need(info, "info", torch.int32)
+    _need(ws, "ws", torch.uint8)
+    _ok(lib().kq_chol_inv(_ptr(H), n, float(damp_rel), _ptr(Lt), _ptr(info), _ptr(ws),
+                          0 if ws is None else ws.numel(), _stream(stream)), "kq_chol_inv")
+
+
+def kq_obs_quantize_workspace(d_out: int, d_in: int, block: int = 128) -> int:
+    return int(lib().kq_obs_quantize_workspace(d_out, d_in, block))
+
+
+def kq_obs_quantize(W, Lt, bits: int, group: int, block: int, codes, scale, zero, col_loss=None,
+                    pre_q=None, ws=None, stream=None) -> None:
+    d_out, d_in = W.shape
+    ng = 1 if group == 0 else -(-d_in // group)
+    _need(W, "W", torch.float32)
+    _need(Lt, "Lt", torch.float32, (d_in, d_in))
+    _need(codes, "codes", torch.uint8, (d_out, d_in))
+    _need(scale, "scale", torch.float32, (d_out, ng))
+    _need(zero, "zero", torch.int32, (d_out, ng))
+    _need(col_loss, "col_loss", torch.float32, (d_in,))
+    _need(pre_q, "pre_q", torch.float32, (d_out, d_in))
+    _need(ws, "ws", torch.uint8)
+    _ok(lib().kq_obs_quantize(_ptr(W), d_out, d_in, _ptr(Lt), bits, group, block, _ptr(codes),
+                              _ptr(scale), _ptr(zero), _ptr(col_loss), _ptr(pre_q), _ptr(ws),
+                              0 if ws is None else ws.numel(), _stream(stream)), "kq_obs_quantize")
+
+
+def kq_dequant_revert(codes, scale, zero, group: int, s_x, s_g, sign_u, sign_v, W_hat, stream=None):
+    d_out, d_in = codes.shape
+    _need(codes, "codes", torch.uint8)
+    _need(scale, "scale", torch.float32)
+    _need(zero, "zero", torch.int32)
+    _need(W_hat, "W_hat", torch.float32, (d_out, d_in))
+    _ok(lib().kq_dequant_revert(_ptr(codes), _ptr(scale), _ptr(zero), d_out, d_in, group, _ptr(s_x),
+                                _ptr(s_g), _ptr(sign_u), _ptr(sign_v), _ptr(W_hat), _stream(stream)),
+        "kq_dequant_revert")
+
+
+def kq_proxy_loss_workspace(d_out: int, d_in: int) -> int:
+    return int(lib().kq_proxy_loss_workspace(d_out, d_in))
+
+
+def kq_proxy_loss(W, W_hat, H_X, H_G, loss, ws, stream=None) -> None:
+    d_out, d_in = W.shape
+    _need(W, "W", torch.float32)
+    _need(W_hat, "W_hat", torch.float32, (d_out, d_in))
+    _need(H_X, "H_X", torch.float32, (d_in, d_in))
+    _need(H_G, "H_G", torch.float32, (d_out, d_out))
+    _need(loss, "loss", torch.float64, (1,))
+    _need(ws, "ws", torch.uint8)
+    _ok(lib().kq_proxy_loss(_ptr(W), _ptr(W_hat), d_out, d_in, _ptr(H_X), _ptr(H_G), _ptr(loss),
+                            _ptr(ws), ws.numel(), _stream(stream)), "kq_proxy_loss")

@@ -1,0 +1,103 @@
+"""One linear layer through the four stages of the KronQ path (Algorithms 1 and 2, GPTQ
+mode), as a sequence of libkronq calls on one CUDA stream. Buffers and workspaces are
+allocated once (torch provides the device memory) and reused across layers of the same
+shape.
+"""
+from __future__ import annotations
+
+import torch
+
+from . import kronq as kq
+
+STAGES = ("factor_x", "factor_g", "scales_traces", "rotate", "chol", "sweep")
+
+
+class LayerPipeline:
+    """Device buffers for one layer shape and the stage sequence that fills them."""
+
+    def __init__(self, d_out: int, d_in: int, bits: int, group: int, block: int = 128,
+                 damp: float = 0.01, device: str = "cuda", want_col_loss: bool = True):
+        self.d_out, self.d_in, self.bits, self.group, self.block, self.damp = d_out, d_in, bits, group, block, damp
+        f32 = dict(dtype=torch.float32, device=device)
+        ng = 1 if group == 0 else -(-d_in // group)
+        self.HX = torch.empty((d_in, d_in), **f32)
+        self.HG = torch.empty((d_out, d_out), **f32)
+        self.Wp = torch.empty((d_out, d_in), **f32)
+        self.s_x = torch.empty((d_in,), **f32)
+        self.s_g = torch.empty((d_out,), **f32)
+        self.Lt = torch.empty((d_in, d_in), **f32)
+        self.codes = torch.empty((d_out, d_in), dtype=torch.uint8, device=device)
+        self.scale = torch.empty((d_out, ng), **f32)
+        self.zero = torch.empty((d_out, ng), dtype=torch.int32, device=device)
+        self.col_loss = torch.empty((d_in,), **f32) if want_col_loss else None
+        self.traces = torch.zeros((6,), dtype=torch.float64, device=device)
+        self.trace_x = torch.zeros((1,), dtype=torch.float64, device=device)
+        self.trace_g = torch.zeros((1,), dtype=torch.float64, device=device)
+        self.info = torch.zeros((4,), dtype=torch.int32, device=device)
+        self.ws_chol = torch.empty((kq.kq_chol_inv_workspace(d_in),), dtype=torch.uint8, device=device)
+        self.ws_obs = torch.empty((kq.kq_obs_quantize_workspace(d_out, d_in, block),), dtype=torch.uint8,
+                                  device=device)
+
+    def run(self, X, G, W, sign_u, sign_v, stream=None, events=None) -> None:
+        """X [T, d_in] bf16, G [T, d_out] bf16, W [d_out, d_in] fp32 (left unchanged), signs
+        int8. `events`, if given, is a list of len(STAGES) + 1 CUDA events recorded at the
+        stage boundaries on the stream."""
+        s = torch.cuda.current_stream() if stream is None else stream
+
+        def mark(i):
+            if events is not None:
+                events[i].record(s)
+
+        info = self.info[0:1]
+        mark(0)
+        kq.kq_accum_factor(X, self.HX, trace=self.trace_x, info=info, stream=s)        # Alg. 1: H_X
+        mark(1)
+        kq.kq_accum_factor(G, self.HG, trace=self.trace_g, info=info, stream=s)        # H_G
+        mark(2)
+        kq.kq_compute_scales(W, self.HX, self.HG, self.s_x, self.s_g, stream=s)      # Eq. (rescale)
+        kq.kq_traces(self.HX, self.s_x, self.HG, self.s_g, self.traces, stream=s)     # Eq. (sensitivity)
+        mark(3)
+        with torch.cuda.stream(s):
+            self.Wp.copy_(W)
+        kq.kq_rotate_in(self.Wp, self.HX, self.s_x, sign_v, kq.KQ_FWD, stream=s)     # Eq. (biip), V side
+        kq.kq_rotate_out(self.Wp, self.HG, self.s_g, sign_u, kq.KQ_FWD, stream=s)    # U side; H_G released
+        mark(4)
+        kq.kq_chol_inv(self.HX, self.damp, self.Lt, self.info[1:2], self.ws_chol, stream=s)  # Alg. 2
+        mark(5)
+        kq.kq_obs_quantize(self.Wp, self.Lt, self.bits, self.group, self.block, self.codes, self.scale,
+                           self.zero, self.col_loss, None, self.ws_obs, stream=s)   # Alg. 2 sweep
+        mark(6)
+
+    def check(self, stream=None) -> None:
+        """Raise if a kernel reported a device-side error (timeout, non-PD pivot)."""
+        for k in range(2):
+            st, raw = kq.kq_check(self.info[k:k + 1], reset=True, stream=stream)
+            if st != kq.KQ_OK:
+                raise kq.KronqError(st, "pipeline", f"device word {raw}")
+
+    def run_host(self, X_h, G_h, W_h, su_h, sv_h, codes_h, scale_h, zero_h, stream=None) -> tuple[int, int]:
+        """End-to-end call with HOST buffers (pinned for asynchronous copies): copy the
+        layer's inputs to the device, run the four stages, copy codes and grids back.
+        Enqueued on `stream`; the caller synchronizes. Returns (bytes in, bytes out)."""
+        s = torch.cuda.current_stream() if stream is None else stream
+        dev = self.HX.device
+        if getattr(self, "_stage", None) is None or self._stage["X"].shape != X_h.shape:
+            self._stage = {
+                "X": torch.empty(X_h.shape, dtype=X_h.dtype, device=dev),
+                "G": torch.empty(G_h.shape, dtype=G_h.dtype, device=dev),
+                "W": torch.empty(W_h.shape, dtype=W_h.dtype, device=dev),
+                "su": torch.empty(su_h.shape, dtype=su_h.dtype, device=dev),
+                "sv": torch.empty(sv_h.shape, dtype=sv_h.dtype, device=dev),
+            }
+        st = self._stage
+        with torch.cuda.stream(s):
+            for k, h in (("X", X_h), ("G", G_h), ("W", W_h), ("su", su_h), ("sv", sv_h)):
+                st[k].copy_(h, non_blocking=True)
+        self.run(st["X"], st["G"], st["W"], st["su"], st["sv"], stream=s)
+        with torch.cuda.stream(s):
+            codes_h.copy_(self.codes, non_blocking=True)
+            scale_h.copy_(self.scale, non_blocking=True)
+            zero_h.copy_(self.zero, non_blocking=True)
+        nin = sum(t.numel() * t.element_size() for t in (X_h, G_h, W_h, su_h, sv_h))
+        nout = sum(t.numel() * t.element_size() for t in (codes_h, scale_h, zero_h))
+        return nin, nout

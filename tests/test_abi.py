@@ -1,0 +1,80 @@
+"""Host-side checks of the C ABI that need no GPU: the library builds and loads, exports
+every entry point include/kronq.h declares, and rejects bad arguments on the host before
+touching the device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "kronq.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2607_07964_gb300 import build, kronq
+    build.build()
+    return kronq.lib()
+
+
+def declared_symbols():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"KQ_API\s+[\w\s\*]+?\b(kq_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_symbols()
+    for required in ["kq_accum_factor", "kq_compute_scales", "kq_rotate_in", "kq_rotate_out",
+                     "kq_chol_inv", "kq_obs_quantize", "kq_traces", "kq_check"]:
+        assert required in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in declared_symbols():
+        assert hasattr(lib, name), name
+        assert ctypes.cast(getattr(lib, name), ctypes.c_void_p).value
+
+
+def test_status_names_and_version(lib):
+    from paper_2607_07964_gb300 import kronq
+    assert kronq.status_name(0) == "KQ_OK"
+    assert kronq.status_name(3) == "KQ_ERR_NOT_PD"
+    assert kronq.version() >= 100
+
+
+def test_workspace_queries(lib):
+    from paper_2607_07964_gb300 import kronq
+    assert kronq.kq_chol_inv_workspace(256) >= 2 * 256 * 256 * 4
+    assert kronq.kq_chol_inv_workspace(200) >= 2 * 256 * 256 * 4   # padded to the block size
+    assert kronq.kq_chol_inv_workspace(0) == 0
+    assert kronq.kq_obs_quantize_workspace(64, 256, 128) >= 64 * 256 * 4
+    assert kronq.kq_proxy_loss_workspace(8, 8) >= 3 * 64 * 4
+
+
+def test_host_side_argument_errors(lib):
+    """Calls with invalid arguments return before any CUDA call (safe without a GPU)."""
+    from paper_2607_07964_gb300 import kronq as K
+    P = ctypes.c_void_p
+    fake = P(256)   # never dereferenced: validation fails first
+    assert lib.kq_accum_factor(None, 16, 8, 8, None, 0, None, None, None) == K.KQ_ERR_INVALID_ARG
+    assert lib.kq_accum_factor(fake, 16, 8, 4, fake, 0, None, None, None) == K.KQ_ERR_INVALID_ARG  # lda < d
+    assert lib.kq_accum_factor(P(258), 16, 8, 8, fake, 0, None, None, None) == K.KQ_ERR_INVALID_ARG
+    assert lib.kq_chol_inv(None, 8, 0.01, None, None, None, 0, None) == K.KQ_ERR_INVALID_ARG
+    assert lib.kq_chol_inv(fake, 8, 0.01, fake, None, None, 0, None) == K.KQ_ERR_WORKSPACE
+    assert lib.kq_chol_inv(fake, 8, -1.0, fake, None, fake, 1 << 20, None) == K.KQ_ERR_INVALID_ARG
+    # rotation sizes without a Hadamard construction
+    assert lib.kq_rotate_in(fake, 4, 100, None, None, fake, 0, None) == K.KQ_ERR_UNSUPPORTED
+    assert lib.kq_rotate_out(fake, 100, 4, None, None, fake, 0, None) == K.KQ_ERR_UNSUPPORTED
+    assert lib.kq_rotate_in(fake, 4, 28 * 2048, None, None, fake, 0, None) == K.KQ_ERR_UNSUPPORTED
+    # sweep: block must be 128 and group in {0, block}
+    args = [fake, 4, 256, fake, 4, 64, 128, fake, fake, fake, None, None, fake, 1 << 30, None]
+    assert lib.kq_obs_quantize(*args) == K.KQ_ERR_UNSUPPORTED
+    args[6] = 64
+    args[5] = 0
+    assert lib.kq_obs_quantize(*args) == K.KQ_ERR_UNSUPPORTED
+    args[6], args[4] = 128, 9
+    assert lib.kq_obs_quantize(*args) == K.KQ_ERR_INVALID_ARG
+    args[4], args[13] = 4, 16
+    assert lib.kq_obs_quantize(*args) == K.KQ_ERR_WORKSPACE
+    assert "workspace" in K.last_error()
