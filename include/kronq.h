@@ -87,7 +87,7 @@ KQ_API kq_status kq_check(int* info, int reset, int* pivot_out, kq_stream_t stre
  *   T == 0 gives H = 0 (accumulate = 0) or leaves H unchanged. `info` (nullable) receives
  *   -KQ_ERR_TIMEOUT if a pipeline wait gave up.
  * ---------------------------------------------------------------------------------- */
-#define KQ_SYRK_CHUNK_TOKENS 2048
+#define KQ_SYRK_CHUNK_TOKENS 512
 KQ_API kq_status kq_accum_factor(const uint16_t* A, int64_t T, int64_t d, int64_t lda, float* H,
                           int accumulate, double* trace, int* info, kq_stream_t stream);
 

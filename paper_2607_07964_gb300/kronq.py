@@ -16,7 +16,7 @@ LIB_PATH = os.path.join(_HERE, "libkronq.so")
 KQ_OK, KQ_ERR_INVALID_ARG, KQ_ERR_UNSUPPORTED, KQ_ERR_NOT_PD = 0, 1, 2, 3
 KQ_ERR_CUDA, KQ_ERR_TIMEOUT, KQ_ERR_WORKSPACE = 4, 5, 6
 KQ_FWD, KQ_INV = 0, 1
-KQ_SYRK_CHUNK_TOKENS = 2048
+KQ_SYRK_CHUNK_TOKENS = 512
 
 _lib = None
 
