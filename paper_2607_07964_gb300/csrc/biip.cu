@@ -91,27 +91,61 @@ __device__ __forceinline__ void mix28(const float (&x)[28], float (&y)[28]) {
     }
 }
 
+// In-register Walsh-Hadamard transform of R = 2, 4 or 8 values (natural order).
+template <int R>
+__device__ __forceinline__ void fwht_reg(float (&x)[8]) {
+#pragma unroll
+    for (int h = 1; h < R; h <<= 1)
+#pragma unroll
+        for (int i = 0; i < R; ++i)
+            if ((i & h) == 0) {
+                const float a = x[i], b = x[i + h];
+                x[i] = a + b;
+                x[i + h] = a - b;
+            }
+}
+__device__ __forceinline__ void fwht_reg_r(float (&x)[8], int r) {
+    if (r == 8) fwht_reg<8>(x);
+    else if (r == 4) fwht_reg<4>(x);
+    else if (r == 2) fwht_reg<2>(x);
+}
+
+// One radix-r pass (span h = 2^lgh) of the Walsh-Hadamard transform over a shared vector
+// of n elements (every h*r-aligned block independently). Index math is shifts and masks.
+__device__ __forceinline__ void fwht_pass(float* v, int n, int lgh, int lgr) {
+    const int h = 1 << lgh, r = 1 << lgr;
+    for (int g = threadIdx.x; g < (n >> lgr); g += blockDim.x) {
+        const int base = ((g >> lgh) << (lgh + lgr)) | (g & (h - 1));
+        float x[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+            if (q < r) x[q] = v[base + q * h];
+        fwht_reg_r(x, r);
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+            if (q < r) v[base + q * h] = x[q];
+    }
+}
+
 // ------------------------------------------------------------------ row transform
 // For each row of M [rows x n]: v <- pre (.) v; v <- (H_28 (x) H_P) v (or H_P); row <-
 // post (.) v / sqrt(n). One CTA per row (grid-stride); n floats of shared memory.
-__global__ void __launch_bounds__(512) rht_rows_kernel(float* __restrict__ M, int64_t rows, int n, int P, int has28,
+// The power-of-two part runs as radix-8 passes (one barrier per pass).
+__global__ void __launch_bounds__(512) rht_rows_kernel(float* __restrict__ M, int64_t rows, int n, int lgP, int has28,
                                 int pre_mode, int post_mode, const int8_t* __restrict__ sign,
                                 const float* __restrict__ s, float inv_sqrt_n) {
     extern __shared__ float v[];
+    const int P = 1 << lgP;
     for (int64_t r = blockIdx.x; r < rows; r += gridDim.x) {
         float* row = M + r * n;
         for (int j = threadIdx.x; j < n; j += blockDim.x)
             v[j] = row[j] * factor(pre_mode, sign, s, j);
         __syncthreads();
-        // Butterflies with span h < P stay inside each P-aligned chunk: I_28 (x) H_P.
-        for (int h = 1; h < P; h <<= 1) {
-            for (int t = threadIdx.x; t < n / 2; t += blockDim.x) {
-                const int i = (t / h) * 2 * h + (t % h);
-                const float a = v[i], b = v[i + h];
-                v[i] = a + b;
-                v[i + h] = a - b;
-            }
+        for (int lgh = 0; lgh < lgP;) {   // I_28 (x) H_P: passes stay inside P-aligned chunks
+            const int lgr = min(3, lgP - lgh);
+            fwht_pass(v, n, lgh, lgr);
             __syncthreads();
+            lgh += lgr;
         }
         if (has28) {   // H_28 (x) I_P
             for (int b = threadIdx.x; b < P; b += blockDim.x) {
@@ -133,20 +167,24 @@ __global__ void __launch_bounds__(512) rht_rows_kernel(float* __restrict__ M, in
 // --------------------------------------------------------------- column transform
 // One radix stage along the row index of M [n x ncols]: for every group base = hi*R*S + lo
 // (lo < S) and CW-column strip, rows base + i*S (i < R) are transformed along i by H_R
-// (R a power of two) or H_28 (R == 28). Shared memory [R][CW].
-__global__ void __launch_bounds__(256) rht_cols_kernel(float* __restrict__ M, int n, int64_t ncols, int R, int S, int CW,
-                                int pre_mode, int post_mode, const int8_t* __restrict__ sign,
+// (R a power of two, as radix-8 passes) or H_28 (R == 28). Shared memory [R][CW], CW a
+// power of two; index math is shifts and masks.
+__global__ void __launch_bounds__(256) rht_cols_kernel(float* __restrict__ M, int n, int64_t ncols, int R, int S,
+                                int lgCW, int pre_mode, int post_mode, const int8_t* __restrict__ sign,
                                 const float* __restrict__ s, float post_scale) {
     extern __shared__ float v[];
-    const int64_t nstrips = (ncols + CW - 1) / CW;
+    const int CW = 1 << lgCW;
+    const int64_t nstrips = (ncols + CW - 1) >> lgCW;
     const int64_t ngroups = n / R;
+    int lgR = 0;
+    while ((1 << lgR) < R) ++lgR;
     for (int64_t w = blockIdx.x; w < ngroups * nstrips; w += gridDim.x) {
         const int64_t g = w / nstrips;
-        const int64_t c0 = (w % nstrips) * CW;
+        const int64_t c0 = (w - g * nstrips) << lgCW;
         const int64_t base = (g / S) * static_cast<int64_t>(R) * S + (g % S);
         const int cw = static_cast<int>(min(static_cast<int64_t>(CW), ncols - c0));
         for (int e = threadIdx.x; e < R * CW; e += blockDim.x) {
-            const int i = e / CW, c = e % CW;
+            const int i = e >> lgCW, c = e & (CW - 1);
             const int64_t r = base + static_cast<int64_t>(i) * S;
             v[e] = c < cw ? M[r * ncols + c0 + c] * factor(pre_mode, sign, s, r) : 0.0f;
         }
@@ -162,19 +200,27 @@ __global__ void __launch_bounds__(256) rht_cols_kernel(float* __restrict__ M, in
             }
             __syncthreads();
         } else {
-            for (int h = 1; h < R; h <<= 1) {
-                for (int e = threadIdx.x; e < (R / 2) * CW; e += blockDim.x) {
-                    const int t = e / CW, c = e % CW;
-                    const int i = (t / h) * 2 * h + (t % h);
-                    const float a = v[i * CW + c], b = v[(i + h) * CW + c];
-                    v[i * CW + c] = a + b;
-                    v[(i + h) * CW + c] = a - b;
+            for (int lgh = 0; lgh < lgR;) {
+                const int lgr = min(3, lgR - lgh);
+                const int h = 1 << lgh, rr = 1 << lgr;
+                for (int gg = threadIdx.x; gg < ((R >> lgr) << lgCW); gg += blockDim.x) {
+                    const int c = gg & (CW - 1), gi = gg >> lgCW;
+                    const int bi = ((gi >> lgh) << (lgh + lgr)) | (gi & (h - 1));
+                    float x[8];
+#pragma unroll
+                    for (int q = 0; q < 8; ++q)
+                        if (q < rr) x[q] = v[((bi + q * h) << lgCW) + c];
+                    fwht_reg_r(x, rr);
+#pragma unroll
+                    for (int q = 0; q < 8; ++q)
+                        if (q < rr) v[((bi + q * h) << lgCW) + c] = x[q];
                 }
                 __syncthreads();
+                lgh += lgr;
             }
         }
         for (int e = threadIdx.x; e < R * CW; e += blockDim.x) {
-            const int i = e / CW, c = e % CW;
+            const int i = e >> lgCW, c = e & (CW - 1);
             if (c < cw) {
                 const int64_t r = base + static_cast<int64_t>(i) * S;
                 M[r * ncols + c0 + c] = v[e] * (factor(post_mode, sign, s, r) * post_scale);
@@ -327,7 +373,7 @@ kq_status rows_transform(float* M, int64_t rows, int64_t n, int pre, int post, c
     const int64_t grid = std::min<int64_t>(rows, static_cast<int64_t>(num_sms()) * 16);
     if (grid > 0) {
         rht_rows_kernel<<<static_cast<unsigned>(grid), threads, smem, stream>>>(
-            M, rows, static_cast<int>(n), p.P, p.has28, pre, post, sign, s,
+            M, rows, static_cast<int>(n), log2i(p.P), p.has28, pre, post, sign, s,
             static_cast<float>(1.0 / sqrt(static_cast<double>(n))));
         KQ_LAUNCH_CHECK("rht_rows_kernel");
     }
@@ -366,7 +412,7 @@ kq_status cols_transform(float* M, int64_t n, int64_t ncols, int pre, int post, 
         const int64_t items = (n / R[st]) * cdiv(ncols, CW);
         const int64_t grid = std::min<int64_t>(items, static_cast<int64_t>(num_sms()) * 8);
         rht_cols_kernel<<<static_cast<unsigned>(grid), 256, smem, stream>>>(
-            M, static_cast<int>(n), ncols, R[st], S[st], CW, st == 0 ? pre : F_NONE,
+            M, static_cast<int>(n), ncols, R[st], S[st], log2i(CW), st == 0 ? pre : F_NONE,
             st == ns - 1 ? post : F_NONE, sign, s, st == ns - 1 ? post_scale : 1.0f);
         KQ_LAUNCH_CHECK("rht_cols_kernel");
     }

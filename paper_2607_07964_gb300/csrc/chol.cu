@@ -72,57 +72,140 @@ __global__ void prep_kernel(const float* __restrict__ H, int64_t n, int64_t npad
 }
 
 // ---------------------------------------------------------------- diag block
-// Factor A_kk (lower) = C C^T in shared memory, write C to A_kk and C^-1 to Z_kk.
-// A non-positive (or NaN) pivot records its index in H's own numbering (1-based).
+// Warp-level Cholesky of a 32 x 32 SPD block held one row per lane (r[c] = S[lane][c],
+// c <= lane). Returns the first non-positive pivot's index, or -1.
+__device__ __forceinline__ int warp_chol32(float (&r)[32], int lane) {
+    int bad = -1;
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+        const float p = __shfl_sync(0xffffffffu, r[j], j);
+        if (!(p > 0.0f) && bad < 0) bad = j;
+        const float d = sqrtf(p);
+        if (lane == j) r[j] = d;
+        else if (lane > j) r[j] = __fdiv_rn(r[j], d);
+#pragma unroll
+        for (int k = j + 1; k < 32; ++k) {
+            const float lkj = __shfl_sync(0xffffffffu, r[j], k);
+            if (lane >= k) r[k] = fmaf(-r[j], lkj, r[k]);
+        }
+    }
+    return bad;
+}
+
+// Warp-level inverse of a lower-triangular 32 x 32 block L (shared, row stride ld): lane c
+// solves L x = e_c by forward substitution and writes column c of X = L^-1.
+__device__ __forceinline__ void warp_trinv32(const float* L, int ld, float* X, int ldx, int lane) {
+    float x[32];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+        float s = (i == lane) ? 1.0f : 0.0f;
+#pragma unroll
+        for (int m = 0; m < i; ++m) s = fmaf(-L[i * ld + m], x[m], s);
+        x[i] = (i >= lane) ? __fdiv_rn(s, L[i * ld + i]) : 0.0f;
+    }
+#pragma unroll
+    for (int i = 0; i < 32; ++i) X[i * ldx + lane] = x[i];
+}
+
+constexpr int SB = 32;                  // sub-block of the diagonal block
+constexpr int TLDD = SB + 1;
+constexpr size_t DIAG_SMEM = (2 * TILE_FLOATS + NB * TLDD) * sizeof(float);
+
+// Factor A_kk = C C^T and invert C, both in shared memory, as 4 x 4 sub-blocks of 32:
+//   for p: warp 0 factors and inverts sub-block (p, p); all warps form the panel
+//          C_qp = A_qp C_pp^-T (q > p) and update A_qr -= C_qp C_rp^T (p < r <= q);
+//   then X_qp = -X_qq sum_{r=p}^{q-1} C_qr X_rp by increasing q - p.
+// Writes C to A_kk and X = C^-1 to Z_kk. A non-positive pivot records its index in H's
+// own numbering (1-based).
 __global__ void __launch_bounds__(512) chol_diag_kernel(Work w, int64_t n, int64_t npad, int k, int* info) {
     extern __shared__ float sm[];
-    float* a = sm;                  // [NB][LD]
-    float* x = sm + TILE_FLOATS;    // [NB][LD] inverse
+    float* a = sm;                        // [NB][LD]  A_kk -> C
+    float* x = sm + TILE_FLOATS;          // [NB][LD]  C^-1
+    float* t = sm + 2 * TILE_FLOATS;      // [NB][TLDD] temporaries
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int64_t off = static_cast<int64_t>(k) * NB;
-    for (int e = threadIdx.x; e < NB * NB; e += blockDim.x) {
+    for (int e = tid; e < NB * NB; e += blockDim.x) {
         const int r = e / NB, c = e % NB;
         a[r * LD + c] = c <= r ? w.A[(off + r) * npad + off + c] : 0.0f;
     }
     __syncthreads();
-    __shared__ float dj;
-    for (int j = 0; j < NB; ++j) {
-        if (threadIdx.x == 0) {
-            const float p = a[j * LD + j];
-            if (!(p > 0.0f)) {
-                const int64_t rev = off + j;
+    for (int p = 0; p < NB / SB; ++p) {
+        const int o = p * SB;
+        if (warp == 0) {
+            float r[32];
+#pragma unroll
+            for (int c = 0; c < 32; ++c) r[c] = a[(o + lane) * LD + o + c];
+            const int bad = warp_chol32(r, lane);
+            if (bad >= 0 && lane == 0) {
+                const int64_t rev = off + o + bad;
                 if (rev < n) record_error(info, static_cast<int>(n - rev));
             }
-            dj = sqrtf(p);
-            a[j * LD + j] = dj;
+#pragma unroll
+            for (int c = 0; c < 32; ++c) a[(o + lane) * LD + o + c] = c <= lane ? r[c] : 0.0f;
+            __syncwarp();
+            warp_trinv32(a + o * LD + o, LD, x + o * LD + o, LD, lane);
         }
         __syncthreads();
-        const float d = dj;
-        for (int r = j + 1 + threadIdx.x; r < NB; r += blockDim.x) a[r * LD + j] = a[r * LD + j] / d;
+        const int nr = NB - o - SB;       // rows below the sub-block
+        // panel into t: C_qp[ro][c] = sum_{m <= c} A[ro][o + m] X_pp[c][m]
+        for (int e = tid; e < nr * SB; e += blockDim.x) {
+            const int ro = e / SB, c = e % SB;
+            const float* arow = a + (o + SB + ro) * LD + o;
+            const float* xrow = x + (o + c) * LD + o;
+            float s = 0.0f;
+            for (int m = 0; m <= c; ++m) s = fmaf(arow[m], xrow[m], s);
+            t[ro * TLDD + c] = s;
+        }
         __syncthreads();
-        const int m = NB - 1 - j;   // trailing size
-        for (int e = threadIdx.x; e < m * m; e += blockDim.x) {
-            const int r = j + 1 + e / m, c = j + 1 + e % m;
-            if (c <= r) a[r * LD + c] = fmaf(-a[r * LD + j], a[c * LD + j], a[r * LD + c]);
+        for (int e = tid; e < nr * SB; e += blockDim.x) {
+            const int ro = e / SB, c = e % SB;
+            a[(o + SB + ro) * LD + o + c] = t[ro * TLDD + c];
+        }
+        __syncthreads();
+        // trailing update of the lower part of rows/cols [o + SB, NB)
+        for (int e = tid; e < nr * nr; e += blockDim.x) {
+            const int ro = e / nr, co = e % nr;
+            if (co > ro) continue;
+            const float* ar = a + (o + SB + ro) * LD + o;
+            const float* ac = a + (o + SB + co) * LD + o;
+            float s = 0.0f;
+#pragma unroll 8
+            for (int m = 0; m < SB; ++m) s = fmaf(ar[m], ac[m], s);
+            a[(o + SB + ro) * LD + o + SB + co] -= s;
         }
         __syncthreads();
     }
-    // Inverse of the lower-triangular C: thread c solves C x = e_c (x lower: rows >= c).
-    for (int c = threadIdx.x; c < NB; c += blockDim.x) {
-        for (int r = 0; r < NB; ++r) {
-            if (r < c) {
-                x[r * LD + c] = 0.0f;
-                continue;
+    // off-diagonal blocks of X = C^-1, by distance d = q - p
+    for (int d = 1; d < NB / SB; ++d) {
+        const int nblk = NB / SB - d;
+        // T_qp = sum_{r=p}^{q-1} C_qr X_rp   (stored in t rows [b*SB, b*SB+SB), b = p)
+        for (int e = tid; e < nblk * SB * SB; e += blockDim.x) {
+            const int b = e / (SB * SB), i = (e / SB) % SB, c = e % SB;
+            const int pp = b, qq = b + d;
+            float s = 0.0f;
+            for (int r2 = pp; r2 < qq; ++r2) {
+                const float* crow = a + (qq * SB + i) * LD + r2 * SB;
+                const float* xcol = x + (r2 * SB) * LD + pp * SB + c;
+                for (int m = 0; m < SB; ++m) s = fmaf(crow[m], xcol[m * LD], s);
             }
-            float s = (r == c) ? 1.0f : 0.0f;
-            for (int m2 = c; m2 < r; ++m2) s = fmaf(-a[r * LD + m2], x[m2 * LD + c], s);
-            x[r * LD + c] = s / a[r * LD + r];
+            t[(b * SB + i) * TLDD + c] = s;
         }
+        __syncthreads();
+        // X_qp = -X_qq T_qp   (X_qq lower)
+        for (int e = tid; e < nblk * SB * SB; e += blockDim.x) {
+            const int b = e / (SB * SB), i = (e / SB) % SB, c = e % SB;
+            const int pp = b, qq = b + d;
+            const float* xrow = x + (qq * SB + i) * LD + qq * SB;
+            float s = 0.0f;
+            for (int m = 0; m <= i; ++m) s = fmaf(xrow[m], t[(b * SB + m) * TLDD + c], s);
+            x[(qq * SB + i) * LD + pp * SB + c] = -s;
+        }
+        __syncthreads();
     }
-    __syncthreads();
-    for (int e = threadIdx.x; e < NB * NB; e += blockDim.x) {
+    for (int e = tid; e < NB * NB; e += blockDim.x) {
         const int r = e / NB, c = e % NB;
         w.A[(off + r) * npad + off + c] = c <= r ? a[r * LD + c] : 0.0f;
-        w.Z[(off + r) * npad + off + c] = x[r * LD + c];
+        w.Z[(off + r) * npad + off + c] = c <= r ? x[r * LD + c] : 0.0f;
     }
 }
 
@@ -277,7 +360,7 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
     static bool attr = false;
     if (!attr) {
         KQ_CUDA(cudaFuncSetAttribute(chol_diag_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     static_cast<int>(GEMM_SMEM)));
+                                     static_cast<int>(DIAG_SMEM)));
         KQ_CUDA(cudaFuncSetAttribute(chol_panel_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(GEMM_SMEM)));
         KQ_CUDA(cudaFuncSetAttribute(chol_update_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -291,7 +374,7 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
     prep_kernel<<<static_cast<unsigned>(pgrid), 256, 0, stream>>>(H, n, npad, damp_rel, w.dsum, w.A, w.Z);
     KQ_LAUNCH_CHECK("prep_kernel");
     for (int k = 0; k < nbk; ++k) {
-        chol_diag_kernel<<<1, 512, GEMM_SMEM, stream>>>(w, n, npad, k, info);
+        chol_diag_kernel<<<1, 512, DIAG_SMEM, stream>>>(w, n, npad, k, info);
         KQ_LAUNCH_CHECK("chol_diag_kernel");
         if (nbk > 1) {
             chol_panel_kernel<<<nbk - 1, GEMM_THREADS, GEMM_SMEM, stream>>>(w, npad, k);

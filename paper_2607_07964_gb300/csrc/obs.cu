@@ -13,7 +13,7 @@
 //   trailing  acc = fma(E_k, R_kc, acc) over ascending k; w_c = w_c - acc
 // Kernels:
 //   rowgrid_kernel   per-row grid (group = 0) from the whole row before the sweep
-//   obs_block_kernel one warp per row; the block's R (128 x 128) in shared memory
+//   obs_block_kernel four rows per warp; the block's R (128 x 128) in shared memory
 //   trailing_kernel  128 x 128 output tiles, K = block, shared-memory operands
 //   colloss_kernel   col_loss[j] = sum over rows of E_j^2, fixed order, fp64
 #include <math.h>
@@ -26,7 +26,6 @@ namespace {
 constexpr int BLK = 128;          // block size B (Algorithm 2); the only supported value
 constexpr int RLD = BLK + 1;
 constexpr int TT = 128;           // trailing tile
-constexpr int TLD = BLK + 1;
 
 struct Grid {
     float scale, zero;
@@ -78,9 +77,24 @@ __global__ void rowgrid_kernel(const float* __restrict__ W, int64_t d_out, int64
     }
 }
 
-// One block [i0, e) of the sweep for all rows. Warp per row (grid-stride over rows); lane l
-// holds columns i0 + 32 s + l (s = 0..3) in registers.
-__global__ void __launch_bounds__(256) obs_block_kernel(
+// One block [i0, e) of the sweep for all rows. Four rows per warp: lanes 8g..8g+7 hold
+// row 4 w + g, lane position lp holding columns i0 + 8 t + lp (t = 0..15) in registers.
+// Per column j the owner lane broadcasts w_j inside its 8-lane group; every lane of the
+// group computes the (identical) quantization, then updates its own later columns.
+constexpr int LPR = 8;                 // lanes per row
+constexpr int CPL = BLK / LPR;         // columns per lane
+constexpr int RPW = 32 / LPR;          // rows per warp
+
+__device__ __forceinline__ float group_min(float v) {
+    for (int o = LPR / 2; o > 0; o >>= 1) v = fminf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+__device__ __forceinline__ float group_max(float v) {
+    for (int o = LPR / 2; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+
+__global__ void __launch_bounds__(128) obs_block_kernel(
     const float* __restrict__ W, int64_t d_out, int64_t d_in, const float* __restrict__ Lt, int64_t i0,
     int bits, int group, const float* __restrict__ gscale, const float* __restrict__ gzero,
     uint8_t* __restrict__ codes, float* __restrict__ scale, int32_t* __restrict__ zero,
@@ -96,90 +110,101 @@ __global__ void __launch_bounds__(256) obs_block_kernel(
     __syncthreads();
     const float maxq = static_cast<float>((1 << bits) - 1);
     const int lane = threadIdx.x & 31;
+    const int lp = lane & (LPR - 1);
+    const int gbase = lane & ~(LPR - 1);
     const int64_t ngroups = group ? (d_in + group - 1) / group : 1;
     const int warps = blockDim.x / 32;
-    for (int64_t r = static_cast<int64_t>(blockIdx.x) * warps + threadIdx.x / 32; r < d_out;
-         r += static_cast<int64_t>(gridDim.x) * warps) {
+    for (int64_t r0 = (static_cast<int64_t>(blockIdx.x) * warps + threadIdx.x / 32) * RPW; r0 < d_out;
+         r0 += static_cast<int64_t>(gridDim.x) * warps * RPW) {
+        const int64_t r = r0 + lane / LPR;
+        const bool live = r < d_out;
         const float* wr = W + r * d_in + i0;
-        float w[4], e[4];
-        uint32_t qv[4];
+        float w[CPL], e[CPL], pq[CPL];
+        uint32_t qv[CPL];
 #pragma unroll
-        for (int s = 0; s < 4; ++s) {
-            const int c = 32 * s + lane;
-            w[s] = c < nb ? wr[c] : 0.0f;
-            e[s] = 0.0f;
-            qv[s] = 0;
+        for (int t = 0; t < CPL; ++t) {
+            const int c = LPR * t + lp;
+            w[t] = (live && c < nb) ? wr[c] : 0.0f;
+            e[t] = 0.0f;
+            pq[t] = 0.0f;
+            qv[t] = 0;
         }
         Grid g;
         if (group) {
             float mn = 0.0f, mx = 0.0f;
 #pragma unroll
-            for (int s = 0; s < 4; ++s)
-                if (32 * s + lane < nb) {
-                    mn = fminf(mn, w[s]);
-                    mx = fmaxf(mx, w[s]);
+            for (int t = 0; t < CPL; ++t)
+                if (LPR * t + lp < nb) {
+                    mn = fminf(mn, w[t]);
+                    mx = fmaxf(mx, w[t]);
                 }
-            g = make_grid(warp_min(mn), warp_max(mx), maxq);
-            if (lane == 0) {
+            g = make_grid(group_min(mn), group_max(mx), maxq);
+            if (live && lp == 0) {
                 const int64_t gi = r * ngroups + i0 / group;
                 scale[gi] = g.scale;
                 zero[gi] = static_cast<int32_t>(g.zero);
             }
         } else {
-            g.scale = gscale[r];
-            g.zero = gzero[r];
+            g.scale = live ? gscale[r] : 1.0f;
+            g.zero = live ? gzero[r] : 0.0f;
         }
-        float pq[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
-        for (int s = 0; s < 4; ++s) {
-            for (int jl = 0; jl < 32; ++jl) {
-                const int j = 32 * s + jl;
-                if (j >= nb) break;
-                const float wj = __shfl_sync(0xffffffffu, w[s], jl);
-                float q = __fadd_rn(rintf(__fdiv_rn(wj, g.scale)), g.zero);
-                q = fminf(fmaxf(q, 0.0f), maxq);
-                const float what = __fmul_rn(g.scale, __fsub_rn(q, g.zero));
+        for (int q = 0; q < CPL; ++q) {
+#pragma unroll
+            for (int jl = 0; jl < LPR; ++jl) {
+                const int j = LPR * q + jl;
+                if (j >= nb) continue;   // uniform across the warp
+                const float wj = __shfl_sync(0xffffffffu, w[q], gbase | jl);
+                float qq = __fadd_rn(rintf(__fdiv_rn(wj, g.scale)), g.zero);
+                qq = fminf(fmaxf(qq, 0.0f), maxq);
+                const float what = __fmul_rn(g.scale, __fsub_rn(qq, g.zero));
                 const float err = __fdiv_rn(__fsub_rn(wj, what), Rs[j * RLD + j]);
-                if (lane == jl) {
-                    e[s] = err;
-                    qv[s] = static_cast<uint32_t>(q);
-                    pq[s] = wj;
+                if (lp == jl) {
+                    e[q] = err;
+                    qv[q] = static_cast<uint32_t>(qq);
+                    pq[q] = wj;
                 }
 #pragma unroll
-                for (int t = s; t < 4; ++t) {
-                    const int k = 32 * t + lane;
+                for (int t = q; t < CPL; ++t) {
+                    const int k = LPR * t + lp;
                     if (k > j) w[t] = __fmaf_rn(-err, Rs[j * RLD + k], w[t]);
                 }
             }
         }
+        if (live) {
 #pragma unroll
-        for (int s = 0; s < 4; ++s) {
-            const int c = 32 * s + lane;
-            if (c < nb) {
-                codes[r * d_in + i0 + c] = static_cast<uint8_t>(qv[s]);
-                E[r * d_in + i0 + c] = e[s];
-                if (pre_q) pre_q[r * d_in + i0 + c] = pq[s];
+            for (int t = 0; t < CPL; ++t) {
+                const int c = LPR * t + lp;
+                if (c < nb) {
+                    codes[r * d_in + i0 + c] = static_cast<uint8_t>(qv[t]);
+                    E[r * d_in + i0 + c] = e[t];
+                    if (pre_q) pre_q[r * d_in + i0 + c] = pq[t];
+                }
             }
         }
     }
 }
 
-// W[:, e0:] -= E[:, i0:e0] R[i0:e0, e0:], R[k][c] = Lt[c][k]. Tile: 128 rows x 128 columns.
-// acc = fma(E_k, R_kc, acc) over ascending k, then w = w - acc.
+// W[:, e0:] -= E[:, i0:e0] R[i0:e0, e0:], R[k][c] = Lt[c][k]. Tile: 128 rows x 128 columns,
+// operands transposed in shared memory (k-major) so each thread reads its 8 rows and 8
+// columns as 128-bit words. Thread (ty, tx) owns rows {4ty..4ty+3, 64+4ty..64+4ty+3} and
+// the same pattern of columns. acc = fma(E_k, R_kc, acc) over ascending k; w = w - acc.
+constexpr int TLK = TT + 4;   // row stride of the k-major tiles (16-byte aligned)
+
 __global__ void __launch_bounds__(256) trailing_kernel(float* __restrict__ W, const float* __restrict__ E,
                                                        const float* __restrict__ Lt, int64_t d_out,
                                                        int64_t d_in, int64_t i0, int kb) {
-    extern __shared__ float sm[];
-    float* es = sm;                 // [TT][TLD]  es[r][k] = E[r0 + r][i0 + k]
-    float* ls = sm + TT * TLD;      // [TT][TLD]  ls[c][k] = Lt[c0 + c][i0 + k]
+    extern __shared__ __align__(16) float sm[];
+    float* es = sm;                 // [BLK][TLK]  es[k][r] = E[r0 + r][i0 + k]
+    float* ls = sm + BLK * TLK;     // [BLK][TLK]  ls[k][c] = Lt[c0 + c][i0 + k]
     const int64_t e0 = i0 + kb;
     const int64_t r0 = static_cast<int64_t>(blockIdx.y) * TT;
     const int64_t c0 = e0 + static_cast<int64_t>(blockIdx.x) * TT;
     for (int idx = threadIdx.x; idx < TT * BLK; idx += blockDim.x) {
         const int a = idx / BLK, k = idx % BLK;
         const int64_t r = r0 + a, c = c0 + a;
-        es[a * TLD + k] = (k < kb && r < d_out) ? E[r * d_in + i0 + k] : 0.0f;
-        ls[a * TLD + k] = (k < kb && c < d_in) ? Lt[c * d_in + i0 + k] : 0.0f;
+        es[k * TLK + a] = (k < kb && r < d_out) ? E[r * d_in + i0 + k] : 0.0f;
+        ls[k * TLK + a] = (k < kb && c < d_in) ? Lt[c * d_in + i0 + k] : 0.0f;
     }
     __syncthreads();
     const int ty = threadIdx.x / 16, tx = threadIdx.x % 16;
@@ -189,11 +214,12 @@ __global__ void __launch_bounds__(256) trailing_kernel(float* __restrict__ W, co
 #pragma unroll
         for (int b = 0; b < 8; ++b) acc[a][b] = 0.0f;
     for (int k = 0; k < kb; ++k) {
-        float ea[8], lb[8];
-#pragma unroll
-        for (int a = 0; a < 8; ++a) ea[a] = es[(ty + 16 * a) * TLD + k];
-#pragma unroll
-        for (int b = 0; b < 8; ++b) lb[b] = ls[(tx + 16 * b) * TLD + k];
+        const float4 ea0 = *reinterpret_cast<const float4*>(es + k * TLK + 4 * ty);
+        const float4 ea1 = *reinterpret_cast<const float4*>(es + k * TLK + 64 + 4 * ty);
+        const float4 lb0 = *reinterpret_cast<const float4*>(ls + k * TLK + 4 * tx);
+        const float4 lb1 = *reinterpret_cast<const float4*>(ls + k * TLK + 64 + 4 * tx);
+        const float ea[8] = {ea0.x, ea0.y, ea0.z, ea0.w, ea1.x, ea1.y, ea1.z, ea1.w};
+        const float lb[8] = {lb0.x, lb0.y, lb0.z, lb0.w, lb1.x, lb1.y, lb1.z, lb1.w};
 #pragma unroll
         for (int a = 0; a < 8; ++a)
 #pragma unroll
@@ -201,11 +227,11 @@ __global__ void __launch_bounds__(256) trailing_kernel(float* __restrict__ W, co
     }
 #pragma unroll
     for (int a = 0; a < 8; ++a) {
-        const int64_t r = r0 + ty + 16 * a;
+        const int64_t r = r0 + (a < 4 ? 4 * ty + a : 64 + 4 * ty + a - 4);
         if (r >= d_out) continue;
 #pragma unroll
         for (int b = 0; b < 8; ++b) {
-            const int64_t c = c0 + tx + 16 * b;
+            const int64_t c = c0 + (b < 4 ? 4 * tx + b : 64 + 4 * tx + b - 4);
             if (c < d_in) {
                 float* o = W + r * d_in + c;
                 *o = __fsub_rn(*o, acc[a][b]);
@@ -214,16 +240,34 @@ __global__ void __launch_bounds__(256) trailing_kernel(float* __restrict__ W, co
     }
 }
 
+// col_loss[j] = sum over rows of E[r][j]^2: fp32 partials over 32 rows, fp64 across them,
+// fixed order. Block (32, 8): 32 columns, 8 row lanes.
 __global__ void colloss_kernel(const float* __restrict__ E, int64_t d_out, int64_t d_in,
                                float* __restrict__ col_loss) {
-    const int64_t j = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-    if (j >= d_in) return;
-    double s = 0.0;
-    for (int64_t r = 0; r < d_out; ++r) {
-        const double v = E[r * d_in + j];
-        s += v * v;
+    __shared__ double part[8][33];
+    const int64_t j = static_cast<int64_t>(blockIdx.x) * 32 + threadIdx.x;
+    double acc = 0.0;
+    if (j < d_in) {
+        float p = 0.0f;
+        int cnt = 0;
+        for (int64_t r = threadIdx.y; r < d_out; r += 8) {
+            const float v = E[r * d_in + j];
+            p = fmaf(v, v, p);
+            if (++cnt == 32) {
+                acc += p;
+                p = 0.0f;
+                cnt = 0;
+            }
+        }
+        acc += p;
     }
-    col_loss[j] = static_cast<float>(s);
+    part[threadIdx.y][threadIdx.x] = acc;
+    __syncthreads();
+    if (threadIdx.y == 0 && j < d_in) {
+        double a = 0.0;
+        for (int y = 0; y < 8; ++y) a += part[y][threadIdx.x];
+        col_loss[j] = static_cast<float>(a);
+    }
 }
 
 struct ObsWs {
@@ -275,7 +319,7 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
         KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      BLK * RLD * 4));
         KQ_CUDA(cudaFuncSetAttribute(trailing_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     2 * TT * TLD * 4));
+                                     2 * BLK * TLK * 4));
         attr = true;
     }
     ObsWs o = carve(ws, d_out, d_in);
@@ -284,21 +328,21 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
                                                                                 zero, o.gscale, o.gzero);
         KQ_LAUNCH_CHECK("rowgrid_kernel");
     }
-    const int64_t row_ctas = std::min<int64_t>(cdiv(d_out, 8), static_cast<int64_t>(num_sms()) * 3);
+    const int64_t row_ctas = std::min<int64_t>(cdiv(d_out, 4 * RPW), static_cast<int64_t>(num_sms()) * 3);
     for (int64_t i0 = 0; i0 < d_in; i0 += BLK) {
         const int kb = static_cast<int>(std::min<int64_t>(BLK, d_in - i0));
-        obs_block_kernel<<<static_cast<unsigned>(row_ctas), 256, BLK * RLD * 4, stream>>>(
+        obs_block_kernel<<<static_cast<unsigned>(row_ctas), 128, BLK * RLD * 4, stream>>>(
             W, d_out, d_in, Lt, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q);
         KQ_LAUNCH_CHECK("obs_block_kernel");
         const int64_t rest = d_in - (i0 + kb);
         if (rest > 0) {
             dim3 grid(static_cast<unsigned>(cdiv(rest, TT)), static_cast<unsigned>(cdiv(d_out, TT)));
-            trailing_kernel<<<grid, 256, 2 * TT * TLD * 4, stream>>>(W, o.E, Lt, d_out, d_in, i0, kb);
+            trailing_kernel<<<grid, 256, 2 * BLK * TLK * 4, stream>>>(W, o.E, Lt, d_out, d_in, i0, kb);
             KQ_LAUNCH_CHECK("trailing_kernel");
         }
     }
     if (col_loss) {
-        colloss_kernel<<<static_cast<unsigned>(cdiv(d_in, 256)), 256, 0, stream>>>(o.E, d_out, d_in, col_loss);
+        colloss_kernel<<<static_cast<unsigned>(cdiv(d_in, 32)), dim3(32, 8), 0, stream>>>(o.E, d_out, d_in, col_loss);
         KQ_LAUNCH_CHECK("colloss_kernel");
     }
     return KQ_OK;
