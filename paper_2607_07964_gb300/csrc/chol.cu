@@ -17,6 +17,7 @@
 #include <math.h>
 
 #include "kq_common.cuh"
+#include "tile_gemm.cuh"
 
 namespace kq {
 namespace {
@@ -24,8 +25,6 @@ namespace {
 constexpr int NB = 128;
 constexpr int LD = NB + 1;                      // padded shared-memory row
 constexpr int TILE_FLOATS = NB * LD;
-constexpr int GEMM_THREADS = 256;               // 16 x 16 threads, 8 x 8 outputs each
-constexpr size_t GEMM_SMEM = 2 * TILE_FLOATS * sizeof(float);
 
 struct Work {
     float* A;      // npad x npad, reversed damped H -> C (lower)
@@ -72,39 +71,42 @@ __global__ void prep_kernel(const float* __restrict__ H, int64_t n, int64_t npad
 }
 
 // ---------------------------------------------------------------- diag block
-// Warp-level Cholesky of a 32 x 32 SPD block held one row per lane (r[c] = S[lane][c],
-// c <= lane). Returns the first non-positive pivot's index, or -1.
-__device__ __forceinline__ int warp_chol32(float (&r)[32], int lane) {
+// One warp factors the 32 x 32 SPD block s (row stride ld, lower part used) in place,
+// lane i owning row i, then writes X = C^-1 to x (lane c solves C x = e_c). The loops stay
+// rolled so the code is small. Returns the first non-positive pivot's index, or -1.
+__device__ __forceinline__ int warp_chol_inv32(float* s, float* x, int ld, int lane) {
     int bad = -1;
-#pragma unroll
+#pragma unroll 1
     for (int j = 0; j < 32; ++j) {
-        const float p = __shfl_sync(0xffffffffu, r[j], j);
+        const float p = s[j * ld + j];
         if (!(p > 0.0f) && bad < 0) bad = j;
         const float d = sqrtf(p);
-        if (lane == j) r[j] = d;
-        else if (lane > j) r[j] = __fdiv_rn(r[j], d);
-#pragma unroll
-        for (int k = j + 1; k < 32; ++k) {
-            const float lkj = __shfl_sync(0xffffffffu, r[j], k);
-            if (lane >= k) r[k] = fmaf(-r[j], lkj, r[k]);
+        __syncwarp();
+        float lij = 0.0f;
+        if (lane > j) {
+            lij = __fdiv_rn(s[lane * ld + j], d);
+            s[lane * ld + j] = lij;
+        } else if (lane == j) {
+            s[j * ld + j] = d;
         }
+        __syncwarp();
+#pragma unroll 4
+        for (int k = j + 1; k <= lane; ++k) s[lane * ld + k] = fmaf(-lij, s[k * ld + j], s[lane * ld + k]);
+        __syncwarp();
     }
-    return bad;
-}
-
-// Warp-level inverse of a lower-triangular 32 x 32 block L (shared, row stride ld): lane c
-// solves L x = e_c by forward substitution and writes column c of X = L^-1.
-__device__ __forceinline__ void warp_trinv32(const float* L, int ld, float* X, int ldx, int lane) {
-    float x[32];
-#pragma unroll
+#pragma unroll 1
     for (int i = 0; i < 32; ++i) {
-        float s = (i == lane) ? 1.0f : 0.0f;
-#pragma unroll
-        for (int m = 0; m < i; ++m) s = fmaf(-L[i * ld + m], x[m], s);
-        x[i] = (i >= lane) ? __fdiv_rn(s, L[i * ld + i]) : 0.0f;
+        float v = 0.0f;
+        if (i >= lane) {
+            float acc = (i == lane) ? 1.0f : 0.0f;
+#pragma unroll 4
+            for (int m = lane; m < i; ++m) acc = fmaf(-s[i * ld + m], x[m * ld + lane], acc);
+            v = __fdiv_rn(acc, s[i * ld + i]);
+        }
+        x[i * ld + lane] = v;
     }
-#pragma unroll
-    for (int i = 0; i < 32; ++i) X[i * ldx + lane] = x[i];
+    __syncwarp();
+    return bad;
 }
 
 constexpr int SB = 32;                  // sub-block of the diagonal block
@@ -132,18 +134,13 @@ __global__ void __launch_bounds__(512) chol_diag_kernel(Work w, int64_t n, int64
     for (int p = 0; p < NB / SB; ++p) {
         const int o = p * SB;
         if (warp == 0) {
-            float r[32];
-#pragma unroll
-            for (int c = 0; c < 32; ++c) r[c] = a[(o + lane) * LD + o + c];
-            const int bad = warp_chol32(r, lane);
+            const int bad = warp_chol_inv32(a + o * LD + o, x + o * LD + o, LD, lane);
             if (bad >= 0 && lane == 0) {
                 const int64_t rev = off + o + bad;
                 if (rev < n) record_error(info, static_cast<int>(n - rev));
             }
-#pragma unroll
-            for (int c = 0; c < 32; ++c) a[(o + lane) * LD + o + c] = c <= lane ? r[c] : 0.0f;
-            __syncwarp();
-            warp_trinv32(a + o * LD + o, LD, x + o * LD + o, LD, lane);
+            // zero the strict upper part of the factored sub-block
+            for (int c = lane + 1; c < SB; ++c) a[(o + lane) * LD + o + c] = 0.0f;
         }
         __syncthreads();
         const int nr = NB - o - SB;       // rows below the sub-block
@@ -209,70 +206,41 @@ __global__ void __launch_bounds__(512) chol_diag_kernel(Work w, int64_t n, int64
     }
 }
 
-// ---------------------------------------------------------------- tile GEMM core
-// acc[a][b] += sum_m P[r_a][m] * Q(m, c_b), r_a = ty + 16 a, c_b = tx + 16 b, m ascending.
-// Q(m, c) = TRANSQ ? q[c][m] : q[m][c]. Both operands are [NB][LD] shared tiles.
-template <bool TRANSQ>
-__device__ __forceinline__ void tile_mac(const float* p, const float* q, float (&acc)[8][8], int ty,
-                                         int tx) {
-#pragma unroll 2
-    for (int m = 0; m < NB; ++m) {
-        float pa[8], qb[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) pa[i] = p[(ty + 16 * i) * LD + m];
-#pragma unroll
-        for (int j = 0; j < 8; ++j) qb[j] = TRANSQ ? q[(tx + 16 * j) * LD + m] : q[m * LD + tx + 16 * j];
-#pragma unroll
-        for (int i = 0; i < 8; ++i)
-#pragma unroll
-            for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(pa[i], qb[j], acc[i][j]);
-    }
-}
-
-__device__ __forceinline__ void load_tile(float* dst, const float* src, int64_t ld_src) {
-    for (int e = threadIdx.x; e < NB * NB; e += blockDim.x) {
-        const int r = e / NB, c = e % NB;
-        dst[r * LD + c] = src[r * ld_src + c];
-    }
-}
-
 // --------------------------------------------------------------------- panel
-// CTA b < k: Z_kb <- C_kk^-1 Z_kb.  CTA b >= k: i = b + 1, A_ik <- A_ik C_kk^-T.
-__global__ void __launch_bounds__(GEMM_THREADS) chol_panel_kernel(Work w, int64_t npad, int k) {
-    extern __shared__ float sm[];
-    float* cinv = sm;
-    float* t = sm + TILE_FLOATS;
+// CTA b < k: Z_kb <- C_kk^-1 Z_kb.  CTA b >= k: i = b + 1, A_ik <- A_ik C_kk^-T. The whole
+// input tile is consumed before the in-place write (gemm_tile ends with a barrier).
+__global__ void __launch_bounds__(G_THREADS, 2) chol_panel_kernel(Work w, int64_t npad, int k) {
+    extern __shared__ __align__(16) float sm[];
     const int b = blockIdx.x;
     const int64_t off = static_cast<int64_t>(k) * NB;
-    load_tile(cinv, w.Z + off * npad + off, npad);
-    const bool zpart = b < k;
-    float* blk = zpart ? w.Z + off * npad + static_cast<int64_t>(b) * NB
-                       : w.A + static_cast<int64_t>(b + 1) * NB * npad + off;
-    load_tile(t, blk, npad);
-    __syncthreads();
-    const int ty = threadIdx.x / 16, tx = threadIdx.x % 16;
+    const float* cinv = w.Z + off * npad + off;
     float acc[8][8];
+    float* out;
+    bool nn;
+    if (b < k) {
+        out = w.Z + off * npad + static_cast<int64_t>(b) * NB;
+        gemm_tile<true, true>(cinv, npad, NB, out, npad, NB, NB, acc, sm);   // C^-1 x B (B N-contiguous)
+        nn = true;
+    } else {
+        out = w.A + static_cast<int64_t>(b + 1) * NB * npad + off;
+        gemm_tile<false, true>(out, npad, NB, cinv, npad, NB, NB, acc, sm);  // A x (C^-1)^T
+        nn = false;
+    }
+    const int ty = threadIdx.x >> 4, tx = threadIdx.x & 15;
 #pragma unroll
     for (int i = 0; i < 8; ++i)
 #pragma unroll
-        for (int j = 0; j < 8; ++j) acc[i][j] = 0.0f;
-    if (zpart)
-        tile_mac<false>(cinv, t, acc, ty, tx);   // C^-1 (rows) x B
-    else
-        tile_mac<true>(t, cinv, acc, ty, tx);    // A x (C^-1)^T
-#pragma unroll
-    for (int i = 0; i < 8; ++i)
-#pragma unroll
-        for (int j = 0; j < 8; ++j) blk[static_cast<int64_t>(ty + 16 * i) * npad + tx + 16 * j] = acc[i][j];
+        for (int j = 0; j < 8; ++j) {
+            const int c = nn ? gt_col<true>(tx, j) : gt_col<false>(tx, j);
+            out[static_cast<int64_t>(gt_row(ty, i)) * npad + c] = acc[i][j];
+        }
 }
 
 // -------------------------------------------------------------------- update
 // Tiles (i, j), k < i < nbk, 0 <= j <= i:
 //   j > k : A_ij -= C_ik C_jk^T;     j <= k : Z_ij -= C_ik Z_kj.
-__global__ void __launch_bounds__(GEMM_THREADS) chol_update_kernel(Work w, int64_t npad, int k) {
-    extern __shared__ float sm[];
-    float* p = sm;
-    float* q = sm + TILE_FLOATS;
+__global__ void __launch_bounds__(G_THREADS, 2) chol_update_kernel(Work w, int64_t npad, int k) {
+    extern __shared__ __align__(16) float sm[];
     int bid = blockIdx.x;
     int i = k + 1;
     while (bid >= i + 1) {
@@ -281,29 +249,21 @@ __global__ void __launch_bounds__(GEMM_THREADS) chol_update_kernel(Work w, int64
     }
     const int j = bid;
     const int64_t ko = static_cast<int64_t>(k) * NB;
-    load_tile(p, w.A + static_cast<int64_t>(i) * NB * npad + ko, npad);   // C_ik
+    const float* cik = w.A + static_cast<int64_t>(i) * NB * npad + ko;
     const bool apart = j > k;
-    if (apart)
-        load_tile(q, w.A + static_cast<int64_t>(j) * NB * npad + ko, npad);   // C_jk
-    else
-        load_tile(q, w.Z + ko * npad + static_cast<int64_t>(j) * NB, npad);   // Z_kj
-    __syncthreads();
-    const int ty = threadIdx.x / 16, tx = threadIdx.x % 16;
     float acc[8][8];
-#pragma unroll
-    for (int a = 0; a < 8; ++a)
-#pragma unroll
-        for (int b = 0; b < 8; ++b) acc[a][b] = 0.0f;
     if (apart)
-        tile_mac<true>(p, q, acc, ty, tx);
+        gemm_tile<false, true>(cik, npad, NB, w.A + static_cast<int64_t>(j) * NB * npad + ko, npad, NB, NB, acc, sm);
     else
-        tile_mac<false>(p, q, acc, ty, tx);
+        gemm_tile<true, true>(cik, npad, NB, w.Z + ko * npad + static_cast<int64_t>(j) * NB, npad, NB, NB, acc, sm);
     float* out = (apart ? w.A : w.Z) + static_cast<int64_t>(i) * NB * npad + static_cast<int64_t>(j) * NB;
+    const int ty = threadIdx.x >> 4, tx = threadIdx.x & 15;
 #pragma unroll
     for (int a = 0; a < 8; ++a)
 #pragma unroll
         for (int b = 0; b < 8; ++b) {
-            float* o = out + static_cast<int64_t>(ty + 16 * a) * npad + tx + 16 * b;
+            const int c = apart ? gt_col<false>(tx, b) : gt_col<true>(tx, b);
+            float* o = out + static_cast<int64_t>(gt_row(ty, a)) * npad + c;
             *o = *o - acc[a][b];
         }
 }
@@ -362,9 +322,9 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
         KQ_CUDA(cudaFuncSetAttribute(chol_diag_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(DIAG_SMEM)));
         KQ_CUDA(cudaFuncSetAttribute(chol_panel_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     static_cast<int>(GEMM_SMEM)));
+                                     static_cast<int>(G_SMEM)));
         KQ_CUDA(cudaFuncSetAttribute(chol_update_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     static_cast<int>(GEMM_SMEM)));
+                                     static_cast<int>(G_SMEM)));
         attr = true;
     }
     diag_sum_kernel<<<1, 1024, 0, stream>>>(H, n, w.dsum);
@@ -377,13 +337,13 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
         chol_diag_kernel<<<1, 512, DIAG_SMEM, stream>>>(w, n, npad, k, info);
         KQ_LAUNCH_CHECK("chol_diag_kernel");
         if (nbk > 1) {
-            chol_panel_kernel<<<nbk - 1, GEMM_THREADS, GEMM_SMEM, stream>>>(w, npad, k);
+            chol_panel_kernel<<<nbk - 1, G_THREADS, G_SMEM, stream>>>(w, npad, k);
             KQ_LAUNCH_CHECK("chol_panel_kernel");
         }
         int64_t tiles = 0;
         for (int i = k + 1; i < nbk; ++i) tiles += i + 1;
         if (tiles > 0) {
-            chol_update_kernel<<<static_cast<unsigned>(tiles), GEMM_THREADS, GEMM_SMEM, stream>>>(w, npad, k);
+            chol_update_kernel<<<static_cast<unsigned>(tiles), G_THREADS, G_SMEM, stream>>>(w, npad, k);
             KQ_LAUNCH_CHECK("chol_update_kernel");
         }
     }

@@ -14,18 +14,18 @@
 // Kernels:
 //   rowgrid_kernel   per-row grid (group = 0) from the whole row before the sweep
 //   obs_block_kernel four rows per warp; the block's R (128 x 128) in shared memory
-//   trailing_kernel  128 x 128 output tiles, K = block, shared-memory operands
+//   trailing_kernel  128 x 128 output tiles of the shared tile GEMM (tile_gemm.cuh)
 //   colloss_kernel   col_loss[j] = sum over rows of E_j^2, fixed order, fp64
 #include <math.h>
 
 #include "kq_common.cuh"
+#include "tile_gemm.cuh"
 
 namespace kq {
 namespace {
 
 constexpr int BLK = 128;          // block size B (Algorithm 2); the only supported value
 constexpr int RLD = BLK + 1;
-constexpr int TT = 128;           // trailing tile
 
 struct Grid {
     float scale, zero;
@@ -119,15 +119,11 @@ __global__ void __launch_bounds__(128) obs_block_kernel(
         const int64_t r = r0 + lane / LPR;
         const bool live = r < d_out;
         const float* wr = W + r * d_in + i0;
-        float w[CPL], e[CPL], pq[CPL];
-        uint32_t qv[CPL];
+        float w[CPL];
 #pragma unroll
         for (int t = 0; t < CPL; ++t) {
             const int c = LPR * t + lp;
             w[t] = (live && c < nb) ? wr[c] : 0.0f;
-            e[t] = 0.0f;
-            pq[t] = 0.0f;
-            qv[t] = 0;
         }
         Grid g;
         if (group) {
@@ -148,93 +144,71 @@ __global__ void __launch_bounds__(128) obs_block_kernel(
             g.scale = live ? gscale[r] : 1.0f;
             g.zero = live ? gzero[r] : 0.0f;
         }
-#pragma unroll
+        // Slot q of the block is always w[0]: after its 8 columns the registers shift down
+        // by one, which keeps the loop rolled (compact code) with register-only indexing.
+#pragma unroll 1
         for (int q = 0; q < CPL; ++q) {
+            float e_cur = 0.0f, pq_cur = 0.0f;
+            uint32_t q_cur = 0;
 #pragma unroll
             for (int jl = 0; jl < LPR; ++jl) {
                 const int j = LPR * q + jl;
-                if (j >= nb) continue;   // uniform across the warp
-                const float wj = __shfl_sync(0xffffffffu, w[q], gbase | jl);
-                float qq = __fadd_rn(rintf(__fdiv_rn(wj, g.scale)), g.zero);
-                qq = fminf(fmaxf(qq, 0.0f), maxq);
-                const float what = __fmul_rn(g.scale, __fsub_rn(qq, g.zero));
-                const float err = __fdiv_rn(__fsub_rn(wj, what), Rs[j * RLD + j]);
-                if (lp == jl) {
-                    e[q] = err;
-                    qv[q] = static_cast<uint32_t>(qq);
-                    pq[q] = wj;
-                }
+                if (j < nb) {   // uniform across the warp
+                    const float wj = __shfl_sync(0xffffffffu, w[0], gbase | jl);
+                    float qq = __fadd_rn(rintf(__fdiv_rn(wj, g.scale)), g.zero);
+                    qq = fminf(fmaxf(qq, 0.0f), maxq);
+                    const float what = __fmul_rn(g.scale, __fsub_rn(qq, g.zero));
+                    const float err = __fdiv_rn(__fsub_rn(wj, what), Rs[j * RLD + j]);
+                    if (lp == jl) {
+                        e_cur = err;
+                        q_cur = static_cast<uint32_t>(qq);
+                        pq_cur = wj;
+                    }
+                    const float* rrow = Rs + j * RLD + LPR * q + lp;
 #pragma unroll
-                for (int t = q; t < CPL; ++t) {
-                    const int k = LPR * t + lp;
-                    if (k > j) w[t] = __fmaf_rn(-err, Rs[j * RLD + k], w[t]);
+                    for (int t = 0; t < CPL; ++t) {
+                        if (t < CPL - q && LPR * (q + t) + lp > j) w[t] = __fmaf_rn(-err, rrow[LPR * t], w[t]);
+                    }
                 }
             }
-        }
-        if (live) {
-#pragma unroll
-            for (int t = 0; t < CPL; ++t) {
-                const int c = LPR * t + lp;
-                if (c < nb) {
-                    codes[r * d_in + i0 + c] = static_cast<uint8_t>(qv[t]);
-                    E[r * d_in + i0 + c] = e[t];
-                    if (pre_q) pre_q[r * d_in + i0 + c] = pq[t];
-                }
+            const int c = LPR * q + lp;
+            if (live && c < nb) {
+                codes[r * d_in + i0 + c] = static_cast<uint8_t>(q_cur);
+                E[r * d_in + i0 + c] = e_cur;
+                if (pre_q) pre_q[r * d_in + i0 + c] = pq_cur;
             }
+#pragma unroll
+            for (int t = 0; t + 1 < CPL; ++t) w[t] = w[t + 1];
+            w[CPL - 1] = 0.0f;
         }
     }
 }
 
-// W[:, e0:] -= E[:, i0:e0] R[i0:e0, e0:], R[k][c] = Lt[c][k]. Tile: 128 rows x 128 columns,
-// operands transposed in shared memory (k-major) so each thread reads its 8 rows and 8
-// columns as 128-bit words. Thread (ty, tx) owns rows {4ty..4ty+3, 64+4ty..64+4ty+3} and
-// the same pattern of columns. acc = fma(E_k, R_kc, acc) over ascending k; w = w - acc.
-constexpr int TLK = TT + 4;   // row stride of the k-major tiles (16-byte aligned)
-
-__global__ void __launch_bounds__(256) trailing_kernel(float* __restrict__ W, const float* __restrict__ E,
-                                                       const float* __restrict__ Lt, int64_t d_out,
-                                                       int64_t d_in, int64_t i0, int kb) {
+// W[:, e0:] -= E[:, i0:e0] R[i0:e0, e0:] with R[k][c] = Lt[c][k]: 128 x 128 output tiles
+// of the shared tile GEMM (acc = fma(E_k, R_kc, acc) over ascending k), then w = w - acc.
+template <bool VEC>
+__global__ void __launch_bounds__(G_THREADS, 2) trailing_kernel(float* __restrict__ W, const float* __restrict__ E,
+                                                                const float* __restrict__ Lt, int64_t d_out,
+                                                                int64_t d_in, int64_t i0, int kb) {
     extern __shared__ __align__(16) float sm[];
-    float* es = sm;                 // [BLK][TLK]  es[k][r] = E[r0 + r][i0 + k]
-    float* ls = sm + BLK * TLK;     // [BLK][TLK]  ls[k][c] = Lt[c0 + c][i0 + k]
     const int64_t e0 = i0 + kb;
-    const int64_t r0 = static_cast<int64_t>(blockIdx.y) * TT;
-    const int64_t c0 = e0 + static_cast<int64_t>(blockIdx.x) * TT;
-    for (int idx = threadIdx.x; idx < TT * BLK; idx += blockDim.x) {
-        const int a = idx / BLK, k = idx % BLK;
-        const int64_t r = r0 + a, c = c0 + a;
-        es[k * TLK + a] = (k < kb && r < d_out) ? E[r * d_in + i0 + k] : 0.0f;
-        ls[k * TLK + a] = (k < kb && c < d_in) ? Lt[c * d_in + i0 + k] : 0.0f;
-    }
-    __syncthreads();
-    const int ty = threadIdx.x / 16, tx = threadIdx.x % 16;
+    const int64_t r0 = static_cast<int64_t>(blockIdx.y) * GT;
+    const int64_t c0 = e0 + static_cast<int64_t>(blockIdx.x) * GT;
+    const int arows = static_cast<int>(min(static_cast<int64_t>(GT), d_out - r0));
+    const int bcols = static_cast<int>(min(static_cast<int64_t>(GT), d_in - c0));
     float acc[8][8];
+    gemm_tile<false, VEC>(E + r0 * d_in + i0, d_in, arows, Lt + c0 * d_in + i0, d_in, bcols, kb, acc, sm);
+    const int ty = threadIdx.x >> 4, tx = threadIdx.x & 15;
 #pragma unroll
-    for (int a = 0; a < 8; ++a)
+    for (int i = 0; i < 8; ++i) {
+        const int rr = gt_row(ty, i);
+        if (rr >= arows) continue;
 #pragma unroll
-        for (int b = 0; b < 8; ++b) acc[a][b] = 0.0f;
-    for (int k = 0; k < kb; ++k) {
-        const float4 ea0 = *reinterpret_cast<const float4*>(es + k * TLK + 4 * ty);
-        const float4 ea1 = *reinterpret_cast<const float4*>(es + k * TLK + 64 + 4 * ty);
-        const float4 lb0 = *reinterpret_cast<const float4*>(ls + k * TLK + 4 * tx);
-        const float4 lb1 = *reinterpret_cast<const float4*>(ls + k * TLK + 64 + 4 * tx);
-        const float ea[8] = {ea0.x, ea0.y, ea0.z, ea0.w, ea1.x, ea1.y, ea1.z, ea1.w};
-        const float lb[8] = {lb0.x, lb0.y, lb0.z, lb0.w, lb1.x, lb1.y, lb1.z, lb1.w};
-#pragma unroll
-        for (int a = 0; a < 8; ++a)
-#pragma unroll
-            for (int b = 0; b < 8; ++b) acc[a][b] = __fmaf_rn(ea[a], lb[b], acc[a][b]);
-    }
-#pragma unroll
-    for (int a = 0; a < 8; ++a) {
-        const int64_t r = r0 + (a < 4 ? 4 * ty + a : 64 + 4 * ty + a - 4);
-        if (r >= d_out) continue;
-#pragma unroll
-        for (int b = 0; b < 8; ++b) {
-            const int64_t c = c0 + (b < 4 ? 4 * tx + b : 64 + 4 * tx + b - 4);
-            if (c < d_in) {
-                float* o = W + r * d_in + c;
-                *o = __fsub_rn(*o, acc[a][b]);
+        for (int j = 0; j < 8; ++j) {
+            const int cc = gt_col<false>(tx, j);
+            if (cc < bcols) {
+                float* o = W + (r0 + rr) * d_in + c0 + cc;
+                *o = __fsub_rn(*o, acc[i][j]);
             }
         }
     }
@@ -318,8 +292,10 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
     if (!attr) {
         KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      BLK * RLD * 4));
-        KQ_CUDA(cudaFuncSetAttribute(trailing_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     2 * BLK * TLK * 4));
+        KQ_CUDA(cudaFuncSetAttribute(trailing_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     static_cast<int>(G_SMEM)));
+        KQ_CUDA(cudaFuncSetAttribute(trailing_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     static_cast<int>(G_SMEM)));
         attr = true;
     }
     ObsWs o = carve(ws, d_out, d_in);
@@ -328,6 +304,7 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
                                                                                 zero, o.gscale, o.gzero);
         KQ_LAUNCH_CHECK("rowgrid_kernel");
     }
+    const bool vec = (d_in % 4 == 0) && (reinterpret_cast<uintptr_t>(Lt) % 16 == 0);
     const int64_t row_ctas = std::min<int64_t>(cdiv(d_out, 4 * RPW), static_cast<int64_t>(num_sms()) * 3);
     for (int64_t i0 = 0; i0 < d_in; i0 += BLK) {
         const int kb = static_cast<int>(std::min<int64_t>(BLK, d_in - i0));
@@ -336,8 +313,11 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
         KQ_LAUNCH_CHECK("obs_block_kernel");
         const int64_t rest = d_in - (i0 + kb);
         if (rest > 0) {
-            dim3 grid(static_cast<unsigned>(cdiv(rest, TT)), static_cast<unsigned>(cdiv(d_out, TT)));
-            trailing_kernel<<<grid, 256, 2 * BLK * TLK * 4, stream>>>(W, o.E, Lt, d_out, d_in, i0, kb);
+            dim3 grid(static_cast<unsigned>(cdiv(rest, GT)), static_cast<unsigned>(cdiv(d_out, GT)));
+            if (vec)
+                trailing_kernel<true><<<grid, G_THREADS, G_SMEM, stream>>>(W, o.E, Lt, d_out, d_in, i0, kb);
+            else
+                trailing_kernel<false><<<grid, G_THREADS, G_SMEM, stream>>>(W, o.E, Lt, d_out, d_in, i0, kb);
             KQ_LAUNCH_CHECK("trailing_kernel");
         }
     }
