@@ -71,55 +71,61 @@ __global__ void prep_kernel(const float* __restrict__ H, int64_t n, int64_t npad
 }
 
 // ---------------------------------------------------------------- diag block
-// One warp factors the 32 x 32 SPD block s (row stride ld, lower part used) in place,
-// lane i owning row i, then writes X = C^-1 to x (lane c solves C x = e_c). The loops stay
-// rolled so the code is small. Returns the first non-positive pivot's index, or -1.
-__device__ __forceinline__ int warp_chol_inv32(float* s, float* x, int ld, int lane) {
+constexpr int DIAG_THREADS = 1024;
+constexpr int SB = 32;                        // leaf size inside the diagonal block
+constexpr int TLDD = SB + 1;
+constexpr size_t DIAG_SMEM = (2 * TILE_FLOATS + NB * TLDD) * sizeof(float);
+
+// One warp factors the 32 x 32 SPD leaf at s (row stride ld) in place: lane i holds the
+// not-yet-eliminated part of row i in registers, shifted so that the current column is
+// always r[0], which keeps the step loop rolled. Returns the first bad pivot, or -1.
+__device__ __forceinline__ int warp_leaf_chol(float* s, int ld, int lane) {
+    float r[SB];
+#pragma unroll
+    for (int t = 0; t < SB; ++t) r[t] = s[lane * ld + t];
     int bad = -1;
 #pragma unroll 1
-    for (int j = 0; j < 32; ++j) {
-        const float p = s[j * ld + j];
+    for (int j = 0; j < SB; ++j) {
+        const float p = __shfl_sync(0xffffffffu, r[0], j);
         if (!(p > 0.0f) && bad < 0) bad = j;
         const float d = sqrtf(p);
-        __syncwarp();
-        float lij = 0.0f;
-        if (lane > j) {
-            lij = __fdiv_rn(s[lane * ld + j], d);
-            s[lane * ld + j] = lij;
-        } else if (lane == j) {
-            s[j * ld + j] = d;
+        const float l = lane > j ? __fdiv_rn(r[0], d) : (lane == j ? d : 0.0f);
+        s[lane * ld + j] = l;                     // column j of the leaf's factor
+#pragma unroll
+        for (int t = 1; t < SB; ++t) {
+            const float lk = __shfl_sync(0xffffffffu, l, (j + t) & (SB - 1));
+            if (t < SB - j && lane >= j + t) r[t] = fmaf(-l, lk, r[t]);
         }
-        __syncwarp();
-#pragma unroll 4
-        for (int k = j + 1; k <= lane; ++k) s[lane * ld + k] = fmaf(-lij, s[k * ld + j], s[lane * ld + k]);
-        __syncwarp();
+#pragma unroll
+        for (int t = 0; t + 1 < SB; ++t) r[t] = r[t + 1];
     }
+    return bad;
+}
+
+// One warp inverts the lower-triangular 32 x 32 leaf L (shared, stride ld) into X (lane c
+// solves L x = e_c; column kept in shared memory, rolled loops).
+__device__ __forceinline__ void warp_leaf_inv(const float* L, float* X, int ld, int lane) {
 #pragma unroll 1
-    for (int i = 0; i < 32; ++i) {
+    for (int i = 0; i < SB; ++i) {
         float v = 0.0f;
         if (i >= lane) {
             float acc = (i == lane) ? 1.0f : 0.0f;
 #pragma unroll 4
-            for (int m = lane; m < i; ++m) acc = fmaf(-s[i * ld + m], x[m * ld + lane], acc);
-            v = __fdiv_rn(acc, s[i * ld + i]);
+            for (int m = lane; m < i; ++m) acc = fmaf(-L[i * ld + m], X[m * ld + lane], acc);
+            v = __fdiv_rn(acc, L[i * ld + i]);
         }
-        x[i * ld + lane] = v;
+        X[i * ld + lane] = v;
     }
-    __syncwarp();
-    return bad;
 }
 
-constexpr int SB = 32;                  // sub-block of the diagonal block
-constexpr int TLDD = SB + 1;
-constexpr size_t DIAG_SMEM = (2 * TILE_FLOATS + NB * TLDD) * sizeof(float);
-
-// Factor A_kk = C C^T and invert C, both in shared memory, as 4 x 4 sub-blocks of 32:
-//   for p: warp 0 factors and inverts sub-block (p, p); all warps form the panel
-//          C_qp = A_qp C_pp^-T (q > p) and update A_qr -= C_qp C_rp^T (p < r <= q);
-//   then X_qp = -X_qq sum_{r=p}^{q-1} C_qr X_rp by increasing q - p.
+// Factor A_kk = C C^T and invert C in shared memory, blocked by 32 x 32 leaves:
+//   for each leaf p: warp 0 factors leaf (p, p); the rows below are solved against it
+//   (C_qp = A_qp C_pp^-T, one thread per row); all warps update the trailing part.
+//   Then warps 0..3 invert the four diagonal leaves and all warps form the off-diagonal
+//   leaves X_qp = -X_qq sum_{r=p}^{q-1} C_qr X_rp by increasing q - p.
 // Writes C to A_kk and X = C^-1 to Z_kk. A non-positive pivot records its index in H's
 // own numbering (1-based).
-__global__ void __launch_bounds__(512) chol_diag_kernel(Work w, int64_t n, int64_t npad, int k, int* info) {
+__global__ void __launch_bounds__(DIAG_THREADS) chol_diag_kernel(Work w, int64_t n, int64_t npad, int k, int* info) {
     extern __shared__ float sm[];
     float* a = sm;                        // [NB][LD]  A_kk -> C
     float* x = sm + TILE_FLOATS;          // [NB][LD]  C^-1
@@ -129,34 +135,31 @@ __global__ void __launch_bounds__(512) chol_diag_kernel(Work w, int64_t n, int64
     for (int e = tid; e < NB * NB; e += blockDim.x) {
         const int r = e / NB, c = e % NB;
         a[r * LD + c] = c <= r ? w.A[(off + r) * npad + off + c] : 0.0f;
+        x[r * LD + c] = 0.0f;
     }
     __syncthreads();
     for (int p = 0; p < NB / SB; ++p) {
         const int o = p * SB;
         if (warp == 0) {
-            const int bad = warp_chol_inv32(a + o * LD + o, x + o * LD + o, LD, lane);
+            const int bad = warp_leaf_chol(a + o * LD + o, LD, lane);
             if (bad >= 0 && lane == 0) {
                 const int64_t rev = off + o + bad;
                 if (rev < n) record_error(info, static_cast<int>(n - rev));
             }
-            // zero the strict upper part of the factored sub-block
-            for (int c = lane + 1; c < SB; ++c) a[(o + lane) * LD + o + c] = 0.0f;
         }
         __syncthreads();
-        const int nr = NB - o - SB;       // rows below the sub-block
-        // panel into t: C_qp[ro][c] = sum_{m <= c} A[ro][o + m] X_pp[c][m]
-        for (int e = tid; e < nr * SB; e += blockDim.x) {
-            const int ro = e / SB, c = e % SB;
-            const float* arow = a + (o + SB + ro) * LD + o;
-            const float* xrow = x + (o + c) * LD + o;
-            float s = 0.0f;
-            for (int m = 0; m <= c; ++m) s = fmaf(arow[m], xrow[m], s);
-            t[ro * TLDD + c] = s;
-        }
-        __syncthreads();
-        for (int e = tid; e < nr * SB; e += blockDim.x) {
-            const int ro = e / SB, c = e % SB;
-            a[(o + SB + ro) * LD + o + c] = t[ro * TLDD + c];
+        const int nr = NB - o - SB;
+        // rows below: forward substitution against the leaf, one thread per row
+        if (tid < nr) {
+            float* row = a + (o + SB + tid) * LD + o;
+            const float* L = a + o * LD + o;
+#pragma unroll 1
+            for (int c = 0; c < SB; ++c) {
+                float acc = row[c];
+#pragma unroll 4
+                for (int m = 0; m < c; ++m) acc = fmaf(-row[m], L[c * LD + m], acc);
+                row[c] = __fdiv_rn(acc, L[c * LD + c]);
+            }
         }
         __syncthreads();
         // trailing update of the lower part of rows/cols [o + SB, NB)
@@ -165,37 +168,37 @@ __global__ void __launch_bounds__(512) chol_diag_kernel(Work w, int64_t n, int64
             if (co > ro) continue;
             const float* ar = a + (o + SB + ro) * LD + o;
             const float* ac = a + (o + SB + co) * LD + o;
-            float s = 0.0f;
+            float acc = 0.0f;
 #pragma unroll 8
-            for (int m = 0; m < SB; ++m) s = fmaf(ar[m], ac[m], s);
-            a[(o + SB + ro) * LD + o + SB + co] -= s;
+            for (int m = 0; m < SB; ++m) acc = fmaf(ar[m], ac[m], acc);
+            a[(o + SB + ro) * LD + o + SB + co] -= acc;
         }
         __syncthreads();
     }
-    // off-diagonal blocks of X = C^-1, by distance d = q - p
+    if (warp < NB / SB) warp_leaf_inv(a + warp * SB * LD + warp * SB, x + warp * SB * LD + warp * SB, LD, lane);
+    __syncthreads();
     for (int d = 1; d < NB / SB; ++d) {
         const int nblk = NB / SB - d;
-        // T_qp = sum_{r=p}^{q-1} C_qr X_rp   (stored in t rows [b*SB, b*SB+SB), b = p)
-        for (int e = tid; e < nblk * SB * SB; e += blockDim.x) {
+        for (int e = tid; e < nblk * SB * SB; e += blockDim.x) {   // T_qp = sum_r C_qr X_rp
             const int b = e / (SB * SB), i = (e / SB) % SB, c = e % SB;
             const int pp = b, qq = b + d;
-            float s = 0.0f;
+            float acc = 0.0f;
             for (int r2 = pp; r2 < qq; ++r2) {
                 const float* crow = a + (qq * SB + i) * LD + r2 * SB;
                 const float* xcol = x + (r2 * SB) * LD + pp * SB + c;
-                for (int m = 0; m < SB; ++m) s = fmaf(crow[m], xcol[m * LD], s);
+#pragma unroll 8
+                for (int m = 0; m < SB; ++m) acc = fmaf(crow[m], xcol[m * LD], acc);
             }
-            t[(b * SB + i) * TLDD + c] = s;
+            t[(b * SB + i) * TLDD + c] = acc;
         }
         __syncthreads();
-        // X_qp = -X_qq T_qp   (X_qq lower)
-        for (int e = tid; e < nblk * SB * SB; e += blockDim.x) {
+        for (int e = tid; e < nblk * SB * SB; e += blockDim.x) {   // X_qp = -X_qq T_qp
             const int b = e / (SB * SB), i = (e / SB) % SB, c = e % SB;
             const int pp = b, qq = b + d;
             const float* xrow = x + (qq * SB + i) * LD + qq * SB;
-            float s = 0.0f;
-            for (int m = 0; m <= i; ++m) s = fmaf(xrow[m], t[(b * SB + m) * TLDD + c], s);
-            x[(qq * SB + i) * LD + pp * SB + c] = -s;
+            float acc = 0.0f;
+            for (int m = 0; m <= i; ++m) acc = fmaf(xrow[m], t[(b * SB + m) * TLDD + c], acc);
+            x[(qq * SB + i) * LD + pp * SB + c] = -acc;
         }
         __syncthreads();
     }
@@ -236,6 +239,26 @@ __global__ void __launch_bounds__(G_THREADS, 2) chol_panel_kernel(Work w, int64_
         }
 }
 
+// out[tile] -= acc, loads of 32 values issued before their stores.
+template <bool BN>
+__device__ __forceinline__ void sub_tile(float* out, int64_t ld, const float (&acc)[8][8]) {
+    const int ty = threadIdx.x >> 4, tx = threadIdx.x & 15;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        float ov[4][8];
+#pragma unroll
+        for (int a = 0; a < 4; ++a)
+#pragma unroll
+            for (int b = 0; b < 8; ++b)
+                ov[a][b] = out[static_cast<int64_t>(gt_row(ty, 4 * h + a)) * ld + gt_col<BN>(tx, b)];
+#pragma unroll
+        for (int a = 0; a < 4; ++a)
+#pragma unroll
+            for (int b = 0; b < 8; ++b)
+                out[static_cast<int64_t>(gt_row(ty, 4 * h + a)) * ld + gt_col<BN>(tx, b)] = ov[a][b] - acc[4 * h + a][b];
+    }
+}
+
 // -------------------------------------------------------------------- update
 // Tiles (i, j), k < i < nbk, 0 <= j <= i:
 //   j > k : A_ij -= C_ik C_jk^T;     j <= k : Z_ij -= C_ik Z_kj.
@@ -257,15 +280,10 @@ __global__ void __launch_bounds__(G_THREADS, 2) chol_update_kernel(Work w, int64
     else
         gemm_tile<true, true>(cik, npad, NB, w.Z + ko * npad + static_cast<int64_t>(j) * NB, npad, NB, NB, acc, sm);
     float* out = (apart ? w.A : w.Z) + static_cast<int64_t>(i) * NB * npad + static_cast<int64_t>(j) * NB;
-    const int ty = threadIdx.x >> 4, tx = threadIdx.x & 15;
-#pragma unroll
-    for (int a = 0; a < 8; ++a)
-#pragma unroll
-        for (int b = 0; b < 8; ++b) {
-            const int c = apart ? gt_col<false>(tx, b) : gt_col<true>(tx, b);
-            float* o = out + static_cast<int64_t>(gt_row(ty, a)) * npad + c;
-            *o = *o - acc[a][b];
-        }
+    if (apart)
+        sub_tile<false>(out, npad, acc);
+    else
+        sub_tile<true>(out, npad, acc);
 }
 
 // -------------------------------------------------------------------- finish
@@ -334,7 +352,7 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
     prep_kernel<<<static_cast<unsigned>(pgrid), 256, 0, stream>>>(H, n, npad, damp_rel, w.dsum, w.A, w.Z);
     KQ_LAUNCH_CHECK("prep_kernel");
     for (int k = 0; k < nbk; ++k) {
-        chol_diag_kernel<<<1, 512, DIAG_SMEM, stream>>>(w, n, npad, k, info);
+        chol_diag_kernel<<<1, DIAG_THREADS, DIAG_SMEM, stream>>>(w, n, npad, k, info);
         KQ_LAUNCH_CHECK("chol_diag_kernel");
         if (nbk > 1) {
             chol_panel_kernel<<<nbk - 1, G_THREADS, G_SMEM, stream>>>(w, npad, k);

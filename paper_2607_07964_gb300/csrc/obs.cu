@@ -199,18 +199,25 @@ __global__ void __launch_bounds__(G_THREADS, 2) trailing_kernel(float* __restric
     float acc[8][8];
     gemm_tile<false, VEC>(E + r0 * d_in + i0, d_in, arows, Lt + c0 * d_in + i0, d_in, bcols, kb, acc, sm);
     const int ty = threadIdx.x >> 4, tx = threadIdx.x & 15;
+    // Read-modify-write of W in two halves of 32 values, all loads of a half issued before
+    // its stores, so the memory latency is paid twice rather than 64 times.
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-        const int rr = gt_row(ty, i);
-        if (rr >= arows) continue;
+    for (int h = 0; h < 2; ++h) {
+        float wv[4][8];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            const int cc = gt_col<false>(tx, j);
-            if (cc < bcols) {
-                float* o = W + (r0 + rr) * d_in + c0 + cc;
-                *o = __fsub_rn(*o, acc[i][j]);
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int rr = gt_row(ty, 4 * h + i), cc = gt_col<false>(tx, j);
+                wv[i][j] = (rr < arows && cc < bcols) ? W[(r0 + rr) * d_in + c0 + cc] : 0.0f;
             }
-        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int rr = gt_row(ty, 4 * h + i), cc = gt_col<false>(tx, j);
+                if (rr < arows && cc < bcols) W[(r0 + rr) * d_in + c0 + cc] = __fsub_rn(wv[i][j], acc[4 * h + i][j]);
+            }
     }
 }
 
