@@ -155,6 +155,26 @@ KQ_API size_t kq_chol_inv_workspace(int64_t n);
 KQ_API kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, float* Lt, int* info, void* ws,
                       size_t ws_bytes, kq_stream_t stream);
 
+/*
+ * kq_chol_inv_noalloc: the same computation and results as kq_chol_inv, for callers that
+ *   cannot hand the library a workspace because they may not allocate device memory when
+ *   they call it -- for example a plugin running inside another runtime that owns every
+ *   device allocation, or a latency-bound loop where a cudaMalloc would synchronize the
+ *   device. The paper has no counterpart; this is a convenience of this library.
+ *   Scratch comes from a fixed array in device memory that the library owns:
+ *   2 * KQ_CHOL_NOALLOC_MAX_N^2 * 4 + 256 bytes (8 MiB), held by every device that loads
+ *   the library until the process exits. n > KQ_CHOL_NOALLOC_MAX_N is rejected with
+ *   KQ_ERR_WORKSPACE and a message; no allocation is ever made.
+ *   The first call on each device looks up the array's device address (cudaGetSymbolAddress,
+ *   with that device current); make that first call before any stream capture.
+ *   All calls share the one array and it keeps the previous call's contents (every byte a
+ *   call reads is written by that call first), so calls whose work overlaps on the GPU --
+ *   on different streams, or from different host threads -- race: serialize them.
+ */
+#define KQ_CHOL_NOALLOC_MAX_N 1024
+KQ_API kq_status kq_chol_inv_noalloc(const float* H, int64_t n, float damp_rel, float* Lt, int* info,
+                                     kq_stream_t stream);
+
 /* ------------------------------------------------------------------------------------
  * Stage 4: column-wise OBS sweep (GPTQ mode; the GPTAQ drift term P is zero).
  * Paper: Sec. 2.1 Eq. (obs_update); Algorithm 2's inner column loop and lazy trailing

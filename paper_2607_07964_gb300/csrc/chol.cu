@@ -370,3 +370,47 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
     KQ_LAUNCH_CHECK("finish_kernel");
     return KQ_OK;
 }
+
+// ------------------------------------------------------------ no-allocation variant
+// kq_chol_inv_noalloc runs the same kernels as kq_chol_inv, with the scratch space taken
+// from a fixed array in device memory that the library owns, so the caller passes only
+// inputs and outputs. The array is sized for n <= KQ_CHOL_NOALLOC_MAX_N and is held by
+// every device that loads the library until the process exits. Its device address is
+// looked up once per device (with that device current) on the first call there.
+#include <mutex>
+
+namespace {
+constexpr size_t kNoallocBytes =
+    2 * static_cast<size_t>(KQ_CHOL_NOALLOC_MAX_N) * KQ_CHOL_NOALLOC_MAX_N * sizeof(float) + 256;
+static __device__ __align__(256) unsigned char g_chol_scratch[kNoallocBytes];
+std::mutex g_noalloc_mu;
+void* g_noalloc_ptr[64] = {};
+}  // namespace
+
+extern "C" kq_status kq_chol_inv_noalloc(const float* H, int64_t n, float damp_rel, float* Lt, int* info,
+                                         kq_stream_t stream) {
+    if (n < 1 || n > KQ_CHOL_NOALLOC_MAX_N) {
+        set_error("kq_chol_inv_noalloc: n=%lld is outside [1, %d], the size its fixed scratch array holds; "
+                  "use kq_chol_inv with a caller workspace",
+                  (long long)n, KQ_CHOL_NOALLOC_MAX_N);
+        return KQ_ERR_WORKSPACE;
+    }
+    int dev = 0;
+    KQ_CUDA(cudaGetDevice(&dev));
+    if (dev < 0 || dev >= 64) {
+        set_error("kq_chol_inv_noalloc: device index %d not supported", dev);
+        return KQ_ERR_INVALID_ARG;
+    }
+    void* ws = nullptr;
+    {
+        std::lock_guard<std::mutex> lock(g_noalloc_mu);
+        if (!g_noalloc_ptr[dev]) {
+            void* p = nullptr;
+            const cudaError_t e = cudaGetSymbolAddress(&p, g_chol_scratch);
+            if (e != cudaSuccess || !p) return cuda_status(e, "cudaGetSymbolAddress(g_chol_scratch)");
+            g_noalloc_ptr[dev] = p;
+        }
+        ws = g_noalloc_ptr[dev];
+    }
+    return kq_chol_inv(H, n, damp_rel, Lt, info, ws, kNoallocBytes, stream);
+}

@@ -49,6 +49,7 @@ def lib() -> ctypes.CDLL:
             "kq_rotate_out": ([P, I64, I64, P, P, P, I, P], I),
             "kq_chol_inv_workspace": ([I64], SZ),
             "kq_chol_inv": ([P, I64, F, P, P, P, SZ, P], I),
+            "kq_chol_inv_noalloc": ([P, I64, F, P, P, P], I),
             "kq_obs_quantize_workspace": ([I64, I64, I], SZ),
             "kq_obs_quantize": ([P, I64, I64, P, I, I, I, P, P, P, P, P, P, SZ, P], I),
             "kq_dequant_revert": ([P, P, P, I64, I64, I, P, P, P, P, P, P], I),
@@ -181,6 +182,20 @@ def kq_chol_inv(H, damp_rel: float, Lt, info, ws, stream=None) -> None:
     _need(ws, "ws", torch.uint8)
     _ok(lib().kq_chol_inv(_ptr(H), n, float(damp_rel), _ptr(Lt), _ptr(info), _ptr(ws),
                           0 if ws is None else ws.numel(), _stream(stream)), "kq_chol_inv")
+
+
+KQ_CHOL_NOALLOC_MAX_N = 1024
+
+
+def kq_chol_inv_noalloc(H, damp_rel: float, Lt, info=None, stream=None) -> None:
+    """kq_chol_inv without a caller workspace (n <= KQ_CHOL_NOALLOC_MAX_N): the library's
+    own fixed device array serves as scratch. Calls must not overlap on the GPU."""
+    n = H.shape[0]
+    _need(H, "H", torch.float32, (n, n))
+    _need(Lt, "Lt", torch.float32, (n, n))
+    _need(info, "info", torch.int32)
+    _ok(lib().kq_chol_inv_noalloc(_ptr(H), n, float(damp_rel), _ptr(Lt), _ptr(info), _stream(stream)),
+        "kq_chol_inv_noalloc")
 
 
 def kq_obs_quantize_workspace(d_out: int, d_in: int, block: int = 128) -> int:
