@@ -112,55 +112,88 @@ __device__ __forceinline__ void fwht_reg_r(float (&x)[8], int r) {
 
 // One radix-r pass (span h = 2^lgh) of the Walsh-Hadamard transform over a shared vector
 // of n elements (every h*r-aligned block independently). Index math is shifts and masks.
-__device__ __forceinline__ void fwht_pass(float* v, int n, int lgh, int lgr) {
+// FIRST: multiply each element by its pre-factor while reading. LAST: instead of writing
+// back, store (value * post-factor * scale) to dst (global).
+template <bool FIRST, bool LAST>
+__device__ __forceinline__ void fwht_pass(float* v, int n, int lgh, int lgr, int pre_mode, int post_mode,
+                                          const int8_t* sign, const float* s, float scale, float* dst) {
     const int h = 1 << lgh, r = 1 << lgr;
     for (int g = threadIdx.x; g < (n >> lgr); g += blockDim.x) {
         const int base = ((g >> lgh) << (lgh + lgr)) | (g & (h - 1));
         float x[8];
 #pragma unroll
         for (int q = 0; q < 8; ++q)
-            if (q < r) x[q] = v[base + q * h];
+            if (q < r) {
+                x[q] = v[base + q * h];
+                if (FIRST) x[q] *= factor(pre_mode, sign, s, base + q * h);
+            }
         fwht_reg_r(x, r);
 #pragma unroll
         for (int q = 0; q < 8; ++q)
-            if (q < r) v[base + q * h] = x[q];
+            if (q < r) {
+                if (LAST) dst[base + q * h] = x[q] * (factor(post_mode, sign, s, base + q * h) * scale);
+                else v[base + q * h] = x[q];
+            }
     }
+}
+
+// Stage n contiguous floats from global into shared memory with 16-byte cp.async copies
+// (scalar copies when the row is not 16-byte aligned).
+__device__ __forceinline__ void stage_row(float* v, const float* src, int n) {
+    if ((reinterpret_cast<uintptr_t>(src) & 15u) == 0 && (n & 3) == 0) {
+        for (int q = threadIdx.x; q < (n >> 2); q += blockDim.x) cp_async16(v + 4 * q, src + 4 * q, 16);
+        cp_async_commit();
+        cp_async_wait<0>();
+    } else {
+        for (int j = threadIdx.x; j < n; j += blockDim.x) v[j] = src[j];
+    }
+    __syncthreads();
 }
 
 // ------------------------------------------------------------------ row transform
 // For each row of M [rows x n]: v <- pre (.) v; v <- (H_28 (x) H_P) v (or H_P); row <-
-// post (.) v / sqrt(n). One CTA per row (grid-stride); n floats of shared memory.
-// The power-of-two part runs as radix-8 passes (one barrier per pass).
-__global__ void __launch_bounds__(512) rht_rows_kernel(float* __restrict__ M, int64_t rows, int n, int lgP, int has28,
+// post (.) v / sqrt(n). One CTA per row (grid-stride); n floats of shared memory. The row
+// is staged with cp.async, the power-of-two part runs as radix-8 passes (one barrier per
+// pass), and the last pass writes straight to global memory.
+template <bool HAS28>
+__global__ void __launch_bounds__(HAS28 ? 256 : 512, HAS28 ? 1 : 2) rht_rows_kernel(float* __restrict__ M, int64_t rows, int n, int lgP,
                                 int pre_mode, int post_mode, const int8_t* __restrict__ sign,
                                 const float* __restrict__ s, float inv_sqrt_n) {
-    extern __shared__ float v[];
+    extern __shared__ __align__(16) float v[];
     const int P = 1 << lgP;
     for (int64_t r = blockIdx.x; r < rows; r += gridDim.x) {
         float* row = M + r * n;
-        for (int j = threadIdx.x; j < n; j += blockDim.x)
-            v[j] = row[j] * factor(pre_mode, sign, s, j);
-        __syncthreads();
+        stage_row(v, row, n);
+        bool first = true;
+        if (!HAS28 && lgP == 0) {   // n == 1
+            for (int j = threadIdx.x; j < n; j += blockDim.x)
+                row[j] = v[j] * factor(pre_mode, sign, s, j) * (factor(post_mode, sign, s, j) * inv_sqrt_n);
+        }
         for (int lgh = 0; lgh < lgP;) {   // I_28 (x) H_P: passes stay inside P-aligned chunks
             const int lgr = min(3, lgP - lgh);
-            fwht_pass(v, n, lgh, lgr);
+            const bool last = !HAS28 && lgh + lgr == lgP;
+            if (first && last) fwht_pass<true, true>(v, n, lgh, lgr, pre_mode, post_mode, sign, s, inv_sqrt_n, row);
+            else if (first) fwht_pass<true, false>(v, n, lgh, lgr, pre_mode, post_mode, sign, s, inv_sqrt_n, row);
+            else if (last) fwht_pass<false, true>(v, n, lgh, lgr, pre_mode, post_mode, sign, s, inv_sqrt_n, row);
+            else fwht_pass<false, false>(v, n, lgh, lgr, pre_mode, post_mode, sign, s, inv_sqrt_n, row);
+            first = false;
             __syncthreads();
             lgh += lgr;
         }
-        if (has28) {   // H_28 (x) I_P
+        if (HAS28) {   // H_28 (x) I_P, written straight to global memory
             for (int b = threadIdx.x; b < P; b += blockDim.x) {
                 float x[28], y[28];
 #pragma unroll
-                for (int a = 0; a < 28; ++a) x[a] = v[a * P + b];
+                for (int a = 0; a < 28; ++a) {
+                    x[a] = v[a * P + b];
+                    if (first) x[a] *= factor(pre_mode, sign, s, a * P + b);
+                }
                 mix28(x, y);
 #pragma unroll
-                for (int a = 0; a < 28; ++a) v[a * P + b] = y[a];
+                for (int a = 0; a < 28; ++a) row[a * P + b] = y[a] * (factor(post_mode, sign, s, a * P + b) * inv_sqrt_n);
             }
             __syncthreads();
         }
-        for (int j = threadIdx.x; j < n; j += blockDim.x)
-            row[j] = v[j] * (factor(post_mode, sign, s, j) * inv_sqrt_n);
-        __syncthreads();
     }
 }
 
@@ -168,62 +201,89 @@ __global__ void __launch_bounds__(512) rht_rows_kernel(float* __restrict__ M, in
 // One radix stage along the row index of M [n x ncols]: for every group base = hi*R*S + lo
 // (lo < S) and CW-column strip, rows base + i*S (i < R) are transformed along i by H_R
 // (R a power of two, as radix-8 passes) or H_28 (R == 28). Shared memory [R][CW], CW a
-// power of two; index math is shifts and masks.
-__global__ void __launch_bounds__(256) rht_cols_kernel(float* __restrict__ M, int n, int64_t ncols, int R, int S,
+// power of two, filled with cp.async; the last pass writes straight to global memory.
+template <bool IS28>
+__global__ void __launch_bounds__(256, IS28 ? 1 : 4) rht_cols_kernel(float* __restrict__ M, int n, int64_t ncols, int R, int S,
                                 int lgCW, int pre_mode, int post_mode, const int8_t* __restrict__ sign,
                                 const float* __restrict__ s, float post_scale) {
-    extern __shared__ float v[];
+    extern __shared__ __align__(16) float v[];
     const int CW = 1 << lgCW;
     const int64_t nstrips = (ncols + CW - 1) >> lgCW;
     const int64_t ngroups = n / R;
     int lgR = 0;
     while ((1 << lgR) < R) ++lgR;
+    const bool vec = (ncols & 3) == 0 && (reinterpret_cast<uintptr_t>(M) & 15u) == 0;
     for (int64_t w = blockIdx.x; w < ngroups * nstrips; w += gridDim.x) {
         const int64_t g = w / nstrips;
         const int64_t c0 = (w - g * nstrips) << lgCW;
         const int64_t base = (g / S) * static_cast<int64_t>(R) * S + (g % S);
         const int cw = static_cast<int>(min(static_cast<int64_t>(CW), ncols - c0));
-        for (int e = threadIdx.x; e < R * CW; e += blockDim.x) {
-            const int i = e >> lgCW, c = e & (CW - 1);
-            const int64_t r = base + static_cast<int64_t>(i) * S;
-            v[e] = c < cw ? M[r * ncols + c0 + c] * factor(pre_mode, sign, s, r) : 0.0f;
+        if (vec) {
+            for (int e = threadIdx.x; e < (R * CW) >> 2; e += blockDim.x) {
+                const int i = (4 * e) >> lgCW, c = (4 * e) & (CW - 1);
+                const int64_t r = base + static_cast<int64_t>(i) * S;
+                const int valid = max(0, min(4, cw - c));
+                cp_async16(v + 4 * e, valid ? static_cast<const void*>(M + r * ncols + c0 + c) : static_cast<const void*>(M),
+                           4 * valid);
+            }
+            cp_async_commit();
+            cp_async_wait<0>();
+        } else {
+            for (int e = threadIdx.x; e < R * CW; e += blockDim.x) {
+                const int i = e >> lgCW, c = e & (CW - 1);
+                v[e] = c < cw ? M[(base + static_cast<int64_t>(i) * S) * ncols + c0 + c] : 0.0f;
+            }
         }
         __syncthreads();
-        if (R == 28) {
+        if (IS28) {
             for (int c = threadIdx.x; c < CW; c += blockDim.x) {
                 float x[28], y[28];
 #pragma unroll
-                for (int a = 0; a < 28; ++a) x[a] = v[a * CW + c];
+                for (int a = 0; a < 28; ++a) x[a] = v[a * CW + c] * factor(pre_mode, sign, s, base + static_cast<int64_t>(a) * S);
                 mix28(x, y);
+                if (c < cw) {
 #pragma unroll
-                for (int a = 0; a < 28; ++a) v[a * CW + c] = y[a];
+                    for (int a = 0; a < 28; ++a) {
+                        const int64_t r = base + static_cast<int64_t>(a) * S;
+                        M[r * ncols + c0 + c] = y[a] * (factor(post_mode, sign, s, r) * post_scale);
+                    }
+                }
             }
-            __syncthreads();
         } else {
             for (int lgh = 0; lgh < lgR;) {
                 const int lgr = min(3, lgR - lgh);
                 const int h = 1 << lgh, rr = 1 << lgr;
+                const bool first = lgh == 0, last = lgh + lgr == lgR;
                 for (int gg = threadIdx.x; gg < ((R >> lgr) << lgCW); gg += blockDim.x) {
                     const int c = gg & (CW - 1), gi = gg >> lgCW;
                     const int bi = ((gi >> lgh) << (lgh + lgr)) | (gi & (h - 1));
                     float x[8];
 #pragma unroll
                     for (int q = 0; q < 8; ++q)
-                        if (q < rr) x[q] = v[((bi + q * h) << lgCW) + c];
+                        if (q < rr) {
+                            x[q] = v[((bi + q * h) << lgCW) + c];
+                            if (first) x[q] *= factor(pre_mode, sign, s, base + static_cast<int64_t>(bi + q * h) * S);
+                        }
                     fwht_reg_r(x, rr);
 #pragma unroll
                     for (int q = 0; q < 8; ++q)
-                        if (q < rr) v[((bi + q * h) << lgCW) + c] = x[q];
+                        if (q < rr) {
+                            if (last) {
+                                if (c < cw) {
+                                    const int64_t r = base + static_cast<int64_t>(bi + q * h) * S;
+                                    M[r * ncols + c0 + c] = x[q] * (factor(post_mode, sign, s, r) * post_scale);
+                                }
+                            } else {
+                                v[((bi + q * h) << lgCW) + c] = x[q];
+                            }
+                        }
                 }
                 __syncthreads();
                 lgh += lgr;
             }
-        }
-        for (int e = threadIdx.x; e < R * CW; e += blockDim.x) {
-            const int i = e >> lgCW, c = e & (CW - 1);
-            if (c < cw) {
-                const int64_t r = base + static_cast<int64_t>(i) * S;
-                M[r * ncols + c0 + c] = v[e] * (factor(post_mode, sign, s, r) * post_scale);
+            if (lgR == 0) {   // R == 1: only the factors apply
+                for (int c = threadIdx.x; c < cw; c += blockDim.x)
+                    M[base * ncols + c0 + c] = v[c] * factor(pre_mode, sign, s, base) * (factor(post_mode, sign, s, base) * post_scale);
             }
         }
         __syncthreads();
@@ -365,16 +425,22 @@ kq_status rows_transform(float* M, int64_t rows, int64_t n, int pre, int post, c
     const size_t smem = static_cast<size_t>(n) * sizeof(float);
     static bool attr = false;
     if (!attr) {
-        KQ_CUDA(cudaFuncSetAttribute(rht_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        KQ_CUDA(cudaFuncSetAttribute(rht_rows_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     32768 * 4));
+        KQ_CUDA(cudaFuncSetAttribute(rht_rows_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      32768 * 4));
         attr = true;
     }
-    const int threads = n >= 2048 ? 512 : (n >= 512 ? 256 : 128);
-    const int64_t grid = std::min<int64_t>(rows, static_cast<int64_t>(num_sms()) * 16);
+    const int threads = p.has28 ? 256 : (n >= 2048 ? 512 : (n >= 512 ? 256 : 128));
+    const int64_t grid = std::min<int64_t>(rows, static_cast<int64_t>(num_sms()) * 32);
     if (grid > 0) {
-        rht_rows_kernel<<<static_cast<unsigned>(grid), threads, smem, stream>>>(
-            M, rows, static_cast<int>(n), log2i(p.P), p.has28, pre, post, sign, s,
-            static_cast<float>(1.0 / sqrt(static_cast<double>(n))));
+        const float isn = static_cast<float>(1.0 / sqrt(static_cast<double>(n)));
+        if (p.has28)
+            rht_rows_kernel<true><<<static_cast<unsigned>(grid), threads, smem, stream>>>(
+                M, rows, static_cast<int>(n), log2i(p.P), pre, post, sign, s, isn);
+        else
+            rht_rows_kernel<false><<<static_cast<unsigned>(grid), threads, smem, stream>>>(
+                M, rows, static_cast<int>(n), log2i(p.P), pre, post, sign, s, isn);
         KQ_LAUNCH_CHECK("rht_rows_kernel");
     }
     return KQ_OK;
@@ -397,7 +463,9 @@ kq_status cols_transform(float* M, int64_t n, int64_t ncols, int pre, int post, 
     if (p.has28) { R[ns] = 28; S[ns] = p.P; ++ns; }
     static bool attr = false;
     if (!attr) {
-        KQ_CUDA(cudaFuncSetAttribute(rht_cols_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        KQ_CUDA(cudaFuncSetAttribute(rht_cols_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     128 * 1024));
+        KQ_CUDA(cudaFuncSetAttribute(rht_cols_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      128 * 1024));
         attr = true;
     }
@@ -410,10 +478,15 @@ kq_status cols_transform(float* M, int64_t n, int64_t ncols, int pre, int post, 
         CW = CW < 32 ? 32 : (CW > 256 ? 256 : CW);
         const size_t smem = static_cast<size_t>(R[st]) * CW * sizeof(float);
         const int64_t items = (n / R[st]) * cdiv(ncols, CW);
-        const int64_t grid = std::min<int64_t>(items, static_cast<int64_t>(num_sms()) * 8);
-        rht_cols_kernel<<<static_cast<unsigned>(grid), 256, smem, stream>>>(
-            M, static_cast<int>(n), ncols, R[st], S[st], log2i(CW), st == 0 ? pre : F_NONE,
-            st == ns - 1 ? post : F_NONE, sign, s, st == ns - 1 ? post_scale : 1.0f);
+        const int64_t grid = std::min<int64_t>(items, static_cast<int64_t>(num_sms()) * 16);
+        const int pm = st == 0 ? pre : F_NONE, qm = st == ns - 1 ? post : F_NONE;
+        const float ps = st == ns - 1 ? post_scale : 1.0f;
+        if (R[st] == 28)
+            rht_cols_kernel<true><<<static_cast<unsigned>(grid), 256, smem, stream>>>(
+                M, static_cast<int>(n), ncols, R[st], S[st], log2i(CW), pm, qm, sign, s, ps);
+        else
+            rht_cols_kernel<false><<<static_cast<unsigned>(grid), 256, smem, stream>>>(
+                M, static_cast<int>(n), ncols, R[st], S[st], log2i(CW), pm, qm, sign, s, ps);
         KQ_LAUNCH_CHECK("rht_cols_kernel");
     }
     return KQ_OK;

@@ -74,55 +74,69 @@ __global__ void prep_kernel(const float* __restrict__ H, int64_t n, int64_t npad
 constexpr int DIAG_THREADS = 1024;
 constexpr int SB = 32;                        // leaf size inside the diagonal block
 constexpr int TLDD = SB + 1;
-constexpr size_t DIAG_SMEM = (2 * TILE_FLOATS + NB * TLDD) * sizeof(float);
+constexpr size_t DIAG_SMEM = (2 * TILE_FLOATS + NB * TLDD + 2 * NB) * sizeof(float);
 
-// One warp factors the 32 x 32 SPD leaf at s (row stride ld) in place: lane i holds the
-// not-yet-eliminated part of row i in registers, shifted so that the current column is
-// always r[0], which keeps the step loop rolled. Returns the first bad pivot, or -1.
-__device__ __forceinline__ int warp_leaf_chol(float* s, int ld, int lane) {
-    float r[SB];
-#pragma unroll
-    for (int t = 0; t < SB; ++t) r[t] = s[lane * ld + t];
+__device__ __forceinline__ void named_barrier(int id, int nthreads) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+// Leaf factor by 128 threads (warps 0..3, named barrier 1): thread t owns row t / 4 of the
+// 32 x 32 leaf at s and the columns k = t (mod 4). Step j updates the trailing part with
+// the pivot scaling deferred, a_ik -= (a_ij / p_j) a_kj; afterwards C_ij = a_ij / sqrt(p_j),
+// C_jj = sqrt(p_j), and dv[j] = 1 / C_jj. Returns the first non-positive pivot, or -1.
+__device__ __forceinline__ int leaf_factor128(float* s, int ld, float* pv, float* dv, int t) {
+    const int i = t >> 2, q = t & 3;
     int bad = -1;
 #pragma unroll 1
     for (int j = 0; j < SB; ++j) {
-        const float p = __shfl_sync(0xffffffffu, r[0], j);
+        const float p = s[j * ld + j];
         if (!(p > 0.0f) && bad < 0) bad = j;
-        const float d = sqrtf(p);
-        const float l = lane > j ? __fdiv_rn(r[0], d) : (lane == j ? d : 0.0f);
-        s[lane * ld + j] = l;                     // column j of the leaf's factor
-#pragma unroll
-        for (int t = 1; t < SB; ++t) {
-            const float lk = __shfl_sync(0xffffffffu, l, (j + t) & (SB - 1));
-            if (t < SB - j && lane >= j + t) r[t] = fmaf(-l, lk, r[t]);
+        if (i > j) {
+            const float f = s[i * ld + j] * __fdiv_rn(1.0f, p);
+            for (int k = j + 1 + q; k <= i; k += 4) s[i * ld + k] = fmaf(-f, s[k * ld + j], s[i * ld + k]);
         }
-#pragma unroll
-        for (int t = 0; t + 1 < SB; ++t) r[t] = r[t + 1];
+        if (t == 0) pv[j] = p;
+        named_barrier(1, 128);
     }
+    for (int e = t; e < SB * SB; e += 128) {
+        const int r = e >> 5, c = e & 31;
+        const float d = sqrtf(pv[c]);
+        if (c < r) s[r * ld + c] = __fdiv_rn(s[r * ld + c], d);
+        else if (c == r) s[r * ld + c] = d;
+        else s[r * ld + c] = 0.0f;
+        if (r == 0) dv[c] = __fdiv_rn(1.0f, d);
+    }
+    named_barrier(1, 128);
     return bad;
 }
 
-// One warp inverts the lower-triangular 32 x 32 leaf L (shared, stride ld) into X (lane c
-// solves L x = e_c; column kept in shared memory, rolled loops).
-__device__ __forceinline__ void warp_leaf_inv(const float* L, float* X, int ld, int lane) {
+// Leaf inverse by 128 threads without block barriers: four lanes per column c (8 columns
+// per warp), lane q of the group owning rows i = q (mod 4). Step i: the owner of row i
+// finalizes x_ic = b_ic / C_ii and shuffles it to the group, which updates
+// b_i'c -= C_i'i x_ic for its rows i' > i. X (stride ld) starts as the identity.
+__device__ __forceinline__ void leaf_inverse128(const float* L, float* X, int ld, const float* dv, int t) {
+    const int c = t >> 2, q = t & 3;
+    const int lane = threadIdx.x & 31, gbase = lane & ~3;
+    for (int r = q; r < SB; r += 4) X[r * ld + c] = (r == c) ? 1.0f : 0.0f;
+    __syncwarp();
 #pragma unroll 1
     for (int i = 0; i < SB; ++i) {
-        float v = 0.0f;
-        if (i >= lane) {
-            float acc = (i == lane) ? 1.0f : 0.0f;
-#pragma unroll 4
-            for (int m = lane; m < i; ++m) acc = fmaf(-L[i * ld + m], X[m * ld + lane], acc);
-            v = __fdiv_rn(acc, L[i * ld + i]);
+        float xi = 0.0f;
+        if ((i & 3) == q) {
+            xi = X[i * ld + c] * dv[i];
+            X[i * ld + c] = xi;
         }
-        X[i * ld + lane] = v;
+        xi = __shfl_sync(0xffffffffu, xi, gbase | (i & 3));
+        for (int r = i + 1 + ((q - i - 1) & 3); r < SB; r += 4) X[r * ld + c] = fmaf(-L[r * ld + i], xi, X[r * ld + c]);
+        __syncwarp();
     }
 }
 
 // Factor A_kk = C C^T and invert C in shared memory, blocked by 32 x 32 leaves:
-//   for each leaf p: warp 0 factors leaf (p, p); the rows below are solved against it
-//   (C_qp = A_qp C_pp^-T, one thread per row); all warps update the trailing part.
-//   Then warps 0..3 invert the four diagonal leaves and all warps form the off-diagonal
-//   leaves X_qp = -X_qq sum_{r=p}^{q-1} C_qr X_rp by increasing q - p.
+//   leaf p: warps 0..3 factor leaf (p, p) while warps 4..7 invert leaf p - 1; then one warp
+//   per row solves the rows below against the leaf (C_qp = A_qp C_pp^-T) and all warps
+//   update the trailing part with 4 x 4 register tiles;
+//   after the last leaf: X_qp = -X_qq sum_{r=p}^{q-1} C_qr X_rp by increasing q - p.
 // Writes C to A_kk and X = C^-1 to Z_kk. A non-positive pivot records its index in H's
 // own numbering (1-based).
 __global__ void __launch_bounds__(DIAG_THREADS) chol_diag_kernel(Work w, int64_t n, int64_t npad, int k, int* info) {
@@ -130,7 +144,10 @@ __global__ void __launch_bounds__(DIAG_THREADS) chol_diag_kernel(Work w, int64_t
     float* a = sm;                        // [NB][LD]  A_kk -> C
     float* x = sm + TILE_FLOATS;          // [NB][LD]  C^-1
     float* t = sm + 2 * TILE_FLOATS;      // [NB][TLDD] temporaries
+    float* pv = t + NB * TLDD;            // [NB] pivots
+    float* dv = pv + NB;                  // [NB] 1 / C_jj
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    constexpr int NW = DIAG_THREADS / 32;
     const int64_t off = static_cast<int64_t>(k) * NB;
     for (int e = tid; e < NB * NB; e += blockDim.x) {
         const int r = e / NB, c = e % NB;
@@ -138,67 +155,124 @@ __global__ void __launch_bounds__(DIAG_THREADS) chol_diag_kernel(Work w, int64_t
         x[r * LD + c] = 0.0f;
     }
     __syncthreads();
-    for (int p = 0; p < NB / SB; ++p) {
+    for (int p = 0; p <= NB / SB; ++p) {
         const int o = p * SB;
-        if (warp == 0) {
-            const int bad = warp_leaf_chol(a + o * LD + o, LD, lane);
-            if (bad >= 0 && lane == 0) {
+        if (p < NB / SB && warp < 4) {
+            const int bad = leaf_factor128(a + o * LD + o, LD, pv + o, dv + o, tid);
+            if (bad >= 0 && tid == 0) {
                 const int64_t rev = off + o + bad;
                 if (rev < n) record_error(info, static_cast<int>(n - rev));
             }
+        } else if (p > 0 && warp >= 4 && warp < 8) {
+            const int po = o - SB;
+            leaf_inverse128(a + po * LD + po, x + po * LD + po, LD, dv + po, tid - 128);
         }
         __syncthreads();
+        if (p == NB / SB) break;
         const int nr = NB - o - SB;
-        // rows below: forward substitution against the leaf, one thread per row
-        if (tid < nr) {
-            float* row = a + (o + SB + tid) * LD + o;
+        // rows below: warp per row (3 rows interleaved), lane = column of the leaf
+        for (int r0 = warp; r0 < nr; r0 += 3 * NW) {
+            float v[3];
+            int rr[3];
+#pragma unroll
+            for (int u = 0; u < 3; ++u) {
+                rr[u] = r0 + u * NW;
+                v[u] = rr[u] < nr ? a[(o + SB + rr[u]) * LD + o + lane] : 0.0f;
+            }
             const float* L = a + o * LD + o;
 #pragma unroll 1
-            for (int c = 0; c < SB; ++c) {
-                float acc = row[c];
-#pragma unroll 4
-                for (int m = 0; m < c; ++m) acc = fmaf(-row[m], L[c * LD + m], acc);
-                row[c] = __fdiv_rn(acc, L[c * LD + c]);
+            for (int m = 0; m < SB; ++m) {
+                const float lm = L[lane * LD + m];
+                const float dm = dv[o + m];
+#pragma unroll
+                for (int u = 0; u < 3; ++u) {
+                    const float vm = __shfl_sync(0xffffffffu, v[u], m) * dm;
+                    if (lane == m) v[u] = vm;
+                    else if (lane > m) v[u] = fmaf(-vm, lm, v[u]);
+                }
             }
+#pragma unroll
+            for (int u = 0; u < 3; ++u)
+                if (rr[u] < nr) a[(o + SB + rr[u]) * LD + o + lane] = v[u];
         }
         __syncthreads();
-        // trailing update of the lower part of rows/cols [o + SB, NB)
-        for (int e = tid; e < nr * nr; e += blockDim.x) {
-            const int ro = e / nr, co = e % nr;
-            if (co > ro) continue;
-            const float* ar = a + (o + SB + ro) * LD + o;
-            const float* ac = a + (o + SB + co) * LD + o;
-            float acc = 0.0f;
-#pragma unroll 8
-            for (int m = 0; m < SB; ++m) acc = fmaf(ar[m], ac[m], acc);
-            a[(o + SB + ro) * LD + o + SB + co] -= acc;
+        // trailing update of rows/cols [o + SB, NB): 4 x 4 register tiles of the lower part
+        const int nt = nr / 4;
+        for (int e = tid; e < nt * nt; e += blockDim.x) {
+            const int tr = e / nt, tc = e % nt;
+            if (tc > tr) continue;
+            const int r0 = o + SB + 4 * tr, c0 = o + SB + 4 * tc;
+            float acc[4][4] = {};
+#pragma unroll 4
+            for (int m = 0; m < SB; ++m) {
+                float ra[4], cb[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    ra[u] = a[(r0 + u) * LD + o + m];
+                    cb[u] = a[(c0 + u) * LD + o + m];
+                }
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+#pragma unroll
+                    for (int v2 = 0; v2 < 4; ++v2) acc[u][v2] = fmaf(ra[u], cb[v2], acc[u][v2]);
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+                for (int v2 = 0; v2 < 4; ++v2)
+                    if (c0 + v2 <= r0 + u) a[(r0 + u) * LD + c0 + v2] -= acc[u][v2];
         }
         __syncthreads();
     }
-    if (warp < NB / SB) warp_leaf_inv(a + warp * SB * LD + warp * SB, x + warp * SB * LD + warp * SB, LD, lane);
-    __syncthreads();
+    // off-diagonal leaves of X, by distance d = q - p, 4 x 4 register tiles
     for (int d = 1; d < NB / SB; ++d) {
         const int nblk = NB / SB - d;
-        for (int e = tid; e < nblk * SB * SB; e += blockDim.x) {   // T_qp = sum_r C_qr X_rp
-            const int b = e / (SB * SB), i = (e / SB) % SB, c = e % SB;
+        for (int e = tid; e < nblk * 64; e += blockDim.x) {   // T_qp = sum_r C_qr X_rp
+            const int b = e >> 6, ti = (e >> 3) & 7, tj = e & 7;
             const int pp = b, qq = b + d;
-            float acc = 0.0f;
+            float acc[4][4] = {};
             for (int r2 = pp; r2 < qq; ++r2) {
-                const float* crow = a + (qq * SB + i) * LD + r2 * SB;
-                const float* xcol = x + (r2 * SB) * LD + pp * SB + c;
-#pragma unroll 8
-                for (int m = 0; m < SB; ++m) acc = fmaf(crow[m], xcol[m * LD], acc);
+#pragma unroll 4
+                for (int m = 0; m < SB; ++m) {
+                    float ca[4], xb[4];
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        ca[u] = a[(qq * SB + 4 * ti + u) * LD + r2 * SB + m];
+                        xb[u] = x[(r2 * SB + m) * LD + pp * SB + 4 * tj + u];
+                    }
+#pragma unroll
+                    for (int u = 0; u < 4; ++u)
+#pragma unroll
+                        for (int v2 = 0; v2 < 4; ++v2) acc[u][v2] = fmaf(ca[u], xb[v2], acc[u][v2]);
+                }
             }
-            t[(b * SB + i) * TLDD + c] = acc;
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+                for (int v2 = 0; v2 < 4; ++v2) t[(b * SB + 4 * ti + u) * TLDD + 4 * tj + v2] = acc[u][v2];
         }
         __syncthreads();
-        for (int e = tid; e < nblk * SB * SB; e += blockDim.x) {   // X_qp = -X_qq T_qp
-            const int b = e / (SB * SB), i = (e / SB) % SB, c = e % SB;
+        for (int e = tid; e < nblk * 64; e += blockDim.x) {   // X_qp = -X_qq T_qp
+            const int b = e >> 6, ti = (e >> 3) & 7, tj = e & 7;
             const int pp = b, qq = b + d;
-            const float* xrow = x + (qq * SB + i) * LD + qq * SB;
-            float acc = 0.0f;
-            for (int m = 0; m <= i; ++m) acc = fmaf(xrow[m], t[(b * SB + m) * TLDD + c], acc);
-            x[(qq * SB + i) * LD + pp * SB + c] = -acc;
+            float acc[4][4] = {};
+#pragma unroll 4
+            for (int m = 0; m < SB; ++m) {
+                float xa[4], tb[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    xa[u] = x[(qq * SB + 4 * ti + u) * LD + qq * SB + m];
+                    tb[u] = t[(b * SB + m) * TLDD + 4 * tj + u];
+                }
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+#pragma unroll
+                    for (int v2 = 0; v2 < 4; ++v2) acc[u][v2] = fmaf(xa[u], tb[v2], acc[u][v2]);
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+                for (int v2 = 0; v2 < 4; ++v2) x[(qq * SB + 4 * ti + u) * LD + pp * SB + 4 * tj + v2] = -acc[u][v2];
         }
         __syncthreads();
     }

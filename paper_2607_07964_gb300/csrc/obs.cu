@@ -25,7 +25,8 @@ namespace kq {
 namespace {
 
 constexpr int BLK = 128;          // block size B (Algorithm 2); the only supported value
-constexpr int RLD = BLK + 1;
+constexpr int RTLD = BLK + 4;     // row stride of the staged L block (16-byte rows)
+constexpr int kRowsPerLane = 1;   // rows per lane group in the block kernel
 
 struct Grid {
     float scale, zero;
@@ -77,13 +78,16 @@ __global__ void rowgrid_kernel(const float* __restrict__ W, int64_t d_out, int64
     }
 }
 
-// One block [i0, e) of the sweep for all rows. Four rows per warp: lanes 8g..8g+7 hold
-// row 4 w + g, lane position lp holding columns i0 + 8 t + lp (t = 0..15) in registers.
-// Per column j the owner lane broadcasts w_j inside its 8-lane group; every lane of the
-// group computes the (identical) quantization, then updates its own later columns.
-constexpr int LPR = 8;                 // lanes per row
+// One block [i0, e) of the sweep for all rows. A group of LPR = 4 lanes handles RPL rows;
+// lane position lp holds columns i0 + 4 t + lp (t = 0..31) of each of its rows in registers.
+// Per column j the owner lane broadcasts w_j inside its group; every lane of the group
+// computes the (identical) quantization, then updates its own later columns. The RPL rows
+// of a lane share the loads of R and give independent instruction chains.
+#ifndef KQ_OBS_LANES_PER_ROW
+#define KQ_OBS_LANES_PER_ROW 8
+#endif
+constexpr int LPR = KQ_OBS_LANES_PER_ROW;   // lanes per row group (4 or 8)
 constexpr int CPL = BLK / LPR;         // columns per lane
-constexpr int RPW = 32 / LPR;          // rows per warp
 
 __device__ __forceinline__ float group_min(float v) {
     for (int o = LPR / 2; o > 0; o >>= 1) v = fminf(v, __shfl_xor_sync(0xffffffffu, v, o));
@@ -94,18 +98,31 @@ __device__ __forceinline__ float group_max(float v) {
     return v;
 }
 
-__global__ void __launch_bounds__(128) obs_block_kernel(
+template <int RPL>
+__global__ void __launch_bounds__(128, 3) obs_block_kernel(
     const float* __restrict__ W, int64_t d_out, int64_t d_in, const float* __restrict__ Lt, int64_t i0,
     int bits, int group, const float* __restrict__ gscale, const float* __restrict__ gzero,
     uint8_t* __restrict__ codes, float* __restrict__ scale, int32_t* __restrict__ zero,
-    float* __restrict__ E, float* __restrict__ pre_q) {
-    extern __shared__ float Rs[];   // [BLK][RLD], Rs[j][k] = R[i0 + j][i0 + k] = Lt[i0 + k][i0 + j]
+    float* __restrict__ E, float* __restrict__ pre_q, bool vec) {
+    // The block of L = R^T in its own layout: Rt[k][j] = Lt[i0 + k][i0 + j] = R[i0 + j][i0 + k],
+    // staged with 16-byte cp.async copies (scalar loads when rows are not 16-byte aligned).
+    extern __shared__ __align__(16) float Rt[];   // [BLK][RTLD]
     const int nb = static_cast<int>(min(static_cast<int64_t>(BLK), d_in - i0));
-    for (int e = threadIdx.x; e < BLK * BLK; e += blockDim.x) {
-        const int k = e / BLK, j = e % BLK;   // coalesced over j along row i0 + k of Lt
-        float v = 0.0f;
-        if (j < nb && k < nb && k >= j) v = Lt[(i0 + k) * d_in + i0 + j];
-        Rs[j * RLD + k] = v;
+    if (vec) {
+        for (int e = threadIdx.x; e < BLK * (BLK / 4); e += blockDim.x) {
+            const int k = e >> 5, j4 = (e & 31) * 4;
+            const int valid = k < nb ? max(0, min(4, nb - j4)) : 0;
+            cp_async16(Rt + k * RTLD + j4,
+                       valid ? static_cast<const void*>(Lt + (i0 + k) * d_in + i0 + j4) : static_cast<const void*>(Lt),
+                       4 * valid);
+        }
+        cp_async_commit();
+        cp_async_wait<0>();
+    } else {
+        for (int e = threadIdx.x; e < BLK * BLK; e += blockDim.x) {
+            const int k = e / BLK, j = e % BLK;
+            Rt[k * RTLD + j] = (j < nb && k < nb) ? Lt[(i0 + k) * d_in + i0 + j] : 0.0f;
+        }
     }
     __syncthreads();
     const float maxq = static_cast<float>((1 << bits) - 1);
@@ -114,72 +131,96 @@ __global__ void __launch_bounds__(128) obs_block_kernel(
     const int gbase = lane & ~(LPR - 1);
     const int64_t ngroups = group ? (d_in + group - 1) / group : 1;
     const int warps = blockDim.x / 32;
-    for (int64_t r0 = (static_cast<int64_t>(blockIdx.x) * warps + threadIdx.x / 32) * RPW; r0 < d_out;
-         r0 += static_cast<int64_t>(gridDim.x) * warps * RPW) {
-        const int64_t r = r0 + lane / LPR;
-        const bool live = r < d_out;
-        const float* wr = W + r * d_in + i0;
-        float w[CPL];
+    constexpr int RPW = (32 / LPR) * RPL;   // rows per warp
+    for (int64_t rw = (static_cast<int64_t>(blockIdx.x) * warps + threadIdx.x / 32) * RPW; rw < d_out;
+         rw += static_cast<int64_t>(gridDim.x) * warps * RPW) {
+        int64_t r[RPL];
+        bool live[RPL];
+        float w[RPL][CPL];
+        Grid g[RPL];
 #pragma unroll
-        for (int t = 0; t < CPL; ++t) {
-            const int c = LPR * t + lp;
-            w[t] = (live && c < nb) ? wr[c] : 0.0f;
-        }
-        Grid g;
-        if (group) {
-            float mn = 0.0f, mx = 0.0f;
+        for (int u = 0; u < RPL; ++u) {
+            r[u] = rw + (lane / LPR) * RPL + u;
+            live[u] = r[u] < d_out;
+            const float* wr = W + r[u] * d_in + i0;
 #pragma unroll
-            for (int t = 0; t < CPL; ++t)
-                if (LPR * t + lp < nb) {
-                    mn = fminf(mn, w[t]);
-                    mx = fmaxf(mx, w[t]);
-                }
-            g = make_grid(group_min(mn), group_max(mx), maxq);
-            if (live && lp == 0) {
-                const int64_t gi = r * ngroups + i0 / group;
-                scale[gi] = g.scale;
-                zero[gi] = static_cast<int32_t>(g.zero);
+            for (int t = 0; t < CPL; ++t) {
+                const int c = LPR * t + lp;
+                w[u][t] = (live[u] && c < nb) ? wr[c] : 0.0f;
             }
-        } else {
-            g.scale = live ? gscale[r] : 1.0f;
-            g.zero = live ? gzero[r] : 0.0f;
+            if (group) {
+                float mn = 0.0f, mx = 0.0f;
+#pragma unroll
+                for (int t = 0; t < CPL; ++t)
+                    if (LPR * t + lp < nb) {
+                        mn = fminf(mn, w[u][t]);
+                        mx = fmaxf(mx, w[u][t]);
+                    }
+                g[u] = make_grid(group_min(mn), group_max(mx), maxq);
+                if (live[u] && lp == 0) {
+                    const int64_t gi = r[u] * ngroups + i0 / group;
+                    scale[gi] = g[u].scale;
+                    zero[gi] = static_cast<int32_t>(g[u].zero);
+                }
+            } else {
+                g[u].scale = live[u] ? gscale[r[u]] : 1.0f;
+                g[u].zero = live[u] ? gzero[r[u]] : 0.0f;
+            }
         }
-        // Slot q of the block is always w[0]: after its 8 columns the registers shift down
-        // by one, which keeps the loop rolled (compact code) with register-only indexing.
+        // Slot q of the block is always w[.][0]: after its 8 columns the registers shift
+        // down by one, which keeps the loop rolled (compact code) with register indexing.
 #pragma unroll 1
         for (int q = 0; q < CPL; ++q) {
-            float e_cur = 0.0f, pq_cur = 0.0f;
-            uint32_t q_cur = 0;
+            float e_cur[RPL], pq_cur[RPL];
+            uint32_t q_cur[RPL];
+#pragma unroll
+            for (int u = 0; u < RPL; ++u) {
+                e_cur[u] = 0.0f;
+                pq_cur[u] = 0.0f;
+                q_cur[u] = 0;
+            }
 #pragma unroll
             for (int jl = 0; jl < LPR; ++jl) {
                 const int j = LPR * q + jl;
                 if (j < nb) {   // uniform across the warp
-                    const float wj = __shfl_sync(0xffffffffu, w[0], gbase | jl);
-                    float qq = __fadd_rn(rintf(__fdiv_rn(wj, g.scale)), g.zero);
-                    qq = fminf(fmaxf(qq, 0.0f), maxq);
-                    const float what = __fmul_rn(g.scale, __fsub_rn(qq, g.zero));
-                    const float err = __fdiv_rn(__fsub_rn(wj, what), Rs[j * RLD + j]);
-                    if (lp == jl) {
-                        e_cur = err;
-                        q_cur = static_cast<uint32_t>(qq);
-                        pq_cur = wj;
+                    const float dj = Rt[j * RTLD + j];
+                    float err[RPL];
+#pragma unroll
+                    for (int u = 0; u < RPL; ++u) {
+                        const float wj = __shfl_sync(0xffffffffu, w[u][0], gbase | jl);
+                        float qq = __fadd_rn(rintf(__fdiv_rn(wj, g[u].scale)), g[u].zero);
+                        qq = fminf(fmaxf(qq, 0.0f), maxq);
+                        const float what = __fmul_rn(g[u].scale, __fsub_rn(qq, g[u].zero));
+                        err[u] = __fdiv_rn(__fsub_rn(wj, what), dj);
+                        if (lp == jl) {
+                            e_cur[u] = err[u];
+                            q_cur[u] = static_cast<uint32_t>(qq);
+                            pq_cur[u] = wj;
+                        }
                     }
-                    const float* rrow = Rs + j * RLD + LPR * q + lp;
+                    const float* rcol = Rt + (LPR * q + lp) * RTLD + j;   // R[j][k] = Rt[k][j]
 #pragma unroll
                     for (int t = 0; t < CPL; ++t) {
-                        if (t < CPL - q && LPR * (q + t) + lp > j) w[t] = __fmaf_rn(-err, rrow[LPR * t], w[t]);
+                        if (t < CPL - q && LPR * (q + t) + lp > j) {
+                            const float rv = rcol[LPR * t * RTLD];
+#pragma unroll
+                            for (int u = 0; u < RPL; ++u) w[u][t] = __fmaf_rn(-err[u], rv, w[u][t]);
+                        }
                     }
                 }
             }
             const int c = LPR * q + lp;
-            if (live && c < nb) {
-                codes[r * d_in + i0 + c] = static_cast<uint8_t>(q_cur);
-                E[r * d_in + i0 + c] = e_cur;
-                if (pre_q) pre_q[r * d_in + i0 + c] = pq_cur;
-            }
 #pragma unroll
-            for (int t = 0; t + 1 < CPL; ++t) w[t] = w[t + 1];
-            w[CPL - 1] = 0.0f;
+            for (int u = 0; u < RPL; ++u) {
+                if (live[u] && c < nb) {
+                    codes[r[u] * d_in + i0 + c] = static_cast<uint8_t>(q_cur[u]);
+                    E[r[u] * d_in + i0 + c] = e_cur[u];
+                    if (pre_q) pre_q[r[u] * d_in + i0 + c] = pq_cur[u];
+                }
+#pragma unroll
+                for (int t = 0; t + 1 < CPL; ++t) w[u][t] = w[u][t + 1];
+                w[u][CPL - 1] = 0.0f;
+            }
         }
     }
 }
@@ -297,8 +338,8 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
     }
     static bool attr = false;
     if (!attr) {
-        KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     BLK * RLD * 4));
+        KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel<kRowsPerLane>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     BLK * RTLD * 4));
         KQ_CUDA(cudaFuncSetAttribute(trailing_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(G_SMEM)));
         KQ_CUDA(cudaFuncSetAttribute(trailing_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -312,11 +353,12 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
         KQ_LAUNCH_CHECK("rowgrid_kernel");
     }
     const bool vec = (d_in % 4 == 0) && (reinterpret_cast<uintptr_t>(Lt) % 16 == 0);
-    const int64_t row_ctas = std::min<int64_t>(cdiv(d_out, 4 * RPW), static_cast<int64_t>(num_sms()) * 3);
+    const int64_t rows_per_cta = 4 * (32 / LPR) * kRowsPerLane;   // 4 warps per CTA
+    const int64_t row_ctas = std::min<int64_t>(cdiv(d_out, rows_per_cta), static_cast<int64_t>(num_sms()) * 3);
     for (int64_t i0 = 0; i0 < d_in; i0 += BLK) {
         const int kb = static_cast<int>(std::min<int64_t>(BLK, d_in - i0));
-        obs_block_kernel<<<static_cast<unsigned>(row_ctas), 128, BLK * RLD * 4, stream>>>(
-            W, d_out, d_in, Lt, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q);
+        obs_block_kernel<kRowsPerLane><<<static_cast<unsigned>(row_ctas), 128, BLK * RTLD * 4, stream>>>(
+            W, d_out, d_in, Lt, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q, vec);
         KQ_LAUNCH_CHECK("obs_block_kernel");
         const int64_t rest = d_in - (i0 + kb);
         if (rest > 0) {
