@@ -71,7 +71,7 @@ __global__ void prep_kernel(const float* __restrict__ H, int64_t n, int64_t npad
 }
 
 // ---------------------------------------------------------------- diag block
-constexpr int DIAG_THREADS = 1024;
+constexpr int DIAG_THREADS = 512;
 constexpr int SB = 32;                        // leaf size inside the diagonal block
 constexpr int TLDD = SB + 1;
 constexpr size_t DIAG_SMEM = (2 * TILE_FLOATS + NB * TLDD + 2 * NB) * sizeof(float);
@@ -93,7 +93,21 @@ __device__ __forceinline__ int leaf_factor128(float* s, int ld, float* pv, float
         if (!(p > 0.0f) && bad < 0) bad = j;
         if (i > j) {
             const float f = s[i * ld + j] * __fdiv_rn(1.0f, p);
-            for (int k = j + 1 + q; k <= i; k += 4) s[i * ld + k] = fmaf(-f, s[k * ld + j], s[i * ld + k]);
+            // at most 8 columns per thread: unrolled so all loads are issued together
+            float sk[8], si[8];
+#pragma unroll
+            for (int m = 0; m < 8; ++m) {
+                const int k = j + 1 + q + 4 * m;
+                if (k <= i) {
+                    sk[m] = s[k * ld + j];
+                    si[m] = s[i * ld + k];
+                }
+            }
+#pragma unroll
+            for (int m = 0; m < 8; ++m) {
+                const int k = j + 1 + q + 4 * m;
+                if (k <= i) s[i * ld + k] = fmaf(-f, sk[m], si[m]);
+            }
         }
         if (t == 0) pv[j] = p;
         named_barrier(1, 128);
@@ -127,7 +141,21 @@ __device__ __forceinline__ void leaf_inverse128(const float* L, float* X, int ld
             X[i * ld + c] = xi;
         }
         xi = __shfl_sync(0xffffffffu, xi, gbase | (i & 3));
-        for (int r = i + 1 + ((q - i - 1) & 3); r < SB; r += 4) X[r * ld + c] = fmaf(-L[r * ld + i], xi, X[r * ld + c]);
+        const int r0 = i + 1 + ((q - i - 1) & 3);   // first row > i owned by this lane
+        float lr[8], xr[8];
+#pragma unroll
+        for (int m = 0; m < 8; ++m) {
+            const int r = r0 + 4 * m;
+            if (r < SB) {
+                lr[m] = L[r * ld + i];
+                xr[m] = X[r * ld + c];
+            }
+        }
+#pragma unroll
+        for (int m = 0; m < 8; ++m) {
+            const int r = r0 + 4 * m;
+            if (r < SB) X[r * ld + c] = fmaf(-lr[m], xi, xr[m]);
+        }
         __syncwarp();
     }
 }
@@ -180,7 +208,7 @@ __global__ void __launch_bounds__(DIAG_THREADS) chol_diag_kernel(Work w, int64_t
                 v[u] = rr[u] < nr ? a[(o + SB + rr[u]) * LD + o + lane] : 0.0f;
             }
             const float* L = a + o * LD + o;
-#pragma unroll 1
+#pragma unroll 4
             for (int m = 0; m < SB; ++m) {
                 const float lm = L[lane * LD + m];
                 const float dm = dv[o + m];
