@@ -106,14 +106,16 @@ KQ_API kq_status kq_accum_factor(const uint16_t* A, int64_t T, int64_t d, int64_
  * kq_compute_scales: s_x [d_in] and s_g [d_out] (fp32) from the ORIGINAL W [d_out x d_in]
  *   fp32 and the diagonals of the raw H_X [d_in x d_in] and H_G [d_out x d_out]. Norms are
  *   summed in fp64; s = sqrt(sqrt(h / a)), and s = 1 when h == 0 or a == 0 (a dead
- *   channel). Must run before either rotation. H_G may be NULL (then s_g = 1; the
- *   one-sided variant).
+ *   channel). Must run before either rotation. Each side is computed only if its output
+ *   is non-NULL (s_x needs H_X); with H_G NULL, s_g = 1 (the one-sided variant). So the
+ *   two sides can run on two streams as soon as their own factor exists.
  *
  * kq_traces: the sensitivity statistics of Sec. 3.3 Eq. (sensitivity), from the raw
  *   factors' diagonals and the scales (call before the rotations overwrite H_X / H_G).
  *   out [6] (device double): tr(H_X), tr(H_G), tr(H_X) tr(H_G), and the post-BiIP
  *   tr(H_X'), tr(H_G'), tr(H_X') tr(H_G') with tr(H') = sum_j H_jj / s_j^2 (the rotations
- *   preserve the trace).
+ *   preserve the trace). A NULL factor leaves its side of out untouched and the products
+ *   use the values already in out, so the sides may come from two calls (X side first).
  *
  * kq_rotate_in (input side, length d_in, sign_v = sigma_V):
  *   dir = KQ_FWD: W <- (W S_X) V^T, and if H_X != NULL: H_X <- V S_X^-1 H_X S_X^-1 V^T.
@@ -121,7 +123,8 @@ KQ_API kq_status kq_accum_factor(const uint16_t* A, int64_t T, int64_t d, int64_
  * kq_rotate_out (output side, length d_out, sign_u = sigma_U):
  *   dir = KQ_FWD: W <- U (S_G W), and if H_G != NULL: H_G <- U S_G^-1 H_G S_G^-1 U^T.
  *   dir = KQ_INV: W <- S_G^-1 (U^T W).
- *   All in place, fp32. s_x / s_g may be NULL for a pure rotation (S = I).
+ *   All in place, fp32. s_x / s_g may be NULL for a pure rotation (S = I). In the FWD
+ *   direction W may be NULL to transform only the factor (H_X or H_G).
  *   Returns KQ_ERR_UNSUPPORTED if the length has no Hadamard construction.
  * ---------------------------------------------------------------------------------- */
 #define KQ_FWD 0
@@ -130,6 +133,21 @@ KQ_API kq_status kq_compute_scales(const float* W, int64_t d_out, int64_t d_in, 
                             const float* H_G, float* s_x, float* s_g, kq_stream_t stream);
 KQ_API kq_status kq_traces(const float* H_X, const float* s_x, int64_t d_in, const float* H_G,
                     const float* s_g, int64_t d_out, double* out, kq_stream_t stream);
+/*
+ * kq_factor_diag: diag(A^T A) alone (the per-channel sums of squares; for G these are the
+ *   only entries of H_G that the quantization reads, through S_G and the traces -- Prop. 1).
+ *   diag [d] fp32 from fp64 sums in a fixed order (deterministic), trace (device double,
+ *   nullable) = their fp64 total. Reads A once. ws: kq_factor_diag_workspace(T, d) bytes.
+ * kq_compute_scales_diag / kq_traces_diag: kq_compute_scales / kq_traces with the factors'
+ *   diagonals given as vectors (stride 1) instead of the full matrices.
+ */
+KQ_API size_t kq_factor_diag_workspace(int64_t T, int64_t d);
+KQ_API kq_status kq_factor_diag(const uint16_t* A, int64_t T, int64_t d, int64_t lda, float* diag, double* trace,
+                                void* ws, size_t ws_bytes, kq_stream_t stream);
+KQ_API kq_status kq_compute_scales_diag(const float* W, int64_t d_out, int64_t d_in, const float* hx_diag,
+                                        const float* hg_diag, float* s_x, float* s_g, kq_stream_t stream);
+KQ_API kq_status kq_traces_diag(const float* hx_diag, const float* s_x, int64_t d_in, const float* hg_diag,
+                                const float* s_g, int64_t d_out, double* out, kq_stream_t stream);
 KQ_API kq_status kq_rotate_in(float* W, int64_t d_out, int64_t d_in, float* H_X, const float* s_x,
                        const int8_t* sign_v, int dir, kq_stream_t stream);
 KQ_API kq_status kq_rotate_out(float* W, int64_t d_out, int64_t d_in, float* H_G, const float* s_g,

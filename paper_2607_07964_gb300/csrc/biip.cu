@@ -13,6 +13,8 @@
 // a Walsh-Hadamard butterfly and the 28-point factor a dense +-1 mix at stride 2^k.
 #include <math.h>
 
+#include <algorithm>
+
 #include "kq_common.cuh"
 
 namespace kq {
@@ -298,7 +300,7 @@ __device__ __forceinline__ float quarter_root_ratio(float h, double a) {
 
 // a_j = ||W[:, j]||^2 and s_x[j] = (H_X[j][j] / a_j)^(1/4). Block (32, 8).
 __global__ void colscale_kernel(const float* __restrict__ W, int64_t d_out, int64_t d_in,
-                                const float* __restrict__ HX, float* __restrict__ s_x) {
+                                const float* __restrict__ HX, int64_t hstride, float* __restrict__ s_x) {
     __shared__ double part[8][33];
     const int64_t j = static_cast<int64_t>(blockIdx.x) * 32 + threadIdx.x;
     double acc = 0.0;
@@ -321,13 +323,13 @@ __global__ void colscale_kernel(const float* __restrict__ W, int64_t d_out, int6
     if (threadIdx.y == 0 && j < d_in) {
         double a = 0.0;
         for (int y = 0; y < 8; ++y) a += part[y][threadIdx.x];
-        s_x[j] = quarter_root_ratio(HX[j * d_in + j], a);
+        s_x[j] = quarter_root_ratio(HX[j * hstride], a);
     }
 }
 
 // r_i = ||W[i, :]||^2 and s_g[i] = (H_G[i][i] / r_i)^(1/4) (1 when H_G is NULL). Warp per row.
 __global__ void rowscale_kernel(const float* __restrict__ W, int64_t d_out, int64_t d_in,
-                                const float* __restrict__ HG, float* __restrict__ s_g) {
+                                const float* __restrict__ HG, int64_t hstride, float* __restrict__ s_g) {
     const int64_t i = static_cast<int64_t>(blockIdx.x) * (blockDim.x / 32) + threadIdx.x / 32;
     const int lane = threadIdx.x & 31;
     if (i >= d_out) return;
@@ -345,27 +347,31 @@ __global__ void rowscale_kernel(const float* __restrict__ W, int64_t d_out, int6
     }
     acc += p;
     for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if (lane == 0) s_g[i] = HG ? quarter_root_ratio(HG[i * d_out + i], acc) : 1.0f;
+    if (lane == 0) s_g[i] = HG ? quarter_root_ratio(HG[i * hstride], acc) : 1.0f;
 }
 
 // out = [tr H_X, tr H_G, product, tr H_X', tr H_G', product'] with tr H' = sum h_j / s_j^2.
-__global__ void traces_kernel(const float* __restrict__ HX, const float* __restrict__ s_x,
-                              int64_t d_in, const float* __restrict__ HG,
+// A NULL factor leaves its entries of out as they are; the products use whatever out then
+// holds for the other side (so the two sides may be filled by two calls, X side first).
+__global__ void traces_kernel(const float* __restrict__ HX, int64_t xstride, const float* __restrict__ s_x,
+                              int64_t d_in, const float* __restrict__ HG, int64_t gstride,
                               const float* __restrict__ s_g, int64_t d_out, double* out) {
     __shared__ double part[4][32];
     double v[4] = {0.0, 0.0, 0.0, 0.0};
-    for (int64_t j = threadIdx.x; j < d_in; j += blockDim.x) {
-        const double h = HX[j * d_in + j];
-        const double sc = s_x ? static_cast<double>(s_x[j]) : 1.0;
-        v[0] += h;
-        v[2] += h / (sc * sc);
-    }
-    for (int64_t i = threadIdx.x; i < d_out; i += blockDim.x) {
-        const double h = HG[i * d_out + i];
-        const double sc = s_g ? static_cast<double>(s_g[i]) : 1.0;
-        v[1] += h;
-        v[3] += h / (sc * sc);
-    }
+    if (HX)
+        for (int64_t j = threadIdx.x; j < d_in; j += blockDim.x) {
+            const double h = HX[j * xstride];
+            const double sc = s_x ? static_cast<double>(s_x[j]) : 1.0;
+            v[0] += h;
+            v[2] += h / (sc * sc);
+        }
+    if (HG)
+        for (int64_t i = threadIdx.x; i < d_out; i += blockDim.x) {
+            const double h = HG[i * gstride];
+            const double sc = s_g ? static_cast<double>(s_g[i]) : 1.0;
+            v[1] += h;
+            v[3] += h / (sc * sc);
+        }
     for (int k = 0; k < 4; ++k) {
         for (int o = 16; o > 0; o >>= 1) v[k] += __shfl_xor_sync(0xffffffffu, v[k], o);
         if ((threadIdx.x & 31) == 0) part[k][threadIdx.x >> 5] = v[k];
@@ -378,14 +384,105 @@ __global__ void traces_kernel(const float* __restrict__ HX, const float* __restr
             v[k] = x;
         }
         if (threadIdx.x == 0) {
-            out[0] = v[0];
-            out[1] = v[1];
-            out[2] = v[0] * v[1];
-            out[3] = v[2];
-            out[4] = v[3];
-            out[5] = v[2] * v[3];
+            if (HX) {
+                out[0] = v[0];
+                out[3] = v[2];
+            }
+            if (HG) {
+                out[1] = v[1];
+                out[4] = v[3];
+            }
+            out[2] = out[0] * out[1];
+            out[5] = out[3] * out[4];
         }
     }
+}
+
+// diag(A^T A): per (row split, 128-column strip) CTA, fp32 partial sums of squares over
+// 32 rows at a time added into fp64; partial[split][j] in the workspace.
+constexpr int DG_COLS = 128;
+constexpr int DG_ROWS = 8;   // row groups per CTA (256 threads = 8 x 32, 4 columns per thread)
+
+__global__ void __launch_bounds__(256) factor_diag_partial_kernel(const uint16_t* __restrict__ A, int64_t T, int64_t d,
+                                                                  int64_t lda, int64_t rows_per_split,
+                                                                  double* __restrict__ partial) {
+    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+    const int64_t c0 = static_cast<int64_t>(blockIdx.x) * DG_COLS + 4 * tx;
+    const int64_t r_begin = static_cast<int64_t>(blockIdx.y) * rows_per_split;
+    const int64_t r_end = min(T, r_begin + rows_per_split);
+    const bool vec = c0 + 4 <= d && (lda & 3) == 0 && (reinterpret_cast<uintptr_t>(A) & 7u) == 0;
+    double acc[4] = {0.0, 0.0, 0.0, 0.0};
+    float p[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    int cnt = 0;
+    // products of bf16 values are exact in fp32; 32-row fp32 partials are added in fp64
+#pragma unroll 4
+    for (int64_t r = r_begin + ty; r < r_end; r += DG_ROWS) {
+        const uint16_t* row = A + r * lda + c0;
+        uint32_t b[4] = {0u, 0u, 0u, 0u};
+        if (vec) {
+            const uint2 v = *reinterpret_cast<const uint2*>(row);
+            b[0] = v.x & 0xFFFFu;
+            b[1] = v.x >> 16;
+            b[2] = v.y & 0xFFFFu;
+            b[3] = v.y >> 16;
+        } else {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) b[u] = (c0 + u < d) ? row[u] : 0u;
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const float x = __uint_as_float(b[u] << 16);
+            p[u] = fmaf(x, x, p[u]);
+        }
+        if (++cnt == 32) {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                acc[u] += p[u];
+                p[u] = 0.0f;
+            }
+            cnt = 0;
+        }
+    }
+    __shared__ double part[DG_ROWS][DG_COLS];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) part[ty][4 * tx + u] = acc[u] + p[u];
+    __syncthreads();
+    if (ty == 0) {
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            double sum = 0.0;
+            for (int y = 0; y < DG_ROWS; ++y) sum += part[y][4 * tx + u];
+            if (c0 + u < d) partial[static_cast<int64_t>(blockIdx.y) * d + c0 + u] = sum;
+        }
+    }
+}
+
+// diag[j] = sum over splits (fixed order), trace = sum_j (one CTA, fixed order per thread).
+__global__ void factor_diag_reduce_kernel(const double* __restrict__ partial, int nsplit, int64_t d,
+                                          float* __restrict__ diag, double* trace) {
+    __shared__ double red[32];
+    double t = 0.0;
+    for (int64_t j = threadIdx.x; j < d; j += blockDim.x) {
+        double s = 0.0;
+        for (int q = 0; q < nsplit; ++q) s += partial[static_cast<int64_t>(q) * d + j];
+        diag[j] = static_cast<float>(s);
+        t += s;
+    }
+    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = t;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        t = threadIdx.x < blockDim.x / 32 ? red[threadIdx.x] : 0.0;
+        for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+        if (threadIdx.x == 0 && trace) *trace = t;
+    }
+}
+
+int diag_splits(int64_t T, int64_t d) {
+    const int64_t strips = cdiv(d, DG_COLS);
+    int64_t s = cdiv(4 * static_cast<int64_t>(num_sms()), strips);
+    s = std::max<int64_t>(1, std::min<int64_t>(s, cdiv(T, 256)));
+    return static_cast<int>(std::min<int64_t>(s, 64));
 }
 
 // ------------------------------------------------------------------ host helpers
@@ -497,40 +594,66 @@ kq_status cols_transform(float* M, int64_t n, int64_t ncols, int pre, int post, 
 
 using namespace kq;
 
-extern "C" kq_status kq_compute_scales(const float* W, int64_t d_out, int64_t d_in, const float* H_X,
-                                       const float* H_G, float* s_x, float* s_g,
-                                       kq_stream_t stream_) {
-    cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
-    if (!W || !H_X || !s_x || !s_g || d_out < 1 || d_in < 1) {
-        set_error("kq_compute_scales: invalid arguments");
+namespace {
+kq_status scales_impl(const float* W, int64_t d_out, int64_t d_in, const float* hx, int64_t xs, const float* hg,
+                      int64_t gs, float* s_x, float* s_g, cudaStream_t stream, const char* who) {
+    if (!W || d_out < 1 || d_in < 1 || (!s_x && !s_g) || (s_x && !hx)) {
+        set_error("%s: invalid arguments", who);
         return KQ_ERR_INVALID_ARG;
     }
-    colscale_kernel<<<static_cast<unsigned>(cdiv(d_in, 32)), dim3(32, 8), 0, stream>>>(W, d_out, d_in,
-                                                                                    H_X, s_x);
-    KQ_LAUNCH_CHECK("colscale_kernel");
-    rowscale_kernel<<<static_cast<unsigned>(cdiv(d_out, 8)), 256, 0, stream>>>(W, d_out, d_in, H_G,
-                                                                              s_g);
-    KQ_LAUNCH_CHECK("rowscale_kernel");
+    if (s_x) {
+        colscale_kernel<<<static_cast<unsigned>(cdiv(d_in, 32)), dim3(32, 8), 0, stream>>>(W, d_out, d_in, hx, xs, s_x);
+        KQ_LAUNCH_CHECK("colscale_kernel");
+    }
+    if (s_g) {
+        rowscale_kernel<<<static_cast<unsigned>(cdiv(d_out, 8)), 256, 0, stream>>>(W, d_out, d_in, hg, gs, s_g);
+        KQ_LAUNCH_CHECK("rowscale_kernel");
+    }
     return KQ_OK;
+}
+
+kq_status traces_impl(const float* hx, int64_t xs, const float* s_x, int64_t d_in, const float* hg, int64_t gs,
+                      const float* s_g, int64_t d_out, double* out, cudaStream_t stream, const char* who) {
+    if ((!hx && !hg) || !out || (hx && d_in < 1) || (hg && d_out < 1)) {
+        set_error("%s: invalid arguments", who);
+        return KQ_ERR_INVALID_ARG;
+    }
+    traces_kernel<<<1, 1024, 0, stream>>>(hx, xs, s_x, d_in, hg, gs, s_g, d_out, out);
+    KQ_LAUNCH_CHECK("traces_kernel");
+    return KQ_OK;
+}
+}  // namespace
+
+extern "C" kq_status kq_compute_scales(const float* W, int64_t d_out, int64_t d_in, const float* H_X,
+                                       const float* H_G, float* s_x, float* s_g, kq_stream_t stream_) {
+    return scales_impl(W, d_out, d_in, H_X, d_in + 1, H_G, d_out + 1, s_x, s_g,
+                       reinterpret_cast<cudaStream_t>(stream_), "kq_compute_scales");
+}
+
+extern "C" kq_status kq_compute_scales_diag(const float* W, int64_t d_out, int64_t d_in, const float* hx_diag,
+                                            const float* hg_diag, float* s_x, float* s_g, kq_stream_t stream_) {
+    return scales_impl(W, d_out, d_in, hx_diag, 1, hg_diag, 1, s_x, s_g, reinterpret_cast<cudaStream_t>(stream_),
+                       "kq_compute_scales_diag");
 }
 
 extern "C" kq_status kq_traces(const float* H_X, const float* s_x, int64_t d_in, const float* H_G,
                                const float* s_g, int64_t d_out, double* out, kq_stream_t stream_) {
-    cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
-    if (!H_X || !H_G || !out || d_in < 1 || d_out < 1) {
-        set_error("kq_traces: invalid arguments");
-        return KQ_ERR_INVALID_ARG;
-    }
-    traces_kernel<<<1, 1024, 0, stream>>>(H_X, s_x, d_in, H_G, s_g, d_out, out);
-    KQ_LAUNCH_CHECK("traces_kernel");
-    return KQ_OK;
+    return traces_impl(H_X, d_in + 1, s_x, d_in, H_G, d_out + 1, s_g, d_out, out,
+                       reinterpret_cast<cudaStream_t>(stream_), "kq_traces");
+}
+
+extern "C" kq_status kq_traces_diag(const float* hx_diag, const float* s_x, int64_t d_in, const float* hg_diag,
+                                    const float* s_g, int64_t d_out, double* out, kq_stream_t stream_) {
+    return traces_impl(hx_diag, 1, s_x, d_in, hg_diag, 1, s_g, d_out, out, reinterpret_cast<cudaStream_t>(stream_),
+                       "kq_traces_diag");
 }
 
 extern "C" kq_status kq_rotate_in(float* W, int64_t d_out, int64_t d_in, float* H_X, const float* s_x,
                                   const int8_t* sign_v, int dir, kq_stream_t stream_) {
     cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
     HadamardPlan p;
-    if (!W || !sign_v || d_out < 1 || d_in < 1 || (dir != KQ_FWD && dir != KQ_INV)) {
+    if ((!W && !(H_X && dir == KQ_FWD)) || !sign_v || d_in < 1 || (W && d_out < 1) ||
+        (dir != KQ_FWD && dir != KQ_INV)) {
         set_error("kq_rotate_in: invalid arguments");
         return KQ_ERR_INVALID_ARG;
     }
@@ -541,8 +664,10 @@ extern "C" kq_status kq_rotate_in(float* W, int64_t d_out, int64_t d_in, float* 
     kq_status st;
     if (dir == KQ_FWD) {
         // W <- (W S_X) V^T: each row times sigma_j s_j, then H_n, then 1/sqrt(n).
-        st = rows_transform(W, d_out, d_in, s_x ? F_SMUL : F_SIGN, F_NONE, sign_v, s_x, stream);
-        if (st != KQ_OK) return st;
+        if (W) {
+            st = rows_transform(W, d_out, d_in, s_x ? F_SMUL : F_SIGN, F_NONE, sign_v, s_x, stream);
+            if (st != KQ_OK) return st;
+        }
         if (H_X) {
             // H_X <- V S_X^-1 H_X S_X^-1 V^T: both sides scaled by sigma / s, then H_n twice.
             st = rows_transform(H_X, d_in, d_in, s_x ? F_SDIV : F_SIGN, F_NONE, sign_v, s_x, stream);
@@ -562,7 +687,8 @@ extern "C" kq_status kq_rotate_out(float* W, int64_t d_out, int64_t d_in, float*
                                    const int8_t* sign_u, int dir, kq_stream_t stream_) {
     cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
     HadamardPlan p;
-    if (!W || !sign_u || d_out < 1 || d_in < 1 || (dir != KQ_FWD && dir != KQ_INV)) {
+    if ((!W && !(H_G && dir == KQ_FWD)) || !sign_u || d_out < 1 || (W && d_in < 1) ||
+        (dir != KQ_FWD && dir != KQ_INV)) {
         set_error("kq_rotate_out: invalid arguments");
         return KQ_ERR_INVALID_ARG;
     }
@@ -573,8 +699,10 @@ extern "C" kq_status kq_rotate_out(float* W, int64_t d_out, int64_t d_in, float*
     kq_status st;
     if (dir == KQ_FWD) {
         // W <- U (S_G W): rows scaled by sigma_i s_i, then H_n along the row index.
-        st = cols_transform(W, d_out, d_in, s_g ? F_SMUL : F_SIGN, F_NONE, sign_u, s_g, stream);
-        if (st != KQ_OK) return st;
+        if (W) {
+            st = cols_transform(W, d_out, d_in, s_g ? F_SMUL : F_SIGN, F_NONE, sign_u, s_g, stream);
+            if (st != KQ_OK) return st;
+        }
         if (H_G) {
             st = rows_transform(H_G, d_out, d_out, s_g ? F_SDIV : F_SIGN, F_NONE, sign_u, s_g, stream);
             if (st != KQ_OK) return st;
@@ -600,3 +728,34 @@ kq_status rotate_cols_inv(float* M, int64_t n, int64_t ncols, const float* s, co
     return cols_transform(M, n, ncols, F_NONE, s ? F_SDIV : F_SIGN, sign, s, stream);
 }
 }  // namespace kq
+
+extern "C" size_t kq_factor_diag_workspace(int64_t T, int64_t d) {
+    if (d < 1 || T < 0) return 0;
+    return 64 * static_cast<size_t>(d) * sizeof(double) + 256;
+}
+
+extern "C" kq_status kq_factor_diag(const uint16_t* A, int64_t T, int64_t d, int64_t lda, float* diag, double* trace,
+                                    void* ws, size_t ws_bytes, kq_stream_t stream_) {
+    cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+    if (!diag || d < 1 || T < 0 || (T > 0 && !A) || lda < d) {
+        set_error("kq_factor_diag: invalid arguments");
+        return KQ_ERR_INVALID_ARG;
+    }
+    if (!ws || ws_bytes < kq_factor_diag_workspace(T, d) || (reinterpret_cast<uintptr_t>(ws) & 15u)) {
+        set_error("kq_factor_diag: workspace must be 16-byte aligned and hold %zu bytes", kq_factor_diag_workspace(T, d));
+        return KQ_ERR_WORKSPACE;
+    }
+    const int nsplit = T > 0 ? diag_splits(T, d) : 1;
+    double* partial = static_cast<double*>(ws);
+    if (T > 0) {
+        const int64_t rows_per_split = cdiv(T, nsplit);
+        dim3 grid(static_cast<unsigned>(cdiv(d, DG_COLS)), static_cast<unsigned>(nsplit));
+        factor_diag_partial_kernel<<<grid, 256, 0, stream>>>(A, T, d, lda, rows_per_split, partial);
+        KQ_LAUNCH_CHECK("factor_diag_partial_kernel");
+    } else {
+        KQ_CUDA(cudaMemsetAsync(partial, 0, sizeof(double) * d, stream));
+    }
+    factor_diag_reduce_kernel<<<1, 1024, 0, stream>>>(partial, nsplit, d, diag, trace);
+    KQ_LAUNCH_CHECK("factor_diag_reduce_kernel");
+    return KQ_OK;
+}

@@ -44,6 +44,10 @@ def lib() -> ctypes.CDLL:
             "kq_check": ([P, I, P, P], I),
             "kq_accum_factor": ([P, I64, I64, I64, P, I, P, P, P], I),
             "kq_compute_scales": ([P, I64, I64, P, P, P, P, P], I),
+            "kq_compute_scales_diag": ([P, I64, I64, P, P, P, P, P], I),
+            "kq_traces_diag": ([P, P, I64, P, P, I64, P, P], I),
+            "kq_factor_diag_workspace": ([I64, I64], SZ),
+            "kq_factor_diag": ([P, I64, I64, I64, P, P, P, SZ, P], I),
             "kq_traces": ([P, P, I64, P, P, I64, P, P], I),
             "kq_rotate_in": ([P, I64, I64, P, P, P, I, P], I),
             "kq_rotate_out": ([P, I64, I64, P, P, P, I, P], I),
@@ -129,6 +133,7 @@ def kq_accum_factor(A, H, accumulate: bool = False, trace=None, info=None, strea
 
 
 def kq_compute_scales(W, H_X, H_G, s_x, s_g, stream=None) -> None:
+    """s_x and/or s_g (each side computed only if its output is given)."""
     d_out, d_in = W.shape
     _need(W, "W", torch.float32)
     _need(H_X, "H_X", torch.float32, (d_in, d_in))
@@ -140,7 +145,9 @@ def kq_compute_scales(W, H_X, H_G, s_x, s_g, stream=None) -> None:
 
 
 def kq_traces(H_X, s_x, H_G, s_g, out, stream=None) -> None:
-    d_in, d_out = H_X.shape[0], H_G.shape[0]
+    """Sensitivity traces; either factor may be None (that side of `out` is kept)."""
+    d_in = 0 if H_X is None else H_X.shape[0]
+    d_out = 0 if H_G is None else H_G.shape[0]
     _need(H_X, "H_X", torch.float32, (d_in, d_in))
     _need(H_G, "H_G", torch.float32, (d_out, d_out))
     _need(s_x, "s_x", torch.float32, (d_in,))
@@ -150,8 +157,52 @@ def kq_traces(H_X, s_x, H_G, s_g, out, stream=None) -> None:
                         _stream(stream)), "kq_traces")
 
 
-def kq_rotate_in(W, H_X, s_x, sign_v, direction: int = KQ_FWD, stream=None) -> None:
+def kq_factor_diag_workspace(T: int, d: int) -> int:
+    return int(lib().kq_factor_diag_workspace(T, d))
+
+
+def kq_factor_diag(A, diag, trace=None, ws=None, stream=None) -> None:
+    """diag(A^T A) (fp64 sums, fp32 result) and optionally its total; A [T, d] bf16."""
+    if A.dim() != 2 or A.stride(1) != 1:
+        raise ValueError("A must be 2-D with unit column stride")
+    T, d = A.shape
+    _need(A, "A", torch.bfloat16, contiguous=False)
+    _need(diag, "diag", torch.float32, (d,))
+    _need(trace, "trace", torch.float64)
+    _need(ws, "ws", torch.uint8)
+    _ok(lib().kq_factor_diag(_ptr(A), T, d, A.stride(0), _ptr(diag), _ptr(trace), _ptr(ws),
+                             0 if ws is None else ws.numel(), _stream(stream)), "kq_factor_diag")
+
+
+def kq_compute_scales_diag(W, hx_diag, hg_diag, s_x, s_g, stream=None) -> None:
     d_out, d_in = W.shape
+    _need(W, "W", torch.float32)
+    _need(hx_diag, "hx_diag", torch.float32, (d_in,))
+    _need(hg_diag, "hg_diag", torch.float32, (d_out,))
+    _need(s_x, "s_x", torch.float32, (d_in,))
+    _need(s_g, "s_g", torch.float32, (d_out,))
+    _ok(lib().kq_compute_scales_diag(_ptr(W), d_out, d_in, _ptr(hx_diag), _ptr(hg_diag), _ptr(s_x), _ptr(s_g),
+                                     _stream(stream)), "kq_compute_scales_diag")
+
+
+def kq_traces_diag(hx_diag, s_x, hg_diag, s_g, out, stream=None) -> None:
+    d_in = 0 if hx_diag is None else hx_diag.shape[0]
+    d_out = 0 if hg_diag is None else hg_diag.shape[0]
+    _need(hx_diag, "hx_diag", torch.float32, (d_in,))
+    _need(hg_diag, "hg_diag", torch.float32, (d_out,))
+    _need(s_x, "s_x", torch.float32, (d_in,))
+    _need(s_g, "s_g", torch.float32, (d_out,))
+    _need(out, "out", torch.float64, (6,))
+    _ok(lib().kq_traces_diag(_ptr(hx_diag), _ptr(s_x), d_in, _ptr(hg_diag), _ptr(s_g), d_out, _ptr(out),
+                             _stream(stream)), "kq_traces_diag")
+
+
+def kq_rotate_in(W, H_X, s_x, sign_v, direction: int = KQ_FWD, stream=None, d_out: int = 0) -> None:
+    """W may be None (then only H_X is transformed, forward direction)."""
+    if W is not None:
+        d_out, d_in = W.shape
+    else:
+        d_in = H_X.shape[0]
     _need(W, "W", torch.float32)
     _need(H_X, "H_X", torch.float32, (d_in, d_in))
     _need(s_x, "s_x", torch.float32, (d_in,))
@@ -160,8 +211,12 @@ def kq_rotate_in(W, H_X, s_x, sign_v, direction: int = KQ_FWD, stream=None) -> N
                            _stream(stream)), "kq_rotate_in")
 
 
-def kq_rotate_out(W, H_G, s_g, sign_u, direction: int = KQ_FWD, stream=None) -> None:
-    d_out, d_in = W.shape
+def kq_rotate_out(W, H_G, s_g, sign_u, direction: int = KQ_FWD, stream=None, d_in: int = 0) -> None:
+    """W may be None (then only H_G is transformed, forward direction)."""
+    if W is not None:
+        d_out, d_in = W.shape
+    else:
+        d_out = H_G.shape[0]
     _need(W, "W", torch.float32)
     _need(H_G, "H_G", torch.float32, (d_out, d_out))
     _need(s_g, "s_g", torch.float32, (d_out,))

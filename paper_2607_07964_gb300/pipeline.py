@@ -16,7 +16,8 @@ class LayerPipeline:
     """Device buffers for one layer shape and the stage sequence that fills them."""
 
     def __init__(self, d_out: int, d_in: int, bits: int, group: int, block: int = 128,
-                 damp: float = 0.01, device: str = "cuda", want_col_loss: bool = True):
+                 damp: float = 0.01, device: str = "cuda", want_col_loss: bool = True,
+                 overlap: bool = True):
         self.d_out, self.d_in, self.bits, self.group, self.block, self.damp = d_out, d_in, bits, group, block, damp
         f32 = dict(dtype=torch.float32, device=device)
         ng = 1 if group == 0 else -(-d_in // group)
@@ -37,30 +38,44 @@ class LayerPipeline:
         self.ws_chol = torch.empty((kq.kq_chol_inv_workspace(d_in),), dtype=torch.uint8, device=device)
         self.ws_obs = torch.empty((kq.kq_obs_quantize_workspace(d_out, d_in, block),), dtype=torch.uint8,
                                   device=device)
+        # Output-side work (H_G, S_G, U) runs on a second stream beside the Cholesky, which
+        # needs only H_X and leaves most SMs idle during its diagonal steps.
+        # The critical path (H_X, Cholesky, sweep) runs on a high-priority stream so SMs freed
+        # by the long-running H_G tiles go to it first.
+        self.overlap = overlap
+        try:
+            lo, hi = torch.cuda.Stream.priority_range()
+        except (AttributeError, RuntimeError):
+            lo, hi = 0, -1
+        self.main = torch.cuda.Stream(device=device, priority=hi) if overlap else None
+        self.side = torch.cuda.Stream(device=device, priority=lo) if overlap else None
+        self._ev = [torch.cuda.Event() for _ in range(6)]
 
     def run(self, X, G, W, sign_u, sign_v, stream=None, events=None) -> None:
         """X [T, d_in] bf16, G [T, d_out] bf16, W [d_out, d_in] fp32 (left unchanged), signs
         int8. `events`, if given, is a list of len(STAGES) + 1 CUDA events recorded at the
         stage boundaries on the stream."""
         s = torch.cuda.current_stream() if stream is None else stream
+        if self.overlap and events is None:
+            self._run_overlapped(X, G, W, sign_u, sign_v, s)
+            return
 
         def mark(i):
             if events is not None:
                 events[i].record(s)
 
-        info = self.info[0:1]
         mark(0)
-        kq.kq_accum_factor(X, self.HX, trace=self.trace_x, info=info, stream=s)        # Alg. 1: H_X
+        kq.kq_accum_factor(X, self.HX, trace=self.trace_x, info=self.info[0:1], stream=s)   # Alg. 1: H_X
         mark(1)
-        kq.kq_accum_factor(G, self.HG, trace=self.trace_g, info=info, stream=s)        # H_G
+        kq.kq_accum_factor(G, self.HG, trace=self.trace_g, info=self.info[2:3], stream=s)   # H_G
         mark(2)
-        kq.kq_compute_scales(W, self.HX, self.HG, self.s_x, self.s_g, stream=s)      # Eq. (rescale)
-        kq.kq_traces(self.HX, self.s_x, self.HG, self.s_g, self.traces, stream=s)     # Eq. (sensitivity)
+        kq.kq_compute_scales(W, self.HX, self.HG, self.s_x, self.s_g, stream=s)          # Eq. (rescale)
+        kq.kq_traces(self.HX, self.s_x, self.HG, self.s_g, self.traces, stream=s)         # Eq. (sensitivity)
         mark(3)
         with torch.cuda.stream(s):
             self.Wp.copy_(W)
-        kq.kq_rotate_in(self.Wp, self.HX, self.s_x, sign_v, kq.KQ_FWD, stream=s)     # Eq. (biip), V side
-        kq.kq_rotate_out(self.Wp, self.HG, self.s_g, sign_u, kq.KQ_FWD, stream=s)    # U side; H_G released
+        kq.kq_rotate_in(self.Wp, self.HX, self.s_x, sign_v, kq.KQ_FWD, stream=s)         # Eq. (biip), V side
+        kq.kq_rotate_out(self.Wp, self.HG, self.s_g, sign_u, kq.KQ_FWD, stream=s)        # U side; H_G released
         mark(4)
         kq.kq_chol_inv(self.HX, self.damp, self.Lt, self.info[1:2], self.ws_chol, stream=s)  # Alg. 2
         mark(5)
@@ -68,9 +83,57 @@ class LayerPipeline:
                            self.zero, self.col_loss, None, self.ws_obs, stream=s)   # Alg. 2 sweep
         mark(6)
 
+    def _run_overlapped(self, X, G, W, sign_u, sign_v, caller) -> None:
+        """The same results on two streams. The Cholesky needs only H_X and leaves most SMs
+        idle during its diagonal steps, so H_G, S_G and U go to a low-priority stream that
+        runs beside it; the high-priority stream does H_X, S_X, V, the Cholesky and (once
+        both sides are done) the sweep. Events order the shared buffers."""
+        s, s2 = self.main, self.side
+        e_in, e_fx, e_tx, e_rin, e_side, e_out = self._ev
+        e_in.record(caller)
+        s.wait_event(e_in)
+        kq.kq_accum_factor(X, self.HX, trace=self.trace_x, info=self.info[0:1], stream=s)
+        e_fx.record(s)
+        kq.kq_compute_scales(W, self.HX, None, self.s_x, None, stream=s)
+        kq.kq_traces(self.HX, self.s_x, None, None, self.traces, stream=s)
+        e_tx.record(s)
+        with torch.cuda.stream(s):
+            self.Wp.copy_(W)
+        kq.kq_rotate_in(self.Wp, self.HX, self.s_x, sign_v, kq.KQ_FWD, stream=s)
+        e_rin.record(s)
+        kq.kq_chol_inv(self.HX, self.damp, self.Lt, self.info[1:2], self.ws_chol, stream=s)
+        s2.wait_event(e_fx)                      # the two factors would only split the SMs
+        kq.kq_accum_factor(G, self.HG, trace=self.trace_g, info=self.info[2:3], stream=s2)
+        kq.kq_compute_scales(W, None, self.HG, None, self.s_g, stream=s2)
+        s2.wait_event(e_tx)
+        kq.kq_traces(None, None, self.HG, self.s_g, self.traces, stream=s2)
+        s2.wait_event(e_rin)
+        kq.kq_rotate_out(self.Wp, self.HG, self.s_g, sign_u, kq.KQ_FWD, stream=s2)
+        e_side.record(s2)
+        s.wait_event(e_side)
+        kq.kq_obs_quantize(self.Wp, self.Lt, self.bits, self.group, self.block, self.codes, self.scale,
+                           self.zero, self.col_loss, None, self.ws_obs, stream=s)
+        e_out.record(s)
+        caller.wait_event(e_out)
+
+    def capture(self, X, G, W, sign_u, sign_v) -> tuple:
+        """Record one layer (both streams) as a CUDA graph on these fixed buffers. Returns
+        (graph, kernels per replay). Run run() once first so one-time set-up is done."""
+        from . import kronq as _kq
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        cap = torch.cuda.Stream(device=self.HX.device)
+        n0 = _kq.launch_count()
+        with torch.cuda.graph(g, stream=cap):
+            self.run(X, G, W, sign_u, sign_v, stream=cap)
+        return g, _kq.launch_count() - n0
+
     def check(self, stream=None) -> None:
         """Raise if a kernel reported a device-side error (timeout, non-PD pivot)."""
-        for k in range(2):
+        if self.side is not None:
+            self.side.synchronize()
+            self.main.synchronize()
+        for k in range(3):
             st, raw = kq.kq_check(self.info[k:k + 1], reset=True, stream=stream)
             if st != kq.KQ_OK:
                 raise kq.KronqError(st, "pipeline", f"device word {raw}")

@@ -287,3 +287,57 @@ def test_pipeline_proxy_loss(name, over):
     t = host(p.traces)
     assert abs(t[5] - o["s_post"]) <= 1e-5 * o["s_post"]
     assert abs(t[2] - o["s"]) <= 1e-5 * o["s"]
+
+
+def test_pipeline_overlap_matches_serial():
+    """The two-stream schedule runs the same kernels on the same buffers in a dependency-
+    respecting order, so every output must be bit-identical to the one-stream schedule."""
+    from paper_2607_07964_gb300.pipeline import STAGES, LayerPipeline
+    cfg = kqsynth.CONFIGS["tiny256"].replace(d_out=512, d_in=896, bits=3, group=128, T=4096, w_bf16=True)
+    L = kqsynth.layer(cfg)
+    X, G, W = bf16_dev(L["X"]), bf16_dev(L["G"]), dev(L["W"])
+    su, sv = dev(L["sign_u"], torch.int8), dev(L["sign_v"], torch.int8)
+    out = []
+    for overlap in (True, False):
+        p = LayerPipeline(cfg.d_out, cfg.d_in, cfg.bits, cfg.group, cfg.block, cfg.damp, overlap=overlap)
+        events = None if overlap else [torch.cuda.Event(enable_timing=True) for _ in range(len(STAGES) + 1)]
+        for _ in range(2):   # twice: buffers reused across layers
+            p.run(X, G, W, su, sv, events=events)
+        p.check()
+        out.append({k: host(getattr(p, k)) for k in ("codes", "scale", "zero", "Lt", "s_x", "s_g", "traces", "col_loss")})
+    for k in out[0]:
+        assert np.array_equal(out[0][k], out[1][k]), k
+
+
+@pytest.mark.parametrize("T,d", [(5000, 640), (130, 8), (0, 64)])
+def test_factor_diag(T, d):
+    """diag(A^T A) from one pass over A: the oracle's fp64 diagonal to fp32 accuracy (the
+    kernel sums 32-row chunks in fp32, exact products of bf16 values, then adds in fp64)."""
+    cfg = kqsynth.CONFIGS["tiny256"].replace(d_in=d, d_out=8, T=max(T, 1), n_outliers=min(4, d))
+    X = kqsynth.activations(cfg)[:T]
+    diag = torch.full((d,), float("nan"), device=DEV)
+    tr = torch.zeros(1, dtype=torch.float64, device=DEV)
+    ws = torch.empty(K().kq_factor_diag_workspace(T, d), dtype=torch.uint8, device=DEV)
+    Xd = bf16_dev(X) if T > 0 else torch.empty((0, d), dtype=torch.bfloat16, device=DEV)
+    K().kq_factor_diag(Xd, diag, trace=tr, ws=ws)
+    want = np.sum(X.astype(np.float64) ** 2, axis=0)
+    got = host(diag)
+    assert np.allclose(got, want.astype(np.float32), rtol=1e-6, atol=0)
+    assert abs(host(tr)[0] - want.sum()) <= 1e-6 * max(want.sum(), 1.0)
+
+
+def test_diag_variants_match_matrix_variants():
+    cfg = kqsynth.CONFIGS["tiny256"].replace(d_out=128, d_in=256, T=1024)
+    L, HX, HG = _layer64(cfg)
+    Wd, HXd, HGd = dev(L["W"]), dev(HX), dev(HG)
+    sx1, sg1 = torch.empty(256, device=DEV), torch.empty(128, device=DEV)
+    sx2, sg2 = torch.empty(256, device=DEV), torch.empty(128, device=DEV)
+    K().kq_compute_scales(Wd, HXd, HGd, sx1, sg1)
+    K().kq_compute_scales_diag(Wd, torch.diagonal(HXd).contiguous(), torch.diagonal(HGd).contiguous(), sx2, sg2)
+    assert torch.equal(sx1, sx2) and torch.equal(sg1, sg2)
+    t1 = torch.zeros(6, dtype=torch.float64, device=DEV)
+    t2 = torch.zeros(6, dtype=torch.float64, device=DEV)
+    K().kq_traces(HXd, sx1, HGd, sg1, t1)
+    K().kq_traces_diag(torch.diagonal(HXd).contiguous(), sx1, None, None, t2)
+    K().kq_traces_diag(None, None, torch.diagonal(HGd).contiguous(), sg1, t2)
+    assert torch.equal(t1, t2)
