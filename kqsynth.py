@@ -64,16 +64,23 @@ def _rng(seed: int, what: str) -> np.random.Generator:
 
 
 def round_bf16(a: np.ndarray) -> np.ndarray:
-    """Round float32 values to the nearest bf16 (ties to even); returns float32."""
+    """Round finite float32 values to the nearest bf16 (ties to even); returns float32."""
     a = np.ascontiguousarray(a, dtype=np.float32)
-    u = a.view(np.uint32).astype(np.uint64)
-    lsb = (u >> 16) & 1
-    u = (u + 0x7FFF + lsb) & 0xFFFF0000
-    out = u.astype(np.uint32).view(np.float32)
-    nan = np.isnan(a)
-    if nan.any():
-        out = out.copy()
-        out[nan] = np.nan
+    u = a.view(np.uint32).copy()
+    u += np.uint32(0x7FFF) + ((u >> np.uint32(16)) & np.uint32(1))
+    u &= np.uint32(0xFFFF0000)
+    return u.view(np.float32)
+
+
+def _scaled_normals(rng: np.random.Generator, T: int, d: int, scale: np.ndarray) -> np.ndarray:
+    """bf16-rounded N(0,1) * scale, drawn in row chunks (same stream as one draw)."""
+    out = np.empty((T, d), dtype=np.float32)
+    step = max(1, (1 << 24) // max(d, 1))
+    for t0 in range(0, T, step):
+        t1 = min(T, t0 + step)
+        z = rng.standard_normal((t1 - t0, d), dtype=np.float32)
+        z *= scale[None, :]
+        out[t0:t1] = round_bf16(z)
     return out
 
 
@@ -96,16 +103,14 @@ def activations(cfg: LayerConfig, T: int | None = None) -> np.ndarray:
     """X [T, d_in], bf16-representable float32, tokens as rows."""
     T = cfg.T if T is None else T
     sx, _ = channel_scales(cfg)
-    z = _rng(cfg.seed, "x").standard_normal((T, cfg.d_in), dtype=np.float32)
-    return round_bf16(z * sx[None, :])
+    return _scaled_normals(_rng(cfg.seed, "x"), T, cfg.d_in, sx)
 
 
 def gradients(cfg: LayerConfig, T: int | None = None) -> np.ndarray:
     """G [T, d_out], bf16-representable float32, tokens as rows."""
     T = cfg.T if T is None else T
     _, sg = channel_scales(cfg)
-    z = _rng(cfg.seed, "g").standard_normal((T, cfg.d_out), dtype=np.float32)
-    return round_bf16(z * sg[None, :])
+    return _scaled_normals(_rng(cfg.seed, "g"), T, cfg.d_out, sg)
 
 
 def weights(cfg: LayerConfig) -> np.ndarray:

@@ -30,7 +30,7 @@ from __future__ import annotations
 import numpy as np
 
 __all__ = [
-    "accum_factor", "sylvester", "paley28", "hadamard_matrix", "rht_matrix",
+    "accum_factor", "factor_entries", "factor_diag", "biip_scales_from_diag", "sylvester", "paley28", "hadamard_matrix", "rht_matrix",
     "biip_scales", "biip", "damp", "inverse_cholesky_upper", "lower_factor",
     "quant_params", "quantize", "obs_sweep", "dequant", "revert", "proxy_loss",
     "traces", "pipeline",
@@ -45,6 +45,32 @@ def accum_factor(A: np.ndarray) -> np.ndarray:
     """H = A^T A for A [T, d] with tokens as rows, in float64 (a library matmul)."""
     A = np.asarray(A, dtype=np.float64)
     return A.T @ A
+
+
+def factor_entries(A, pairs) -> np.ndarray:
+    """Selected entries H[i, j] = sum_t A[t, i] A[t, j] of the factor, each a float64 dot
+    product over all tokens (for checking very large factors entry by entry)."""
+    out = np.empty(len(pairs))
+    cache = {}
+
+    def col(j):
+        if j not in cache:
+            cache[j] = np.asarray(A[:, j], dtype=np.float64)
+        return cache[j]
+
+    for k, (i, j) in enumerate(pairs):
+        out[k] = float(np.dot(col(i), col(j)))
+    return out
+
+
+def factor_diag(A, chunk: int = 8192) -> np.ndarray:
+    """diag(A^T A) = per-channel sums of squares in float64, over row chunks."""
+    A = np.asarray(A)
+    acc = np.zeros(A.shape[1])
+    for t0 in range(0, A.shape[0], chunk):
+        blk = np.asarray(A[t0:t0 + chunk], dtype=np.float64)
+        acc += np.einsum("ij,ij->j", blk, blk)
+    return acc
 
 
 # ----------------------------------------------------------------------------------
@@ -123,6 +149,11 @@ def biip_scales(W: np.ndarray, HX: np.ndarray, HG: np.ndarray):
         sx = np.where((hx > 0) & (a > 0), (hx / a) ** 0.25, 1.0)
         sg = np.where((hg > 0) & (r > 0), (hg / r) ** 0.25, 1.0)
     return sx, sg
+
+
+def biip_scales_from_diag(W: np.ndarray, hx: np.ndarray, hg: np.ndarray):
+    """Eq. (rescale) from the factors' diagonals alone (all that the scales read)."""
+    return biip_scales(W, np.diag(np.asarray(hx, np.float64)), np.diag(np.asarray(hg, np.float64)))
 
 
 def biip(W, HX, HG, sign_u, sign_v):
