@@ -17,7 +17,8 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libkronq.so")
 SOURCES = ["kq_api.cu", "syrk.cu", "biip.cu", "chol.cu", "obs.cu", "check.cu"]
-HEADERS = [os.path.join(CSRC, "kq_common.cuh"), os.path.join(ROOT, "include", "kronq.h")]
+HEADERS = sorted(os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith(".cuh")) + [
+    os.path.join(ROOT, "include", "kronq.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
          "-I" + os.path.join(ROOT, "include")]

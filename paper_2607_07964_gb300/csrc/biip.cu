@@ -16,6 +16,7 @@
 #include <algorithm>
 
 #include "kq_common.cuh"
+#include "sumsq.cuh"
 
 namespace kq {
 namespace {
@@ -298,56 +299,21 @@ __device__ __forceinline__ float quarter_root_ratio(float h, double a) {
     return static_cast<float>(sqrt(sqrt(static_cast<double>(h) / a)));
 }
 
-// a_j = ||W[:, j]||^2 and s_x[j] = (H_X[j][j] / a_j)^(1/4). Block (32, 8).
+// a_j = ||W[:, j]||^2 and s_x[j] = (H_X[j][j] / a_j)^(1/4). Block (CS_X, CS_Y).
 __global__ void colscale_kernel(const float* __restrict__ W, int64_t d_out, int64_t d_in,
                                 const float* __restrict__ HX, int64_t hstride, float* __restrict__ s_x) {
-    __shared__ double part[8][33];
-    const int64_t j = static_cast<int64_t>(blockIdx.x) * 32 + threadIdx.x;
-    double acc = 0.0;
-    if (j < d_in) {
-        float p = 0.0f;
-        int cnt = 0;
-        for (int64_t r = threadIdx.y; r < d_out; r += 8) {
-            const float w = W[r * d_in + j];
-            p = fmaf(w, w, p);
-            if (++cnt == 32) {
-                acc += p;
-                p = 0.0f;
-                cnt = 0;
-            }
-        }
-        acc += p;
-    }
-    part[threadIdx.y][threadIdx.x] = acc;
-    __syncthreads();
-    if (threadIdx.y == 0 && j < d_in) {
-        double a = 0.0;
-        for (int y = 0; y < 8; ++y) a += part[y][threadIdx.x];
-        s_x[j] = quarter_root_ratio(HX[j * hstride], a);
-    }
+    const int64_t j = static_cast<int64_t>(blockIdx.x) * CS_X + threadIdx.x;
+    const double a = col_sumsq(W, d_out, d_in, j);
+    if (threadIdx.y == 0 && j < d_in) s_x[j] = quarter_root_ratio(HX[j * hstride], a);
 }
 
 // r_i = ||W[i, :]||^2 and s_g[i] = (H_G[i][i] / r_i)^(1/4) (1 when H_G is NULL). Warp per row.
 __global__ void rowscale_kernel(const float* __restrict__ W, int64_t d_out, int64_t d_in,
                                 const float* __restrict__ HG, int64_t hstride, float* __restrict__ s_g) {
     const int64_t i = static_cast<int64_t>(blockIdx.x) * (blockDim.x / 32) + threadIdx.x / 32;
-    const int lane = threadIdx.x & 31;
     if (i >= d_out) return;
-    double acc = 0.0;
-    float p = 0.0f;
-    int cnt = 0;
-    for (int64_t j = lane; j < d_in; j += 32) {
-        const float w = W[i * d_in + j];
-        p = fmaf(w, w, p);
-        if (++cnt == 32) {
-            acc += p;
-            p = 0.0f;
-            cnt = 0;
-        }
-    }
-    acc += p;
-    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if (lane == 0) s_g[i] = HG ? quarter_root_ratio(HG[i * hstride], acc) : 1.0f;
+    const double acc = row_sumsq(W + i * d_in, d_in);
+    if ((threadIdx.x & 31) == 0) s_g[i] = HG ? quarter_root_ratio(HG[i * hstride], acc) : 1.0f;
 }
 
 // out = [tr H_X, tr H_G, product, tr H_X', tr H_G', product'] with tr H' = sum h_j / s_j^2.
@@ -602,7 +568,7 @@ kq_status scales_impl(const float* W, int64_t d_out, int64_t d_in, const float* 
         return KQ_ERR_INVALID_ARG;
     }
     if (s_x) {
-        colscale_kernel<<<static_cast<unsigned>(cdiv(d_in, 32)), dim3(32, 8), 0, stream>>>(W, d_out, d_in, hx, xs, s_x);
+        colscale_kernel<<<static_cast<unsigned>(cdiv(d_in, CS_X)), dim3(CS_X, CS_Y), 0, stream>>>(W, d_out, d_in, hx, xs, s_x);
         KQ_LAUNCH_CHECK("colscale_kernel");
     }
     if (s_g) {

@@ -13,6 +13,10 @@
 //           update-- A_ij -= C_ik C_jk^T (k < j <= i) and B_ij -= C_ik Z_kj (j <= k < i),
 // where B (stored in Z's blocks) is the right-hand side I of C Z = I after the earlier
 // steps' eliminations. The matrix is padded to a multiple of nb with an identity block.
+// Look-ahead: the update is split into the tiles step k + 1 reads first (row and column
+// block k + 1, on the caller's stream, on the critical path) and the rest (on a library
+// side stream, beside step k + 1's diagonal factorization and panel); step k + 1's own
+// first tiles wait for that rest, which also writes them.
 // All arithmetic is fp32 with fused multiply-add.
 #include <math.h>
 
@@ -362,17 +366,9 @@ __device__ __forceinline__ void sub_tile(float* out, int64_t ld, const float (&a
 }
 
 // -------------------------------------------------------------------- update
-// Tiles (i, j), k < i < nbk, 0 <= j <= i:
+// Tile (i, j) of step k, k < i < nbk, 0 <= j <= i:
 //   j > k : A_ij -= C_ik C_jk^T;     j <= k : Z_ij -= C_ik Z_kj.
-__global__ void __launch_bounds__(G_THREADS, 2) chol_update_kernel(Work w, int64_t npad, int k) {
-    extern __shared__ __align__(16) float sm[];
-    int bid = blockIdx.x;
-    int i = k + 1;
-    while (bid >= i + 1) {
-        bid -= i + 1;
-        ++i;
-    }
-    const int j = bid;
+__device__ __forceinline__ void update_tile(const Work& w, int64_t npad, int k, int i, int j, float* sm) {
     const int64_t ko = static_cast<int64_t>(k) * NB;
     const float* cik = w.A + static_cast<int64_t>(i) * NB * npad + ko;
     const bool apart = j > k;
@@ -386,6 +382,29 @@ __global__ void __launch_bounds__(G_THREADS, 2) chol_update_kernel(Work w, int64
         sub_tile<false>(out, npad, acc);
     else
         sub_tile<true>(out, npad, acc);
+}
+
+// The tiles that step k + 1 reads first: row block k + 1 (tiles (k + 1, j), j <= k + 1)
+// and block column k + 1 below it (tiles (i, k + 1), i > k + 1). nbk CTAs.
+__global__ void __launch_bounds__(G_THREADS, 2) chol_next_kernel(Work w, int64_t npad, int k) {
+    extern __shared__ __align__(16) float sm[];
+    const int bid = blockIdx.x;
+    if (bid < k + 2)
+        update_tile(w, npad, k, k + 1, bid, sm);
+    else
+        update_tile(w, npad, k, bid, k + 1, sm);
+}
+
+// The other tiles of step k: (i, j) with i > k + 1 and j != k + 1 (i tiles in row block i).
+__global__ void __launch_bounds__(G_THREADS, 2) chol_rest_kernel(Work w, int64_t npad, int k) {
+    extern __shared__ __align__(16) float sm[];
+    int bid = blockIdx.x;
+    int i = k + 2;
+    while (bid >= i) {
+        bid -= i;
+        ++i;
+    }
+    update_tile(w, npad, k, i, bid < k + 1 ? bid : bid + 1, sm);
 }
 
 // -------------------------------------------------------------------- finish
@@ -443,7 +462,9 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
                                      static_cast<int>(DIAG_SMEM)));
         KQ_CUDA(cudaFuncSetAttribute(chol_panel_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(G_SMEM)));
-        KQ_CUDA(cudaFuncSetAttribute(chol_update_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        KQ_CUDA(cudaFuncSetAttribute(chol_next_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     static_cast<int>(G_SMEM)));
+        KQ_CUDA(cudaFuncSetAttribute(chol_rest_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(G_SMEM)));
         attr = true;
     }
@@ -453,6 +474,8 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
     const int64_t pgrid = std::min<int64_t>(cdiv(total, 256), static_cast<int64_t>(num_sms()) * 32);
     prep_kernel<<<static_cast<unsigned>(pgrid), 256, 0, stream>>>(H, n, npad, damp_rel, w.dsum, w.A, w.Z);
     KQ_LAUNCH_CHECK("prep_kernel");
+    SideStream* side = nbk > 2 ? side_stream(stream) : nullptr;
+    bool forked = false;
     for (int k = 0; k < nbk; ++k) {
         chol_diag_kernel<<<1, DIAG_THREADS, DIAG_SMEM, stream>>>(w, n, npad, k, info);
         KQ_LAUNCH_CHECK("chol_diag_kernel");
@@ -460,13 +483,29 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
             chol_panel_kernel<<<nbk - 1, G_THREADS, G_SMEM, stream>>>(w, npad, k);
             KQ_LAUNCH_CHECK("chol_panel_kernel");
         }
-        int64_t tiles = 0;
-        for (int i = k + 1; i < nbk; ++i) tiles += i + 1;
-        if (tiles > 0) {
-            chol_update_kernel<<<static_cast<unsigned>(tiles), G_THREADS, G_SMEM, stream>>>(w, npad, k);
-            KQ_LAUNCH_CHECK("chol_update_kernel");
+        if (k + 1 >= nbk) break;
+        int64_t rest = 0;
+        for (int i = k + 2; i < nbk; ++i) rest += i;
+        const bool fork = side && rest > 0;
+        if (fork) KQ_CUDA(cudaEventRecord(side->ev[0], stream));      // panel k done
+        if (forked) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));  // rest of step k - 1 done
+        chol_next_kernel<<<nbk, G_THREADS, G_SMEM, stream>>>(w, npad, k);
+        KQ_LAUNCH_CHECK("chol_next_kernel");
+        if (rest > 0) {
+            cudaStream_t rs = stream;
+            if (fork) {
+                KQ_CUDA(cudaStreamWaitEvent(side->s, side->ev[0], 0));
+                rs = side->s;
+            }
+            chol_rest_kernel<<<static_cast<unsigned>(rest), G_THREADS, G_SMEM, rs>>>(w, npad, k);
+            KQ_LAUNCH_CHECK("chol_rest_kernel");
+            if (fork) {
+                KQ_CUDA(cudaEventRecord(side->ev[1], side->s));
+                forked = true;
+            }
         }
     }
+    if (forked) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));
     finish_kernel<<<dim3(static_cast<unsigned>(cdiv(n, 32)), static_cast<unsigned>(cdiv(n, 32))),
                     dim3(32, 8), 0, stream>>>(w.Z, n, npad, Lt);
     KQ_LAUNCH_CHECK("finish_kernel");

@@ -39,6 +39,39 @@ int num_sms() {
     return cache[dev];
 }
 
+SideStream* side_stream(cudaStream_t caller) {
+    static thread_local SideStream cache[64][8] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    int prio = 0, least = 0, greatest = 0;
+    if (cudaStreamGetPriority(caller, &prio) != cudaSuccess ||
+        cudaDeviceGetStreamPriorityRange(&least, &greatest) != cudaSuccess) {
+        cudaGetLastError();
+        return nullptr;
+    }
+    // Larger numbers are lower priorities.
+    const int side_prio = prio < least ? prio + 1 : least;
+    const int idx = side_prio - greatest;
+    if (idx < 0 || idx >= 8) return nullptr;
+    SideStream& c = cache[dev][idx];
+    if (!c.tried) {
+        cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+        if (cudaStreamIsCapturing(caller, &cap) != cudaSuccess) {
+            cudaGetLastError();
+            return nullptr;
+        }
+        if (cap != cudaStreamCaptureStatusNone) return nullptr;
+        c.tried = true;
+        if (cudaStreamCreateWithPriority(&c.s, cudaStreamNonBlocking, side_prio) != cudaSuccess ||
+            cudaEventCreateWithFlags(&c.ev[0], cudaEventDisableTiming) != cudaSuccess ||
+            cudaEventCreateWithFlags(&c.ev[1], cudaEventDisableTiming) != cudaSuccess) {
+            cudaGetLastError();
+            c.s = nullptr;
+        }
+    }
+    return c.s ? &c : nullptr;
+}
+
 }  // namespace kq
 
 extern "C" const char* kq_last_error(void) { return kq::g_err; }

@@ -34,6 +34,21 @@ inline int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
 // Number of SMs of the current device (cached per device).
 int num_sms();
 
+// A library-owned stream for work that can run beside the caller's stream. An entry point
+// forks to it with an event recorded on the caller's stream and joins back (the caller's
+// stream waits on an event recorded on it) before returning, so the caller sees one
+// ordered stream, and a CUDA graph captured from the caller's stream records both
+// branches. One per host thread, device and priority; its priority is one level below the
+// caller's stream. side_stream returns nullptr (the caller then runs everything on its own
+// stream) when the stream cannot be made, or when the caller's stream is being captured
+// and the side stream does not exist yet.
+struct SideStream {
+    cudaStream_t s;
+    cudaEvent_t ev[2];
+    bool tried;
+};
+SideStream* side_stream(cudaStream_t caller);
+
 // ------------------------------------------------------------------------- device side
 // Device error words: info == 0 ok; > 0 a 1-based pivot index (Cholesky); < 0 minus a
 // kq_status recorded by a kernel (for example -KQ_ERR_TIMEOUT).

@@ -13,20 +13,20 @@
 //   trailing  acc = fma(E_k, R_kc, acc) over ascending k; w_c = w_c - acc
 // Kernels:
 //   rowgrid_kernel   per-row grid (group = 0) from the whole row before the sweep
-//   obs_block_kernel four rows per warp; the block's R (128 x 128) in shared memory
+//   pack_r_kernel    the diagonal 128 x 128 blocks of R in the block kernel's layout
+//   obs_block_kernel 8 lanes per row, 16 columns per lane; the block's R in shared memory
 //   trailing_kernel  128 x 128 output tiles of the shared tile GEMM (tile_gemm.cuh)
-//   colloss_kernel   col_loss[j] = sum over rows of E_j^2, fixed order, fp64
+//   colloss_kernel   col_loss[j] = sum over rows of E_j^2, fixed order (sumsq.cuh)
 #include <math.h>
 
 #include "kq_common.cuh"
 #include "tile_gemm.cuh"
+#include "sumsq.cuh"
 
 namespace kq {
 namespace {
 
 constexpr int BLK = 128;          // block size B (Algorithm 2); the only supported value
-constexpr int RTLD = BLK + 4;     // row stride of the staged L block (16-byte rows)
-constexpr int kRowsPerLane = 1;   // rows per lane group in the block kernel
 
 struct Grid {
     float scale, zero;
@@ -78,16 +78,46 @@ __global__ void rowgrid_kernel(const float* __restrict__ W, int64_t d_out, int64
     }
 }
 
-// One block [i0, e) of the sweep for all rows. A group of LPR = 4 lanes handles RPL rows;
-// lane position lp holds columns i0 + 4 t + lp (t = 0..31) of each of its rows in registers.
-// Per column j the owner lane broadcasts w_j inside its group; every lane of the group
-// computes the (identical) quantization, then updates its own later columns. The RPL rows
-// of a lane share the loads of R and give independent instruction chains.
+// One block [i0, e) of the sweep for all rows. A group of LPR = 8 lanes handles one row;
+// lane position lp holds the CPL = 16 consecutive columns i0 + CPL lp + t of it in
+// registers. Column j = CPL o + jj is owned by lane o: for each o (rolled loop) the 16
+// columns are an unrolled loop, so every register index is a compile-time constant. Per
+// column the owner's w_j is broadcast in the group, every lane computes the (identical)
+// quantization and error, and every lane updates all CPL of its registers with R_jk. The
+// updates of columns k < j (lanes before the owner, or the owner's own earlier columns)
+// read R_jk = 0 or hit values that are no longer read, so no update needs a predicate and
+// the live columns k > j see exactly the operations of the definition.
 #ifndef KQ_OBS_LANES_PER_ROW
 #define KQ_OBS_LANES_PER_ROW 8
 #endif
-constexpr int LPR = KQ_OBS_LANES_PER_ROW;   // lanes per row group (4 or 8)
-constexpr int CPL = BLK / LPR;         // columns per lane
+constexpr int LPR = KQ_OBS_LANES_PER_ROW;   // lanes per row (8 or 16)
+constexpr int CPL = BLK / LPR;              // columns per lane
+constexpr int NV = CPL / 4;                 // float4 slots per lane
+static_assert(LPR == 8 || LPR == 16, "lanes per row must be 8 or 16");
+
+// Packed layout of one diagonal block of R: row j holds R[i0 + j][i0 + c] at pos(c). The
+// CPL columns of lane lp fill slots [lp NV, lp NV + NV) of 16 bytes, rotated by lane so
+// that the NV float4 loads of 8 consecutive lanes hit 8 distinct bank groups.
+__host__ __device__ constexpr int slot_of(int lp, int v) { return lp * NV + ((v + ((lp * NV) >> 3)) & (NV - 1)); }
+__device__ __forceinline__ int pos_of(int c) { return 4 * slot_of(c / CPL, (c % CPL) >> 2) + (c & 3); }
+
+// Rp[b][j][pos(c)] = R[i0 + j][i0 + c] = Lt[i0 + c][i0 + j] (0 outside the matrix),
+// i0 = b BLK. Block (32, 8) transposes one 32 x 32 tile through shared memory.
+__global__ void pack_r_kernel(const float* __restrict__ Lt, int64_t n, float* __restrict__ Rp) {
+    __shared__ float t[32][33];
+    const int64_t i0 = static_cast<int64_t>(blockIdx.z) * BLK;
+    const int c0 = blockIdx.y * 32, j0 = blockIdx.x * 32;
+    for (int r = threadIdx.y; r < 32; r += 8) {
+        const int64_t c = i0 + c0 + r, j = i0 + j0 + threadIdx.x;
+        t[r][threadIdx.x] = (c < n && j < n) ? Lt[c * n + j] : 0.0f;
+    }
+    __syncthreads();
+    float* out = Rp + static_cast<int64_t>(blockIdx.z) * BLK * BLK;
+    for (int r = threadIdx.y; r < 32; r += 8) {
+        const int j = j0 + r, c = c0 + threadIdx.x;
+        out[j * BLK + pos_of(c)] = t[threadIdx.x][r];
+    }
+}
 
 __device__ __forceinline__ float group_min(float v) {
     for (int o = LPR / 2; o > 0; o >>= 1) v = fminf(v, __shfl_xor_sync(0xffffffffu, v, o));
@@ -98,128 +128,131 @@ __device__ __forceinline__ float group_max(float v) {
     return v;
 }
 
-template <int RPL>
+// A lane's CPL columns [cb, cb + CPL) of row r of the block starting at column i0 (0 past
+// the block end nb or past the last row).
+template <bool VEC>
+__device__ __forceinline__ void load_cols(const float* __restrict__ W, int64_t r, int64_t d_out, int64_t d_in,
+                                          int64_t i0, int cb, int nb, float (&w)[CPL]) {
+    const bool live = r < d_out;
+    const float* src = W + r * d_in + i0 + cb;
+    if (VEC && cb + CPL <= nb) {
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+            const float4 x = live ? __ldg(reinterpret_cast<const float4*>(src) + v) : make_float4(0.f, 0.f, 0.f, 0.f);
+            w[4 * v] = x.x;
+            w[4 * v + 1] = x.y;
+            w[4 * v + 2] = x.z;
+            w[4 * v + 3] = x.w;
+        }
+    } else {
+#pragma unroll
+        for (int t = 0; t < CPL; ++t) w[t] = (live && cb + t < nb) ? src[t] : 0.0f;
+    }
+}
+
+// VEC: d_in % 16 == 0 and W, codes (and pre_q) 16-byte aligned, so a lane's CPL columns
+// of W, E and codes move as 16-byte vectors.
+template <bool VEC>
 __global__ void __launch_bounds__(128, 3) obs_block_kernel(
-    const float* __restrict__ W, int64_t d_out, int64_t d_in, const float* __restrict__ Lt, int64_t i0,
+    const float* __restrict__ W, int64_t d_out, int64_t d_in, const float* __restrict__ Rp, int64_t i0,
     int bits, int group, const float* __restrict__ gscale, const float* __restrict__ gzero,
     uint8_t* __restrict__ codes, float* __restrict__ scale, int32_t* __restrict__ zero,
-    float* __restrict__ E, float* __restrict__ pre_q, bool vec) {
-    // The block of L = R^T in its own layout: Rt[k][j] = Lt[i0 + k][i0 + j] = R[i0 + j][i0 + k],
-    // staged with 16-byte cp.async copies (scalar loads when rows are not 16-byte aligned).
-    extern __shared__ __align__(16) float Rt[];   // [BLK][RTLD]
+    float* __restrict__ E, float* __restrict__ pre_q) {
+    extern __shared__ __align__(16) float Rs[];   // [BLK][BLK], packed (pack_r_kernel)
+    for (int e = threadIdx.x; e < BLK * BLK / 4; e += blockDim.x) cp_async16(Rs + 4 * e, Rp + 4 * e, 16);
+    cp_async_commit();
     const int nb = static_cast<int>(min(static_cast<int64_t>(BLK), d_in - i0));
-    if (vec) {
-        for (int e = threadIdx.x; e < BLK * (BLK / 4); e += blockDim.x) {
-            const int k = e >> 5, j4 = (e & 31) * 4;
-            const int valid = k < nb ? max(0, min(4, nb - j4)) : 0;
-            cp_async16(Rt + k * RTLD + j4,
-                       valid ? static_cast<const void*>(Lt + (i0 + k) * d_in + i0 + j4) : static_cast<const void*>(Lt),
-                       4 * valid);
-        }
-        cp_async_commit();
-        cp_async_wait<0>();
-    } else {
-        for (int e = threadIdx.x; e < BLK * BLK; e += blockDim.x) {
-            const int k = e / BLK, j = e % BLK;
-            Rt[k * RTLD + j] = (j < nb && k < nb) ? Lt[(i0 + k) * d_in + i0 + j] : 0.0f;
-        }
-    }
-    __syncthreads();
     const float maxq = static_cast<float>((1 << bits) - 1);
     const int lane = threadIdx.x & 31;
     const int lp = lane & (LPR - 1);
     const int gbase = lane & ~(LPR - 1);
+    const int cb = CPL * lp;                       // first column of this lane in the block
     const int64_t ngroups = group ? (d_in + group - 1) / group : 1;
     const int warps = blockDim.x / 32;
-    constexpr int RPW = (32 / LPR) * RPL;   // rows per warp
-    for (int64_t rw = (static_cast<int64_t>(blockIdx.x) * warps + threadIdx.x / 32) * RPW; rw < d_out;
-         rw += static_cast<int64_t>(gridDim.x) * warps * RPW) {
-        int64_t r[RPL];
-        bool live[RPL];
-        float w[RPL][CPL];
-        Grid g[RPL];
+    constexpr int RPW = 32 / LPR;                  // rows per warp
+    const int64_t rstride = static_cast<int64_t>(gridDim.x) * warps * RPW;
+    const int64_t rw0 = (static_cast<int64_t>(blockIdx.x) * warps + threadIdx.x / 32) * RPW;
+    float w[CPL];
+    // The first row's weights load while R is staged; every thread reaches the barrier.
+    load_cols<VEC>(W, rw0 + lane / LPR, d_out, d_in, i0, cb, nb, w);
+    cp_async_wait<0>();
+    __syncthreads();
+    for (int64_t rw = rw0; rw < d_out; rw += rstride) {
+        const int64_t r = rw + lane / LPR;
+        const bool live = r < d_out;
+        if (rw != rw0) load_cols<VEC>(W, r, d_out, d_in, i0, cb, nb, w);
+        Grid g;
+        if (group) {
+            float mn = 0.0f, mx = 0.0f;
 #pragma unroll
-        for (int u = 0; u < RPL; ++u) {
-            r[u] = rw + (lane / LPR) * RPL + u;
-            live[u] = r[u] < d_out;
-            const float* wr = W + r[u] * d_in + i0;
-#pragma unroll
-            for (int t = 0; t < CPL; ++t) {
-                const int c = LPR * t + lp;
-                w[u][t] = (live[u] && c < nb) ? wr[c] : 0.0f;
-            }
-            if (group) {
-                float mn = 0.0f, mx = 0.0f;
-#pragma unroll
-                for (int t = 0; t < CPL; ++t)
-                    if (LPR * t + lp < nb) {
-                        mn = fminf(mn, w[u][t]);
-                        mx = fmaxf(mx, w[u][t]);
-                    }
-                g[u] = make_grid(group_min(mn), group_max(mx), maxq);
-                if (live[u] && lp == 0) {
-                    const int64_t gi = r[u] * ngroups + i0 / group;
-                    scale[gi] = g[u].scale;
-                    zero[gi] = static_cast<int32_t>(g[u].zero);
+            for (int t = 0; t < CPL; ++t)
+                if (cb + t < nb) {
+                    mn = fminf(mn, w[t]);
+                    mx = fmaxf(mx, w[t]);
                 }
-            } else {
-                g[u].scale = live[u] ? gscale[r[u]] : 1.0f;
-                g[u].zero = live[u] ? gzero[r[u]] : 0.0f;
+            g = make_grid(group_min(mn), group_max(mx), maxq);
+            if (live && lp == 0) {
+                const int64_t gi = r * ngroups + i0 / group;
+                scale[gi] = g.scale;
+                zero[gi] = static_cast<int32_t>(g.zero);
             }
+        } else {
+            g.scale = live ? gscale[r] : 1.0f;
+            g.zero = live ? gzero[r] : 0.0f;
         }
-        // Slot q of the block is always w[.][0]: after its 8 columns the registers shift
-        // down by one, which keeps the loop rolled (compact code) with register indexing.
 #pragma unroll 1
-        for (int q = 0; q < CPL; ++q) {
-            float e_cur[RPL], pq_cur[RPL];
-            uint32_t q_cur[RPL];
+        for (int o = 0; o < LPR; ++o) {
+            if (CPL * o >= nb) break;   // uniform across the CTA
+            float e[CPL];
+            uint32_t cq[NV];
 #pragma unroll
-            for (int u = 0; u < RPL; ++u) {
-                e_cur[u] = 0.0f;
-                pq_cur[u] = 0.0f;
-                q_cur[u] = 0;
-            }
+            for (int v = 0; v < NV; ++v) cq[v] = 0u;
 #pragma unroll
-            for (int jl = 0; jl < LPR; ++jl) {
-                const int j = LPR * q + jl;
-                if (j < nb) {   // uniform across the warp
-                    const float dj = Rt[j * RTLD + j];
-                    float err[RPL];
+            for (int jj = 0; jj < CPL; ++jj) {
+                const int j = CPL * o + jj;
+                e[jj] = 0.0f;
+                if (j < nb) {   // uniform across the CTA
+                    const float* rr = Rs + j * BLK;
+                    const float dj = rr[4 * slot_of(o, jj >> 2) + (jj & 3)];
+                    float4 rv[NV];
 #pragma unroll
-                    for (int u = 0; u < RPL; ++u) {
-                        const float wj = __shfl_sync(0xffffffffu, w[u][0], gbase | jl);
-                        float qq = __fadd_rn(rintf(__fdiv_rn(wj, g[u].scale)), g[u].zero);
-                        qq = fminf(fmaxf(qq, 0.0f), maxq);
-                        const float what = __fmul_rn(g[u].scale, __fsub_rn(qq, g[u].zero));
-                        err[u] = __fdiv_rn(__fsub_rn(wj, what), dj);
-                        if (lp == jl) {
-                            e_cur[u] = err[u];
-                            q_cur[u] = static_cast<uint32_t>(qq);
-                            pq_cur[u] = wj;
-                        }
-                    }
-                    const float* rcol = Rt + (LPR * q + lp) * RTLD + j;   // R[j][k] = Rt[k][j]
+                    for (int v = 0; v < NV; ++v) rv[v] = *reinterpret_cast<const float4*>(rr + 4 * slot_of(lp, v));
+                    const float wj = __shfl_sync(0xffffffffu, w[jj], gbase | o);
+                    float qq = __fadd_rn(rintf(__fdiv_rn(wj, g.scale)), g.zero);
+                    qq = fminf(fmaxf(qq, 0.0f), maxq);
+                    const float what = __fmul_rn(g.scale, __fsub_rn(qq, g.zero));
+                    const float err = __fdiv_rn(__fsub_rn(wj, what), dj);
+                    e[jj] = err;
+                    cq[jj >> 2] |= static_cast<uint32_t>(qq) << (8 * (jj & 3));
+                    if (pre_q && live && lp == o) pre_q[r * d_in + i0 + j] = wj;
 #pragma unroll
-                    for (int t = 0; t < CPL; ++t) {
-                        if (t < CPL - q && LPR * (q + t) + lp > j) {
-                            const float rv = rcol[LPR * t * RTLD];
-#pragma unroll
-                            for (int u = 0; u < RPL; ++u) w[u][t] = __fmaf_rn(-err[u], rv, w[u][t]);
-                        }
+                    for (int v = 0; v < NV; ++v) {
+                        w[4 * v] = __fmaf_rn(-err, rv[v].x, w[4 * v]);
+                        w[4 * v + 1] = __fmaf_rn(-err, rv[v].y, w[4 * v + 1]);
+                        w[4 * v + 2] = __fmaf_rn(-err, rv[v].z, w[4 * v + 2]);
+                        w[4 * v + 3] = __fmaf_rn(-err, rv[v].w, w[4 * v + 3]);
                     }
                 }
             }
-            const int c = LPR * q + lp;
+            if (live && lp == o) {
+                const int64_t ob = r * d_in + i0 + CPL * o;
+                if (VEC && CPL * o + CPL <= nb) {
 #pragma unroll
-            for (int u = 0; u < RPL; ++u) {
-                if (live[u] && c < nb) {
-                    codes[r[u] * d_in + i0 + c] = static_cast<uint8_t>(q_cur[u]);
-                    E[r[u] * d_in + i0 + c] = e_cur[u];
-                    if (pre_q) pre_q[r[u] * d_in + i0 + c] = pq_cur[u];
+                    for (int v = 0; v < NV; ++v)
+                        reinterpret_cast<float4*>(E + ob)[v] = make_float4(e[4 * v], e[4 * v + 1], e[4 * v + 2], e[4 * v + 3]);
+                    if constexpr (NV == 4) {
+                        *reinterpret_cast<uint4*>(codes + ob) = make_uint4(cq[0], cq[1], cq[2], cq[3]);
+                    } else {
+                        *reinterpret_cast<uint2*>(codes + ob) = make_uint2(cq[0], cq[1]);
+                    }
+                } else {
+#pragma unroll
+                    for (int t = 0; t < CPL; ++t)
+                        if (CPL * o + t < nb) {
+                            E[ob + t] = e[t];
+                            codes[ob + t] = static_cast<uint8_t>(cq[t >> 2] >> (8 * (t & 3)));
+                        }
                 }
-#pragma unroll
-                for (int t = 0; t + 1 < CPL; ++t) w[u][t] = w[u][t + 1];
-                w[u][CPL - 1] = 0.0f;
             }
         }
     }
@@ -262,45 +295,26 @@ __global__ void __launch_bounds__(G_THREADS, 2) trailing_kernel(float* __restric
     }
 }
 
-// col_loss[j] = sum over rows of E[r][j]^2: fp32 partials over 32 rows, fp64 across them,
-// fixed order. Block (32, 8): 32 columns, 8 row lanes.
+// col_loss[j] = sum over rows of E[r][j]^2 in a fixed order (fp32 runs, fp64 across them).
+// Block (CS_X, CS_Y).
 __global__ void colloss_kernel(const float* __restrict__ E, int64_t d_out, int64_t d_in,
                                float* __restrict__ col_loss) {
-    __shared__ double part[8][33];
-    const int64_t j = static_cast<int64_t>(blockIdx.x) * 32 + threadIdx.x;
-    double acc = 0.0;
-    if (j < d_in) {
-        float p = 0.0f;
-        int cnt = 0;
-        for (int64_t r = threadIdx.y; r < d_out; r += 8) {
-            const float v = E[r * d_in + j];
-            p = fmaf(v, v, p);
-            if (++cnt == 32) {
-                acc += p;
-                p = 0.0f;
-                cnt = 0;
-            }
-        }
-        acc += p;
-    }
-    part[threadIdx.y][threadIdx.x] = acc;
-    __syncthreads();
-    if (threadIdx.y == 0 && j < d_in) {
-        double a = 0.0;
-        for (int y = 0; y < 8; ++y) a += part[y][threadIdx.x];
-        col_loss[j] = static_cast<float>(a);
-    }
+    const int64_t j = static_cast<int64_t>(blockIdx.x) * CS_X + threadIdx.x;
+    const double a = col_sumsq(E, d_out, d_in, j);
+    if (threadIdx.y == 0 && j < d_in) col_loss[j] = static_cast<float>(a);
 }
 
 struct ObsWs {
-    float* E;
-    float* gscale;
-    float* gzero;
+    float* Rp;      // packed diagonal blocks of R, nblk x BLK x BLK
+    float* E;       // d_out x d_in
+    float* gscale;  // d_out
+    float* gzero;   // d_out
 };
 
 ObsWs carve(void* ws, int64_t d_out, int64_t d_in) {
     ObsWs o;
-    o.E = static_cast<float*>(ws);
+    o.Rp = static_cast<float*>(ws);
+    o.E = o.Rp + cdiv(d_in, BLK) * BLK * BLK;
     o.gscale = o.E + d_out * d_in;
     o.gzero = o.gscale + d_out;
     return o;
@@ -314,7 +328,8 @@ using namespace kq;
 extern "C" size_t kq_obs_quantize_workspace(int64_t d_out, int64_t d_in, int block) {
     (void)block;
     if (d_out < 1 || d_in < 1) return 0;
-    return static_cast<size_t>(d_out) * d_in * sizeof(float) + 2 * static_cast<size_t>(d_out) * sizeof(float) + 256;
+    return (static_cast<size_t>(cdiv(d_in, BLK)) * BLK * BLK + static_cast<size_t>(d_out) * d_in +
+            2 * static_cast<size_t>(d_out)) * sizeof(float) + 256;
 }
 
 extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, const float* Lt, int bits,
@@ -338,8 +353,10 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
     }
     static bool attr = false;
     if (!attr) {
-        KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel<kRowsPerLane>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     BLK * RTLD * 4));
+        KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     BLK * BLK * 4));
+        KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     BLK * BLK * 4));
         KQ_CUDA(cudaFuncSetAttribute(trailing_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(G_SMEM)));
         KQ_CUDA(cudaFuncSetAttribute(trailing_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -352,13 +369,23 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
                                                                                 zero, o.gscale, o.gzero);
         KQ_LAUNCH_CHECK("rowgrid_kernel");
     }
+    const int64_t nblk = cdiv(d_in, BLK);
+    pack_r_kernel<<<dim3(BLK / 32, BLK / 32, static_cast<unsigned>(nblk)), dim3(32, 8), 0, stream>>>(Lt, d_in, o.Rp);
+    KQ_LAUNCH_CHECK("pack_r_kernel");
     const bool vec = (d_in % 4 == 0) && (reinterpret_cast<uintptr_t>(Lt) % 16 == 0);
-    const int64_t rows_per_cta = 4 * (32 / LPR) * kRowsPerLane;   // 4 warps per CTA
+    const bool bvec = (d_in % 16 == 0) && (reinterpret_cast<uintptr_t>(W) % 16 == 0) &&
+                      (reinterpret_cast<uintptr_t>(codes) % 16 == 0);
+    const int64_t rows_per_cta = 4 * (32 / LPR);   // 4 warps per CTA
     const int64_t row_ctas = std::min<int64_t>(cdiv(d_out, rows_per_cta), static_cast<int64_t>(num_sms()) * 3);
     for (int64_t i0 = 0; i0 < d_in; i0 += BLK) {
         const int kb = static_cast<int>(std::min<int64_t>(BLK, d_in - i0));
-        obs_block_kernel<kRowsPerLane><<<static_cast<unsigned>(row_ctas), 128, BLK * RTLD * 4, stream>>>(
-            W, d_out, d_in, Lt, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q, vec);
+        const float* rp = o.Rp + (i0 / BLK) * BLK * BLK;
+        if (bvec)
+            obs_block_kernel<true><<<static_cast<unsigned>(row_ctas), 128, BLK * BLK * 4, stream>>>(
+                W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q);
+        else
+            obs_block_kernel<false><<<static_cast<unsigned>(row_ctas), 128, BLK * BLK * 4, stream>>>(
+                W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q);
         KQ_LAUNCH_CHECK("obs_block_kernel");
         const int64_t rest = d_in - (i0 + kb);
         if (rest > 0) {
@@ -371,7 +398,7 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
         }
     }
     if (col_loss) {
-        colloss_kernel<<<static_cast<unsigned>(cdiv(d_in, 32)), dim3(32, 8), 0, stream>>>(o.E, d_out, d_in, col_loss);
+        colloss_kernel<<<static_cast<unsigned>(cdiv(d_in, CS_X)), dim3(CS_X, CS_Y), 0, stream>>>(o.E, d_out, d_in, col_loss);
         KQ_LAUNCH_CHECK("colloss_kernel");
     }
     return KQ_OK;
