@@ -8,7 +8,7 @@
 // reversal, the lower Cholesky factor C of A = J H J gives H = (J C J)(J C J)^T, J C J
 // upper, hence H^-1 = (J C^-T J)(J C^-T J)^T and L = J C^-T J, i.e. L[i][j] = C^-1[n-1-j][n-1-i].
 // One right-looking blocked sweep (block nb = 128) computes C and Z = C^-1 together:
-//   step k: diag  -- factor A_kk = C_kk C_kk^T and invert C_kk in shared memory (1 CTA);
+//   step k: diag  -- factor A_kk = C_kk C_kk^T and invert C_kk in registers (1 CTA);
 //           panel -- C_ik = A_ik C_kk^-T (i > k) and Z_kj = C_kk^-1 B_kj (j < k);
 //           update-- A_ij -= C_ik C_jk^T (k < j <= i) and B_ij -= C_ik Z_kj (j <= k < i),
 // where B (stored in Z's blocks) is the right-hand side I of C Z = I after the earlier
@@ -28,7 +28,6 @@ namespace {
 
 constexpr int NB = 128;
 constexpr int LD = NB + 1;                      // padded shared-memory row
-constexpr int TILE_FLOATS = NB * LD;
 
 struct Work {
     float* A;      // npad x npad, reversed damped H -> C (lower)
@@ -75,274 +74,439 @@ __global__ void prep_kernel(const float* __restrict__ H, int64_t n, int64_t npad
 }
 
 // ---------------------------------------------------------------- diag block
-constexpr int DIAG_THREADS = 512;
-constexpr int SB = 32;                        // leaf size inside the diagonal block
-constexpr int TLDD = SB + 1;
-constexpr size_t DIAG_SMEM = (2 * TILE_FLOATS + NB * TLDD + 2 * NB) * sizeof(float);
+// Factor A_kk = C C^T and invert C on one CTA, as an L D L^T sweep that builds L^-1 in
+// place (Gauss-Jordan on the lower triangle), four columns per barrier.
+//
+// Scalar step j (the definition): with the "hook" h (row j left of the diagonal, column j
+// below it, h_j = 0), pivot d_j and multipliers u_i = M_ij / d_j, every row i > j updates
+//   M_ik -= u_i h_k      (k != j; k > j: Schur complement, k < j: rows of L^-1)
+// and column j keeps its value, the unscaled column j of L D. So M ends up holding, below
+// the diagonal, R = -L^-1 D (column-scaled), and C = L D^1/2 has C_ij = (column j at step j)
+// / sqrt(d_j), while C^-1 = D^-1/2 L^-1 has entries -R_ik / (d_k sqrt(d_i)).
+//
+// Four steps at once (block column q, rows j..j+3, j = 4q): with the 4 x 4 pivot block
+// factored as L_b D_b L_b^T (raw columns g = L_b D_b, raw inverse rows b of the block),
+// a panel row p below it gives w = L_b^-1 p (the raw hook values of the four steps) and
+// u = w / d; a block-row column x (left of the block) gives h = L_b^-1 x; the four scalar
+// updates of a below-block entry sum to M_ik -= sum_t u_i^t h_k^t with h = w for columns
+// right of the block. Panel entries end as w_s - sum_{t>s} u^t b_ts, block-row entries as
+// h, and the pivot block as b. The pivot block's owner factors it once and publishes the
+// record; panel rows and block-row rows are published raw by their owners. One barrier
+// per block column; the staging is double-buffered.
+//
+// Thread t < 528 owns one 4 x 4 block of the lower triangle (row-major block order) in
+// registers. Pivots are checked by thread 0 (first non-positive one reported).
+constexpr int DIAG_THREADS = 544;                            // 528 owners + 16 idle lanes
+constexpr int DG_OWNERS = (NB / 4) * (NB / 4 + 1) / 2;       // 528
+constexpr int DG_LD = NB + 4;                                // craw row stride (16-byte rows)
+constexpr int DG_PIV = 32;                                   // floats per pivot record
+constexpr size_t DIAG_SMEM =
+    (static_cast<size_t>(NB) * DG_LD + 2 * NB * 4 + 2 * 4 * NB + 2 * DG_PIV + NB) * sizeof(float);
 
-__device__ __forceinline__ void named_barrier(int id, int nthreads) {
-    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+struct Piv4 {   // factored 4 x 4 pivot block: 1 / d, unit-lower L_b, raw inverse rows b
+    float rd[4], l10, l20, l30, l21, l31, l32, b10, b20, b30, b21, b31, b32;
+};
+
+__device__ __forceinline__ float rcp_approx(float x) {
+    float r;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+    return r;
 }
 
-// Leaf factor by 128 threads (warps 0..3, named barrier 1): thread t owns row t / 4 of the
-// 32 x 32 leaf at s and the columns k = t (mod 4). Step j updates the trailing part with
-// the pivot scaling deferred, a_ik -= (a_ij / p_j) a_kj; afterwards C_ij = a_ij / sqrt(p_j),
-// C_jj = sqrt(p_j), and dv[j] = 1 / C_jj. Returns the first non-positive pivot, or -1.
-__device__ __forceinline__ int leaf_factor128(float* s, int ld, float* pv, float* dv, int t) {
-    const int i = t >> 2, q = t & 3;
-    int bad = -1;
-#pragma unroll 1
-    for (int j = 0; j < SB; ++j) {
-        const float p = s[j * ld + j];
-        if (!(p > 0.0f) && bad < 0) bad = j;
-        if (i > j) {
-            const float f = s[i * ld + j] * __fdiv_rn(1.0f, p);
-            // at most 8 columns per thread: unrolled so all loads are issued together
-            float sk[8], si[8];
-#pragma unroll
-            for (int m = 0; m < 8; ++m) {
-                const int k = j + 1 + q + 4 * m;
-                if (k <= i) {
-                    sk[m] = s[k * ld + j];
-                    si[m] = s[i * ld + k];
-                }
-            }
-#pragma unroll
-            for (int m = 0; m < 8; ++m) {
-                const int k = j + 1 + q + 4 * m;
-                if (k <= i) s[i * ld + k] = fmaf(-f, sk[m], si[m]);
-            }
-        }
-        if (t == 0) pv[j] = p;
-        named_barrier(1, 128);
-    }
-    for (int e = t; e < SB * SB; e += 128) {
-        const int r = e >> 5, c = e & 31;
-        const float d = sqrtf(pv[c]);
-        if (c < r) s[r * ld + c] = __fdiv_rn(s[r * ld + c], d);
-        else if (c == r) s[r * ld + c] = d;
-        else s[r * ld + c] = 0.0f;
-        if (r == 0) dv[c] = __fdiv_rn(1.0f, d);
-    }
-    named_barrier(1, 128);
-    return bad;
+// x <- L_b^-1 x
+__device__ __forceinline__ void unit_lower_solve(float& x0, float& x1, float& x2, float& x3, const Piv4& p) {
+    x1 = fmaf(-p.l10, x0, x1);
+    x2 = fmaf(-p.l20, x0, x2);
+    x3 = fmaf(-p.l30, x0, x3);
+    x2 = fmaf(-p.l21, x1, x2);
+    x3 = fmaf(-p.l31, x1, x3);
+    x3 = fmaf(-p.l32, x2, x3);
 }
 
-// Leaf inverse by 128 threads without block barriers: four lanes per column c (8 columns
-// per warp), lane q of the group owning rows i = q (mod 4). Step i: the owner of row i
-// finalizes x_ic = b_ic / C_ii and shuffles it to the group, which updates
-// b_i'c -= C_i'i x_ic for its rows i' > i. X (stride ld) starts as the identity.
-__device__ __forceinline__ void leaf_inverse128(const float* L, float* X, int ld, const float* dv, int t) {
-    const int c = t >> 2, q = t & 3;
-    const int lane = threadIdx.x & 31, gbase = lane & ~3;
-    for (int r = q; r < SB; r += 4) X[r * ld + c] = (r == c) ? 1.0f : 0.0f;
-    __syncwarp();
-#pragma unroll 1
-    for (int i = 0; i < SB; ++i) {
-        float xi = 0.0f;
-        if ((i & 3) == q) {
-            xi = X[i * ld + c] * dv[i];
-            X[i * ld + c] = xi;
-        }
-        xi = __shfl_sync(0xffffffffu, xi, gbase | (i & 3));
-        const int r0 = i + 1 + ((q - i - 1) & 3);   // first row > i owned by this lane
-        float lr[8], xr[8];
+// Publish the inputs of block step q (buffer q & 1): block-row rows (left of the pivot),
+// panel rows (below it), and the factored pivot, whose owner also sets its block final.
+__device__ __forceinline__ void diag_publish(int q, float (&m)[4][4], int bi, int bk, float* Pst, float* Qst,
+                                             float* Pv, float* craw) {
+    const int buf = q & 1;
+    const int i0 = 4 * bi, k0 = 4 * bk;
+    if (bi == q && bk < q) {
 #pragma unroll
-        for (int m = 0; m < 8; ++m) {
-            const int r = r0 + 4 * m;
-            if (r < SB) {
-                lr[m] = L[r * ld + i];
-                xr[m] = X[r * ld + c];
-            }
-        }
+        for (int r = 0; r < 4; ++r)
+            *reinterpret_cast<float4*>(Qst + buf * 4 * NB + r * NB + k0) = make_float4(m[r][0], m[r][1], m[r][2], m[r][3]);
+    }
+    if (bk == q && bi > q) {
 #pragma unroll
-        for (int m = 0; m < 8; ++m) {
-            const int r = r0 + 4 * m;
-            if (r < SB) X[r * ld + c] = fmaf(-lr[m], xi, xr[m]);
-        }
-        __syncwarp();
+        for (int r = 0; r < 4; ++r)
+            *reinterpret_cast<float4*>(Pst + buf * NB * 4 + (i0 + r) * 4) = make_float4(m[r][0], m[r][1], m[r][2], m[r][3]);
+    }
+    if (bi == q && bk == q) {
+        float a11 = m[1][1], a21 = m[2][1], a31 = m[3][1], a22 = m[2][2], a32 = m[3][2], a33 = m[3][3];
+        const float d0 = m[0][0], g10 = m[1][0], g20 = m[2][0], g30 = m[3][0];
+        const float r0 = rcp_approx(d0);
+        const float l10 = g10 * r0, l20 = g20 * r0, l30 = g30 * r0;
+        a11 = fmaf(-l10, g10, a11);
+        a21 = fmaf(-l20, g10, a21);
+        a31 = fmaf(-l30, g10, a31);
+        a22 = fmaf(-l20, g20, a22);
+        a32 = fmaf(-l30, g20, a32);
+        a33 = fmaf(-l30, g30, a33);
+        const float d1 = a11, g21 = a21, g31 = a31;
+        const float r1 = rcp_approx(d1);
+        const float l21 = g21 * r1, l31 = g31 * r1;
+        a22 = fmaf(-l21, g21, a22);
+        a32 = fmaf(-l31, g21, a32);
+        a33 = fmaf(-l31, g31, a33);
+        const float d2 = a22, g32 = a32;
+        const float r2 = rcp_approx(d2);
+        const float l32 = g32 * r2;
+        a33 = fmaf(-l32, g32, a33);
+        const float d3 = a33;
+        const float r3 = rcp_approx(d3);
+        const float b10 = g10, b21 = g21, b32 = g32;
+        const float b20 = fmaf(-l21, b10, g20);
+        const float b31 = fmaf(-l32, b21, g31);
+        const float b30 = fmaf(-l32, b20, fmaf(-l31, b10, g30));
+        float* pv = Pv + buf * DG_PIV;
+        *reinterpret_cast<float4*>(pv) = make_float4(r0, r1, r2, r3);
+        *reinterpret_cast<float4*>(pv + 4) = make_float4(l10, l20, l30, l21);
+        *reinterpret_cast<float4*>(pv + 8) = make_float4(l31, l32, b10, b20);
+        *reinterpret_cast<float4*>(pv + 12) = make_float4(b30, b21, b31, b32);
+        *reinterpret_cast<float4*>(pv + 16) = make_float4(d0, d1, d2, d3);
+        m[1][0] = b10;
+        m[2][0] = b20;
+        m[3][0] = b30;
+        m[2][1] = b21;
+        m[3][1] = b31;
+        m[3][2] = b32;
+        craw[(i0 + 1) * DG_LD + k0] = g10;
+        craw[(i0 + 2) * DG_LD + k0] = g20;
+        craw[(i0 + 3) * DG_LD + k0] = g30;
+        craw[(i0 + 2) * DG_LD + k0 + 1] = g21;
+        craw[(i0 + 3) * DG_LD + k0 + 1] = g31;
+        craw[(i0 + 3) * DG_LD + k0 + 2] = g32;
     }
 }
 
-// Factor A_kk = C C^T and invert C in shared memory, blocked by 32 x 32 leaves:
-//   leaf p: warps 0..3 factor leaf (p, p) while warps 4..7 invert leaf p - 1; then one warp
-//   per row solves the rows below against the leaf (C_qp = A_qp C_pp^-T) and all warps
-//   update the trailing part with 4 x 4 register tiles;
-//   after the last leaf: X_qp = -X_qq sum_{r=p}^{q-1} C_qr X_rp by increasing q - p.
-// Writes C to A_kk and X = C^-1 to Z_kk. A non-positive pivot records its index in H's
-// own numbering (1-based).
 __global__ void __launch_bounds__(DIAG_THREADS) chol_diag_kernel(Work w, int64_t n, int64_t npad, int k, int* info) {
-    extern __shared__ float sm[];
-    float* a = sm;                        // [NB][LD]  A_kk -> C
-    float* x = sm + TILE_FLOATS;          // [NB][LD]  C^-1
-    float* t = sm + 2 * TILE_FLOATS;      // [NB][TLDD] temporaries
-    float* pv = t + NB * TLDD;            // [NB] pivots
-    float* dv = pv + NB;                  // [NB] 1 / C_jj
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    constexpr int NW = DIAG_THREADS / 32;
+    extern __shared__ __align__(16) float sm[];
+    float* craw = sm;                     // [NB][DG_LD]  columns of L D at their own step
+    float* Pst = craw + NB * DG_LD;       // [2][NB][4]   panel rows
+    float* Qst = Pst + 2 * NB * 4;        // [2][4][NB]   block-row rows
+    float* Pv = Qst + 2 * 4 * NB;         // [2][DG_PIV]  pivot records
+    float* dv = Pv + 2 * DG_PIV;          // [NB]         pivots d
+    const int tid = threadIdx.x;
     const int64_t off = static_cast<int64_t>(k) * NB;
-    for (int e = tid; e < NB * NB; e += blockDim.x) {
-        const int r = e / NB, c = e % NB;
-        a[r * LD + c] = c <= r ? w.A[(off + r) * npad + off + c] : 0.0f;
-        x[r * LD + c] = 0.0f;
+    const bool owner = tid < DG_OWNERS;
+    int bi = 0, bk = 0;
+    if (owner) {
+        int rem = tid;
+        while (rem > bi) {
+            rem -= bi + 1;
+            ++bi;
+        }
+        bk = rem;
+    }
+    const int i0 = 4 * bi, k0 = 4 * bk;
+    float m[4][4];
+    if (owner) {
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            const float4 v = *reinterpret_cast<const float4*>(w.A + (off + i0 + r) * npad + off + k0);
+            m[r][0] = v.x;
+            m[r][1] = v.y;
+            m[r][2] = v.z;
+            m[r][3] = v.w;
+        }
+        diag_publish(0, m, bi, bk, Pst, Qst, Pv, craw);
     }
     __syncthreads();
-    for (int p = 0; p <= NB / SB; ++p) {
-        const int o = p * SB;
-        if (p < NB / SB && warp < 4) {
-            const int bad = leaf_factor128(a + o * LD + o, LD, pv + o, dv + o, tid);
-            if (bad >= 0 && tid == 0) {
-                const int64_t rev = off + o + bad;
-                if (rev < n) record_error(info, static_cast<int>(n - rev));
-            }
-        } else if (p > 0 && warp >= 4 && warp < 8) {
-            const int po = o - SB;
-            leaf_inverse128(a + po * LD + po, x + po * LD + po, LD, dv + po, tid - 128);
-        }
-        __syncthreads();
-        if (p == NB / SB) break;
-        const int nr = NB - o - SB;
-        // rows below: warp per row (3 rows interleaved), lane = column of the leaf
-        for (int r0 = warp; r0 < nr; r0 += 3 * NW) {
-            float v[3];
-            int rr[3];
+#pragma unroll 1
+    for (int q = 0; q < NB / 4; ++q) {
+        const int buf = q & 1;
+        const float* pv = Pv + buf * DG_PIV;
+        if (tid == 0) {
 #pragma unroll
-            for (int u = 0; u < 3; ++u) {
-                rr[u] = r0 + u * NW;
-                v[u] = rr[u] < nr ? a[(o + SB + rr[u]) * LD + o + lane] : 0.0f;
-            }
-            const float* L = a + o * LD + o;
-#pragma unroll 4
-            for (int m = 0; m < SB; ++m) {
-                const float lm = L[lane * LD + m];
-                const float dm = dv[o + m];
-#pragma unroll
-                for (int u = 0; u < 3; ++u) {
-                    const float vm = __shfl_sync(0xffffffffu, v[u], m) * dm;
-                    if (lane == m) v[u] = vm;
-                    else if (lane > m) v[u] = fmaf(-vm, lm, v[u]);
+            for (int t = 0; t < 4; ++t) {
+                const float d = pv[16 + t];
+                dv[4 * q + t] = d;
+                if (!(d > 0.0f)) {
+                    const int64_t rev = off + 4 * q + t;
+                    if (rev < n) record_error(info, static_cast<int>(n - rev));
                 }
             }
-#pragma unroll
-            for (int u = 0; u < 3; ++u)
-                if (rr[u] < nr) a[(o + SB + rr[u]) * LD + o + lane] = v[u];
         }
-        __syncthreads();
-        // trailing update of rows/cols [o + SB, NB): 4 x 4 register tiles of the lower part
-        const int nt = nr / 4;
-        for (int e = tid; e < nt * nt; e += blockDim.x) {
-            const int tr = e / nt, tc = e % nt;
-            if (tc > tr) continue;
-            const int r0 = o + SB + 4 * tr, c0 = o + SB + 4 * tc;
-            float acc[4][4] = {};
-#pragma unroll 4
-            for (int m = 0; m < SB; ++m) {
-                float ra[4], cb[4];
-#pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    ra[u] = a[(r0 + u) * LD + o + m];
-                    cb[u] = a[(c0 + u) * LD + o + m];
-                }
-#pragma unroll
-                for (int u = 0; u < 4; ++u)
-#pragma unroll
-                    for (int v2 = 0; v2 < 4; ++v2) acc[u][v2] = fmaf(ra[u], cb[v2], acc[u][v2]);
+        if (owner && bi >= q && !(bi == q && bk >= q)) {
+            Piv4 p;
+            {
+                const float4 v0 = *reinterpret_cast<const float4*>(pv);
+                const float4 v1 = *reinterpret_cast<const float4*>(pv + 4);
+                const float4 v2 = *reinterpret_cast<const float4*>(pv + 8);
+                const float4 v3 = *reinterpret_cast<const float4*>(pv + 12);
+                p.rd[0] = v0.x;
+                p.rd[1] = v0.y;
+                p.rd[2] = v0.z;
+                p.rd[3] = v0.w;
+                p.l10 = v1.x;
+                p.l20 = v1.y;
+                p.l30 = v1.z;
+                p.l21 = v1.w;
+                p.l31 = v2.x;
+                p.l32 = v2.y;
+                p.b10 = v2.z;
+                p.b20 = v2.w;
+                p.b30 = v3.x;
+                p.b21 = v3.y;
+                p.b31 = v3.z;
+                p.b32 = v3.w;
             }
+            if (bi == q) {
+                // block row, left of the pivot: rows become L_b^-1 x (final)
 #pragma unroll
-            for (int u = 0; u < 4; ++u)
+                for (int c = 0; c < 4; ++c) unit_lower_solve(m[0][c], m[1][c], m[2][c], m[3][c], p);
+            } else {
+                // my rows below the pivot: w = L_b^-1 p, u = w / d
+                float u[4][4], wv[4][4];
+                const float* pr = Pst + buf * NB * 4 + i0 * 4;
 #pragma unroll
-                for (int v2 = 0; v2 < 4; ++v2)
-                    if (c0 + v2 <= r0 + u) a[(r0 + u) * LD + c0 + v2] -= acc[u][v2];
-        }
-        __syncthreads();
-    }
-    // off-diagonal leaves of X, by distance d = q - p, 4 x 4 register tiles
-    for (int d = 1; d < NB / SB; ++d) {
-        const int nblk = NB / SB - d;
-        for (int e = tid; e < nblk * 64; e += blockDim.x) {   // T_qp = sum_r C_qr X_rp
-            const int b = e >> 6, ti = (e >> 3) & 7, tj = e & 7;
-            const int pp = b, qq = b + d;
-            float acc[4][4] = {};
-            for (int r2 = pp; r2 < qq; ++r2) {
-#pragma unroll 4
-                for (int m = 0; m < SB; ++m) {
-                    float ca[4], xb[4];
+                for (int r = 0; r < 4; ++r) {
+                    const float4 x = *reinterpret_cast<const float4*>(pr + 4 * r);
+                    float x0 = x.x, x1 = x.y, x2 = x.z, x3 = x.w;
+                    unit_lower_solve(x0, x1, x2, x3, p);
+                    wv[r][0] = x0;
+                    wv[r][1] = x1;
+                    wv[r][2] = x2;
+                    wv[r][3] = x3;
+                    u[r][0] = x0 * p.rd[0];
+                    u[r][1] = x1 * p.rd[1];
+                    u[r][2] = x2 * p.rd[2];
+                    u[r][3] = x3 * p.rd[3];
+                }
+                if (bk == q) {
+                    // panel: final raw inverse columns; w is column block q of L D
 #pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        ca[u] = a[(qq * SB + 4 * ti + u) * LD + r2 * SB + m];
-                        xb[u] = x[(r2 * SB + m) * LD + pp * SB + 4 * tj + u];
+                    for (int r = 0; r < 4; ++r) {
+                        m[r][0] = fmaf(-u[r][3], p.b30, fmaf(-u[r][2], p.b20, fmaf(-u[r][1], p.b10, wv[r][0])));
+                        m[r][1] = fmaf(-u[r][3], p.b31, fmaf(-u[r][2], p.b21, wv[r][1]));
+                        m[r][2] = fmaf(-u[r][3], p.b32, wv[r][2]);
+                        m[r][3] = wv[r][3];
+                        *reinterpret_cast<float4*>(craw + (i0 + r) * DG_LD + k0) =
+                            make_float4(wv[r][0], wv[r][1], wv[r][2], wv[r][3]);
+                    }
+                } else {
+                    // h = L_b^-1 x, x from the block row (left columns) or the panel (right)
+                    float h[4][4];   // h[t][c]
+                    if (bk < q) {
+                        const float* qr = Qst + buf * 4 * NB + k0;
+#pragma unroll
+                        for (int t = 0; t < 4; ++t) {
+                            const float4 x = *reinterpret_cast<const float4*>(qr + t * NB);
+                            h[t][0] = x.x;
+                            h[t][1] = x.y;
+                            h[t][2] = x.z;
+                            h[t][3] = x.w;
+                        }
+                    } else {
+                        const float* pc = Pst + buf * NB * 4 + k0 * 4;
+#pragma unroll
+                        for (int c = 0; c < 4; ++c) {
+                            const float4 x = *reinterpret_cast<const float4*>(pc + 4 * c);
+                            h[0][c] = x.x;
+                            h[1][c] = x.y;
+                            h[2][c] = x.z;
+                            h[3][c] = x.w;
+                        }
                     }
 #pragma unroll
-                    for (int u = 0; u < 4; ++u)
+                    for (int c = 0; c < 4; ++c) unit_lower_solve(h[0][c], h[1][c], h[2][c], h[3][c], p);
 #pragma unroll
-                        for (int v2 = 0; v2 < 4; ++v2) acc[u][v2] = fmaf(ca[u], xb[v2], acc[u][v2]);
+                    for (int t = 0; t < 4; ++t)
+#pragma unroll
+                        for (int r = 0; r < 4; ++r)
+#pragma unroll
+                            for (int c = 0; c < 4; ++c) m[r][c] = fmaf(-u[r][t], h[t][c], m[r][c]);
                 }
             }
-#pragma unroll
-            for (int u = 0; u < 4; ++u)
-#pragma unroll
-                for (int v2 = 0; v2 < 4; ++v2) t[(b * SB + 4 * ti + u) * TLDD + 4 * tj + v2] = acc[u][v2];
         }
-        __syncthreads();
-        for (int e = tid; e < nblk * 64; e += blockDim.x) {   // X_qp = -X_qq T_qp
-            const int b = e >> 6, ti = (e >> 3) & 7, tj = e & 7;
-            const int pp = b, qq = b + d;
-            float acc[4][4] = {};
-#pragma unroll 4
-            for (int m = 0; m < SB; ++m) {
-                float xa[4], tb[4];
-#pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    xa[u] = x[(qq * SB + 4 * ti + u) * LD + qq * SB + m];
-                    tb[u] = t[(b * SB + m) * TLDD + 4 * tj + u];
-                }
-#pragma unroll
-                for (int u = 0; u < 4; ++u)
-#pragma unroll
-                    for (int v2 = 0; v2 < 4; ++v2) acc[u][v2] = fmaf(xa[u], tb[v2], acc[u][v2]);
-            }
-#pragma unroll
-            for (int u = 0; u < 4; ++u)
-#pragma unroll
-                for (int v2 = 0; v2 < 4; ++v2) x[(qq * SB + 4 * ti + u) * LD + pp * SB + 4 * tj + v2] = -acc[u][v2];
-        }
+        if (owner && q + 1 < NB / 4) diag_publish(q + 1, m, bi, bk, Pst, Qst, Pv, craw);
         __syncthreads();
     }
-    for (int e = tid; e < NB * NB; e += blockDim.x) {
-        const int r = e / NB, c = e % NB;
-        w.A[(off + r) * npad + off + c] = c <= r ? a[r * LD + c] : 0.0f;
-        w.Z[(off + r) * npad + off + c] = c <= r ? x[r * LD + c] : 0.0f;
+    // Scales (the staging is free now): sqrt(d), 1 / sqrt(d), 1 / d.
+    float* sq = Pst;
+    float* isq = Pst + NB;
+    float* idv = Qst;
+    if (tid < NB) {
+        const float d = dv[tid];
+        const float r = sqrtf(d);
+        sq[tid] = r;
+        isq[tid] = __frcp_rn(r);
+        idv[tid] = __frcp_rn(d);
+    }
+    __syncthreads();
+    // C^-1 = D^-1/2 L^-1 with L^-1_ik = -R_ik / d_k (k < i); the upper blocks of Z stay 0.
+    if (owner) {
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            const int i = i0 + r;
+            const float si = isq[i];
+            float o[4];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                const int kk = k0 + c;
+                o[c] = kk < i ? -m[r][c] * idv[kk] * si : (kk == i ? si : 0.0f);
+            }
+            *reinterpret_cast<float4*>(w.Z + (off + i) * npad + off + k0) = make_float4(o[0], o[1], o[2], o[3]);
+        }
+    }
+    // C = (L D) D^-1/2, upper part 0.
+    for (int e = tid; e < NB * NB / 4; e += blockDim.x) {
+        const int r = e / (NB / 4), c0 = 4 * (e % (NB / 4));
+        float o[4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int cc = c0 + c;
+            o[c] = cc < r ? craw[r * DG_LD + cc] * isq[cc] : (cc == r ? sq[r] : 0.0f);
+        }
+        *reinterpret_cast<float4*>(w.A + (off + r) * npad + off + c0) = make_float4(o[0], o[1], o[2], o[3]);
+    }
+}
+
+// ---------------------------------------------------------- strips of one tile
+// The panel and the first tiles of the next step are on the critical path and come in
+// ~nbk tiles, so each 128 x 128 tile is split over 4 CTAs (strips or quadrants) with the
+// whole K = 128 staged in shared memory at once (two cp.async groups of 64).
+constexpr int SK = NB;
+constexpr int SLD = SK + 4;   // row stride of K-contiguous slabs (conflict-free float4 rows)
+
+template <int BM, int BNc, bool BNL>
+struct Strip {
+    static constexpr int RM = BM / 16, CN = BNc / 16;
+    static constexpr int A_FLOATS = BM * SLD;
+    static constexpr int B_FLOATS = BNL ? SK * (BNc + 4) : BNc * SLD;
+    static constexpr size_t SMEM = static_cast<size_t>(A_FLOATS + B_FLOATS) * sizeof(float);
+};
+constexpr size_t smax(size_t a, size_t b) { return a > b ? a : b; }
+constexpr size_t STRIP_SMEM = smax(smax(Strip<128, 32, true>::SMEM, Strip<32, 128, false>::SMEM),
+                                   smax(Strip<64, 64, true>::SMEM, Strip<64, 64, false>::SMEM));
+
+// acc[i][j] = sum over k < 128 of A[ty + 16 i][k] * B(k, col_j), 256 threads (ty, tx) =
+// (tid / 16, tid % 16). A is K-contiguous (row r at A + r ld). BNL = false: B(k, c) at
+// B + c ld + k, col_j = tx + 16 j; BNL = true: B(k, c) at B + k ld + c, col_j = CN tx + j.
+// All global reads finish before the function returns (the output may alias an input
+// row or column strip of this CTA).
+template <int BM, int BNc, bool BNL>
+__device__ __forceinline__ void strip_gemm(const float* __restrict__ A, const float* __restrict__ B, int64_t ld,
+                                           float (&acc)[BM / 16][BNc / 16], float* sm) {
+    using S = Strip<BM, BNc, BNL>;
+    constexpr int RM = S::RM, CN = S::CN, BLD = BNc + 4;
+    float* As = sm;
+    float* Bs = sm + S::A_FLOATS;
+    const int tid = threadIdx.x, ty = tid >> 4, tx = tid & 15;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int kh = h * (SK / 2);
+        for (int q = tid; q < BM * (SK / 8); q += G_THREADS) {
+            const int r = q / (SK / 8), k4 = q % (SK / 8);
+            cp_async16(As + r * SLD + kh + 4 * k4, A + r * ld + kh + 4 * k4, 16);
+        }
+        if (BNL) {
+            for (int q = tid; q < (SK / 2) * (BNc / 4); q += G_THREADS) {
+                const int kk = q / (BNc / 4), c4 = q % (BNc / 4);
+                cp_async16(Bs + (kh + kk) * BLD + 4 * c4, B + (kh + kk) * ld + 4 * c4, 16);
+            }
+        } else {
+            for (int q = tid; q < BNc * (SK / 8); q += G_THREADS) {
+                const int c = q / (SK / 8), k4 = q % (SK / 8);
+                cp_async16(Bs + c * SLD + kh + 4 * k4, B + c * ld + kh + 4 * k4, 16);
+            }
+        }
+        cp_async_commit();
+    }
+#pragma unroll
+    for (int i = 0; i < RM; ++i)
+#pragma unroll
+        for (int j = 0; j < CN; ++j) acc[i][j] = 0.0f;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        if (h == 0)
+            cp_async_wait<1>();
+        else
+            cp_async_wait<0>();
+        __syncthreads();
+#pragma unroll 2
+        for (int k4 = h * (SK / 8); k4 < (h + 1) * (SK / 8); ++k4) {
+            float4 a[RM];
+#pragma unroll
+            for (int i = 0; i < RM; ++i) a[i] = *reinterpret_cast<const float4*>(As + (ty + 16 * i) * SLD + 4 * k4);
+            if (!BNL) {
+#pragma unroll
+                for (int j = 0; j < CN; ++j) {
+                    const float4 b = *reinterpret_cast<const float4*>(Bs + (tx + 16 * j) * SLD + 4 * k4);
+#pragma unroll
+                    for (int i = 0; i < RM; ++i) {
+                        acc[i][j] = fmaf(a[i].x, b.x, acc[i][j]);
+                        acc[i][j] = fmaf(a[i].y, b.y, acc[i][j]);
+                        acc[i][j] = fmaf(a[i].z, b.z, acc[i][j]);
+                        acc[i][j] = fmaf(a[i].w, b.w, acc[i][j]);
+                    }
+                }
+            } else {
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk) {
+                    const float* brow = Bs + (4 * k4 + kk) * BLD + CN * tx;
+                    float bv[CN];
+                    if constexpr (CN % 4 == 0) {
+#pragma unroll
+                        for (int j4 = 0; j4 < CN / 4; ++j4) {
+                            const float4 t = *reinterpret_cast<const float4*>(brow + 4 * j4);
+                            bv[4 * j4] = t.x;
+                            bv[4 * j4 + 1] = t.y;
+                            bv[4 * j4 + 2] = t.z;
+                            bv[4 * j4 + 3] = t.w;
+                        }
+                    } else {
+                        static_assert(CN == 2, "strip width");
+                        const float2 t = *reinterpret_cast<const float2*>(brow);
+                        bv[0] = t.x;
+                        bv[1] = t.y;
+                    }
+#pragma unroll
+                    for (int i = 0; i < RM; ++i) {
+                        const float av = kk == 0 ? a[i].x : kk == 1 ? a[i].y : kk == 2 ? a[i].z : a[i].w;
+#pragma unroll
+                        for (int j = 0; j < CN; ++j) acc[i][j] = fmaf(av, bv[j], acc[i][j]);
+                    }
+                }
+            }
+        }
     }
 }
 
 // --------------------------------------------------------------------- panel
-// CTA b < k: Z_kb <- C_kk^-1 Z_kb.  CTA b >= k: i = b + 1, A_ik <- A_ik C_kk^-T. The whole
-// input tile is consumed before the in-place write (gemm_tile ends with a barrier).
+// CTA (b, s), b < k: column strip s (32 columns) of Z_kb <- C_kk^-1 Z_kb.
+// CTA (b, s), b >= k: row strip s (32 rows) of A_ik <- A_ik C_kk^-T, i = b + 1.
+// Each CTA reads and writes only its own strip, so the in-place update is race-free.
 __global__ void __launch_bounds__(G_THREADS, 2) chol_panel_kernel(Work w, int64_t npad, int k) {
     extern __shared__ __align__(16) float sm[];
-    const int b = blockIdx.x;
+    const int b = blockIdx.x, s = blockIdx.y;
     const int64_t off = static_cast<int64_t>(k) * NB;
     const float* cinv = w.Z + off * npad + off;
-    float acc[8][8];
-    float* out;
-    bool nn;
-    if (b < k) {
-        out = w.Z + off * npad + static_cast<int64_t>(b) * NB;
-        gemm_tile<true, true>(cinv, npad, NB, out, npad, NB, NB, acc, sm);   // C^-1 x B (B N-contiguous)
-        nn = true;
-    } else {
-        out = w.A + static_cast<int64_t>(b + 1) * NB * npad + off;
-        gemm_tile<false, true>(out, npad, NB, cinv, npad, NB, NB, acc, sm);  // A x (C^-1)^T
-        nn = false;
-    }
     const int ty = threadIdx.x >> 4, tx = threadIdx.x & 15;
+    if (b < k) {
+        float* out = w.Z + off * npad + static_cast<int64_t>(b) * NB + 32 * s;
+        float acc[8][2];
+        strip_gemm<128, 32, true>(cinv, out, npad, acc, sm);
 #pragma unroll
-    for (int i = 0; i < 8; ++i)
+        for (int i = 0; i < 8; ++i)
+            *reinterpret_cast<float2*>(out + (ty + 16 * i) * npad + 2 * tx) = make_float2(acc[i][0], acc[i][1]);
+    } else {
+        float* out = w.A + (static_cast<int64_t>(b + 1) * NB + 32 * s) * npad + off;
+        float acc[2][8];
+        strip_gemm<32, 128, false>(out, cinv, npad, acc, sm);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            const int c = nn ? gt_col<true>(tx, j) : gt_col<false>(tx, j);
-            out[static_cast<int64_t>(gt_row(ty, i)) * npad + c] = acc[i][j];
-        }
+        for (int i = 0; i < 2; ++i)
+#pragma unroll
+            for (int j = 0; j < 8; ++j) out[(ty + 16 * i) * npad + tx + 16 * j] = acc[i][j];
+    }
 }
 
 // out[tile] -= acc, loads of 32 values issued before their stores.
@@ -384,15 +548,48 @@ __device__ __forceinline__ void update_tile(const Work& w, int64_t npad, int k, 
         sub_tile<true>(out, npad, acc);
 }
 
+// Quadrant q (rows 64 (q / 2), columns 64 (q % 2)) of update tile (i, j) of step k.
+__device__ __forceinline__ void update_quad(const Work& w, int64_t npad, int k, int i, int j, int q, float* sm) {
+    const int64_t ko = static_cast<int64_t>(k) * NB;
+    const int64_t r0 = static_cast<int64_t>(i) * NB + 64 * (q >> 1);
+    const int64_t c0 = static_cast<int64_t>(j) * NB + 64 * (q & 1);
+    const int ty = threadIdx.x >> 4, tx = threadIdx.x & 15;
+    const float* cik = w.A + r0 * npad + ko;
+    float acc[4][4];
+    if (j > k) {
+        strip_gemm<64, 64, false>(cik, w.A + c0 * npad + ko, npad, acc, sm);
+        float* out = w.A + r0 * npad + c0;
+        float o[4][4];
+#pragma unroll
+        for (int a = 0; a < 4; ++a)
+#pragma unroll
+            for (int c = 0; c < 4; ++c) o[a][c] = out[(ty + 16 * a) * npad + tx + 16 * c];
+#pragma unroll
+        for (int a = 0; a < 4; ++a)
+#pragma unroll
+            for (int c = 0; c < 4; ++c) out[(ty + 16 * a) * npad + tx + 16 * c] = o[a][c] - acc[a][c];
+    } else {
+        strip_gemm<64, 64, true>(cik, w.Z + ko * npad + c0, npad, acc, sm);
+        float* out = w.Z + r0 * npad + c0;
+        float4 o[4];
+#pragma unroll
+        for (int a = 0; a < 4; ++a) o[a] = *reinterpret_cast<const float4*>(out + (ty + 16 * a) * npad + 4 * tx);
+#pragma unroll
+        for (int a = 0; a < 4; ++a)
+            *reinterpret_cast<float4*>(out + (ty + 16 * a) * npad + 4 * tx) =
+                make_float4(o[a].x - acc[a][0], o[a].y - acc[a][1], o[a].z - acc[a][2], o[a].w - acc[a][3]);
+    }
+}
+
 // The tiles that step k + 1 reads first: row block k + 1 (tiles (k + 1, j), j <= k + 1)
-// and block column k + 1 below it (tiles (i, k + 1), i > k + 1). nbk CTAs.
+// and block column k + 1 below it (tiles (i, k + 1), i > k + 1); nbk tiles x 4 quadrants.
 __global__ void __launch_bounds__(G_THREADS, 2) chol_next_kernel(Work w, int64_t npad, int k) {
     extern __shared__ __align__(16) float sm[];
     const int bid = blockIdx.x;
     if (bid < k + 2)
-        update_tile(w, npad, k, k + 1, bid, sm);
+        update_quad(w, npad, k, k + 1, bid, blockIdx.y, sm);
     else
-        update_tile(w, npad, k, bid, k + 1, sm);
+        update_quad(w, npad, k, bid, k + 1, blockIdx.y, sm);
 }
 
 // The other tiles of step k: (i, j) with i > k + 1 and j != k + 1 (i tiles in row block i).
@@ -461,9 +658,9 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
         KQ_CUDA(cudaFuncSetAttribute(chol_diag_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(DIAG_SMEM)));
         KQ_CUDA(cudaFuncSetAttribute(chol_panel_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     static_cast<int>(G_SMEM)));
+                                     static_cast<int>(STRIP_SMEM)));
         KQ_CUDA(cudaFuncSetAttribute(chol_next_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     static_cast<int>(G_SMEM)));
+                                     static_cast<int>(STRIP_SMEM)));
         KQ_CUDA(cudaFuncSetAttribute(chol_rest_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(G_SMEM)));
         attr = true;
@@ -480,7 +677,7 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
         chol_diag_kernel<<<1, DIAG_THREADS, DIAG_SMEM, stream>>>(w, n, npad, k, info);
         KQ_LAUNCH_CHECK("chol_diag_kernel");
         if (nbk > 1) {
-            chol_panel_kernel<<<nbk - 1, G_THREADS, G_SMEM, stream>>>(w, npad, k);
+            chol_panel_kernel<<<dim3(nbk - 1, 4), G_THREADS, STRIP_SMEM, stream>>>(w, npad, k);
             KQ_LAUNCH_CHECK("chol_panel_kernel");
         }
         if (k + 1 >= nbk) break;
@@ -489,7 +686,7 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
         const bool fork = side && rest > 0;
         if (fork) KQ_CUDA(cudaEventRecord(side->ev[0], stream));      // panel k done
         if (forked) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));  // rest of step k - 1 done
-        chol_next_kernel<<<nbk, G_THREADS, G_SMEM, stream>>>(w, npad, k);
+        chol_next_kernel<<<dim3(nbk, 4), G_THREADS, STRIP_SMEM, stream>>>(w, npad, k);
         KQ_LAUNCH_CHECK("chol_next_kernel");
         if (rest > 0) {
             cudaStream_t rs = stream;

@@ -94,6 +94,8 @@ constexpr int LPR = KQ_OBS_LANES_PER_ROW;   // lanes per row (8 or 16)
 constexpr int CPL = BLK / LPR;              // columns per lane
 constexpr int NV = CPL / 4;                 // float4 slots per lane
 static_assert(LPR == 8 || LPR == 16, "lanes per row must be 8 or 16");
+constexpr int OBS_ROWS = 16;                // rows per CTA
+constexpr int OBS_THREADS = OBS_ROWS * LPR; // 128 or 256
 
 // Packed layout of one diagonal block of R: row j holds R[i0 + j][i0 + c] at pos(c). The
 // CPL columns of lane lp fill slots [lp NV, lp NV + NV) of 16 bytes, rotated by lane so
@@ -153,7 +155,7 @@ __device__ __forceinline__ void load_cols(const float* __restrict__ W, int64_t r
 // VEC: d_in % 16 == 0 and W, codes (and pre_q) 16-byte aligned, so a lane's CPL columns
 // of W, E and codes move as 16-byte vectors.
 template <bool VEC>
-__global__ void __launch_bounds__(128, 3) obs_block_kernel(
+__global__ void __launch_bounds__(OBS_THREADS, 3) obs_block_kernel(
     const float* __restrict__ W, int64_t d_out, int64_t d_in, const float* __restrict__ Rp, int64_t i0,
     int bits, int group, const float* __restrict__ gscale, const float* __restrict__ gzero,
     uint8_t* __restrict__ codes, float* __restrict__ scale, int32_t* __restrict__ zero,
@@ -375,16 +377,15 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
     const bool vec = (d_in % 4 == 0) && (reinterpret_cast<uintptr_t>(Lt) % 16 == 0);
     const bool bvec = (d_in % 16 == 0) && (reinterpret_cast<uintptr_t>(W) % 16 == 0) &&
                       (reinterpret_cast<uintptr_t>(codes) % 16 == 0);
-    const int64_t rows_per_cta = 4 * (32 / LPR);   // 4 warps per CTA
-    const int64_t row_ctas = std::min<int64_t>(cdiv(d_out, rows_per_cta), static_cast<int64_t>(num_sms()) * 3);
+    const int64_t row_ctas = std::min<int64_t>(cdiv(d_out, OBS_ROWS), static_cast<int64_t>(num_sms()) * 3);
     for (int64_t i0 = 0; i0 < d_in; i0 += BLK) {
         const int kb = static_cast<int>(std::min<int64_t>(BLK, d_in - i0));
         const float* rp = o.Rp + (i0 / BLK) * BLK * BLK;
         if (bvec)
-            obs_block_kernel<true><<<static_cast<unsigned>(row_ctas), 128, BLK * BLK * 4, stream>>>(
+            obs_block_kernel<true><<<static_cast<unsigned>(row_ctas), OBS_THREADS, BLK * BLK * 4, stream>>>(
                 W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q);
         else
-            obs_block_kernel<false><<<static_cast<unsigned>(row_ctas), 128, BLK * BLK * 4, stream>>>(
+            obs_block_kernel<false><<<static_cast<unsigned>(row_ctas), OBS_THREADS, BLK * BLK * 4, stream>>>(
                 W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q);
         KQ_LAUNCH_CHECK("obs_block_kernel");
         const int64_t rest = d_in - (i0 + kb);
