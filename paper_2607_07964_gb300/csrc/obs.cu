@@ -260,18 +260,18 @@ __global__ void __launch_bounds__(OBS_THREADS, 3) obs_block_kernel(
     }
 }
 
-// W[:, e0:] -= E[:, i0:e0] R[i0:e0, e0:] with R[k][c] = Lt[c][k]: 128 x 128 output tiles
-// of the shared tile GEMM (acc = fma(E_k, R_kc, acc) over ascending k), then w = w - acc.
+// W[:, cb:ce] -= E[:, i0:i0+kb] R[i0:i0+kb, cb:ce] with R[k][c] = Lt[c][k]: 128 x 128 output
+// tiles of the shared tile GEMM (acc = fma(E_k, R_kc, acc) over ascending k), then w = w - acc.
 template <bool VEC>
 __global__ void __launch_bounds__(G_THREADS, 2) trailing_kernel(float* __restrict__ W, const float* __restrict__ E,
                                                                 const float* __restrict__ Lt, int64_t d_out,
-                                                                int64_t d_in, int64_t i0, int kb) {
+                                                                int64_t d_in, int64_t i0, int kb, int64_t cb,
+                                                                int64_t ce) {
     extern __shared__ __align__(16) float sm[];
-    const int64_t e0 = i0 + kb;
     const int64_t r0 = static_cast<int64_t>(blockIdx.y) * GT;
-    const int64_t c0 = e0 + static_cast<int64_t>(blockIdx.x) * GT;
+    const int64_t c0 = cb + static_cast<int64_t>(blockIdx.x) * GT;
     const int arows = static_cast<int>(min(static_cast<int64_t>(GT), d_out - r0));
-    const int bcols = static_cast<int>(min(static_cast<int64_t>(GT), d_in - c0));
+    const int bcols = static_cast<int>(min(static_cast<int64_t>(GT), ce - c0));
     float acc[8][8];
     gemm_tile<false, VEC>(E + r0 * d_in + i0, d_in, arows, Lt + c0 * d_in + i0, d_in, bcols, kb, acc, sm);
     const int ty = threadIdx.x >> 4, tx = threadIdx.x & 15;
@@ -378,6 +378,22 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
     const bool bvec = (d_in % 16 == 0) && (reinterpret_cast<uintptr_t>(W) % 16 == 0) &&
                       (reinterpret_cast<uintptr_t>(codes) % 16 == 0);
     const int64_t row_ctas = std::min<int64_t>(cdiv(d_out, OBS_ROWS), static_cast<int64_t>(num_sms()) * 3);
+    // Look-ahead: after block b, the update of block column b + 1 runs on the caller's stream
+    // (the next block kernel waits for it); the columns beyond run on a library side stream
+    // beside block b + 1. Every column still receives the block updates in block order
+    // (block column b + 2 gets E_b from the side stream before E_b+1 from the next step's
+    // first update, which waits for it), so the results are the same bits.
+    SideStream* side = nblk > 2 ? side_stream(stream) : nullptr;
+    bool forked = false;
+    auto trailing = [&](int64_t i0, int kb, int64_t cb, int64_t ce, cudaStream_t st) -> kq_status {
+        dim3 grid(static_cast<unsigned>(cdiv(ce - cb, GT)), static_cast<unsigned>(cdiv(d_out, GT)));
+        if (vec)
+            trailing_kernel<true><<<grid, G_THREADS, G_SMEM, st>>>(W, o.E, Lt, d_out, d_in, i0, kb, cb, ce);
+        else
+            trailing_kernel<false><<<grid, G_THREADS, G_SMEM, st>>>(W, o.E, Lt, d_out, d_in, i0, kb, cb, ce);
+        KQ_LAUNCH_CHECK("trailing_kernel");
+        return KQ_OK;
+    };
     for (int64_t i0 = 0; i0 < d_in; i0 += BLK) {
         const int kb = static_cast<int>(std::min<int64_t>(BLK, d_in - i0));
         const float* rp = o.Rp + (i0 / BLK) * BLK * BLK;
@@ -388,16 +404,29 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
             obs_block_kernel<false><<<static_cast<unsigned>(row_ctas), OBS_THREADS, BLK * BLK * 4, stream>>>(
                 W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q);
         KQ_LAUNCH_CHECK("obs_block_kernel");
-        const int64_t rest = d_in - (i0 + kb);
-        if (rest > 0) {
-            dim3 grid(static_cast<unsigned>(cdiv(rest, GT)), static_cast<unsigned>(cdiv(d_out, GT)));
-            if (vec)
-                trailing_kernel<true><<<grid, G_THREADS, G_SMEM, stream>>>(W, o.E, Lt, d_out, d_in, i0, kb);
-            else
-                trailing_kernel<false><<<grid, G_THREADS, G_SMEM, stream>>>(W, o.E, Lt, d_out, d_in, i0, kb);
-            KQ_LAUNCH_CHECK("trailing_kernel");
+        const int64_t nb0 = i0 + kb;                                // next block column
+        if (nb0 >= d_in) break;
+        const int64_t nb1 = std::min<int64_t>(d_in, nb0 + BLK);    // columns beyond it: [nb1, d_in)
+        const bool fork = side && nb1 < d_in;
+        if (fork) KQ_CUDA(cudaEventRecord(side->ev[0], stream));           // E of this block ready
+        if (forked) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));  // previous far update done
+        kq_status st = trailing(i0, kb, nb0, nb1, stream);
+        if (st != KQ_OK) return st;
+        if (nb1 < d_in) {
+            cudaStream_t fs = stream;
+            if (fork) {
+                KQ_CUDA(cudaStreamWaitEvent(side->s, side->ev[0], 0));
+                fs = side->s;
+            }
+            st = trailing(i0, kb, nb1, d_in, fs);
+            if (st != KQ_OK) return st;
+            if (fork) {
+                KQ_CUDA(cudaEventRecord(side->ev[1], side->s));
+                forked = true;
+            }
         }
     }
+    if (forked) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));
     if (col_loss) {
         colloss_kernel<<<static_cast<unsigned>(cdiv(d_in, CS_X)), dim3(CS_X, CS_Y), 0, stream>>>(o.E, d_out, d_in, col_loss);
         KQ_LAUNCH_CHECK("colloss_kernel");
