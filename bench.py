@@ -42,6 +42,10 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-graph", action="store_true", help="launch kernels directly instead of replaying a CUDA graph")
+    ap.add_argument("--x-chunk-tokens", type=int, default=0,
+                    help="token chunk of the H_X accumulation (0: one call)")
+    ap.add_argument("--g-chunk-tokens", type=int, default=32768,
+                    help="token chunk of the H_G accumulation (0: one call)")
     return ap.parse_args()
 
 
@@ -51,9 +55,10 @@ def workload_name(cfg) -> str:
             f"damp {cfg.damp}")
 
 
-def config_dict(cfg) -> dict:
+def config_dict(cfg, x_chunk: int = 0, g_chunk: int = 0) -> dict:
     return {"workload": workload_name(cfg), "d_out": cfg.d_out, "d_in": cfg.d_in, "T": cfg.T,
             "bits": cfg.bits, "group": cfg.group, "block": cfg.block, "damp": cfg.damp,
+            "factor_chunk_tokens": {"X": x_chunk, "G": g_chunk},
             "l2": "inputs larger than L2 (X and G are T x d bf16, >= 1 GiB each); no flush"}
 
 
@@ -74,21 +79,18 @@ def measured_peaks():
         return dict(FALLBACK_PEAKS), "fallback"
 
 
-def syrk_traffic(cfg):
-    """DRAM bytes per SYRK launch from a committed ncu capture, if it was taken on the
-    current kernel source (else None)."""
+def syrk_traffic(cfg, launch_tokens: int):
+    """DRAM bytes per SYRK launch from a committed ncu capture of a launch of the same
+    shape (d, tokens per launch), taken on the current kernel source; else None."""
     src = os.path.join(ROOT, "paper_2607_07964_gb300", "csrc", "syrk.cu")
     rec = os.path.join(ROOT, "profiles", "syrk_traffic.json")
     try:
         with open(rec) as f:
             r = json.load(f)
         h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-        if r.get("syrk_cu_sha256_16") != h:
+        if r.get("syrk_cu_sha256_16") != h or r.get("d") != cfg.d_in or r.get("T") != launch_tokens:
             return None
-        per_token = r["dram_bytes_per_launch"] / r["T"]
-        if r.get("d") != cfg.d_in:
-            return None
-        return per_token * cfg.T
+        return float(r["dram_bytes_per_launch"])
     except (OSError, ValueError, KeyError):
         return None
 
@@ -225,7 +227,7 @@ def run_reference(args):
     out = {"impl": "reference", "metric": METRIC, "value": v, "unit": "ms", "n_gpus": args.gpus,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": v, "higher_is_better": False,
            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-           "config": config_dict(cfg),
+           "config": config_dict(cfg, args.x_chunk_tokens, args.g_chunk_tokens),
            "cpu_baseline": {"value": v, "unit": "ms", "cores": last["cores"], "kind": "oracle",
                             "sample": last["sample"], "stages_ms": last["stages_ms"]},
            "e2e": {"value": v, "unit": "ms", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -246,7 +248,8 @@ def run_ours(args):
     dev = f"cuda:{local}"
     cfg = kqsynth.CONFIGS[args.config].replace(seed=rank)
     inp = kqsynth.device_layer(cfg, device=dev)
-    p = LayerPipeline(cfg.d_out, cfg.d_in, cfg.bits, cfg.group, cfg.block, cfg.damp, device=dev)
+    p = LayerPipeline(cfg.d_out, cfg.d_in, cfg.bits, cfg.group, cfg.block, cfg.damp, device=dev,
+                      x_chunk_tokens=args.x_chunk_tokens, g_chunk_tokens=args.g_chunk_tokens)
     stream = torch.cuda.current_stream()
 
     def barrier():
@@ -305,12 +308,14 @@ def run_ours(args):
               "sweep_trailing": fl["sweep"] / stage_ms["sweep"] / 1e9}
     peaks, peak_src = measured_peaks()
     peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+    # factor_x is one SYRK launch per token chunk: flops per launch / mean launch time.
+    n_launch = len(p._chunks("X", cfg.T))
     achieved = tflops["factor_x"]
-    traffic = syrk_traffic(cfg)
+    traffic = syrk_traffic(cfg, cfg.T // n_launch)
     roofline = {"kernel": "syrk_tc_kernel (H_X = X^T X)", "bound": "tensor", "achieved": achieved,
                 "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak, "traffic": traffic,
                 "peak_source": f"{peak_src} bf16 dense burst",
-                "algorithmic_flops_per_launch": fl["factor_x"]}
+                "algorithmic_flops_per_launch": fl["factor_x"] / n_launch, "launches_per_factor": n_launch}
 
     e2e = None
     if not args.no_e2e:
@@ -350,7 +355,7 @@ def run_ours(args):
                "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
                "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
                "dtype": "bf16 products, f32 accumulate/arithmetic", "data": "synthetic",
-               "config": config_dict(cfg), "stages_ms": stage_ms, "tflops": tflops,
+               "config": config_dict(cfg, args.x_chunk_tokens, args.g_chunk_tokens), "stages_ms": stage_ms, "tflops": tflops,
                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
                "launch_mode": "cuda graph replay (one graph per layer, two streams)" if graph is not None
                else "direct launches (two streams)",

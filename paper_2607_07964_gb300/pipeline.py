@@ -17,7 +17,7 @@ class LayerPipeline:
 
     def __init__(self, d_out: int, d_in: int, bits: int, group: int, block: int = 128,
                  damp: float = 0.01, device: str = "cuda", want_col_loss: bool = True,
-                 overlap: bool = True):
+                 overlap: bool = True, x_chunk_tokens: int = 0, g_chunk_tokens: int = 32768):
         self.d_out, self.d_in, self.bits, self.group, self.block, self.damp = d_out, d_in, bits, group, block, damp
         f32 = dict(dtype=torch.float32, device=device)
         ng = 1 if group == 0 else -(-d_in // group)
@@ -43,13 +43,35 @@ class LayerPipeline:
         # The critical path (H_X, Cholesky, sweep) runs on a high-priority stream so SMs freed
         # by the long-running H_G tiles go to it first.
         self.overlap = overlap
+        # H_X and H_G are accumulated over token chunks of these sizes (0: one call). The host
+        # path copies X, then G, and accumulates each chunk as soon as it has arrived; G is
+        # the last input, so chunking it hides its accumulation under its own copy, while
+        # H_X's single call already hides under G's copy. In the device-resident schedule
+        # H_G runs on the side stream, where the cost of the shorter calls is mostly hidden.
+        self.chunk_tokens = {"X": x_chunk_tokens, "G": g_chunk_tokens}
         try:
             lo, hi = torch.cuda.Stream.priority_range()
         except (AttributeError, RuntimeError):
             lo, hi = 0, -1
         self.main = torch.cuda.Stream(device=device, priority=hi) if overlap else None
         self.side = torch.cuda.Stream(device=device, priority=lo) if overlap else None
-        self._ev = [torch.cuda.Event() for _ in range(6)]
+        self.copy = None
+        self._ev = [torch.cuda.Event() for _ in range(7)]
+
+    def _chunks(self, which: str, T: int) -> list[tuple[int, int]]:
+        c = self.chunk_tokens[which]
+        c = c if c > 0 else max(T, 1)
+        return [(t0, min(T, t0 + c)) for t0 in range(0, max(T, 1), c)]
+
+    def _factor(self, which, A, H, trace, info, stream, ready=None) -> None:
+        """H = A^T A over the token chunks (Alg. 1 online statistic); `ready`, if given,
+        holds one event per chunk that the stream waits on before using it."""
+        ch = self._chunks(which, A.shape[0])
+        for c, (t0, t1) in enumerate(ch):
+            if ready is not None:
+                stream.wait_event(ready[c])
+            kq.kq_accum_factor(A[t0:t1], H, accumulate=c > 0, trace=trace if c == len(ch) - 1 else None,
+                               info=info, stream=stream)
 
     def run(self, X, G, W, sign_u, sign_v, stream=None, events=None) -> None:
         """X [T, d_in] bf16, G [T, d_out] bf16, W [d_out, d_in] fp32 (left unchanged), signs
@@ -65,9 +87,9 @@ class LayerPipeline:
                 events[i].record(s)
 
         mark(0)
-        kq.kq_accum_factor(X, self.HX, trace=self.trace_x, info=self.info[0:1], stream=s)   # Alg. 1: H_X
+        self._factor("X", X, self.HX, self.trace_x, self.info[0:1], s)                           # Alg. 1: H_X
         mark(1)
-        kq.kq_accum_factor(G, self.HG, trace=self.trace_g, info=self.info[2:3], stream=s)   # H_G
+        self._factor("G", G, self.HG, self.trace_g, self.info[2:3], s)                           # H_G
         mark(2)
         kq.kq_compute_scales(W, self.HX, self.HG, self.s_x, self.s_g, stream=s)          # Eq. (rescale)
         kq.kq_traces(self.HX, self.s_x, self.HG, self.s_g, self.traces, stream=s)         # Eq. (sensitivity)
@@ -75,7 +97,8 @@ class LayerPipeline:
         with torch.cuda.stream(s):
             self.Wp.copy_(W)
         kq.kq_rotate_in(self.Wp, self.HX, self.s_x, sign_v, kq.KQ_FWD, stream=s)         # Eq. (biip), V side
-        kq.kq_rotate_out(self.Wp, self.HG, self.s_g, sign_u, kq.KQ_FWD, stream=s)        # U side; H_G released
+        kq.kq_rotate_out(self.Wp, None, self.s_g, sign_u, kq.KQ_FWD, stream=s)           # U side
+        kq.kq_rotate_out(None, self.HG, self.s_g, sign_u, kq.KQ_FWD, stream=s)           # H_G, then released
         mark(4)
         kq.kq_chol_inv(self.HX, self.damp, self.Lt, self.info[1:2], self.ws_chol, stream=s)  # Alg. 2
         mark(5)
@@ -83,17 +106,22 @@ class LayerPipeline:
                            self.zero, self.col_loss, None, self.ws_obs, stream=s)   # Alg. 2 sweep
         mark(6)
 
-    def _run_overlapped(self, X, G, W, sign_u, sign_v, caller) -> None:
+    def _run_overlapped(self, X, G, W, sign_u, sign_v, caller, x_ready=None, g_ready=None, w_ready=None) -> None:
         """The same results on two streams. The Cholesky needs only H_X and leaves most SMs
         idle during its diagonal steps, so H_G, S_G and U go to a low-priority stream that
         runs beside it; the high-priority stream does H_X, S_X, V, the Cholesky and (once
-        both sides are done) the sweep. Events order the shared buffers."""
+        U is applied to W) the sweep, while H_G's own rotation finishes beside the sweep.
+        Events order the shared buffers; x_ready / g_ready / w_ready are the host path's
+        copy events."""
         s, s2 = self.main, self.side
-        e_in, e_fx, e_tx, e_rin, e_side, e_out = self._ev
+        e_in, e_fx, e_tx, e_rin, e_side, e_out, e_hg = self._ev
         e_in.record(caller)
         s.wait_event(e_in)
-        kq.kq_accum_factor(X, self.HX, trace=self.trace_x, info=self.info[0:1], stream=s)
+        s2.wait_event(e_in)
+        self._factor("X", X, self.HX, self.trace_x, self.info[0:1], s, x_ready)
         e_fx.record(s)
+        if w_ready is not None:
+            s.wait_event(w_ready)
         kq.kq_compute_scales(W, self.HX, None, self.s_x, None, stream=s)
         kq.kq_traces(self.HX, self.s_x, None, None, self.traces, stream=s)
         e_tx.record(s)
@@ -103,18 +131,21 @@ class LayerPipeline:
         e_rin.record(s)
         kq.kq_chol_inv(self.HX, self.damp, self.Lt, self.info[1:2], self.ws_chol, stream=s)
         s2.wait_event(e_fx)                      # the two factors would only split the SMs
-        kq.kq_accum_factor(G, self.HG, trace=self.trace_g, info=self.info[2:3], stream=s2)
+        self._factor("G", G, self.HG, self.trace_g, self.info[2:3], s2, g_ready)
+        s2.wait_event(e_tx)                      # W (host path) and the X side of the traces
         kq.kq_compute_scales(W, None, self.HG, None, self.s_g, stream=s2)
-        s2.wait_event(e_tx)
         kq.kq_traces(None, None, self.HG, self.s_g, self.traces, stream=s2)
         s2.wait_event(e_rin)
-        kq.kq_rotate_out(self.Wp, self.HG, self.s_g, sign_u, kq.KQ_FWD, stream=s2)
+        kq.kq_rotate_out(self.Wp, None, self.s_g, sign_u, kq.KQ_FWD, stream=s2)
         e_side.record(s2)
+        kq.kq_rotate_out(None, self.HG, self.s_g, sign_u, kq.KQ_FWD, stream=s2)
+        e_hg.record(s2)
         s.wait_event(e_side)
         kq.kq_obs_quantize(self.Wp, self.Lt, self.bits, self.group, self.block, self.codes, self.scale,
                            self.zero, self.col_loss, None, self.ws_obs, stream=s)
         e_out.record(s)
         caller.wait_event(e_out)
+        caller.wait_event(e_hg)
 
     def capture(self, X, G, W, sign_u, sign_v) -> tuple:
         """Record one layer (both streams) as a CUDA graph on these fixed buffers. Returns
@@ -141,7 +172,12 @@ class LayerPipeline:
     def run_host(self, X_h, G_h, W_h, su_h, sv_h, codes_h, scale_h, zero_h, stream=None) -> tuple[int, int]:
         """End-to-end call with HOST buffers (pinned for asynchronous copies): copy the
         layer's inputs to the device, run the four stages, copy codes and grids back.
-        Enqueued on `stream`; the caller synchronizes. Returns (bytes in, bytes out)."""
+        Enqueued on `stream`; the caller synchronizes. Returns (bytes in, bytes out).
+
+        The copies run on their own stream in the order W, signs, X chunks, G chunks, and
+        each chunk's factor accumulation starts as soon as that chunk has arrived, so the
+        host link (the bound at these sizes) overlaps the factor, rescale, rotation and
+        Cholesky work; without the two-stream schedule the copies simply precede the run."""
         s = torch.cuda.current_stream() if stream is None else stream
         dev = self.HX.device
         if getattr(self, "_stage", None) is None or self._stage["X"].shape != X_h.shape:
@@ -153,14 +189,37 @@ class LayerPipeline:
                 "sv": torch.empty(sv_h.shape, dtype=sv_h.dtype, device=dev),
             }
         st = self._stage
-        with torch.cuda.stream(s):
-            for k, h in (("X", X_h), ("G", G_h), ("W", W_h), ("su", su_h), ("sv", sv_h)):
-                st[k].copy_(h, non_blocking=True)
-        self.run(st["X"], st["G"], st["W"], st["su"], st["sv"], stream=s)
+        nin = sum(t.numel() * t.element_size() for t in (X_h, G_h, W_h, su_h, sv_h))
+        nout = sum(t.numel() * t.element_size() for t in (codes_h, scale_h, zero_h))
+        if not self.overlap:
+            with torch.cuda.stream(s):
+                for k, h in (("X", X_h), ("G", G_h), ("W", W_h), ("su", su_h), ("sv", sv_h)):
+                    st[k].copy_(h, non_blocking=True)
+            self.run(st["X"], st["G"], st["W"], st["su"], st["sv"], stream=s)
+        else:
+            if self.copy is None:
+                self.copy = torch.cuda.Stream(device=dev)
+            cs = self.copy
+            e0 = torch.cuda.Event()
+            e0.record(s)
+            cs.wait_event(e0)
+            with torch.cuda.stream(cs):
+                for k, h in (("W", W_h), ("su", su_h), ("sv", sv_h)):
+                    st[k].copy_(h, non_blocking=True)
+                w_ready = torch.cuda.Event()
+                w_ready.record(cs)
+                ready = {}
+                for k, h in (("X", X_h), ("G", G_h)):
+                    ready[k] = []
+                    for t0, t1 in self._chunks(k, h.shape[0]):
+                        st[k][t0:t1].copy_(h[t0:t1], non_blocking=True)
+                        ev = torch.cuda.Event()
+                        ev.record(cs)
+                        ready[k].append(ev)
+            self._run_overlapped(st["X"], st["G"], st["W"], st["su"], st["sv"], s, x_ready=ready["X"],
+                                 g_ready=ready["G"], w_ready=w_ready)
         with torch.cuda.stream(s):
             codes_h.copy_(self.codes, non_blocking=True)
             scale_h.copy_(self.scale, non_blocking=True)
             zero_h.copy_(self.zero, non_blocking=True)
-        nin = sum(t.numel() * t.element_size() for t in (X_h, G_h, W_h, su_h, sv_h))
-        nout = sum(t.numel() * t.element_size() for t in (codes_h, scale_h, zero_h))
         return nin, nout

@@ -299,7 +299,8 @@ def test_pipeline_overlap_matches_serial():
     su, sv = dev(L["sign_u"], torch.int8), dev(L["sign_v"], torch.int8)
     out = []
     for overlap in (True, False):
-        p = LayerPipeline(cfg.d_out, cfg.d_in, cfg.bits, cfg.group, cfg.block, cfg.damp, overlap=overlap)
+        p = LayerPipeline(cfg.d_out, cfg.d_in, cfg.bits, cfg.group, cfg.block, cfg.damp, overlap=overlap,
+                          x_chunk_tokens=1024, g_chunk_tokens=1536)
         events = None if overlap else [torch.cuda.Event(enable_timing=True) for _ in range(len(STAGES) + 1)]
         for _ in range(2):   # twice: buffers reused across layers
             p.run(X, G, W, su, sv, events=events)
@@ -307,6 +308,38 @@ def test_pipeline_overlap_matches_serial():
         out.append({k: host(getattr(p, k)) for k in ("codes", "scale", "zero", "Lt", "s_x", "s_g", "traces", "col_loss")})
     for k in out[0]:
         assert np.array_equal(out[0][k], out[1][k]), k
+
+
+@pytest.mark.parametrize("overlap", [True, False])
+def test_pipeline_host_path_matches_device_path(overlap):
+    """run_host (host buffers, chunked copies overlapped with the factor accumulation)
+    gives the same bits as run on device-resident inputs with the same token chunks."""
+    from paper_2607_07964_gb300.pipeline import LayerPipeline
+    cfg = kqsynth.CONFIGS["tiny256"].replace(d_out=448, d_in=896, bits=4, group=128, T=5000, w_bf16=True)
+    L = kqsynth.layer(cfg)
+    X, G, W = bf16_dev(L["X"]), bf16_dev(L["G"]), dev(L["W"])
+    su, sv = dev(L["sign_u"], torch.int8), dev(L["sign_v"], torch.int8)
+    p = LayerPipeline(cfg.d_out, cfg.d_in, cfg.bits, cfg.group, cfg.block, cfg.damp, overlap=overlap,
+                      x_chunk_tokens=2048, g_chunk_tokens=1536)
+    p.run(X, G, W, su, sv)
+    p.check()
+    want = {k: host(getattr(p, k)) for k in ("codes", "scale", "zero", "Lt", "traces", "col_loss")}
+    Xh, Gh, Wh = X.cpu().pin_memory(), G.cpu().pin_memory(), W.cpu().pin_memory()
+    suh, svh = su.cpu().pin_memory(), sv.cpu().pin_memory()
+    ch = torch.empty(p.codes.shape, dtype=p.codes.dtype).pin_memory()
+    sh = torch.empty(p.scale.shape, dtype=p.scale.dtype).pin_memory()
+    zh = torch.empty(p.zero.shape, dtype=p.zero.dtype).pin_memory()
+    p.codes.zero_()
+    nin, nout = p.run_host(Xh, Gh, Wh, suh, svh, ch, sh, zh)
+    torch.cuda.synchronize()
+    p.check()
+    assert nin == sum(t.numel() * t.element_size() for t in (Xh, Gh, Wh, suh, svh))
+    assert nout == ch.numel() + 4 * sh.numel() + 4 * zh.numel()
+    assert np.array_equal(ch.numpy(), want["codes"])
+    assert np.array_equal(sh.numpy(), want["scale"])
+    assert np.array_equal(zh.numpy(), want["zero"])
+    for k in ("Lt", "traces", "col_loss"):
+        assert np.array_equal(host(getattr(p, k)), want[k]), k
 
 
 @pytest.mark.parametrize("T,d", [(5000, 640), (130, 8), (0, 64)])
