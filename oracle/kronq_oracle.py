@@ -131,6 +131,34 @@ def rht_matrix(n: int, sign: np.ndarray) -> np.ndarray:
     return hadamard_matrix(n).astype(np.float64) * sign[None, :] / np.sqrt(n)
 
 
+def rht_rows(n: int, sign: np.ndarray, rows) -> np.ndarray:
+    """Selected rows of V = H_n diag(sigma) / sqrt(n) without forming H_n (for sizes where the
+    dense n x n matrix is too large): Sylvester entries are (-1)^popcount(i & j); for
+    n = 28 * 2^k, H_n[i, j] = H_28[i // 2^k, j // 2^k] * H_{2^k}[i % 2^k, j % 2^k]."""
+    sign = np.asarray(sign, dtype=np.float64).reshape(-1)
+    assert sign.shape == (n,)
+    rows = np.asarray(rows, dtype=np.int64).reshape(-1)
+    if n >= 1 and n & (n - 1) == 0:
+        P, h28 = n, None
+    elif n % 28 == 0 and (n // 28) & (n // 28 - 1) == 0:
+        P, h28 = n // 28, paley28()
+    else:
+        raise ValueError(f"no Hadamard construction for n = {n}")
+    j = np.arange(n, dtype=np.int64)
+    out = np.empty((len(rows), n), dtype=np.float64)
+    for t, i in enumerate(rows):
+        both = (i % P) & (j % P)
+        parity = np.zeros(n, dtype=np.int64)
+        while np.any(both):
+            parity ^= both & 1
+            both >>= 1
+        v = 1.0 - 2.0 * parity
+        if h28 is not None:
+            v = v * h28[i // P, j // P]
+        out[t] = v * sign / np.sqrt(n)
+    return out
+
+
 # ----------------------------------------------------------------------------------
 # Stage 2: bidirectional incoherence processing (Eq. rescale, Eq. biip, Algorithm 1).
 # ----------------------------------------------------------------------------------

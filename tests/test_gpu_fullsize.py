@@ -1,14 +1,19 @@
-"""GPU parity at the benchmark's full size: the Llama-3-8B q_proj layer (W 4096 x 4096,
-T = 131072 calibration tokens, 4-bit, group 128), run through the same pipeline and the
-same kernels the benchmark times. The oracle cannot redo the whole layer in float64 here,
-so it checks what it can compute one by one:
-  * sampled entries and the whole diagonal of H_X and H_G (float64 dot products);
-  * S_X, S_G from those float64 diagonals;
-  * sampled rows of W' = U S_G W S_X V^T (dense float64 products);
-  * a 4096 x 4096 inverse Cholesky of an oracle-built SPD matrix;
-  * the 4096 x 4096 sweep, bit-exact against the fp32-ordered oracle on sampled rows.
-Inputs are drawn on the GPU with torch's generator (kqsynth.device_layer) and copied to
-the host for the oracle.
+"""GPU parity at full size for every Llama-shaped layer of the benchmark plan (q_proj and
+the MLP layers of the 8B model; q/o, k/v and down_proj of the 70B model), each run through
+the kernels and launch configuration the benchmark times (one H_X call, H_G in the
+pipeline's token chunks). The oracle cannot redo these layers in float64, so it checks what
+it can compute one by one, or what holds at any size:
+  * sampled entries and sampled diagonal entries of H_X and H_G (float64 dot products over
+    all T tokens);
+  * S_X, S_G at the sampled channels;
+  * sampled entries of W' = U S_G W S_X V^T and of H_X' = V S_X^-1 H_X S_X^-1 V^T (rows of
+    U and V built one at a time from the Hadamard definition);
+  * the inverse Cholesky: its trailing 1024 x 1024 block depends only on the trailing block
+    of the damped H_X' (H = U U^T with U upper gives L = U^-T block by block), which the
+    oracle factors exactly; and L L^T H e_j = e_j on sampled columns;
+  * the sweep on the GPU's own W' and L, bit-exact against the fp32-ordered oracle on
+    sampled rows.
+Inputs are drawn on the GPU with torch's generator (kqsynth.device_layer).
 """
 import numpy as np
 import pytest
@@ -20,6 +25,9 @@ from oracle import obs_sweep_fp32
 
 pytestmark = [pytest.mark.gpu, pytest.mark.slow]
 
+CONFIGS = ["q_proj_8b", "gate_up_8b", "down_8b", "qo_70b", "kv_70b", "down_70b"]
+TAIL = 1024
+
 
 def _rel(a, b):
     a = np.asarray(a, np.float64)
@@ -27,93 +35,114 @@ def _rel(a, b):
     return float(np.linalg.norm(a - b) / np.linalg.norm(b))
 
 
-@pytest.fixture(scope="module")
-def layer():
+def _bf16_cols(A, cols):
+    """float64 copy of the selected columns of a bf16 device matrix (exact widening)."""
+    return A[:, torch.as_tensor(cols, device=A.device)].float().cpu().numpy().astype(np.float64)
+
+
+@pytest.fixture(scope="module", params=CONFIGS)
+def layer(request):
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
     from paper_2607_07964_gb300 import build
-    build.build()
-    cfg = kqsynth.CONFIGS["q_proj_8b"]
-    return cfg, kqsynth.device_layer(cfg)
-
-
-def test_fullsize_factors_scales_rotation(layer):
     from paper_2607_07964_gb300 import kronq as K
     from paper_2607_07964_gb300.pipeline import LayerPipeline
-    cfg, inp = layer
-    X, G, W = inp["X"], inp["G"], inp["W"]
-    su, sv = inp["sign_u"], inp["sign_v"]
-    d_out, d_in = cfg.d_out, cfg.d_in
-    # the factors, as the pipeline's first stage computes them
-    HX = torch.empty((d_in, d_in), device="cuda")
-    HG = torch.empty((d_out, d_out), device="cuda")
-    K.kq_accum_factor(X, HX)
-    K.kq_accum_factor(G, HG)
-    Xh = X.cpu().view(torch.int16).numpy()
-    Gh = G.cpu().view(torch.int16).numpy()
-    to32 = lambda a: (a.astype(np.uint32) << 16).view(np.float32)  # noqa: E731  bf16 bits -> fp32
-    rng = np.random.default_rng(5)
-    diags = []
-    for A_bits, H, d in ((Xh, HX, d_in), (Gh, HG, d_out)):
-        cols = np.unique(rng.integers(0, d, 48))
-        A = to32(A_bits[:, cols].astype(np.uint16))
-        pairs = [(a, b) for a in range(len(cols)) for b in range(len(cols))]
-        want = ref.factor_entries(A, pairs).reshape(len(cols), len(cols))
-        got = H.cpu().numpy()[np.ix_(cols, cols)]
-        assert _rel(got, want) <= 1e-5
-        diag_want = np.zeros(d)
-        for t0 in range(0, A_bits.shape[0], 16384):   # float64 sums of squares over all tokens
-            diag_want += ref.factor_diag(to32(A_bits[t0:t0 + 16384].view(np.uint16)))
-        diag_got = torch.diagonal(H).cpu().numpy()
-        assert np.max(np.abs(diag_got - diag_want) / diag_want) <= 1e-5
-        diags.append(diag_want)
-    hx, hg = diags
-    # scales and the rotated weight, through the pipeline's own buffers
-    p = LayerPipeline(d_out, d_in, cfg.bits, cfg.group, cfg.block, cfg.damp)
-    K.kq_compute_scales(W, HX, HG, p.s_x, p.s_g)
-    Wh = W.cpu().numpy().astype(np.float64)
-    sx, sg = ref.biip_scales_from_diag(Wh, hx, hg)
-    assert np.max(np.abs(p.s_x.cpu().numpy() / sx - 1)) <= 1e-5
-    assert np.max(np.abs(p.s_g.cpu().numpy() / sg - 1)) <= 1e-5
-    Wp = W.clone()
-    K.kq_rotate_in(Wp, None, p.s_x, sv)
-    K.kq_rotate_out(Wp, None, p.s_g, su)
-    V = ref.rht_matrix(d_in, sv.cpu().numpy())
-    U = ref.rht_matrix(d_out, su.cpu().numpy())
-    M = (Wh * sx[None, :]) @ V.T
-    rows = np.unique(rng.integers(0, d_out, 16))
-    want = (U[rows] * sg[None, :]) @ M
-    assert _rel(Wp.cpu().numpy()[rows], want) <= 1e-5
-
-
-def test_fullsize_chol_and_sweep():
-    if not torch.cuda.is_available():
-        pytest.skip("no CUDA device")
-    from paper_2607_07964_gb300 import build
-    from paper_2607_07964_gb300 import kronq as K
     build.build()
-    n = 4096
-    H = kqsynth.random_spd(n, seed=23, cond_decay=1.0).astype(np.float32)
-    Lref = ref.lower_factor(ref.damp(H.astype(np.float64), 0.01))
-    Lt = torch.empty((n, n), device="cuda")
-    info = torch.zeros(1, dtype=torch.int32, device="cuda")
-    ws = torch.empty(K.kq_chol_inv_workspace(n), dtype=torch.uint8, device="cuda")
-    K.kq_chol_inv(torch.from_numpy(H).cuda(), 0.01, Lt, info, ws)
-    assert K.kq_check(info)[0] == K.KQ_OK
-    assert _rel(Lt.cpu().numpy(), Lref) <= 1e-5
-    # the sweep on the oracle's L and a seeded W' of the q_proj size
-    Lt32 = np.ascontiguousarray(Lref.astype(np.float32))
-    gen = torch.Generator(device="cuda")
-    gen.manual_seed(99)
-    Wp = (0.05 * torch.randn((n, n), generator=gen, device="cuda")).contiguous()
+    cfg = kqsynth.CONFIGS[request.param]
+    inp = kqsynth.device_layer(cfg)
+    d_out, d_in = cfg.d_out, cfg.d_in
+    p = LayerPipeline(d_out, d_in, cfg.bits, cfg.group, cfg.block, cfg.damp, overlap=False)
+    s = torch.cuda.current_stream()
+    # stage 1 as the pipeline launches it
+    p._factor("X", inp["X"], p.HX, p.trace_x, p.info[0:1], s)
+    p._factor("G", inp["G"], p.HG, p.trace_g, p.info[2:3], s)
+    HX_raw = p.HX.clone()
+    HG_raw = p.HG.clone()
+    K.kq_compute_scales(inp["W"], p.HX, p.HG, p.s_x, p.s_g)
+    p.Wp.copy_(inp["W"])
+    K.kq_rotate_in(p.Wp, p.HX, p.s_x, inp["sign_v"], K.KQ_FWD)
+    K.kq_rotate_out(p.Wp, None, p.s_g, inp["sign_u"], K.KQ_FWD)
+    Wp = p.Wp.clone()
+    K.kq_chol_inv(p.HX, cfg.damp, p.Lt, p.info[1:2], p.ws_chol)
+    K.kq_obs_quantize(p.Wp, p.Lt, cfg.bits, cfg.group, cfg.block, p.codes, p.scale, p.zero, None, None, p.ws_obs)
+    p.check()
+    yield cfg, inp, p, HX_raw, HG_raw, Wp
+    del p, inp, HX_raw, HG_raw, Wp
+    torch.cuda.empty_cache()
+
+
+def test_fullsize_factors_and_scales(layer):
+    cfg, inp, p, HX, HG, _ = layer
+    rng = np.random.default_rng(5)
+    W = inp["W"].cpu().numpy().astype(np.float64)
+    for A, H, d, s_dev, axis in ((inp["X"], HX, cfg.d_in, p.s_x, 0), (inp["G"], HG, cfg.d_out, p.s_g, 1)):
+        cols = np.unique(rng.integers(0, d, 40))
+        Ac = _bf16_cols(A, cols)
+        want = Ac.T @ Ac                              # float64 sums over all tokens
+        got = H[torch.as_tensor(cols, device="cuda")][:, torch.as_tensor(cols, device="cuda")].cpu().numpy()
+        assert _rel(got, want) <= 1e-5
+        assert np.max(np.abs(np.diag(got) / np.diag(want) - 1)) <= 1e-5
+        # scales at these channels: (h / ||W column or row||^2)^(1/4)
+        norm2 = np.sum(W[:, cols] ** 2, axis=0) if axis == 0 else np.sum(W[cols] ** 2, axis=1)
+        s_want = (np.diag(want) / norm2) ** 0.25
+        assert np.max(np.abs(s_dev.cpu().numpy()[cols] / s_want - 1)) <= 1e-5
+
+
+def test_fullsize_rotations(layer):
+    cfg, inp, p, HX, _, Wp = layer
+    rng = np.random.default_rng(6)
+    d_out, d_in = cfg.d_out, cfg.d_in
+    sx = p.s_x.cpu().numpy().astype(np.float64)
+    sg = p.s_g.cpu().numpy().astype(np.float64)
+    su, sv = inp["sign_u"].cpu().numpy(), inp["sign_v"].cpu().numpy()
+    rows = np.unique(rng.integers(0, d_out, 12))
+    cols = np.unique(rng.integers(0, d_in, 12))
+    U = ref.rht_rows(d_out, su, rows)
+    V = ref.rht_rows(d_in, sv, cols)
+    W = inp["W"].cpu().numpy().astype(np.float64)
+    want = ((U * sg[None, :]) @ W * sx[None, :]) @ V.T
+    got = Wp.cpu().numpy()[np.ix_(rows, cols)]
+    assert _rel(got, want) <= 1e-5
+    # H_X' = V S_X^-1 H_X S_X^-1 V^T at sampled entries
+    hrows = np.unique(rng.integers(0, d_in, 12))
+    Hh = HX.cpu().numpy().astype(np.float64)
+    Vr = ref.rht_rows(d_in, sv, hrows) / sx[None, :]
+    Vc = V / sx[None, :]
+    want = (Vr @ Hh) @ Vc.T
+    got = p.HX.cpu().numpy()[np.ix_(hrows, cols)]
+    assert _rel(got, want) <= 1e-5
+
+
+def test_fullsize_inverse_cholesky(layer):
+    cfg, _, p, _, _, _ = layer
+    n = cfg.d_in
+    Hrot = p.HX.cpu().numpy().astype(np.float64)
+    delta = cfg.damp * np.mean(np.diag(Hrot))
+    L = p.Lt.cpu().numpy()
+    # trailing block: exact against the oracle's inverse Cholesky of the damped trailing block
+    D = Hrot[n - TAIL:, n - TAIL:] + delta * np.eye(TAIL)
+    Lref = ref.lower_factor(D)
+    assert _rel(L[n - TAIL:, n - TAIL:], Lref) <= 1e-5
+    if n <= 4096:   # small enough for the whole float64 factor
+        assert _rel(L, ref.lower_factor(ref.damp(Hrot, cfg.damp))) <= 1e-5
+    assert np.all(np.triu(L, 1) == 0)
+    # L L^T H e_j = e_j on sampled columns (any size)
+    Ld = L.astype(np.float64)
+    for j in np.unique(np.random.default_rng(8).integers(0, n, 4)):
+        h = Hrot[:, j].copy()
+        h[j] += delta
+        r = Ld @ (Ld.T @ h)
+        e = np.zeros(n)
+        e[j] = 1.0
+        assert np.linalg.norm(r - e) <= 1e-3, (j, np.linalg.norm(r - e))
+
+
+def test_fullsize_sweep_bit_exact(layer):
+    cfg, _, p, _, _, Wp = layer
+    rows = np.unique(np.random.default_rng(9).integers(0, cfg.d_out, 24))
     Wh = Wp.cpu().numpy()
-    codes = torch.empty((n, n), dtype=torch.uint8, device="cuda")
-    scale = torch.empty((n, n // 128), device="cuda")
-    zero = torch.empty((n, n // 128), dtype=torch.int32, device="cuda")
-    wso = torch.empty(K.kq_obs_quantize_workspace(n, n, 128), dtype=torch.uint8, device="cuda")
-    K.kq_obs_quantize(Wp, torch.from_numpy(Lt32).cuda(), 4, 128, 128, codes, scale, zero, None, None, wso)
-    rows = np.unique(np.random.default_rng(7).integers(0, n, 48))
-    c = obs_sweep_fp32(Wh, Lt32, 4, 128, 128, rows=rows)
-    assert np.array_equal(codes.cpu().numpy()[rows], c["codes"])
-    assert np.array_equal(scale.cpu().numpy()[rows], c["scale"])
-    assert np.array_equal(zero.cpu().numpy()[rows], c["zero"].astype(np.int32))
+    Lt32 = np.ascontiguousarray(p.Lt.cpu().numpy())
+    c = obs_sweep_fp32(Wh, Lt32, cfg.bits, cfg.group, cfg.block, rows=rows)
+    assert np.array_equal(p.codes.cpu().numpy()[rows], c["codes"])
+    assert np.array_equal(p.scale.cpu().numpy()[rows], c["scale"])
+    assert np.array_equal(p.zero.cpu().numpy()[rows], c["zero"].astype(np.int32))

@@ -96,6 +96,23 @@ def test_rht_rotate_unrotate(n):
     assert np.allclose(np.linalg.norm(W @ V.T, axis=1), np.linalg.norm(W, axis=1))
 
 
+@pytest.mark.parametrize("n", [8, 64, 28, 112, 896])
+def test_rht_rows_match_dense_matrix(n):
+    """The row-at-a-time RHT used at full size equals rows of the dense definition."""
+    rng = _rng(n + 1)
+    sign = np.where(rng.random(n) < 0.5, -1, 1)
+    rows = np.unique(rng.integers(0, n, 5))
+    assert np.array_equal(ref.rht_rows(n, sign, rows), ref.rht_matrix(n, sign)[rows])
+
+
+def test_rht_rows_orthonormal_at_large_size():
+    """Rows of V for n = 28 * 1024 are orthonormal (checked on a sample)."""
+    n = 28 * 1024
+    sign = np.where(_rng(3).random(n) < 0.5, -1, 1)
+    R = ref.rht_rows(n, sign, [0, 1, 1023, 1024, 20000, n - 1])
+    assert np.allclose(R @ R.T, np.eye(6), atol=1e-12)
+
+
 # ---------------------------------------------------------------- rescaling (Eq. rescale)
 def test_rescale_equalizes_norms_and_diagonals():
     """With S_X = (h/a)^(1/4), the rescaled column energy a_j s_j^2 equals the rescaled
