@@ -46,6 +46,8 @@ def parse():
                     help="token chunk of the H_X accumulation (0: one call)")
     ap.add_argument("--g-chunk-tokens", type=int, default=32768,
                     help="token chunk of the H_G accumulation (0: one call)")
+    ap.add_argument("--trailing", default="fp32", choices=["fp32", "3xtf32"],
+                    help="sweep trailing update: fp32-ordered SIMT (bit-exact) or 3xTF32 tensor cores")
     return ap.parse_args()
 
 
@@ -55,10 +57,10 @@ def workload_name(cfg) -> str:
             f"damp {cfg.damp}")
 
 
-def config_dict(cfg, x_chunk: int = 0, g_chunk: int = 0) -> dict:
+def config_dict(cfg, x_chunk: int = 0, g_chunk: int = 0, trailing: str = "fp32") -> dict:
     return {"workload": workload_name(cfg), "d_out": cfg.d_out, "d_in": cfg.d_in, "T": cfg.T,
             "bits": cfg.bits, "group": cfg.group, "block": cfg.block, "damp": cfg.damp,
-            "factor_chunk_tokens": {"X": x_chunk, "G": g_chunk},
+            "factor_chunk_tokens": {"X": x_chunk, "G": g_chunk}, "sweep_trailing_update": trailing,
             "l2": "inputs larger than L2 (X and G are T x d bf16, >= 1 GiB each); no flush"}
 
 
@@ -227,7 +229,7 @@ def run_reference(args):
     out = {"impl": "reference", "metric": METRIC, "value": v, "unit": "ms", "n_gpus": args.gpus,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": v, "higher_is_better": False,
            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-           "config": config_dict(cfg, args.x_chunk_tokens, args.g_chunk_tokens),
+           "config": config_dict(cfg, args.x_chunk_tokens, args.g_chunk_tokens, args.trailing),
            "cpu_baseline": {"value": v, "unit": "ms", "cores": last["cores"], "kind": "oracle",
                             "sample": last["sample"], "stages_ms": last["stages_ms"]},
            "e2e": {"value": v, "unit": "ms", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -249,7 +251,8 @@ def run_ours(args):
     cfg = kqsynth.CONFIGS[args.config].replace(seed=rank)
     inp = kqsynth.device_layer(cfg, device=dev)
     p = LayerPipeline(cfg.d_out, cfg.d_in, cfg.bits, cfg.group, cfg.block, cfg.damp, device=dev,
-                      x_chunk_tokens=args.x_chunk_tokens, g_chunk_tokens=args.g_chunk_tokens)
+                      x_chunk_tokens=args.x_chunk_tokens, g_chunk_tokens=args.g_chunk_tokens,
+                      trailing=args.trailing)
     stream = torch.cuda.current_stream()
 
     def barrier():
@@ -355,7 +358,7 @@ def run_ours(args):
                "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
                "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
                "dtype": "bf16 products, f32 accumulate/arithmetic", "data": "synthetic",
-               "config": config_dict(cfg, args.x_chunk_tokens, args.g_chunk_tokens), "stages_ms": stage_ms, "tflops": tflops,
+               "config": config_dict(cfg, args.x_chunk_tokens, args.g_chunk_tokens, args.trailing), "stages_ms": stage_ms, "tflops": tflops,
                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
                "launch_mode": "cuda graph replay (one graph per layer, two streams)" if graph is not None
                else "direct launches (two streams)",

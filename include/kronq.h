@@ -211,17 +211,28 @@ KQ_API kq_status kq_chol_inv_noalloc(const float* H, int64_t n, float damp_rel, 
  *   Outputs: codes [d_out x d_in] uint8; scale fp32 and zero int32 as above; col_loss
  *   [d_in] (nullable) = sum over rows of E_j^2; pre_q [d_out x d_in] (nullable) = the value
  *   w_j just before it was quantized.
- *   Every fp32 operation and its order are fixed (IEEE division, rintf, one fmaf per
- *   intra-block update; trailing update as acc = fmaf(E_k, R_kc, acc) over ascending k,
- *   then w_c - acc), so results are reproducible bit for bit.
+ *   mode selects the arithmetic of the lazy trailing update (the column loop is the same):
+ *   KQ_TRAIL_FP32: every fp32 operation and its order are fixed (IEEE division, rintf, one
+ *     fmaf per intra-block update; trailing update as acc = fmaf(E_k, R_kc, acc) over
+ *     ascending k, then w_c - acc), so results are reproducible bit for bit and equal to
+ *     the fp32-ordered definition.
+ *   KQ_TRAIL_3XTF32: the trailing update runs on the tensor cores with the 3xTF32 split
+ *     (E R ~= E_hi R_hi + E_hi R_lo + E_lo R_hi, hi = rounded to tf32, lo = the exact
+ *     remainder; fp32 accumulation). Its sums differ from the fp32 order in the last bits,
+ *     so a code can differ from the fp32-ordered definition where w / scale falls on a
+ *     rounding tie, and the rest of that row then follows a slightly different error path.
+ *     Needs d_in % 4 == 0 and a 16-byte aligned W.
  *   Requirements: 1 <= bits <= 8, block == 128, group in {0, block}.
- *   ws: kq_obs_quantize_workspace(d_out, d_in, block) bytes.
+ *   info (nullable, device int): -KQ_ERR_TIMEOUT if a tensor-core pipeline wait gave up.
+ *   ws: kq_obs_quantize_workspace(d_out, d_in, block, mode) bytes, 256-byte aligned.
  * ---------------------------------------------------------------------------------- */
-KQ_API size_t kq_obs_quantize_workspace(int64_t d_out, int64_t d_in, int block);
+#define KQ_TRAIL_FP32 0
+#define KQ_TRAIL_3XTF32 1
+KQ_API size_t kq_obs_quantize_workspace(int64_t d_out, int64_t d_in, int block, int mode);
 KQ_API kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, const float* Lt, int bits,
-                          int group, int block, uint8_t* codes, float* scale, int32_t* zero,
-                          float* col_loss, float* pre_q, void* ws, size_t ws_bytes,
-                          kq_stream_t stream);
+                                 int group, int block, int mode, uint8_t* codes, float* scale, int32_t* zero,
+                                 float* col_loss, float* pre_q, int* info, void* ws, size_t ws_bytes,
+                                 kq_stream_t stream);
 
 /* ------------------------------------------------------------------------------------
  * Check-only calls (not part of the timed path).

@@ -22,6 +22,7 @@
 #include "kq_common.cuh"
 #include "tile_gemm.cuh"
 #include "sumsq.cuh"
+#include "trail_tc.cuh"
 
 namespace kq {
 namespace {
@@ -159,7 +160,7 @@ __global__ void __launch_bounds__(OBS_THREADS, 3) obs_block_kernel(
     const float* __restrict__ W, int64_t d_out, int64_t d_in, const float* __restrict__ Rp, int64_t i0,
     int bits, int group, const float* __restrict__ gscale, const float* __restrict__ gzero,
     uint8_t* __restrict__ codes, float* __restrict__ scale, int32_t* __restrict__ zero,
-    float* __restrict__ E, float* __restrict__ pre_q) {
+    float* __restrict__ E, float* __restrict__ pre_q, float* __restrict__ Eh, float* __restrict__ El) {
     extern __shared__ __align__(16) float Rs[];   // [BLK][BLK], packed (pack_r_kernel)
     for (int e = threadIdx.x; e < BLK * BLK / 4; e += blockDim.x) cp_async16(Rs + 4 * e, Rp + 4 * e, 16);
     cp_async_commit();
@@ -247,12 +248,30 @@ __global__ void __launch_bounds__(OBS_THREADS, 3) obs_block_kernel(
                     } else {
                         *reinterpret_cast<uint2*>(codes + ob) = make_uint2(cq[0], cq[1]);
                     }
+                    if (Eh) {   // tensor-core trailing update: E = E_hi + E_lo
+#pragma unroll
+                        for (int v = 0; v < NV; ++v) {
+                            float h[4], l[4];
+#pragma unroll
+                            for (int t = 0; t < 4; ++t) {
+                                h[t] = tf32_hi(e[4 * v + t]);
+                                l[t] = e[4 * v + t] - h[t];
+                            }
+                            reinterpret_cast<float4*>(Eh + ob)[v] = make_float4(h[0], h[1], h[2], h[3]);
+                            reinterpret_cast<float4*>(El + ob)[v] = make_float4(l[0], l[1], l[2], l[3]);
+                        }
+                    }
                 } else {
 #pragma unroll
                     for (int t = 0; t < CPL; ++t)
                         if (CPL * o + t < nb) {
                             E[ob + t] = e[t];
                             codes[ob + t] = static_cast<uint8_t>(cq[t >> 2] >> (8 * (t & 3)));
+                            if (Eh) {
+                                const float h = tf32_hi(e[t]);
+                                Eh[ob + t] = h;
+                                El[ob + t] = e[t] - h;
+                            }
                         }
                 }
             }
@@ -311,14 +330,43 @@ struct ObsWs {
     float* E;       // d_out x d_in
     float* gscale;  // d_out
     float* gzero;   // d_out
+    float* Eh;      // tensor-core mode: E_hi, E_lo [d_out x d_in], Lt_hi, Lt_lo [d_in x d_in]
+    float* El;
+    float* Lh;
+    float* Ll;
 };
 
-ObsWs carve(void* ws, int64_t d_out, int64_t d_in) {
+inline size_t align256(size_t b) { return (b + 255) & ~static_cast<size_t>(255); }
+
+size_t ws_base_bytes(int64_t d_out, int64_t d_in) {
+    return align256((static_cast<size_t>(cdiv(d_in, BLK)) * BLK * BLK + static_cast<size_t>(d_out) * d_in +
+                     2 * static_cast<size_t>(d_out)) * sizeof(float));
+}
+
+size_t ws_bytes_of(int64_t d_out, int64_t d_in, int mode) {
+    size_t b = ws_base_bytes(d_out, d_in);
+    if (mode == KQ_TRAIL_3XTF32)
+        b += 2 * align256(static_cast<size_t>(d_out) * d_in * sizeof(float)) +
+             2 * align256(static_cast<size_t>(d_in) * d_in * sizeof(float));
+    return b + 256;
+}
+
+ObsWs carve(void* ws, int64_t d_out, int64_t d_in, int mode) {
     ObsWs o;
     o.Rp = static_cast<float*>(ws);
     o.E = o.Rp + cdiv(d_in, BLK) * BLK * BLK;
     o.gscale = o.E + d_out * d_in;
     o.gzero = o.gscale + d_out;
+    o.Eh = o.El = o.Lh = o.Ll = nullptr;
+    if (mode == KQ_TRAIL_3XTF32) {
+        uint8_t* p = static_cast<uint8_t*>(ws) + ws_base_bytes(d_out, d_in);
+        const size_t eb = align256(static_cast<size_t>(d_out) * d_in * sizeof(float));
+        const size_t lb = align256(static_cast<size_t>(d_in) * d_in * sizeof(float));
+        o.Eh = reinterpret_cast<float*>(p);
+        o.El = reinterpret_cast<float*>(p + eb);
+        o.Lh = reinterpret_cast<float*>(p + 2 * eb);
+        o.Ll = reinterpret_cast<float*>(p + 2 * eb + lb);
+    }
     return o;
 }
 
@@ -327,16 +375,15 @@ ObsWs carve(void* ws, int64_t d_out, int64_t d_in) {
 
 using namespace kq;
 
-extern "C" size_t kq_obs_quantize_workspace(int64_t d_out, int64_t d_in, int block) {
+extern "C" size_t kq_obs_quantize_workspace(int64_t d_out, int64_t d_in, int block, int mode) {
     (void)block;
-    if (d_out < 1 || d_in < 1) return 0;
-    return (static_cast<size_t>(cdiv(d_in, BLK)) * BLK * BLK + static_cast<size_t>(d_out) * d_in +
-            2 * static_cast<size_t>(d_out)) * sizeof(float) + 256;
+    if (d_out < 1 || d_in < 1 || (mode != KQ_TRAIL_FP32 && mode != KQ_TRAIL_3XTF32)) return 0;
+    return ws_bytes_of(d_out, d_in, mode);
 }
 
 extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, const float* Lt, int bits,
-                                     int group, int block, uint8_t* codes, float* scale, int32_t* zero,
-                                     float* col_loss, float* pre_q, void* ws, size_t ws_bytes,
+                                     int group, int block, int mode, uint8_t* codes, float* scale, int32_t* zero,
+                                     float* col_loss, float* pre_q, int* info, void* ws, size_t ws_bytes,
                                      kq_stream_t stream_) {
     cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
     if (!W || !Lt || !codes || !scale || !zero || d_out < 1 || d_in < 1 || bits < 1 || bits > 8) {
@@ -347,10 +394,18 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
         set_error("kq_obs_quantize: block must be %d and group 0 or equal to block", BLK);
         return KQ_ERR_UNSUPPORTED;
     }
-    if (!ws || ws_bytes < kq_obs_quantize_workspace(d_out, d_in, block) ||
-        (reinterpret_cast<uintptr_t>(ws) & 15u)) {
-        set_error("kq_obs_quantize: workspace must be 16-byte aligned and hold %zu bytes",
-                  kq_obs_quantize_workspace(d_out, d_in, block));
+    if (mode != KQ_TRAIL_FP32 && mode != KQ_TRAIL_3XTF32) {
+        set_error("kq_obs_quantize: unknown trailing-update mode %d", mode);
+        return KQ_ERR_INVALID_ARG;
+    }
+    const bool tc = mode == KQ_TRAIL_3XTF32;
+    if (tc && ((d_in % 4) != 0 || (reinterpret_cast<uintptr_t>(W) & 15u) != 0)) {
+        set_error("kq_obs_quantize: the tensor-core trailing update needs d_in %% 4 == 0 and a 16-byte aligned W");
+        return KQ_ERR_UNSUPPORTED;
+    }
+    if (!ws || ws_bytes < ws_bytes_of(d_out, d_in, mode) || (reinterpret_cast<uintptr_t>(ws) & 255u)) {
+        set_error("kq_obs_quantize: workspace must be 256-byte aligned and hold %zu bytes",
+                  ws_bytes_of(d_out, d_in, mode));
         return KQ_ERR_WORKSPACE;
     }
     static bool attr = false;
@@ -365,7 +420,13 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
                                      static_cast<int>(G_SMEM)));
         attr = true;
     }
-    ObsWs o = carve(ws, d_out, d_in);
+    ObsWs o = carve(ws, d_out, d_in, mode);
+    TrailMaps maps;
+    if (tc) {
+        kq_status st0 = split_tf32(Lt, d_in * d_in, o.Lh, o.Ll, stream);
+        if (st0 != KQ_OK) return st0;
+        if ((st0 = maps.init(o.Eh, o.El, o.Lh, o.Ll, d_out, d_in)) != KQ_OK) return st0;
+    }
     if (group == 0) {
         rowgrid_kernel<<<static_cast<unsigned>(cdiv(d_out, 8)), 256, 0, stream>>>(W, d_out, d_in, bits, scale,
                                                                                 zero, o.gscale, o.gzero);
@@ -386,6 +447,7 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
     SideStream* side = nblk > 2 ? side_stream(stream) : nullptr;
     bool forked = false;
     auto trailing = [&](int64_t i0, int kb, int64_t cb, int64_t ce, cudaStream_t st) -> kq_status {
+        if (tc) return trail_tc(maps, W, d_out, d_in, i0, cb, ce, info, st);
         dim3 grid(static_cast<unsigned>(cdiv(ce - cb, GT)), static_cast<unsigned>(cdiv(d_out, GT)));
         if (vec)
             trailing_kernel<true><<<grid, G_THREADS, G_SMEM, st>>>(W, o.E, Lt, d_out, d_in, i0, kb, cb, ce);
@@ -399,10 +461,10 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
         const float* rp = o.Rp + (i0 / BLK) * BLK * BLK;
         if (bvec)
             obs_block_kernel<true><<<static_cast<unsigned>(row_ctas), OBS_THREADS, BLK * BLK * 4, stream>>>(
-                W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q);
+                W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q, o.Eh, o.El);
         else
             obs_block_kernel<false><<<static_cast<unsigned>(row_ctas), OBS_THREADS, BLK * BLK * 4, stream>>>(
-                W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q);
+                W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q, o.Eh, o.El);
         KQ_LAUNCH_CHECK("obs_block_kernel");
         const int64_t nb0 = i0 + kb;                                // next block column
         if (nb0 >= d_in) break;

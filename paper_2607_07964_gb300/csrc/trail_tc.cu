@@ -1,0 +1,296 @@
+// Stage 4, tensor-core variant of the OBS sweep's lazy trailing update (Algorithm 2):
+//   W[:, cols] -= E_blk R_blk,   E_blk = E[:, i0:i0+128], R_blk[k][c] = Lt[c][i0 + k],
+// on the 5th-generation tensor cores with fp32-accurate products from the 3xTF32 split
+// (Markidis et al. 2018; Ootomo & Yokota 2022): with x_hi = x rounded to tf32 and
+// x_lo = x - x_hi (exact in fp32),  E R ~= E_hi R_hi + E_hi R_lo + E_lo R_hi, accumulated in
+// fp32 in TMEM. The dropped E_lo R_lo term and the tf32 truncation of the lo parts are
+// ~2^-22 of each product.
+//
+// One CTA per 128 x BN output tile, K = 128 in four 32-wide slabs through a 2-stage ring:
+//   warp 0: TMA loads of E_hi, E_lo (128 rows x 32 k) and Lt_hi, Lt_lo (BN rows x 32 k),
+//           K-major with 128-byte swizzle (a 32-float row is one swizzle atom);
+//   warp 1: allocates BN TMEM columns, issues tcgen05.mma kind::tf32 (M 128, N BN, K 8),
+//           three per k step, into one fp32 accumulator;
+//   warps 2..5: read the accumulator (one row per thread) and update W in place for the
+//           rows < d_out and columns in [cb, ce).
+// Every mbarrier wait is bounded; a timeout sets -KQ_ERR_TIMEOUT in *info and the CTA
+// drains its copies and MMAs before it exits.
+#include <algorithm>
+#include <cstring>
+
+#include "trail_tc.cuh"
+
+namespace kq {
+namespace {
+
+constexpr int TBM = 128;                 // rows per tile (MMA M, TMEM lanes)
+constexpr int TBK = 32;                  // k per slab (one 128-byte swizzle row)
+constexpr int TK = 128;                  // block size: the K of every trailing update
+constexpr int TNSLAB = TK / TBK;         // 4
+constexpr int TSTAGES = 2;
+constexpr int T_THREADS = 192;           // 6 warps
+constexpr int A_SLAB = TBM * TBK * 4;    // 16 KB
+
+template <int BN>
+struct TrailCfg {
+    static constexpr int B_SLAB = BN * TBK * 4;                    // 16 or 32 KB
+    static constexpr int STAGE = 2 * A_SLAB + 2 * B_SLAB;          // hi + lo of both
+    static constexpr int SMEM = TSTAGES * STAGE + 1024 + 256;
+};
+
+// Instruction descriptor, kind::tf32: fp32 accumulator, tf32 A and B, both K-major.
+__host__ __device__ constexpr uint32_t idesc_tf32_k_major(int M, int N) {
+    return (1u << 4)                                // D format: f32
+           | (2u << 7)                              // A format: tf32
+           | (2u << 10)                             // B format: tf32
+           | (static_cast<uint32_t>(N >> 3) << 17)  // N / 8
+           | (static_cast<uint32_t>(M >> 4) << 24); // M / 16
+}
+
+__device__ __forceinline__ void tc_mma_tf32(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                            uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+__device__ __forceinline__ bool wait_quiet(uint64_t* bar, uint32_t parity) {
+    int dummy = 0;
+    return mbar_wait(bar, parity, &dummy);
+}
+
+template <int BN>
+__global__ void __launch_bounds__(T_THREADS, 1)
+trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__ CUtensorMap mEl,
+                const __grid_constant__ CUtensorMap mRh, const __grid_constant__ CUtensorMap mRl,
+                float* __restrict__ W, int64_t d_out, int64_t d_in, int i0, int64_t cb, int64_t ce, int* info) {
+    using C = TrailCfg<BN>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + TSTAGES * C::STAGE);
+    uint64_t* empty = full + TSTAGES;
+    uint64_t* mma_done = empty + TSTAGES;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int64_t r0 = static_cast<int64_t>(blockIdx.y) * TBM;
+    const int64_t c0 = cb + static_cast<int64_t>(blockIdx.x) * BN;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < TSTAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        mbar_init(mma_done, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(tmem_slot, BN);
+        tmem_relinquish();
+    }
+    if (warp == 0 && lane == 0) {
+        tma_prefetch_desc(&mEh);
+        tma_prefetch_desc(&mEl);
+        tma_prefetch_desc(&mRh);
+        tma_prefetch_desc(&mRl);
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            int issued = 0;
+            for (int s = 0; s < TNSLAB; ++s) {
+                const int st = s % TSTAGES;
+                const uint32_t u = static_cast<uint32_t>(s / TSTAGES);
+                if (!mbar_wait(&empty[st], (u & 1u) ^ 1u, abort_flag)) break;
+                mbar_arrive_expect_tx(&full[st], C::STAGE);
+                uint8_t* base = smem + st * C::STAGE;
+                const int x = i0 + s * TBK;
+                tma_load_2d(base, &mEh, &full[st], x, static_cast<int>(r0));
+                tma_load_2d(base + A_SLAB, &mEl, &full[st], x, static_cast<int>(r0));
+                tma_load_2d(base + 2 * A_SLAB, &mRh, &full[st], x, static_cast<int>(c0));
+                tma_load_2d(base + 2 * A_SLAB + C::B_SLAB, &mRl, &full[st], x, static_cast<int>(c0));
+                issued = s + 1;
+            }
+            for (int s = (issued > TSTAGES ? issued - TSTAGES : 0); s < issued; ++s)
+                wait_quiet(&full[s % TSTAGES], static_cast<uint32_t>(s / TSTAGES) & 1u);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_tf32_k_major(TBM, BN);
+            for (int s = 0; s < TNSLAB; ++s) {
+                const int st = s % TSTAGES;
+                if (!mbar_wait(&full[st], static_cast<uint32_t>(s / TSTAGES) & 1u, abort_flag)) break;
+                tc_fence_after();
+                const uint32_t a_hi = smem_u32(smem + st * C::STAGE);
+                const uint32_t a_lo = a_hi + A_SLAB;
+                const uint32_t b_hi = a_hi + 2 * A_SLAB;
+                const uint32_t b_lo = b_hi + C::B_SLAB;
+#pragma unroll
+                for (int k = 0; k < TBK / 8; ++k) {   // 8 tf32 = 32 bytes per MMA
+                    const uint32_t ko = static_cast<uint32_t>(k * 32);
+                    const uint64_t dah = smem_desc_sw128(a_hi + ko, 16, 1024);
+                    const uint64_t dal = smem_desc_sw128(a_lo + ko, 16, 1024);
+                    const uint64_t dbh = smem_desc_sw128(b_hi + ko, 16, 1024);
+                    const uint64_t dbl = smem_desc_sw128(b_lo + ko, 16, 1024);
+                    tc_mma_tf32(tmem, dal, dbh, idesc, (s > 0 || k > 0) ? 1u : 0u);
+                    tc_mma_tf32(tmem, dah, dbl, idesc, 1u);
+                    tc_mma_tf32(tmem, dah, dbh, idesc, 1u);
+                }
+                tc_commit(&empty[st]);
+            }
+            tc_commit(mma_done);
+            wait_quiet(mma_done, 0);
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue (4 warps)
+        const int q = warp & 3;
+        const int64_t row = r0 + q * 32 + lane;
+        bool ok = mbar_wait(mma_done, 0, abort_flag);
+        ok = __all_sync(0xffffffffu, ok) && !*abort_flag;
+        if (ok) {
+            tc_fence_after();
+            float* wrow = W + row * d_in;
+            const bool live = row < d_out;
+#pragma unroll 1
+            for (int p = 0; p < BN / 32; ++p) {
+                float v[32];
+                tmem_ld32(tmem + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(p * 32), v);
+                tc_wait_ld();
+                const int64_t cp = c0 + p * 32;
+                if (!live) continue;
+                if (cp + 32 <= ce && (d_in & 3) == 0) {
+                    float4* w4 = reinterpret_cast<float4*>(wrow + cp);
+                    float4 o[8];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) o[i] = w4[i];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i)
+                        w4[i] = make_float4(o[i].x - v[4 * i], o[i].y - v[4 * i + 1], o[i].z - v[4 * i + 2],
+                                            o[i].w - v[4 * i + 3]);
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i)
+                        if (cp + i < ce) wrow[cp + i] -= v[i];
+                }
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (*abort_flag && threadIdx.x == 0) record_error(info, -KQ_ERR_TIMEOUT);
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, BN);
+    }
+}
+
+__global__ void split_tf32_kernel(const float* __restrict__ src, int64_t n, float* __restrict__ hi,
+                                  float* __restrict__ lo) {
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const float x = src[i];
+        const float h = tf32_hi(x);
+        hi[i] = h;
+        lo[i] = x - h;
+    }
+}
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_tiled() {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    }
+    return fn;
+}
+
+// 2-D fp32 tensor map over a row-major [rows x cols] matrix, box = box_rows x 32 columns.
+kq_status make_map(CUtensorMap* m, const float* base, int64_t rows, int64_t cols, int box_rows) {
+    EncodeTiledFn enc = encode_tiled();
+    if (!enc) {
+        set_error("trailing update: cuTensorMapEncodeTiled is unavailable");
+        return KQ_ERR_CUDA;
+    }
+    std::memset(m, 0, sizeof(*m));
+    cuuint64_t gdim[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+    cuuint64_t gstride[1] = {static_cast<cuuint64_t>(cols) * 4};
+    cuuint32_t box[2] = {static_cast<cuuint32_t>(TBK), static_cast<cuuint32_t>(box_rows)};
+    cuuint32_t estride[2] = {1, 1};
+    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(base), gdim, gstride, box, estride,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+        set_error("trailing update: cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
+        return KQ_ERR_CUDA;
+    }
+    return KQ_OK;
+}
+
+}  // namespace
+
+kq_status split_tf32(const float* src, int64_t n, float* hi, float* lo, cudaStream_t stream) {
+    const int64_t grid = std::min<int64_t>(cdiv(n, 256), static_cast<int64_t>(num_sms()) * 16);
+    split_tf32_kernel<<<static_cast<unsigned>(std::max<int64_t>(grid, 1)), 256, 0, stream>>>(src, n, hi, lo);
+    KQ_LAUNCH_CHECK("split_tf32_kernel");
+    return KQ_OK;
+}
+
+kq_status TrailMaps::init(const float* E_hi, const float* E_lo, const float* Lt_hi, const float* Lt_lo,
+                          int64_t d_out, int64_t d_in) {
+    kq_status st;
+    if ((st = make_map(&eh, E_hi, d_out, d_in, TBM)) != KQ_OK) return st;
+    if ((st = make_map(&el, E_lo, d_out, d_in, TBM)) != KQ_OK) return st;
+    if ((st = make_map(&rh_wide, Lt_hi, d_in, d_in, 256)) != KQ_OK) return st;
+    if ((st = make_map(&rl_wide, Lt_lo, d_in, d_in, 256)) != KQ_OK) return st;
+    if ((st = make_map(&rh_narrow, Lt_hi, d_in, d_in, 128)) != KQ_OK) return st;
+    if ((st = make_map(&rl_narrow, Lt_lo, d_in, d_in, 128)) != KQ_OK) return st;
+    return KQ_OK;
+}
+
+kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, int64_t i0, int64_t cb, int64_t ce,
+                   int* info, cudaStream_t stream) {
+    static bool attr = false;
+    if (!attr) {
+        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     TrailCfg<256>::SMEM));
+        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     TrailCfg<128>::SMEM));
+        attr = true;
+    }
+    const unsigned gy = static_cast<unsigned>(cdiv(d_out, TBM));
+    if (ce - cb <= 128) {
+        dim3 grid(static_cast<unsigned>(cdiv(ce - cb, 128)), gy);
+        trail_tc_kernel<128><<<grid, T_THREADS, TrailCfg<128>::SMEM, stream>>>(
+            m.eh, m.el, m.rh_narrow, m.rl_narrow, W, d_out, d_in, static_cast<int>(i0), cb, ce, info);
+    } else {
+        dim3 grid(static_cast<unsigned>(cdiv(ce - cb, 256)), gy);
+        trail_tc_kernel<256><<<grid, T_THREADS, TrailCfg<256>::SMEM, stream>>>(
+            m.eh, m.el, m.rh_wide, m.rl_wide, W, d_out, d_in, static_cast<int>(i0), cb, ce, info);
+    }
+    KQ_LAUNCH_CHECK("trail_tc_kernel");
+    return KQ_OK;
+}
+
+}  // namespace kq

@@ -16,6 +16,7 @@ LIB_PATH = os.path.join(_HERE, "libkronq.so")
 KQ_OK, KQ_ERR_INVALID_ARG, KQ_ERR_UNSUPPORTED, KQ_ERR_NOT_PD = 0, 1, 2, 3
 KQ_ERR_CUDA, KQ_ERR_TIMEOUT, KQ_ERR_WORKSPACE = 4, 5, 6
 KQ_FWD, KQ_INV = 0, 1
+KQ_TRAIL_FP32, KQ_TRAIL_3XTF32 = 0, 1
 KQ_SYRK_CHUNK_TOKENS = 512
 
 _lib = None
@@ -54,8 +55,8 @@ def lib() -> ctypes.CDLL:
             "kq_chol_inv_workspace": ([I64], SZ),
             "kq_chol_inv": ([P, I64, F, P, P, P, SZ, P], I),
             "kq_chol_inv_noalloc": ([P, I64, F, P, P, P], I),
-            "kq_obs_quantize_workspace": ([I64, I64, I], SZ),
-            "kq_obs_quantize": ([P, I64, I64, P, I, I, I, P, P, P, P, P, P, SZ, P], I),
+            "kq_obs_quantize_workspace": ([I64, I64, I, I], SZ),
+            "kq_obs_quantize": ([P, I64, I64, P, I, I, I, I, P, P, P, P, P, P, P, SZ, P], I),
             "kq_dequant_revert": ([P, P, P, I64, I64, I, P, P, P, P, P, P], I),
             "kq_proxy_loss_workspace": ([I64, I64], SZ),
             "kq_proxy_loss": ([P, P, I64, I64, P, P, P, P, SZ, P], I),
@@ -253,12 +254,13 @@ def kq_chol_inv_noalloc(H, damp_rel: float, Lt, info=None, stream=None) -> None:
         "kq_chol_inv_noalloc")
 
 
-def kq_obs_quantize_workspace(d_out: int, d_in: int, block: int = 128) -> int:
-    return int(lib().kq_obs_quantize_workspace(d_out, d_in, block))
+def kq_obs_quantize_workspace(d_out: int, d_in: int, block: int = 128, mode: int = KQ_TRAIL_FP32) -> int:
+    return int(lib().kq_obs_quantize_workspace(d_out, d_in, block, mode))
 
 
 def kq_obs_quantize(W, Lt, bits: int, group: int, block: int, codes, scale, zero, col_loss=None,
-                    pre_q=None, ws=None, stream=None) -> None:
+                    pre_q=None, ws=None, stream=None, mode: int = KQ_TRAIL_FP32, info=None) -> None:
+    """mode: KQ_TRAIL_FP32 (fp32-ordered trailing update, bit-exact) or KQ_TRAIL_3XTF32."""
     d_out, d_in = W.shape
     ng = 1 if group == 0 else -(-d_in // group)
     _need(W, "W", torch.float32)
@@ -269,8 +271,9 @@ def kq_obs_quantize(W, Lt, bits: int, group: int, block: int, codes, scale, zero
     _need(col_loss, "col_loss", torch.float32, (d_in,))
     _need(pre_q, "pre_q", torch.float32, (d_out, d_in))
     _need(ws, "ws", torch.uint8)
-    _ok(lib().kq_obs_quantize(_ptr(W), d_out, d_in, _ptr(Lt), bits, group, block, _ptr(codes),
-                              _ptr(scale), _ptr(zero), _ptr(col_loss), _ptr(pre_q), _ptr(ws),
+    _need(info, "info", torch.int32)
+    _ok(lib().kq_obs_quantize(_ptr(W), d_out, d_in, _ptr(Lt), bits, group, block, mode, _ptr(codes),
+                              _ptr(scale), _ptr(zero), _ptr(col_loss), _ptr(pre_q), _ptr(info), _ptr(ws),
                               0 if ws is None else ws.numel(), _stream(stream)), "kq_obs_quantize")
 
 

@@ -17,7 +17,8 @@ class LayerPipeline:
 
     def __init__(self, d_out: int, d_in: int, bits: int, group: int, block: int = 128,
                  damp: float = 0.01, device: str = "cuda", want_col_loss: bool = True,
-                 overlap: bool = True, x_chunk_tokens: int = 0, g_chunk_tokens: int = 32768):
+                 overlap: bool = True, x_chunk_tokens: int = 0, g_chunk_tokens: int = 32768,
+                 trailing: str = "fp32"):
         self.d_out, self.d_in, self.bits, self.group, self.block, self.damp = d_out, d_in, bits, group, block, damp
         f32 = dict(dtype=torch.float32, device=device)
         ng = 1 if group == 0 else -(-d_in // group)
@@ -36,7 +37,10 @@ class LayerPipeline:
         self.trace_g = torch.zeros((1,), dtype=torch.float64, device=device)
         self.info = torch.zeros((4,), dtype=torch.int32, device=device)
         self.ws_chol = torch.empty((kq.kq_chol_inv_workspace(d_in),), dtype=torch.uint8, device=device)
-        self.ws_obs = torch.empty((kq.kq_obs_quantize_workspace(d_out, d_in, block),), dtype=torch.uint8,
+        # the sweep's lazy trailing update: "fp32" (the fp32-ordered definition, bit-exact) or
+        # "3xtf32" (tensor cores, 3xTF32 split)
+        self.trail_mode = {"fp32": kq.KQ_TRAIL_FP32, "3xtf32": kq.KQ_TRAIL_3XTF32}[trailing]
+        self.ws_obs = torch.empty((kq.kq_obs_quantize_workspace(d_out, d_in, block, self.trail_mode),), dtype=torch.uint8,
                                   device=device)
         # Output-side work (H_G, S_G, U) runs on a second stream beside the Cholesky, which
         # needs only H_X and leaves most SMs idle during its diagonal steps.
@@ -103,7 +107,8 @@ class LayerPipeline:
         kq.kq_chol_inv(self.HX, self.damp, self.Lt, self.info[1:2], self.ws_chol, stream=s)  # Alg. 2
         mark(5)
         kq.kq_obs_quantize(self.Wp, self.Lt, self.bits, self.group, self.block, self.codes, self.scale,
-                           self.zero, self.col_loss, None, self.ws_obs, stream=s)   # Alg. 2 sweep
+                           self.zero, self.col_loss, None, self.ws_obs, stream=s, mode=self.trail_mode,
+                           info=self.info[3:4])   # Alg. 2 sweep
         mark(6)
 
     def _run_overlapped(self, X, G, W, sign_u, sign_v, caller, x_ready=None, g_ready=None, w_ready=None) -> None:
@@ -142,7 +147,8 @@ class LayerPipeline:
         e_hg.record(s2)
         s.wait_event(e_side)
         kq.kq_obs_quantize(self.Wp, self.Lt, self.bits, self.group, self.block, self.codes, self.scale,
-                           self.zero, self.col_loss, None, self.ws_obs, stream=s)
+                           self.zero, self.col_loss, None, self.ws_obs, stream=s, mode=self.trail_mode,
+                           info=self.info[3:4])
         e_out.record(s)
         caller.wait_event(e_out)
         caller.wait_event(e_hg)
@@ -164,7 +170,7 @@ class LayerPipeline:
         if self.side is not None:
             self.side.synchronize()
             self.main.synchronize()
-        for k in range(3):
+        for k in range(4):
             st, raw = kq.kq_check(self.info[k:k + 1], reset=True, stream=stream)
             if st != kq.KQ_OK:
                 raise kq.KronqError(st, "pipeline", f"device word {raw}")

@@ -49,6 +49,8 @@ def test_workspace_queries(lib):
     assert kronq.kq_chol_inv_workspace(200) >= 2 * 256 * 256 * 4   # padded to the block size
     assert kronq.kq_chol_inv_workspace(0) == 0
     assert kronq.kq_obs_quantize_workspace(64, 256, 128) >= 64 * 256 * 4
+    assert kronq.kq_obs_quantize_workspace(64, 256, 128, kronq.KQ_TRAIL_3XTF32) >= 3 * 64 * 256 * 4 + 2 * 256 * 256 * 4
+    assert kronq.kq_obs_quantize_workspace(64, 256, 128, 5) == 0
     assert kronq.kq_proxy_loss_workspace(8, 8) >= 3 * 64 * 4
 
 
@@ -68,13 +70,17 @@ def test_host_side_argument_errors(lib):
     assert lib.kq_rotate_out(fake, 100, 4, None, None, fake, 0, None) == K.KQ_ERR_UNSUPPORTED
     assert lib.kq_rotate_in(fake, 4, 28 * 2048, None, None, fake, 0, None) == K.KQ_ERR_UNSUPPORTED
     # sweep: block must be 128 and group in {0, block}
-    args = [fake, 4, 256, fake, 4, 64, 128, fake, fake, fake, None, None, fake, 1 << 30, None]
+    args = [fake, 4, 256, fake, 4, 64, 128, 0, fake, fake, fake, None, None, None, fake, 1 << 30, None]
     assert lib.kq_obs_quantize(*args) == K.KQ_ERR_UNSUPPORTED
     args[6] = 64
     args[5] = 0
     assert lib.kq_obs_quantize(*args) == K.KQ_ERR_UNSUPPORTED
     args[6], args[4] = 128, 9
     assert lib.kq_obs_quantize(*args) == K.KQ_ERR_INVALID_ARG
-    args[4], args[13] = 4, 16
+    args[4], args[7] = 4, 7                       # unknown trailing-update mode
+    assert lib.kq_obs_quantize(*args) == K.KQ_ERR_INVALID_ARG
+    args[7], args[2] = K.KQ_TRAIL_3XTF32, 258     # tensor-core mode needs d_in % 4 == 0
+    assert lib.kq_obs_quantize(*args) == K.KQ_ERR_UNSUPPORTED
+    args[7], args[2], args[15] = 0, 256, 16
     assert lib.kq_obs_quantize(*args) == K.KQ_ERR_WORKSPACE
     assert "workspace" in K.last_error()
