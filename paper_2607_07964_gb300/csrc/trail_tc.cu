@@ -11,8 +11,10 @@
 //           K-major with 128-byte swizzle (a 32-float row is one swizzle atom);
 //   warp 1: allocates BN TMEM columns, issues tcgen05.mma kind::tf32 (M 128, N BN, K 8),
 //           three per k step, into one fp32 accumulator;
-//   warps 2..5: read the accumulator (one row per thread) and update W in place for the
-//           rows < d_out and columns in [cb, ce).
+//   warps 2..9: two per TMEM lane quadrant, each thread one row and BN / 2 columns: they
+//           load their slice of W into registers before the MMAs finish (the loads overlap
+//           the TMA/MMA pipeline), then subtract the accumulator and store, for the rows
+//           < d_out and columns in [cb, ce).
 // Every mbarrier wait is bounded; a timeout sets -KQ_ERR_TIMEOUT in *info and the CTA
 // drains its copies and MMAs before it exits.
 #include <algorithm>
@@ -27,15 +29,14 @@ constexpr int TBM = 128;                 // rows per tile (MMA M, TMEM lanes)
 constexpr int TBK = 32;                  // k per slab (one 128-byte swizzle row)
 constexpr int TK = 128;                  // block size: the K of every trailing update
 constexpr int TNSLAB = TK / TBK;         // 4
-constexpr int TSTAGES = 2;
-constexpr int T_THREADS = 192;           // 6 warps
+constexpr int T_THREADS = 320;           // 10 warps: TMA, MMA, 8 epilogue
 constexpr int A_SLAB = TBM * TBK * 4;    // 16 KB
 
-template <int BN>
+template <int BN, int STAGES>
 struct TrailCfg {
     static constexpr int B_SLAB = BN * TBK * 4;                    // 16 or 32 KB
     static constexpr int STAGE = 2 * A_SLAB + 2 * B_SLAB;          // hi + lo of both
-    static constexpr int SMEM = TSTAGES * STAGE + 1024 + 256;
+    static constexpr int SMEM = STAGES * STAGE + 1024 + 256;
 };
 
 // Instruction descriptor, kind::tf32: fp32 accumulator, tf32 A and B, both K-major.
@@ -62,12 +63,12 @@ __device__ __forceinline__ bool wait_quiet(uint64_t* bar, uint32_t parity) {
     return mbar_wait(bar, parity, &dummy);
 }
 
-template <int BN>
+template <int BN, int TSTAGES>
 __global__ void __launch_bounds__(T_THREADS, 1)
 trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__ CUtensorMap mEl,
                 const __grid_constant__ CUtensorMap mRh, const __grid_constant__ CUtensorMap mRl,
                 float* __restrict__ W, int64_t d_out, int64_t d_in, int i0, int64_t cb, int64_t ce, int* info) {
-    using C = TrailCfg<BN>;
+    using C = TrailCfg<BN, TSTAGES>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -155,35 +156,41 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
             wait_quiet(mma_done, 0);
         }
     } else {
-        // ------------------------------------------------------------ epilogue (4 warps)
-        const int q = warp & 3;
+        // ------------------------------------------------------------ epilogue (8 warps)
+        constexpr int HALF = BN / 2;            // columns per thread
+        const int q = warp & 3;                 // TMEM lane quadrant this warp may access
+        const int h = (warp - 2) >> 2;          // which half of the columns
         const int64_t row = r0 + q * 32 + lane;
+        const int64_t cs = c0 + h * HALF;       // first column of this thread
+        const bool live = row < d_out;
+        const bool vec = live && cs + HALF <= ce && (d_in & 3) == 0;
+        float* wrow = W + row * d_in + cs;
+        float4 wv[HALF / 4];
+        if (vec) {
+#pragma unroll
+            for (int i = 0; i < HALF / 4; ++i) wv[i] = reinterpret_cast<const float4*>(wrow)[i];
+        }
         bool ok = mbar_wait(mma_done, 0, abort_flag);
         ok = __all_sync(0xffffffffu, ok) && !*abort_flag;
         if (ok) {
             tc_fence_after();
-            float* wrow = W + row * d_in;
-            const bool live = row < d_out;
-#pragma unroll 1
-            for (int p = 0; p < BN / 32; ++p) {
+            const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(h * HALF);
+#pragma unroll
+            for (int p = 0; p < HALF / 32; ++p) {
                 float v[32];
-                tmem_ld32(tmem + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(p * 32), v);
+                tmem_ld32(taddr + static_cast<uint32_t>(p * 32), v);
                 tc_wait_ld();
-                const int64_t cp = c0 + p * 32;
-                if (!live) continue;
-                if (cp + 32 <= ce && (d_in & 3) == 0) {
-                    float4* w4 = reinterpret_cast<float4*>(wrow + cp);
-                    float4 o[8];
+                if (vec) {
 #pragma unroll
-                    for (int i = 0; i < 8; ++i) o[i] = w4[i];
-#pragma unroll
-                    for (int i = 0; i < 8; ++i)
-                        w4[i] = make_float4(o[i].x - v[4 * i], o[i].y - v[4 * i + 1], o[i].z - v[4 * i + 2],
-                                            o[i].w - v[4 * i + 3]);
-                } else {
+                    for (int i = 0; i < 8; ++i) {
+                        const float4 o = wv[8 * p + i];
+                        reinterpret_cast<float4*>(wrow)[8 * p + i] =
+                            make_float4(o.x - v[4 * i], o.y - v[4 * i + 1], o.z - v[4 * i + 2], o.w - v[4 * i + 3]);
+                    }
+                } else if (live) {
 #pragma unroll
                     for (int i = 0; i < 32; ++i)
-                        if (cp + i < ce) wrow[cp + i] -= v[i];
+                        if (cs + 32 * p + i < ce) wrow[32 * p + i] -= v[i];
                 }
             }
         }
@@ -271,22 +278,27 @@ kq_status TrailMaps::init(const float* E_hi, const float* E_lo, const float* Lt_
 
 kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, int64_t i0, int64_t cb, int64_t ce,
                    int* info, cudaStream_t stream) {
+    // The next block column (critical path, few tiles): 128-column tiles, 2-stage ring.
+    // The far columns: 256-column tiles with a 1-stage ring (97 KB), so a tile fits on an SM
+    // beside the next block kernel's CTAs (64 KB each) that run at the same time.
+    using Narrow = TrailCfg<128, 2>;
+    using Wide = TrailCfg<256, 1>;
     static bool attr = false;
     if (!attr) {
-        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     TrailCfg<256>::SMEM));
-        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     TrailCfg<128>::SMEM));
+        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<256, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     Wide::SMEM));
+        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<128, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     Narrow::SMEM));
         attr = true;
     }
     const unsigned gy = static_cast<unsigned>(cdiv(d_out, TBM));
     if (ce - cb <= 128) {
         dim3 grid(static_cast<unsigned>(cdiv(ce - cb, 128)), gy);
-        trail_tc_kernel<128><<<grid, T_THREADS, TrailCfg<128>::SMEM, stream>>>(
+        trail_tc_kernel<128, 2><<<grid, T_THREADS, Narrow::SMEM, stream>>>(
             m.eh, m.el, m.rh_narrow, m.rl_narrow, W, d_out, d_in, static_cast<int>(i0), cb, ce, info);
     } else {
         dim3 grid(static_cast<unsigned>(cdiv(ce - cb, 256)), gy);
-        trail_tc_kernel<256><<<grid, T_THREADS, TrailCfg<256>::SMEM, stream>>>(
+        trail_tc_kernel<256, 1><<<grid, T_THREADS, Wide::SMEM, stream>>>(
             m.eh, m.el, m.rh_wide, m.rl_wide, W, d_out, d_in, static_cast<int>(i0), cb, ce, info);
     }
     KQ_LAUNCH_CHECK("trail_tc_kernel");
