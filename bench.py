@@ -46,7 +46,7 @@ def parse():
                     help="token chunk of the H_X accumulation (0: one call)")
     ap.add_argument("--g-chunk-tokens", type=int, default=32768,
                     help="token chunk of the H_G accumulation (0: one call)")
-    ap.add_argument("--trailing", default="fp32", choices=["fp32", "3xtf32"],
+    ap.add_argument("--trailing", default="3xtf32", choices=["fp32", "3xtf32"],
                     help="sweep trailing update: fp32-ordered SIMT (bit-exact) or 3xTF32 tensor cores")
     return ap.parse_args()
 
@@ -57,7 +57,7 @@ def workload_name(cfg) -> str:
             f"damp {cfg.damp}")
 
 
-def config_dict(cfg, x_chunk: int = 0, g_chunk: int = 0, trailing: str = "fp32") -> dict:
+def config_dict(cfg, x_chunk: int = 0, g_chunk: int = 0, trailing: str = "3xtf32") -> dict:
     return {"workload": workload_name(cfg), "d_out": cfg.d_out, "d_in": cfg.d_in, "T": cfg.T,
             "bits": cfg.bits, "group": cfg.group, "block": cfg.block, "damp": cfg.damp,
             "factor_chunk_tokens": {"X": x_chunk, "G": g_chunk}, "sweep_trailing_update": trailing,

@@ -6,15 +6,17 @@
 // fp32 in TMEM. The dropped E_lo R_lo term and the tf32 truncation of the lo parts are
 // ~2^-22 of each product.
 //
-// One CTA per 128 x BN output tile, K = 128 in four 32-wide slabs through a 2-stage ring:
+// Persistent CTAs (one per SM) walk 128 x BN output tiles, K = 128 in four 32-wide slabs
+// through a 2-stage ring, with two TMEM accumulators so a tile's epilogue overlaps the next
+// tile's loads and MMAs:
 //   warp 0: TMA loads of E_hi, E_lo (128 rows x 32 k) and Lt_hi, Lt_lo (BN rows x 32 k),
 //           K-major with 128-byte swizzle (a 32-float row is one swizzle atom);
-//   warp 1: allocates BN TMEM columns, issues tcgen05.mma kind::tf32 (M 128, N BN, K 8),
-//           three per k step, into one fp32 accumulator;
+//   warp 1: allocates 2 BN TMEM columns, issues tcgen05.mma kind::tf32 (M 128, N BN, K 8),
+//           three per k step, into the accumulator the epilogue has released;
 //   warps 2..9: two per TMEM lane quadrant, each thread one row and BN / 2 columns: they
-//           load their slice of W into registers before the MMAs finish (the loads overlap
-//           the TMA/MMA pipeline), then subtract the accumulator and store, for the rows
-//           < d_out and columns in [cb, ce).
+//           load their slice of W into registers before the tile's MMAs finish (the loads
+//           overlap the TMA/MMA pipeline), then subtract the accumulator and store, for the
+//           rows < d_out and columns in [cb, ce).
 // Every mbarrier wait is bounded; a timeout sets -KQ_ERR_TIMEOUT in *info and the CTA
 // drains its copies and MMAs before it exits.
 #include <algorithm>
@@ -37,6 +39,7 @@ struct TrailCfg {
     static constexpr int B_SLAB = BN * TBK * 4;                    // 16 or 32 KB
     static constexpr int STAGE = 2 * A_SLAB + 2 * B_SLAB;          // hi + lo of both
     static constexpr int SMEM = STAGES * STAGE + 1024 + 256;
+    static_assert(2 * BN <= 512, "two accumulators must fit in TMEM");
 };
 
 // Instruction descriptor, kind::tf32: fp32 accumulator, tf32 A and B, both K-major.
@@ -67,33 +70,38 @@ template <int BN, int TSTAGES>
 __global__ void __launch_bounds__(T_THREADS, 1)
 trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__ CUtensorMap mEl,
                 const __grid_constant__ CUtensorMap mRh, const __grid_constant__ CUtensorMap mRl,
-                float* __restrict__ W, int64_t d_out, int64_t d_in, int i0, int64_t cb, int64_t ce, int* info) {
+                float* __restrict__ W, int64_t d_out, int64_t d_in, int i0, int64_t cb, int64_t ce,
+                int n_col_tiles, int n_tiles, int* info) {
     using C = TrailCfg<BN, TSTAGES>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     uint64_t* full = reinterpret_cast<uint64_t*>(smem + TSTAGES * C::STAGE);
     uint64_t* empty = full + TSTAGES;
-    uint64_t* mma_done = empty + TSTAGES;
+    uint64_t* tfull = empty + TSTAGES;     // accumulator b holds a finished tile
+    uint64_t* tempty = tfull + 2;          // the epilogue has read accumulator b
+    uint64_t* mma_done = tempty + 2;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int64_t r0 = static_cast<int64_t>(blockIdx.y) * TBM;
-    const int64_t c0 = cb + static_cast<int64_t>(blockIdx.x) * BN;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < TSTAGES; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
         }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&tfull[b], 1);
+            mbar_init(&tempty[b], 8);
+        }
         mbar_init(mma_done, 1);
         *abort_flag = 0;
         fence_mbar_init();
     }
     if (warp == 1) {
-        tmem_alloc(tmem_slot, BN);
+        tmem_alloc(tmem_slot, 2 * BN);
         tmem_relinquish();
     }
     if (warp == 0 && lane == 0) {
@@ -110,47 +118,67 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
-            int issued = 0;
-            for (int s = 0; s < TNSLAB; ++s) {
-                const int st = s % TSTAGES;
-                const uint32_t u = static_cast<uint32_t>(s / TSTAGES);
-                if (!mbar_wait(&empty[st], (u & 1u) ^ 1u, abort_flag)) break;
-                mbar_arrive_expect_tx(&full[st], C::STAGE);
-                uint8_t* base = smem + st * C::STAGE;
-                const int x = i0 + s * TBK;
-                tma_load_2d(base, &mEh, &full[st], x, static_cast<int>(r0));
-                tma_load_2d(base + A_SLAB, &mEl, &full[st], x, static_cast<int>(r0));
-                tma_load_2d(base + 2 * A_SLAB, &mRh, &full[st], x, static_cast<int>(c0));
-                tma_load_2d(base + 2 * A_SLAB + C::B_SLAB, &mRl, &full[st], x, static_cast<int>(c0));
-                issued = s + 1;
+            int k = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+                const int r0 = (t / n_col_tiles) * TBM;
+                const int c0 = static_cast<int>(cb) + (t % n_col_tiles) * BN;
+                for (int s = 0; s < TNSLAB; ++s, ++k) {
+                    const int st = k % TSTAGES;
+                    const uint32_t u = static_cast<uint32_t>(k / TSTAGES);
+                    if (!mbar_wait(&empty[st], (u & 1u) ^ 1u, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(&full[st], C::STAGE);
+                    uint8_t* base = smem + st * C::STAGE;
+                    const int x = i0 + s * TBK;
+                    tma_load_2d(base, &mEh, &full[st], x, r0);
+                    tma_load_2d(base + A_SLAB, &mEl, &full[st], x, r0);
+                    tma_load_2d(base + 2 * A_SLAB, &mRh, &full[st], x, c0);
+                    tma_load_2d(base + 2 * A_SLAB + C::B_SLAB, &mRl, &full[st], x, c0);
+                }
             }
-            for (int s = (issued > TSTAGES ? issued - TSTAGES : 0); s < issued; ++s)
-                wait_quiet(&full[s % TSTAGES], static_cast<uint32_t>(s / TSTAGES) & 1u);
+            // every issued load must land before the CTA exits
+            for (int j = (k > TSTAGES ? k - TSTAGES : 0); j < k; ++j)
+                wait_quiet(&full[j % TSTAGES], static_cast<uint32_t>(j / TSTAGES) & 1u);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
             constexpr uint32_t idesc = idesc_tf32_k_major(TBM, BN);
-            for (int s = 0; s < TNSLAB; ++s) {
-                const int st = s % TSTAGES;
-                if (!mbar_wait(&full[st], static_cast<uint32_t>(s / TSTAGES) & 1u, abort_flag)) break;
+            int k = 0, li = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++li) {
+                const int buf = li & 1;
+                if (!mbar_wait(&tempty[buf], ((static_cast<uint32_t>(li) >> 1) & 1u) ^ 1u, abort_flag)) break;
                 tc_fence_after();
-                const uint32_t a_hi = smem_u32(smem + st * C::STAGE);
-                const uint32_t a_lo = a_hi + A_SLAB;
-                const uint32_t b_hi = a_hi + 2 * A_SLAB;
-                const uint32_t b_lo = b_hi + C::B_SLAB;
+                const uint32_t dt = tmem + static_cast<uint32_t>(buf * BN);
+                for (int s = 0; s < TNSLAB; ++s, ++k) {
+                    const int st = k % TSTAGES;
+                    if (!mbar_wait(&full[st], static_cast<uint32_t>(k / TSTAGES) & 1u, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a_hi = smem_u32(smem + st * C::STAGE);
+                    const uint32_t a_lo = a_hi + A_SLAB;
+                    const uint32_t b_hi = a_hi + 2 * A_SLAB;
+                    const uint32_t b_lo = b_hi + C::B_SLAB;
 #pragma unroll
-                for (int k = 0; k < TBK / 8; ++k) {   // 8 tf32 = 32 bytes per MMA
-                    const uint32_t ko = static_cast<uint32_t>(k * 32);
-                    const uint64_t dah = smem_desc_sw128(a_hi + ko, 16, 1024);
-                    const uint64_t dal = smem_desc_sw128(a_lo + ko, 16, 1024);
-                    const uint64_t dbh = smem_desc_sw128(b_hi + ko, 16, 1024);
-                    const uint64_t dbl = smem_desc_sw128(b_lo + ko, 16, 1024);
-                    tc_mma_tf32(tmem, dal, dbh, idesc, (s > 0 || k > 0) ? 1u : 0u);
-                    tc_mma_tf32(tmem, dah, dbl, idesc, 1u);
-                    tc_mma_tf32(tmem, dah, dbh, idesc, 1u);
+                    for (int kk = 0; kk < TBK / 8; ++kk) {   // 8 tf32 = 32 bytes per MMA
+                        const uint32_t ko = static_cast<uint32_t>(kk * 32);
+                        const uint64_t dah = smem_desc_sw128(a_hi + ko, 16, 1024);
+                        const uint64_t dal = smem_desc_sw128(a_lo + ko, 16, 1024);
+                        const uint64_t dbh = smem_desc_sw128(b_hi + ko, 16, 1024);
+                        const uint64_t dbl = smem_desc_sw128(b_lo + ko, 16, 1024);
+                        tc_mma_tf32(dt, dal, dbh, idesc, (s > 0 || kk > 0) ? 1u : 0u);
+                        tc_mma_tf32(dt, dah, dbl, idesc, 1u);
+                        tc_mma_tf32(dt, dah, dbh, idesc, 1u);
+                    }
+                    tc_commit(&empty[st]);
                 }
-                tc_commit(&empty[st]);
+                if (ok) tc_commit(&tfull[buf]);
             }
             tc_commit(mma_done);
             wait_quiet(mma_done, 0);
@@ -160,21 +188,25 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
         constexpr int HALF = BN / 2;            // columns per thread
         const int q = warp & 3;                 // TMEM lane quadrant this warp may access
         const int h = (warp - 2) >> 2;          // which half of the columns
-        const int64_t row = r0 + q * 32 + lane;
-        const int64_t cs = c0 + h * HALF;       // first column of this thread
-        const bool live = row < d_out;
-        const bool vec = live && cs + HALF <= ce && (d_in & 3) == 0;
-        float* wrow = W + row * d_in + cs;
-        float4 wv[HALF / 4];
-        if (vec) {
+        int li = 0;
+        for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++li) {
+            const int buf = li & 1;
+            const int64_t row = static_cast<int64_t>(t / n_col_tiles) * TBM + q * 32 + lane;
+            const int64_t cs = cb + static_cast<int64_t>(t % n_col_tiles) * BN + h * HALF;
+            const bool live = row < d_out;
+            const bool vec = live && cs + HALF <= ce && (d_in & 3) == 0;
+            float* wrow = W + row * d_in + cs;
+            float4 wv[HALF / 4];
+            if (vec) {   // W loads overlap the MMAs of this tile
 #pragma unroll
-            for (int i = 0; i < HALF / 4; ++i) wv[i] = reinterpret_cast<const float4*>(wrow)[i];
-        }
-        bool ok = mbar_wait(mma_done, 0, abort_flag);
-        ok = __all_sync(0xffffffffu, ok) && !*abort_flag;
-        if (ok) {
+                for (int i = 0; i < HALF / 4; ++i) wv[i] = reinterpret_cast<const float4*>(wrow)[i];
+            }
+            bool ok = mbar_wait(&tfull[buf], (static_cast<uint32_t>(li) >> 1) & 1u, abort_flag);
+            ok = __all_sync(0xffffffffu, ok) && !*abort_flag;
+            if (!ok) break;
             tc_fence_after();
-            const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(h * HALF);
+            const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) +
+                                   static_cast<uint32_t>(buf * BN + h * HALF);
 #pragma unroll
             for (int p = 0; p < HALF / 32; ++p) {
                 float v[32];
@@ -193,6 +225,9 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
                         if (cs + 32 * p + i < ce) wrow[32 * p + i] -= v[i];
                 }
             }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty[buf]);
         }
     }
 
@@ -201,7 +236,7 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
     if (*abort_flag && threadIdx.x == 0) record_error(info, -KQ_ERR_TIMEOUT);
     if (warp == 1) {
         tc_fence_after();
-        tmem_dealloc(tmem, BN);
+        tmem_dealloc(tmem, 2 * BN);
     }
 }
 
@@ -278,28 +313,31 @@ kq_status TrailMaps::init(const float* E_hi, const float* E_lo, const float* Lt_
 
 kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, int64_t i0, int64_t cb, int64_t ce,
                    int* info, cudaStream_t stream) {
-    // The next block column (critical path, few tiles): 128-column tiles, 2-stage ring.
-    // The far columns: 256-column tiles with a 1-stage ring (97 KB), so a tile fits on an SM
-    // beside the next block kernel's CTAs (64 KB each) that run at the same time.
+    // The next block column (critical path, few tiles): 128-column tiles; the far columns:
+    // 256-column tiles; both with a 2-stage ring.
     using Narrow = TrailCfg<128, 2>;
-    using Wide = TrailCfg<256, 1>;
+    using Wide = TrailCfg<256, 2>;
     static bool attr = false;
     if (!attr) {
-        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<256, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<256, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      Wide::SMEM));
         KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<128, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      Narrow::SMEM));
         attr = true;
     }
-    const unsigned gy = static_cast<unsigned>(cdiv(d_out, TBM));
+    // Persistent: at most one CTA per SM, each walking the tiles t, t + grid, ... (column
+    // tile fastest, so the CTAs running together share row and column operands in L2).
+    const int n_row = static_cast<int>(cdiv(d_out, TBM));
     if (ce - cb <= 128) {
-        dim3 grid(static_cast<unsigned>(cdiv(ce - cb, 128)), gy);
-        trail_tc_kernel<128, 2><<<grid, T_THREADS, Narrow::SMEM, stream>>>(
-            m.eh, m.el, m.rh_narrow, m.rl_narrow, W, d_out, d_in, static_cast<int>(i0), cb, ce, info);
+        const int n_col = static_cast<int>(cdiv(ce - cb, 128));
+        const int n = n_row * n_col;
+        trail_tc_kernel<128, 2><<<static_cast<unsigned>(std::min(n, num_sms())), T_THREADS, Narrow::SMEM, stream>>>(
+            m.eh, m.el, m.rh_narrow, m.rl_narrow, W, d_out, d_in, static_cast<int>(i0), cb, ce, n_col, n, info);
     } else {
-        dim3 grid(static_cast<unsigned>(cdiv(ce - cb, 256)), gy);
-        trail_tc_kernel<256, 1><<<grid, T_THREADS, Wide::SMEM, stream>>>(
-            m.eh, m.el, m.rh_wide, m.rl_wide, W, d_out, d_in, static_cast<int>(i0), cb, ce, info);
+        const int n_col = static_cast<int>(cdiv(ce - cb, 256));
+        const int n = n_row * n_col;
+        trail_tc_kernel<256, 2><<<static_cast<unsigned>(std::min(n, num_sms())), T_THREADS, Wide::SMEM, stream>>>(
+            m.eh, m.el, m.rh_wide, m.rl_wide, W, d_out, d_in, static_cast<int>(i0), cb, ce, n_col, n, info);
     }
     KQ_LAUNCH_CHECK("trail_tc_kernel");
     return KQ_OK;

@@ -18,7 +18,7 @@ class LayerPipeline:
     def __init__(self, d_out: int, d_in: int, bits: int, group: int, block: int = 128,
                  damp: float = 0.01, device: str = "cuda", want_col_loss: bool = True,
                  overlap: bool = True, x_chunk_tokens: int = 0, g_chunk_tokens: int = 32768,
-                 trailing: str = "fp32"):
+                 trailing: str = "3xtf32"):
         self.d_out, self.d_in, self.bits, self.group, self.block, self.damp = d_out, d_in, bits, group, block, damp
         f32 = dict(dtype=torch.float32, device=device)
         ng = 1 if group == 0 else -(-d_in // group)
