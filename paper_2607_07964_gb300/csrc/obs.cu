@@ -426,6 +426,7 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
         kq_status st0 = split_tf32(Lt, d_in * d_in, o.Lh, o.Ll, stream);
         if (st0 != KQ_OK) return st0;
         if ((st0 = maps.init(o.Eh, o.El, o.Lh, o.Ll, d_out, d_in)) != KQ_OK) return st0;
+        if ((st0 = maps.set_w(W, d_out, d_in)) != KQ_OK) return st0;
     }
     if (group == 0) {
         rowgrid_kernel<<<static_cast<unsigned>(cdiv(d_out, 8)), 256, 0, stream>>>(W, d_out, d_in, bits, scale,

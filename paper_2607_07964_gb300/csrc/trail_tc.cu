@@ -36,11 +36,23 @@ constexpr int A_SLAB = TBM * TBK * 4;    // 16 KB
 
 template <int BN, int STAGES>
 struct TrailCfg {
-    static constexpr int B_SLAB = BN * TBK * 4;                    // 16 or 32 KB
+    static constexpr int B_SLAB = BN * TBK * 4;                    // 16 KB for BN = 128
     static constexpr int STAGE = 2 * A_SLAB + 2 * B_SLAB;          // hi + lo of both
-    static constexpr int SMEM = STAGES * STAGE + 1024 + 256;
+    static constexpr int WTILE = TBM * BN * 4;                     // the tile of W (64 KB)
+    static constexpr int SMEM = STAGES * STAGE + WTILE + 1024 + 256;
     static_assert(2 * BN <= 512, "two accumulators must fit in TMEM");
+    static_assert(BN % 32 == 0, "W moves in 32-column boxes");
 };
+
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* m, const void* src, int x, int y) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                     reinterpret_cast<uint64_t>(m)),
+                 "r"(smem_u32(src)), "r"(x), "r"(y)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
 // Instruction descriptor, kind::tf32: fp32 accumulator, tf32 A and B, both K-major.
 __host__ __device__ constexpr uint32_t idesc_tf32_k_major(int M, int N) {
@@ -70,17 +82,22 @@ template <int BN, int TSTAGES>
 __global__ void __launch_bounds__(T_THREADS, 1)
 trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__ CUtensorMap mEl,
                 const __grid_constant__ CUtensorMap mRh, const __grid_constant__ CUtensorMap mRl,
-                float* __restrict__ W, int64_t d_out, int64_t d_in, int i0, int64_t cb, int64_t ce,
-                int n_col_tiles, int n_tiles, int* info) {
+                const __grid_constant__ CUtensorMap mW, int d_out, int i0, int cb, int n_col_tiles, int n_tiles,
+                int* info) {
     using C = TrailCfg<BN, TSTAGES>;
+    constexpr int WBOX = TBM * 32 * 4;     // one 128-row x 32-column box of W (16 KB)
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-    uint64_t* full = reinterpret_cast<uint64_t*>(smem + TSTAGES * C::STAGE);
+    uint8_t* wtile = smem + TSTAGES * C::STAGE;                   // BN / 32 boxes, 128-byte swizzled
+    uint64_t* full = reinterpret_cast<uint64_t*>(wtile + C::WTILE);
     uint64_t* empty = full + TSTAGES;
     uint64_t* tfull = empty + TSTAGES;     // accumulator b holds a finished tile
     uint64_t* tempty = tfull + 2;          // the epilogue has read accumulator b
-    uint64_t* mma_done = tempty + 2;
+    uint64_t* wfull = tempty + 2;          // the W tile has arrived
+    uint64_t* wfree = wfull + 1;           // the W tile has been stored (buffer reusable)
+    uint64_t* wdone = wfree + 1;           // all 8 epilogue warps have updated the W tile
+    uint64_t* mma_done = wdone + 1;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
@@ -96,6 +113,9 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
             mbar_init(&tfull[b], 1);
             mbar_init(&tempty[b], 8);
         }
+        mbar_init(wfull, 1);
+        mbar_init(wfree, 1);
+        mbar_init(wdone, 8);
         mbar_init(mma_done, 1);
         *abort_flag = 0;
         fence_mbar_init();
@@ -109,6 +129,7 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
         tma_prefetch_desc(&mEl);
         tma_prefetch_desc(&mRh);
         tma_prefetch_desc(&mRl);
+        tma_prefetch_desc(&mW);
     }
     tc_fence_before();
     __syncthreads();
@@ -118,11 +139,17 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
-            int k = 0;
+            int k = 0, li = 0, w_issued = 0;
             bool ok = true;
-            for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+            for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++li) {
                 const int r0 = (t / n_col_tiles) * TBM;
-                const int c0 = static_cast<int>(cb) + (t % n_col_tiles) * BN;
+                const int c0 = cb + (t % n_col_tiles) * BN;
+                // the tile of W, once the previous tile has been stored from the buffer
+                if (!mbar_wait(wfree, (static_cast<uint32_t>(li) & 1u) ^ 1u, abort_flag)) break;
+                mbar_arrive_expect_tx(wfull, C::WTILE);
+#pragma unroll
+                for (int j = 0; j < BN / 32; ++j) tma_load_2d(wtile + j * WBOX, &mW, wfull, c0 + 32 * j, r0);
+                w_issued = li + 1;
                 for (int s = 0; s < TNSLAB; ++s, ++k) {
                     const int st = k % TSTAGES;
                     const uint32_t u = static_cast<uint32_t>(k / TSTAGES);
@@ -142,6 +169,7 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
             // every issued load must land before the CTA exits
             for (int j = (k > TSTAGES ? k - TSTAGES : 0); j < k; ++j)
                 wait_quiet(&full[j % TSTAGES], static_cast<uint32_t>(j / TSTAGES) & 1u);
+            if (w_issued > 0) wait_quiet(wfull, static_cast<uint32_t>(w_issued - 1) & 1u);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
@@ -185,23 +213,18 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
         }
     } else {
         // ------------------------------------------------------------ epilogue (8 warps)
-        constexpr int HALF = BN / 2;            // columns per thread
+        // Thread = one row of the tile (TMEM lane) and BN / 2 columns. W sits in shared
+        // memory as 128-byte swizzled rows (16-byte chunk c of row r at c ^ (r & 7)), so the
+        // float4 accesses of 8 consecutive rows hit distinct banks.
+        constexpr int HALF = BN / 2;
         const int q = warp & 3;                 // TMEM lane quadrant this warp may access
         const int h = (warp - 2) >> 2;          // which half of the columns
+        const int r = q * 32 + lane;            // row within the tile
         int li = 0;
         for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++li) {
             const int buf = li & 1;
-            const int64_t row = static_cast<int64_t>(t / n_col_tiles) * TBM + q * 32 + lane;
-            const int64_t cs = cb + static_cast<int64_t>(t % n_col_tiles) * BN + h * HALF;
-            const bool live = row < d_out;
-            const bool vec = live && cs + HALF <= ce && (d_in & 3) == 0;
-            float* wrow = W + row * d_in + cs;
-            float4 wv[HALF / 4];
-            if (vec) {   // W loads overlap the MMAs of this tile
-#pragma unroll
-                for (int i = 0; i < HALF / 4; ++i) wv[i] = reinterpret_cast<const float4*>(wrow)[i];
-            }
-            bool ok = mbar_wait(&tfull[buf], (static_cast<uint32_t>(li) >> 1) & 1u, abort_flag);
+            bool ok = mbar_wait(&tfull[buf], (static_cast<uint32_t>(li) >> 1) & 1u, abort_flag) &&
+                      mbar_wait(wfull, static_cast<uint32_t>(li) & 1u, abort_flag);
             ok = __all_sync(0xffffffffu, ok) && !*abort_flag;
             if (!ok) break;
             tc_fence_after();
@@ -212,23 +235,35 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
                 float v[32];
                 tmem_ld32(taddr + static_cast<uint32_t>(p * 32), v);
                 tc_wait_ld();
-                if (vec) {
+                float4* rowp = reinterpret_cast<float4*>(wtile + (h * (HALF / 32) + p) * WBOX + r * 128);
 #pragma unroll
-                    for (int i = 0; i < 8; ++i) {
-                        const float4 o = wv[8 * p + i];
-                        reinterpret_cast<float4*>(wrow)[8 * p + i] =
-                            make_float4(o.x - v[4 * i], o.y - v[4 * i + 1], o.z - v[4 * i + 2], o.w - v[4 * i + 3]);
-                    }
-                } else if (live) {
-#pragma unroll
-                    for (int i = 0; i < 32; ++i)
-                        if (cs + 32 * p + i < ce) wrow[32 * p + i] -= v[i];
+                for (int c = 0; c < 8; ++c) {
+                    float4* cp = rowp + (c ^ (r & 7));
+                    const float4 o = *cp;
+                    *cp = make_float4(o.x - v[4 * c], o.y - v[4 * c + 1], o.z - v[4 * c + 2], o.w - v[4 * c + 3]);
                 }
             }
             tc_fence_before();
+            fence_proxy_async();                        // this thread's W updates -> TMA
             __syncwarp();
-            if (lane == 0) mbar_arrive(&tempty[buf]);
+            if (lane == 0) {
+                mbar_arrive(&tempty[buf]);              // the accumulator may be reused
+                mbar_arrive(wdone);
+            }
+            if (warp == 2 && lane == 0) {
+                // store the tile once every warp has updated it, then free the buffer
+                if (mbar_wait(wdone, static_cast<uint32_t>(li) & 1u, abort_flag)) {
+                    const int r0 = (t / n_col_tiles) * TBM;
+                    const int c0 = cb + (t % n_col_tiles) * BN;
+#pragma unroll
+                    for (int j = 0; j < BN / 32; ++j) tma_store_2d(&mW, wtile + j * WBOX, c0 + 32 * j, r0);
+                    bulk_commit();
+                    bulk_wait_read0();
+                    mbar_arrive(wfree);
+                }
+            }
         }
+        if (warp == 2 && lane == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
     }
 
     tc_fence_before();
@@ -304,41 +339,37 @@ kq_status TrailMaps::init(const float* E_hi, const float* E_lo, const float* Lt_
     kq_status st;
     if ((st = make_map(&eh, E_hi, d_out, d_in, TBM)) != KQ_OK) return st;
     if ((st = make_map(&el, E_lo, d_out, d_in, TBM)) != KQ_OK) return st;
-    if ((st = make_map(&rh_wide, Lt_hi, d_in, d_in, 256)) != KQ_OK) return st;
-    if ((st = make_map(&rl_wide, Lt_lo, d_in, d_in, 256)) != KQ_OK) return st;
     if ((st = make_map(&rh_narrow, Lt_hi, d_in, d_in, 128)) != KQ_OK) return st;
     if ((st = make_map(&rl_narrow, Lt_lo, d_in, d_in, 128)) != KQ_OK) return st;
     return KQ_OK;
 }
 
+kq_status TrailMaps::set_w(float* W, int64_t d_out, int64_t d_in) {
+    return make_map(&w, W, d_out, d_in, TBM);
+}
+
 kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, int64_t i0, int64_t cb, int64_t ce,
                    int* info, cudaStream_t stream) {
-    // The next block column (critical path, few tiles): 128-column tiles; the far columns:
-    // 256-column tiles; both with a 2-stage ring.
-    using Narrow = TrailCfg<128, 2>;
-    using Wide = TrailCfg<256, 2>;
-    static bool attr = false;
-    if (!attr) {
-        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<256, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     Wide::SMEM));
-        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<128, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     Narrow::SMEM));
-        attr = true;
-    }
     // Persistent: at most one CTA per SM, each walking the tiles t, t + grid, ... (column
     // tile fastest, so the CTAs running together share row and column operands in L2).
-    const int n_row = static_cast<int>(cdiv(d_out, TBM));
-    if (ce - cb <= 128) {
-        const int n_col = static_cast<int>(cdiv(ce - cb, 128));
-        const int n = n_row * n_col;
-        trail_tc_kernel<128, 2><<<static_cast<unsigned>(std::min(n, num_sms())), T_THREADS, Narrow::SMEM, stream>>>(
-            m.eh, m.el, m.rh_narrow, m.rl_narrow, W, d_out, d_in, static_cast<int>(i0), cb, ce, n_col, n, info);
-    } else {
-        const int n_col = static_cast<int>(cdiv(ce - cb, 256));
-        const int n = n_row * n_col;
-        trail_tc_kernel<256, 2><<<static_cast<unsigned>(std::min(n, num_sms())), T_THREADS, Wide::SMEM, stream>>>(
-            m.eh, m.el, m.rh_wide, m.rl_wide, W, d_out, d_in, static_cast<int>(i0), cb, ce, n_col, n, info);
+    // 128-column tiles; a range either is a whole number of tiles or ends at d_in (the TMA
+    // copies clip the last tile there).
+    using Cfg = TrailCfg<128, 2>;
+    if ((ce - cb) % 128 != 0 && ce != d_in) {
+        set_error("trailing update: column range [%lld, %lld) is not whole tiles", (long long)cb, (long long)ce);
+        return KQ_ERR_INVALID_ARG;
     }
+    static bool attr = false;
+    if (!attr) {
+        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<128, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
+        attr = true;
+    }
+    const int n_row = static_cast<int>(cdiv(d_out, TBM));
+    const int n_col = static_cast<int>(cdiv(ce - cb, 128));
+    const int n = n_row * n_col;
+    trail_tc_kernel<128, 2><<<static_cast<unsigned>(std::min(n, num_sms())), T_THREADS, Cfg::SMEM, stream>>>(
+        m.eh, m.el, m.rh_narrow, m.rl_narrow, m.w, static_cast<int>(d_out), static_cast<int>(i0),
+        static_cast<int>(cb), n_col, n, info);
     KQ_LAUNCH_CHECK("trail_tc_kernel");
     return KQ_OK;
 }
