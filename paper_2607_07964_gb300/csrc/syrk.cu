@@ -194,17 +194,53 @@ syrk_tc_kernel(const __grid_constant__ CUtensorMap tmap, float* __restrict__ H, 
             __syncwarp();
             if (lane == 0) mbar_arrive(&tempty[buf]);
         }
-        if (ok && !*abort_flag && row < d) {
-            const int cbase = j0 + half * 128;
+        // Write-out through shared memory (the pipeline stages are idle now): each warp stages
+        // its 32 rows x 128 columns, then updates the lower tile one 128-byte row segment at a
+        // time (coalesced, also for the accumulate read) and writes the mirror from the staged
+        // results (lanes on consecutive rows of H^T: coalesced too).
+        ok = __all_sync(0xffffffffu, ok && !*abort_flag);
+        if (ok) {
+            constexpr int SLD = 129;
+            float* st = reinterpret_cast<float*>(smem) + (warp - 2) * 32 * SLD;
 #pragma unroll
-            for (int i = 0; i < 128; ++i) {
-                const int col = cbase + i;
-                if (col < d && col <= row) {
-                    float v = acc[i];
-                    float* dst = H + static_cast<int64_t>(row) * d + col;
-                    if (accumulate) v += *dst;
-                    *dst = v;
-                    if (col < row) H[static_cast<int64_t>(col) * d + row] = v;
+            for (int i = 0; i < 128; ++i) st[lane * SLD + i] = acc[i];
+            __syncwarp();
+            const int cbase = j0 + half * 128;
+            const int rbase = i0 + q * 32;
+            // eight rows at a time, so 32 loads per lane are in flight (accumulate mode)
+#pragma unroll 1
+            for (int r8 = 0; r8 < 32; r8 += 8) {
+                float old[8][4];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const int rr = rbase + r8 + u;
+#pragma unroll
+                    for (int m = 0; m < 4; ++m) {
+                        const int col = cbase + lane + 32 * m;
+                        old[u][m] = (accumulate && rr < d && col < d && col <= rr)
+                                        ? H[static_cast<int64_t>(rr) * d + col] : 0.0f;
+                    }
+                }
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const int rr = rbase + r8 + u;
+#pragma unroll
+                    for (int m = 0; m < 4; ++m) {
+                        const int col = cbase + lane + 32 * m;
+                        if (rr < d && col < d && col <= rr) {
+                            const float v = st[(r8 + u) * SLD + lane + 32 * m] + old[u][m];
+                            H[static_cast<int64_t>(rr) * d + col] = v;
+                            st[(r8 + u) * SLD + lane + 32 * m] = v;
+                        }
+                    }
+                }
+            }
+            __syncwarp();
+            if (row < d) {
+#pragma unroll 4
+                for (int i = 0; i < 128; ++i) {
+                    const int col = cbase + i;
+                    if (col < d && col < row) H[static_cast<int64_t>(col) * d + row] = st[lane * SLD + i];
                 }
             }
         }
