@@ -8,7 +8,7 @@
 // reversal, the lower Cholesky factor C of A = J H J gives H = (J C J)(J C J)^T, J C J
 // upper, hence H^-1 = (J C^-T J)(J C^-T J)^T and L = J C^-T J, i.e. L[i][j] = C^-1[n-1-j][n-1-i].
 // One right-looking blocked sweep (block nb = 128) computes C and Z = C^-1 together:
-//   step k: diag  -- factor A_kk = C_kk C_kk^T and invert C_kk in registers (1 CTA);
+//   step k: diag  -- factor A_kk = C_kk C_kk^T in registers and keep C_kk^-1 (1 CTA);
 //           panel -- C_ik = A_ik C_kk^-T (i > k) and Z_kj = C_kk^-1 B_kj (j < k);
 //           update-- A_ij -= C_ik C_jk^T (k < j <= i) and B_ij -= C_ik Z_kj (j <= k < i),
 // where B (stored in Z's blocks) is the right-hand side I of C Z = I after the earlier
@@ -81,8 +81,9 @@ __global__ void prep_kernel(const float* __restrict__ H, int64_t n, int64_t npad
 // below it, h_j = 0), pivot d_j and multipliers u_i = M_ij / d_j, every row i > j updates
 //   M_ik -= u_i h_k      (k != j; k > j: Schur complement, k < j: rows of L^-1)
 // and column j keeps its value, the unscaled column j of L D. So M ends up holding, below
-// the diagonal, R = -L^-1 D (column-scaled), and C = L D^1/2 has C_ij = (column j at step j)
-// / sqrt(d_j), while C^-1 = D^-1/2 L^-1 has entries -R_ik / (d_k sqrt(d_i)).
+// the diagonal, R = -L^-1 D (column-scaled), and C^-1 = D^-1/2 L^-1 has entries
+// -R_ik / (d_k sqrt(d_i)). C = L D^1/2 itself is not stored: the panel and the updates read
+// only C^-1 of the diagonal block.
 //
 // Four steps at once (block column q, rows j..j+3, j = 4q): with the 4 x 4 pivot block
 // factored as L_b D_b L_b^T (raw columns g = L_b D_b, raw inverse rows b of the block),
@@ -98,10 +99,9 @@ __global__ void prep_kernel(const float* __restrict__ H, int64_t n, int64_t npad
 // registers. Pivots are checked by thread 0 (first non-positive one reported).
 constexpr int DIAG_THREADS = 544;                            // 528 owners + 16 idle lanes
 constexpr int DG_OWNERS = (NB / 4) * (NB / 4 + 1) / 2;       // 528
-constexpr int DG_LD = NB + 4;                                // craw row stride (16-byte rows)
 constexpr int DG_PIV = 32;                                   // floats per pivot record
 constexpr size_t DIAG_SMEM =
-    (static_cast<size_t>(NB) * DG_LD + 2 * NB * 4 + 2 * 4 * NB + 2 * DG_PIV + NB) * sizeof(float);
+    (2 * NB * 4 + 2 * 4 * NB + 2 * DG_PIV + NB) * sizeof(float);
 
 struct Piv4 {   // factored 4 x 4 pivot block: 1 / d, unit-lower L_b, raw inverse rows b
     float rd[4], l10, l20, l30, l21, l31, l32, b10, b20, b30, b21, b31, b32;
@@ -126,7 +126,7 @@ __device__ __forceinline__ void unit_lower_solve(float& x0, float& x1, float& x2
 // Publish the inputs of block step q (buffer q & 1): block-row rows (left of the pivot),
 // panel rows (below it), and the factored pivot, whose owner also sets its block final.
 __device__ __forceinline__ void diag_publish(int q, float (&m)[4][4], int bi, int bk, float* Pst, float* Qst,
-                                             float* Pv, float* craw) {
+                                             float* Pv) {
     const int buf = q & 1;
     const int i0 = 4 * bi, k0 = 4 * bk;
     if (bi == q && bk < q) {
@@ -178,19 +178,12 @@ __device__ __forceinline__ void diag_publish(int q, float (&m)[4][4], int bi, in
         m[2][1] = b21;
         m[3][1] = b31;
         m[3][2] = b32;
-        craw[(i0 + 1) * DG_LD + k0] = g10;
-        craw[(i0 + 2) * DG_LD + k0] = g20;
-        craw[(i0 + 3) * DG_LD + k0] = g30;
-        craw[(i0 + 2) * DG_LD + k0 + 1] = g21;
-        craw[(i0 + 3) * DG_LD + k0 + 1] = g31;
-        craw[(i0 + 3) * DG_LD + k0 + 2] = g32;
     }
 }
 
 __global__ void __launch_bounds__(DIAG_THREADS) chol_diag_kernel(Work w, int64_t n, int64_t npad, int k, int* info) {
     extern __shared__ __align__(16) float sm[];
-    float* craw = sm;                     // [NB][DG_LD]  columns of L D at their own step
-    float* Pst = craw + NB * DG_LD;       // [2][NB][4]   panel rows
+    float* Pst = sm;                      // [2][NB][4]   panel rows
     float* Qst = Pst + 2 * NB * 4;        // [2][4][NB]   block-row rows
     float* Pv = Qst + 2 * 4 * NB;         // [2][DG_PIV]  pivot records
     float* dv = Pv + 2 * DG_PIV;          // [NB]         pivots d
@@ -217,7 +210,7 @@ __global__ void __launch_bounds__(DIAG_THREADS) chol_diag_kernel(Work w, int64_t
             m[r][2] = v.z;
             m[r][3] = v.w;
         }
-        diag_publish(0, m, bi, bk, Pst, Qst, Pv, craw);
+        diag_publish(0, m, bi, bk, Pst, Qst, Pv);
     }
     __syncthreads();
 #pragma unroll 1
@@ -282,15 +275,13 @@ __global__ void __launch_bounds__(DIAG_THREADS) chol_diag_kernel(Work w, int64_t
                     u[r][3] = x3 * p.rd[3];
                 }
                 if (bk == q) {
-                    // panel: final raw inverse columns; w is column block q of L D
+                    // panel: final raw inverse columns
 #pragma unroll
                     for (int r = 0; r < 4; ++r) {
                         m[r][0] = fmaf(-u[r][3], p.b30, fmaf(-u[r][2], p.b20, fmaf(-u[r][1], p.b10, wv[r][0])));
                         m[r][1] = fmaf(-u[r][3], p.b31, fmaf(-u[r][2], p.b21, wv[r][1]));
                         m[r][2] = fmaf(-u[r][3], p.b32, wv[r][2]);
                         m[r][3] = wv[r][3];
-                        *reinterpret_cast<float4*>(craw + (i0 + r) * DG_LD + k0) =
-                            make_float4(wv[r][0], wv[r][1], wv[r][2], wv[r][3]);
                     }
                 } else {
                     // h = L_b^-1 x, x from the block row (left columns) or the panel (right)
@@ -327,22 +318,20 @@ __global__ void __launch_bounds__(DIAG_THREADS) chol_diag_kernel(Work w, int64_t
                 }
             }
         }
-        if (owner && q + 1 < NB / 4) diag_publish(q + 1, m, bi, bk, Pst, Qst, Pv, craw);
+        if (owner && q + 1 < NB / 4) diag_publish(q + 1, m, bi, bk, Pst, Qst, Pv);
         __syncthreads();
     }
-    // Scales (the staging is free now): sqrt(d), 1 / sqrt(d), 1 / d.
-    float* sq = Pst;
-    float* isq = Pst + NB;
+    // Scales (the staging is free now): 1 / sqrt(d), 1 / d.
+    float* isq = Pst;
     float* idv = Qst;
     if (tid < NB) {
         const float d = dv[tid];
-        const float r = sqrtf(d);
-        sq[tid] = r;
-        isq[tid] = __frcp_rn(r);
+        isq[tid] = __frcp_rn(sqrtf(d));
         idv[tid] = __frcp_rn(d);
     }
     __syncthreads();
     // C^-1 = D^-1/2 L^-1 with L^-1_ik = -R_ik / d_k (k < i); the upper blocks of Z stay 0.
+    // C_kk itself is not stored: later steps read only C^-1_kk and the blocks below it.
     if (owner) {
 #pragma unroll
         for (int r = 0; r < 4; ++r) {
@@ -356,17 +345,6 @@ __global__ void __launch_bounds__(DIAG_THREADS) chol_diag_kernel(Work w, int64_t
             }
             *reinterpret_cast<float4*>(w.Z + (off + i) * npad + off + k0) = make_float4(o[0], o[1], o[2], o[3]);
         }
-    }
-    // C = (L D) D^-1/2, upper part 0.
-    for (int e = tid; e < NB * NB / 4; e += blockDim.x) {
-        const int r = e / (NB / 4), c0 = 4 * (e % (NB / 4));
-        float o[4];
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-            const int cc = c0 + c;
-            o[c] = cc < r ? craw[r * DG_LD + cc] * isq[cc] : (cc == r ? sq[r] : 0.0f);
-        }
-        *reinterpret_cast<float4*>(w.A + (off + r) * npad + off + c0) = make_float4(o[0], o[1], o[2], o[3]);
     }
 }
 
