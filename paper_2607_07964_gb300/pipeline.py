@@ -65,7 +65,14 @@ class LayerPipeline:
     def _chunks(self, which: str, T: int) -> list[tuple[int, int]]:
         c = self.chunk_tokens[which]
         c = c if c > 0 else max(T, 1)
-        return [(t0, min(T, t0 + c)) for t0 in range(0, max(T, 1), c)]
+        ch = [(t0, min(T, t0 + c)) for t0 in range(0, max(T, 1), c)]
+        if which == "G" and self.chunk_tokens["G"] > 0 and len(ch) > 1:
+            # the last chunk in four: after G's last bytes arrive on the host path, only a
+            # quarter chunk of accumulation stands before S_G, U and the sweep
+            t0, t1 = ch.pop()
+            q = max(1, -(-(t1 - t0) // 4))
+            ch += [(a, min(t1, a + q)) for a in range(t0, t1, q)]
+        return ch
 
     def _factor(self, which, A, H, trace, info, stream, ready=None) -> None:
         """H = A^T A over the token chunks (Alg. 1 online statistic); `ready`, if given,
