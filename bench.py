@@ -211,6 +211,16 @@ def dist_setup(backend: str):
     return ws, rank, local
 
 
+def max_over_ranks(v: float, ws: int, device: str = "cpu") -> float:
+    """The slowest rank's value (the job's time); v itself when there is one rank."""
+    if ws <= 1:
+        return v
+    import torch
+    t = torch.tensor([v], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
 def run_reference(args):
     ws, rank, _ = dist_setup("gloo")
     cfg = kqsynth.CONFIGS[args.config]
@@ -289,11 +299,7 @@ def run_ours(args):
     launches = per_step * args.steps if graph is not None else kq.launch_count() - n0
     clocks = sampler.stop()
     p.check(stream)
-    total_ms = t_start.elapsed_time(t_end)
-    if ws > 1:
-        t = torch.tensor([total_ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(t_start.elapsed_time(t_end), ws, dev)
     # Per-stage times and the SYRK roofline come from a second, serialized pass (each stage
     # alone on the stream, bracketed by events); the headline value above overlaps stages.
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(len(STAGES) + 1)] for _ in range(args.steps)]
@@ -341,11 +347,7 @@ def run_ours(args):
         e1.record(stream)
         torch.cuda.synchronize()
         barrier()
-        e_ms = e0.elapsed_time(e1)
-        if ws > 1:
-            t = torch.tensor([e_ms], device=dev)
-            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-            e_ms = float(t.item())
+        e_ms = max_over_ranks(e0.elapsed_time(e1), ws, dev)
         e2e = {"value": e_ms / (ws * args.steps), "unit": "ms", "h2d_bytes_per_step": nin,
                "d2h_bytes_per_step": nout}
 
