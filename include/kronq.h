@@ -71,6 +71,16 @@ KQ_API uint64_t kq_launch_count(void);
  */
 KQ_API kq_status kq_check(int* info, int reset, int* pivot_out, kq_stream_t stream);
 
+/*
+ * kq_selftest_timeout: a diagnostic with no counterpart in the paper. Launches one kernel
+ *   that waits on an mbarrier nothing arrives on, using the same bounded wait as every
+ *   pipeline kernel (TMA/tcgen05 producers, consumers and epilogues), which gives up after
+ *   limit_us microseconds (1 .. 2e6) and records -KQ_ERR_TIMEOUT in *info (device int). Read
+ *   it with kq_check. It shows, without faulting or hanging the GPU, that a stalled pipeline
+ *   returns an error status and leaves the context usable.
+ */
+KQ_API kq_status kq_selftest_timeout(int* info, int64_t limit_us, kq_stream_t stream);
+
 /* ------------------------------------------------------------------------------------
  * Stage 1: Kronecker factors.
  * Paper: Sec. 2.1 Eq. (ptq_obj) defines H_X = X X^T; Sec. 3.1 Eq. (kfac) the factor pair

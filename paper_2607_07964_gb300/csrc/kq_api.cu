@@ -72,7 +72,32 @@ SideStream* side_stream(cudaStream_t caller) {
     return c.s ? &c : nullptr;
 }
 
+// Waits on an mbarrier that nothing ever arrives on, with the bounded wait every pipeline
+// kernel uses, and reports the timeout the way those kernels do.
+__global__ void selftest_timeout_kernel(int* info, uint64_t limit_ns) {
+    __shared__ uint64_t bar;
+    __shared__ int abort_flag;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        abort_flag = 0;
+        fence_mbar_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0 && !mbar_wait(&bar, 0, &abort_flag, limit_ns)) record_error(info, -KQ_ERR_TIMEOUT);
+}
+
 }  // namespace kq
+
+extern "C" kq_status kq_selftest_timeout(int* info, int64_t limit_us, kq_stream_t stream_) {
+    if (!info || limit_us < 1 || limit_us > 2000000) {
+        kq::set_error("kq_selftest_timeout: info must be a device int and 1 <= limit_us <= 2e6");
+        return KQ_ERR_INVALID_ARG;
+    }
+    kq::selftest_timeout_kernel<<<1, 32, 0, reinterpret_cast<cudaStream_t>(stream_)>>>(
+        info, static_cast<uint64_t>(limit_us) * 1000u);
+    KQ_LAUNCH_CHECK("selftest_timeout_kernel");
+    return KQ_OK;
+}
 
 extern "C" const char* kq_last_error(void) { return kq::g_err; }
 

@@ -98,13 +98,14 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 // Bounded wait for the phase with the given parity. Returns false (and raises *abort)
 // when the limit is reached or another thread has already raised *abort.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                          uint64_t limit_ns = kWaitLimitNs) {
     if (mbar_try_wait(bar, parity)) return true;
     uint64_t t0 = global_timer_ns();
     for (uint32_t it = 0; it < kWaitLimitIters; ++it) {
         if (mbar_try_wait(bar, parity)) return true;
         if (*abort) return false;
-        if ((it & 255u) == 255u && global_timer_ns() - t0 > kWaitLimitNs) break;
+        if ((it & 255u) == 255u && global_timer_ns() - t0 > limit_ns) break;
     }
     *abort = 1;
     return false;

@@ -43,6 +43,7 @@ def lib() -> ctypes.CDLL:
             "kq_version": ([], I),
             "kq_launch_count": ([], ctypes.c_uint64),
             "kq_check": ([P, I, P, P], I),
+            "kq_selftest_timeout": ([P, I64, P], I),
             "kq_accum_factor": ([P, I64, I64, I64, P, I, P, P, P], I),
             "kq_compute_scales": ([P, I64, I64, P, P, P, P, P], I),
             "kq_compute_scales_diag": ([P, I64, I64, P, P, P, P, P], I),
@@ -118,6 +119,12 @@ def kq_check(info=None, reset: bool = True, stream=None) -> tuple[int, int]:
     raw = ctypes.c_int(0)
     st = lib().kq_check(_ptr(info), int(reset), ctypes.byref(raw), _stream(stream))
     return st, raw.value
+
+
+def kq_selftest_timeout(info, limit_us: int, stream=None) -> None:
+    """A kernel whose bounded wait runs out (nothing arrives); *info gets -KQ_ERR_TIMEOUT."""
+    _need(info, "info", torch.int32)
+    _ok(lib().kq_selftest_timeout(_ptr(info), int(limit_us), _stream(stream)), "kq_selftest_timeout")
 
 
 def kq_accum_factor(A, H, accumulate: bool = False, trace=None, info=None, stream=None) -> None:

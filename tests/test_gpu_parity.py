@@ -430,3 +430,19 @@ def test_diag_variants_match_matrix_variants():
     K().kq_traces_diag(torch.diagonal(HXd).contiguous(), sx1, None, None, t2)
     K().kq_traces_diag(None, None, torch.diagonal(HGd).contiguous(), sg1, t2)
     assert torch.equal(t1, t2)
+
+
+# ------------------------------------------------------------ failure detection
+def test_bounded_wait_reports_timeout_and_context_survives():
+    """A wait that nothing satisfies (no GPU fault, no hang): the kernel gives up after its
+    limit, the status reaches the host through kq_check, and the next calls still work."""
+    info = torch.zeros(1, dtype=torch.int32, device=DEV)
+    K().kq_selftest_timeout(info, 20000)          # 20 ms
+    st, raw = K().kq_check(info, reset=True)
+    assert st == K().KQ_ERR_TIMEOUT
+    assert raw == -K().KQ_ERR_TIMEOUT
+    assert K().kq_check(info)[0] == K().KQ_OK     # reset cleared the word
+    X = kqsynth.activations(kqsynth.CONFIGS["tiny256"].replace(T=256, d_in=64))
+    H = torch.empty((64, 64), device=DEV)
+    K().kq_accum_factor(bf16_dev(X), H)
+    assert rel_fro(host(H), ref.accum_factor(X)) <= 1e-5
