@@ -13,7 +13,10 @@ Llama weights, Sec. 5.1; neither is available here):
   * weights     W[i, j] = 0.02 * z, each entry multiplied by 10 with probability 0.001;
   * X and G are rounded to bf16 (round-to-nearest-even); W is rounded to bf16 unless
     `w_bf16` is False (then it stays fp32);
-  * RHT sign vectors are +-1 (int8), one per side.
+  * RHT sign vectors are +-1 (int8), one per side;
+  * for the GPTAQ drift correction, the full-precision model's input is
+    x~[t, j] = x[t, j] + drift * sigma_j * z (drift = 0.1 by default), rounded to bf16: X is
+    read as the running quantized model's input and X~ - X as its drift.
 Every tensor has its own sub-seed, so changing one shape does not change the others.
 """
 from __future__ import annotations
@@ -23,7 +26,7 @@ import dataclasses
 import numpy as np
 
 _SUB = {"xscale": 1, "xperm": 2, "x": 3, "gscale": 4, "g": 5, "w": 6, "wbern": 7,
-        "sign_u": 8, "sign_v": 9}
+        "sign_u": 8, "sign_v": 9, "xdrift": 10}
 
 
 @dataclasses.dataclass(frozen=True)
@@ -106,6 +109,15 @@ def activations(cfg: LayerConfig, T: int | None = None) -> np.ndarray:
     return _scaled_normals(_rng(cfg.seed, "x"), T, cfg.d_in, sx)
 
 
+def fp_activations(cfg: LayerConfig, X: np.ndarray, drift: float = 0.1) -> np.ndarray:
+    """X~ [T, d_in] = bf16(X + drift * sigma_j * z): the full-precision model's input to the
+    layer whose running quantized input is X (bf16-representable float32)."""
+    sx, _ = channel_scales(cfg)
+    T = X.shape[0]
+    noise = _scaled_normals(_rng(cfg.seed, "xdrift"), T, cfg.d_in, (drift * sx).astype(np.float32))
+    return round_bf16(np.asarray(X, np.float32) + noise)
+
+
 def gradients(cfg: LayerConfig, T: int | None = None) -> np.ndarray:
     """G [T, d_out], bf16-representable float32, tokens as rows."""
     T = cfg.T if T is None else T
@@ -171,3 +183,21 @@ def device_layer(cfg: LayerConfig, device: str = "cuda"):
     su, sv = signs(cfg)
     return {"X": X, "G": G, "W": w.contiguous(),
             "sign_u": torch.from_numpy(su).to(device), "sign_v": torch.from_numpy(sv).to(device)}
+
+
+def device_fp_activations(cfg: LayerConfig, X, drift: float = 0.1):
+    """X~ = bf16(X + drift * sigma_j * z) drawn on the GPU with torch's generator (the device
+    counterpart of `fp_activations`)."""
+    import torch
+
+    gen = torch.Generator(device=X.device)
+    gen.manual_seed(cfg.seed * 7919 + 23)
+    sx, _ = channel_scales(cfg)
+    sx_t = torch.from_numpy(drift * sx).to(X.device)
+    Xt = torch.empty_like(X)
+    chunk = max(1, (1 << 26) // cfg.d_in)
+    for t0 in range(0, X.shape[0], chunk):
+        t1 = min(X.shape[0], t0 + chunk)
+        z = torch.randn((t1 - t0, cfg.d_in), generator=gen, device=X.device)
+        Xt[t0:t1] = (X[t0:t1].float() + z * sx_t).to(torch.bfloat16)
+    return Xt

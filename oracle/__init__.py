@@ -43,7 +43,7 @@ def _load():
         f = lib.kqref_sweep32
         P = ctypes.c_void_p
         I64 = ctypes.c_int64
-        f.argtypes = [P, I64, I64, P, ctypes.c_int, ctypes.c_int, ctypes.c_int, P, I64,
+        f.argtypes = [P, I64, I64, P, P, ctypes.c_int, ctypes.c_int, ctypes.c_int, P, I64,
                       P, P, P, P, P]
         f.restype = ctypes.c_int
         _lib = lib
@@ -51,13 +51,17 @@ def _load():
 
 
 def obs_sweep_fp32(W, Lt, bits: int, group: int, block: int = 128, rows=None,
-                   want_pre_q: bool = False) -> dict:
+                   want_pre_q: bool = False, Pt=None) -> dict:
     """fp32-ordered sweep of Algorithm 2 (see sweep32.c) on float32 W [m, n] and
-    Lt = R^T [n, n]. `rows` selects a subset of rows (all rows by default)."""
+    Lt = R^T [n, n]; with the GPTAQ correction when Pt = P^T [n, n] is given. `rows`
+    selects a subset of rows (all rows by default)."""
     W = np.ascontiguousarray(W, dtype=np.float32)
     Lt = np.ascontiguousarray(Lt, dtype=np.float32)
     m, n = W.shape
     assert Lt.shape == (n, n)
+    if Pt is not None:
+        Pt = np.ascontiguousarray(Pt, dtype=np.float32)
+        assert Pt.shape == (n, n)
     if rows is None:
         rows_arr = None
         nrows = m
@@ -71,7 +75,7 @@ def obs_sweep_fp32(W, Lt, bits: int, group: int, block: int = 128, rows=None,
     E = np.zeros((nrows, n), np.float32)
     pre_q = np.zeros((nrows, n), np.float32) if want_pre_q else None
     ptr = lambda a: None if a is None else a.ctypes.data  # noqa: E731
-    rc = _load().kqref_sweep32(ptr(W), m, n, ptr(Lt), bits, group, block, ptr(rows_arr), nrows,
+    rc = _load().kqref_sweep32(ptr(W), m, n, ptr(Lt), ptr(Pt), bits, group, block, ptr(rows_arr), nrows,
                                ptr(codes), ptr(scale), ptr(zero), ptr(E), ptr(pre_q))
     if rc != 0:
         raise ValueError("kqref_sweep32 rejected its arguments")

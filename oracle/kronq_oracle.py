@@ -10,6 +10,8 @@ It follows "KronQ: LLM Quantization via Kronecker-Factored Hessian":
   * randomized Hadamard (BiIP) Sec. 3.2 Eq. (biip), Algorithm 1
   * damping, inverse Cholesky  Algorithm 2, Proposition 1
   * column-wise OBS sweep      Sec. 2.1 Eq. (obs_update), Algorithm 2 (GPTQ mode, P = 0)
+  * GPTAQ drift correction     Sec. 2.1 Eq. (gptaq_obj), Sec. 3.1 Eq. (kronq_full),
+                               Proposition 1 (P), Algorithms 1 and 2 (Delta X X^T, P)
   * revert and proxy loss      Algorithm 2, Sec. 3.1 Eq. (kron_obj), Theorem 1
   * sensitivity traces         Sec. 3.3 Eq. (sensitivity)
 Tokens are stored as rows here (X is T x d_in), so the paper's X X^T is X^T X.
@@ -23,7 +25,10 @@ Readings of points the paper leaves open (all listed in the design notes):
   * the quantizer is the asymmetric min-max grid of GPTQ/GPTAQ with round-half-even;
   * per-row grids come from the whole rotated row before the sweep; group grids
     (group == block) from the current, compensated block at block start;
-  * the per-column loss is sum over rows of E_j^2 (no 1/2).
+  * the per-column loss is sum over rows of E_j^2 (no 1/2);
+  * the drift statistic is D = (X~ - X)^T X (tokens as rows), transformed like H_X;
+  * W_{:,j} in the P terms of Proposition 1 and Algorithm 2 is column j's value just
+    before it is quantized, in the column update and in the lazy trailing update alike.
 """
 from __future__ import annotations
 
@@ -33,7 +38,7 @@ __all__ = [
     "accum_factor", "factor_entries", "factor_diag", "biip_scales_from_diag", "sylvester", "paley28", "hadamard_matrix", "rht_matrix",
     "biip_scales", "biip", "damp", "inverse_cholesky_upper", "lower_factor",
     "quant_params", "quantize", "obs_sweep", "dequant", "revert", "proxy_loss",
-    "traces", "pipeline",
+    "traces", "pipeline", "drift_factor", "gptaq_p", "objective",
 ]
 
 
@@ -71,6 +76,16 @@ def factor_diag(A, chunk: int = 8192) -> np.ndarray:
         blk = np.asarray(A[t0:t0 + chunk], dtype=np.float64)
         acc += np.einsum("ij,ij->j", blk, blk)
     return acc
+
+
+def drift_factor(Xt, X) -> np.ndarray:
+    """Algorithm 1's drift statistic Delta X X^T = (X~ - X) X^T, with tokens as rows here:
+    D = (X~ - X)^T X, D[a, b] = sum_t (x~_t[a] - x_t[a]) x_t[b] (not symmetric). X~ is the
+    full-precision model's input to the layer, X the running quantized model's (Sec. 2.1,
+    Eq. gptaq_obj)."""
+    Xt = np.asarray(Xt, dtype=np.float64)
+    X = np.asarray(X, dtype=np.float64)
+    return (Xt - X).T @ X
 
 
 # ----------------------------------------------------------------------------------
@@ -184,10 +199,10 @@ def biip_scales_from_diag(W: np.ndarray, hx: np.ndarray, hg: np.ndarray):
     return biip_scales(W, np.diag(np.asarray(hx, np.float64)), np.diag(np.asarray(hg, np.float64)))
 
 
-def biip(W, HX, HG, sign_u, sign_v):
-    """Algorithm 1 without the drift statistic (X-tilde = X):
-    W <- S_G W S_X; H_X <- S_X^-1 H_X S_X^-1; H_G <- S_G^-1 H_G S_G^-1;
-    W <- U W V^T; H_X <- V H_X V^T; H_G <- U H_G U^T (dense products)."""
+def biip(W, HX, HG, sign_u, sign_v, D=None):
+    """Algorithm 1: W <- S_G W S_X; H_X <- S_X^-1 H_X S_X^-1; H_G <- S_G^-1 H_G S_G^-1;
+    W <- U W V^T; H_X <- V H_X V^T; H_G <- U H_G U^T (dense products). With the drift
+    statistic D (Delta X X^T), also D <- V S_X^-1 D S_X^-1 V^T."""
     W = np.asarray(W, dtype=np.float64)
     HX = np.asarray(HX, dtype=np.float64)
     HG = np.asarray(HG, dtype=np.float64)
@@ -198,8 +213,12 @@ def biip(W, HX, HG, sign_u, sign_v):
     HGs = HG / sg[:, None] / sg[None, :]
     U = rht_matrix(d_out, sign_u)
     V = rht_matrix(d_in, sign_v)
-    return {"W": U @ Ws @ V.T, "HX": V @ HXs @ V.T, "HG": U @ HGs @ U.T,
-            "s_x": sx, "s_g": sg, "U": U, "V": V}
+    out = {"W": U @ Ws @ V.T, "HX": V @ HXs @ V.T, "HG": U @ HGs @ U.T,
+           "s_x": sx, "s_g": sg, "U": U, "V": V}
+    if D is not None:
+        Ds = np.asarray(D, dtype=np.float64) / sx[:, None] / sx[None, :]
+        out["D"] = V @ Ds @ V.T
+    return out
 
 
 # ----------------------------------------------------------------------------------
@@ -225,6 +244,18 @@ def lower_factor(Hd: np.ndarray) -> np.ndarray:
     return inverse_cholesky_upper(Hd).T
 
 
+def gptaq_p(Dp: np.ndarray, L: np.ndarray, alpha: float) -> np.ndarray:
+    """The GPTAQ correction of Proposition 1 and Algorithm 2:
+    P = alpha ((D' L) o M_U) L^T, with D' the rescaled, rotated drift statistic, L the
+    lower factor of the damped H^-1 = L L^T and M_U the strictly upper-triangular mask.
+    P is strictly upper triangular."""
+    Dp = np.asarray(Dp, dtype=np.float64)
+    L = np.asarray(L, dtype=np.float64)
+    n = L.shape[0]
+    M_U = np.triu(np.ones((n, n)), 1)
+    return alpha * ((Dp @ L) * M_U) @ L.T
+
+
 # ----------------------------------------------------------------------------------
 # Stage 4: quantizer and the blocked OBS sweep (Eq. obs_update, Algorithm 2 with P = 0).
 # ----------------------------------------------------------------------------------
@@ -247,17 +278,21 @@ def quantize(w, scale, zero, bits):
     return np.clip(np.rint(np.asarray(w, np.float64) / scale) + zero, 0, 2 ** bits - 1)
 
 
-def obs_sweep(Wp: np.ndarray, R: np.ndarray, bits: int, group: int, block: int):
-    """Column-wise OBS sweep of Algorithm 2 in GPTQ mode (no P term).
+def obs_sweep(Wp: np.ndarray, R: np.ndarray, bits: int, group: int, block: int, P=None):
+    """Column-wise OBS sweep of Algorithm 2; GPTQ mode when P is None.
 
     For each block [i, e): for j in the block, quantize column j, E_j = (w_j - w^_j)/R_jj,
-    update the rest of the block by -E_j R[j, j+1:e]; then the lazy trailing update
-    W[:, e:] -= E_blk R[i:e, e:]. Returns codes, scale, zero (per row or per group)
-    and E for every column (the per-column loss is sum over rows of E^2), and pre_q,
-    the value of each column just before it is quantized.
+    update the rest of the block by -E_j R[j, j+1:e] + w_j P[j, j+1:e]; then the lazy
+    trailing update W[:, e:] -= E_blk R[i:e, e:] - Wpre_blk P[i:e, e:], where w_j and Wpre
+    are the columns' values just before they were quantized (Proposition 1's W_{:,p}).
+    Returns codes, scale, zero (per row or per group) and E for every column (the
+    per-column loss is sum over rows of E^2), and pre_q, the value of each column just
+    before it is quantized.
     """
     W = np.array(Wp, dtype=np.float64, copy=True)
     R = np.asarray(R, dtype=np.float64)
+    if P is not None:
+        P = np.asarray(P, dtype=np.float64)
     m, n = W.shape
     if group not in (0, block):
         raise ValueError("group must be 0 (per row) or equal to the block size")
@@ -284,8 +319,12 @@ def obs_sweep(Wp: np.ndarray, R: np.ndarray, bits: int, group: int, block: int):
             what = scale[:, gidx] * (q - zero[:, gidx])
             E[:, j] = (w - what) / R[j, j]
             W[:, j + 1:e] -= np.outer(E[:, j], R[j, j + 1:e])
+            if P is not None:
+                W[:, j + 1:e] += np.outer(pre_q[:, j], P[j, j + 1:e])
         if e < n:
             W[:, e:] -= E[:, i:e] @ R[i:e, e:]
+            if P is not None:
+                W[:, e:] += pre_q[:, i:e] @ P[i:e, e:]
     return {"codes": codes, "scale": scale, "zero": zero, "E": E, "pre_q": pre_q}
 
 
@@ -311,6 +350,18 @@ def proxy_loss(W, What, HX, HG) -> float:
     return float(np.trace(np.asarray(HG, np.float64) @ dW @ np.asarray(HX, np.float64) @ dW.T))
 
 
+def objective(W, What, HX, HG, D=None) -> float:
+    """The full objective of Eq. (kronq_full): tr[H_G (dW H_X dW^T + 2 W D dW^T)], dW = W - W^,
+    D = Delta X X^T (the second term is absent when D is None)."""
+    W = np.asarray(W, np.float64)
+    dW = W - np.asarray(What, np.float64)
+    HG = np.asarray(HG, np.float64)
+    val = np.trace(HG @ dW @ np.asarray(HX, np.float64) @ dW.T)
+    if D is not None:
+        val += 2.0 * np.trace(HG @ W @ np.asarray(D, np.float64) @ dW.T)
+    return float(val)
+
+
 def traces(HX, HG, HXp, HGp) -> dict:
     """Sensitivity s = tr(H_G) tr(H_X) (Eq. sensitivity), raw and after BiIP."""
     tx, tg = float(np.trace(HX)), float(np.trace(HG))
@@ -320,14 +371,17 @@ def traces(HX, HG, HXp, HGp) -> dict:
 
 
 def pipeline(X, G, W, sign_u, sign_v, bits: int, group: int, block: int = 128,
-             lam: float = 0.01) -> dict:
-    """Algorithms 1 and 2 end to end (GPTQ mode, X-tilde = X), all in float64."""
+             lam: float = 0.01, Xt=None, alpha: float = 0.25) -> dict:
+    """Algorithms 1 and 2 end to end, all in float64: GPTQ mode when Xt (X~) is None,
+    else with the GPTAQ drift correction P of scaling alpha."""
     HX = accum_factor(X)
     HG = accum_factor(G)
-    b = biip(W, HX, HG, sign_u, sign_v)
+    D = None if Xt is None else drift_factor(Xt, X)
+    b = biip(W, HX, HG, sign_u, sign_v, D)
     Hd = damp(b["HX"], lam)
     R = inverse_cholesky_upper(Hd)
-    sw = obs_sweep(b["W"], R, bits, group, block)
+    P = None if D is None else gptaq_p(b["D"], R.T, alpha)
+    sw = obs_sweep(b["W"], R, bits, group, block, P)
     Qp = dequant(sw["codes"], sw["scale"], sw["zero"], group)
     What = revert(Qp, b["s_x"], b["s_g"], b["U"], b["V"])
     out = {"HX": HX, "HG": HG, "Wp": b["W"], "HXp": b["HX"], "HGp": b["HG"],
@@ -335,6 +389,8 @@ def pipeline(X, G, W, sign_u, sign_v, bits: int, group: int, block: int = 128,
            "What": What, "loss": proxy_loss(W, What, HX, HG),
            "loss_rot": proxy_loss(b["W"], Qp, b["HX"], b["HG"]),
            "col_loss": np.sum(sw["E"] ** 2, axis=0)}
+    if D is not None:
+        out.update({"D": D, "Dp": b["D"], "P": P, "objective": objective(W, What, HX, HG, D)})
     out.update(sw)
     out.update(traces(HX, HG, b["HX"], b["HG"]))
     return out

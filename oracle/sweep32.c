@@ -1,7 +1,8 @@
 /*
- * fp32-ordered OBS sweep: the oracle's statement of Algorithm 2 (GPTQ mode, no P term;
- * Eq. obs_update) with every float32 operation and its order written out, so that a
- * float32 implementation that follows the same order gives the same bits.
+ * fp32-ordered OBS sweep: the oracle's statement of Algorithm 2 (Eq. obs_update; with
+ * the GPTAQ correction P of Proposition 1 when Pt is given) with every float32 operation
+ * and its order written out, so that a float32 implementation that follows the same
+ * order gives the same bits.
  *
  * TEST INFRASTRUCTURE ONLY: called by the tests and the benchmark's CPU-baseline leg,
  * never by the product path. Compiled with -ffp-contract=off; division is the IEEE
@@ -14,10 +15,14 @@
  *   column j:   q = clamp(rintf(w / scale) + zero, 0, 2^b - 1)
  *               what = scale * (q - zero);  E = (w - what) / R_jj
  *               w_k = fmaf(-E, R_jk, w_k) for k = j+1 .. block end - 1
+ *               with P:  w_k = fmaf(w, P_jk, fmaf(-E, R_jk, w_k)), w = column j's value
+ *               before it was quantized
  *   after the block [i, e): for each column c >= e:
  *               acc = 0; acc = fmaf(E_k, R_kc, acc) for k = i .. e-1 (ascending)
+ *               with P, continuing: acc = fmaf(-wpre_k, P_kc, acc) for k = i .. e-1
  *               w_c = w_c - acc
- * R is read from Lt = R^T (row-major, lower), R_jk = Lt[k * n + j].
+ * R is read from Lt = R^T (row-major, lower), R_jk = Lt[k * n + j]; P from Pt = P^T
+ * (row-major, strictly lower), P_jk = Pt[k * n + j].
  */
 #include <math.h>
 #include <stdint.h>
@@ -39,8 +44,9 @@ static void grid(const float *x, int64_t len, int bits, float *scale, float *zer
 }
 
 /* One row of the sweep. w: the row (n floats, updated in place as the sweep goes). */
-static void sweep_row(float *w, const float *Lt, int64_t n, int bits, int group, int block,
-                      uint8_t *codes, float *scale, float *zero, float *E, float *pre_q)
+static void sweep_row(float *w, const float *Lt, const float *Pt, int64_t n, int bits, int group,
+                      int block, uint8_t *codes, float *scale, float *zero, float *E, float *pre_q,
+                      float *wpre)
 {
     float maxq = (float)((1 << bits) - 1);
     float s = 0.0f, z = 0.0f;
@@ -59,6 +65,7 @@ static void sweep_row(float *w, const float *Lt, int64_t n, int bits, int group,
         for (int64_t j = i; j < e; ++j) {
             float wj = w[j];
             if (pre_q) pre_q[j] = wj;
+            wpre[j - i] = wj;
             float q = rintf(wj / s) + z;
             if (q < 0.0f) q = 0.0f;
             if (q > maxq) q = maxq;
@@ -66,13 +73,21 @@ static void sweep_row(float *w, const float *Lt, int64_t n, int bits, int group,
             float what = s * (q - z);
             float err = (wj - what) / Lt[j * n + j];
             E[j] = err;
-            for (int64_t k = j + 1; k < e; ++k)
-                w[k] = fmaf(-err, Lt[k * n + j], w[k]);
+            if (Pt) {
+                for (int64_t k = j + 1; k < e; ++k)
+                    w[k] = fmaf(wj, Pt[k * n + j], fmaf(-err, Lt[k * n + j], w[k]));
+            } else {
+                for (int64_t k = j + 1; k < e; ++k)
+                    w[k] = fmaf(-err, Lt[k * n + j], w[k]);
+            }
         }
         for (int64_t c = e; c < n; ++c) {
             float acc = 0.0f;
             for (int64_t k = i; k < e; ++k)
                 acc = fmaf(E[k], Lt[c * n + k], acc);
+            if (Pt)
+                for (int64_t k = i; k < e; ++k)
+                    acc = fmaf(-wpre[k - i], Pt[c * n + k], acc);
             w[c] = w[c] - acc;
         }
     }
@@ -80,12 +95,13 @@ static void sweep_row(float *w, const float *Lt, int64_t n, int bits, int group,
 
 /*
  * Sweep the rows listed in `rows` (nrows of them; NULL = rows 0..nrows-1) of W [m x n].
- * Outputs are indexed by position in the row list: codes/E/pre_q [nrows x n],
- * scale/zero [nrows x ngroups]. W itself is not modified. Returns 0, or -1 on bad args.
+ * Pt = P^T (NULL: GPTQ mode, no drift correction). Outputs are indexed by position in the
+ * row list: codes/E/pre_q [nrows x n], scale/zero [nrows x ngroups]. W itself is not
+ * modified. Returns 0, or -1 on bad args.
  */
-int kqref_sweep32(const float *W, int64_t m, int64_t n, const float *Lt, int bits, int group,
-                  int block, const int64_t *rows, int64_t nrows, uint8_t *codes, float *scale,
-                  float *zero, float *E, float *pre_q)
+int kqref_sweep32(const float *W, int64_t m, int64_t n, const float *Lt, const float *Pt, int bits,
+                  int group, int block, const int64_t *rows, int64_t nrows, uint8_t *codes,
+                  float *scale, float *zero, float *E, float *pre_q)
 {
     if (bits < 1 || bits > 8 || block < 1 || (group != 0 && group != block) || n < 1)
         return -1;
@@ -95,11 +111,11 @@ int kqref_sweep32(const float *W, int64_t m, int64_t n, const float *Lt, int bit
     for (int64_t t = 0; t < nrows; ++t) {
         int64_t r = rows ? rows[t] : t;
         if (r < 0 || r >= m) { bad = 1; continue; }
-        float *w = (float *)malloc((size_t)n * sizeof(float));
+        float *w = (float *)malloc((size_t)(n + block) * sizeof(float));
         if (!w) { bad = 1; continue; }
         memcpy(w, W + r * n, (size_t)n * sizeof(float));
-        sweep_row(w, Lt, n, bits, group, block, codes + t * n, scale + t * ngroups,
-                  zero + t * ngroups, E + t * n, pre_q ? pre_q + t * n : NULL);
+        sweep_row(w, Lt, Pt, n, bits, group, block, codes + t * n, scale + t * ngroups,
+                  zero + t * ngroups, E + t * n, pre_q ? pre_q + t * n : NULL, w + n);
         free(w);
     }
     return bad ? -1 : 0;

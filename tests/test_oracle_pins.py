@@ -400,3 +400,135 @@ def test_fp32_sweep_row_subset():
     part = obs_sweep_fp32(W, Lt, 3, 16, 16, rows=rows)
     assert np.array_equal(part["codes"], full["codes"][rows])
     assert np.array_equal(part["E"], full["E"][rows])
+
+
+# ---------------------------------------------------------------- GPTAQ drift correction
+def _drift_problem(seed, T=60, n=10, m=3, drift=0.1):
+    """Tiny layer with a drifted full-precision input: X, X~, and the damped H as the
+    Gram matrix of X with sqrt(delta) I appended (X~ gets the same rows, so they carry no
+    drift): H = X_aug^T X_aug = X^T X + delta I."""
+    rng = _rng(seed)
+    sc = np.exp(rng.standard_normal(n))
+    X = rng.standard_normal((T, n)) * sc
+    Xt = X + drift * rng.standard_normal((T, n)) * sc
+    delta = 0.01 * np.mean(np.diag(X.T @ X))
+    X_aug = np.vstack([X, np.sqrt(delta) * np.eye(n)])
+    dX_aug = np.vstack([Xt - X, np.zeros((n, n))])
+    H = ref.damp(X.T @ X, 0.01)
+    W = rng.standard_normal((m, n)) * 0.05
+    return X, Xt, X_aug, dX_aug, H, W
+
+
+def test_drift_factor_brute_force_integers():
+    """Delta X X^T of Algorithm 1 with tokens as rows: D[a, b] = sum_t (x~_t[a] - x_t[a]) x_t[b],
+    by Python integer loops (D is not symmetric)."""
+    rng = _rng(31)
+    T, d = 23, 5
+    X = rng.integers(-9, 10, size=(T, d))
+    Xt = X + rng.integers(-3, 4, size=(T, d))
+    D = ref.drift_factor(Xt.astype(np.float64), X.astype(np.float64))
+    brute = [[sum(int(Xt[t, a] - X[t, a]) * int(X[t, b]) for t in range(T)) for b in range(d)]
+             for a in range(d)]
+    assert np.array_equal(D, np.array(brute, dtype=np.float64))
+    assert not np.array_equal(D, D.T)
+
+
+def test_p_rows_are_least_squares_projection_of_drift():
+    """GPTAQ's sequential residual reading of Prop. 1: row p of P (alpha = 1) holds the
+    least-squares coefficients of column p's drift Delta x_p on the later columns x_{p+1:},
+    i.e. P[p, p+1:] = D[p, p+1:] H[p+1:, p+1:]^-1; P is strictly upper triangular and
+    linear in alpha."""
+    X, Xt, X_aug, dX_aug, H, _ = _drift_problem(41, n=12)
+    n = H.shape[0]
+    L = ref.lower_factor(H)
+    P = ref.gptaq_p(ref.drift_factor(Xt, X), L, 1.0)
+    assert np.all(np.tril(P) == 0)
+    for p in range(n - 1):
+        c, *_ = np.linalg.lstsq(X_aug[:, p + 1:], dX_aug[:, p], rcond=None)
+        assert np.allclose(P[p, p + 1:], c, rtol=1e-9, atol=1e-12)
+    P4 = ref.gptaq_p(ref.drift_factor(Xt, X), L, 0.25)
+    assert np.allclose(P4, 0.25 * P, rtol=1e-12, atol=0)
+
+
+@pytest.mark.parametrize("block", [3, 4, 16])
+def test_sweep_with_p_is_sequential_residual_compensation(block):
+    """Algorithm 2 with P (alpha = 1, per-row grid), blocked with a lazy trailing update,
+    equals the column-by-column compensation of Prop. 1 restated as least squares: after
+    quantizing column p, the later columns absorb the residual x_p (w_p - w^_p) + Delta x_p w_p
+    (w_p the column's value just before quantization) by a least-squares fit on x_{p+1:}."""
+    X, Xt, X_aug, dX_aug, H, W = _drift_problem(43, n=10)
+    n = H.shape[0]
+    R = ref.inverse_cholesky_upper(H)
+    P = ref.gptaq_p(ref.drift_factor(Xt, X), R.T, 1.0)
+    bits = 3
+    sw = ref.obs_sweep(W, R, bits, 0, block, P)
+    for r in range(W.shape[0]):
+        s, z = ref.quant_params(W[r:r + 1], bits)
+        v = W[r].copy()
+        for p in range(n):
+            assert np.isclose(sw["pre_q"][r, p], v[p], rtol=1e-9, atol=1e-12)
+            q = ref.quantize(v[p], s[0], z[0], bits)
+            assert sw["codes"][r, p] == q
+            what = s[0] * (q - z[0])
+            if p + 1 < n:
+                resid = X_aug[:, p] * (v[p] - what) + dX_aug[:, p] * v[p]
+                c, *_ = np.linalg.lstsq(X_aug[:, p + 1:], resid, rcond=None)
+                v[p + 1:] += c
+
+
+def test_zero_drift_gives_gptq_sweep():
+    """X~ = X: D = 0, P = 0 and the sweep is the GPTQ-mode sweep, code for code."""
+    cfg = kqsynth.CONFIGS["tiny256"].replace(d_in=32, d_out=28, T=300)
+    L = kqsynth.layer(cfg)
+    a = ref.pipeline(L["X"], L["G"], L["W"], L["sign_u"], L["sign_v"], 3, 16, 16)
+    b = ref.pipeline(L["X"], L["G"], L["W"], L["sign_u"], L["sign_v"], 3, 16, 16, Xt=L["X"])
+    assert np.all(b["D"] == 0) and np.all(b["P"] == 0)
+    assert np.array_equal(a["codes"], b["codes"])
+
+
+def test_theorem1_invariance_with_drift_term():
+    """Theorem 1 (both terms, appendix proof): the full objective of Eq. (kronq_full) is the
+    same in the original space and after BiIP, with D carried as V S_X^-1 D S_X^-1 V^T."""
+    cfg = kqsynth.CONFIGS["tiny256"].replace(d_in=32, d_out=28, T=300)
+    L = kqsynth.layer(cfg)
+    Xt = kqsynth.fp_activations(cfg, L["X"])
+    HX, HG = ref.accum_factor(L["X"]), ref.accum_factor(L["G"])
+    D = ref.drift_factor(Xt, L["X"])
+    W = L["W"].astype(np.float64)
+    What = W + _rng(3).standard_normal(W.shape) * 0.01
+    b = ref.biip(W, HX, HG, L["sign_u"], L["sign_v"], D)
+    Whatp = b["U"] @ (b["s_g"][:, None] * What * b["s_x"][None, :]) @ b["V"].T
+    j0 = ref.objective(W, What, HX, HG, D)
+    j1 = ref.objective(b["W"], Whatp, b["HX"], b["HG"], b["D"])
+    assert np.isclose(j0, j1, rtol=1e-9)
+    # the drift term is really present: dropping it changes the value
+    assert not np.isclose(j0, ref.objective(W, What, HX, HG), rtol=1e-6)
+    # and the plain expansion of Eq. (gptaq_obj) with H_G = I: ||W X~^T - W^ X^T||^2 minus the
+    # constant ||W (X~ - X)^T||^2
+    Xd, Xtd = L["X"].astype(np.float64), Xt.astype(np.float64)
+    full = np.sum((W @ Xtd.T - What @ Xd.T) ** 2) - np.sum((W @ (Xtd - Xd).T) ** 2)
+    assert np.isclose(ref.objective(W, What, HX, np.eye(W.shape[0]), D), full, rtol=1e-9)
+
+
+@pytest.mark.parametrize("group", [0, 32])
+def test_fp32_sweep_with_p_matches_fp64_off_ties(group):
+    """The fp32-ordered sweep with P agrees with the fp64 sweep wherever the decision is
+    not within fp32 noise of a rounding tie."""
+    X, Xt, _, _, H, _ = _drift_problem(47, T=400, n=64)
+    R = ref.inverse_cholesky_upper(H)
+    P = ref.gptaq_p(ref.drift_factor(Xt, X), R.T, 0.25)
+    R32, P32 = R.astype(np.float32), P.astype(np.float32)
+    W32 = (_rng(8).standard_normal((40, 64)) * 0.02).astype(np.float32)
+    s64 = ref.obs_sweep(W32.astype(np.float64), R32.astype(np.float64), 4, group, 32,
+                        P32.astype(np.float64))
+    s32 = obs_sweep_fp32(W32, R32.T, 4, group, 32, Pt=P32.T)
+    diff = s64["codes"] != s32["codes"]
+    for r in np.nonzero(diff.any(1))[0]:
+        j = np.argmax(diff[r])
+        g = 0 if group == 0 else j // group
+        t = s64["pre_q"][r, j] / s64["scale"][r, g]
+        assert abs(abs(t - np.floor(t)) - 0.5) < 1e-3
+    assert diff.mean() < 0.02
+    # P really changes the result
+    s0 = obs_sweep_fp32(W32, R32.T, 4, group, 32)
+    assert not np.array_equal(s0["codes"], s32["codes"])
