@@ -48,7 +48,14 @@ def parse():
                     help="token chunk of the H_G accumulation (0: one call)")
     ap.add_argument("--trailing", default="3xtf32", choices=["fp32", "3xtf32"],
                     help="sweep trailing update: fp32-ordered SIMT (bit-exact) or 3xTF32 tensor cores")
+    ap.add_argument("--drift", type=float, default=None, metavar="ALPHA",
+                    help="with the GPTAQ drift correction of scaling ALPHA (full-precision input X~ = "
+                         "X + 0.1 sigma z); default: GPTQ mode")
     return ap.parse_args()
+
+
+def metric_of(alpha) -> str:
+    return METRIC if alpha is None else "ms per linear layer (factors+drift+rotate+chol+P+OBS sweep)"
 
 
 def workload_name(cfg) -> str:
@@ -57,18 +64,26 @@ def workload_name(cfg) -> str:
             f"damp {cfg.damp}")
 
 
-def config_dict(cfg, x_chunk: int = 0, g_chunk: int = 0, trailing: str = "3xtf32") -> dict:
-    return {"workload": workload_name(cfg), "d_out": cfg.d_out, "d_in": cfg.d_in, "T": cfg.T,
-            "bits": cfg.bits, "group": cfg.group, "block": cfg.block, "damp": cfg.damp,
-            "factor_chunk_tokens": {"X": x_chunk, "G": g_chunk}, "sweep_trailing_update": trailing,
-            "l2": "inputs larger than L2 (X and G are T x d bf16, >= 1 GiB each); no flush"}
+def config_dict(cfg, x_chunk: int = 0, g_chunk: int = 0, trailing: str = "3xtf32", alpha=None) -> dict:
+    d = {"workload": workload_name(cfg), "d_out": cfg.d_out, "d_in": cfg.d_in, "T": cfg.T,
+         "bits": cfg.bits, "group": cfg.group, "block": cfg.block, "damp": cfg.damp,
+         "factor_chunk_tokens": {"X": x_chunk, "G": g_chunk}, "sweep_trailing_update": trailing,
+         "l2": "inputs larger than L2 (X and G are T x d bf16, >= 1 GiB each); no flush"}
+    if alpha is not None:
+        d["workload"] += f" + GPTAQ drift correction (alpha {alpha}, X~ = X + 0.1 sigma z)"
+        d["drift_alpha"] = alpha
+    return d
 
 
-def algorithmic_flops(cfg) -> dict:
-    return {"factor_x": cfg.T * cfg.d_in * (cfg.d_in + 1),
-            "factor_g": cfg.T * cfg.d_out * (cfg.d_out + 1),
-            "chol": 2 * cfg.d_in ** 3 / 3,
-            "sweep": cfg.d_out * cfg.d_in * max(cfg.d_in - cfg.block, 0)}
+def algorithmic_flops(cfg, drift: bool = False) -> dict:
+    fl = {"factor_x": cfg.T * cfg.d_in * (cfg.d_in + 1),
+          "factor_g": cfg.T * cfg.d_out * (cfg.d_out + 1),
+          "chol": 2 * cfg.d_in ** 3 / 3,
+          "sweep": cfg.d_out * cfg.d_in * max(cfg.d_in - cfg.block, 0) * (2 if drift else 1)}
+    if drift:
+        fl["drift"] = 2 * cfg.T * cfg.d_in ** 2       # (X~ - X)^T X
+        fl["p"] = 2 * cfg.d_in ** 3 / 3               # two triangular products
+    return fl
 
 
 def measured_peaks():
@@ -152,7 +167,7 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------- CPU oracle timing
-def oracle_sample_ms(cfg, repeats: int = 1, T_s: int = 4096, f: int = 2, rows_s: int = 128) -> dict:
+def oracle_sample_ms(cfg, repeats: int = 1, T_s: int = 4096, f: int = 2, rows_s: int = 128, alpha=None) -> dict:
     """Time the oracle on a bounded sample of the workload and extrapolate each stage to
     the full layer by its cost model: the factors run on T_s of the T tokens at full width
     (linear in tokens); BiIP, Cholesky and the fp32-ordered sweep run on a layer shrunk by
@@ -168,25 +183,43 @@ def oracle_sample_ms(cfg, repeats: int = 1, T_s: int = 4096, f: int = 2, rows_s:
     rows_s = min(sub.d_out, rows_s)
     L = kqsynth.layer(cfg.replace(T=T_s))
     Ls = kqsynth.layer(sub)
+    drift = alpha is not None
+    if drift:
+        Xt = kqsynth.fp_activations(cfg, L["X"])
+        Xts = kqsynth.fp_activations(sub, Ls["X"])
     stage = {"factors": [], "biip": [], "chol": [], "sweep": []}
+    if drift:
+        stage.update({"drift": [], "p": []})
     for _ in range(repeats):
         t0 = time.perf_counter()
         HX = ref.accum_factor(L["X"])
         HG = ref.accum_factor(L["G"])
         t1 = time.perf_counter()
         stage["factors"].append((t1 - t0) * cfg.T / T_s)
+        Ds = None
+        if drift:
+            t1 = time.perf_counter()
+            ref.drift_factor(Xt, L["X"])
+            stage["drift"].append((time.perf_counter() - t1) * cfg.T / T_s)
+            Ds = ref.drift_factor(Xts, Ls["X"])
         HXs, HGs = ref.accum_factor(Ls["X"]), ref.accum_factor(Ls["G"])
         t1 = time.perf_counter()
-        b = ref.biip(Ls["W"], HXs, HGs, Ls["sign_u"], Ls["sign_v"])
+        b = ref.biip(Ls["W"], HXs, HGs, Ls["sign_u"], Ls["sign_v"], Ds)
         t2 = time.perf_counter()
         stage["biip"].append((t2 - t1) * f ** 3)
         R = ref.inverse_cholesky_upper(ref.damp(b["HX"], cfg.damp))
         t3 = time.perf_counter()
         stage["chol"].append((t3 - t2) * f ** 3)
+        Pt = None
+        if drift:
+            P = ref.gptaq_p(b["D"], R.T, alpha)
+            t3b = time.perf_counter()
+            stage["p"].append((t3b - t3) * f ** 3)
+            Pt = P.T.astype("float32")
         Wp = b["W"][:rows_s].astype("float32")
         Lt = R.T.astype("float32")
         t4 = time.perf_counter()
-        oracle.obs_sweep_fp32(Wp, Lt, cfg.bits, cfg.group, cfg.block)
+        oracle.obs_sweep_fp32(Wp, Lt, cfg.bits, cfg.group, cfg.block, Pt=Pt)
         t5 = time.perf_counter()
         stage["sweep"].append((t5 - t4) * (cfg.d_out / rows_s) * f ** 2)
         del HX, HG, HXs, HGs, b, R
@@ -196,7 +229,9 @@ def oracle_sample_ms(cfg, repeats: int = 1, T_s: int = 4096, f: int = 2, rows_s:
             "sample": (f"factors on {T_s} of {cfg.T} tokens at full width (x{cfg.T / T_s:g}); BiIP dense "
                        f"products, Cholesky and fp32-ordered sweep ({rows_s} rows) on the "
                        f"{sub.d_out}x{sub.d_in} layer (x{f}^3, x{f}^3, x{f}^2*{cfg.d_out / rows_s:g}); "
-                       f"{repeats} repeat(s), mean")}
+                       f"{repeats} repeat(s), mean" + ("; drift statistic on the same tokens as the "
+                                                        "factors, P on the shrunk layer (x" + str(f) + "^3)"
+                                                        if drift else ""))}
 
 
 # --------------------------------------------------------------------- distributed
@@ -226,7 +261,7 @@ def run_reference(args):
     cfg = kqsynth.CONFIGS[args.config]
     if rank != 0:
         return
-    small = dict(T_s=2048, f=4, rows_s=64)
+    small = dict(T_s=2048, f=4, rows_s=64, alpha=args.drift)
     for _ in range(args.warmup):
         oracle_sample_ms(cfg, **small)
     vals, last = [], None
@@ -236,10 +271,10 @@ def run_reference(args):
         vals.append(last["value"])
     wall = time.perf_counter() - t0
     v = statistics.mean(vals)
-    out = {"impl": "reference", "metric": METRIC, "value": v, "unit": "ms", "n_gpus": args.gpus,
+    out = {"impl": "reference", "metric": metric_of(args.drift), "value": v, "unit": "ms", "n_gpus": args.gpus,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": v, "higher_is_better": False,
            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-           "config": config_dict(cfg, args.x_chunk_tokens, args.g_chunk_tokens, args.trailing),
+           "config": config_dict(cfg, args.x_chunk_tokens, args.g_chunk_tokens, args.trailing, args.drift),
            "cpu_baseline": {"value": v, "unit": "ms", "cores": last["cores"], "kind": "oracle",
                             "sample": last["sample"], "stages_ms": last["stages_ms"]},
            "e2e": {"value": v, "unit": "ms", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -254,15 +289,18 @@ def run_ours(args):
     ws, rank, local = dist_setup("nccl")
     kbuild.build()
     from paper_2607_07964_gb300 import kronq as kq
-    from paper_2607_07964_gb300.pipeline import STAGES, LayerPipeline
+    from paper_2607_07964_gb300.pipeline import LayerPipeline
 
     torch.cuda.set_device(local)
     dev = f"cuda:{local}"
     cfg = kqsynth.CONFIGS[args.config].replace(seed=rank)
     inp = kqsynth.device_layer(cfg, device=dev)
+    drift = args.drift is not None
+    Xt = kqsynth.device_fp_activations(cfg, inp["X"]) if drift else None
     p = LayerPipeline(cfg.d_out, cfg.d_in, cfg.bits, cfg.group, cfg.block, cfg.damp, device=dev,
                       x_chunk_tokens=args.x_chunk_tokens, g_chunk_tokens=args.g_chunk_tokens,
-                      trailing=args.trailing)
+                      trailing=args.trailing, alpha=args.drift)
+    STAGES = p.stages
     stream = torch.cuda.current_stream()
 
     def barrier():
@@ -270,7 +308,7 @@ def run_ours(args):
             torch.distributed.barrier()
 
     for _ in range(args.warmup):
-        p.run(inp["X"], inp["G"], inp["W"], inp["sign_u"], inp["sign_v"], stream=stream)
+        p.run(inp["X"], inp["G"], inp["W"], inp["sign_u"], inp["sign_v"], stream=stream, Xt=Xt)
     p.check(stream)
 
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -280,7 +318,7 @@ def run_ours(args):
     torch.cuda.synchronize()
     graph = None
     if not args.no_graph:
-        graph, per_step = p.capture(inp["X"], inp["G"], inp["W"], inp["sign_u"], inp["sign_v"])
+        graph, per_step = p.capture(inp["X"], inp["G"], inp["W"], inp["sign_u"], inp["sign_v"], Xt=Xt)
         for _ in range(2):
             graph.replay()
         torch.cuda.synchronize()
@@ -292,7 +330,7 @@ def run_ours(args):
         if graph is not None:
             graph.replay()
         else:
-            p.run(inp["X"], inp["G"], inp["W"], inp["sign_u"], inp["sign_v"], stream=stream)
+            p.run(inp["X"], inp["G"], inp["W"], inp["sign_u"], inp["sign_v"], stream=stream, Xt=Xt)
     t_end.record(stream)
     torch.cuda.synchronize()
     barrier()
@@ -305,16 +343,19 @@ def run_ours(args):
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(len(STAGES) + 1)] for _ in range(args.steps)]
     torch.cuda.synchronize()
     for k in range(args.steps):
-        p.run(inp["X"], inp["G"], inp["W"], inp["sign_u"], inp["sign_v"], stream=stream, events=evs[k])
+        p.run(inp["X"], inp["G"], inp["W"], inp["sign_u"], inp["sign_v"], stream=stream, events=evs[k], Xt=Xt)
     torch.cuda.synchronize()
     p.check(stream)
     stage_ms = {name: statistics.mean(evs[k][i].elapsed_time(evs[k][i + 1]) for k in range(args.steps))
                 for i, name in enumerate(STAGES)}
-    fl = algorithmic_flops(cfg)
+    fl = algorithmic_flops(cfg, drift)
     tflops = {"factor_x": fl["factor_x"] / stage_ms["factor_x"] / 1e9,
               "factor_g": fl["factor_g"] / stage_ms["factor_g"] / 1e9,
               "chol": fl["chol"] / stage_ms["chol"] / 1e9,
               "sweep_trailing": fl["sweep"] / stage_ms["sweep"] / 1e9}
+    if drift:
+        tflops["drift"] = fl["drift"] / stage_ms["drift"] / 1e9
+        tflops["p"] = fl["p"] / stage_ms["p"] / 1e9
     peaks, peak_src = measured_peaks()
     peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
     # factor_x is one SYRK launch per token chunk: flops per launch / mean launch time.
@@ -325,17 +366,27 @@ def run_ours(args):
                 "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak, "traffic": traffic,
                 "peak_source": f"{peak_src} bf16 dense burst",
                 "algorithmic_flops_per_launch": fl["factor_x"] / n_launch, "launches_per_factor": n_launch}
+    if drift:
+        # the drift stage (one split pass + one drift_tc_kernel launch with K = 2 T): algorithmic
+        # flops of (X~ - X)^T X over the stage time; the split pair executes twice as many
+        a = tflops["drift"]
+        roofline = {"kernel": "drift stage (drift_split_kernel + drift_tc_kernel, D = (X~ - X)^T X)",
+                    "bound": "tensor", "achieved": a, "peak": peak, "unit": "TFLOP/s", "frac": a / peak,
+                    "traffic": None, "peak_source": f"{peak_src} bf16 dense burst",
+                    "algorithmic_flops_per_launch": fl["drift"], "executed_flops_per_launch": 2 * fl["drift"],
+                    "executed_frac": 2 * a / peak, "syrk_h_x": roofline}
 
     e2e = None
     if not args.no_e2e:
         Xh = inp["X"].cpu().pin_memory()
+        Xth = Xt.cpu().pin_memory() if drift else None
         Gh = inp["G"].cpu().pin_memory()
         Wh = inp["W"].cpu().pin_memory()
         suh, svh = inp["sign_u"].cpu().pin_memory(), inp["sign_v"].cpu().pin_memory()
         ch = torch.empty(p.codes.shape, dtype=p.codes.dtype).pin_memory()
         sh = torch.empty(p.scale.shape, dtype=p.scale.dtype).pin_memory()
         zh = torch.empty(p.zero.shape, dtype=p.zero.dtype).pin_memory()
-        p.run_host(Xh, Gh, Wh, suh, svh, ch, sh, zh, stream=stream)
+        p.run_host(Xh, Gh, Wh, suh, svh, ch, sh, zh, stream=stream, Xt_h=Xth)
         torch.cuda.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         barrier()
@@ -343,7 +394,7 @@ def run_ours(args):
         e0.record(stream)
         nin = nout = 0
         for _ in range(args.steps):
-            nin, nout = p.run_host(Xh, Gh, Wh, suh, svh, ch, sh, zh, stream=stream)
+            nin, nout = p.run_host(Xh, Gh, Wh, suh, svh, ch, sh, zh, stream=stream, Xt_h=Xth)
         e1.record(stream)
         torch.cuda.synchronize()
         barrier()
@@ -353,14 +404,15 @@ def run_ours(args):
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        cpu = oracle_sample_ms(cfg, repeats=2)
+        cpu = oracle_sample_ms(cfg, repeats=2, alpha=args.drift)
 
     if rank == 0:
-        out = {"metric": METRIC, "value": total_ms / (ws * args.steps), "unit": "ms", "n_gpus": ws,
+        out = {"metric": metric_of(args.drift), "value": total_ms / (ws * args.steps), "unit": "ms", "n_gpus": ws,
                "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
                "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
                "dtype": "bf16 products, f32 accumulate/arithmetic", "data": "synthetic",
-               "config": config_dict(cfg, args.x_chunk_tokens, args.g_chunk_tokens, args.trailing), "stages_ms": stage_ms, "tflops": tflops,
+               "config": config_dict(cfg, args.x_chunk_tokens, args.g_chunk_tokens, args.trailing, args.drift),
+               "stages_ms": stage_ms, "tflops": tflops,
                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
                "launch_mode": "cuda graph replay (one graph per layer, two streams)" if graph is not None
                else "direct launches (two streams)",

@@ -8,7 +8,9 @@
  *                                                              kq_rotate_in, kq_rotate_out)
  *   3. damped inverse Cholesky                                (kq_chol_inv)
  *   4. column-wise OBS sweep with b-bit asymmetric grids      (kq_obs_quantize)
- * plus two check-only calls (kq_dequant_revert, kq_proxy_loss).
+ * with the GPTAQ drift correction as an option (kq_accum_drift, kq_gptaq_p, and the Pt
+ * argument of kq_obs_quantize), plus two check-only calls (kq_dequant_revert,
+ * kq_proxy_loss).
  *
  * Conventions shared by every call
  *   - Tokens are rows: X is [T x d_in], G is [T x d_out]; the paper stacks tokens as
@@ -100,6 +102,32 @@ KQ_API kq_status kq_selftest_timeout(int* info, int64_t limit_us, kq_stream_t st
 #define KQ_SYRK_CHUNK_TOKENS 512
 KQ_API kq_status kq_accum_factor(const uint16_t* A, int64_t T, int64_t d, int64_t lda, float* H,
                           int accumulate, double* trace, int* info, kq_stream_t stream);
+
+/* ------------------------------------------------------------------------------------
+ * GPTAQ drift statistic (optional; the full objective of Sec. 3.1 Eq. kronq_full).
+ * Paper: Sec. 2.1 Eq. (gptaq_obj) (Delta X = X~ - X, X~ the full-precision model's input to
+ * the layer, X the running quantized model's); Algorithm 1 computes Delta X X^T online.
+ *
+ * kq_accum_drift: D (+)= (X~ - X)^T X for X~, X [T x d] bf16 (row t = token t, common row
+ *   stride `ld` elements); D [d x d] fp32 row-major, D[a][b] = sum_t (x~_t[a] - x_t[a]) x_t[b]
+ *   (not symmetric). The drift is split exactly into a bf16 pair hi + lo (x~ - x is exact
+ *   in fp32; the pair holds it to 16 significant bits, exactly unless the two exponents are
+ *   more than 8 apart), and D = hi^T X + lo^T X runs on the tensor cores (bf16 products,
+ *   exact in fp32; fp32 sums drained every KQ_SYRK_CHUNK_TOKENS tokens).
+ *   accumulate = 0 overwrites D, 1 adds to it. Requirements: X~, X 16-byte aligned,
+ *   d % 8 == 0, ld % 8 == 0, ld >= d, 1 <= d <= 65536, 0 <= T < 2^31. T == 0 gives D = 0
+ *   (accumulate = 0) or leaves D unchanged.
+ *   ws (256-byte aligned) holds the split drift of a chunk of tokens: with
+ *   kq_accum_drift_workspace(T, d) bytes all T tokens go through one pass; a smaller ws
+ *   (at least 4 * d * 64 bytes) processes the tokens in chunks of what it holds.
+ *   info (nullable): -KQ_ERR_TIMEOUT if a pipeline wait gave up.
+ * The drift statistic is rescaled and rotated like H_X (Algorithm 1): pass D as the
+ * H_X argument of kq_rotate_in (W = NULL, dir = KQ_FWD) to get D' = V S_X^-1 D S_X^-1 V^T.
+ * ---------------------------------------------------------------------------------- */
+KQ_API size_t kq_accum_drift_workspace(int64_t T, int64_t d);
+KQ_API kq_status kq_accum_drift(const uint16_t* Xt, const uint16_t* X, int64_t T, int64_t d, int64_t ld,
+                                float* D, int accumulate, int* info, void* ws, size_t ws_bytes,
+                                kq_stream_t stream);
 
 /* ------------------------------------------------------------------------------------
  * Stage 2: bidirectional incoherence processing.
@@ -204,15 +232,37 @@ KQ_API kq_status kq_chol_inv_noalloc(const float* H, int64_t n, float damp_rel, 
                                      kq_stream_t stream);
 
 /* ------------------------------------------------------------------------------------
- * Stage 4: column-wise OBS sweep (GPTQ mode; the GPTAQ drift term P is zero).
+ * GPTAQ correction matrix (optional).
+ * Paper: Proposition 1 and Algorithm 2: P = alpha ((D' L) o M_U) L^T with D' the rescaled,
+ * rotated drift statistic, H^-1 = L L^T (L from kq_chol_inv of the damped H_X') and M_U
+ * the strictly upper-triangular mask. Row p of P (alpha = 1) holds the least-squares
+ * coefficients of column p's drift on the later columns.
+ *
+ * kq_gptaq_p: Pt [n x n] fp32 row-major receives P^T (strictly lower triangular; the upper
+ *   triangle and the diagonal are written as 0). Dp = D' [n x n], Lt = L [n x n] row-major
+ *   (lower; its strict upper triangle must be 0, as kq_chol_inv leaves it). Both triangular
+ *   products run on the tensor cores with the 3xTF32 split (fp32-accurate products, fp32
+ *   sums). Requirements: n % 4 == 0, 1 <= n <= 65536, Dp and Lt 16-byte aligned.
+ *   ws: kq_gptaq_p_workspace(n) bytes (6 n^2 floats), 256-byte aligned.
+ *   info (nullable): -KQ_ERR_TIMEOUT if a pipeline wait gave up.
+ * ---------------------------------------------------------------------------------- */
+KQ_API size_t kq_gptaq_p_workspace(int64_t n);
+KQ_API kq_status kq_gptaq_p(const float* Dp, const float* Lt, int64_t n, float alpha, float* Pt, int* info,
+                            void* ws, size_t ws_bytes, kq_stream_t stream);
+
+/* ------------------------------------------------------------------------------------
+ * Stage 4: column-wise OBS sweep, GPTQ mode (Pt = NULL) or with the GPTAQ correction P.
  * Paper: Sec. 2.1 Eq. (obs_update); Algorithm 2's inner column loop and lazy trailing
- * update; Proposition 1 (H_G cancels, so the sweep reads only L).
+ * update; Proposition 1 (H_G cancels, so the sweep reads only L, and P with the drift).
  *
  * kq_obs_quantize: W [d_out x d_in] fp32 (the rotated, rescaled W'; destroyed), Lt from
- *   kq_chol_inv. For each block of `block` columns and each column j of it:
+ *   kq_chol_inv, Pt from kq_gptaq_p or NULL. For each block of `block` columns and each
+ *   column j of it:
  *     q_j = clamp(rint(w_j / scale) + zero, 0, 2^bits - 1)        (round half to even)
  *     E_j = (w_j - scale * (q_j - zero)) / R_jj,  w_k -= E_j R_jk for k in (j, block end)
- *   then W[:, block end:] -= E_block R[block, block end:].
+ *     with P:  w_k += w_j P_jk as well (w_j = column j's value just before quantization)
+ *   then W[:, block end:] -= E_block R[block, block end:]
+ *     with P:  W[:, block end:] += Wpre_block P[block, block end:] as well.
  *   Grid (asymmetric min-max): xmin = min(0, min x), xmax = max(0, max x), (-1, 1) if both
  *   are 0; scale = (xmax - xmin) / (2^bits - 1); zero = rint(-xmin / scale).
  *   group = 0: one grid per row from the whole row before the sweep (scale/zero [d_out]).
@@ -223,26 +273,29 @@ KQ_API kq_status kq_chol_inv_noalloc(const float* H, int64_t n, float damp_rel, 
  *   w_j just before it was quantized.
  *   mode selects the arithmetic of the lazy trailing update (the column loop is the same):
  *   KQ_TRAIL_FP32: every fp32 operation and its order are fixed (IEEE division, rintf, one
- *     fmaf per intra-block update; trailing update as acc = fmaf(E_k, R_kc, acc) over
- *     ascending k, then w_c - acc), so results are reproducible bit for bit and equal to
- *     the fp32-ordered definition.
+ *     fmaf per intra-block update, with P w_k = fmaf(w_j, P_jk, fmaf(-E_j, R_jk, w_k));
+ *     trailing update as acc = fmaf(E_k, R_kc, acc) over ascending k, with P continuing
+ *     acc = fmaf(-wpre_k, P_kc, acc) over ascending k, then w_c - acc), so results are
+ *     reproducible bit for bit and equal to the fp32-ordered definition.
  *   KQ_TRAIL_3XTF32: the trailing update runs on the tensor cores with the 3xTF32 split
  *     (E R ~= E_hi R_hi + E_hi R_lo + E_lo R_hi, hi = rounded to tf32, lo = the exact
  *     remainder; fp32 accumulation). Its sums differ from the fp32 order in the last bits,
  *     so a code can differ from the fp32-ordered definition where w / scale falls on a
  *     rounding tie, and the rest of that row then follows a slightly different error path.
  *     Needs d_in % 4 == 0 and a 16-byte aligned W.
- *   Requirements: 1 <= bits <= 8, block == 128, group in {0, block}.
+ *   Requirements: 1 <= bits <= 8, block == 128, group in {0, block}; with P also
+ *   d_in % 16 == 0 and W, codes, Pt 16-byte aligned.
  *   info (nullable, device int): -KQ_ERR_TIMEOUT if a tensor-core pipeline wait gave up.
- *   ws: kq_obs_quantize_workspace(d_out, d_in, block, mode) bytes, 256-byte aligned.
+ *   ws: kq_obs_quantize_workspace(d_out, d_in, block, mode, with_p) bytes (with_p = 1 when
+ *   Pt will be passed), 256-byte aligned.
  * ---------------------------------------------------------------------------------- */
 #define KQ_TRAIL_FP32 0
 #define KQ_TRAIL_3XTF32 1
-KQ_API size_t kq_obs_quantize_workspace(int64_t d_out, int64_t d_in, int block, int mode);
-KQ_API kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, const float* Lt, int bits,
-                                 int group, int block, int mode, uint8_t* codes, float* scale, int32_t* zero,
-                                 float* col_loss, float* pre_q, int* info, void* ws, size_t ws_bytes,
-                                 kq_stream_t stream);
+KQ_API size_t kq_obs_quantize_workspace(int64_t d_out, int64_t d_in, int block, int mode, int with_p);
+KQ_API kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, const float* Lt, const float* Pt,
+                                 int bits, int group, int block, int mode, uint8_t* codes, float* scale,
+                                 int32_t* zero, float* col_loss, float* pre_q, int* info, void* ws,
+                                 size_t ws_bytes, kq_stream_t stream);
 
 /* ------------------------------------------------------------------------------------
  * Check-only calls (not part of the timed path).

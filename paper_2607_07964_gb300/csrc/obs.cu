@@ -1,16 +1,20 @@
-// Stage 4: the column-wise OBS sweep with b-bit asymmetric grids (GPTQ mode).
+// Stage 4: the column-wise OBS sweep with b-bit asymmetric grids.
 //
 // Paper: Sec. 2.1 Eq. (obs_update) (compensation -(w_p - q_p)/[H^-1]_pp [H^-1]_{p,p+1:}),
 // Algorithm 2 (inner column loop over a block of B columns with error E, then the lazy
 // trailing update W[:, i+B:] -= E R[i:i+B, i+B:]), Proposition 1 (H_G cancels, so only
-// L = R^T enters). The GPTAQ drift term P is zero here (one input set, X-tilde = X).
+// L = R^T enters). With the GPTAQ correction P (Proposition 1, Algorithm 2) each column j
+// also adds w_j P[j, k] to the later columns k, w_j being column j's value just before it
+// is quantized; the lazy update then subtracts [E | -Wpre] [R ; P]. GPTQ mode: no P.
 //
 // Every fp32 operation is written with an explicit round-to-nearest intrinsic so the
 // compiler cannot contract or reorder it; the order is:
 //   grid      scale = (xmax - xmin) / (2^b - 1), zero = rint(-xmin / scale)
 //   column j  q = clamp(rint(w / scale) + zero, 0, 2^b - 1); what = scale * (q - zero)
 //             E = (w - what) / R_jj;  w_k = fma(-E, R_jk, w_k) for k in (j, block end)
-//   trailing  acc = fma(E_k, R_kc, acc) over ascending k; w_c = w_c - acc
+//             with P: w_k = fma(w_j, P_jk, fma(-E, R_jk, w_k))
+//   trailing  acc = fma(E_k, R_kc, acc) over ascending k; with P continuing
+//             acc = fma(-wpre_k, P_kc, acc) over ascending k; w_c = w_c - acc
 // Kernels:
 //   rowgrid_kernel   per-row grid (group = 0) from the whole row before the sweep
 //   pack_r_kernel    the diagonal 128 x 128 blocks of R in the block kernel's layout
@@ -97,6 +101,10 @@ constexpr int NV = CPL / 4;                 // float4 slots per lane
 static_assert(LPR == 8 || LPR == 16, "lanes per row must be 8 or 16");
 constexpr int OBS_ROWS = 16;                // rows per CTA
 constexpr int OBS_THREADS = OBS_ROWS * LPR; // 128 or 256
+// With P the CTA holds both diagonal blocks (R and P, 128 KB), so one CTA fits an SM; it
+// takes twice the rows to keep as many warps per SM.
+constexpr int OBS_ROWS_P = 2 * OBS_ROWS;
+constexpr int OBS_THREADS_P = OBS_ROWS_P * LPR;
 
 // Packed layout of one diagonal block of R: row j holds R[i0 + j][i0 + c] at pos(c). The
 // CPL columns of lane lp fill slots [lp NV, lp NV + NV) of 16 bytes, rotated by lane so
@@ -154,15 +162,21 @@ __device__ __forceinline__ void load_cols(const float* __restrict__ W, int64_t r
 }
 
 // VEC: d_in % 16 == 0 and W, codes (and pre_q) 16-byte aligned, so a lane's CPL columns
-// of W, E and codes move as 16-byte vectors.
-template <bool VEC>
-__global__ void __launch_bounds__(OBS_THREADS, 3) obs_block_kernel(
+// of W, E and codes move as 16-byte vectors. HASP: with the GPTAQ correction; Pp is P's
+// diagonal block packed like R's, and the block's -Wpre goes to Q (fp32 trailing update)
+// or to Qh + Ql (tensor-core trailing update).
+template <bool VEC, bool HASP>
+__global__ void __launch_bounds__(HASP ? OBS_THREADS_P : OBS_THREADS, HASP ? 1 : 3) obs_block_kernel(
     const float* __restrict__ W, int64_t d_out, int64_t d_in, const float* __restrict__ Rp, int64_t i0,
     int bits, int group, const float* __restrict__ gscale, const float* __restrict__ gzero,
     uint8_t* __restrict__ codes, float* __restrict__ scale, int32_t* __restrict__ zero,
-    float* __restrict__ E, float* __restrict__ pre_q, float* __restrict__ Eh, float* __restrict__ El) {
-    extern __shared__ __align__(16) float Rs[];   // [BLK][BLK], packed (pack_r_kernel)
+    float* __restrict__ E, float* __restrict__ pre_q, float* __restrict__ Eh, float* __restrict__ El,
+    const float* __restrict__ Pp, float* __restrict__ Q, float* __restrict__ Qh, float* __restrict__ Ql) {
+    extern __shared__ __align__(16) float Rs[];   // [BLK][BLK], packed (pack_r_kernel); then P's
+    float* Ps = Rs + BLK * BLK;
     for (int e = threadIdx.x; e < BLK * BLK / 4; e += blockDim.x) cp_async16(Rs + 4 * e, Rp + 4 * e, 16);
+    if (HASP)
+        for (int e = threadIdx.x; e < BLK * BLK / 4; e += blockDim.x) cp_async16(Ps + 4 * e, Pp + 4 * e, 16);
     cp_async_commit();
     const int nb = static_cast<int>(min(static_cast<int64_t>(BLK), d_in - i0));
     const float maxq = static_cast<float>((1 << bits) - 1);
@@ -207,6 +221,7 @@ __global__ void __launch_bounds__(OBS_THREADS, 3) obs_block_kernel(
         for (int o = 0; o < LPR; ++o) {
             if (CPL * o >= nb) break;   // uniform across the CTA
             float e[CPL];
+            float wq[HASP ? CPL : 1];
             uint32_t cq[NV];
 #pragma unroll
             for (int v = 0; v < NV; ++v) cq[v] = 0u;
@@ -228,13 +243,30 @@ __global__ void __launch_bounds__(OBS_THREADS, 3) obs_block_kernel(
                     e[jj] = err;
                     cq[jj >> 2] |= static_cast<uint32_t>(qq) << (8 * (jj & 3));
                     if (pre_q && live && lp == o) pre_q[r * d_in + i0 + j] = wj;
+                    if constexpr (HASP) {
+                        wq[jj] = wj;
+                        const float* pr = Ps + j * BLK;
+                        float4 pv[NV];
 #pragma unroll
-                    for (int v = 0; v < NV; ++v) {
-                        w[4 * v] = __fmaf_rn(-err, rv[v].x, w[4 * v]);
-                        w[4 * v + 1] = __fmaf_rn(-err, rv[v].y, w[4 * v + 1]);
-                        w[4 * v + 2] = __fmaf_rn(-err, rv[v].z, w[4 * v + 2]);
-                        w[4 * v + 3] = __fmaf_rn(-err, rv[v].w, w[4 * v + 3]);
+                        for (int v = 0; v < NV; ++v) pv[v] = *reinterpret_cast<const float4*>(pr + 4 * slot_of(lp, v));
+#pragma unroll
+                        for (int v = 0; v < NV; ++v) {
+                            w[4 * v] = __fmaf_rn(wj, pv[v].x, __fmaf_rn(-err, rv[v].x, w[4 * v]));
+                            w[4 * v + 1] = __fmaf_rn(wj, pv[v].y, __fmaf_rn(-err, rv[v].y, w[4 * v + 1]));
+                            w[4 * v + 2] = __fmaf_rn(wj, pv[v].z, __fmaf_rn(-err, rv[v].z, w[4 * v + 2]));
+                            w[4 * v + 3] = __fmaf_rn(wj, pv[v].w, __fmaf_rn(-err, rv[v].w, w[4 * v + 3]));
+                        }
+                    } else {
+#pragma unroll
+                        for (int v = 0; v < NV; ++v) {
+                            w[4 * v] = __fmaf_rn(-err, rv[v].x, w[4 * v]);
+                            w[4 * v + 1] = __fmaf_rn(-err, rv[v].y, w[4 * v + 1]);
+                            w[4 * v + 2] = __fmaf_rn(-err, rv[v].z, w[4 * v + 2]);
+                            w[4 * v + 3] = __fmaf_rn(-err, rv[v].w, w[4 * v + 3]);
+                        }
                     }
+                } else if constexpr (HASP) {
+                    wq[jj] = 0.0f;
                 }
             }
             if (live && lp == o) {
@@ -261,6 +293,26 @@ __global__ void __launch_bounds__(OBS_THREADS, 3) obs_block_kernel(
                             reinterpret_cast<float4*>(El + ob)[v] = make_float4(l[0], l[1], l[2], l[3]);
                         }
                     }
+                    if constexpr (HASP) {   // -Wpre of the block, for the trailing update
+                        if (Qh) {
+#pragma unroll
+                            for (int v = 0; v < NV; ++v) {
+                                float h[4], l[4];
+#pragma unroll
+                                for (int t = 0; t < 4; ++t) {
+                                    h[t] = tf32_hi(-wq[4 * v + t]);
+                                    l[t] = -wq[4 * v + t] - h[t];
+                                }
+                                reinterpret_cast<float4*>(Qh + ob)[v] = make_float4(h[0], h[1], h[2], h[3]);
+                                reinterpret_cast<float4*>(Ql + ob)[v] = make_float4(l[0], l[1], l[2], l[3]);
+                            }
+                        } else {
+#pragma unroll
+                            for (int v = 0; v < NV; ++v)
+                                reinterpret_cast<float4*>(Q + ob)[v] =
+                                    make_float4(-wq[4 * v], -wq[4 * v + 1], -wq[4 * v + 2], -wq[4 * v + 3]);
+                        }
+                    }
                 } else {
 #pragma unroll
                     for (int t = 0; t < CPL; ++t)
@@ -272,6 +324,15 @@ __global__ void __launch_bounds__(OBS_THREADS, 3) obs_block_kernel(
                                 Eh[ob + t] = h;
                                 El[ob + t] = e[t] - h;
                             }
+                            if constexpr (HASP) {
+                                if (Qh) {
+                                    const float h = tf32_hi(-wq[t]);
+                                    Qh[ob + t] = h;
+                                    Ql[ob + t] = -wq[t] - h;
+                                } else {
+                                    Q[ob + t] = -wq[t];
+                                }
+                            }
                         }
                 }
             }
@@ -281,11 +342,13 @@ __global__ void __launch_bounds__(OBS_THREADS, 3) obs_block_kernel(
 
 // W[:, cb:ce] -= E[:, i0:i0+kb] R[i0:i0+kb, cb:ce] with R[k][c] = Lt[c][k]: 128 x 128 output
 // tiles of the shared tile GEMM (acc = fma(E_k, R_kc, acc) over ascending k), then w = w - acc.
+// With P (Q = -Wpre, P[k][c] = Pt[c][k]) the sum continues with acc = fma(Q_k, P_kc, acc).
 template <bool VEC>
 __global__ void __launch_bounds__(G_THREADS, 2) trailing_kernel(float* __restrict__ W, const float* __restrict__ E,
                                                                 const float* __restrict__ Lt, int64_t d_out,
                                                                 int64_t d_in, int64_t i0, int kb, int64_t cb,
-                                                                int64_t ce) {
+                                                                int64_t ce, const float* __restrict__ Q,
+                                                                const float* __restrict__ Pt) {
     extern __shared__ __align__(16) float sm[];
     const int64_t r0 = static_cast<int64_t>(blockIdx.y) * GT;
     const int64_t c0 = cb + static_cast<int64_t>(blockIdx.x) * GT;
@@ -293,6 +356,7 @@ __global__ void __launch_bounds__(G_THREADS, 2) trailing_kernel(float* __restric
     const int bcols = static_cast<int>(min(static_cast<int64_t>(GT), ce - c0));
     float acc[8][8];
     gemm_tile<false, VEC>(E + r0 * d_in + i0, d_in, arows, Lt + c0 * d_in + i0, d_in, bcols, kb, acc, sm);
+    if (Pt) gemm_tile<false, VEC, false>(Q + r0 * d_in + i0, d_in, arows, Pt + c0 * d_in + i0, d_in, bcols, kb, acc, sm);
     const int ty = threadIdx.x >> 4, tx = threadIdx.x & 15;
     // Read-modify-write of W in two halves of 32 values, all loads of a half issued before
     // its stores, so the memory latency is paid twice rather than 64 times.
@@ -334,6 +398,12 @@ struct ObsWs {
     float* El;
     float* Lh;
     float* Ll;
+    float* Pp;      // with P: packed diagonal blocks of P; -Wpre [d_out x d_in] (fp32 mode)
+    float* Q;
+    float* Qh;      // with P, tensor-core mode: (-Wpre)_hi, _lo [d_out x d_in], Pt_hi, Pt_lo
+    float* Ql;
+    float* Ph;
+    float* Pl;
 };
 
 inline size_t align256(size_t b) { return (b + 255) & ~static_cast<size_t>(255); }
@@ -343,29 +413,59 @@ size_t ws_base_bytes(int64_t d_out, int64_t d_in) {
                      2 * static_cast<size_t>(d_out)) * sizeof(float));
 }
 
-size_t ws_bytes_of(int64_t d_out, int64_t d_in, int mode) {
-    size_t b = ws_base_bytes(d_out, d_in);
-    if (mode == KQ_TRAIL_3XTF32)
-        b += 2 * align256(static_cast<size_t>(d_out) * d_in * sizeof(float)) +
-             2 * align256(static_cast<size_t>(d_in) * d_in * sizeof(float));
+// Byte sizes of the parts in carve order.
+struct WsParts {
+    size_t base, blk, wide, sq;
+};
+WsParts parts_of(int64_t d_out, int64_t d_in) {
+    WsParts p;
+    p.base = ws_base_bytes(d_out, d_in);
+    p.blk = align256(static_cast<size_t>(cdiv(d_in, BLK)) * BLK * BLK * sizeof(float));
+    p.wide = align256(static_cast<size_t>(d_out) * d_in * sizeof(float));
+    p.sq = align256(static_cast<size_t>(d_in) * d_in * sizeof(float));
+    return p;
+}
+
+size_t ws_bytes_of(int64_t d_out, int64_t d_in, int mode, bool with_p) {
+    const WsParts p = parts_of(d_out, d_in);
+    const bool tc = mode == KQ_TRAIL_3XTF32;
+    size_t b = p.base;
+    if (tc) b += 2 * p.wide + 2 * p.sq;
+    if (with_p) b += p.blk + (tc ? 2 * p.wide + 2 * p.sq : p.wide);
     return b + 256;
 }
 
-ObsWs carve(void* ws, int64_t d_out, int64_t d_in, int mode) {
+ObsWs carve(void* ws, int64_t d_out, int64_t d_in, int mode, bool with_p) {
+    const WsParts sz = parts_of(d_out, d_in);
+    const bool tc = mode == KQ_TRAIL_3XTF32;
     ObsWs o;
     o.Rp = static_cast<float*>(ws);
     o.E = o.Rp + cdiv(d_in, BLK) * BLK * BLK;
     o.gscale = o.E + d_out * d_in;
     o.gzero = o.gscale + d_out;
-    o.Eh = o.El = o.Lh = o.Ll = nullptr;
-    if (mode == KQ_TRAIL_3XTF32) {
-        uint8_t* p = static_cast<uint8_t*>(ws) + ws_base_bytes(d_out, d_in);
-        const size_t eb = align256(static_cast<size_t>(d_out) * d_in * sizeof(float));
-        const size_t lb = align256(static_cast<size_t>(d_in) * d_in * sizeof(float));
-        o.Eh = reinterpret_cast<float*>(p);
-        o.El = reinterpret_cast<float*>(p + eb);
-        o.Lh = reinterpret_cast<float*>(p + 2 * eb);
-        o.Ll = reinterpret_cast<float*>(p + 2 * eb + lb);
+    o.Eh = o.El = o.Lh = o.Ll = o.Pp = o.Q = o.Qh = o.Ql = o.Ph = o.Pl = nullptr;
+    uint8_t* p = static_cast<uint8_t*>(ws) + sz.base;
+    auto take = [&](size_t bytes) {
+        float* f = reinterpret_cast<float*>(p);
+        p += bytes;
+        return f;
+    };
+    if (tc) {
+        o.Eh = take(sz.wide);
+        o.El = take(sz.wide);
+        o.Lh = take(sz.sq);
+        o.Ll = take(sz.sq);
+    }
+    if (with_p) {
+        o.Pp = take(sz.blk);
+        if (tc) {
+            o.Qh = take(sz.wide);
+            o.Ql = take(sz.wide);
+            o.Ph = take(sz.sq);
+            o.Pl = take(sz.sq);
+        } else {
+            o.Q = take(sz.wide);
+        }
     }
     return o;
 }
@@ -375,16 +475,16 @@ ObsWs carve(void* ws, int64_t d_out, int64_t d_in, int mode) {
 
 using namespace kq;
 
-extern "C" size_t kq_obs_quantize_workspace(int64_t d_out, int64_t d_in, int block, int mode) {
+extern "C" size_t kq_obs_quantize_workspace(int64_t d_out, int64_t d_in, int block, int mode, int with_p) {
     (void)block;
     if (d_out < 1 || d_in < 1 || (mode != KQ_TRAIL_FP32 && mode != KQ_TRAIL_3XTF32)) return 0;
-    return ws_bytes_of(d_out, d_in, mode);
+    return ws_bytes_of(d_out, d_in, mode, with_p != 0);
 }
 
-extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, const float* Lt, int bits,
-                                     int group, int block, int mode, uint8_t* codes, float* scale, int32_t* zero,
-                                     float* col_loss, float* pre_q, int* info, void* ws, size_t ws_bytes,
-                                     kq_stream_t stream_) {
+extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, const float* Lt, const float* Pt,
+                                     int bits, int group, int block, int mode, uint8_t* codes, float* scale,
+                                     int32_t* zero, float* col_loss, float* pre_q, int* info, void* ws,
+                                     size_t ws_bytes, kq_stream_t stream_) {
     cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
     if (!W || !Lt || !codes || !scale || !zero || d_out < 1 || d_in < 1 || bits < 1 || bits > 8) {
         set_error("kq_obs_quantize: invalid arguments");
@@ -399,34 +499,46 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
         return KQ_ERR_INVALID_ARG;
     }
     const bool tc = mode == KQ_TRAIL_3XTF32;
+    const bool hp = Pt != nullptr;
     if (tc && ((d_in % 4) != 0 || (reinterpret_cast<uintptr_t>(W) & 15u) != 0)) {
         set_error("kq_obs_quantize: the tensor-core trailing update needs d_in %% 4 == 0 and a 16-byte aligned W");
         return KQ_ERR_UNSUPPORTED;
     }
-    if (!ws || ws_bytes < ws_bytes_of(d_out, d_in, mode) || (reinterpret_cast<uintptr_t>(ws) & 255u)) {
+    if (hp && ((d_in % 16) != 0 || (reinterpret_cast<uintptr_t>(W) & 15u) || (reinterpret_cast<uintptr_t>(codes) & 15u) ||
+               (reinterpret_cast<uintptr_t>(Pt) & 15u))) {
+        set_error("kq_obs_quantize: the drift correction needs d_in %% 16 == 0 and 16-byte aligned W, codes, Pt");
+        return KQ_ERR_UNSUPPORTED;
+    }
+    if (!ws || ws_bytes < ws_bytes_of(d_out, d_in, mode, hp) || (reinterpret_cast<uintptr_t>(ws) & 255u)) {
         set_error("kq_obs_quantize: workspace must be 256-byte aligned and hold %zu bytes",
-                  ws_bytes_of(d_out, d_in, mode));
+                  ws_bytes_of(d_out, d_in, mode, hp));
         return KQ_ERR_WORKSPACE;
     }
     static bool attr = false;
     if (!attr) {
-        KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      BLK * BLK * 4));
-        KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      BLK * BLK * 4));
+        KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     2 * BLK * BLK * 4));
         KQ_CUDA(cudaFuncSetAttribute(trailing_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(G_SMEM)));
         KQ_CUDA(cudaFuncSetAttribute(trailing_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(G_SMEM)));
         attr = true;
     }
-    ObsWs o = carve(ws, d_out, d_in, mode);
+    ObsWs o = carve(ws, d_out, d_in, mode, hp);
     TrailMaps maps;
     if (tc) {
         kq_status st0 = split_tf32(Lt, d_in * d_in, o.Lh, o.Ll, stream);
         if (st0 != KQ_OK) return st0;
         if ((st0 = maps.init(o.Eh, o.El, o.Lh, o.Ll, d_out, d_in)) != KQ_OK) return st0;
         if ((st0 = maps.set_w(W, d_out, d_in)) != KQ_OK) return st0;
+        if (hp) {
+            if ((st0 = split_tf32(Pt, d_in * d_in, o.Ph, o.Pl, stream)) != KQ_OK) return st0;
+            if ((st0 = maps.init_p(o.Qh, o.Ql, o.Ph, o.Pl, d_out, d_in)) != KQ_OK) return st0;
+        }
     }
     if (group == 0) {
         rowgrid_kernel<<<static_cast<unsigned>(cdiv(d_out, 8)), 256, 0, stream>>>(W, d_out, d_in, bits, scale,
@@ -436,10 +548,15 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
     const int64_t nblk = cdiv(d_in, BLK);
     pack_r_kernel<<<dim3(BLK / 32, BLK / 32, static_cast<unsigned>(nblk)), dim3(32, 8), 0, stream>>>(Lt, d_in, o.Rp);
     KQ_LAUNCH_CHECK("pack_r_kernel");
+    if (hp) {   // P[i0 + j][i0 + c] = Pt[i0 + c][i0 + j]: the same packing as R from Lt
+        pack_r_kernel<<<dim3(BLK / 32, BLK / 32, static_cast<unsigned>(nblk)), dim3(32, 8), 0, stream>>>(Pt, d_in, o.Pp);
+        KQ_LAUNCH_CHECK("pack_r_kernel");
+    }
     const bool vec = (d_in % 4 == 0) && (reinterpret_cast<uintptr_t>(Lt) % 16 == 0);
     const bool bvec = (d_in % 16 == 0) && (reinterpret_cast<uintptr_t>(W) % 16 == 0) &&
                       (reinterpret_cast<uintptr_t>(codes) % 16 == 0);
-    const int64_t row_ctas = std::min<int64_t>(cdiv(d_out, OBS_ROWS), static_cast<int64_t>(num_sms()) * 3);
+    const int64_t row_ctas = hp ? std::min<int64_t>(cdiv(d_out, OBS_ROWS_P), static_cast<int64_t>(num_sms()))
+                                : std::min<int64_t>(cdiv(d_out, OBS_ROWS), static_cast<int64_t>(num_sms()) * 3);
     // Look-ahead: after block b, the update of block column b + 1 runs on the caller's stream
     // (the next block kernel waits for it); the columns beyond run on a library side stream
     // beside block b + 1. Every column still receives the block updates in block order
@@ -448,24 +565,30 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
     SideStream* side = nblk > 2 ? side_stream(stream) : nullptr;
     bool forked = false;
     auto trailing = [&](int64_t i0, int kb, int64_t cb, int64_t ce, cudaStream_t st) -> kq_status {
-        if (tc) return trail_tc(maps, W, d_out, d_in, i0, cb, ce, info, st);
+        if (tc) return trail_tc(maps, W, d_out, d_in, i0, cb, ce, hp, info, st);
         dim3 grid(static_cast<unsigned>(cdiv(ce - cb, GT)), static_cast<unsigned>(cdiv(d_out, GT)));
         if (vec)
-            trailing_kernel<true><<<grid, G_THREADS, G_SMEM, st>>>(W, o.E, Lt, d_out, d_in, i0, kb, cb, ce);
+            trailing_kernel<true><<<grid, G_THREADS, G_SMEM, st>>>(W, o.E, Lt, d_out, d_in, i0, kb, cb, ce, o.Q, Pt);
         else
-            trailing_kernel<false><<<grid, G_THREADS, G_SMEM, st>>>(W, o.E, Lt, d_out, d_in, i0, kb, cb, ce);
+            trailing_kernel<false><<<grid, G_THREADS, G_SMEM, st>>>(W, o.E, Lt, d_out, d_in, i0, kb, cb, ce, o.Q, Pt);
         KQ_LAUNCH_CHECK("trailing_kernel");
         return KQ_OK;
     };
     for (int64_t i0 = 0; i0 < d_in; i0 += BLK) {
         const int kb = static_cast<int>(std::min<int64_t>(BLK, d_in - i0));
         const float* rp = o.Rp + (i0 / BLK) * BLK * BLK;
-        if (bvec)
-            obs_block_kernel<true><<<static_cast<unsigned>(row_ctas), OBS_THREADS, BLK * BLK * 4, stream>>>(
-                W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q, o.Eh, o.El);
+        if (hp)
+            obs_block_kernel<true, true><<<static_cast<unsigned>(row_ctas), OBS_THREADS_P, 2 * BLK * BLK * 4, stream>>>(
+                W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q, o.Eh, o.El,
+                o.Pp + (i0 / BLK) * BLK * BLK, o.Q, o.Qh, o.Ql);
+        else if (bvec)
+            obs_block_kernel<true, false><<<static_cast<unsigned>(row_ctas), OBS_THREADS, BLK * BLK * 4, stream>>>(
+                W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q, o.Eh, o.El,
+                nullptr, nullptr, nullptr, nullptr);
         else
-            obs_block_kernel<false><<<static_cast<unsigned>(row_ctas), OBS_THREADS, BLK * BLK * 4, stream>>>(
-                W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q, o.Eh, o.El);
+            obs_block_kernel<false, false><<<static_cast<unsigned>(row_ctas), OBS_THREADS, BLK * BLK * 4, stream>>>(
+                W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q, o.Eh, o.El,
+                nullptr, nullptr, nullptr, nullptr);
         KQ_LAUNCH_CHECK("obs_block_kernel");
         const int64_t nb0 = i0 + kb;                                // next block column
         if (nb0 >= d_in) break;

@@ -59,9 +59,16 @@ __device__ __forceinline__ bool wait_noabort(uint64_t* bar, uint32_t parity) {
     return mbar_wait(bar, parity, &dummy);
 }
 
-__global__ void __launch_bounds__(NUM_THREADS, 1)
-syrk_tc_kernel(const __grid_constant__ CUtensorMap tmap, float* __restrict__ H, int d, int T,
-               int n_row_tiles, int chunk_stages, int accumulate, int* info) {
+// The body shared by the two Gram products.
+//   CROSS = false (SYRK): H (+)= A^T A, lower 128 x 256 tiles mirrored on write-out; every
+//     operand box comes from map a0.
+//   CROSS = true: D (+)= (A_hi + A_lo)^T B over all tiles, no symmetry: the K loop runs over
+//     the T tokens of the pair (a0 = A_hi, b) and then over the pair (a1 = A_lo, b).
+template <bool CROSS>
+__device__ __forceinline__ void gram_tc_body(const CUtensorMap* a0, const CUtensorMap* a1,
+                                             const CUtensorMap* bmap, float* __restrict__ H, int d,
+                                             int T, int n_row_tiles, int chunk_stages, int accumulate,
+                                             int* info) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -76,10 +83,16 @@ syrk_tc_kernel(const __grid_constant__ CUtensorMap tmap, float* __restrict__ H, 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     int ti, tj;
-    tile_of(blockIdx.x, n_row_tiles, &ti, &tj);
+    if (CROSS) {
+        ti = static_cast<int>(blockIdx.x) % n_row_tiles;
+        tj = static_cast<int>(blockIdx.x) / n_row_tiles;
+    } else {
+        tile_of(blockIdx.x, n_row_tiles, &ti, &tj);
+    }
     const int i0 = ti * BM;
     const int j0 = tj * BN;
-    const int nk = (T + BK - 1) / BK;
+    const int nk1 = (T + BK - 1) / BK;          // stages per pass over the tokens
+    const int nk = CROSS ? 2 * nk1 : nk1;
     const int nchunks = (nk + chunk_stages - 1) / chunk_stages;
 
     if (threadIdx.x == 0) {
@@ -99,7 +112,13 @@ syrk_tc_kernel(const __grid_constant__ CUtensorMap tmap, float* __restrict__ H, 
         tmem_alloc(tmem_slot, TMEM_COLS);
         tmem_relinquish();
     }
-    if (warp == 0 && lane == 0) tma_prefetch_desc(&tmap);
+    if (warp == 0 && lane == 0) {
+        tma_prefetch_desc(a0);
+        if (CROSS) {
+            tma_prefetch_desc(a1);
+            tma_prefetch_desc(bmap);
+        }
+    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -116,12 +135,15 @@ syrk_tc_kernel(const __grid_constant__ CUtensorMap tmap, float* __restrict__ H, 
                 mbar_arrive_expect_tx(&full[s], STAGE_BYTES);
                 uint8_t* a = smem + s * STAGE_BYTES;
                 uint8_t* b = a + A_BYTES;
-                const int y = k * BK;
-                tma_load_2d(a, &tmap, &full[s], i0, y);
-                tma_load_2d(a + BOX_BYTES, &tmap, &full[s], i0 + 64, y);
+                const bool second = CROSS && k >= nk1;
+                const int y = (second ? k - nk1 : k) * BK;
+                const CUtensorMap* am = second ? a1 : a0;
+                const CUtensorMap* bm = CROSS ? bmap : a0;
+                tma_load_2d(a, am, &full[s], i0, y);
+                tma_load_2d(a + BOX_BYTES, am, &full[s], i0 + 64, y);
 #pragma unroll
                 for (int q = 0; q < 4; ++q)
-                    tma_load_2d(b + q * BOX_BYTES, &tmap, &full[s], j0 + 64 * q, y);
+                    tma_load_2d(b + q * BOX_BYTES, bm, &full[s], j0 + 64 * q, y);
                 issued = k + 1;
             }
             // Drain: every issued load must have landed before the CTA may exit.
@@ -217,7 +239,7 @@ syrk_tc_kernel(const __grid_constant__ CUtensorMap tmap, float* __restrict__ H, 
 #pragma unroll
                     for (int m = 0; m < 4; ++m) {
                         const int col = cbase + lane + 32 * m;
-                        old[u][m] = (accumulate && rr < d && col < d && col <= rr)
+                        old[u][m] = (accumulate && rr < d && col < d && (CROSS || col <= rr))
                                         ? H[static_cast<int64_t>(rr) * d + col] : 0.0f;
                     }
                 }
@@ -227,7 +249,7 @@ syrk_tc_kernel(const __grid_constant__ CUtensorMap tmap, float* __restrict__ H, 
 #pragma unroll
                     for (int m = 0; m < 4; ++m) {
                         const int col = cbase + lane + 32 * m;
-                        if (rr < d && col < d && col <= rr) {
+                        if (rr < d && col < d && (CROSS || col <= rr)) {
                             const float v = st[(r8 + u) * SLD + lane + 32 * m] + old[u][m];
                             H[static_cast<int64_t>(rr) * d + col] = v;
                             st[(r8 + u) * SLD + lane + 32 * m] = v;
@@ -236,7 +258,7 @@ syrk_tc_kernel(const __grid_constant__ CUtensorMap tmap, float* __restrict__ H, 
                 }
             }
             __syncwarp();
-            if (row < d) {
+            if (!CROSS && row < d) {
 #pragma unroll 4
                 for (int i = 0; i < 128; ++i) {
                     const int col = cbase + i;
@@ -251,6 +273,64 @@ syrk_tc_kernel(const __grid_constant__ CUtensorMap tmap, float* __restrict__ H, 
     if (warp == 1) {
         tc_fence_after();
         tmem_dealloc(tmem, TMEM_COLS);
+    }
+}
+
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+syrk_tc_kernel(const __grid_constant__ CUtensorMap tmap, float* __restrict__ H, int d, int T,
+               int n_row_tiles, int chunk_stages, int accumulate, int* info) {
+    gram_tc_body<false>(&tmap, &tmap, &tmap, H, d, T, n_row_tiles, chunk_stages, accumulate, info);
+}
+
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+drift_tc_kernel(const __grid_constant__ CUtensorMap a_hi, const __grid_constant__ CUtensorMap a_lo,
+                const __grid_constant__ CUtensorMap b, float* __restrict__ D, int d, int T,
+                int n_row_tiles, int chunk_stages, int accumulate, int* info) {
+    gram_tc_body<true>(&a_hi, &a_lo, &b, D, d, T, n_row_tiles, chunk_stages, accumulate, info);
+}
+
+// Round a finite fp32 value to the nearest bf16, ties to even; returns the 16 bf16 bits.
+__device__ __forceinline__ uint32_t bf16_rn_bits(float f) {
+    const uint32_t u = __float_as_uint(f);
+    return (u + 0x7fffu + ((u >> 16) & 1u)) >> 16;
+}
+
+// Exact split of the drift X~ - X into a bf16 pair: hi = bf16(x~ - x), lo = bf16((x~ - x) - hi).
+// x~ - x of two bf16 values is exact in fp32 (their significands have 8 bits), and hi + lo
+// carries 16 significant bits, which holds the difference exactly unless the two exponents
+// are more than 8 apart (then the pair is within 2^-17 of it). Eight elements per thread.
+__global__ void drift_split_kernel(const uint16_t* __restrict__ Xt, const uint16_t* __restrict__ X,
+                                   int64_t T, int64_t d, int64_t ld, uint16_t* __restrict__ hi,
+                                   uint16_t* __restrict__ lo) {
+    const int64_t per_row = d >> 3;
+    const int64_t total = T * per_row;
+    for (int64_t v = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; v < total;
+         v += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t t = v / per_row;
+        const int64_t c = (v - t * per_row) << 3;
+        const uint4 a = __ldg(reinterpret_cast<const uint4*>(Xt + t * ld + c));
+        const uint4 b = __ldg(reinterpret_cast<const uint4*>(X + t * ld + c));
+        const uint32_t aw[4] = {a.x, a.y, a.z, a.w};
+        const uint32_t bw[4] = {b.x, b.y, b.z, b.w};
+        uint32_t hw[4], lw[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            uint32_t h2 = 0, l2 = 0;
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                const float xa = __uint_as_float(((aw[q] >> (16 * e)) & 0xffffu) << 16);
+                const float xb = __uint_as_float(((bw[q] >> (16 * e)) & 0xffffu) << 16);
+                const float df = xa - xb;
+                const uint32_t h = bf16_rn_bits(df);
+                const uint32_t l = bf16_rn_bits(df - __uint_as_float(h << 16));
+                h2 |= h << (16 * e);
+                l2 |= l << (16 * e);
+            }
+            hw[q] = h2;
+            lw[q] = l2;
+        }
+        *reinterpret_cast<uint4*>(hi + t * d + c) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+        *reinterpret_cast<uint4*>(lo + t * d + c) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
     }
 }
 
@@ -287,6 +367,30 @@ EncodeTiledFn encode_fn() {
     return fn;
 }
 
+// 2D map over a [rows x d] bf16 matrix (row stride ld elements): 64-feature x BK-token
+// boxes, 128-byte swizzle, zero fill past the last row.
+kq_status make_bf16_map(CUtensorMap* m, const uint16_t* base, int64_t d, int64_t rows, int64_t ld,
+                        const char* who) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) {
+        set_error("%s: cuTensorMapEncodeTiled is unavailable", who);
+        return KQ_ERR_CUDA;
+    }
+    std::memset(m, 0, sizeof(*m));
+    cuuint64_t gdim[2] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(rows)};
+    cuuint64_t gstride[1] = {static_cast<cuuint64_t>(ld) * 2};
+    cuuint32_t box[2] = {64, static_cast<cuuint32_t>(BK)};
+    cuuint32_t estride[2] = {1, 1};
+    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<uint16_t*>(base), gdim, gstride,
+                     box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+        set_error("%s: cuTensorMapEncodeTiled failed (%d)", who, static_cast<int>(r));
+        return KQ_ERR_CUDA;
+    }
+    return KQ_OK;
+}
+
 }  // namespace
 
 kq_status launch_trace(const float* H, int64_t n, double* out, cudaStream_t stream) {
@@ -314,25 +418,9 @@ extern "C" kq_status kq_accum_factor(const uint16_t* A, int64_t T, int64_t d, in
     if (T == 0) {
         if (!accumulate) KQ_CUDA(cudaMemsetAsync(H, 0, sizeof(float) * d * d, stream));
     } else {
-        EncodeTiledFn enc = encode_fn();
-        if (!enc) {
-            set_error("kq_accum_factor: cuTensorMapEncodeTiled is unavailable");
-            return KQ_ERR_CUDA;
-        }
         CUtensorMap tmap;
-        std::memset(&tmap, 0, sizeof(tmap));
-        cuuint64_t gdim[2] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(T)};
-        cuuint64_t gstride[1] = {static_cast<cuuint64_t>(lda) * 2};
-        cuuint32_t box[2] = {64, static_cast<cuuint32_t>(BK)};
-        cuuint32_t estride[2] = {1, 1};
-        CUresult r = enc(&tmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<uint16_t*>(A), gdim,
-                         gstride, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                         CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-        if (r != CUDA_SUCCESS) {
-            set_error("kq_accum_factor: cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
-            return KQ_ERR_CUDA;
-        }
+        kq_status st = make_bf16_map(&tmap, A, d, T, lda, "kq_accum_factor");
+        if (st != KQ_OK) return st;
         static bool attr_set = false;
         if (!attr_set) {
             KQ_CUDA(cudaFuncSetAttribute(syrk_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -349,5 +437,71 @@ extern "C" kq_status kq_accum_factor(const uint16_t* A, int64_t T, int64_t d, in
         KQ_LAUNCH_CHECK("syrk_tc_kernel");
     }
     if (trace) return launch_trace(H, d, trace, stream);
+    return KQ_OK;
+}
+
+// ---------------------------------------------------------------------------- drift statistic
+extern "C" size_t kq_accum_drift_workspace(int64_t T, int64_t d) {
+    using namespace kq;
+    if (T < 1 || d < 1) return 0;
+    const int64_t Tr = cdiv(T, BK) * BK;
+    return 2 * static_cast<size_t>(Tr) * static_cast<size_t>(d) * sizeof(uint16_t);
+}
+
+extern "C" kq_status kq_accum_drift(const uint16_t* Xt, const uint16_t* X, int64_t T, int64_t d, int64_t ld,
+                                    float* D, int accumulate, int* info, void* ws, size_t ws_bytes,
+                                    kq_stream_t stream_) {
+    using namespace kq;
+    cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+    if (!D || d < 1 || d > 65536 || T < 0 || (T > 0 && (!Xt || !X)) || ld < d) {
+        set_error("kq_accum_drift: invalid arguments (d=%lld T=%lld ld=%lld)", (long long)d, (long long)T,
+                  (long long)ld);
+        return KQ_ERR_INVALID_ARG;
+    }
+    if (T > 0 && ((reinterpret_cast<uintptr_t>(Xt) & 15u) || (reinterpret_cast<uintptr_t>(X) & 15u) ||
+                  (ld % 8) != 0 || (d % 8) != 0 || T > (1ll << 31) - 64)) {
+        set_error("kq_accum_drift: X~ and X must be 16-byte aligned, d and ld multiples of 8, T < 2^31");
+        return KQ_ERR_INVALID_ARG;
+    }
+    if (T == 0) {
+        if (!accumulate) KQ_CUDA(cudaMemsetAsync(D, 0, sizeof(float) * d * d, stream));
+        return KQ_OK;
+    }
+    // token chunk: what the workspace holds (a multiple of BK tokens), at most all of T
+    const int64_t per_token = 2 * d * static_cast<int64_t>(sizeof(uint16_t));
+    int64_t Tc = ws ? static_cast<int64_t>(ws_bytes / per_token) / BK * BK : 0;
+    if (Tc > cdiv(T, BK) * BK) Tc = cdiv(T, BK) * BK;
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || Tc < BK) {
+        set_error("kq_accum_drift: workspace must be 256-byte aligned and hold at least %lld bytes "
+                  "(%zu for one pass)", (long long)(per_token * BK), kq_accum_drift_workspace(T, d));
+        return KQ_ERR_WORKSPACE;
+    }
+    uint16_t* hi = static_cast<uint16_t*>(ws);
+    uint16_t* lo = hi + Tc * d;
+    static bool attr_set = false;
+    if (!attr_set) {
+        KQ_CUDA(cudaFuncSetAttribute(drift_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES));
+        attr_set = true;
+    }
+    const int n_row = static_cast<int>(cdiv(d, BM));
+    const int n_col = static_cast<int>(cdiv(d, BN));
+    const int chunk_stages = KQ_SYRK_CHUNK_TOKENS / BK;
+    for (int64_t t0 = 0; t0 < T; t0 += Tc) {
+        const int64_t tn = std::min<int64_t>(Tc, T - t0);
+        const int64_t vecs = tn * (d / 8);
+        const int64_t grid = std::min<int64_t>(cdiv(vecs, 256), static_cast<int64_t>(num_sms()) * 16);
+        drift_split_kernel<<<static_cast<unsigned>(grid), 256, 0, stream>>>(Xt + t0 * ld, X + t0 * ld, tn, d, ld,
+                                                                            hi, lo);
+        KQ_LAUNCH_CHECK("drift_split_kernel");
+        CUtensorMap mh, ml, mb;
+        kq_status st = make_bf16_map(&mh, hi, d, tn, d, "kq_accum_drift");
+        if (st == KQ_OK) st = make_bf16_map(&ml, lo, d, tn, d, "kq_accum_drift");
+        if (st == KQ_OK) st = make_bf16_map(&mb, X + t0 * ld, d, tn, ld, "kq_accum_drift");
+        if (st != KQ_OK) return st;
+        drift_tc_kernel<<<static_cast<unsigned>(n_row * n_col), NUM_THREADS, SMEM_BYTES, stream>>>(
+            mh, ml, mb, D, static_cast<int>(d), static_cast<int>(tn), n_row, chunk_stages,
+            (accumulate || t0 > 0) ? 1 : 0, info);
+        KQ_LAUNCH_CHECK("drift_tc_kernel");
+    }
     return KQ_OK;
 }

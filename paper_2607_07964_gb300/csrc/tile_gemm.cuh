@@ -114,15 +114,18 @@ __device__ __forceinline__ void g_compute_chunk(const float* smem, int stage, in
     }
 }
 
-// acc = sum over k < kb of A-tile x B-tile, in ascending k. smem: G_SMEM bytes, 16-aligned.
-template <bool BN, bool VEC>
+// acc = sum over k < kb of A-tile x B-tile, in ascending k (INIT = false: the sum continues
+// from the acc passed in). smem: G_SMEM bytes, 16-aligned.
+template <bool BN, bool VEC, bool INIT = true>
 __device__ __forceinline__ void gemm_tile(const float* A, int64_t lda, int arows, const float* B, int64_t ldb, int bcols,
                                           int kb, float (&acc)[8][8], float* smem) {
     const int ty = threadIdx.x >> 4, tx = threadIdx.x & 15;
+    if (INIT) {
 #pragma unroll
-    for (int i = 0; i < 8; ++i)
+        for (int i = 0; i < 8; ++i)
 #pragma unroll
-        for (int j = 0; j < 8; ++j) acc[i][j] = 0.0f;
+            for (int j = 0; j < 8; ++j) acc[i][j] = 0.0f;
+    }
     const int nch = (kb + GK - 1) / GK;
     for (int c = 0; c < GSTAGES - 1; ++c) {
         if (c < nch) g_load_chunk<BN, VEC>(smem, c, c, A, lda, arows, B, ldb, bcols, kb);

@@ -1,5 +1,7 @@
 // Stage 4, tensor-core variant of the OBS sweep's lazy trailing update (Algorithm 2):
 //   W[:, cols] -= E_blk R_blk,   E_blk = E[:, i0:i0+128], R_blk[k][c] = Lt[c][i0 + k],
+// and with the GPTAQ correction also -= Q_blk P_blk (Q = -Wpre, P_blk[k][c] = Pt[c][i0 + k]),
+// i.e. K = 256 over [E | Q] and [R ; P],
 // on the 5th-generation tensor cores with fp32-accurate products from the 3xTF32 split
 // (Markidis et al. 2018; Ootomo & Yokota 2022): with x_hi = x rounded to tf32 and
 // x_lo = x - x_hi (exact in fp32),  E R ~= E_hi R_hi + E_hi R_lo + E_lo R_hi, accumulated in
@@ -44,35 +46,6 @@ struct TrailCfg {
     static_assert(BN % 32 == 0, "W moves in 32-column boxes");
 };
 
-__device__ __forceinline__ void tma_store_2d(const CUtensorMap* m, const void* src, int x, int y) {
-    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
-                     reinterpret_cast<uint64_t>(m)),
-                 "r"(smem_u32(src)), "r"(x), "r"(y)
-                 : "memory");
-}
-__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
-__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
-
-// Instruction descriptor, kind::tf32: fp32 accumulator, tf32 A and B, both K-major.
-__host__ __device__ constexpr uint32_t idesc_tf32_k_major(int M, int N) {
-    return (1u << 4)                                // D format: f32
-           | (2u << 7)                              // A format: tf32
-           | (2u << 10)                             // B format: tf32
-           | (static_cast<uint32_t>(N >> 3) << 17)  // N / 8
-           | (static_cast<uint32_t>(M >> 4) << 24); // M / 16
-}
-
-__device__ __forceinline__ void tc_mma_tf32(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
-                                            uint32_t accumulate) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-        : "memory");
-}
-
 __device__ __forceinline__ bool wait_quiet(uint64_t* bar, uint32_t parity) {
     int dummy = 0;
     return mbar_wait(bar, parity, &dummy);
@@ -82,8 +55,10 @@ template <int BN, int TSTAGES>
 __global__ void __launch_bounds__(T_THREADS, 1)
 trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__ CUtensorMap mEl,
                 const __grid_constant__ CUtensorMap mRh, const __grid_constant__ CUtensorMap mRl,
+                const __grid_constant__ CUtensorMap mQh, const __grid_constant__ CUtensorMap mQl,
+                const __grid_constant__ CUtensorMap mPh, const __grid_constant__ CUtensorMap mPl,
                 const __grid_constant__ CUtensorMap mW, int d_out, int i0, int cb, int n_col_tiles, int n_tiles,
-                int* info) {
+                int nslab, int* info) {
     using C = TrailCfg<BN, TSTAGES>;
     constexpr int WBOX = TBM * 32 * 4;     // one 128-row x 32-column box of W (16 KB)
     extern __shared__ uint8_t smem_raw[];
@@ -130,6 +105,12 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
         tma_prefetch_desc(&mRh);
         tma_prefetch_desc(&mRl);
         tma_prefetch_desc(&mW);
+        if (nslab > TNSLAB) {
+            tma_prefetch_desc(&mQh);
+            tma_prefetch_desc(&mQl);
+            tma_prefetch_desc(&mPh);
+            tma_prefetch_desc(&mPl);
+        }
     }
     tc_fence_before();
     __syncthreads();
@@ -150,7 +131,7 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
 #pragma unroll
                 for (int j = 0; j < BN / 32; ++j) tma_load_2d(wtile + j * WBOX, &mW, wfull, c0 + 32 * j, r0);
                 w_issued = li + 1;
-                for (int s = 0; s < TNSLAB; ++s, ++k) {
+                for (int s = 0; s < nslab; ++s, ++k) {
                     const int st = k % TSTAGES;
                     const uint32_t u = static_cast<uint32_t>(k / TSTAGES);
                     if (!mbar_wait(&empty[st], (u & 1u) ^ 1u, abort_flag)) {
@@ -159,11 +140,13 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
                     }
                     mbar_arrive_expect_tx(&full[st], C::STAGE);
                     uint8_t* base = smem + st * C::STAGE;
-                    const int x = i0 + s * TBK;
-                    tma_load_2d(base, &mEh, &full[st], x, r0);
-                    tma_load_2d(base + A_SLAB, &mEl, &full[st], x, r0);
-                    tma_load_2d(base + 2 * A_SLAB, &mRh, &full[st], x, c0);
-                    tma_load_2d(base + 2 * A_SLAB + C::B_SLAB, &mRl, &full[st], x, c0);
+                    // slabs 0..3: E and R; slabs 4..7 (with P): -Wpre and P
+                    const bool second = s >= TNSLAB;
+                    const int x = i0 + (second ? s - TNSLAB : s) * TBK;
+                    tma_load_2d(base, second ? &mQh : &mEh, &full[st], x, r0);
+                    tma_load_2d(base + A_SLAB, second ? &mQl : &mEl, &full[st], x, r0);
+                    tma_load_2d(base + 2 * A_SLAB, second ? &mPh : &mRh, &full[st], x, c0);
+                    tma_load_2d(base + 2 * A_SLAB + C::B_SLAB, second ? &mPl : &mRl, &full[st], x, c0);
                 }
             }
             // every issued load must land before the CTA exits
@@ -182,7 +165,7 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
                 if (!mbar_wait(&tempty[buf], ((static_cast<uint32_t>(li) >> 1) & 1u) ^ 1u, abort_flag)) break;
                 tc_fence_after();
                 const uint32_t dt = tmem + static_cast<uint32_t>(buf * BN);
-                for (int s = 0; s < TNSLAB; ++s, ++k) {
+                for (int s = 0; s < nslab; ++s, ++k) {
                     const int st = k % TSTAGES;
                     if (!mbar_wait(&full[st], static_cast<uint32_t>(k / TSTAGES) & 1u, abort_flag)) {
                         ok = false;
@@ -303,8 +286,9 @@ EncodeTiledFn encode_tiled() {
     return fn;
 }
 
-// 2-D fp32 tensor map over a row-major [rows x cols] matrix, box = box_rows x 32 columns.
-kq_status make_map(CUtensorMap* m, const float* base, int64_t rows, int64_t cols, int box_rows) {
+}  // namespace
+
+kq_status make_f32_map(CUtensorMap* m, const float* base, int64_t rows, int64_t cols, int box_rows) {
     EncodeTiledFn enc = encode_tiled();
     if (!enc) {
         set_error("trailing update: cuTensorMapEncodeTiled is unavailable");
@@ -325,8 +309,6 @@ kq_status make_map(CUtensorMap* m, const float* base, int64_t rows, int64_t cols
     return KQ_OK;
 }
 
-}  // namespace
-
 kq_status split_tf32(const float* src, int64_t n, float* hi, float* lo, cudaStream_t stream) {
     const int64_t grid = std::min<int64_t>(cdiv(n, 256), static_cast<int64_t>(num_sms()) * 16);
     split_tf32_kernel<<<static_cast<unsigned>(std::max<int64_t>(grid, 1)), 256, 0, stream>>>(src, n, hi, lo);
@@ -337,19 +319,29 @@ kq_status split_tf32(const float* src, int64_t n, float* hi, float* lo, cudaStre
 kq_status TrailMaps::init(const float* E_hi, const float* E_lo, const float* Lt_hi, const float* Lt_lo,
                           int64_t d_out, int64_t d_in) {
     kq_status st;
-    if ((st = make_map(&eh, E_hi, d_out, d_in, TBM)) != KQ_OK) return st;
-    if ((st = make_map(&el, E_lo, d_out, d_in, TBM)) != KQ_OK) return st;
-    if ((st = make_map(&rh_narrow, Lt_hi, d_in, d_in, 128)) != KQ_OK) return st;
-    if ((st = make_map(&rl_narrow, Lt_lo, d_in, d_in, 128)) != KQ_OK) return st;
+    if ((st = make_f32_map(&eh, E_hi, d_out, d_in, TBM)) != KQ_OK) return st;
+    if ((st = make_f32_map(&el, E_lo, d_out, d_in, TBM)) != KQ_OK) return st;
+    if ((st = make_f32_map(&rh_narrow, Lt_hi, d_in, d_in, 128)) != KQ_OK) return st;
+    if ((st = make_f32_map(&rl_narrow, Lt_lo, d_in, d_in, 128)) != KQ_OK) return st;
+    return KQ_OK;
+}
+
+kq_status TrailMaps::init_p(const float* Q_hi, const float* Q_lo, const float* Pt_hi, const float* Pt_lo,
+                            int64_t d_out, int64_t d_in) {
+    kq_status st;
+    if ((st = make_f32_map(&qh, Q_hi, d_out, d_in, TBM)) != KQ_OK) return st;
+    if ((st = make_f32_map(&ql, Q_lo, d_out, d_in, TBM)) != KQ_OK) return st;
+    if ((st = make_f32_map(&ph, Pt_hi, d_in, d_in, 128)) != KQ_OK) return st;
+    if ((st = make_f32_map(&pl, Pt_lo, d_in, d_in, 128)) != KQ_OK) return st;
     return KQ_OK;
 }
 
 kq_status TrailMaps::set_w(float* W, int64_t d_out, int64_t d_in) {
-    return make_map(&w, W, d_out, d_in, TBM);
+    return make_f32_map(&w, W, d_out, d_in, TBM);
 }
 
 kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, int64_t i0, int64_t cb, int64_t ce,
-                   int* info, cudaStream_t stream) {
+                   bool with_p, int* info, cudaStream_t stream) {
     // Persistent: at most one CTA per SM, each walking the tiles t, t + grid, ... (column
     // tile fastest, so the CTAs running together share row and column operands in L2).
     // 128-column tiles; a range either is a whole number of tiles or ends at d_in (the TMA
@@ -368,8 +360,9 @@ kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, in
     const int n_col = static_cast<int>(cdiv(ce - cb, 128));
     const int n = n_row * n_col;
     trail_tc_kernel<128, 2><<<static_cast<unsigned>(std::min(n, num_sms())), T_THREADS, Cfg::SMEM, stream>>>(
-        m.eh, m.el, m.rh_narrow, m.rl_narrow, m.w, static_cast<int>(d_out), static_cast<int>(i0),
-        static_cast<int>(cb), n_col, n, info);
+        m.eh, m.el, m.rh_narrow, m.rl_narrow, with_p ? m.qh : m.eh, with_p ? m.ql : m.el,
+        with_p ? m.ph : m.rh_narrow, with_p ? m.pl : m.rl_narrow, m.w, static_cast<int>(d_out), static_cast<int>(i0),
+        static_cast<int>(cb), n_col, n, with_p ? 2 * TNSLAB : TNSLAB, info);
     KQ_LAUNCH_CHECK("trail_tc_kernel");
     return KQ_OK;
 }

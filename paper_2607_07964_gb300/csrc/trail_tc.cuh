@@ -12,22 +12,59 @@ __device__ __forceinline__ float tf32_hi(float x) {
     return __uint_as_float(r);
 }
 
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* m, const void* src, int x, int y) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                     reinterpret_cast<uint64_t>(m)),
+                 "r"(smem_u32(src)), "r"(x), "r"(y)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+// Instruction descriptor, kind::tf32: fp32 accumulator, tf32 A and B, both K-major.
+__host__ __device__ constexpr uint32_t idesc_tf32_k_major(int M, int N) {
+    return (1u << 4)                                // D format: f32
+           | (2u << 7)                              // A format: tf32
+           | (2u << 10)                             // B format: tf32
+           | (static_cast<uint32_t>(N >> 3) << 17)  // N / 8
+           | (static_cast<uint32_t>(M >> 4) << 24); // M / 16
+}
+
+__device__ __forceinline__ void tc_mma_tf32(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                            uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// 2-D fp32 tensor map over a row-major [rows x cols] matrix: box = box_rows x 32 columns,
+// 128-byte swizzle (a 32-float row is one swizzle atom), zero fill outside the matrix.
+kq_status make_f32_map(CUtensorMap* m, const float* base, int64_t rows, int64_t cols, int box_rows);
+
 // Tensor maps over the split error block and the split L, encoded once per sweep.
 struct TrailMaps {
     CUtensorMap eh, el;                  // E_hi, E_lo [d_out x d_in], 128-row boxes
     CUtensorMap rh_narrow, rl_narrow;    // Lt_hi, Lt_lo [d_in x d_in], 128-row boxes
     CUtensorMap w;                       // W [d_out x d_in], 128-row boxes (read and written)
+    CUtensorMap qh, ql, ph, pl;          // with P: (-Wpre)_hi, _lo [d_out x d_in], Pt_hi, Pt_lo [d_in x d_in]
     kq_status init(const float* E_hi, const float* E_lo, const float* Lt_hi, const float* Lt_lo, int64_t d_out,
                    int64_t d_in);
+    kq_status init_p(const float* Q_hi, const float* Q_lo, const float* Pt_hi, const float* Pt_lo, int64_t d_out,
+                     int64_t d_in);
     kq_status set_w(float* W, int64_t d_out, int64_t d_in);
 };
 
 // hi = src rounded to tf32, lo = src - hi (n elements).
 kq_status split_tf32(const float* src, int64_t n, float* hi, float* lo, cudaStream_t stream);
 
-// W[:, cb:ce] -= E[:, i0:i0+128] R[i0:i0+128, cb:ce] (R[k][c] = Lt[c][k]) on tensor cores;
-// [cb, ce) must be whole 128-column tiles or end at d_in. W is the one set_w was given.
+// W[:, cb:ce] -= E[:, i0:i0+128] R[i0:i0+128, cb:ce] (R[k][c] = Lt[c][k]) on tensor cores,
+// and with_p: also -= Q[:, i0:i0+128] P[i0:i0+128, cb:ce] (P[k][c] = Pt[c][k]); [cb, ce) must
+// be whole 128-column tiles or end at d_in. W is the one set_w was given.
 kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, int64_t i0, int64_t cb, int64_t ce,
-                   int* info, cudaStream_t stream);
+                   bool with_p, int* info, cudaStream_t stream);
 
 }  // namespace kq

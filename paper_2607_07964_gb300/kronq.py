@@ -56,8 +56,12 @@ def lib() -> ctypes.CDLL:
             "kq_chol_inv_workspace": ([I64], SZ),
             "kq_chol_inv": ([P, I64, F, P, P, P, SZ, P], I),
             "kq_chol_inv_noalloc": ([P, I64, F, P, P, P], I),
-            "kq_obs_quantize_workspace": ([I64, I64, I, I], SZ),
-            "kq_obs_quantize": ([P, I64, I64, P, I, I, I, I, P, P, P, P, P, P, P, SZ, P], I),
+            "kq_obs_quantize_workspace": ([I64, I64, I, I, I], SZ),
+            "kq_obs_quantize": ([P, I64, I64, P, P, I, I, I, I, P, P, P, P, P, P, P, SZ, P], I),
+            "kq_accum_drift_workspace": ([I64, I64], SZ),
+            "kq_accum_drift": ([P, P, I64, I64, I64, P, I, P, P, SZ, P], I),
+            "kq_gptaq_p_workspace": ([I64], SZ),
+            "kq_gptaq_p": ([P, P, I64, F, P, P, P, SZ, P], I),
             "kq_dequant_revert": ([P, P, P, I64, I64, I, P, P, P, P, P, P], I),
             "kq_proxy_loss_workspace": ([I64, I64], SZ),
             "kq_proxy_loss": ([P, P, I64, I64, P, P, P, P, SZ, P], I),
@@ -138,6 +142,41 @@ def kq_accum_factor(A, H, accumulate: bool = False, trace=None, info=None, strea
     _need(info, "info", torch.int32)
     _ok(lib().kq_accum_factor(_ptr(A), T, d, A.stride(0), _ptr(H), int(accumulate), _ptr(trace),
                               _ptr(info), _stream(stream)), "kq_accum_factor")
+
+
+def kq_accum_drift_workspace(T: int, d: int) -> int:
+    """Bytes for one pass over all T tokens (a smaller workspace makes token chunks)."""
+    return int(lib().kq_accum_drift_workspace(T, d))
+
+
+def kq_accum_drift(Xt, X, D, accumulate: bool = False, info=None, ws=None, stream=None) -> None:
+    """D (+)= (X~ - X)^T X; Xt (X~) and X [T, d] bf16 with the same row stride, D [d, d] fp32."""
+    if X.dim() != 2 or X.stride(1) != 1 or Xt.shape != X.shape or Xt.stride() != X.stride():
+        raise ValueError("X~ and X must be 2-D, same shape and strides, unit column stride")
+    T, d = X.shape
+    _need(Xt, "Xt", torch.bfloat16, contiguous=False)
+    _need(X, "X", torch.bfloat16, contiguous=False)
+    _need(D, "D", torch.float32, (d, d))
+    _need(info, "info", torch.int32)
+    _need(ws, "ws", torch.uint8)
+    _ok(lib().kq_accum_drift(_ptr(Xt), _ptr(X), T, d, X.stride(0), _ptr(D), int(accumulate), _ptr(info),
+                             _ptr(ws), 0 if ws is None else ws.numel(), _stream(stream)), "kq_accum_drift")
+
+
+def kq_gptaq_p_workspace(n: int) -> int:
+    return int(lib().kq_gptaq_p_workspace(n))
+
+
+def kq_gptaq_p(Dp, Lt, alpha: float, Pt, ws, info=None, stream=None) -> None:
+    """Pt = P^T with P = alpha ((D' L) o M_U) L^T (Proposition 1, Algorithm 2)."""
+    n = Lt.shape[0]
+    _need(Dp, "Dp", torch.float32, (n, n))
+    _need(Lt, "Lt", torch.float32, (n, n))
+    _need(Pt, "Pt", torch.float32, (n, n))
+    _need(ws, "ws", torch.uint8)
+    _need(info, "info", torch.int32)
+    _ok(lib().kq_gptaq_p(_ptr(Dp), _ptr(Lt), n, float(alpha), _ptr(Pt), _ptr(info), _ptr(ws),
+                         0 if ws is None else ws.numel(), _stream(stream)), "kq_gptaq_p")
 
 
 def kq_compute_scales(W, H_X, H_G, s_x, s_g, stream=None) -> None:
@@ -261,17 +300,20 @@ def kq_chol_inv_noalloc(H, damp_rel: float, Lt, info=None, stream=None) -> None:
         "kq_chol_inv_noalloc")
 
 
-def kq_obs_quantize_workspace(d_out: int, d_in: int, block: int = 128, mode: int = KQ_TRAIL_FP32) -> int:
-    return int(lib().kq_obs_quantize_workspace(d_out, d_in, block, mode))
+def kq_obs_quantize_workspace(d_out: int, d_in: int, block: int = 128, mode: int = KQ_TRAIL_FP32,
+                              with_p: bool = False) -> int:
+    return int(lib().kq_obs_quantize_workspace(d_out, d_in, block, mode, int(with_p)))
 
 
 def kq_obs_quantize(W, Lt, bits: int, group: int, block: int, codes, scale, zero, col_loss=None,
-                    pre_q=None, ws=None, stream=None, mode: int = KQ_TRAIL_FP32, info=None) -> None:
-    """mode: KQ_TRAIL_FP32 (fp32-ordered trailing update, bit-exact) or KQ_TRAIL_3XTF32."""
+                    pre_q=None, ws=None, stream=None, mode: int = KQ_TRAIL_FP32, info=None, Pt=None) -> None:
+    """mode: KQ_TRAIL_FP32 (fp32-ordered trailing update, bit-exact) or KQ_TRAIL_3XTF32.
+    Pt: P^T from kq_gptaq_p for the GPTAQ drift correction, or None (GPTQ mode)."""
     d_out, d_in = W.shape
     ng = 1 if group == 0 else -(-d_in // group)
     _need(W, "W", torch.float32)
     _need(Lt, "Lt", torch.float32, (d_in, d_in))
+    _need(Pt, "Pt", torch.float32, (d_in, d_in))
     _need(codes, "codes", torch.uint8, (d_out, d_in))
     _need(scale, "scale", torch.float32, (d_out, ng))
     _need(zero, "zero", torch.int32, (d_out, ng))
@@ -279,7 +321,7 @@ def kq_obs_quantize(W, Lt, bits: int, group: int, block: int, codes, scale, zero
     _need(pre_q, "pre_q", torch.float32, (d_out, d_in))
     _need(ws, "ws", torch.uint8)
     _need(info, "info", torch.int32)
-    _ok(lib().kq_obs_quantize(_ptr(W), d_out, d_in, _ptr(Lt), bits, group, block, mode, _ptr(codes),
+    _ok(lib().kq_obs_quantize(_ptr(W), d_out, d_in, _ptr(Lt), _ptr(Pt), bits, group, block, mode, _ptr(codes),
                               _ptr(scale), _ptr(zero), _ptr(col_loss), _ptr(pre_q), _ptr(info), _ptr(ws),
                               0 if ws is None else ws.numel(), _stream(stream)), "kq_obs_quantize")
 

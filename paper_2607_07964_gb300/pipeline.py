@@ -1,7 +1,8 @@
-"""One linear layer through the four stages of the KronQ path (Algorithms 1 and 2, GPTQ
-mode), as a sequence of libkronq calls on one CUDA stream. Buffers and workspaces are
-allocated once (torch provides the device memory) and reused across layers of the same
-shape.
+"""One linear layer through the four stages of the KronQ path (Algorithms 1 and 2), as a
+sequence of libkronq calls on one or two CUDA streams: GPTQ mode, or with the GPTAQ drift
+correction (the full objective of Eq. kronq_full) when a scaling alpha is given and the
+full-precision input X~ is passed to run(). Buffers and workspaces are allocated once
+(torch provides the device memory) and reused across layers of the same shape.
 """
 from __future__ import annotations
 
@@ -10,6 +11,8 @@ import torch
 from . import kronq as kq
 
 STAGES = ("factor_x", "factor_g", "scales_traces", "rotate", "chol", "sweep")
+# with the drift correction: the drift statistic after H_X, and P after the Cholesky
+STAGES_DRIFT = ("factor_x", "drift", "factor_g", "scales_traces", "rotate", "chol", "p", "sweep")
 
 
 class LayerPipeline:
@@ -18,8 +21,11 @@ class LayerPipeline:
     def __init__(self, d_out: int, d_in: int, bits: int, group: int, block: int = 128,
                  damp: float = 0.01, device: str = "cuda", want_col_loss: bool = True,
                  overlap: bool = True, x_chunk_tokens: int = 0, g_chunk_tokens: int = 32768,
-                 trailing: str = "3xtf32"):
+                 trailing: str = "3xtf32", alpha: float | None = None, drift_chunk_tokens: int = 0):
         self.d_out, self.d_in, self.bits, self.group, self.block, self.damp = d_out, d_in, bits, group, block, damp
+        # GPTAQ drift correction (Prop. 1, Alg. 2) with scaling alpha; None = GPTQ mode
+        self.alpha = alpha
+        self.stages = STAGES if alpha is None else STAGES_DRIFT
         f32 = dict(dtype=torch.float32, device=device)
         ng = 1 if group == 0 else -(-d_in // group)
         self.HX = torch.empty((d_in, d_in), **f32)
@@ -40,8 +46,19 @@ class LayerPipeline:
         # the sweep's lazy trailing update: "fp32" (the fp32-ordered definition, bit-exact) or
         # "3xtf32" (tensor cores, 3xTF32 split)
         self.trail_mode = {"fp32": kq.KQ_TRAIL_FP32, "3xtf32": kq.KQ_TRAIL_3XTF32}[trailing]
-        self.ws_obs = torch.empty((kq.kq_obs_quantize_workspace(d_out, d_in, block, self.trail_mode),), dtype=torch.uint8,
-                                  device=device)
+        self.ws_obs = torch.empty((kq.kq_obs_quantize_workspace(d_out, d_in, block, self.trail_mode,
+                                                                alpha is not None),),
+                                  dtype=torch.uint8, device=device)
+        if alpha is not None:
+            self.D = torch.empty((d_in, d_in), **f32)      # drift statistic, then D'
+            self.Pt = torch.empty((d_in, d_in), **f32)
+            self.ws_p = torch.empty((kq.kq_gptaq_p_workspace(d_in),), dtype=torch.uint8, device=device)
+        else:
+            self.D = self.Pt = None
+        # the split drift of this many tokens at a time (0: all tokens of the first run; the
+        # call chunks the tokens itself when its workspace holds fewer)
+        self.drift_chunk_tokens = drift_chunk_tokens
+        self.ws_drift = None
         # Output-side work (H_G, S_G, U) runs on a second stream beside the Cholesky, which
         # needs only H_X and leaves most SMs idle during its diagonal steps.
         # The critical path (H_X, Cholesky, sweep) runs on a high-priority stream so SMs freed
@@ -60,7 +77,7 @@ class LayerPipeline:
         self.main = torch.cuda.Stream(device=device, priority=hi) if overlap else None
         self.side = torch.cuda.Stream(device=device, priority=lo) if overlap else None
         self.copy = None
-        self._ev = [torch.cuda.Event() for _ in range(7)]
+        self._ev = [torch.cuda.Event() for _ in range(8)]
 
     def _chunks(self, which: str, T: int) -> list[tuple[int, int]]:
         c = self.chunk_tokens[which]
@@ -84,49 +101,71 @@ class LayerPipeline:
             kq.kq_accum_factor(A[t0:t1], H, accumulate=c > 0, trace=trace if c == len(ch) - 1 else None,
                                info=info, stream=stream)
 
-    def run(self, X, G, W, sign_u, sign_v, stream=None, events=None) -> None:
+    def _need_xt(self, Xt) -> None:
+        if (self.alpha is None) != (Xt is None):
+            raise ValueError("X~ must be given exactly when the pipeline has a drift scaling alpha")
+        if Xt is not None and self.ws_drift is None:   # sized once, before any graph capture
+            tokens = self.drift_chunk_tokens if self.drift_chunk_tokens > 0 else Xt.shape[0]
+            self.ws_drift = torch.empty((kq.kq_accum_drift_workspace(tokens, self.d_in),), dtype=torch.uint8,
+                                        device=self.HX.device)
+
+    def run(self, X, G, W, sign_u, sign_v, stream=None, events=None, Xt=None) -> None:
         """X [T, d_in] bf16, G [T, d_out] bf16, W [d_out, d_in] fp32 (left unchanged), signs
-        int8. `events`, if given, is a list of len(STAGES) + 1 CUDA events recorded at the
-        stage boundaries on the stream."""
+        int8; Xt = X~ [T, d_in] bf16 with the drift correction. `events`, if given, is a list
+        of len(self.stages) + 1 CUDA events recorded at the stage boundaries on the stream."""
+        self._need_xt(Xt)
         s = torch.cuda.current_stream() if stream is None else stream
         if self.overlap and events is None:
-            self._run_overlapped(X, G, W, sign_u, sign_v, s)
+            self._run_overlapped(X, G, W, sign_u, sign_v, s, Xt=Xt)
             return
+        marks = iter(range(len(self.stages) + 1))
 
-        def mark(i):
+        def mark():
+            i = next(marks)
             if events is not None:
                 events[i].record(s)
 
-        mark(0)
+        mark()
         self._factor("X", X, self.HX, self.trace_x, self.info[0:1], s)                           # Alg. 1: H_X
-        mark(1)
+        mark()
+        if Xt is not None:                                                                        # Alg. 1: Delta X X^T
+            kq.kq_accum_drift(Xt, X, self.D, info=self.info[0:1], ws=self.ws_drift, stream=s)
+            mark()
         self._factor("G", G, self.HG, self.trace_g, self.info[2:3], s)                           # H_G
-        mark(2)
+        mark()
         kq.kq_compute_scales(W, self.HX, self.HG, self.s_x, self.s_g, stream=s)          # Eq. (rescale)
         kq.kq_traces(self.HX, self.s_x, self.HG, self.s_g, self.traces, stream=s)         # Eq. (sensitivity)
-        mark(3)
+        mark()
         with torch.cuda.stream(s):
             self.Wp.copy_(W)
         kq.kq_rotate_in(self.Wp, self.HX, self.s_x, sign_v, kq.KQ_FWD, stream=s)         # Eq. (biip), V side
+        if Xt is not None:
+            kq.kq_rotate_in(None, self.D, self.s_x, sign_v, kq.KQ_FWD, stream=s)         # D' = V S^-1 D S^-1 V^T
         kq.kq_rotate_out(self.Wp, None, self.s_g, sign_u, kq.KQ_FWD, stream=s)           # U side
         kq.kq_rotate_out(None, self.HG, self.s_g, sign_u, kq.KQ_FWD, stream=s)           # H_G, then released
-        mark(4)
+        mark()
         kq.kq_chol_inv(self.HX, self.damp, self.Lt, self.info[1:2], self.ws_chol, stream=s)  # Alg. 2
-        mark(5)
+        mark()
+        if Xt is not None:
+            kq.kq_gptaq_p(self.D, self.Lt, self.alpha, self.Pt, self.ws_p, info=self.info[1:2], stream=s)  # P
+            mark()
         kq.kq_obs_quantize(self.Wp, self.Lt, self.bits, self.group, self.block, self.codes, self.scale,
                            self.zero, self.col_loss, None, self.ws_obs, stream=s, mode=self.trail_mode,
-                           info=self.info[3:4])   # Alg. 2 sweep
-        mark(6)
+                           info=self.info[3:4], Pt=self.Pt if Xt is not None else None)   # Alg. 2 sweep
+        mark()
 
-    def _run_overlapped(self, X, G, W, sign_u, sign_v, caller, x_ready=None, g_ready=None, w_ready=None) -> None:
+    def _run_overlapped(self, X, G, W, sign_u, sign_v, caller, x_ready=None, g_ready=None, w_ready=None,
+                        Xt=None, xt_ready=None) -> None:
         """The same results on two streams. The Cholesky needs only H_X and leaves most SMs
         idle during its diagonal steps, so H_G, S_G and U go to a low-priority stream that
         runs beside it; the high-priority stream does H_X, S_X, V, the Cholesky and (once
         U is applied to W) the sweep, while H_G's own rotation finishes beside the sweep.
-        Events order the shared buffers; x_ready / g_ready / w_ready are the host path's
-        copy events."""
+        With the drift correction the drift statistic and its rotation run first on the
+        low-priority stream and P on the high-priority one after the Cholesky.
+        Events order the shared buffers; x_ready / g_ready / w_ready / xt_ready are the host
+        path's copy events."""
         s, s2 = self.main, self.side
-        e_in, e_fx, e_tx, e_rin, e_side, e_out, e_hg = self._ev
+        e_in, e_fx, e_tx, e_rin, e_side, e_out, e_hg, e_d = self._ev
         e_in.record(caller)
         s.wait_event(e_in)
         s2.wait_event(e_in)
@@ -143,6 +182,13 @@ class LayerPipeline:
         e_rin.record(s)
         kq.kq_chol_inv(self.HX, self.damp, self.Lt, self.info[1:2], self.ws_chol, stream=s)
         s2.wait_event(e_fx)                      # the two factors would only split the SMs
+        if Xt is not None:
+            if xt_ready is not None:
+                s2.wait_event(xt_ready)
+            kq.kq_accum_drift(Xt, X, self.D, info=self.info[2:3], ws=self.ws_drift, stream=s2)
+            s2.wait_event(e_tx)                  # S_X
+            kq.kq_rotate_in(None, self.D, self.s_x, sign_v, kq.KQ_FWD, stream=s2)
+            e_d.record(s2)
         self._factor("G", G, self.HG, self.trace_g, self.info[2:3], s2, g_ready)
         s2.wait_event(e_tx)                      # W (host path) and the X side of the traces
         kq.kq_compute_scales(W, None, self.HG, None, self.s_g, stream=s2)
@@ -152,15 +198,18 @@ class LayerPipeline:
         e_side.record(s2)
         kq.kq_rotate_out(None, self.HG, self.s_g, sign_u, kq.KQ_FWD, stream=s2)
         e_hg.record(s2)
+        if Xt is not None:
+            s.wait_event(e_d)
+            kq.kq_gptaq_p(self.D, self.Lt, self.alpha, self.Pt, self.ws_p, info=self.info[1:2], stream=s)
         s.wait_event(e_side)
         kq.kq_obs_quantize(self.Wp, self.Lt, self.bits, self.group, self.block, self.codes, self.scale,
                            self.zero, self.col_loss, None, self.ws_obs, stream=s, mode=self.trail_mode,
-                           info=self.info[3:4])
+                           info=self.info[3:4], Pt=self.Pt if Xt is not None else None)
         e_out.record(s)
         caller.wait_event(e_out)
         caller.wait_event(e_hg)
 
-    def capture(self, X, G, W, sign_u, sign_v) -> tuple:
+    def capture(self, X, G, W, sign_u, sign_v, Xt=None) -> tuple:
         """Record one layer (both streams) as a CUDA graph on these fixed buffers. Returns
         (graph, kernels per replay). Run run() once first so one-time set-up is done."""
         from . import kronq as _kq
@@ -169,7 +218,7 @@ class LayerPipeline:
         cap = torch.cuda.Stream(device=self.HX.device)
         n0 = _kq.launch_count()
         with torch.cuda.graph(g, stream=cap):
-            self.run(X, G, W, sign_u, sign_v, stream=cap)
+            self.run(X, G, W, sign_u, sign_v, stream=cap, Xt=Xt)
         return g, _kq.launch_count() - n0
 
     def check(self, stream=None) -> None:
@@ -182,7 +231,7 @@ class LayerPipeline:
             if st != kq.KQ_OK:
                 raise kq.KronqError(st, "pipeline", f"device word {raw}")
 
-    def run_host(self, X_h, G_h, W_h, su_h, sv_h, codes_h, scale_h, zero_h, stream=None) -> tuple[int, int]:
+    def run_host(self, X_h, G_h, W_h, su_h, sv_h, codes_h, scale_h, zero_h, stream=None, Xt_h=None) -> tuple[int, int]:
         """End-to-end call with HOST buffers (pinned for asynchronous copies): copy the
         layer's inputs to the device, run the four stages, copy codes and grids back.
         Enqueued on `stream`; the caller synchronizes. Returns (bytes in, bytes out).
@@ -191,9 +240,11 @@ class LayerPipeline:
         each chunk's factor accumulation starts as soon as that chunk has arrived, so the
         host link (the bound at these sizes) overlaps the factor, rescale, rotation and
         Cholesky work; without the two-stream schedule the copies simply precede the run."""
+        self._need_xt(Xt_h)
         s = torch.cuda.current_stream() if stream is None else stream
         dev = self.HX.device
-        if getattr(self, "_stage", None) is None or self._stage["X"].shape != X_h.shape:
+        if getattr(self, "_stage", None) is None or self._stage["X"].shape != X_h.shape or \
+                (Xt_h is not None) != ("Xt" in self._stage):
             self._stage = {
                 "X": torch.empty(X_h.shape, dtype=X_h.dtype, device=dev),
                 "G": torch.empty(G_h.shape, dtype=G_h.dtype, device=dev),
@@ -201,14 +252,18 @@ class LayerPipeline:
                 "su": torch.empty(su_h.shape, dtype=su_h.dtype, device=dev),
                 "sv": torch.empty(sv_h.shape, dtype=sv_h.dtype, device=dev),
             }
+            if Xt_h is not None:
+                self._stage["Xt"] = torch.empty(Xt_h.shape, dtype=Xt_h.dtype, device=dev)
         st = self._stage
-        nin = sum(t.numel() * t.element_size() for t in (X_h, G_h, W_h, su_h, sv_h))
+        ins = [X_h, G_h, W_h, su_h, sv_h] + ([] if Xt_h is None else [Xt_h])
+        nin = sum(t.numel() * t.element_size() for t in ins)
         nout = sum(t.numel() * t.element_size() for t in (codes_h, scale_h, zero_h))
         if not self.overlap:
             with torch.cuda.stream(s):
-                for k, h in (("X", X_h), ("G", G_h), ("W", W_h), ("su", su_h), ("sv", sv_h)):
+                pairs = [("X", X_h), ("G", G_h), ("W", W_h), ("su", su_h), ("sv", sv_h)]
+                for k, h in pairs + ([] if Xt_h is None else [("Xt", Xt_h)]):
                     st[k].copy_(h, non_blocking=True)
-            self.run(st["X"], st["G"], st["W"], st["su"], st["sv"], stream=s)
+            self.run(st["X"], st["G"], st["W"], st["su"], st["sv"], stream=s, Xt=st.get("Xt"))
         else:
             if self.copy is None:
                 self.copy = torch.cuda.Stream(device=dev)
@@ -229,8 +284,13 @@ class LayerPipeline:
                         ev = torch.cuda.Event()
                         ev.record(cs)
                         ready[k].append(ev)
+                    if k == "X" and Xt_h is not None:   # X~ right after X: the drift needs both
+                        st["Xt"].copy_(Xt_h, non_blocking=True)
+                        xt_ready = torch.cuda.Event()
+                        xt_ready.record(cs)
             self._run_overlapped(st["X"], st["G"], st["W"], st["su"], st["sv"], s, x_ready=ready["X"],
-                                 g_ready=ready["G"], w_ready=w_ready)
+                                 g_ready=ready["G"], w_ready=w_ready, Xt=st.get("Xt"),
+                                 xt_ready=xt_ready if Xt_h is not None else None)
         with torch.cuda.stream(s):
             codes_h.copy_(self.codes, non_blocking=True)
             scale_h.copy_(self.scale, non_blocking=True)

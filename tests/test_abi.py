@@ -26,7 +26,8 @@ def declared_symbols():
 def test_header_declares_the_boundary():
     names = declared_symbols()
     for required in ["kq_accum_factor", "kq_compute_scales", "kq_rotate_in", "kq_rotate_out",
-                     "kq_chol_inv", "kq_obs_quantize", "kq_traces", "kq_check"]:
+                     "kq_chol_inv", "kq_obs_quantize", "kq_traces", "kq_check", "kq_accum_drift",
+                     "kq_gptaq_p"]:
         assert required in names
 
 
@@ -51,7 +52,16 @@ def test_workspace_queries(lib):
     assert kronq.kq_obs_quantize_workspace(64, 256, 128) >= 64 * 256 * 4
     assert kronq.kq_obs_quantize_workspace(64, 256, 128, kronq.KQ_TRAIL_3XTF32) >= 3 * 64 * 256 * 4 + 2 * 256 * 256 * 4
     assert kronq.kq_obs_quantize_workspace(64, 256, 128, 5) == 0
+    # with P: packed P blocks and -Wpre (fp32), or its split and the split P (tensor cores)
+    assert (kronq.kq_obs_quantize_workspace(64, 256, 128, kronq.KQ_TRAIL_FP32, True) >=
+            kronq.kq_obs_quantize_workspace(64, 256, 128) + 2 * 128 * 128 * 4 + 64 * 256 * 4)
+    assert (kronq.kq_obs_quantize_workspace(64, 256, 128, kronq.KQ_TRAIL_3XTF32, True) >=
+            kronq.kq_obs_quantize_workspace(64, 256, 128, kronq.KQ_TRAIL_3XTF32) + 2 * 128 * 128 * 4
+            + 2 * 64 * 256 * 4 + 2 * 256 * 256 * 4)
     assert kronq.kq_proxy_loss_workspace(8, 8) >= 3 * 64 * 4
+    assert kronq.kq_accum_drift_workspace(100, 64) == 2 * 128 * 64 * 2   # tokens padded to 64
+    assert kronq.kq_accum_drift_workspace(0, 64) == 0
+    assert kronq.kq_gptaq_p_workspace(256) >= 6 * 256 * 256 * 4
 
 
 def test_host_side_argument_errors(lib):
@@ -70,17 +80,31 @@ def test_host_side_argument_errors(lib):
     assert lib.kq_rotate_out(fake, 100, 4, None, None, fake, 0, None) == K.KQ_ERR_UNSUPPORTED
     assert lib.kq_rotate_in(fake, 4, 28 * 2048, None, None, fake, 0, None) == K.KQ_ERR_UNSUPPORTED
     # sweep: block must be 128 and group in {0, block}
-    args = [fake, 4, 256, fake, 4, 64, 128, 0, fake, fake, fake, None, None, None, fake, 1 << 30, None]
+    # (W, d_out, d_in, Lt, Pt, bits, group, block, mode, codes, scale, zero, col_loss, pre_q,
+    #  info, ws, ws_bytes, stream)
+    args = [fake, 4, 256, fake, None, 4, 64, 128, 0, fake, fake, fake, None, None, None, fake, 1 << 30, None]
     assert lib.kq_obs_quantize(*args) == K.KQ_ERR_UNSUPPORTED
-    args[6] = 64
-    args[5] = 0
+    args[7] = 64
+    args[6] = 0
     assert lib.kq_obs_quantize(*args) == K.KQ_ERR_UNSUPPORTED
-    args[6], args[4] = 128, 9
+    args[7], args[5] = 128, 9
     assert lib.kq_obs_quantize(*args) == K.KQ_ERR_INVALID_ARG
-    args[4], args[7] = 4, 7                       # unknown trailing-update mode
+    args[5], args[8] = 4, 7                       # unknown trailing-update mode
     assert lib.kq_obs_quantize(*args) == K.KQ_ERR_INVALID_ARG
-    args[7], args[2] = K.KQ_TRAIL_3XTF32, 258     # tensor-core mode needs d_in % 4 == 0
+    args[8], args[2] = K.KQ_TRAIL_3XTF32, 258     # tensor-core mode needs d_in % 4 == 0
     assert lib.kq_obs_quantize(*args) == K.KQ_ERR_UNSUPPORTED
-    args[7], args[2], args[15] = 0, 256, 16
+    args[8], args[2], args[4] = 0, 264, fake      # the drift correction needs d_in % 16 == 0
+    assert lib.kq_obs_quantize(*args) == K.KQ_ERR_UNSUPPORTED
+    args[2], args[4], args[16] = 256, None, 16
     assert lib.kq_obs_quantize(*args) == K.KQ_ERR_WORKSPACE
     assert "workspace" in K.last_error()
+    # drift statistic: X~ and X needed, d % 8 == 0, 16-byte alignment, a workspace
+    assert lib.kq_accum_drift(None, fake, 16, 8, 8, fake, 0, None, fake, 1 << 20, None) == K.KQ_ERR_INVALID_ARG
+    assert lib.kq_accum_drift(fake, fake, 16, 12, 16, fake, 0, None, fake, 1 << 20, None) == K.KQ_ERR_INVALID_ARG
+    assert lib.kq_accum_drift(P(264), fake, 16, 8, 8, fake, 0, None, fake, 1 << 20, None) == K.KQ_ERR_INVALID_ARG
+    assert lib.kq_accum_drift(fake, fake, 16, 8, 8, fake, 0, None, None, 0, None) == K.KQ_ERR_WORKSPACE
+    assert lib.kq_accum_drift(fake, fake, 16, 8, 8, fake, 0, None, fake, 100, None) == K.KQ_ERR_WORKSPACE
+    # correction matrix: n % 4 == 0 and a workspace
+    assert lib.kq_gptaq_p(None, fake, 8, 0.25, fake, None, fake, 1 << 20, None) == K.KQ_ERR_INVALID_ARG
+    assert lib.kq_gptaq_p(fake, fake, 6, 0.25, fake, None, fake, 1 << 20, None) == K.KQ_ERR_UNSUPPORTED
+    assert lib.kq_gptaq_p(fake, fake, 8, 0.25, fake, None, fake, 16, None) == K.KQ_ERR_WORKSPACE
