@@ -305,7 +305,7 @@ def test_pipeline_with_drift_objective(trailing):
 def test_pipeline_with_drift_schedules_agree():
     """Serialized, two-stream and host-path runs of the drift pipeline give the same bits
     (fp32-ordered trailing update: every result is deterministic)."""
-    cfg, L = _layer(192, 768, 3000, 4, 128, seed=2)
+    cfg, L = _layer(224, 896, 3000, 4, 128, seed=2)
     a = _gpu_pipeline(cfg, L, overlap=False)
     b = _gpu_pipeline(cfg, L, overlap=True)
     c = _gpu_pipeline(cfg, L, overlap=True, host_path=True)
