@@ -48,6 +48,10 @@ def parse():
                     help="token chunk of the H_G accumulation (0: one call)")
     ap.add_argument("--trailing", default="3xtf32", choices=["fp32", "3xtf32"],
                     help="sweep trailing update: fp32-ordered SIMT (bit-exact) or 3xTF32 tensor cores")
+    ap.add_argument("--drift-chunk-tokens", type=int, default=0,
+                    help="token chunk of the drift statistic's launches (0: one launch)")
+    ap.add_argument("--tokens", type=int, default=0,
+                    help="override the workload's token count (small cases for profiling captures)")
     ap.add_argument("--drift", type=float, default=None, metavar="ALPHA",
                     help="with the GPTAQ drift correction of scaling ALPHA (full-precision input X~ = "
                          "X + 0.1 sigma z); default: GPTQ mode")
@@ -259,6 +263,8 @@ def max_over_ranks(v: float, ws: int, device: str = "cpu") -> float:
 def run_reference(args):
     ws, rank, _ = dist_setup("gloo")
     cfg = kqsynth.CONFIGS[args.config]
+    if args.tokens > 0:
+        cfg = cfg.replace(T=args.tokens)
     if rank != 0:
         return
     small = dict(T_s=2048, f=4, rows_s=64, alpha=args.drift)
@@ -294,12 +300,14 @@ def run_ours(args):
     torch.cuda.set_device(local)
     dev = f"cuda:{local}"
     cfg = kqsynth.CONFIGS[args.config].replace(seed=rank)
+    if args.tokens > 0:
+        cfg = cfg.replace(T=args.tokens)
     inp = kqsynth.device_layer(cfg, device=dev)
     drift = args.drift is not None
     Xt = kqsynth.device_fp_activations(cfg, inp["X"]) if drift else None
     p = LayerPipeline(cfg.d_out, cfg.d_in, cfg.bits, cfg.group, cfg.block, cfg.damp, device=dev,
                       x_chunk_tokens=args.x_chunk_tokens, g_chunk_tokens=args.g_chunk_tokens,
-                      trailing=args.trailing, alpha=args.drift)
+                      trailing=args.trailing, alpha=args.drift, drift_chunk_tokens=args.drift_chunk_tokens)
     STAGES = p.stages
     stream = torch.cuda.current_stream()
 
