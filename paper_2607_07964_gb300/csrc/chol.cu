@@ -17,25 +17,35 @@
 // block k + 1, on the caller's stream, on the critical path) and the rest (on a library
 // side stream, beside step k + 1's diagonal factorization and panel); step k + 1's own
 // first tiles wait for that rest, which also writes them.
-// All arithmetic is fp32 with fused multiply-add.
+// The diagonal, panel and first-tile kernels are fp32 SIMT with fused multiply-add. The
+// rest of each update (the bulk of the 2 n^3 / 3 flops) runs on the tensor cores with the
+// 3xTF32 split (trail_tc.cu, Cholesky mode): chol_split_kernel writes the tf32 hi / lo of
+// the panel C_{.k} and of Z_{k.} transposed (the K-major operands), then the persistent
+// tensor-core kernel updates the tiles in place (TMA load, subtract, TMA store).
 #include <math.h>
 
 #include "kq_common.cuh"
 #include "tile_gemm.cuh"
+#include "trail_tc.cuh"
 
 namespace kq {
 namespace {
 
 constexpr int NB = 128;
-constexpr int LD = NB + 1;                      // padded shared-memory row
 
 struct Work {
     float* A;      // npad x npad, reversed damped H -> C (lower)
     float* Z;      // npad x npad, B -> C^-1 (lower)
+    float* Ch;     // npad x NB each: split C_{.k} (rows of the step's update), and the split
+    float* Cl;     // transpose of Z_{k.} (row j NB + c holds Z[k NB + .][j NB + c])
+    float* Zh;
+    float* Zl;
     double* dsum;  // sum of diag(H)
 };
 
 inline size_t npad_of(int64_t n) { return static_cast<size_t>(cdiv(n, NB) * NB); }
+
+constexpr size_t ws_bytes_for(size_t np) { return (2 * np * np + 4 * np * NB) * sizeof(float) + 256; }
 
 // --------------------------------------------------------------------- prep
 __global__ void diag_sum_kernel(const float* __restrict__ H, int64_t n, double* out) {
@@ -487,45 +497,6 @@ __global__ void __launch_bounds__(G_THREADS, 2) chol_panel_kernel(Work w, int64_
     }
 }
 
-// out[tile] -= acc, loads of 32 values issued before their stores.
-template <bool BN>
-__device__ __forceinline__ void sub_tile(float* out, int64_t ld, const float (&acc)[8][8]) {
-    const int ty = threadIdx.x >> 4, tx = threadIdx.x & 15;
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-        float ov[4][8];
-#pragma unroll
-        for (int a = 0; a < 4; ++a)
-#pragma unroll
-            for (int b = 0; b < 8; ++b)
-                ov[a][b] = out[static_cast<int64_t>(gt_row(ty, 4 * h + a)) * ld + gt_col<BN>(tx, b)];
-#pragma unroll
-        for (int a = 0; a < 4; ++a)
-#pragma unroll
-            for (int b = 0; b < 8; ++b)
-                out[static_cast<int64_t>(gt_row(ty, 4 * h + a)) * ld + gt_col<BN>(tx, b)] = ov[a][b] - acc[4 * h + a][b];
-    }
-}
-
-// -------------------------------------------------------------------- update
-// Tile (i, j) of step k, k < i < nbk, 0 <= j <= i:
-//   j > k : A_ij -= C_ik C_jk^T;     j <= k : Z_ij -= C_ik Z_kj.
-__device__ __forceinline__ void update_tile(const Work& w, int64_t npad, int k, int i, int j, float* sm) {
-    const int64_t ko = static_cast<int64_t>(k) * NB;
-    const float* cik = w.A + static_cast<int64_t>(i) * NB * npad + ko;
-    const bool apart = j > k;
-    float acc[8][8];
-    if (apart)
-        gemm_tile<false, true>(cik, npad, NB, w.A + static_cast<int64_t>(j) * NB * npad + ko, npad, NB, NB, acc, sm);
-    else
-        gemm_tile<true, true>(cik, npad, NB, w.Z + ko * npad + static_cast<int64_t>(j) * NB, npad, NB, NB, acc, sm);
-    float* out = (apart ? w.A : w.Z) + static_cast<int64_t>(i) * NB * npad + static_cast<int64_t>(j) * NB;
-    if (apart)
-        sub_tile<false>(out, npad, acc);
-    else
-        sub_tile<true>(out, npad, acc);
-}
-
 // Quadrant q (rows 64 (q / 2), columns 64 (q % 2)) of update tile (i, j) of step k.
 __device__ __forceinline__ void update_quad(const Work& w, int64_t npad, int k, int i, int j, int q, float* sm) {
     const int64_t ko = static_cast<int64_t>(k) * NB;
@@ -570,16 +541,38 @@ __global__ void __launch_bounds__(G_THREADS, 2) chol_next_kernel(Work w, int64_t
         update_quad(w, npad, k, bid, k + 1, blockIdx.y, sm);
 }
 
-// The other tiles of step k: (i, j) with i > k + 1 and j != k + 1 (i tiles in row block i).
-__global__ void __launch_bounds__(G_THREADS, 2) chol_rest_kernel(Work w, int64_t npad, int k) {
-    extern __shared__ __align__(16) float sm[];
-    int bid = blockIdx.x;
-    int i = k + 2;
-    while (bid >= i) {
-        bid -= i;
-        ++i;
+// Operands of step k's tensor-core update, tf32 hi / lo: Ch/Cl rows r >= (k + 2) NB hold
+// C[r][k NB + c] (column block k of A); Zh/Zl rows q = j NB + c < (k + 1) NB hold
+// Z[k NB + c'][q] at column c' (row block k of Z, transposed through a 32 x 33 tile).
+// Block (32, 8); one 32 x 32 tile per CTA.
+__global__ void chol_split_kernel(const float* __restrict__ A, const float* __restrict__ Z, int64_t npad, int k,
+                                  float* __restrict__ Ch, float* __restrict__ Cl, float* __restrict__ Zh,
+                                  float* __restrict__ Zl) {
+    __shared__ float t[32][33];
+    const int64_t ko = static_cast<int64_t>(k) * NB;
+    const int64_t crow0 = static_cast<int64_t>(k + 2) * NB;
+    const int64_t nct = (npad - crow0) / 32 * (NB / 32);
+    int64_t b = blockIdx.x;
+    if (b < nct) {
+        const int64_t r0 = crow0 + (b / (NB / 32)) * 32, c0 = (b % (NB / 32)) * 32;
+        for (int r = threadIdx.y; r < 32; r += 8) {
+            const float x = A[(r0 + r) * npad + ko + c0 + threadIdx.x];
+            const float h = tf32_hi(x);
+            Ch[(r0 + r) * NB + c0 + threadIdx.x] = h;
+            Cl[(r0 + r) * NB + c0 + threadIdx.x] = x - h;
+        }
+        return;
     }
-    update_tile(w, npad, k, i, bid < k + 1 ? bid : bid + 1, sm);
+    b -= nct;
+    const int64_t kc0 = (b % (NB / 32)) * 32, q0 = (b / (NB / 32)) * 32;
+    for (int r = threadIdx.y; r < 32; r += 8) t[r][threadIdx.x] = Z[(ko + kc0 + r) * npad + q0 + threadIdx.x];
+    __syncthreads();
+    for (int r = threadIdx.y; r < 32; r += 8) {
+        const float x = t[threadIdx.x][r];   // Z[ko + kc0 + threadIdx.x][q0 + r]
+        const float h = tf32_hi(x);
+        Zh[(q0 + r) * NB + kc0 + threadIdx.x] = h;
+        Zl[(q0 + r) * NB + kc0 + threadIdx.x] = x - h;
+    }
 }
 
 // -------------------------------------------------------------------- finish
@@ -609,8 +602,7 @@ using namespace kq;
 
 extern "C" size_t kq_chol_inv_workspace(int64_t n) {
     if (n < 1) return 0;
-    const size_t np = npad_of(n);
-    return 2 * np * np * sizeof(float) + 256;
+    return ws_bytes_for(npad_of(n));
 }
 
 extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, float* Lt, int* info, void* ws,
@@ -630,7 +622,16 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
     Work w;
     w.A = static_cast<float*>(ws);
     w.Z = w.A + npad * npad;
-    w.dsum = reinterpret_cast<double*>(w.Z + npad * npad);
+    w.Ch = w.Z + npad * npad;
+    w.Cl = w.Ch + npad * NB;
+    w.Zh = w.Cl + npad * NB;
+    w.Zl = w.Zh + npad * NB;
+    w.dsum = reinterpret_cast<double*>(w.Zl + npad * NB);
+    CholTcMaps maps;
+    if (nbk > 2) {
+        kq_status st = maps.init(w.A, w.Z, w.Ch, w.Cl, w.Zh, w.Zl, npad);
+        if (st != KQ_OK) return st;
+    }
     static bool attr = false;
     if (!attr) {
         KQ_CUDA(cudaFuncSetAttribute(chol_diag_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -639,8 +640,6 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
                                      static_cast<int>(STRIP_SMEM)));
         KQ_CUDA(cudaFuncSetAttribute(chol_next_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(STRIP_SMEM)));
-        KQ_CUDA(cudaFuncSetAttribute(chol_rest_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     static_cast<int>(G_SMEM)));
         attr = true;
     }
     diag_sum_kernel<<<1, 1024, 0, stream>>>(H, n, w.dsum);
@@ -672,8 +671,13 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
                 KQ_CUDA(cudaStreamWaitEvent(side->s, side->ev[0], 0));
                 rs = side->s;
             }
-            chol_rest_kernel<<<static_cast<unsigned>(rest), G_THREADS, G_SMEM, rs>>>(w, npad, k);
-            KQ_LAUNCH_CHECK("chol_rest_kernel");
+            const int64_t split_tiles = (npad - static_cast<int64_t>(k + 2) * NB) / 32 * (NB / 32) +
+                                        static_cast<int64_t>(k + 1) * NB / 32 * (NB / 32);
+            chol_split_kernel<<<static_cast<unsigned>(split_tiles), dim3(32, 8), 0, rs>>>(w.A, w.Z, npad, k, w.Ch, w.Cl,
+                                                                                          w.Zh, w.Zl);
+            KQ_LAUNCH_CHECK("chol_split_kernel");
+            kq_status st = chol_rest_tc(maps, nbk, k, info, rs);
+            if (st != KQ_OK) return st;
             if (fork) {
                 KQ_CUDA(cudaEventRecord(side->ev[1], side->s));
                 forked = true;
@@ -696,8 +700,7 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
 #include <mutex>
 
 namespace {
-constexpr size_t kNoallocBytes =
-    2 * static_cast<size_t>(KQ_CHOL_NOALLOC_MAX_N) * KQ_CHOL_NOALLOC_MAX_N * sizeof(float) + 256;
+constexpr size_t kNoallocBytes = kq::ws_bytes_for(KQ_CHOL_NOALLOC_MAX_N);
 static __device__ __align__(256) unsigned char g_chol_scratch[kNoallocBytes];
 std::mutex g_noalloc_mu;
 void* g_noalloc_ptr[64] = {};

@@ -51,14 +51,50 @@ __device__ __forceinline__ bool wait_quiet(uint64_t* bar, uint32_t parity) {
     return mbar_wait(bar, parity, &dummy);
 }
 
+// Which output tiles a launch updates, and from which operand maps.
+//   mode 0 (the sweep): a row x column grid over W[:, cb:], K slabs at columns i0 + 32 s of
+//     the first pair (E with R) and, for slabs >= 4, of the second pair (-Wpre with P).
+//   mode 1 (a Cholesky step k, see chol.cu): the lower tiles (i, j) of the padded matrix
+//     with i >= k + 2, j <= i, j != k + 1; K = 128 slabs at columns 32 s of the split
+//     column block C_{.k}; B from the C pair (j > k, output A) or from the transposed Z_{k.}
+//     pair (j <= k, output Z).
+struct TileSet {
+    int mode;
+    int n_tiles;
+    int n_col_tiles, cb, i0;   // mode 0
+    int k;                     // mode 1
+};
+
+// Tile t: top-left corner (row r0, column c0) and whether it takes the second B pair and
+// the second W map.
+__device__ __forceinline__ void tile_at(const TileSet& ts, int t, int bn, int* r0, int* c0, bool* alt) {
+    if (ts.mode == 0) {
+        *r0 = (t / ts.n_col_tiles) * TBM;
+        *c0 = ts.cb + (t % ts.n_col_tiles) * bn;
+        *alt = false;
+        return;
+    }
+    int i = ts.k + 2;
+    while (t >= i) {
+        t -= i;
+        ++i;
+    }
+    const int j = t < ts.k + 1 ? t : t + 1;
+    *r0 = i * TBM;
+    *c0 = j * TBM;
+    *alt = j <= ts.k;
+}
+
 template <int BN, int TSTAGES>
 __global__ void __launch_bounds__(T_THREADS, 1)
 trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__ CUtensorMap mEl,
                 const __grid_constant__ CUtensorMap mRh, const __grid_constant__ CUtensorMap mRl,
                 const __grid_constant__ CUtensorMap mQh, const __grid_constant__ CUtensorMap mQl,
                 const __grid_constant__ CUtensorMap mPh, const __grid_constant__ CUtensorMap mPl,
-                const __grid_constant__ CUtensorMap mW, int d_out, int i0, int cb, int n_col_tiles, int n_tiles,
+                const __grid_constant__ CUtensorMap mW, const __grid_constant__ CUtensorMap mW2, TileSet ts,
                 int nslab, int* info) {
+    const int n_tiles = ts.n_tiles;
+    const int xk = ts.mode == 0 ? ts.i0 : 0;
     using C = TrailCfg<BN, TSTAGES>;
     constexpr int WBOX = TBM * 32 * 4;     // one 128-row x 32-column box of W (16 KB)
     extern __shared__ uint8_t smem_raw[];
@@ -105,7 +141,8 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
         tma_prefetch_desc(&mRh);
         tma_prefetch_desc(&mRl);
         tma_prefetch_desc(&mW);
-        if (nslab > TNSLAB) {
+        if (ts.mode == 1) tma_prefetch_desc(&mW2);
+        if (nslab > TNSLAB || ts.mode == 1) {
             tma_prefetch_desc(&mQh);
             tma_prefetch_desc(&mQl);
             tma_prefetch_desc(&mPh);
@@ -123,13 +160,15 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
             int k = 0, li = 0, w_issued = 0;
             bool ok = true;
             for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++li) {
-                const int r0 = (t / n_col_tiles) * TBM;
-                const int c0 = cb + (t % n_col_tiles) * BN;
+                int r0, c0;
+                bool alt;
+                tile_at(ts, t, BN, &r0, &c0, &alt);
+                const CUtensorMap* wm = alt ? &mW2 : &mW;
                 // the tile of W, once the previous tile has been stored from the buffer
                 if (!mbar_wait(wfree, (static_cast<uint32_t>(li) & 1u) ^ 1u, abort_flag)) break;
                 mbar_arrive_expect_tx(wfull, C::WTILE);
 #pragma unroll
-                for (int j = 0; j < BN / 32; ++j) tma_load_2d(wtile + j * WBOX, &mW, wfull, c0 + 32 * j, r0);
+                for (int j = 0; j < BN / 32; ++j) tma_load_2d(wtile + j * WBOX, wm, wfull, c0 + 32 * j, r0);
                 w_issued = li + 1;
                 for (int s = 0; s < nslab; ++s, ++k) {
                     const int st = k % TSTAGES;
@@ -140,13 +179,15 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
                     }
                     mbar_arrive_expect_tx(&full[st], C::STAGE);
                     uint8_t* base = smem + st * C::STAGE;
-                    // slabs 0..3: E and R; slabs 4..7 (with P): -Wpre and P
+                    // slabs 0..3: E and R; slabs 4..7 (with P): -Wpre and P. Cholesky tiles
+                    // with j <= k take B from the second pair.
                     const bool second = s >= TNSLAB;
-                    const int x = i0 + (second ? s - TNSLAB : s) * TBK;
+                    const bool bsec = second || alt;
+                    const int x = xk + (second ? s - TNSLAB : s) * TBK;
                     tma_load_2d(base, second ? &mQh : &mEh, &full[st], x, r0);
                     tma_load_2d(base + A_SLAB, second ? &mQl : &mEl, &full[st], x, r0);
-                    tma_load_2d(base + 2 * A_SLAB, second ? &mPh : &mRh, &full[st], x, c0);
-                    tma_load_2d(base + 2 * A_SLAB + C::B_SLAB, second ? &mPl : &mRl, &full[st], x, c0);
+                    tma_load_2d(base + 2 * A_SLAB, bsec ? &mPh : &mRh, &full[st], x, c0);
+                    tma_load_2d(base + 2 * A_SLAB + C::B_SLAB, bsec ? &mPl : &mRl, &full[st], x, c0);
                 }
             }
             // every issued load must land before the CTA exits
@@ -236,10 +277,12 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
             if (warp == 2 && lane == 0) {
                 // store the tile once every warp has updated it, then free the buffer
                 if (mbar_wait(wdone, static_cast<uint32_t>(li) & 1u, abort_flag)) {
-                    const int r0 = (t / n_col_tiles) * TBM;
-                    const int c0 = cb + (t % n_col_tiles) * BN;
+                    int r0, c0;
+                    bool alt;
+                    tile_at(ts, t, BN, &r0, &c0, &alt);
+                    const CUtensorMap* wm = alt ? &mW2 : &mW;
 #pragma unroll
-                    for (int j = 0; j < BN / 32; ++j) tma_store_2d(&mW, wtile + j * WBOX, c0 + 32 * j, r0);
+                    for (int j = 0; j < BN / 32; ++j) tma_store_2d(wm, wtile + j * WBOX, c0 + 32 * j, r0);
                     bulk_commit();
                     bulk_wait_read0();
                     mbar_arrive(wfree);
@@ -358,11 +401,46 @@ kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, in
     }
     const int n_row = static_cast<int>(cdiv(d_out, TBM));
     const int n_col = static_cast<int>(cdiv(ce - cb, 128));
-    const int n = n_row * n_col;
-    trail_tc_kernel<128, 2><<<static_cast<unsigned>(std::min(n, num_sms())), T_THREADS, Cfg::SMEM, stream>>>(
+    TileSet ts{};
+    ts.mode = 0;
+    ts.n_tiles = n_row * n_col;
+    ts.n_col_tiles = n_col;
+    ts.cb = static_cast<int>(cb);
+    ts.i0 = static_cast<int>(i0);
+    trail_tc_kernel<128, 2><<<static_cast<unsigned>(std::min(ts.n_tiles, num_sms())), T_THREADS, Cfg::SMEM, stream>>>(
         m.eh, m.el, m.rh_narrow, m.rl_narrow, with_p ? m.qh : m.eh, with_p ? m.ql : m.el,
-        with_p ? m.ph : m.rh_narrow, with_p ? m.pl : m.rl_narrow, m.w, static_cast<int>(d_out), static_cast<int>(i0),
-        static_cast<int>(cb), n_col, n, with_p ? 2 * TNSLAB : TNSLAB, info);
+        with_p ? m.ph : m.rh_narrow, with_p ? m.pl : m.rl_narrow, m.w, m.w, ts, with_p ? 2 * TNSLAB : TNSLAB, info);
+    KQ_LAUNCH_CHECK("trail_tc_kernel");
+    return KQ_OK;
+}
+
+// ------------------------------------------------------------ Cholesky step updates
+kq_status CholTcMaps::init(float* A, float* Z, const float* Ch, const float* Cl, const float* Zh, const float* Zl,
+                           int64_t npad) {
+    kq_status st;
+    if ((st = make_f32_map(&a, A, npad, npad, TBM)) != KQ_OK) return st;
+    if ((st = make_f32_map(&z, Z, npad, npad, TBM)) != KQ_OK) return st;
+    if ((st = make_f32_map(&ch, Ch, npad, 128, TBM)) != KQ_OK) return st;
+    if ((st = make_f32_map(&cl, Cl, npad, 128, TBM)) != KQ_OK) return st;
+    if ((st = make_f32_map(&zh, Zh, npad, 128, TBM)) != KQ_OK) return st;
+    if ((st = make_f32_map(&zl, Zl, npad, 128, TBM)) != KQ_OK) return st;
+    return KQ_OK;
+}
+
+kq_status chol_rest_tc(const CholTcMaps& m, int nbk, int k, int* info, cudaStream_t stream) {
+    using Cfg = TrailCfg<128, 2>;
+    static bool attr = false;
+    if (!attr) {
+        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<128, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
+        attr = true;
+    }
+    TileSet ts{};
+    ts.mode = 1;
+    ts.k = k;
+    for (int i = k + 2; i < nbk; ++i) ts.n_tiles += i;
+    if (ts.n_tiles == 0) return KQ_OK;
+    trail_tc_kernel<128, 2><<<static_cast<unsigned>(std::min(ts.n_tiles, num_sms())), T_THREADS, Cfg::SMEM, stream>>>(
+        m.ch, m.cl, m.ch, m.cl, m.ch, m.cl, m.zh, m.zl, m.a, m.z, ts, TNSLAB, info);
     KQ_LAUNCH_CHECK("trail_tc_kernel");
     return KQ_OK;
 }

@@ -58,6 +58,19 @@ struct TrailMaps {
     kq_status set_w(float* W, int64_t d_out, int64_t d_in);
 };
 
+// Tensor maps of one inverse-Cholesky call (chol.cu): the padded A (-> C) and Z, and the
+// split operands of a step's update, C_{.k} and the transposed Z_{k.} ([npad x 128] each).
+struct CholTcMaps {
+    CUtensorMap a, z, ch, cl, zh, zl;
+    kq_status init(float* A, float* Z, const float* Ch, const float* Cl, const float* Zh, const float* Zl,
+                   int64_t npad);
+};
+
+// Step k's update of every tile the next step does not read first: A_ij -= C_ik C_jk^T
+// (j > k) and Z_ij -= C_ik Z_kj (j <= k) for block rows i >= k + 2, j <= i, j != k + 1, on
+// the tensor cores (3xTF32, K = 128), from the split operands in Ch/Cl and Zh/Zl.
+kq_status chol_rest_tc(const CholTcMaps& m, int nbk, int k, int* info, cudaStream_t stream);
+
 // hi = src rounded to tf32, lo = src - hi (n elements).
 kq_status split_tf32(const float* src, int64_t n, float* hi, float* lo, cudaStream_t stream);
 
