@@ -48,6 +48,10 @@ def parse():
                     help="token chunk of the H_G accumulation (0: one call)")
     ap.add_argument("--trailing", default="3xtf32", choices=["fp32", "3xtf32"],
                     help="sweep trailing update: fp32-ordered SIMT (bit-exact) or 3xTF32 tensor cores")
+    ap.add_argument("--block", default=None, choices=sorted(kqsynth.BLOCKS),
+                    help="a whole transformer block (seven sublayers, shared H_X, W2/W3 allocation) "
+                         "instead of one layer")
+    ap.add_argument("--lanes", type=int, default=2, help="sublayers quantized concurrently in --block mode")
     ap.add_argument("--drift-chunk-tokens", type=int, default=0,
                     help="token chunk of the drift statistic's launches (0: one launch)")
     ap.add_argument("--tokens", type=int, default=0,
@@ -430,9 +434,181 @@ def run_ours(args):
         torch.distributed.destroy_process_group()
 
 
+# ------------------------------------------------------------------ transformer block
+BLOCK_METRIC = "ms per transformer block (7 sublayers: shared H_X, W2/W3 allocation, rotate+chol+sweep)"
+
+
+def block_config_dict(bc, lanes) -> dict:
+    return {"workload": (f"{bc.name}: d_model {bc.d_model}, d_kv {bc.d_kv}, d_ff {bc.d_ff}, T={bc.T} tokens, "
+                         f"W{bc.low_bits}/W{bc.high_bits} at mean {bc.budget} bits, group {bc.group}"),
+            "d_model": bc.d_model, "d_kv": bc.d_kv, "d_ff": bc.d_ff, "T": bc.T, "group": bc.group,
+            "bits": [bc.low_bits, bc.high_bits], "budget_bits": bc.budget, "lanes": lanes,
+            "l2": "inputs larger than L2 (every X and G is T x d bf16); no flush"}
+
+
+def block_flops(bc) -> dict:
+    spec = kqsynth.block_spec(bc)
+    d_in = {grp: d for _, grp, _, d in spec}
+    fx = sum(bc.T * d * (d + 1) for d in d_in.values())
+    fg = sum(bc.T * d_out * (d_out + 1) for _, _, d_out, _ in spec)
+    return {"factors": fx + fg, "factor_x": fx, "factor_g": fg}
+
+
+def oracle_block_ms(bc, small: bool = False) -> dict:
+    """The oracle's time for a block: the layer estimate of oracle_sample_ms per sublayer,
+    minus the H_X accumulations the shared inputs do not repeat."""
+    spec = kqsynth.block_spec(bc)
+    kw = dict(T_s=2048, f=4, rows_s=64) if small else {}
+    total, seen, parts = 0.0, set(), {}
+    for name, grp, d_out, d_in in spec:
+        c = kqsynth.LayerConfig(name, d_out, d_in, bc.T, bc.low_bits, bc.group, bc.n_outliers, bc.g_sigma,
+                                block=bc.block, damp=bc.damp)
+        r = oracle_sample_ms(c, **kw)
+        v = r["value"]
+        if grp in seen:   # H_X of a shared input is accumulated once: drop this layer's X share
+            v -= r["stages_ms"]["factors"] * d_in * d_in / (d_in * d_in + d_out * d_out)
+        seen.add(grp)
+        parts[name] = v
+        total += v
+    return {"value": total, "unit": "ms", "cores": os.cpu_count(), "kind": "oracle", "sublayers_ms": parts,
+            "sample": "per sublayer the single-layer sample of oracle_sample_ms" + (" (reduced)" if small else "")
+                      + "; shared H_X counted once"}
+
+
+def run_block(args):
+    import torch
+
+    from paper_2607_07964_gb300 import build as kbuild
+    ws, rank, local = dist_setup("nccl")
+    kbuild.build()
+    from paper_2607_07964_gb300 import kronq as kq
+    from paper_2607_07964_gb300.block import BlockQuantizer
+
+    torch.cuda.set_device(local)
+    dev = f"cuda:{local}"
+    bc = kqsynth.BLOCKS[args.block].replace(seed=rank)
+    if args.tokens > 0:
+        bc = bc.replace(T=args.tokens)
+    spec = kqsynth.block_spec(bc)
+    inp = kqsynth.device_block(bc, device=dev)
+    q = BlockQuantizer(spec, bc.group, bc.block, bc.damp, bc.low_bits, bc.high_bits, bc.budget, device=dev,
+                       trailing=args.trailing, lanes=args.lanes)
+    stream = torch.cuda.current_stream()
+    args_in = (inp["X"], inp["G"], inp["W"], inp["sign_u"], inp["sign_v"])
+    for _ in range(args.warmup):
+        q.run(*args_in, stream=stream)
+    q.check()
+
+    def barrier():
+        if ws > 1:
+            torch.distributed.barrier()
+
+    sampler = ClockSampler(None)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    fac_ms, tot_ms = [], []
+    barrier()
+    torch.cuda.synchronize()
+    sampler.start()
+    n0 = kq.launch_count()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(args.steps):
+        ev[0].record(stream)
+        q.factors(inp["X"], inp["G"], stream)
+        ev[1].record(stream)
+        sc = q.scores(inp["W"], stream)
+        bits = q.allocate(sc)
+        q.quantize(inp["W"], inp["sign_u"], inp["sign_v"], bits, stream)
+        ev[2].record(stream)
+        torch.cuda.synchronize()
+        fac_ms.append(ev[0].elapsed_time(ev[1]))
+        tot_ms.append(ev[0].elapsed_time(ev[2]))
+    t1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    launches = kq.launch_count() - n0
+    clocks = sampler.stop()
+    q.check()
+    total = max_over_ranks(t0.elapsed_time(t1), ws, dev)
+    fl = block_flops(bc)
+    peaks, peak_src = measured_peaks()
+    peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+    fac = statistics.mean(fac_ms)
+    achieved = fl["factors"] / fac / 1e9
+    roofline = {"kernel": "syrk_tc_kernel (the block's 4 H_X and 7 H_G accumulations, back to back)",
+                "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
+                "traffic": None, "peak_source": f"{peak_src} bf16 dense burst",
+                "algorithmic_flops_per_launch": fl["factors"] / 11, "launches": 11}
+    e2e = None
+    if not args.no_e2e:
+        hosts = {k: {n: t.cpu().pin_memory() for n, t in d.items()} for k, d in zip(
+            ("X", "G", "W", "sign_u", "sign_v"), args_in)}
+        outs = {n: (torch.empty(p.codes.shape, dtype=torch.uint8).pin_memory(),
+                    torch.empty(p.scale.shape).pin_memory(), torch.empty(p.zero.shape, dtype=torch.int32).pin_memory())
+                for n, p in q.pipes.items()}
+        nin = sum(t.numel() * t.element_size() for d in hosts.values() for t in d.values())
+        nout = sum(t.numel() * t.element_size() for o in outs.values() for t in o)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(args.steps):
+            for key, d in hosts.items():
+                for n, t in d.items():
+                    args_in[("X", "G", "W", "sign_u", "sign_v").index(key)][n].copy_(t, non_blocking=True)
+            q.run(*args_in, stream=stream)
+            for n, (c, s_, z) in outs.items():
+                p = q.pipes[n]
+                c.copy_(p.codes, non_blocking=True)
+                s_.copy_(p.scale, non_blocking=True)
+                z.copy_(p.zero, non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e2e = {"value": max_over_ranks(e0.elapsed_time(e1), ws, dev) / (ws * args.steps), "unit": "ms",
+               "h2d_bytes_per_step": nin, "d2h_bytes_per_step": nout,
+               "note": "copies, then the block (no overlap of copies with compute)"}
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        cpu = oracle_block_ms(bc)
+    if rank == 0:
+        out = {"metric": BLOCK_METRIC, "value": total / (ws * args.steps), "unit": "ms", "n_gpus": ws,
+               "steps": args.steps, "warmup": args.warmup, "ms_per_step": total / args.steps,
+               "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
+               "dtype": "bf16 products, f32 accumulate/arithmetic", "data": "synthetic",
+               "config": block_config_dict(bc, args.lanes),
+               "stages_ms": {"factors": fac, "scores_alloc_quantize": statistics.mean(tot_ms) - fac},
+               "bits": bits, "scores_post_biip": {n: sc[n][5] for n in sc},
+               "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches // args.steps,
+               "launch_mode": "direct launches; one host sync per block for the allocation", "clocks": clocks}
+        print(json.dumps(out), flush=True)
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+
+
 def main():
     args = parse()
-    if args.impl == "reference":
+    if args.block is not None:
+        if args.impl == "reference":
+            ws, rank, _ = dist_setup("gloo")
+            if rank == 0:
+                bc = kqsynth.BLOCKS[args.block]
+                if args.tokens > 0:
+                    bc = bc.replace(T=args.tokens)
+                t0 = time.perf_counter()
+                vals = [oracle_block_ms(bc, small=True)["value"] for _ in range(args.steps)]
+                v = statistics.mean(vals)
+                print(json.dumps({"impl": "reference", "metric": BLOCK_METRIC, "value": v, "unit": "ms",
+                                  "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+                                  "ms_per_step": v, "higher_is_better": False, "scaling": "weak",
+                                  "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+                                  "config": block_config_dict(bc, args.lanes),
+                                  "cpu_baseline": {"value": v, "unit": "ms", "cores": os.cpu_count(),
+                                                   "kind": "oracle", "sample": "reduced single-layer samples"},
+                                  "e2e": {"value": v, "unit": "ms", "h2d_bytes_per_step": 0,
+                                          "d2h_bytes_per_step": 0},
+                                  "wall_s": time.perf_counter() - t0}), flush=True)
+        else:
+            run_block(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_ours(args)

@@ -201,3 +201,85 @@ def device_fp_activations(cfg: LayerConfig, X, drift: float = 0.1):
         z = torch.randn((t1 - t0, cfg.d_in), generator=gen, device=X.device)
         Xt[t0:t1] = (X[t0:t1].float() + z * sx_t).to(torch.bfloat16)
     return Xt
+
+
+# ------------------------------------------------------------------ transformer blocks
+@dataclasses.dataclass(frozen=True)
+class BlockConfig:
+    """One Llama-style transformer block: attention q, k, v (shared input), o, and MLP
+    gate, up (shared input), down; the bit widths and the mean-bits budget of the W2 -> W3
+    allocation."""
+    name: str
+    d_model: int
+    d_kv: int
+    d_ff: int
+    T: int
+    group: int = 128
+    block: int = 128
+    damp: float = 0.01
+    low_bits: int = 2
+    high_bits: int = 3
+    budget: float = 2.5
+    n_outliers: int = 16
+    g_sigma: float = 1.5
+    w_bf16: bool = True
+    seed: int = 0
+
+    def replace(self, **kw) -> "BlockConfig":
+        return dataclasses.replace(self, **kw)
+
+
+BLOCKS = {
+    "tiny_block": BlockConfig("tiny_block", 256, 64, 512, 2048, n_outliers=4),
+    "llama3_8b_block": BlockConfig("llama3_8b_block", 4096, 1024, 14336, 131072),
+}
+
+INPUTS = ("attn", "o", "mlp", "down")
+
+
+def block_spec(cfg: BlockConfig) -> list[tuple[str, str, int, int]]:
+    """(sublayer, input group, d_out, d_in) of the seven linear sublayers: q, k, v read the
+    attention input, gate and up the MLP input."""
+    m, kv, ff = cfg.d_model, cfg.d_kv, cfg.d_ff
+    return [("q", "attn", m, m), ("k", "attn", kv, m), ("v", "attn", kv, m), ("o", "o", m, m),
+            ("gate", "mlp", ff, m), ("up", "mlp", ff, m), ("down", "down", m, ff)]
+
+
+def _input_dim(cfg: BlockConfig, group: str) -> int:
+    return cfg.d_ff if group == "down" else cfg.d_model
+
+
+def _sub_cfg(cfg: BlockConfig, d_out: int, d_in: int, k: int) -> LayerConfig:
+    return LayerConfig(f"{cfg.name}.{k}", d_out, d_in, cfg.T, cfg.low_bits, cfg.group, cfg.n_outliers,
+                       cfg.g_sigma, w_bf16=cfg.w_bf16, block=cfg.block, damp=cfg.damp, seed=cfg.seed * 64 + k)
+
+
+def block_inputs(cfg: BlockConfig) -> dict:
+    """Host inputs of a block: X per input group, and G, W, signs per sublayer (each tensor
+    drawn from its own sub-seed with the single-layer recipe)."""
+    X = {g: activations(_sub_cfg(cfg, 8, _input_dim(cfg, g), 1 + i)) for i, g in enumerate(INPUTS)}
+    out = {"X": X, "G": {}, "W": {}, "sign_u": {}, "sign_v": {}}
+    for k, (name, _, d_out, d_in) in enumerate(block_spec(cfg)):
+        c = _sub_cfg(cfg, d_out, d_in, 16 + k)
+        out["G"][name] = gradients(c)
+        out["W"][name] = weights(c)
+        out["sign_u"][name], out["sign_v"][name] = signs(c)
+    return out
+
+
+def device_block(cfg: BlockConfig, device: str = "cuda") -> dict:
+    """The block's inputs drawn on the GPU (same recipe as block_inputs, torch's generator)."""
+    import torch
+
+    X = {}
+    for i, g in enumerate(INPUTS):
+        X[g] = device_layer(_sub_cfg(cfg, 8, _input_dim(cfg, g), 1 + i), device)["X"]
+        torch.cuda.empty_cache()
+    out = {"X": X, "G": {}, "W": {}, "sign_u": {}, "sign_v": {}}
+    for k, (name, _, d_out, d_in) in enumerate(block_spec(cfg)):
+        d = device_layer(_sub_cfg(cfg, d_out, d_in, 16 + k).replace(T=cfg.T), device)
+        out["G"][name], out["W"][name] = d["G"], d["W"]
+        out["sign_u"][name], out["sign_v"][name] = d["sign_u"], d["sign_v"]
+        del d
+        torch.cuda.empty_cache()
+    return out

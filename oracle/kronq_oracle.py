@@ -14,6 +14,7 @@ It follows "KronQ: LLM Quantization via Kronecker-Factored Hessian":
                                Proposition 1 (P), Algorithms 1 and 2 (Delta X X^T, P)
   * revert and proxy loss      Algorithm 2, Sec. 3.1 Eq. (kron_obj), Theorem 1
   * sensitivity traces         Sec. 3.3 Eq. (sensitivity)
+  * mixed-precision allocation Sec. 3.3, Sec. 5 "Results on Mixed-precision" (W2 -> W3)
 Tokens are stored as rows here (X is T x d_in), so the paper's X X^T is X^T X.
 
 Readings of points the paper leaves open (all listed in the design notes):
@@ -28,7 +29,10 @@ Readings of points the paper leaves open (all listed in the design notes):
   * the per-column loss is sum over rows of E_j^2 (no 1/2);
   * the drift statistic is D = (X~ - X)^T X (tokens as rows), transformed like H_X;
   * W_{:,j} in the P terms of Proposition 1 and Algorithm 2 is column j's value just
-    before it is quantized, in the column update and in the lazy trailing update alike.
+    before it is quantized, in the column update and in the lazy trailing update alike;
+  * the W2 -> W3 allocation upgrades sublayers in descending post-BiIP score while the
+    parameter-weighted mean bit width stays within the budget, stopping at the first
+    upgrade that would exceed it (ties keep the listed order).
 """
 from __future__ import annotations
 
@@ -38,7 +42,8 @@ __all__ = [
     "accum_factor", "factor_entries", "factor_diag", "biip_scales_from_diag", "sylvester", "paley28", "hadamard_matrix", "rht_matrix",
     "biip_scales", "biip", "damp", "inverse_cholesky_upper", "lower_factor",
     "quant_params", "quantize", "obs_sweep", "dequant", "revert", "proxy_loss",
-    "traces", "pipeline", "drift_factor", "gptaq_p", "objective",
+    "traces", "pipeline", "drift_factor", "gptaq_p", "objective", "allocate_bits", "block_scores",
+    "block_pipeline",
 ]
 
 
@@ -394,3 +399,56 @@ def pipeline(X, G, W, sign_u, sign_v, bits: int, group: int, block: int = 128,
     out.update(sw)
     out.update(traces(HX, HG, b["HX"], b["HG"]))
     return out
+
+
+# ----------------------------------------------------------------------------------
+# Mixed-precision allocation across the sublayers of a block (Sec. 3.3 Eq. sensitivity;
+# Sec. 5 "Results on Mixed-precision": the most sensitive sublayers go from W2 to W3).
+# ----------------------------------------------------------------------------------
+def allocate_bits(scores: dict, params: dict, low: int, high: int, budget: float) -> dict:
+    """Upgrade sublayers from `low` to `high` bits in descending score, one at a time, while
+    the parameter-weighted mean bit width sum(bits * params) / sum(params) stays within
+    `budget`; the first upgrade that would exceed it ends the allocation. Equal scores keep
+    the order of `scores`."""
+    names = list(scores)
+    order = sorted(range(len(names)), key=lambda i: -scores[names[i]])   # stable
+    total = float(sum(params[n] for n in names))
+    bits = {n: low for n in names}
+    used = low * total
+    for i in order:
+        n = names[i]
+        if (used + (high - low) * params[n]) / total > budget:
+            break
+        bits[n] = high
+        used += (high - low) * params[n]
+    return bits
+
+
+def block_scores(X: dict, G: dict, W: dict, spec) -> dict:
+    """Per sublayer: raw and post-BiIP traces and the sensitivity s = tr(H_G) tr(H_X)
+    (Eq. sensitivity, computed post-BiIP). spec lists (name, input group, d_out, d_in);
+    sublayers of one input group share H_X."""
+    HX = {g: accum_factor(X[g]) for g in {grp for _, grp, _, _ in spec}}
+    out = {}
+    for name, grp, _, _ in spec:
+        HG = accum_factor(G[name])
+        sx, sg = biip_scales(W[name], HX[grp], HG)
+        hx, hg = np.diag(HX[grp]), np.diag(HG)
+        out[name] = {"trHX": float(np.sum(hx)), "trHG": float(np.sum(hg)),
+                     "trHX_post": float(np.sum(hx / sx ** 2)), "trHG_post": float(np.sum(hg / sg ** 2))}
+        out[name]["s"] = out[name]["trHX"] * out[name]["trHG"]
+        out[name]["s_post"] = out[name]["trHX_post"] * out[name]["trHG_post"]
+    return out
+
+
+def block_pipeline(X: dict, G: dict, W: dict, sign_u: dict, sign_v: dict, spec, group: int, low: int, high: int,
+                   budget: float, block: int = 128, lam: float = 0.01) -> dict:
+    """A transformer block: scores, the W2 -> W3 allocation, then each sublayer through
+    Algorithms 1 and 2 at its allocated bit width."""
+    sc = block_scores(X, G, W, spec)
+    params = {name: d_out * d_in for name, _, d_out, d_in in spec}
+    bits = allocate_bits({n: sc[n]["s_post"] for n, _, _, _ in spec}, params, low, high, budget)
+    res = {}
+    for name, grp, _, _ in spec:
+        res[name] = pipeline(X[grp], G[name], W[name], sign_u[name], sign_v[name], bits[name], group, block, lam)
+    return {"scores": sc, "bits": bits, "layers": res}

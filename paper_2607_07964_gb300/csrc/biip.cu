@@ -14,6 +14,7 @@
 #include <math.h>
 
 #include <algorithm>
+#include <utility>
 
 #include "kq_common.cuh"
 #include "sumsq.cuh"
@@ -70,7 +71,6 @@ constexpr bool h28_is_hadamard() {
     return true;
 }
 static_assert(h28_is_hadamard(), "H_28 must satisfy H H^T = 28 I and be symmetric");
-__constant__ H28Masks c_h28 = make_h28();
 
 // Factor applied to element index j before (pre) or after (post) a transform.
 enum FactorMode { F_NONE = 0, F_SMUL = 1, F_SDIV = 2, F_SIGN = 3 };
@@ -82,16 +82,27 @@ __device__ __forceinline__ float factor(int mode, const int8_t* sign, const floa
     return mode == F_SMUL ? sg * s[j] : sg / s[j];
 }
 
-// y = H_28 x for 28 values in registers.
-__device__ __forceinline__ void mix28(const float (&x)[28], float (&y)[28]) {
+// y = H_28 x for 28 values in registers, each output handed to out(r, y_r) as soon as it is
+// formed (only x stays live). Each row's sign mask is a template argument taken from the
+// compile-time table kH28, so every term is a plain add or subtract.
+constexpr H28Masks kH28 = make_h28();
+
+template <uint32_t M>
+__device__ __forceinline__ float pm_sum28(const float (&x)[28]) {
+    float acc = 0.0f;
 #pragma unroll
-    for (int r = 0; r < 28; ++r) {
-        const uint32_t m = c_h28.m[r];
-        float acc = 0.0f;
-#pragma unroll
-        for (int a = 0; a < 28; ++a) acc += ((m >> a) & 1u) ? -x[a] : x[a];
-        y[r] = acc;
-    }
+    for (int a = 0; a < 28; ++a) acc = ((M >> a) & 1u) ? acc - x[a] : acc + x[a];
+    return acc;
+}
+
+template <typename Out, int... R>
+__device__ __forceinline__ void mix28_rows(const float (&x)[28], Out& out, std::integer_sequence<int, R...>) {
+    (out(R, pm_sum28<kH28.m[R]>(x)), ...);
+}
+
+template <typename Out>
+__device__ __forceinline__ void mix28(const float (&x)[28], Out out) {
+    mix28_rows(x, out, std::make_integer_sequence<int, 28>{});
 }
 
 // In-register Walsh-Hadamard transform of R = 2, 4 or 8 values (natural order).
@@ -155,18 +166,40 @@ __device__ __forceinline__ void stage_row(float* v, const float* src, int n) {
 
 // ------------------------------------------------------------------ row transform
 // For each row of M [rows x n]: v <- pre (.) v; v <- (H_28 (x) H_P) v (or H_P); row <-
-// post (.) v / sqrt(n). One CTA per row (grid-stride); n floats of shared memory. The row
-// is staged with cp.async, the power-of-two part runs as radix-8 passes (one barrier per
-// pass), and the last pass writes straight to global memory.
+// post (.) v / sqrt(n). A CTA walks rows r = blockIdx.x, + gridDim.x, ... with two shared
+// row buffers when they fit (DBL): the next row's cp.async copy is issued before the
+// current row's butterflies, so loads overlap compute within the CTA. The power-of-two
+// part runs as radix-8 passes (one barrier per pass); the last pass (or the 28-point mix)
+// writes straight to global memory.
 template <bool HAS28>
-__global__ void __launch_bounds__(HAS28 ? 256 : 512, HAS28 ? 1 : 2) rht_rows_kernel(float* __restrict__ M, int64_t rows, int n, int lgP,
+__global__ void __launch_bounds__(256, HAS28 ? 2 : 4) rht_rows_kernel(float* __restrict__ M, int64_t rows, int n, int lgP,
                                 int pre_mode, int post_mode, const int8_t* __restrict__ sign,
-                                const float* __restrict__ s, float inv_sqrt_n) {
-    extern __shared__ __align__(16) float v[];
+                                const float* __restrict__ s, float inv_sqrt_n, int dbl) {
+    extern __shared__ __align__(16) float smem_rows[];
     const int P = 1 << lgP;
-    for (int64_t r = blockIdx.x; r < rows; r += gridDim.x) {
+    const bool async = (reinterpret_cast<uintptr_t>(M) & 15u) == 0 && (n & 3) == 0;
+    auto issue = [&](int64_t r, float* dst) {
+        const float* src = M + r * n;
+        for (int q = threadIdx.x; q < (n >> 2); q += blockDim.x) cp_async16(dst + 4 * q, src + 4 * q, 16);
+        cp_async_commit();
+    };
+    int it = 0;
+    if (async && dbl && blockIdx.x < rows) issue(blockIdx.x, smem_rows);
+    for (int64_t r = blockIdx.x; r < rows; r += gridDim.x, ++it) {
         float* row = M + r * n;
-        stage_row(v, row, n);
+        float* v = smem_rows + ((async && dbl) ? (it & 1) * n : 0);
+        if (async && dbl) {
+            const int64_t nxt = r + gridDim.x;
+            if (nxt < rows) {
+                issue(nxt, smem_rows + ((it + 1) & 1) * n);
+                cp_async_wait<1>();
+            } else {
+                cp_async_wait<0>();
+            }
+            __syncthreads();
+        } else {
+            stage_row(v, row, n);
+        }
         bool first = true;
         if (!HAS28 && lgP == 0) {   // n == 1
             for (int j = threadIdx.x; j < n; j += blockDim.x)
@@ -185,15 +218,15 @@ __global__ void __launch_bounds__(HAS28 ? 256 : 512, HAS28 ? 1 : 2) rht_rows_ker
         }
         if (HAS28) {   // H_28 (x) I_P, written straight to global memory
             for (int b = threadIdx.x; b < P; b += blockDim.x) {
-                float x[28], y[28];
+                float x[28];
 #pragma unroll
                 for (int a = 0; a < 28; ++a) {
                     x[a] = v[a * P + b];
                     if (first) x[a] *= factor(pre_mode, sign, s, a * P + b);
                 }
-                mix28(x, y);
-#pragma unroll
-                for (int a = 0; a < 28; ++a) row[a * P + b] = y[a] * (factor(post_mode, sign, s, a * P + b) * inv_sqrt_n);
+                mix28(x, [&](int a, float y) {
+                    row[a * P + b] = y * (factor(post_mode, sign, s, a * P + b) * inv_sqrt_n);
+                });
             }
             __syncthreads();
         }
@@ -206,7 +239,7 @@ __global__ void __launch_bounds__(HAS28 ? 256 : 512, HAS28 ? 1 : 2) rht_rows_ker
 // (R a power of two, as radix-8 passes) or H_28 (R == 28). Shared memory [R][CW], CW a
 // power of two, filled with cp.async; the last pass writes straight to global memory.
 template <bool IS28>
-__global__ void __launch_bounds__(256, IS28 ? 1 : 4) rht_cols_kernel(float* __restrict__ M, int n, int64_t ncols, int R, int S,
+__global__ void __launch_bounds__(256, IS28 ? 2 : 4) rht_cols_kernel(float* __restrict__ M, int n, int64_t ncols, int R, int S,
                                 int lgCW, int pre_mode, int post_mode, const int8_t* __restrict__ sign,
                                 const float* __restrict__ s, float post_scale) {
     extern __shared__ __align__(16) float v[];
@@ -239,17 +272,32 @@ __global__ void __launch_bounds__(256, IS28 ? 1 : 4) rht_cols_kernel(float* __re
         }
         __syncthreads();
         if (IS28) {
+            // the 28 rows' pre- and post-factors, once per work item
+            float* pf = v + 28 * CW;
+            if (threadIdx.x < 28) {
+                const int64_t r = base + static_cast<int64_t>(threadIdx.x) * S;
+                pf[threadIdx.x] = factor(pre_mode, sign, s, r);
+                pf[28 + threadIdx.x] = factor(post_mode, sign, s, r) * post_scale;
+            }
+            __syncthreads();
+            // mix in place (each thread owns its columns), then store the tile row by row
             for (int c = threadIdx.x; c < CW; c += blockDim.x) {
-                float x[28], y[28];
+                float x[28];
 #pragma unroll
-                for (int a = 0; a < 28; ++a) x[a] = v[a * CW + c] * factor(pre_mode, sign, s, base + static_cast<int64_t>(a) * S);
-                mix28(x, y);
-                if (c < cw) {
-#pragma unroll
-                    for (int a = 0; a < 28; ++a) {
-                        const int64_t r = base + static_cast<int64_t>(a) * S;
-                        M[r * ncols + c0 + c] = y[a] * (factor(post_mode, sign, s, r) * post_scale);
-                    }
+                for (int a = 0; a < 28; ++a) x[a] = v[a * CW + c] * pf[a];
+                mix28(x, [&](int a, float y) { v[a * CW + c] = y * pf[28 + a]; });
+            }
+            __syncthreads();
+            if (vec && cw == CW) {
+                for (int e = threadIdx.x; e < (28 * CW) >> 2; e += blockDim.x) {
+                    const int i = (4 * e) >> lgCW, c = (4 * e) & (CW - 1);
+                    *reinterpret_cast<float4*>(M + (base + static_cast<int64_t>(i) * S) * ncols + c0 + c) =
+                        *reinterpret_cast<const float4*>(v + 4 * e);
+                }
+            } else {
+                for (int e = threadIdx.x; e < 28 * CW; e += blockDim.x) {
+                    const int i = e >> lgCW, c = e & (CW - 1);
+                    if (c < cw) M[(base + static_cast<int64_t>(i) * S) * ncols + c0 + c] = v[e];
                 }
             }
         } else {
@@ -485,25 +533,30 @@ kq_status rows_transform(float* M, int64_t rows, int64_t n, int pre, int post, c
                          const float* s, cudaStream_t stream) {
     HadamardPlan p;
     if (!plan_of(n, &p)) return KQ_ERR_UNSUPPORTED;
-    const size_t smem = static_cast<size_t>(n) * sizeof(float);
+    constexpr size_t kMaxSmem = 227 * 1024;
+    const size_t row_bytes = static_cast<size_t>(n) * sizeof(float);
+    const int dbl = 2 * row_bytes <= kMaxSmem ? 1 : 0;
+    const size_t smem = (dbl ? 2 : 1) * row_bytes;
     static bool attr = false;
     if (!attr) {
         KQ_CUDA(cudaFuncSetAttribute(rht_rows_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     32768 * 4));
+                                     static_cast<int>(kMaxSmem)));
         KQ_CUDA(cudaFuncSetAttribute(rht_rows_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     32768 * 4));
+                                     static_cast<int>(kMaxSmem)));
         attr = true;
     }
-    const int threads = p.has28 ? 256 : (n >= 2048 ? 512 : (n >= 512 ? 256 : 128));
-    const int64_t grid = std::min<int64_t>(rows, static_cast<int64_t>(num_sms()) * 32);
+    const int threads = n >= 512 ? 256 : 128;
+    // as many CTAs as fit on an SM by shared memory (at most 8), each walking rows
+    const int64_t per_sm = std::max<int64_t>(1, std::min<int64_t>(8, static_cast<int64_t>(kMaxSmem / smem)));
+    const int64_t grid = std::min<int64_t>(rows, static_cast<int64_t>(num_sms()) * per_sm);
     if (grid > 0) {
         const float isn = static_cast<float>(1.0 / sqrt(static_cast<double>(n)));
         if (p.has28)
             rht_rows_kernel<true><<<static_cast<unsigned>(grid), threads, smem, stream>>>(
-                M, rows, static_cast<int>(n), log2i(p.P), pre, post, sign, s, isn);
+                M, rows, static_cast<int>(n), log2i(p.P), pre, post, sign, s, isn, dbl);
         else
             rht_rows_kernel<false><<<static_cast<unsigned>(grid), threads, smem, stream>>>(
-                M, rows, static_cast<int>(n), log2i(p.P), pre, post, sign, s, isn);
+                M, rows, static_cast<int>(n), log2i(p.P), pre, post, sign, s, isn, dbl);
         KQ_LAUNCH_CHECK("rht_rows_kernel");
     }
     return KQ_OK;
@@ -514,14 +567,18 @@ kq_status cols_transform(float* M, int64_t n, int64_t ncols, int pre, int post, 
     HadamardPlan p;
     if (!plan_of(n, &p)) return KQ_ERR_UNSUPPORTED;
     // Radix stages: (R, S) pairs applied in order; S = product of earlier radices.
-    int R[3], S[3], ns = 0;
+    // Radix at most 64 per stage: a [64 x 256] tile (64 KB) leaves room for three CTAs per
+    // SM, so one CTA's loads overlap another's butterflies (a single 512- or 1024-row stage,
+    // one CTA per SM, ran below 0.7 TB/s).
+    int R[4], S[4], ns = 0;
     const int kp = log2i(p.P);
-    if (kp <= 10) {
-        if (p.P > 1) { R[ns] = p.P; S[ns] = 1; ++ns; }
-    } else {
-        const int k1 = kp - kp / 2, k2 = kp / 2;
-        R[ns] = 1 << k1; S[ns] = 1; ++ns;
-        R[ns] = 1 << k2; S[ns] = 1 << k1; ++ns;
+    const int nst = (kp + 5) / 6;
+    for (int st = 0, done = 0; st < nst; ++st) {
+        const int kb = (kp - done) / (nst - st);   // as even as possible
+        R[ns] = 1 << kb;
+        S[ns] = 1 << done;
+        ++ns;
+        done += kb;
     }
     if (p.has28) { R[ns] = 28; S[ns] = p.P; ++ns; }
     static bool attr = false;
@@ -539,7 +596,7 @@ kq_status cols_transform(float* M, int64_t n, int64_t ncols, int pre, int post, 
     for (int st = 0; st < ns; ++st) {
         int CW = 32768 / R[st];
         CW = CW < 32 ? 32 : (CW > 256 ? 256 : CW);
-        const size_t smem = static_cast<size_t>(R[st]) * CW * sizeof(float);
+        const size_t smem = (static_cast<size_t>(R[st]) * CW + (R[st] == 28 ? 56 : 0)) * sizeof(float);
         const int64_t items = (n / R[st]) * cdiv(ncols, CW);
         const int64_t grid = std::min<int64_t>(items, static_cast<int64_t>(num_sms()) * 16);
         const int pm = st == 0 ? pre : F_NONE, qm = st == ns - 1 ? post : F_NONE;

@@ -40,36 +40,43 @@ int num_sms() {
 }
 
 SideStream* side_stream(cudaStream_t caller) {
-    static thread_local SideStream cache[64][8] = {};
+    // One side stream per (device, caller stream) and host thread, so calls on different
+    // caller streams (concurrent layers) fork to different side streams.
+    struct Entry {
+        int dev;
+        cudaStream_t caller;
+        SideStream side;
+    };
+    constexpr int kMax = 64;
+    static thread_local Entry table[kMax];
+    static thread_local int used = 0;
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    if (cudaGetDevice(&dev) != cudaSuccess) return nullptr;
+    for (int i = 0; i < used; ++i)
+        if (table[i].dev == dev && table[i].caller == caller) return table[i].side.s ? &table[i].side : nullptr;
+    if (used == kMax) return nullptr;   // beyond kMax caller streams: no fork, all work in order
     int prio = 0, least = 0, greatest = 0;
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
     if (cudaStreamGetPriority(caller, &prio) != cudaSuccess ||
-        cudaDeviceGetStreamPriorityRange(&least, &greatest) != cudaSuccess) {
+        cudaDeviceGetStreamPriorityRange(&least, &greatest) != cudaSuccess ||
+        cudaStreamIsCapturing(caller, &cap) != cudaSuccess) {
         cudaGetLastError();
         return nullptr;
     }
-    // Larger numbers are lower priorities.
+    if (cap != cudaStreamCaptureStatusNone) return nullptr;   // made only outside a capture
+    // Larger numbers are lower priorities: one level below the caller's.
     const int side_prio = prio < least ? prio + 1 : least;
-    const int idx = side_prio - greatest;
-    if (idx < 0 || idx >= 8) return nullptr;
-    SideStream& c = cache[dev][idx];
-    if (!c.tried) {
-        cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
-        if (cudaStreamIsCapturing(caller, &cap) != cudaSuccess) {
-            cudaGetLastError();
-            return nullptr;
-        }
-        if (cap != cudaStreamCaptureStatusNone) return nullptr;
-        c.tried = true;
-        if (cudaStreamCreateWithPriority(&c.s, cudaStreamNonBlocking, side_prio) != cudaSuccess ||
-            cudaEventCreateWithFlags(&c.ev[0], cudaEventDisableTiming) != cudaSuccess ||
-            cudaEventCreateWithFlags(&c.ev[1], cudaEventDisableTiming) != cudaSuccess) {
-            cudaGetLastError();
-            c.s = nullptr;
-        }
+    Entry& e = table[used++];
+    e.dev = dev;
+    e.caller = caller;
+    e.side.tried = true;
+    if (cudaStreamCreateWithPriority(&e.side.s, cudaStreamNonBlocking, side_prio) != cudaSuccess ||
+        cudaEventCreateWithFlags(&e.side.ev[0], cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&e.side.ev[1], cudaEventDisableTiming) != cudaSuccess) {
+        cudaGetLastError();
+        e.side.s = nullptr;
     }
-    return c.s ? &c : nullptr;
+    return e.side.s ? &e.side : nullptr;
 }
 
 // Waits on an mbarrier that nothing ever arrives on, with the bounded wait every pipeline

@@ -38,10 +38,11 @@ int num_sms();
 // forks to it with an event recorded on the caller's stream and joins back (the caller's
 // stream waits on an event recorded on it) before returning, so the caller sees one
 // ordered stream, and a CUDA graph captured from the caller's stream records both
-// branches. One per host thread, device and priority; its priority is one level below the
-// caller's stream. side_stream returns nullptr (the caller then runs everything on its own
-// stream) when the stream cannot be made, or when the caller's stream is being captured
-// and the side stream does not exist yet.
+// branches. One per host thread, device and caller stream (so concurrent calls on
+// different caller streams fork to different side streams); its priority is one level below
+// the caller's stream. side_stream returns nullptr (the caller then runs everything on its
+// own stream) when the stream cannot be made, or when the caller's stream is being captured
+// and its side stream does not exist yet.
 struct SideStream {
     cudaStream_t s;
     cudaEvent_t ev[2];

@@ -214,6 +214,50 @@ class LayerPipeline:
         caller.wait_event(e_out)
         caller.wait_event(e_hg)
 
+    def run_from_factors(self, HX_raw, HG_raw, W, sign_u, sign_v, stream=None, scales_ready: bool = False) -> None:
+        """Stages 2-4 from factors accumulated elsewhere (a factor shared by several
+        sublayers, Sec. 3.3: q, k and v read the same input). HX_raw / HG_raw are copied
+        into this pipeline's buffers (the rotations work in place). scales_ready: s_x, s_g
+        and the traces are already in this pipeline's buffers (computed from the same raw
+        factors). The Cholesky runs on this pipeline's high-priority stream with the H_G
+        side beside it, as in run()."""
+        s = torch.cuda.current_stream() if stream is None else stream
+        main = self.main if self.overlap else s
+        side = self.side if self.overlap else s
+        e_in, e_fx, e_tx, e_rin, e_side, e_out, e_hg, _ = self._ev
+        e_in.record(s)
+        main.wait_event(e_in)
+        side.wait_event(e_in)
+        with torch.cuda.stream(main):
+            self.HX.copy_(HX_raw)
+        if not scales_ready:
+            kq.kq_compute_scales(W, self.HX, None, self.s_x, None, stream=main)
+            kq.kq_traces(self.HX, self.s_x, None, None, self.traces, stream=main)
+        e_tx.record(main)
+        with torch.cuda.stream(main):
+            self.Wp.copy_(W)
+        kq.kq_rotate_in(self.Wp, self.HX, self.s_x, sign_v, kq.KQ_FWD, stream=main)
+        e_rin.record(main)
+        kq.kq_chol_inv(self.HX, self.damp, self.Lt, self.info[1:2], self.ws_chol, stream=main)
+        with torch.cuda.stream(side):
+            self.HG.copy_(HG_raw)
+        side.wait_event(e_tx)
+        if not scales_ready:
+            kq.kq_compute_scales(W, None, self.HG, None, self.s_g, stream=side)
+            kq.kq_traces(None, None, self.HG, self.s_g, self.traces, stream=side)
+        side.wait_event(e_rin)
+        kq.kq_rotate_out(self.Wp, None, self.s_g, sign_u, kq.KQ_FWD, stream=side)
+        e_side.record(side)
+        kq.kq_rotate_out(None, self.HG, self.s_g, sign_u, kq.KQ_FWD, stream=side)
+        e_hg.record(side)
+        main.wait_event(e_side)
+        kq.kq_obs_quantize(self.Wp, self.Lt, self.bits, self.group, self.block, self.codes, self.scale,
+                           self.zero, self.col_loss, None, self.ws_obs, stream=main, mode=self.trail_mode,
+                           info=self.info[3:4])
+        e_out.record(main)
+        s.wait_event(e_out)
+        s.wait_event(e_hg)
+
     def capture(self, X, G, W, sign_u, sign_v, Xt=None) -> tuple:
         """Record one layer (both streams) as a CUDA graph on these fixed buffers. Returns
         (graph, kernels per replay). Run run() once first so one-time set-up is done."""

@@ -532,3 +532,51 @@ def test_fp32_sweep_with_p_matches_fp64_off_ties(group):
     # P really changes the result
     s0 = obs_sweep_fp32(W32, R32.T, 4, group, 32)
     assert not np.array_equal(s0["codes"], s32["codes"])
+
+
+# ------------------------------------------------------- mixed-precision allocation
+def test_allocation_worked_examples_golden():
+    """Hand-worked W2 -> W3 allocations (tests/golden/mp_allocation_worked.json)."""
+    g = json.load(open(os.path.join(GOLDEN, "mp_allocation_worked.json")))
+    for c in g["cases"]:
+        assert ref.allocate_bits(c["scores"], c["params"], g["low"], g["high"], c["budget"]) == c["bits"], c["work"]
+
+
+def test_allocation_limits_and_monotone_budget():
+    rng = _rng(12)
+    names = [f"s{i}" for i in range(7)]
+    scores = dict(zip(names, rng.random(7)))
+    params = dict(zip(names, rng.integers(1, 20, 7).tolist()))
+    assert set(ref.allocate_bits(scores, params, 2, 3, 2.0).values()) == {2}
+    assert set(ref.allocate_bits(scores, params, 2, 3, 3.0).values()) == {3}
+    prev = set()
+    for budget in np.linspace(2.0, 3.0, 41):
+        b = ref.allocate_bits(scores, params, 2, 3, budget)
+        up = {n for n in names if b[n] == 3}
+        assert prev <= up                           # a larger budget never downgrades
+        mean = sum(b[n] * params[n] for n in names) / sum(params.values())
+        assert mean <= budget + 1e-12
+        # the upgraded set is a prefix of the descending-score order
+        order = sorted(names, key=lambda n: -scores[n])
+        assert up == set(order[:len(up)])
+        prev = up
+
+
+def test_block_scores_shared_input_degeneracy():
+    """Sec. 3.3: q, k, v read the same input, so every activation-only score (raw tr(H_X))
+    is identical for them; the joint score differs through tr(H_G)."""
+    cfg = kqsynth.BLOCKS["tiny_block"].replace(T=256)
+    b = kqsynth.block_inputs(cfg)
+    sc = ref.block_scores(b["X"], b["G"], b["W"], kqsynth.block_spec(cfg))
+    assert sc["q"]["trHX"] == sc["k"]["trHX"] == sc["v"]["trHX"]
+    assert sc["gate"]["trHX"] == sc["up"]["trHX"]
+    assert len({sc[n]["trHG"] for n in ("q", "k", "v")}) == 3
+    for n, v in sc.items():
+        assert np.isclose(v["s"], v["trHX"] * v["trHG"], rtol=1e-12)
+        # post-BiIP traces follow the rescale identity sum_j h_j / s_j^2 (checked against
+        # the dense rotated factor of that sublayer)
+    name, grp, _, _ = kqsynth.block_spec(cfg)[1]
+    su, sv = b["sign_u"][name], b["sign_v"][name]
+    r = ref.biip(b["W"][name], ref.accum_factor(b["X"][grp]), ref.accum_factor(b["G"][name]), su, sv)
+    assert np.isclose(np.trace(r["HX"]), sc[name]["trHX_post"], rtol=1e-10)
+    assert np.isclose(np.trace(r["HG"]), sc[name]["trHG_post"], rtol=1e-10)
