@@ -52,6 +52,11 @@ def parse():
                     help="a whole transformer block (seven sublayers, shared H_X, W2/W3 allocation) "
                          "instead of one layer")
     ap.add_argument("--lanes", type=int, default=2, help="sublayers quantized concurrently in --block mode")
+    ap.add_argument("--infer", type=int, default=None, metavar="BITS",
+                    help="decode with quantized layers instead: one token through every linear sublayer of "
+                         "--infer-blocks Llama-3-8B blocks (kq_infer, online BiIP revert)")
+    ap.add_argument("--infer-blocks", type=int, default=32)
+    ap.add_argument("--infer-tokens", type=int, default=1)
     ap.add_argument("--drift-chunk-tokens", type=int, default=0,
                     help="token chunk of the drift statistic's launches (0: one launch)")
     ap.add_argument("--tokens", type=int, default=0,
@@ -584,8 +589,120 @@ def run_block(args):
         torch.distributed.destroy_process_group()
 
 
+# ------------------------------------------------------------------ decode (inference)
+INFER_METRIC = "ms per decode step (B tokens through every linear sublayer, online BiIP revert)"
+
+
+def run_infer(args):
+    import torch
+
+    from paper_2607_07964_gb300 import build as kbuild
+    ws, rank, local = dist_setup("nccl")
+    kbuild.build()
+    from paper_2607_07964_gb300 import kronq as kq
+
+    torch.cuda.set_device(local)
+    dev = f"cuda:{local}"
+    bc = kqsynth.BLOCKS["llama3_8b_block"]
+    spec = kqsynth.block_spec(bc)
+    bits, B, nb = args.infer, args.infer_tokens, args.infer_blocks
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(1234 + rank)
+    layers = []
+    wbytes = 0
+    for blk in range(nb):
+        for name, _, d_out, d_in in spec:
+            ng = d_in // 128
+            codes = torch.randint(0, 2 ** bits, (d_out, d_in), generator=gen, device=dev, dtype=torch.int32).to(torch.uint8)
+            packed = torch.empty(kq.kq_packed_codes_bytes(d_out, d_in, bits) // 4, dtype=torch.int32, device=dev)
+            kq.kq_pack_codes(codes, bits, packed)
+            del codes
+            L = {"packed": packed, "d_out": d_out, "d_in": d_in,
+                 "scale": torch.rand((d_out, ng), generator=gen, device=dev) * 0.01 + 1e-3,
+                 "zero": torch.randint(0, 2 ** bits, (d_out, ng), generator=gen, device=dev, dtype=torch.int32),
+                 "s_x": torch.rand(d_in, generator=gen, device=dev) + 0.5, "s_g": torch.rand(d_out, generator=gen, device=dev) + 0.5,
+                 "su": (torch.randint(0, 2, (d_out,), generator=gen, device=dev) * 2 - 1).to(torch.int8),
+                 "sv": (torch.randint(0, 2, (d_in,), generator=gen, device=dev) * 2 - 1).to(torch.int8)}
+            L["x"] = torch.randn((B, d_in), generator=gen, device=dev)
+            L["y"] = torch.empty((B, d_out), device=dev)
+            L["ws"] = torch.empty(kq.kq_infer_workspace(B, d_in, d_out), dtype=torch.uint8, device=dev)
+            wbytes += packed.numel() * 4 + L["scale"].numel() * 4 + L["zero"].numel() * 4
+            layers.append(L)
+    stream = torch.cuda.current_stream()
+    # A block's decode step in dependency order: q, k, v read the same input (concurrent), then
+    # o, then gate and up (concurrent), then down.
+    phases = [["q", "k", "v"], ["o"], ["gate", "up"], ["down"]]
+    names = [name for name, _, _, _ in spec]
+    lanes = [torch.cuda.Stream(device=dev) for _ in range(3)]
+
+    def call(L, s):
+        kq.kq_infer(L["packed"], L["scale"], L["zero"], L["d_out"], L["d_in"], bits, 128, L["s_x"], L["s_g"],
+                    L["su"], L["sv"], L["x"], L["y"], L["ws"], stream=s)
+
+    def step(s):
+        for blk in range(nb):
+            for ph in phases:
+                if len(ph) == 1:
+                    call(layers[blk * len(names) + names.index(ph[0])], s)
+                    continue
+                ev = torch.cuda.Event()
+                ev.record(s)
+                for i, name in enumerate(ph):
+                    lanes[i].wait_event(ev)
+                    call(layers[blk * len(names) + names.index(name)], lanes[i])
+                for i in range(len(ph)):
+                    s.wait_stream(lanes[i])
+
+    for _ in range(args.warmup):
+        step(stream)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    cap = torch.cuda.Stream(device=dev)
+    n0 = kq.launch_count()
+    with torch.cuda.graph(g, stream=cap):
+        step(cap)
+    per_step = kq.launch_count() - n0
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(None)
+    sampler.start()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(args.steps):
+        g.replay()
+    t1.record(stream)
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    ms = max_over_ranks(t0.elapsed_time(t1), ws, dev) / args.steps
+    peaks, peak_src = measured_peaks()
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+    ach = wbytes / ms / 1e6
+    if rank == 0:
+        out = {"metric": INFER_METRIC, "value": ms / ws, "unit": "ms", "n_gpus": ws, "steps": args.steps,
+               "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": False, "scaling": "weak",
+               "vs_baseline": None, "dtype": "f32 arithmetic on packed integer codes", "data": "synthetic",
+               "config": {"workload": f"Llama-3-8B linear sublayers x {nb} blocks, {bits}-bit codes "
+                                      f"({'4-bit lanes' if bits == 3 else 'packed'}), group 128, B = {B}; per block "
+                                      f"q|k|v concurrent, o, gate|up concurrent, down",
+                          "blocks": nb, "bits": bits, "tokens": B,
+                          "l2": f"{wbytes / 1e9:.2f} GB of packed weights per step, larger than L2; no flush"},
+               "roofline": {"kernel": "kq_infer (Hadamard in, dequant_gemv_kernel, Hadamard out) over all sublayers",
+                            "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm,
+                            "traffic": None, "peak_source": f"{peak_src} HBM copy",
+                            "bytes_per_step": wbytes},
+               "cpu_baseline": None, "e2e": None, "gpu_launches": per_step,
+               "launch_mode": "cuda graph replay", "clocks": clocks}
+        print(json.dumps(out), flush=True)
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+
+
 def main():
     args = parse()
+    if args.infer is not None:
+        run_infer(args)
+        return
     if args.block is not None:
         if args.impl == "reference":
             ws, rank, _ = dist_setup("gloo")

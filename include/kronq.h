@@ -9,8 +9,8 @@
  *   3. damped inverse Cholesky                                (kq_chol_inv)
  *   4. column-wise OBS sweep with b-bit asymmetric grids      (kq_obs_quantize)
  * with the GPTAQ drift correction as an option (kq_accum_drift, kq_gptaq_p, and the Pt
- * argument of kq_obs_quantize), plus two check-only calls (kq_dequant_revert,
- * kq_proxy_loss).
+ * argument of kq_obs_quantize), inference with the quantized layer (kq_pack_codes,
+ * kq_infer), plus two check-only calls (kq_dequant_revert, kq_proxy_loss).
  *
  * Conventions shared by every call
  *   - Tokens are rows: X is [T x d_in], G is [T x d_out]; the paper stacks tokens as
@@ -296,6 +296,35 @@ KQ_API kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, const fl
                                  int bits, int group, int block, int mode, uint8_t* codes, float* scale,
                                  int32_t* zero, float* col_loss, float* pre_q, int* info, void* ws,
                                  size_t ws_bytes, kq_stream_t stream);
+
+/* ------------------------------------------------------------------------------------
+ * Inference with a quantized layer.
+ * Paper: Algorithm 2's revert W^ = S_G^-1 U^T Q' V S_X^-1 (Q' the dequantized codes) and
+ * Sec. 3.2 (at inference the diagonal scales are reverted elementwise and U, V cost
+ * O(d log d) per layer). y = W^ x is computed without forming W^:
+ *   x' = V S_X^-1 x (fast Hadamard transform), y' = Q' x' (dequantizing product over the
+ *   packed codes), y = S_G^-1 U^T y' (fast Hadamard transform).
+ *
+ * kq_pack_codes: codes [d_out x d_in] uint8 (from kq_obs_quantize) -> packed, 32-bit words
+ *   along each row: word w of a row holds codes w * (32 / pb) .. + 32 / pb - 1, code t of the
+ *   word in bits [t pb, t pb + pb), pb = bits for 2-, 4- and 8-bit codes and 4 for 3-bit
+ *   codes. kq_packed_codes_bytes(d_out, d_in, bits) bytes (0 for unsupported bits).
+ *   Requirements: bits in {2, 3, 4, 8}, d_in % 128 == 0, packed 16-byte aligned.
+ * kq_infer: y [B x d_out] fp32 = W^ x for B tokens x [B x d_in] fp32 (1 <= B <= 8), from
+ *   the packed codes, scale fp32 and zero int32 ([d_out] for group 0, [d_out x d_in / 128]
+ *   for group 128), s_x [d_in], s_g [d_out] and the RHT signs of the quantization.
+ *   All arithmetic fp32 (codes are exact as floats; per group scale (sum q x' - zero sum x')).
+ *   ws: kq_infer_workspace(B, d_in, d_out) bytes, 256-byte aligned. packed, x, y, s_x, s_g
+ *   16-byte aligned, the signs 4-byte aligned, d_out % 4 == 0; s_x, s_g required (not NULL). d_in and d_out need Hadamard constructions (2^k or 28 * 2^k).
+ * ---------------------------------------------------------------------------------- */
+KQ_API size_t kq_packed_codes_bytes(int64_t d_out, int64_t d_in, int bits);
+KQ_API kq_status kq_pack_codes(const uint8_t* codes, int64_t d_out, int64_t d_in, int bits, uint32_t* packed,
+                               kq_stream_t stream);
+KQ_API size_t kq_infer_workspace(int64_t B, int64_t d_in, int64_t d_out);
+KQ_API kq_status kq_infer(const uint32_t* packed, const float* scale, const int32_t* zero, int64_t d_out,
+                          int64_t d_in, int bits, int group, const float* s_x, const float* s_g,
+                          const int8_t* sign_u, const int8_t* sign_v, const float* x, int64_t B, float* y,
+                          void* ws, size_t ws_bytes, kq_stream_t stream);
 
 /* ------------------------------------------------------------------------------------
  * Check-only calls (not part of the timed path).

@@ -15,6 +15,7 @@ It follows "KronQ: LLM Quantization via Kronecker-Factored Hessian":
   * revert and proxy loss      Algorithm 2, Sec. 3.1 Eq. (kron_obj), Theorem 1
   * sensitivity traces         Sec. 3.3 Eq. (sensitivity)
   * mixed-precision allocation Sec. 3.3, Sec. 5 "Results on Mixed-precision" (W2 -> W3)
+  * inference y = W^ x         Algorithm 2's revert applied to tokens (Sec. 3.2)
 Tokens are stored as rows here (X is T x d_in), so the paper's X X^T is X^T X.
 
 Readings of points the paper leaves open (all listed in the design notes):
@@ -43,7 +44,7 @@ __all__ = [
     "biip_scales", "biip", "damp", "inverse_cholesky_upper", "lower_factor",
     "quant_params", "quantize", "obs_sweep", "dequant", "revert", "proxy_loss",
     "traces", "pipeline", "drift_factor", "gptaq_p", "objective", "allocate_bits", "block_scores",
-    "block_pipeline",
+    "block_pipeline", "infer",
 ]
 
 
@@ -452,3 +453,18 @@ def block_pipeline(X: dict, G: dict, W: dict, sign_u: dict, sign_v: dict, spec, 
     for name, grp, _, _ in spec:
         res[name] = pipeline(X[grp], G[name], W[name], sign_u[name], sign_v[name], bits[name], group, block, lam)
     return {"scores": sc, "bits": bits, "layers": res}
+
+
+# ----------------------------------------------------------------------------------
+# Inference with the quantized layer (Algorithm 2's revert; Sec. 3.2: the scales are
+# reverted elementwise and U, V applied to activations at inference).
+# ----------------------------------------------------------------------------------
+def infer(codes, scale, zero, group: int, s_x, s_g, sign_u, sign_v, x) -> np.ndarray:
+    """y = W^ x^T for tokens x [B, d_in] (returned [B, d_out]), W^ the dense reverted
+    weight S_G^-1 U^T Q' V S_X^-1 in float64."""
+    d_out, d_in = np.asarray(codes).shape
+    U = rht_matrix(d_out, sign_u)
+    V = rht_matrix(d_in, sign_v)
+    What = revert(dequant(codes, np.asarray(scale, np.float64), np.asarray(zero, np.float64), group),
+                  np.asarray(s_x, np.float64), np.asarray(s_g, np.float64), U, V)
+    return np.asarray(x, np.float64) @ What.T

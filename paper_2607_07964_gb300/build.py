@@ -16,7 +16,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libkronq.so")
-SOURCES = ["kq_api.cu", "syrk.cu", "biip.cu", "chol.cu", "obs.cu", "trail_tc.cu", "gptaq.cu", "check.cu"]
+SOURCES = ["kq_api.cu", "syrk.cu", "biip.cu", "chol.cu", "obs.cu", "trail_tc.cu", "gptaq.cu", "infer.cu", "check.cu"]
 HEADERS = sorted(os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith(".cuh")) + [
     os.path.join(ROOT, "include", "kronq.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

@@ -14,155 +14,13 @@
 #include <math.h>
 
 #include <algorithm>
-#include <utility>
 
 #include "kq_common.cuh"
+#include "rht.cuh"
 #include "sumsq.cuh"
 
 namespace kq {
 namespace {
-
-// ---------------------------------------------------------------------------------------
-// H_28 by Paley's second construction over GF(13): the symmetric conference matrix
-// C = [[0, 1^T], [1, Q]], Q[i][j] = chi(j - i) (chi = quadratic character mod 13), with
-// every entry replaced by a 2 x 2 block: 0 -> [[1,-1],[-1,-1]], c = +-1 -> c [[1,1],[1,-1]].
-// Stored as 28 row masks; bit a of row r is set when H_28[r][a] = -1.
-constexpr int chi13(int a) {
-    a %= 13;
-    if (a < 0) a += 13;
-    if (a == 0) return 0;
-    for (int x = 1; x < 13; ++x)
-        if ((x * x) % 13 == a) return 1;
-    return -1;
-}
-constexpr int conf14(int i, int j) {
-    if (i == 0 && j == 0) return 0;
-    if (i == 0 || j == 0) return 1;
-    return chi13((j - 1) - (i - 1));
-}
-constexpr int h28_entry(int r, int a) {
-    const int c = conf14(r / 2, a / 2);
-    const int u = r % 2, v = a % 2;
-    if (c == 0) return (u == 0 && v == 0) ? 1 : -1;   // [[1,-1],[-1,-1]]
-    const int blk = (u == 1 && v == 1) ? -1 : 1;     // [[1,1],[1,-1]]
-    return c * blk;
-}
-struct H28Masks {
-    uint32_t m[28];
-};
-constexpr H28Masks make_h28() {
-    H28Masks t{};
-    for (int r = 0; r < 28; ++r) {
-        uint32_t m = 0;
-        for (int a = 0; a < 28; ++a)
-            if (h28_entry(r, a) < 0) m |= 1u << a;
-        t.m[r] = m;
-    }
-    return t;
-}
-constexpr bool h28_is_hadamard() {
-    for (int r = 0; r < 28; ++r)
-        for (int q = 0; q < 28; ++q) {
-            int dot = 0;
-            for (int a = 0; a < 28; ++a) dot += h28_entry(r, a) * h28_entry(q, a);
-            if (dot != (r == q ? 28 : 0)) return false;
-            if (h28_entry(r, q) != h28_entry(q, r)) return false;
-        }
-    return true;
-}
-static_assert(h28_is_hadamard(), "H_28 must satisfy H H^T = 28 I and be symmetric");
-
-// Factor applied to element index j before (pre) or after (post) a transform.
-enum FactorMode { F_NONE = 0, F_SMUL = 1, F_SDIV = 2, F_SIGN = 3 };
-
-__device__ __forceinline__ float factor(int mode, const int8_t* sign, const float* s, int64_t j) {
-    if (mode == F_NONE) return 1.0f;
-    const float sg = static_cast<float>(sign[j]);
-    if (mode == F_SIGN || s == nullptr) return sg;
-    return mode == F_SMUL ? sg * s[j] : sg / s[j];
-}
-
-// y = H_28 x for 28 values in registers, each output handed to out(r, y_r) as soon as it is
-// formed (only x stays live). Each row's sign mask is a template argument taken from the
-// compile-time table kH28, so every term is a plain add or subtract.
-constexpr H28Masks kH28 = make_h28();
-
-template <uint32_t M>
-__device__ __forceinline__ float pm_sum28(const float (&x)[28]) {
-    float acc = 0.0f;
-#pragma unroll
-    for (int a = 0; a < 28; ++a) acc = ((M >> a) & 1u) ? acc - x[a] : acc + x[a];
-    return acc;
-}
-
-template <typename Out, int... R>
-__device__ __forceinline__ void mix28_rows(const float (&x)[28], Out& out, std::integer_sequence<int, R...>) {
-    (out(R, pm_sum28<kH28.m[R]>(x)), ...);
-}
-
-template <typename Out>
-__device__ __forceinline__ void mix28(const float (&x)[28], Out out) {
-    mix28_rows(x, out, std::make_integer_sequence<int, 28>{});
-}
-
-// In-register Walsh-Hadamard transform of R = 2, 4 or 8 values (natural order).
-template <int R>
-__device__ __forceinline__ void fwht_reg(float (&x)[8]) {
-#pragma unroll
-    for (int h = 1; h < R; h <<= 1)
-#pragma unroll
-        for (int i = 0; i < R; ++i)
-            if ((i & h) == 0) {
-                const float a = x[i], b = x[i + h];
-                x[i] = a + b;
-                x[i + h] = a - b;
-            }
-}
-__device__ __forceinline__ void fwht_reg_r(float (&x)[8], int r) {
-    if (r == 8) fwht_reg<8>(x);
-    else if (r == 4) fwht_reg<4>(x);
-    else if (r == 2) fwht_reg<2>(x);
-}
-
-// One radix-r pass (span h = 2^lgh) of the Walsh-Hadamard transform over a shared vector
-// of n elements (every h*r-aligned block independently). Index math is shifts and masks.
-// FIRST: multiply each element by its pre-factor while reading. LAST: instead of writing
-// back, store (value * post-factor * scale) to dst (global).
-template <bool FIRST, bool LAST>
-__device__ __forceinline__ void fwht_pass(float* v, int n, int lgh, int lgr, int pre_mode, int post_mode,
-                                          const int8_t* sign, const float* s, float scale, float* dst) {
-    const int h = 1 << lgh, r = 1 << lgr;
-    for (int g = threadIdx.x; g < (n >> lgr); g += blockDim.x) {
-        const int base = ((g >> lgh) << (lgh + lgr)) | (g & (h - 1));
-        float x[8];
-#pragma unroll
-        for (int q = 0; q < 8; ++q)
-            if (q < r) {
-                x[q] = v[base + q * h];
-                if (FIRST) x[q] *= factor(pre_mode, sign, s, base + q * h);
-            }
-        fwht_reg_r(x, r);
-#pragma unroll
-        for (int q = 0; q < 8; ++q)
-            if (q < r) {
-                if (LAST) dst[base + q * h] = x[q] * (factor(post_mode, sign, s, base + q * h) * scale);
-                else v[base + q * h] = x[q];
-            }
-    }
-}
-
-// Stage n contiguous floats from global into shared memory with 16-byte cp.async copies
-// (scalar copies when the row is not 16-byte aligned).
-__device__ __forceinline__ void stage_row(float* v, const float* src, int n) {
-    if ((reinterpret_cast<uintptr_t>(src) & 15u) == 0 && (n & 3) == 0) {
-        for (int q = threadIdx.x; q < (n >> 2); q += blockDim.x) cp_async16(v + 4 * q, src + 4 * q, 16);
-        cp_async_commit();
-        cp_async_wait<0>();
-    } else {
-        for (int j = threadIdx.x; j < n; j += blockDim.x) v[j] = src[j];
-    }
-    __syncthreads();
-}
 
 // ------------------------------------------------------------------ row transform
 // For each row of M [rows x n]: v <- pre (.) v; v <- (H_28 (x) H_P) v (or H_P); row <-
@@ -742,6 +600,11 @@ extern "C" kq_status kq_rotate_out(float* W, int64_t d_out, int64_t d_in, float*
 
 // Used by the check-only revert (check.cu).
 namespace kq {
+// Used by the inference call (infer.cu): rows <- V S^-1 rows (pre-factor sigma / s).
+kq_status rotate_rows_pre_div(float* M, int64_t rows, int64_t n, const float* s, const int8_t* sign,
+                              cudaStream_t stream) {
+    return rows_transform(M, rows, n, s ? F_SDIV : F_SIGN, F_NONE, sign, s, stream);
+}
 kq_status rotate_rows_inv(float* M, int64_t rows, int64_t n, const float* s, const int8_t* sign,
                           cudaStream_t stream) {
     return rows_transform(M, rows, n, F_NONE, s ? F_SDIV : F_SIGN, sign, s, stream);

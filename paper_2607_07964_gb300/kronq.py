@@ -60,6 +60,10 @@ def lib() -> ctypes.CDLL:
             "kq_obs_quantize": ([P, I64, I64, P, P, I, I, I, I, P, P, P, P, P, P, P, SZ, P], I),
             "kq_accum_drift_workspace": ([I64, I64], SZ),
             "kq_accum_drift": ([P, P, I64, I64, I64, P, I, P, P, SZ, P], I),
+            "kq_packed_codes_bytes": ([I64, I64, I], SZ),
+            "kq_pack_codes": ([P, I64, I64, I, P, P], I),
+            "kq_infer_workspace": ([I64, I64, I64], SZ),
+            "kq_infer": ([P, P, P, I64, I64, I, I, P, P, P, P, P, I64, P, P, SZ, P], I),
             "kq_gptaq_p_workspace": ([I64], SZ),
             "kq_gptaq_p": ([P, P, I64, F, P, P, P, SZ, P], I),
             "kq_dequant_revert": ([P, P, P, I64, I64, I, P, P, P, P, P, P], I),
@@ -324,6 +328,42 @@ def kq_obs_quantize(W, Lt, bits: int, group: int, block: int, codes, scale, zero
     _ok(lib().kq_obs_quantize(_ptr(W), d_out, d_in, _ptr(Lt), _ptr(Pt), bits, group, block, mode, _ptr(codes),
                               _ptr(scale), _ptr(zero), _ptr(col_loss), _ptr(pre_q), _ptr(info), _ptr(ws),
                               0 if ws is None else ws.numel(), _stream(stream)), "kq_obs_quantize")
+
+
+def kq_packed_codes_bytes(d_out: int, d_in: int, bits: int) -> int:
+    return int(lib().kq_packed_codes_bytes(d_out, d_in, bits))
+
+
+def kq_pack_codes(codes, bits: int, packed, stream=None) -> None:
+    """codes [d_out, d_in] uint8 -> packed words (int32 tensor of kq_packed_codes_bytes / 4)."""
+    d_out, d_in = codes.shape
+    _need(codes, "codes", torch.uint8)
+    _need(packed, "packed", torch.int32, (kq_packed_codes_bytes(d_out, d_in, bits) // 4,))
+    _ok(lib().kq_pack_codes(_ptr(codes), d_out, d_in, bits, _ptr(packed), _stream(stream)), "kq_pack_codes")
+
+
+def kq_infer_workspace(B: int, d_in: int, d_out: int) -> int:
+    return int(lib().kq_infer_workspace(B, d_in, d_out))
+
+
+def kq_infer(packed, scale, zero, d_out: int, d_in: int, bits: int, group: int, s_x, s_g, sign_u, sign_v, x, y,
+             ws, stream=None) -> None:
+    """y [B, d_out] = W^ x for x [B, d_in]: the reverted quantized layer applied with online
+    Hadamard transforms (Algorithm 2's revert, Sec. 3.2)."""
+    B = x.shape[0]
+    _need(packed, "packed", torch.int32)
+    _need(scale, "scale", torch.float32)
+    _need(zero, "zero", torch.int32)
+    _need(s_x, "s_x", torch.float32, (d_in,))
+    _need(s_g, "s_g", torch.float32, (d_out,))
+    _need(sign_u, "sign_u", torch.int8, (d_out,))
+    _need(sign_v, "sign_v", torch.int8, (d_in,))
+    _need(x, "x", torch.float32, (B, d_in))
+    _need(y, "y", torch.float32, (B, d_out))
+    _need(ws, "ws", torch.uint8)
+    _ok(lib().kq_infer(_ptr(packed), _ptr(scale), _ptr(zero), d_out, d_in, bits, group, _ptr(s_x), _ptr(s_g),
+                       _ptr(sign_u), _ptr(sign_v), _ptr(x), B, _ptr(y), _ptr(ws), 0 if ws is None else ws.numel(),
+                       _stream(stream)), "kq_infer")
 
 
 def kq_dequant_revert(codes, scale, zero, group: int, s_x, s_g, sign_u, sign_v, W_hat, stream=None):

@@ -580,3 +580,25 @@ def test_block_scores_shared_input_degeneracy():
     r = ref.biip(b["W"][name], ref.accum_factor(b["X"][grp]), ref.accum_factor(b["G"][name]), su, sv)
     assert np.isclose(np.trace(r["HX"]), sc[name]["trHX_post"], rtol=1e-10)
     assert np.isclose(np.trace(r["HG"]), sc[name]["trHG_post"], rtol=1e-10)
+
+
+# ------------------------------------------------------------------------ inference
+def test_infer_reproduces_the_layer_within_the_grid_bound():
+    """8-bit per-row codes of W' = U S_G W S_X V^T reverted and applied to tokens give W x
+    up to the rounding of the grid: |W^ - W| is the reverted error of |Q' - W'| <= scale / 2
+    (rotations are orthogonal, so ||(W^ - W) x|| <= ||S_G^-1|| ||Q' - W'||_2 ||S_X^-1 x||)."""
+    cfg = kqsynth.CONFIGS["tiny256"].replace(d_out=64, d_in=128, T=512)
+    L = kqsynth.layer(cfg)
+    HX, HG = ref.accum_factor(L["X"]), ref.accum_factor(L["G"])
+    b = ref.biip(L["W"], HX, HG, L["sign_u"], L["sign_v"])
+    s, z = ref.quant_params(b["W"], 8)
+    codes = ref.quantize(b["W"], s[:, None], z[:, None], 8).astype(np.uint8)
+    x = _rng(4).standard_normal((3, 128))
+    y = ref.infer(codes, s[:, None], z[:, None], 0, b["s_x"], b["s_g"], L["sign_u"], L["sign_v"], x)
+    W = L["W"].astype(np.float64)
+    dWp = ref.dequant(codes, s[:, None], z[:, None], 0) - b["W"]
+    assert np.max(np.abs(dWp) / s[:, None]) <= 0.5 + 1e-9
+    bound = np.linalg.norm(dWp, 2) / np.min(b["s_g"]) * np.linalg.norm(x / b["s_x"][None, :], axis=1)
+    err = np.linalg.norm(y - x @ W.T, axis=1)
+    assert np.all(err <= bound * (1 + 1e-9))
+    assert np.all(err > 0)
