@@ -56,6 +56,9 @@ def parse():
                     help="decode with quantized layers instead: one token through every linear sublayer of "
                          "--infer-blocks Llama-3-8B blocks (kq_infer, online BiIP revert)")
     ap.add_argument("--infer-blocks", type=int, default=32)
+    ap.add_argument("--validate", action="store_true",
+                    help="Prop. 2 checks on the --config layer: output-side exponent sweep of the rescale, "
+                         "rho, CV of column/row norms (not a timing run)")
     ap.add_argument("--infer-tokens", type=int, default=1)
     ap.add_argument("--drift-chunk-tokens", type=int, default=0,
                     help="token chunk of the drift statistic's launches (0: one launch)")
@@ -698,8 +701,36 @@ def run_infer(args):
         torch.distributed.destroy_process_group()
 
 
+def run_validate(args):
+    import torch
+
+    from paper_2607_07964_gb300 import build as kbuild
+    kbuild.build()
+    from paper_2607_07964_gb300.validate import exponent_sweep
+
+    cfg = kqsynth.CONFIGS[args.config]
+    if args.tokens > 0:
+        cfg = cfg.replace(T=args.tokens)
+    inp = kqsynth.device_layer(cfg)
+    alphas = [0.0, 0.125, 0.25, 0.375, 0.5]
+    t0 = time.perf_counter()
+    res = exponent_sweep(inp["X"], inp["G"], inp["W"], inp["sign_u"], inp["sign_v"], cfg.bits, cfg.group, alphas,
+                         cfg.block, cfg.damp, args.trailing)
+    wall = time.perf_counter() - t0
+    base = res["loss"][alphas.index(0.25)]
+    out = {"metric": "Prop. 2 output-side exponent sweep: proxy loss relative to alpha = 1/4",
+           "config": config_dict(cfg, trailing=args.trailing), "data": "synthetic",
+           "alphas": alphas, "loss": res["loss"], "loss_rel": [v / base for v in res["loss"]],
+           "argmin_alpha": alphas[min(range(len(alphas)), key=lambda i: res["loss"][i])],
+           "stats": res["stats"], "wall_s": wall}
+    print(json.dumps(out), flush=True)
+
+
 def main():
     args = parse()
+    if args.validate:
+        run_validate(args)
+        return
     if args.infer is not None:
         run_infer(args)
         return

@@ -165,6 +165,24 @@ KQ_API kq_status kq_accum_drift(const uint16_t* Xt, const uint16_t* X, int64_t T
  *   direction W may be NULL to transform only the factor (H_X or H_G).
  *   Returns KQ_ERR_UNSUPPORTED if the length has no Hadamard construction.
  * ---------------------------------------------------------------------------------- */
+KQ_API kq_status kq_compute_scales_exp(const float* W, int64_t d_out, int64_t d_in, const float* H_X,
+                                       const float* H_G, float* s_x, float* s_g, float ex, float eg,
+                                       kq_stream_t stream);
+
+/* BiIP statistics (Prop. 2 and Sec. 3.2; no counterpart in the quantization path itself):
+ * kq_compute_scales_exp: the scales of kq_compute_scales with the exponent as a parameter,
+ *   s_x = (h_x / a)^ex, s_g = (h_g / r)^eg, ex, eg in [0, 1] (1/4 gives kq_compute_scales'
+ *   bits exactly; 0 gives no rescale). Prop. 2's exponent sweep varies eg.
+ * kq_biip_stats: out [4] (device double) = [CV_in, CV_out, rho_in, rho_out]: the coefficient
+ *   of variation (population standard deviation over mean) of the column norms and of the
+ *   row norms of W [d_out x d_in], and rho = (sum sqrt(h a))^2 / (sum h sum a) <= 1 (Prop. 2's
+ *   gain of the rescale over none) from the diagonal h of H_X (input side, a = squared
+ *   column norms) or H_G (output side, a = squared row norms); a NULL factor leaves its rho
+ *   entry untouched. fp64 sums. ws: kq_biip_stats_workspace(d_out, d_in) bytes. */
+KQ_API size_t kq_biip_stats_workspace(int64_t d_out, int64_t d_in);
+KQ_API kq_status kq_biip_stats(const float* W, int64_t d_out, int64_t d_in, const float* H_X, const float* H_G,
+                               double* out, void* ws, size_t ws_bytes, kq_stream_t stream);
+
 #define KQ_FWD 0
 #define KQ_INV 1
 KQ_API kq_status kq_compute_scales(const float* W, int64_t d_out, int64_t d_in, const float* H_X,

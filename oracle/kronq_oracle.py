@@ -16,6 +16,8 @@ It follows "KronQ: LLM Quantization via Kronecker-Factored Hessian":
   * sensitivity traces         Sec. 3.3 Eq. (sensitivity)
   * mixed-precision allocation Sec. 3.3, Sec. 5 "Results on Mixed-precision" (W2 -> W3)
   * inference y = W^ x         Algorithm 2's revert applied to tokens (Sec. 3.2)
+  * BiIP statistics            Prop. 2 (rho, the exponent of the rescale), Sec. 3.2 and
+                               the appendix on weight distributions (CV_in, CV_out)
 Tokens are stored as rows here (X is T x d_in), so the paper's X X^T is X^T X.
 
 Readings of points the paper leaves open (all listed in the design notes):
@@ -44,7 +46,7 @@ __all__ = [
     "biip_scales", "biip", "damp", "inverse_cholesky_upper", "lower_factor",
     "quant_params", "quantize", "obs_sweep", "dequant", "revert", "proxy_loss",
     "traces", "pipeline", "drift_factor", "gptaq_p", "objective", "allocate_bits", "block_scores",
-    "block_pipeline", "infer",
+    "block_pipeline", "infer", "biip_scales_exp", "norm_cv", "rho", "prop2_bound",
 ]
 
 
@@ -205,15 +207,19 @@ def biip_scales_from_diag(W: np.ndarray, hx: np.ndarray, hg: np.ndarray):
     return biip_scales(W, np.diag(np.asarray(hx, np.float64)), np.diag(np.asarray(hg, np.float64)))
 
 
-def biip(W, HX, HG, sign_u, sign_v, D=None):
+def biip(W, HX, HG, sign_u, sign_v, D=None, ex: float = 0.25, eg: float = 0.25):
     """Algorithm 1: W <- S_G W S_X; H_X <- S_X^-1 H_X S_X^-1; H_G <- S_G^-1 H_G S_G^-1;
     W <- U W V^T; H_X <- V H_X V^T; H_G <- U H_G U^T (dense products). With the drift
-    statistic D (Delta X X^T), also D <- V S_X^-1 D S_X^-1 V^T."""
+    statistic D (Delta X X^T), also D <- V S_X^-1 D S_X^-1 V^T. ex, eg: the rescale's
+    exponents (1/4 in Eq. rescale; Prop. 2's sweep varies them)."""
     W = np.asarray(W, dtype=np.float64)
     HX = np.asarray(HX, dtype=np.float64)
     HG = np.asarray(HG, dtype=np.float64)
     d_out, d_in = W.shape
-    sx, sg = biip_scales(W, HX, HG)
+    if ex == 0.25 and eg == 0.25:
+        sx, sg = biip_scales(W, HX, HG)
+    else:
+        sx, sg = biip_scales_exp(W, np.diag(HX), np.diag(HG), ex, eg)
     Ws = sg[:, None] * W * sx[None, :]
     HXs = HX / sx[:, None] / sx[None, :]
     HGs = HG / sg[:, None] / sg[None, :]
@@ -377,13 +383,13 @@ def traces(HX, HG, HXp, HGp) -> dict:
 
 
 def pipeline(X, G, W, sign_u, sign_v, bits: int, group: int, block: int = 128,
-             lam: float = 0.01, Xt=None, alpha: float = 0.25) -> dict:
+             lam: float = 0.01, Xt=None, alpha: float = 0.25, ex: float = 0.25, eg: float = 0.25) -> dict:
     """Algorithms 1 and 2 end to end, all in float64: GPTQ mode when Xt (X~) is None,
-    else with the GPTAQ drift correction P of scaling alpha."""
+    else with the GPTAQ drift correction P of scaling alpha; ex, eg the rescale exponents."""
     HX = accum_factor(X)
     HG = accum_factor(G)
     D = None if Xt is None else drift_factor(Xt, X)
-    b = biip(W, HX, HG, sign_u, sign_v, D)
+    b = biip(W, HX, HG, sign_u, sign_v, D, ex, eg)
     Hd = damp(b["HX"], lam)
     R = inverse_cholesky_upper(Hd)
     P = None if D is None else gptaq_p(b["D"], R.T, alpha)
@@ -468,3 +474,44 @@ def infer(codes, scale, zero, group: int, s_x, s_g, sign_u, sign_v, x) -> np.nda
     What = revert(dequant(codes, np.asarray(scale, np.float64), np.asarray(zero, np.float64), group),
                   np.asarray(s_x, np.float64), np.asarray(s_g, np.float64), U, V)
     return np.asarray(x, np.float64) @ What.T
+
+
+# ----------------------------------------------------------------------------------
+# BiIP statistics (Prop. 2; Sec. 3.2 "CV_in / CV_out"; the appendix on weight distributions).
+# ----------------------------------------------------------------------------------
+def biip_scales_exp(W, hx, hg, ex: float, eg: float):
+    """Eq. (rescale) with the exponent as a parameter: s_x = (h_x / a)^ex, s_g = (h_g / r)^eg
+    (ex = eg = 1/4 is the paper's; Prop. 2's sweep varies it). Dead channels get 1."""
+    W = np.asarray(W, dtype=np.float64)
+    a = np.sum(W * W, axis=0)
+    r = np.sum(W * W, axis=1)
+    hx = np.asarray(hx, np.float64)
+    hg = np.asarray(hg, np.float64)
+    with np.errstate(divide="ignore", invalid="ignore"):
+        sx = np.where((hx > 0) & (a > 0), (hx / a) ** ex, 1.0)
+        sg = np.where((hg > 0) & (r > 0), (hg / r) ** eg, 1.0)
+    return sx, sg
+
+
+def norm_cv(W) -> tuple:
+    """(CV_in, CV_out): coefficient of variation (population standard deviation over mean)
+    of the column norms ||W[:, j]|| and of the row norms ||W[i, :]||."""
+    W = np.asarray(W, dtype=np.float64)
+    c = np.sqrt(np.sum(W * W, axis=0))
+    r = np.sqrt(np.sum(W * W, axis=1))
+    return float(np.std(c) / np.mean(c)), float(np.std(r) / np.mean(r))
+
+
+def rho(h, a) -> float:
+    """Prop. 2's gain of the rescale over none: (sum sqrt(h a))^2 / (sum h sum a) <= 1."""
+    h = np.asarray(h, np.float64)
+    a = np.asarray(a, np.float64)
+    return float(np.sum(np.sqrt(h * a)) ** 2 / (np.sum(h) * np.sum(a)))
+
+
+def prop2_bound(h, a, s) -> float:
+    """The rescale-dependent factor of Prop. 2's expected loss: (sum h / s^2)(sum s^2 a)."""
+    h = np.asarray(h, np.float64)
+    a = np.asarray(a, np.float64)
+    s = np.asarray(s, np.float64)
+    return float(np.sum(h / s ** 2) * np.sum(s ** 2 * a))

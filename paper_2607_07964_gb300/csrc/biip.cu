@@ -205,21 +205,84 @@ __device__ __forceinline__ float quarter_root_ratio(float h, double a) {
     return static_cast<float>(sqrt(sqrt(static_cast<double>(h) / a)));
 }
 
-// a_j = ||W[:, j]||^2 and s_x[j] = (H_X[j][j] / a_j)^(1/4). Block (CS_X, CS_Y).
-__global__ void colscale_kernel(const float* __restrict__ W, int64_t d_out, int64_t d_in,
-                                const float* __restrict__ HX, int64_t hstride, float* __restrict__ s_x) {
-    const int64_t j = static_cast<int64_t>(blockIdx.x) * CS_X + threadIdx.x;
-    const double a = col_sumsq(W, d_out, d_in, j);
-    if (threadIdx.y == 0 && j < d_in) s_x[j] = quarter_root_ratio(HX[j * hstride], a);
+// (h / a)^e; e == 1/4 takes the same sqrt(sqrt()) as Eq. (rescale)'s scales.
+__device__ __forceinline__ float ratio_pow(float h, double a, float e) {
+    if (e == 0.25f) return quarter_root_ratio(h, a);
+    if (!(h > 0.0f) || !(a > 0.0)) return 1.0f;
+    return static_cast<float>(pow(static_cast<double>(h) / a, static_cast<double>(e)));
 }
 
-// r_i = ||W[i, :]||^2 and s_g[i] = (H_G[i][i] / r_i)^(1/4) (1 when H_G is NULL). Warp per row.
+// a_j = ||W[:, j]||^2 and s_x[j] = (H_X[j][j] / a_j)^e (e = 1/4: Eq. rescale). Block (CS_X, CS_Y).
+__global__ void colscale_kernel(const float* __restrict__ W, int64_t d_out, int64_t d_in,
+                                const float* __restrict__ HX, int64_t hstride, float* __restrict__ s_x, float e) {
+    const int64_t j = static_cast<int64_t>(blockIdx.x) * CS_X + threadIdx.x;
+    const double a = col_sumsq(W, d_out, d_in, j);
+    if (threadIdx.y == 0 && j < d_in) s_x[j] = ratio_pow(HX[j * hstride], a, e);
+}
+
+// r_i = ||W[i, :]||^2 and s_g[i] = (H_G[i][i] / r_i)^e (1 when H_G is NULL). Warp per row.
 __global__ void rowscale_kernel(const float* __restrict__ W, int64_t d_out, int64_t d_in,
-                                const float* __restrict__ HG, int64_t hstride, float* __restrict__ s_g) {
+                                const float* __restrict__ HG, int64_t hstride, float* __restrict__ s_g, float e) {
     const int64_t i = static_cast<int64_t>(blockIdx.x) * (blockDim.x / 32) + threadIdx.x / 32;
     if (i >= d_out) return;
     const double acc = row_sumsq(W + i * d_in, d_in);
-    if ((threadIdx.x & 31) == 0) s_g[i] = HG ? quarter_root_ratio(HG[i * hstride], acc) : 1.0f;
+    if ((threadIdx.x & 31) == 0) s_g[i] = HG ? ratio_pow(HG[i * hstride], acc, e) : 1.0f;
+}
+
+// Squared column norms (a) and squared row norms (r) of W in fp64, for the BiIP statistics.
+__global__ void colnorm2_kernel(const float* __restrict__ W, int64_t d_out, int64_t d_in, double* __restrict__ a) {
+    const int64_t j = static_cast<int64_t>(blockIdx.x) * CS_X + threadIdx.x;
+    const double v = col_sumsq(W, d_out, d_in, j);
+    if (threadIdx.y == 0 && j < d_in) a[j] = v;
+}
+__global__ void rownorm2_kernel(const float* __restrict__ W, int64_t d_out, int64_t d_in, double* __restrict__ r) {
+    const int64_t i = static_cast<int64_t>(blockIdx.x) * (blockDim.x / 32) + threadIdx.x / 32;
+    if (i >= d_out) return;
+    const double v = row_sumsq(W + i * d_in, d_in);
+    if ((threadIdx.x & 31) == 0) r[i] = v;
+}
+
+// out = [CV_in, CV_out, rho_in, rho_out]: coefficient of variation (population standard
+// deviation over mean) of the column and row norms sqrt(a), sqrt(r), and
+// rho = (sum sqrt(h a))^2 / (sum h sum a) with h the factor's diagonal (entries 2 and 3 are
+// left as they are when the factor is NULL). One CTA, fp64, fixed order.
+__global__ void biip_stats_kernel(const double* __restrict__ a, int64_t d_in, const double* __restrict__ r,
+                                  int64_t d_out, const float* __restrict__ HX, int64_t xs,
+                                  const float* __restrict__ HG, int64_t gs, double* __restrict__ out) {
+    __shared__ double part[6][32];
+    double v[6];
+    for (int side = 0; side < 2; ++side) {
+        const double* n2 = side == 0 ? a : r;
+        const int64_t n = side == 0 ? d_in : d_out;
+        const float* H = side == 0 ? HX : HG;
+        const int64_t hs = side == 0 ? xs : gs;
+        for (int k = 0; k < 6; ++k) v[k] = 0.0;
+        for (int64_t j = threadIdx.x; j < n; j += blockDim.x) {
+            const double nn = sqrt(n2[j]);
+            v[0] += nn;                       // sum of norms
+            v[1] += n2[j];                    // sum of squared norms
+            if (H) {
+                const double h = static_cast<double>(H[j * hs]);
+                v[2] += sqrt(h * n2[j]);
+                v[3] += h;
+            }
+        }
+        for (int k = 0; k < 4; ++k) {
+            for (int o = 16; o > 0; o >>= 1) v[k] += __shfl_xor_sync(0xffffffffu, v[k], o);
+            if ((threadIdx.x & 31) == 0) part[k][threadIdx.x >> 5] = v[k];
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            double t[4] = {0.0, 0.0, 0.0, 0.0};
+            for (int w = 0; w < static_cast<int>(blockDim.x / 32); ++w)
+                for (int k = 0; k < 4; ++k) t[k] += part[k][w];
+            const double mean = t[0] / static_cast<double>(n);
+            const double var = fmax(t[1] / static_cast<double>(n) - mean * mean, 0.0);
+            out[side] = sqrt(var) / mean;
+            if (H) out[2 + side] = t[2] * t[2] / (t[3] * t[1]);
+        }
+        __syncthreads();
+    }
 }
 
 // out = [tr H_X, tr H_G, product, tr H_X', tr H_G', product'] with tr H' = sum h_j / s_j^2.
@@ -477,17 +540,19 @@ using namespace kq;
 
 namespace {
 kq_status scales_impl(const float* W, int64_t d_out, int64_t d_in, const float* hx, int64_t xs, const float* hg,
-                      int64_t gs, float* s_x, float* s_g, cudaStream_t stream, const char* who) {
+                      int64_t gs, float* s_x, float* s_g, cudaStream_t stream, const char* who, float ex = 0.25f,
+                      float eg = 0.25f) {
     if (!W || d_out < 1 || d_in < 1 || (!s_x && !s_g) || (s_x && !hx)) {
         set_error("%s: invalid arguments", who);
         return KQ_ERR_INVALID_ARG;
     }
     if (s_x) {
-        colscale_kernel<<<static_cast<unsigned>(cdiv(d_in, CS_X)), dim3(CS_X, CS_Y), 0, stream>>>(W, d_out, d_in, hx, xs, s_x);
+        colscale_kernel<<<static_cast<unsigned>(cdiv(d_in, CS_X)), dim3(CS_X, CS_Y), 0, stream>>>(W, d_out, d_in, hx, xs, s_x,
+                                                                                               ex);
         KQ_LAUNCH_CHECK("colscale_kernel");
     }
     if (s_g) {
-        rowscale_kernel<<<static_cast<unsigned>(cdiv(d_out, 8)), 256, 0, stream>>>(W, d_out, d_in, hg, gs, s_g);
+        rowscale_kernel<<<static_cast<unsigned>(cdiv(d_out, 8)), 256, 0, stream>>>(W, d_out, d_in, hg, gs, s_g, eg);
         KQ_LAUNCH_CHECK("rowscale_kernel");
     }
     return KQ_OK;
@@ -515,6 +580,44 @@ extern "C" kq_status kq_compute_scales_diag(const float* W, int64_t d_out, int64
                                             const float* hg_diag, float* s_x, float* s_g, kq_stream_t stream_) {
     return scales_impl(W, d_out, d_in, hx_diag, 1, hg_diag, 1, s_x, s_g, reinterpret_cast<cudaStream_t>(stream_),
                        "kq_compute_scales_diag");
+}
+
+extern "C" kq_status kq_compute_scales_exp(const float* W, int64_t d_out, int64_t d_in, const float* H_X,
+                                           const float* H_G, float* s_x, float* s_g, float ex, float eg,
+                                           kq_stream_t stream_) {
+    if (!(ex >= 0.0f && ex <= 1.0f) || !(eg >= 0.0f && eg <= 1.0f)) {
+        set_error("kq_compute_scales_exp: exponents must lie in [0, 1]");
+        return KQ_ERR_INVALID_ARG;
+    }
+    return scales_impl(W, d_out, d_in, H_X, d_in + 1, H_G, d_out + 1, s_x, s_g, reinterpret_cast<cudaStream_t>(stream_),
+                       "kq_compute_scales_exp", ex, eg);
+}
+
+extern "C" size_t kq_biip_stats_workspace(int64_t d_out, int64_t d_in) {
+    if (d_out < 1 || d_in < 1) return 0;
+    return static_cast<size_t>(d_out + d_in) * sizeof(double) + 256;
+}
+
+extern "C" kq_status kq_biip_stats(const float* W, int64_t d_out, int64_t d_in, const float* H_X, const float* H_G,
+                                   double* out, void* ws, size_t ws_bytes, kq_stream_t stream_) {
+    cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+    if (!W || !out || d_out < 1 || d_in < 1) {
+        set_error("kq_biip_stats: invalid arguments");
+        return KQ_ERR_INVALID_ARG;
+    }
+    if (!ws || ws_bytes < kq_biip_stats_workspace(d_out, d_in) || (reinterpret_cast<uintptr_t>(ws) & 15u)) {
+        set_error("kq_biip_stats: workspace must be 16-byte aligned and hold %zu bytes", kq_biip_stats_workspace(d_out, d_in));
+        return KQ_ERR_WORKSPACE;
+    }
+    double* a = static_cast<double*>(ws);
+    double* r = a + d_in;
+    colnorm2_kernel<<<static_cast<unsigned>(cdiv(d_in, CS_X)), dim3(CS_X, CS_Y), 0, stream>>>(W, d_out, d_in, a);
+    KQ_LAUNCH_CHECK("colnorm2_kernel");
+    rownorm2_kernel<<<static_cast<unsigned>(cdiv(d_out, 8)), 256, 0, stream>>>(W, d_out, d_in, r);
+    KQ_LAUNCH_CHECK("rownorm2_kernel");
+    biip_stats_kernel<<<1, 1024, 0, stream>>>(a, d_in, r, d_out, H_X, d_in + 1, H_G, d_out + 1, out);
+    KQ_LAUNCH_CHECK("biip_stats_kernel");
+    return KQ_OK;
 }
 
 extern "C" kq_status kq_traces(const float* H_X, const float* s_x, int64_t d_in, const float* H_G,

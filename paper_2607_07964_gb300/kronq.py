@@ -47,6 +47,9 @@ def lib() -> ctypes.CDLL:
             "kq_accum_factor": ([P, I64, I64, I64, P, I, P, P, P], I),
             "kq_compute_scales": ([P, I64, I64, P, P, P, P, P], I),
             "kq_compute_scales_diag": ([P, I64, I64, P, P, P, P, P], I),
+            "kq_compute_scales_exp": ([P, I64, I64, P, P, P, P, F, F, P], I),
+            "kq_biip_stats_workspace": ([I64, I64], SZ),
+            "kq_biip_stats": ([P, I64, I64, P, P, P, P, SZ, P], I),
             "kq_traces_diag": ([P, P, I64, P, P, I64, P, P], I),
             "kq_factor_diag_workspace": ([I64, I64], SZ),
             "kq_factor_diag": ([P, I64, I64, I64, P, P, P, SZ, P], I),
@@ -193,6 +196,34 @@ def kq_compute_scales(W, H_X, H_G, s_x, s_g, stream=None) -> None:
     _need(s_g, "s_g", torch.float32, (d_out,))
     _ok(lib().kq_compute_scales(_ptr(W), d_out, d_in, _ptr(H_X), _ptr(H_G), _ptr(s_x), _ptr(s_g),
                                 _stream(stream)), "kq_compute_scales")
+
+
+def kq_compute_scales_exp(W, H_X, H_G, s_x, s_g, ex: float, eg: float, stream=None) -> None:
+    """Scales with the exponent as a parameter (1/4: kq_compute_scales)."""
+    d_out, d_in = W.shape
+    _need(W, "W", torch.float32)
+    _need(H_X, "H_X", torch.float32, (d_in, d_in))
+    _need(H_G, "H_G", torch.float32, (d_out, d_out))
+    _need(s_x, "s_x", torch.float32, (d_in,))
+    _need(s_g, "s_g", torch.float32, (d_out,))
+    _ok(lib().kq_compute_scales_exp(_ptr(W), d_out, d_in, _ptr(H_X), _ptr(H_G), _ptr(s_x), _ptr(s_g), float(ex),
+                                    float(eg), _stream(stream)), "kq_compute_scales_exp")
+
+
+def kq_biip_stats_workspace(d_out: int, d_in: int) -> int:
+    return int(lib().kq_biip_stats_workspace(d_out, d_in))
+
+
+def kq_biip_stats(W, H_X, H_G, out, ws, stream=None) -> None:
+    """out [4] float64 = [CV_in, CV_out, rho_in, rho_out] of W with the factors' diagonals."""
+    d_out, d_in = W.shape
+    _need(W, "W", torch.float32)
+    _need(H_X, "H_X", torch.float32, (d_in, d_in))
+    _need(H_G, "H_G", torch.float32, (d_out, d_out))
+    _need(out, "out", torch.float64, (4,))
+    _need(ws, "ws", torch.uint8)
+    _ok(lib().kq_biip_stats(_ptr(W), d_out, d_in, _ptr(H_X), _ptr(H_G), _ptr(out), _ptr(ws),
+                            0 if ws is None else ws.numel(), _stream(stream)), "kq_biip_stats")
 
 
 def kq_traces(H_X, s_x, H_G, s_g, out, stream=None) -> None:

@@ -602,3 +602,58 @@ def test_infer_reproduces_the_layer_within_the_grid_bound():
     err = np.linalg.norm(y - x @ W.T, axis=1)
     assert np.all(err <= bound * (1 + 1e-9))
     assert np.all(err > 0)
+
+
+# --------------------------------------------------------------- BiIP statistics (Prop. 2)
+def test_norm_cv_closed_forms():
+    """Columns with norms 1, 2, 3, 4 (and rows all equal): CV_in = std/mean of (1, 2, 3, 4)
+    = sqrt(1.25) / 2.5; CV_out = 0."""
+    W = np.zeros((4, 4))
+    for j, nrm in enumerate([1.0, 2.0, 3.0, 4.0]):
+        W[:, j] = nrm / 2.0             # each column: four entries of nrm / 2 -> norm nrm
+    W = W[:, [0, 1, 2, 3]]
+    cv_in, cv_out = ref.norm_cv(W)
+    assert np.isclose(cv_in, np.sqrt(1.25) / 2.5, rtol=1e-12)
+    assert np.isclose(cv_out, 0.0, atol=1e-15)
+    # orthogonal rotations on the column side keep every row norm (CV_out unchanged)
+    Wr = np.random.default_rng(0).standard_normal((16, 32)) * np.exp(np.linspace(0, 3, 32))
+    V = ref.rht_matrix(32, np.ones(32))
+    assert np.isclose(ref.norm_cv(Wr @ V.T)[1], ref.norm_cv(Wr)[1], rtol=1e-12)
+
+
+def test_rho_bounds_and_equality():
+    """rho <= 1 (Cauchy-Schwarz), = 1 iff h is proportional to a, ~k/d when the curvature sits
+    on k channels of equal row energy (the appendix's concentration remark)."""
+    rng = _rng(14)
+    h, a = rng.random(50) + 0.01, rng.random(50) + 0.01
+    assert ref.rho(h, a) < 1.0
+    assert np.isclose(ref.rho(3.0 * a, a), 1.0, rtol=1e-14)
+    d, k = 1000, 10
+    hk = np.zeros(d)
+    hk[:k] = 1.0
+    assert np.isclose(ref.rho(hk, np.ones(d)), k / d, rtol=1e-12)
+
+
+def test_prop2_bound_minimized_at_quarter_exponent():
+    """Prop. 2: over s = (h/a)^alpha the factor (sum h/s^2)(sum s^2 a) is smallest at
+    alpha = 1/4, where it equals (sum sqrt(h a))^2; a fine sweep finds the minimum there."""
+    rng = _rng(15)
+    h = np.exp(rng.standard_normal(200) * 1.5)
+    a = np.exp(rng.standard_normal(200) * 0.7)
+    alphas = np.linspace(0.0, 0.5, 201)
+    vals = [ref.prop2_bound(h, a, (h / a) ** al) for al in alphas]
+    assert np.isclose(alphas[int(np.argmin(vals))], 0.25, atol=1e-9)
+    assert np.isclose(min(vals), np.sum(np.sqrt(h * a)) ** 2, rtol=1e-12)
+    assert np.isclose(vals[0] , np.sum(h) * np.sum(a), rtol=1e-12)          # alpha = 0: s = 1
+    assert np.isclose(min(vals) / vals[0], ref.rho(h, a), rtol=1e-12)
+
+
+def test_scales_exponent_quarter_is_the_paper_rescale():
+    cfg = kqsynth.CONFIGS["tiny256"].replace(d_in=64, d_out=32, T=200)
+    L = kqsynth.layer(cfg)
+    HX, HG = ref.accum_factor(L["X"]), ref.accum_factor(L["G"])
+    sx, sg = ref.biip_scales(L["W"], HX, HG)
+    sx2, sg2 = ref.biip_scales_exp(L["W"], np.diag(HX), np.diag(HG), 0.25, 0.25)
+    assert np.allclose(sx, sx2, rtol=1e-14) and np.allclose(sg, sg2, rtol=1e-14)
+    sx0, sg0 = ref.biip_scales_exp(L["W"], np.diag(HX), np.diag(HG), 0.0, 0.0)
+    assert np.all(sx0 == 1.0) and np.all(sg0 == 1.0)
