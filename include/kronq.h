@@ -218,8 +218,10 @@ KQ_API kq_status kq_rotate_out(float* W, int64_t d_out, int64_t d_in, float* H_G
  *   Lt [n x n] fp32, the lower-triangular L with (H + damp_rel * mean(diag H) I)^-1 = L L^T
  *   and positive diagonal; the strict upper triangle of Lt is written with zeros. R = L^T
  *   is the upper factor whose row j drives the OBS update of column j. Computed as the
- *   Cholesky factorization of the index-reversed matrix followed by a triangular inverse
- *   (2 n^3 / 3 flops), fp32.
+ *   Cholesky factorization of the index-reversed matrix with its triangular inverse formed in
+ *   the same sweep (2 n^3 / 3 flops): fp32 on the diagonal blocks and panels, the trailing
+ *   updates on the tensor cores with the 3xTF32 split (fp32-accurate products, fp32 sums),
+ *   grouped into K = 1024 updates beyond each 1024-column super-panel when n > 1024.
  *   On a non-positive pivot, *info (required for that report) receives the 1-based index
  *   (in H's own indexing) of the failing pivot; Lt is then undefined. The caller may retry
  *   with a larger damp_rel.

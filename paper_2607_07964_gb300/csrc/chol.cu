@@ -22,6 +22,15 @@
 // 3xTF32 split (trail_tc.cu, Cholesky mode): chol_split_kernel writes the tf32 hi / lo of
 // the panel C_{.k} and of Z_{k.} transposed (the K-major operands), then the persistent
 // tensor-core kernel updates the tiles in place (TMA load, subtract, TMA store).
+// Two levels when n > 8 NB: steps are grouped in super-panels of 8 blocks. Inside a
+// super-panel the per-step update touches only its block columns (all rows below) and its
+// block rows of Z; the tiles beyond get the whole super-panel's update at once (K = 8 NB):
+// first the next super-panel's columns and rows (on the caller's stream: the next steps
+// read them), the remaining ones on a second library stream beside the next super-panel.
+// The trailing matrix is then read and written once per super-panel rather than once per
+// step (at n = 28672, ~90 GB of HBM traffic instead of ~700 GB), and the K = 1024 products
+// keep the tensor cores busy. The split sets alternate between super-panels, so a
+// super-panel's split does not overwrite the operands the previous remote update reads.
 #include <math.h>
 
 #include "kq_common.cuh"
@@ -33,19 +42,24 @@ namespace {
 
 constexpr int NB = 128;
 
+constexpr int SPB = 8;                          // blocks per super-panel
+
 struct Work {
     float* A;      // npad x npad, reversed damped H -> C (lower)
     float* Z;      // npad x npad, B -> C^-1 (lower)
-    float* Ch;     // npad x NB each: split C_{.k} (rows of the step's update), and the split
-    float* Cl;     // transpose of Z_{k.} (row j NB + c holds Z[k NB + .][j NB + c])
-    float* Zh;
-    float* Zl;
+    float* split[8];  // per set: Ch, Cl (split C panel), Zh, Zl (split Z rows, transposed)
     double* dsum;  // sum of diag(H)
 };
 
 inline size_t npad_of(int64_t n) { return static_cast<size_t>(cdiv(n, NB) * NB); }
 
-constexpr size_t ws_bytes_for(size_t np) { return (2 * np * np + 4 * np * NB) * sizeof(float) + 256; }
+// Split panel width and number of sets: one 128-column slice when one super-panel covers
+// the matrix, else two sets of a super-panel's width.
+constexpr size_t split_width(size_t np) { return np / NB > static_cast<size_t>(SPB) ? static_cast<size_t>(SPB) * NB : NB; }
+constexpr size_t split_sets(size_t np) { return np / NB > static_cast<size_t>(SPB) ? 2 : 1; }
+constexpr size_t ws_bytes_for(size_t np) {
+    return (2 * np * np + split_sets(np) * 4 * np * split_width(np)) * sizeof(float) + 256;
+}
 
 // --------------------------------------------------------------------- prep
 __global__ void diag_sum_kernel(const float* __restrict__ H, int64_t n, double* out) {
@@ -541,38 +555,50 @@ __global__ void __launch_bounds__(G_THREADS, 2) chol_next_kernel(Work w, int64_t
         update_quad(w, npad, k, bid, k + 1, blockIdx.y, sm);
 }
 
-// Operands of step k's tensor-core update, tf32 hi / lo: Ch/Cl rows r >= (k + 2) NB hold
-// C[r][k NB + c] (column block k of A); Zh/Zl rows q = j NB + c < (k + 1) NB hold
-// Z[k NB + c'][q] at column c' (row block k of Z, transposed through a 32 x 33 tile).
+// Operands of step k's tensor-core updates, tf32 hi / lo, into columns [col, col + NB) of
+// the [npad x width] split buffers: Ch/Cl rows r >= (k + 1) NB hold C[r][k NB + c] (column
+// block k of A); Zh/Zl rows q < (k + 1) NB hold Z[k NB + c][q] (row block k of Z, transposed
+// through a 32 x 33 tile) and rows q in [(k + 1) NB, zero_to) are zero (Z_kj = 0 for j > k).
 // Block (32, 8); one 32 x 32 tile per CTA.
 __global__ void chol_split_kernel(const float* __restrict__ A, const float* __restrict__ Z, int64_t npad, int k,
-                                  float* __restrict__ Ch, float* __restrict__ Cl, float* __restrict__ Zh,
-                                  float* __restrict__ Zl) {
+                                  int width, int col, int64_t zero_to, float* __restrict__ Ch, float* __restrict__ Cl,
+                                  float* __restrict__ Zh, float* __restrict__ Zl) {
     __shared__ float t[32][33];
     const int64_t ko = static_cast<int64_t>(k) * NB;
-    const int64_t crow0 = static_cast<int64_t>(k + 2) * NB;
+    const int64_t crow0 = static_cast<int64_t>(k + 1) * NB;
     const int64_t nct = (npad - crow0) / 32 * (NB / 32);
+    const int64_t nzt = (ko + NB) / 32 * (NB / 32);
     int64_t b = blockIdx.x;
     if (b < nct) {
         const int64_t r0 = crow0 + (b / (NB / 32)) * 32, c0 = (b % (NB / 32)) * 32;
         for (int r = threadIdx.y; r < 32; r += 8) {
             const float x = A[(r0 + r) * npad + ko + c0 + threadIdx.x];
             const float h = tf32_hi(x);
-            Ch[(r0 + r) * NB + c0 + threadIdx.x] = h;
-            Cl[(r0 + r) * NB + c0 + threadIdx.x] = x - h;
+            Ch[(r0 + r) * width + col + c0 + threadIdx.x] = h;
+            Cl[(r0 + r) * width + col + c0 + threadIdx.x] = x - h;
         }
         return;
     }
     b -= nct;
-    const int64_t kc0 = (b % (NB / 32)) * 32, q0 = (b / (NB / 32)) * 32;
-    for (int r = threadIdx.y; r < 32; r += 8) t[r][threadIdx.x] = Z[(ko + kc0 + r) * npad + q0 + threadIdx.x];
-    __syncthreads();
-    for (int r = threadIdx.y; r < 32; r += 8) {
-        const float x = t[threadIdx.x][r];   // Z[ko + kc0 + threadIdx.x][q0 + r]
-        const float h = tf32_hi(x);
-        Zh[(q0 + r) * NB + kc0 + threadIdx.x] = h;
-        Zl[(q0 + r) * NB + kc0 + threadIdx.x] = x - h;
+    if (b < nzt) {
+        const int64_t kc0 = (b % (NB / 32)) * 32, q0 = (b / (NB / 32)) * 32;
+        for (int r = threadIdx.y; r < 32; r += 8) t[r][threadIdx.x] = Z[(ko + kc0 + r) * npad + q0 + threadIdx.x];
+        __syncthreads();
+        for (int r = threadIdx.y; r < 32; r += 8) {
+            const float x = t[threadIdx.x][r];   // Z[ko + kc0 + threadIdx.x][q0 + r]
+            const float h = tf32_hi(x);
+            Zh[(q0 + r) * width + col + kc0 + threadIdx.x] = h;
+            Zl[(q0 + r) * width + col + kc0 + threadIdx.x] = x - h;
+        }
+        return;
     }
+    b -= nzt;
+    const int64_t q0 = ko + NB + (b / (NB / 32)) * 32, kc0 = (b % (NB / 32)) * 32;
+    if (q0 < zero_to)
+        for (int r = threadIdx.y; r < 32; r += 8) {
+            Zh[(q0 + r) * width + col + kc0 + threadIdx.x] = 0.0f;
+            Zl[(q0 + r) * width + col + kc0 + threadIdx.x] = 0.0f;
+        }
 }
 
 // -------------------------------------------------------------------- finish
@@ -619,17 +645,18 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
     }
     const int64_t npad = static_cast<int64_t>(npad_of(n));
     const int nbk = static_cast<int>(npad / NB);
+    const int width = static_cast<int>(split_width(static_cast<size_t>(npad)));
+    const int nsets = static_cast<int>(split_sets(static_cast<size_t>(npad)));
+    const bool two_level = nbk > SPB;
     Work w;
     w.A = static_cast<float*>(ws);
     w.Z = w.A + npad * npad;
-    w.Ch = w.Z + npad * npad;
-    w.Cl = w.Ch + npad * NB;
-    w.Zh = w.Cl + npad * NB;
-    w.Zl = w.Zh + npad * NB;
-    w.dsum = reinterpret_cast<double*>(w.Zl + npad * NB);
+    float* sp = w.Z + npad * npad;
+    for (int q = 0; q < 4 * nsets; ++q, sp += npad * width) w.split[q] = sp;
+    w.dsum = reinterpret_cast<double*>(sp);
     CholTcMaps maps;
     if (nbk > 2) {
-        kq_status st = maps.init(w.A, w.Z, w.Ch, w.Cl, w.Zh, w.Zl, npad);
+        kq_status st = maps.init(w.A, w.Z, npad, width, nsets, w.split);
         if (st != KQ_OK) return st;
     }
     static bool attr = false;
@@ -649,42 +676,83 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
     prep_kernel<<<static_cast<unsigned>(pgrid), 256, 0, stream>>>(H, n, npad, damp_rel, w.dsum, w.A, w.Z);
     KQ_LAUNCH_CHECK("prep_kernel");
     SideStream* side = nbk > 2 ? side_stream(stream) : nullptr;
-    bool forked = false;
-    for (int k = 0; k < nbk; ++k) {
-        chol_diag_kernel<<<1, DIAG_THREADS, DIAG_SMEM, stream>>>(w, n, npad, k, info);
-        KQ_LAUNCH_CHECK("chol_diag_kernel");
-        if (nbk > 1) {
-            chol_panel_kernel<<<dim3(nbk - 1, 4), G_THREADS, STRIP_SMEM, stream>>>(w, npad, k);
-            KQ_LAUNCH_CHECK("chol_panel_kernel");
-        }
-        if (k + 1 >= nbk) break;
-        int64_t rest = 0;
-        for (int i = k + 2; i < nbk; ++i) rest += i;
-        const bool fork = side && rest > 0;
-        if (fork) KQ_CUDA(cudaEventRecord(side->ev[0], stream));      // panel k done
-        if (forked) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));  // rest of step k - 1 done
-        chol_next_kernel<<<dim3(nbk, 4), G_THREADS, STRIP_SMEM, stream>>>(w, npad, k);
-        KQ_LAUNCH_CHECK("chol_next_kernel");
-        if (rest > 0) {
-            cudaStream_t rs = stream;
-            if (fork) {
-                KQ_CUDA(cudaStreamWaitEvent(side->s, side->ev[0], 0));
-                rs = side->s;
+    bool forked = false, remote_pending = false;
+    for (int k0 = 0; k0 < nbk; k0 += (two_level ? SPB : nbk)) {
+        const int k1 = two_level ? std::min(nbk, k0 + SPB) : nbk;   // this super-panel: blocks [k0, k1)
+        const int set = two_level ? (k0 / SPB) & 1 : 0;
+        const bool far_after = two_level && k1 < nbk;
+        for (int k = k0; k < k1; ++k) {
+            chol_diag_kernel<<<1, DIAG_THREADS, DIAG_SMEM, stream>>>(w, n, npad, k, info);
+            KQ_LAUNCH_CHECK("chol_diag_kernel");
+            if (nbk > 1) {
+                chol_panel_kernel<<<dim3(nbk - 1, 4), G_THREADS, STRIP_SMEM, stream>>>(w, npad, k);
+                KQ_LAUNCH_CHECK("chol_panel_kernel");
             }
-            const int64_t split_tiles = (npad - static_cast<int64_t>(k + 2) * NB) / 32 * (NB / 32) +
-                                        static_cast<int64_t>(k + 1) * NB / 32 * (NB / 32);
-            chol_split_kernel<<<static_cast<unsigned>(split_tiles), dim3(32, 8), 0, rs>>>(w.A, w.Z, npad, k, w.Ch, w.Cl,
-                                                                                          w.Zh, w.Zl);
-            KQ_LAUNCH_CHECK("chol_split_kernel");
-            kq_status st = chol_rest_tc(maps, nbk, k, info, rs);
+            if (k + 1 >= nbk) break;
+            const bool has_rest = k + 2 < k1;                 // tiles of this super-panel beyond k + 1
+            const bool need_split = has_rest || far_after;   // the super-panel update reads every slice
+            const bool fork = side && need_split;
+            if (fork) KQ_CUDA(cudaEventRecord(side->ev[0], stream));      // panel k done
+            if (forked) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));  // update of step k - 1 done
+            if (k + 1 < k1) {
+                chol_next_kernel<<<dim3(nbk, 4), G_THREADS, STRIP_SMEM, stream>>>(w, npad, k);
+                KQ_LAUNCH_CHECK("chol_next_kernel");
+            }
+            if (need_split) {
+                cudaStream_t rs = stream;
+                if (fork) {
+                    KQ_CUDA(cudaStreamWaitEvent(side->s, side->ev[0], 0));
+                    rs = side->s;
+                }
+                const int col = two_level ? (k - k0) * NB : 0;
+                const int64_t zero_to = far_after ? static_cast<int64_t>(k1) * NB : 0;
+                const int64_t tiles = (npad - static_cast<int64_t>(k + 1) * NB) / 32 * (NB / 32) +
+                                      static_cast<int64_t>(k + 1) * NB / 32 * (NB / 32) +
+                                      std::max<int64_t>(0, zero_to - static_cast<int64_t>(k + 1) * NB) / 32 * (NB / 32);
+                float* const* sp4 = w.split + 4 * set;
+                chol_split_kernel<<<static_cast<unsigned>(tiles), dim3(32, 8), 0, rs>>>(
+                    w.A, w.Z, npad, k, width, col, zero_to, sp4[0], sp4[1], sp4[2], sp4[3]);
+                KQ_LAUNCH_CHECK("chol_split_kernel");
+                if (has_rest) {
+                    // A: block columns [k + 2, k1), all rows below; Z: block rows [k + 2, k1), j <= k
+                    kq_status st = chol_update_tc(maps, set, nbk, k + 2, k1, k + 2, k1, k + 1, col, NB / 32, info, rs);
+                    if (st != KQ_OK) return st;
+                }
+                if (fork) {
+                    KQ_CUDA(cudaEventRecord(side->ev[1], side->s));
+                    forked = true;
+                }
+            }
+        }
+        if (!far_after) continue;
+        // The super-panel's update of every tile beyond it, K = (k1 - k0) NB: the next
+        // super-panel's block columns and rows first, on the caller's stream, then the rest on
+        // the second library stream beside the next super-panel (which touches none of it).
+        const int k2 = std::min(nbk, k1 + SPB);
+        const int nslab = (k1 - k0) * NB / 32;
+        if (side) {
+            KQ_CUDA(cudaEventRecord(side->ev2[0], side->s));                 // this super-panel's splits
+            KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[0], 0));
+            if (remote_pending) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[1], 0));   // previous remote part
+        }
+        kq_status st = chol_update_tc(maps, set, nbk, k1, k2, k1, k2, k1, 0, nslab, info, stream);
+        if (st != KQ_OK) return st;
+        if (k2 < nbk) {
+            cudaStream_t rs = stream;
+            if (side) {
+                KQ_CUDA(cudaStreamWaitEvent(side->s2, side->ev2[0], 0));
+                rs = side->s2;
+            }
+            st = chol_update_tc(maps, set, nbk, k2, nbk, k2, nbk, k1, 0, nslab, info, rs);
             if (st != KQ_OK) return st;
-            if (fork) {
-                KQ_CUDA(cudaEventRecord(side->ev[1], side->s));
-                forked = true;
+            if (side) {
+                KQ_CUDA(cudaEventRecord(side->ev2[1], side->s2));
+                remote_pending = true;
             }
         }
     }
     if (forked) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));
+    if (remote_pending) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[1], 0));
     finish_kernel<<<dim3(static_cast<unsigned>(cdiv(n, 32)), static_cast<unsigned>(cdiv(n, 32))),
                     dim3(32, 8), 0, stream>>>(w.Z, n, npad, Lt);
     KQ_LAUNCH_CHECK("finish_kernel");

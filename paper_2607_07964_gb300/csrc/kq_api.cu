@@ -71,8 +71,12 @@ SideStream* side_stream(cudaStream_t caller) {
     e.caller = caller;
     e.side.tried = true;
     if (cudaStreamCreateWithPriority(&e.side.s, cudaStreamNonBlocking, side_prio) != cudaSuccess ||
+        cudaStreamCreateWithPriority(&e.side.s2, cudaStreamNonBlocking, side_prio) != cudaSuccess ||
         cudaEventCreateWithFlags(&e.side.ev[0], cudaEventDisableTiming) != cudaSuccess ||
-        cudaEventCreateWithFlags(&e.side.ev[1], cudaEventDisableTiming) != cudaSuccess) {
+        cudaEventCreateWithFlags(&e.side.ev[1], cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&e.side.ev2[0], cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&e.side.ev2[1], cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&e.side.ev2[2], cudaEventDisableTiming) != cudaSuccess) {
         cudaGetLastError();
         e.side.s = nullptr;
     }

@@ -46,6 +46,8 @@ int num_sms();
 struct SideStream {
     cudaStream_t s;
     cudaEvent_t ev[2];
+    cudaStream_t s2;        // a second side stream (same priority) for long-running work
+    cudaEvent_t ev2[3];
     bool tried;
 };
 SideStream* side_stream(cudaStream_t caller);

@@ -54,15 +54,16 @@ __device__ __forceinline__ bool wait_quiet(uint64_t* bar, uint32_t parity) {
 // Which output tiles a launch updates, and from which operand maps.
 //   mode 0 (the sweep): a row x column grid over W[:, cb:], K slabs at columns i0 + 32 s of
 //     the first pair (E with R) and, for slabs >= 4, of the second pair (-Wpre with P).
-//   mode 1 (a Cholesky step k, see chol.cu): the lower tiles (i, j) of the padded matrix
-//     with i >= k + 2, j <= i, j != k + 1; K = 128 slabs at columns 32 s of the split
-//     column block C_{.k}; B from the C pair (j > k, output A) or from the transposed Z_{k.}
-//     pair (j <= k, output Z).
+//   mode 1 (a Cholesky update, see chol.cu): first the A region -- lower tiles (i, j) with
+//     j in [a_j0, a_j1) and i >= j, output A, B operand from the split C rows j -- then the
+//     B region -- tiles (i, j) with i in [b_i0, b_i1), j < b_j1, output Z, B operand from the
+//     split transposed Z rows j. The A operand is the split C rows i; K slabs at columns
+//     kx + 32 s of the split buffers.
 struct TileSet {
     int mode;
     int n_tiles;
-    int n_col_tiles, cb, i0;   // mode 0
-    int k;                     // mode 1
+    int n_col_tiles, cb, i0;                          // mode 0
+    int nbk, a_j0, a_j1, n_a, b_i0, b_i1, b_j1, kx;   // mode 1
 };
 
 // Tile t: top-left corner (row r0, column c0) and whether it takes the second B pair and
@@ -74,15 +75,21 @@ __device__ __forceinline__ void tile_at(const TileSet& ts, int t, int bn, int* r
         *alt = false;
         return;
     }
-    int i = ts.k + 2;
-    while (t >= i) {
-        t -= i;
-        ++i;
+    if (t < ts.n_a) {
+        int j = ts.a_j0;
+        while (t >= ts.nbk - j) {
+            t -= ts.nbk - j;
+            ++j;
+        }
+        *r0 = (j + t) * TBM;
+        *c0 = j * TBM;
+        *alt = false;
+        return;
     }
-    const int j = t < ts.k + 1 ? t : t + 1;
-    *r0 = i * TBM;
-    *c0 = j * TBM;
-    *alt = j <= ts.k;
+    t -= ts.n_a;
+    *r0 = (ts.b_i0 + t / ts.b_j1) * TBM;
+    *c0 = (t % ts.b_j1) * TBM;
+    *alt = true;
 }
 
 template <int BN, int TSTAGES>
@@ -92,9 +99,9 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
                 const __grid_constant__ CUtensorMap mQh, const __grid_constant__ CUtensorMap mQl,
                 const __grid_constant__ CUtensorMap mPh, const __grid_constant__ CUtensorMap mPl,
                 const __grid_constant__ CUtensorMap mW, const __grid_constant__ CUtensorMap mW2, TileSet ts,
-                int nslab, int* info) {
+                int nslab, int drain, int* info) {
     const int n_tiles = ts.n_tiles;
-    const int xk = ts.mode == 0 ? ts.i0 : 0;
+    const int xk = ts.mode == 0 ? ts.i0 : ts.kx;
     using C = TrailCfg<BN, TSTAGES>;
     constexpr int WBOX = TBM * 32 * 4;     // one 128-row x 32-column box of W (16 KB)
     extern __shared__ uint8_t smem_raw[];
@@ -181,7 +188,7 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
                     uint8_t* base = smem + st * C::STAGE;
                     // slabs 0..3: E and R; slabs 4..7 (with P): -Wpre and P. Cholesky tiles
                     // with j <= k take B from the second pair.
-                    const bool second = s >= TNSLAB;
+                    const bool second = ts.mode == 0 && s >= TNSLAB;
                     const bool bsec = second || alt;
                     const int x = xk + (second ? s - TNSLAB : s) * TBK;
                     tma_load_2d(base, second ? &mQh : &mEh, &full[st], x, r0);
@@ -199,38 +206,44 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
             constexpr uint32_t idesc = idesc_tf32_k_major(TBM, BN);
-            int k = 0, li = 0;
+            int k = 0, cc = 0;   // cc: accumulator chunks issued (the two buffers alternate per chunk)
             bool ok = true;
-            for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++li) {
-                const int buf = li & 1;
-                if (!mbar_wait(&tempty[buf], ((static_cast<uint32_t>(li) >> 1) & 1u) ^ 1u, abort_flag)) break;
-                tc_fence_after();
-                const uint32_t dt = tmem + static_cast<uint32_t>(buf * BN);
-                for (int s = 0; s < nslab; ++s, ++k) {
-                    const int st = k % TSTAGES;
-                    if (!mbar_wait(&full[st], static_cast<uint32_t>(k / TSTAGES) & 1u, abort_flag)) {
+            for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+                for (int s0 = 0; s0 < nslab && ok; s0 += drain, ++cc) {
+                    const int buf = cc & 1;
+                    if (!mbar_wait(&tempty[buf], ((static_cast<uint32_t>(cc) >> 1) & 1u) ^ 1u, abort_flag)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t a_hi = smem_u32(smem + st * C::STAGE);
-                    const uint32_t a_lo = a_hi + A_SLAB;
-                    const uint32_t b_hi = a_hi + 2 * A_SLAB;
-                    const uint32_t b_lo = b_hi + C::B_SLAB;
+                    const uint32_t dt = tmem + static_cast<uint32_t>(buf * BN);
+                    const int s1 = min(nslab, s0 + drain);
+                    for (int s = s0; s < s1; ++s, ++k) {
+                        const int st = k % TSTAGES;
+                        if (!mbar_wait(&full[st], static_cast<uint32_t>(k / TSTAGES) & 1u, abort_flag)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t a_hi = smem_u32(smem + st * C::STAGE);
+                        const uint32_t a_lo = a_hi + A_SLAB;
+                        const uint32_t b_hi = a_hi + 2 * A_SLAB;
+                        const uint32_t b_lo = b_hi + C::B_SLAB;
 #pragma unroll
-                    for (int kk = 0; kk < TBK / 8; ++kk) {   // 8 tf32 = 32 bytes per MMA
-                        const uint32_t ko = static_cast<uint32_t>(kk * 32);
-                        const uint64_t dah = smem_desc_sw128(a_hi + ko, 16, 1024);
-                        const uint64_t dal = smem_desc_sw128(a_lo + ko, 16, 1024);
-                        const uint64_t dbh = smem_desc_sw128(b_hi + ko, 16, 1024);
-                        const uint64_t dbl = smem_desc_sw128(b_lo + ko, 16, 1024);
-                        tc_mma_tf32(dt, dal, dbh, idesc, (s > 0 || kk > 0) ? 1u : 0u);
-                        tc_mma_tf32(dt, dah, dbl, idesc, 1u);
-                        tc_mma_tf32(dt, dah, dbh, idesc, 1u);
+                        for (int kk = 0; kk < TBK / 8; ++kk) {   // 8 tf32 = 32 bytes per MMA
+                            const uint32_t ko = static_cast<uint32_t>(kk * 32);
+                            const uint64_t dah = smem_desc_sw128(a_hi + ko, 16, 1024);
+                            const uint64_t dal = smem_desc_sw128(a_lo + ko, 16, 1024);
+                            const uint64_t dbh = smem_desc_sw128(b_hi + ko, 16, 1024);
+                            const uint64_t dbl = smem_desc_sw128(b_lo + ko, 16, 1024);
+                            tc_mma_tf32(dt, dal, dbh, idesc, (s > s0 || kk > 0) ? 1u : 0u);
+                            tc_mma_tf32(dt, dah, dbl, idesc, 1u);
+                            tc_mma_tf32(dt, dah, dbh, idesc, 1u);
+                        }
+                        tc_commit(&empty[st]);
                     }
-                    tc_commit(&empty[st]);
+                    if (ok) tc_commit(&tfull[buf]);
                 }
-                if (ok) tc_commit(&tfull[buf]);
             }
             tc_commit(mma_done);
             wait_quiet(mma_done, 0);
@@ -244,36 +257,42 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
         const int q = warp & 3;                 // TMEM lane quadrant this warp may access
         const int h = (warp - 2) >> 2;          // which half of the columns
         const int r = q * 32 + lane;            // row within the tile
-        int li = 0;
-        for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++li) {
-            const int buf = li & 1;
-            bool ok = mbar_wait(&tfull[buf], (static_cast<uint32_t>(li) >> 1) & 1u, abort_flag) &&
-                      mbar_wait(wfull, static_cast<uint32_t>(li) & 1u, abort_flag);
+        int li = 0, cc = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++li) {
+            ok = mbar_wait(wfull, static_cast<uint32_t>(li) & 1u, abort_flag);
             ok = __all_sync(0xffffffffu, ok) && !*abort_flag;
             if (!ok) break;
-            tc_fence_after();
-            const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) +
-                                   static_cast<uint32_t>(buf * BN + h * HALF);
+            // W -= each accumulator chunk in turn (K = drain * 32 per chunk)
+            for (int s0 = 0; s0 < nslab; s0 += drain, ++cc) {
+                const int buf = cc & 1;
+                ok = mbar_wait(&tfull[buf], (static_cast<uint32_t>(cc) >> 1) & 1u, abort_flag);
+                ok = __all_sync(0xffffffffu, ok) && !*abort_flag;
+                if (!ok) break;
+                tc_fence_after();
+                const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) +
+                                       static_cast<uint32_t>(buf * BN + h * HALF);
 #pragma unroll
-            for (int p = 0; p < HALF / 32; ++p) {
-                float v[32];
-                tmem_ld32(taddr + static_cast<uint32_t>(p * 32), v);
-                tc_wait_ld();
-                float4* rowp = reinterpret_cast<float4*>(wtile + (h * (HALF / 32) + p) * WBOX + r * 128);
+                for (int p = 0; p < HALF / 32; ++p) {
+                    float v[32];
+                    tmem_ld32(taddr + static_cast<uint32_t>(p * 32), v);
+                    tc_wait_ld();
+                    float4* rowp = reinterpret_cast<float4*>(wtile + (h * (HALF / 32) + p) * WBOX + r * 128);
 #pragma unroll
-                for (int c = 0; c < 8; ++c) {
-                    float4* cp = rowp + (c ^ (r & 7));
-                    const float4 o = *cp;
-                    *cp = make_float4(o.x - v[4 * c], o.y - v[4 * c + 1], o.z - v[4 * c + 2], o.w - v[4 * c + 3]);
+                    for (int c = 0; c < 8; ++c) {
+                        float4* cp = rowp + (c ^ (r & 7));
+                        const float4 o = *cp;
+                        *cp = make_float4(o.x - v[4 * c], o.y - v[4 * c + 1], o.z - v[4 * c + 2], o.w - v[4 * c + 3]);
+                    }
                 }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&tempty[buf]);   // the accumulator may be reused
             }
-            tc_fence_before();
+            if (!ok) break;
             fence_proxy_async();                        // this thread's W updates -> TMA
             __syncwarp();
-            if (lane == 0) {
-                mbar_arrive(&tempty[buf]);              // the accumulator may be reused
-                mbar_arrive(wdone);
-            }
+            if (lane == 0) mbar_arrive(wdone);
             if (warp == 2 && lane == 0) {
                 // store the tile once every warp has updated it, then free the buffer
                 if (mbar_wait(wdone, static_cast<uint32_t>(li) & 1u, abort_flag)) {
@@ -409,25 +428,28 @@ kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, in
     ts.i0 = static_cast<int>(i0);
     trail_tc_kernel<128, 2><<<static_cast<unsigned>(std::min(ts.n_tiles, num_sms())), T_THREADS, Cfg::SMEM, stream>>>(
         m.eh, m.el, m.rh_narrow, m.rl_narrow, with_p ? m.qh : m.eh, with_p ? m.ql : m.el,
-        with_p ? m.ph : m.rh_narrow, with_p ? m.pl : m.rl_narrow, m.w, m.w, ts, with_p ? 2 * TNSLAB : TNSLAB, info);
+        with_p ? m.ph : m.rh_narrow, with_p ? m.pl : m.rl_narrow, m.w, m.w, ts, with_p ? 2 * TNSLAB : TNSLAB,
+        with_p ? 2 * TNSLAB : TNSLAB, info);
     KQ_LAUNCH_CHECK("trail_tc_kernel");
     return KQ_OK;
 }
 
 // ------------------------------------------------------------ Cholesky step updates
-kq_status CholTcMaps::init(float* A, float* Z, const float* Ch, const float* Cl, const float* Zh, const float* Zl,
-                           int64_t npad) {
+kq_status CholTcMaps::init(float* A, float* Z, int64_t npad, int width, int nsets, float* const* split) {
     kq_status st;
     if ((st = make_f32_map(&a, A, npad, npad, TBM)) != KQ_OK) return st;
     if ((st = make_f32_map(&z, Z, npad, npad, TBM)) != KQ_OK) return st;
-    if ((st = make_f32_map(&ch, Ch, npad, 128, TBM)) != KQ_OK) return st;
-    if ((st = make_f32_map(&cl, Cl, npad, 128, TBM)) != KQ_OK) return st;
-    if ((st = make_f32_map(&zh, Zh, npad, 128, TBM)) != KQ_OK) return st;
-    if ((st = make_f32_map(&zl, Zl, npad, 128, TBM)) != KQ_OK) return st;
+    for (int q = 0; q < nsets; ++q) {
+        if ((st = make_f32_map(&ch[q], split[4 * q + 0], npad, width, TBM)) != KQ_OK) return st;
+        if ((st = make_f32_map(&cl[q], split[4 * q + 1], npad, width, TBM)) != KQ_OK) return st;
+        if ((st = make_f32_map(&zh[q], split[4 * q + 2], npad, width, TBM)) != KQ_OK) return st;
+        if ((st = make_f32_map(&zl[q], split[4 * q + 3], npad, width, TBM)) != KQ_OK) return st;
+    }
     return KQ_OK;
 }
 
-kq_status chol_rest_tc(const CholTcMaps& m, int nbk, int k, int* info, cudaStream_t stream) {
+kq_status chol_update_tc(const CholTcMaps& m, int set, int nbk, int a_j0, int a_j1, int b_i0, int b_i1, int b_j1,
+                         int kx, int nslab, int* info, cudaStream_t stream) {
     using Cfg = TrailCfg<128, 2>;
     static bool attr = false;
     if (!attr) {
@@ -436,11 +458,19 @@ kq_status chol_rest_tc(const CholTcMaps& m, int nbk, int k, int* info, cudaStrea
     }
     TileSet ts{};
     ts.mode = 1;
-    ts.k = k;
-    for (int i = k + 2; i < nbk; ++i) ts.n_tiles += i;
+    ts.nbk = nbk;
+    ts.a_j0 = a_j0;
+    ts.a_j1 = a_j1;
+    for (int j = a_j0; j < a_j1; ++j) ts.n_a += nbk - j;
+    ts.b_i0 = b_i0;
+    ts.b_i1 = b_i1;
+    ts.b_j1 = b_j1;
+    ts.kx = kx;
+    ts.n_tiles = ts.n_a + ((b_i1 > b_i0 && b_j1 > 0) ? (b_i1 - b_i0) * b_j1 : 0);
     if (ts.n_tiles == 0) return KQ_OK;
     trail_tc_kernel<128, 2><<<static_cast<unsigned>(std::min(ts.n_tiles, num_sms())), T_THREADS, Cfg::SMEM, stream>>>(
-        m.ch, m.cl, m.ch, m.cl, m.ch, m.cl, m.zh, m.zl, m.a, m.z, ts, TNSLAB, info);
+        m.ch[set], m.cl[set], m.ch[set], m.cl[set], m.ch[set], m.cl[set], m.zh[set], m.zl[set], m.a, m.z, ts, nslab,
+        TNSLAB, info);
     KQ_LAUNCH_CHECK("trail_tc_kernel");
     return KQ_OK;
 }

@@ -58,18 +58,20 @@ struct TrailMaps {
     kq_status set_w(float* W, int64_t d_out, int64_t d_in);
 };
 
-// Tensor maps of one inverse-Cholesky call (chol.cu): the padded A (-> C) and Z, and the
-// split operands of a step's update, C_{.k} and the transposed Z_{k.} ([npad x 128] each).
+// Tensor maps of one inverse-Cholesky call (chol.cu): the padded A (-> C) and Z, and per
+// split set the tf32 hi / lo of a block column panel of C and of the matching block rows of
+// Z transposed ([npad x width] each). split[] lists Ch, Cl, Zh, Zl of set 0, then set 1.
 struct CholTcMaps {
-    CUtensorMap a, z, ch, cl, zh, zl;
-    kq_status init(float* A, float* Z, const float* Ch, const float* Cl, const float* Zh, const float* Zl,
-                   int64_t npad);
+    CUtensorMap a, z;
+    CUtensorMap ch[2], cl[2], zh[2], zl[2];
+    kq_status init(float* A, float* Z, int64_t npad, int width, int nsets, float* const* split);
 };
 
-// Step k's update of every tile the next step does not read first: A_ij -= C_ik C_jk^T
-// (j > k) and Z_ij -= C_ik Z_kj (j <= k) for block rows i >= k + 2, j <= i, j != k + 1, on
-// the tensor cores (3xTF32, K = 128), from the split operands in Ch/Cl and Zh/Zl.
-kq_status chol_rest_tc(const CholTcMaps& m, int nbk, int k, int* info, cudaStream_t stream);
+// A Cholesky update on the tensor cores (3xTF32): A_ij -= C_i. C_j.^T for the lower tiles with
+// j in [a_j0, a_j1), i >= j, and Z_ij -= C_i. Z_.j for i in [b_i0, b_i1), j < b_j1, where the
+// dot runs over the nslab * 32 split columns starting at kx of split set `set`.
+kq_status chol_update_tc(const CholTcMaps& m, int set, int nbk, int a_j0, int a_j1, int b_i0, int b_i1, int b_j1,
+                         int kx, int nslab, int* info, cudaStream_t stream);
 
 // hi = src rounded to tf32, lo = src - hi (n elements).
 kq_status split_tf32(const float* src, int64_t n, float* hi, float* lo, cudaStream_t stream);
