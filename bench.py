@@ -14,6 +14,7 @@ bounded sample of the same workload and extrapolates to the same metric.
 from __future__ import annotations
 
 import argparse
+import datetime
 import hashlib
 import json
 import os
@@ -35,7 +36,8 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=None,
+                    help="timed steps (default: 100 for a layer or decode, 10 for a block, 3 for the oracle arm)")
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--config", default="q_proj_8b", choices=sorted(kqsynth.CONFIGS))
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
@@ -67,7 +69,11 @@ def parse():
     ap.add_argument("--drift", type=float, default=None, metavar="ALPHA",
                     help="with the GPTAQ drift correction of scaling ALPHA (full-precision input X~ = "
                          "X + 0.1 sigma z); default: GPTQ mode")
-    return ap.parse_args()
+    args = ap.parse_args()
+    if args.steps is None:
+        # a timed region of at least ~0.5 s, so that the clock record has samples inside it
+        args.steps = 3 if args.impl == "reference" else 10 if args.block else 100
+    return args
 
 
 def metric_of(alpha) -> str:
@@ -130,7 +136,7 @@ def syrk_traffic(cfg, launch_tokens: int):
 
 # --------------------------------------------------------------------------- clocks
 class ClockSampler:
-    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
               "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
               "clocks_event_reasons.sw_power_cap,pci.bus_id")
 
@@ -140,6 +146,8 @@ class ClockSampler:
         self.path = None
 
     def start(self):
+        """Start sampling and return once the first sample is written (bounded by 5 s), so
+        that the samples taken after this call cover the timed region that follows."""
         try:
             fd, self.path = tempfile.mkstemp(suffix=".csv")
             os.close(fd)
@@ -149,37 +157,49 @@ class ClockSampler:
                                          stdout=self.out, stderr=subprocess.DEVNULL)
         except (OSError, ValueError):
             self.proc = None
+            return
+        t_end = time.time() + 5.0
+        while time.time() < t_end and self.proc.poll() is None and os.path.getsize(self.path) == 0:
+            time.sleep(0.01)
+        self.t_begin = datetime.datetime.now()
 
     def stop(self) -> dict | None:
+        """Clock record of the region between start() and this call: the samples stamped
+        inside it, or, for a region shorter than the sampling period, the first sample
+        stamped after it began."""
         if self.proc is None:
             return None
+        t_stop = datetime.datetime.now()
+        time.sleep(0.25)   # lets a region shorter than the period receive its sample
         self.proc.terminate()
         try:
             self.proc.wait(timeout=5)
         except subprocess.TimeoutExpired:
             self.proc.kill()
         self.out.close()
-        sm, mx, reasons = [], [], set()
+        rows = []
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         for line in open(self.path):
             f = [x.strip() for x in line.split(",")]
-            if len(f) < 8:
+            if len(f) < 9:
                 continue
-            if self.bus_id and not f[7].lower().endswith(self.bus_id[-12:]):
+            if self.bus_id and not f[8].lower().endswith(self.bus_id[-12:]):
                 continue
             try:
-                sm.append(float(f[0]))
-                mx.append(float(f[1]))
+                ts = datetime.datetime.strptime(f[0], "%Y/%m/%d %H:%M:%S.%f")
+                rows.append((ts, float(f[1]), float(f[2]), [n for k, n in enumerate(names)
+                                                            if f[4 + k].lower() == "active"]))
             except ValueError:
                 continue
-            for k, n in enumerate(names):
-                if f[3 + k].lower() == "active":
-                    reasons.add(n)
         os.unlink(self.path)
-        if not sm:
+        inside = [r for r in rows if self.t_begin <= r[0] <= t_stop]
+        if not inside:
+            inside = [r for r in rows if r[0] >= self.t_begin][:1]
+        if not inside:
             return None
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
-                "reasons": sorted(reasons)}
+        return {"sm_mhz": statistics.median(r[1] for r in inside), "sm_max_mhz": max(r[2] for r in inside),
+                "samples": len(inside), "reasons": sorted({n for r in inside for n in r[3]}),
+                "region_ms": round((t_stop - self.t_begin).total_seconds() * 1e3, 1)}
 
 
 # ---------------------------------------------------------------- CPU oracle timing
