@@ -83,6 +83,18 @@ KQ_API kq_status kq_check(int* info, int reset, int* pivot_out, kq_stream_t stre
  */
 KQ_API kq_status kq_selftest_timeout(int* info, int64_t limit_us, kq_stream_t stream);
 
+/*
+ * kq_selftest_div: a diagnostic with no counterpart in the paper. The OBS sweep (Sec. 2.1
+ *   Eq. (obs_update)) divides by the grid scale and by [H^-1]_pp on its sequential chain; it
+ *   does so with a reciprocal and two Markstein corrections, which must equal IEEE
+ *   round-to-nearest division bit for bit. For n pairs a[i], b[i] (device fp32) this adds to
+ *   *mismatches (device uint64) the number of i where that division differs from the
+ *   correctly rounded a[i] / b[i] in any bit. n = 0 is a no-op; NULL pointers or n < 0 give
+ *   KQ_ERR_INVALID_ARG.
+ */
+KQ_API kq_status kq_selftest_div(const float* a, const float* b, int64_t n, unsigned long long* mismatches,
+                                 kq_stream_t stream);
+
 /* ------------------------------------------------------------------------------------
  * Stage 1: Kronecker factors.
  * Paper: Sec. 2.1 Eq. (ptq_obj) defines H_X = X X^T; Sec. 3.1 Eq. (kfac) the factor pair

@@ -110,6 +110,38 @@ extern "C" kq_status kq_selftest_timeout(int* info, int64_t limit_us, kq_stream_
     return KQ_OK;
 }
 
+namespace kq {
+namespace {
+// mismatches (+)= the number of i with div_rn(a_i, b_i, div_recip(b_i)) != __fdiv_rn(a_i, b_i)
+// bit for bit.
+__global__ void selftest_div_kernel(const float* __restrict__ a, const float* __restrict__ b, int64_t n,
+                                    unsigned long long* __restrict__ mismatches) {
+    unsigned long long bad = 0;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const float x = a[i], y = b[i];
+        bad += __float_as_uint(div_rn(x, y, div_recip(y))) != __float_as_uint(__fdiv_rn(x, y));
+    }
+    for (int o = 16; o > 0; o >>= 1) bad += __shfl_xor_sync(0xffffffffu, bad, o);
+    if ((threadIdx.x & 31) == 0 && bad) atomicAdd(mismatches, bad);
+}
+}  // namespace
+}  // namespace kq
+
+extern "C" kq_status kq_selftest_div(const float* a, const float* b, int64_t n, unsigned long long* mismatches,
+                                     kq_stream_t stream_) {
+    if (!a || !b || !mismatches || n < 0) {
+        kq::set_error("kq_selftest_div: invalid arguments");
+        return KQ_ERR_INVALID_ARG;
+    }
+    if (n == 0) return KQ_OK;
+    const int64_t blocks = std::min<int64_t>(kq::cdiv(n, 256), static_cast<int64_t>(kq::num_sms()) * 8);
+    kq::selftest_div_kernel<<<static_cast<unsigned>(blocks), 256, 0, reinterpret_cast<cudaStream_t>(stream_)>>>(
+        a, b, n, mismatches);
+    KQ_LAUNCH_CHECK("selftest_div_kernel");
+    return KQ_OK;
+}
+
 extern "C" const char* kq_last_error(void) { return kq::g_err; }
 
 extern "C" const char* kq_status_name(int s) {

@@ -59,6 +59,29 @@ __device__ __forceinline__ void record_error(int* info, int code) {
     if (info) atomicCAS(info, 0, code);
 }
 
+// Correctly rounded a / b from y = __frcp_rn(b), after Markstein's theorem (P. W. Markstein,
+// "Computation of elementary functions on the IBM RISC System/6000 processor", IBM J. Res.
+// Dev. 34(1), 1990): when y is within half an ulp of 1/b and q within one ulp of a/b, the
+// residual a - b q is exact under an fma and RN(q + (a - b q) y) = RN(a / b). q0 = RN(a y)
+// can be 1.5 ulp off, so one correction brings it within one ulp and a second one rounds
+// correctly. Every intermediate must stay normal: callers pass y = 0 for a divisor outside
+// [2^-60, 2^60] (div_recip), and a dividend outside that range (zero, subnormal, inf, NaN
+// included) also takes __fdiv_rn. Two dependent fma pairs replace the division on the
+// sequential chain of the OBS sweep; the reciprocal is computed once per divisor.
+__device__ __forceinline__ float div_recip(float b) {
+    const float ab = fabsf(b);
+    return (ab >= 0x1p-60f && ab <= 0x1p60f) ? __frcp_rn(b) : 0.0f;
+}
+__device__ __forceinline__ float div_rn(float a, float b, float y) {
+    const float aa = fabsf(a);
+    if (y != 0.0f && aa >= 0x1p-60f && aa <= 0x1p60f) {
+        const float q0 = __fmul_rn(a, y);
+        const float q1 = __fmaf_rn(__fmaf_rn(-q0, b, a), y, q0);
+        return __fmaf_rn(__fmaf_rn(-q1, b, a), y, q1);
+    }
+    return __fdiv_rn(a, b);
+}
+
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }

@@ -99,11 +99,14 @@ constexpr int LPR = KQ_OBS_LANES_PER_ROW;   // lanes per row (8 or 16)
 constexpr int CPL = BLK / LPR;              // columns per lane
 constexpr int NV = CPL / 4;                 // float4 slots per lane
 static_assert(LPR == 8 || LPR == 16, "lanes per row must be 8 or 16");
-constexpr int OBS_ROWS = 16;                // rows per CTA
-constexpr int OBS_THREADS = OBS_ROWS * LPR; // 128 or 256
-// With P the CTA holds both diagonal blocks (R and P, 128 KB), so one CTA fits an SM; it
-// takes twice the rows to keep as many warps per SM.
-constexpr int OBS_ROWS_P = 2 * OBS_ROWS;
+// 32 rows per CTA (8 warps): with 64 KB of shared memory and at most 128 registers a
+// thread, a CTA fits beside one CTA of the 3xTF32 far-column update (129 KB, 320 threads),
+// so block b + 1 runs while block b's far columns are updated (one CTA per SM up to 4864
+// rows, two beyond).
+constexpr int OBS_ROWS = 32;                // rows per CTA
+constexpr int OBS_THREADS = OBS_ROWS * LPR; // 256 or 512
+// With P the CTA holds both diagonal blocks (R and P, 128 KB): one CTA per SM, alone.
+constexpr int OBS_ROWS_P = 32;
 constexpr int OBS_THREADS_P = OBS_ROWS_P * LPR;
 
 // Packed layout of one diagonal block of R: row j holds R[i0 + j][i0 + c] at pos(c). The
@@ -112,14 +115,16 @@ constexpr int OBS_THREADS_P = OBS_ROWS_P * LPR;
 __host__ __device__ constexpr int slot_of(int lp, int v) { return lp * NV + ((v + ((lp * NV) >> 3)) & (NV - 1)); }
 __device__ __forceinline__ int pos_of(int c) { return 4 * slot_of(c / CPL, (c % CPL) >> 2) + (c & 3); }
 
-// Rp[b][j][pos(c)] = R[i0 + j][i0 + c] = Lt[i0 + c][i0 + j] (0 outside the matrix),
-// i0 = b BLK. Block (32, 8) transposes one 32 x 32 tile through shared memory.
-__global__ void pack_r_kernel(const float* __restrict__ Lt, int64_t n, float* __restrict__ Rp) {
+// Rp[b][j][pos(c)] = R[i0 + j][i1 + c] = Lt[i1 + c][i0 + j] (0 outside the matrix),
+// i0 = b BLK, i1 = i0 + coff BLK: the diagonal blocks (coff = 0) or the blocks right of them
+// (coff = 1). Block (32, 8) transposes one 32 x 32 tile through shared memory.
+__global__ void pack_r_kernel(const float* __restrict__ Lt, int64_t n, float* __restrict__ Rp, int coff) {
     __shared__ float t[32][33];
     const int64_t i0 = static_cast<int64_t>(blockIdx.z) * BLK;
+    const int64_t i1 = i0 + static_cast<int64_t>(coff) * BLK;
     const int c0 = blockIdx.y * 32, j0 = blockIdx.x * 32;
     for (int r = threadIdx.y; r < 32; r += 8) {
-        const int64_t c = i0 + c0 + r, j = i0 + j0 + threadIdx.x;
+        const int64_t c = i1 + c0 + r, j = i0 + j0 + threadIdx.x;
         t[r][threadIdx.x] = (c < n && j < n) ? Lt[c * n + j] : 0.0f;
     }
     __syncthreads();
@@ -141,7 +146,8 @@ __device__ __forceinline__ float group_max(float v) {
 
 // A lane's CPL columns [cb, cb + CPL) of row r of the block starting at column i0 (0 past
 // the block end nb or past the last row).
-template <bool VEC>
+// NC: through the read-only path (data this kernel does not write); else plain loads.
+template <bool VEC, bool NC = true>
 __device__ __forceinline__ void load_cols(const float* __restrict__ W, int64_t r, int64_t d_out, int64_t d_in,
                                           int64_t i0, int cb, int nb, float (&w)[CPL]) {
     const bool live = r < d_out;
@@ -149,7 +155,8 @@ __device__ __forceinline__ void load_cols(const float* __restrict__ W, int64_t r
     if (VEC && cb + CPL <= nb) {
 #pragma unroll
         for (int v = 0; v < NV; ++v) {
-            const float4 x = live ? __ldg(reinterpret_cast<const float4*>(src) + v) : make_float4(0.f, 0.f, 0.f, 0.f);
+            const float4* p = reinterpret_cast<const float4*>(src) + v;
+            const float4 x = live ? (NC ? __ldg(p) : *p) : make_float4(0.f, 0.f, 0.f, 0.f);
             w[4 * v] = x.x;
             w[4 * v + 1] = x.y;
             w[4 * v + 2] = x.z;
@@ -161,20 +168,68 @@ __device__ __forceinline__ void load_cols(const float* __restrict__ W, int64_t r
     }
 }
 
+template <bool VEC>
+__device__ __forceinline__ void store_cols(float* W, int64_t r, int64_t d_out, int64_t d_in, int64_t i0, int cb,
+                                           int nb, const float (&w)[CPL]) {
+    if (r >= d_out) return;
+    float* dst = W + r * d_in + i0 + cb;
+    if (VEC && cb + CPL <= nb) {
+#pragma unroll
+        for (int v = 0; v < NV; ++v)
+            reinterpret_cast<float4*>(dst)[v] = make_float4(w[4 * v], w[4 * v + 1], w[4 * v + 2], w[4 * v + 3]);
+    } else {
+#pragma unroll
+        for (int t = 0; t < CPL; ++t)
+            if (cb + t < nb) dst[t] = w[t];
+    }
+}
+
+// w -= E_prev R_prev,this for one row: the previous block's lazy update of this block
+// column, in the order of the trailing update (acc = fma(E_k, R_kc, acc) over ascending k,
+// then w - acc). Rq: the block of R (rows = the previous block's columns) packed like the
+// diagonal blocks, in shared memory; ep: this lane's CPL entries of the row of E_prev.
+__device__ __forceinline__ void prev_block_update(const float* Rq, const float (&ep)[CPL], int lp, int gbase,
+                                                  float (&w)[CPL]) {
+    float acc[CPL];
+#pragma unroll
+    for (int t = 0; t < CPL; ++t) acc[t] = 0.0f;
+#pragma unroll 1
+    for (int o = 0; o < LPR; ++o) {
+#pragma unroll
+        for (int jj = 0; jj < CPL; ++jj) {
+            const float ek = __shfl_sync(0xffffffffu, ep[jj], gbase | o);
+            const float* rr = Rq + (CPL * o + jj) * BLK;
+#pragma unroll
+            for (int v = 0; v < NV; ++v) {
+                const float4 x = *reinterpret_cast<const float4*>(rr + 4 * slot_of(lp, v));
+                acc[4 * v] = __fmaf_rn(ek, x.x, acc[4 * v]);
+                acc[4 * v + 1] = __fmaf_rn(ek, x.y, acc[4 * v + 1]);
+                acc[4 * v + 2] = __fmaf_rn(ek, x.z, acc[4 * v + 2]);
+                acc[4 * v + 3] = __fmaf_rn(ek, x.w, acc[4 * v + 3]);
+            }
+        }
+    }
+#pragma unroll
+    for (int t = 0; t < CPL; ++t) w[t] = __fsub_rn(w[t], acc[t]);
+}
+
 // VEC: d_in % 16 == 0 and W, codes (and pre_q) 16-byte aligned, so a lane's CPL columns
 // of W, E and codes move as 16-byte vectors. HASP: with the GPTAQ correction; Pp is P's
 // diagonal block packed like R's, and the block's -Wpre goes to Q (fp32 trailing update)
 // or to Qh + Ql (tensor-core trailing update).
 template <bool VEC, bool HASP>
-__global__ void __launch_bounds__(HASP ? OBS_THREADS_P : OBS_THREADS, HASP ? 1 : 3) obs_block_kernel(
-    const float* __restrict__ W, int64_t d_out, int64_t d_in, const float* __restrict__ Rp, int64_t i0,
+__global__ void __launch_bounds__(HASP ? OBS_THREADS_P : OBS_THREADS, HASP ? 1 : 2) obs_block_kernel(
+    float* __restrict__ W, int64_t d_out, int64_t d_in, const float* __restrict__ Rp, int64_t i0,
     int bits, int group, const float* __restrict__ gscale, const float* __restrict__ gzero,
     uint8_t* __restrict__ codes, float* __restrict__ scale, int32_t* __restrict__ zero,
     float* __restrict__ E, float* __restrict__ pre_q, float* __restrict__ Eh, float* __restrict__ El,
-    const float* __restrict__ Pp, float* __restrict__ Q, float* __restrict__ Qh, float* __restrict__ Ql) {
+    const float* __restrict__ Pp, float* __restrict__ Q, float* __restrict__ Qh, float* __restrict__ Ql,
+    const float* __restrict__ Rq) {
     extern __shared__ __align__(16) float Rs[];   // [BLK][BLK], packed (pack_r_kernel); then P's
     float* Ps = Rs + BLK * BLK;
-    for (int e = threadIdx.x; e < BLK * BLK / 4; e += blockDim.x) cp_async16(Rs + 4 * e, Rp + 4 * e, 16);
+    const bool fused = !HASP && Rq != nullptr;
+    // With Rq, the buffer first holds the previous block's R_prev,this for the fused update.
+    for (int e = threadIdx.x; e < BLK * BLK / 4; e += blockDim.x) cp_async16(Rs + 4 * e, (fused ? Rq : Rp) + 4 * e, 16);
     if (HASP)
         for (int e = threadIdx.x; e < BLK * BLK / 4; e += blockDim.x) cp_async16(Ps + 4 * e, Pp + 4 * e, 16);
     cp_async_commit();
@@ -190,14 +245,38 @@ __global__ void __launch_bounds__(HASP ? OBS_THREADS_P : OBS_THREADS, HASP ? 1 :
     const int64_t rstride = static_cast<int64_t>(gridDim.x) * warps * RPW;
     const int64_t rw0 = (static_cast<int64_t>(blockIdx.x) * warps + threadIdx.x / 32) * RPW;
     float w[CPL];
-    // The first row's weights load while R is staged; every thread reaches the barrier.
-    load_cols<VEC>(W, rw0 + lane / LPR, d_out, d_in, i0, cb, nb, w);
+    if (fused) {
+        // Each row of this CTA goes back to W updated, and the sweep below reads it with
+        // plain loads; then the diagonal block replaces R_prev,this in shared memory.
+        cp_async_wait<0>();
+        __syncthreads();
+        for (int64_t rw = rw0; rw < d_out; rw += rstride) {
+            const int64_t r = rw + lane / LPR;
+            float ep[CPL];
+            load_cols<VEC>(E, r, d_out, d_in, i0 - BLK, cb, BLK, ep);
+            load_cols<VEC>(W, r, d_out, d_in, i0, cb, nb, w);
+            prev_block_update(Rs, ep, lp, gbase, w);
+            store_cols<VEC>(W, r, d_out, d_in, i0, cb, nb, w);
+        }
+        __syncthreads();
+        for (int e = threadIdx.x; e < BLK * BLK / 4; e += blockDim.x) cp_async16(Rs + 4 * e, Rp + 4 * e, 16);
+        cp_async_commit();
+        load_cols<VEC, false>(W, rw0 + lane / LPR, d_out, d_in, i0, cb, nb, w);
+    } else {
+        // The first row's weights load while R is staged.
+        load_cols<VEC>(W, rw0 + lane / LPR, d_out, d_in, i0, cb, nb, w);
+    }
     cp_async_wait<0>();
-    __syncthreads();
+    __syncthreads();   // every thread reaches it
     for (int64_t rw = rw0; rw < d_out; rw += rstride) {
         const int64_t r = rw + lane / LPR;
         const bool live = r < d_out;
-        if (rw != rw0) load_cols<VEC>(W, r, d_out, d_in, i0, cb, nb, w);
+        if (rw != rw0) {
+            if (fused)
+                load_cols<VEC, false>(W, r, d_out, d_in, i0, cb, nb, w);
+            else
+                load_cols<VEC>(W, r, d_out, d_in, i0, cb, nb, w);
+        }
         Grid g;
         if (group) {
             float mn = 0.0f, mx = 0.0f;
@@ -391,6 +470,7 @@ __global__ void colloss_kernel(const float* __restrict__ E, int64_t d_out, int64
 
 struct ObsWs {
     float* Rp;      // packed diagonal blocks of R, nblk x BLK x BLK
+    float* Rq;      // packed blocks of R right of them (block b: rows of b, columns of b + 1)
     float* E;       // d_out x d_in
     float* gscale;  // d_out
     float* gzero;   // d_out
@@ -409,7 +489,7 @@ struct ObsWs {
 inline size_t align256(size_t b) { return (b + 255) & ~static_cast<size_t>(255); }
 
 size_t ws_base_bytes(int64_t d_out, int64_t d_in) {
-    return align256((static_cast<size_t>(cdiv(d_in, BLK)) * BLK * BLK + static_cast<size_t>(d_out) * d_in +
+    return align256((2 * static_cast<size_t>(cdiv(d_in, BLK)) * BLK * BLK + static_cast<size_t>(d_out) * d_in +
                      2 * static_cast<size_t>(d_out)) * sizeof(float));
 }
 
@@ -440,7 +520,8 @@ ObsWs carve(void* ws, int64_t d_out, int64_t d_in, int mode, bool with_p) {
     const bool tc = mode == KQ_TRAIL_3XTF32;
     ObsWs o;
     o.Rp = static_cast<float*>(ws);
-    o.E = o.Rp + cdiv(d_in, BLK) * BLK * BLK;
+    o.Rq = o.Rp + cdiv(d_in, BLK) * BLK * BLK;
+    o.E = o.Rq + cdiv(d_in, BLK) * BLK * BLK;
     o.gscale = o.E + d_out * d_in;
     o.gzero = o.gscale + d_out;
     o.Eh = o.El = o.Lh = o.Ll = o.Pp = o.Q = o.Qh = o.Ql = o.Ph = o.Pl = nullptr;
@@ -520,6 +601,11 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
                                      BLK * BLK * 4));
         KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      BLK * BLK * 4));
+        // Whole shared memory on the SM, so that a CTA fits beside a far-update CTA.
+        KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel<true, false>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                     cudaSharedmemCarveoutMaxShared));
+        KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel<false, false>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                     cudaSharedmemCarveoutMaxShared));
         KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      2 * BLK * BLK * 4));
         KQ_CUDA(cudaFuncSetAttribute(trailing_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -546,26 +632,46 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
         KQ_LAUNCH_CHECK("rowgrid_kernel");
     }
     const int64_t nblk = cdiv(d_in, BLK);
-    pack_r_kernel<<<dim3(BLK / 32, BLK / 32, static_cast<unsigned>(nblk)), dim3(32, 8), 0, stream>>>(Lt, d_in, o.Rp);
+    const int64_t row_ctas = hp ? std::min<int64_t>(cdiv(d_out, OBS_ROWS_P), static_cast<int64_t>(num_sms()))
+                                : std::min<int64_t>(cdiv(d_out, OBS_ROWS), 2 * static_cast<int64_t>(num_sms()));
+    pack_r_kernel<<<dim3(BLK / 32, BLK / 32, static_cast<unsigned>(nblk)), dim3(32, 8), 0, stream>>>(Lt, d_in, o.Rp, 0);
     KQ_LAUNCH_CHECK("pack_r_kernel");
+    if (!hp && nblk > 1 && row_ctas <= static_cast<int64_t>(num_sms()) && d_out * d_in <= (int64_t{24} << 20)) {
+        pack_r_kernel<<<dim3(BLK / 32, BLK / 32, static_cast<unsigned>(nblk - 1)), dim3(32, 8), 0, stream>>>(Lt, d_in,
+                                                                                                          o.Rq, 1);
+        KQ_LAUNCH_CHECK("pack_r_kernel");
+    }
     if (hp) {   // P[i0 + j][i0 + c] = Pt[i0 + c][i0 + j]: the same packing as R from Lt
-        pack_r_kernel<<<dim3(BLK / 32, BLK / 32, static_cast<unsigned>(nblk)), dim3(32, 8), 0, stream>>>(Pt, d_in, o.Pp);
+        pack_r_kernel<<<dim3(BLK / 32, BLK / 32, static_cast<unsigned>(nblk)), dim3(32, 8), 0, stream>>>(Pt, d_in, o.Pp, 0);
         KQ_LAUNCH_CHECK("pack_r_kernel");
     }
     const bool vec = (d_in % 4 == 0) && (reinterpret_cast<uintptr_t>(Lt) % 16 == 0);
     const bool bvec = (d_in % 16 == 0) && (reinterpret_cast<uintptr_t>(W) % 16 == 0) &&
                       (reinterpret_cast<uintptr_t>(codes) % 16 == 0);
-    const int64_t row_ctas = hp ? std::min<int64_t>(cdiv(d_out, OBS_ROWS_P), static_cast<int64_t>(num_sms()))
-                                : std::min<int64_t>(cdiv(d_out, OBS_ROWS), static_cast<int64_t>(num_sms()) * 3);
-    // Look-ahead: after block b, the update of block column b + 1 runs on the caller's stream
-    // (the next block kernel waits for it); the columns beyond run on a library side stream
-    // beside block b + 1. Every column still receives the block updates in block order
-    // (block column b + 2 gets E_b from the side stream before E_b+1 from the next step's
-    // first update, which waits for it), so the results are the same bits.
+    // GPTQ mode: block b's kernel first applies the previous block's update of its own
+    // columns (E_{b-1} R_{b-1,b}, fused), and the update of the columns beyond block b + 1
+    // runs on a library side stream beside block b + 1, whose CTAs share the SMs with it.
+    // Block b waits only for the far update of block b - 2 (the last one that writes its
+    // columns); the two far-update events alternate. With P: after block b the update of
+    // block column b + 1 runs on the caller's stream (the next block kernel waits for it),
+    // the columns beyond on the side stream beside block b + 1.
+    // Every column receives the block updates in block order either way. The fused update
+    // is fp32 in the trailing update's order in both modes (the far ones are 3xTF32 in the
+    // tensor-core mode).
     SideStream* side = nblk > 2 ? side_stream(stream) : nullptr;
     bool forked = false;
+    bool far_pending[2] = {false, false};
+    // 128 x 64 far-update tiles (a CTA fits beside a block-kernel CTA) while the block kernel
+    // runs one CTA per SM and the far updates take about as long as the block kernels
+    // (their mean, ~d_out d_in / 2 multiply-adds per block, against ~35 us a block: up to
+    // d_out d_in ~ 24M). Otherwise nothing fits beside the block kernel, or the sweep waits
+    // on the far updates, and 128 x 128 tiles are faster.
+    const bool narrow = !hp && row_ctas <= static_cast<int64_t>(num_sms()) && d_out * d_in <= (int64_t{24} << 20);
+    // The previous block's update fused into the block kernel: only then, so that nothing
+    // but the far update shares the SMs with the block kernel.
+    const bool fuse = narrow;
     auto trailing = [&](int64_t i0, int kb, int64_t cb, int64_t ce, cudaStream_t st) -> kq_status {
-        if (tc) return trail_tc(maps, W, d_out, d_in, i0, cb, ce, hp, info, st);
+        if (tc) return trail_tc(maps, W, d_out, d_in, i0, cb, ce, hp, narrow, info, st);
         dim3 grid(static_cast<unsigned>(cdiv(ce - cb, GT)), static_cast<unsigned>(cdiv(d_out, GT)));
         if (vec)
             trailing_kernel<true><<<grid, G_THREADS, G_SMEM, st>>>(W, o.E, Lt, d_out, d_in, i0, kb, cb, ce, o.Q, Pt);
@@ -575,29 +681,38 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
         return KQ_OK;
     };
     for (int64_t i0 = 0; i0 < d_in; i0 += BLK) {
+        const int64_t b = i0 / BLK;
         const int kb = static_cast<int>(std::min<int64_t>(BLK, d_in - i0));
-        const float* rp = o.Rp + (i0 / BLK) * BLK * BLK;
+        const float* rp = o.Rp + b * BLK * BLK;
+        const float* rq = fuse && b > 0 ? o.Rq + (b - 1) * BLK * BLK : nullptr;
+        if (fuse && far_pending[b & 1]) {   // the far update of block b - 2
+            KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[b & 1], 0));
+            far_pending[b & 1] = false;
+        }
         if (hp)
             obs_block_kernel<true, true><<<static_cast<unsigned>(row_ctas), OBS_THREADS_P, 2 * BLK * BLK * 4, stream>>>(
                 W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q, o.Eh, o.El,
-                o.Pp + (i0 / BLK) * BLK * BLK, o.Q, o.Qh, o.Ql);
+                o.Pp + b * BLK * BLK, o.Q, o.Qh, o.Ql, nullptr);
         else if (bvec)
             obs_block_kernel<true, false><<<static_cast<unsigned>(row_ctas), OBS_THREADS, BLK * BLK * 4, stream>>>(
                 W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q, o.Eh, o.El,
-                nullptr, nullptr, nullptr, nullptr);
+                nullptr, nullptr, nullptr, nullptr, rq);
         else
             obs_block_kernel<false, false><<<static_cast<unsigned>(row_ctas), OBS_THREADS, BLK * BLK * 4, stream>>>(
                 W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q, o.Eh, o.El,
-                nullptr, nullptr, nullptr, nullptr);
+                nullptr, nullptr, nullptr, nullptr, rq);
         KQ_LAUNCH_CHECK("obs_block_kernel");
         const int64_t nb0 = i0 + kb;                                // next block column
         if (nb0 >= d_in) break;
         const int64_t nb1 = std::min<int64_t>(d_in, nb0 + BLK);    // columns beyond it: [nb1, d_in)
         const bool fork = side && nb1 < d_in;
         if (fork) KQ_CUDA(cudaEventRecord(side->ev[0], stream));           // E of this block ready
-        if (forked) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));  // previous far update done
-        kq_status st = trailing(i0, kb, nb0, nb1, stream);
-        if (st != KQ_OK) return st;
+        kq_status st;
+        if (!fuse) {
+            if (forked) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));  // previous far update done
+            st = trailing(i0, kb, nb0, nb1, stream);
+            if (st != KQ_OK) return st;
+        }
         if (nb1 < d_in) {
             cudaStream_t fs = stream;
             if (fork) {
@@ -607,11 +722,16 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
             st = trailing(i0, kb, nb1, d_in, fs);
             if (st != KQ_OK) return st;
             if (fork) {
-                KQ_CUDA(cudaEventRecord(side->ev[1], side->s));
-                forked = true;
+                KQ_CUDA(cudaEventRecord(fuse ? side->ev2[b & 1] : side->ev[1], side->s));
+                if (fuse)
+                    far_pending[b & 1] = true;
+                else
+                    forked = true;
             }
         }
     }
+    for (int q = 0; q < 2; ++q)
+        if (far_pending[q]) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[q], 0));
     if (forked) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));
     if (col_loss) {
         colloss_kernel<<<static_cast<unsigned>(cdiv(d_in, CS_X)), dim3(CS_X, CS_Y), 0, stream>>>(o.E, d_out, d_in, col_loss);

@@ -385,6 +385,8 @@ kq_status TrailMaps::init(const float* E_hi, const float* E_lo, const float* Lt_
     if ((st = make_f32_map(&el, E_lo, d_out, d_in, TBM)) != KQ_OK) return st;
     if ((st = make_f32_map(&rh_narrow, Lt_hi, d_in, d_in, 128)) != KQ_OK) return st;
     if ((st = make_f32_map(&rl_narrow, Lt_lo, d_in, d_in, 128)) != KQ_OK) return st;
+    if ((st = make_f32_map(&rh64, Lt_hi, d_in, d_in, 64)) != KQ_OK) return st;
+    if ((st = make_f32_map(&rl64, Lt_lo, d_in, d_in, 64)) != KQ_OK) return st;
     return KQ_OK;
 }
 
@@ -402,36 +404,49 @@ kq_status TrailMaps::set_w(float* W, int64_t d_out, int64_t d_in) {
     return make_f32_map(&w, W, d_out, d_in, TBM);
 }
 
-kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, int64_t i0, int64_t cb, int64_t ce,
-                   bool with_p, int* info, cudaStream_t stream) {
-    // Persistent: at most one CTA per SM, each walking the tiles t, t + grid, ... (column
-    // tile fastest, so the CTAs running together share row and column operands in L2).
-    // 128-column tiles; a range either is a whole number of tiles or ends at d_in (the TMA
-    // copies clip the last tile there).
-    using Cfg = TrailCfg<128, 2>;
-    if ((ce - cb) % 128 != 0 && ce != d_in) {
-        set_error("trailing update: column range [%lld, %lld) is not whole tiles", (long long)cb, (long long)ce);
-        return KQ_ERR_INVALID_ARG;
-    }
+namespace {
+template <int BN>
+kq_status launch_trail(const TrailMaps& m, const CUtensorMap& rh, const CUtensorMap& rl, int64_t d_out, int64_t i0,
+                       int64_t cb, int64_t ce, bool with_p, int* info, cudaStream_t stream) {
+    using Cfg = TrailCfg<BN, 2>;
     static bool attr = false;
     if (!attr) {
-        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<128, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
+        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<BN, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
+        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<BN, 2>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                     cudaSharedmemCarveoutMaxShared));
         attr = true;
     }
     const int n_row = static_cast<int>(cdiv(d_out, TBM));
-    const int n_col = static_cast<int>(cdiv(ce - cb, 128));
+    const int n_col = static_cast<int>(cdiv(ce - cb, BN));
     TileSet ts{};
     ts.mode = 0;
     ts.n_tiles = n_row * n_col;
     ts.n_col_tiles = n_col;
     ts.cb = static_cast<int>(cb);
     ts.i0 = static_cast<int>(i0);
-    trail_tc_kernel<128, 2><<<static_cast<unsigned>(std::min(ts.n_tiles, num_sms())), T_THREADS, Cfg::SMEM, stream>>>(
-        m.eh, m.el, m.rh_narrow, m.rl_narrow, with_p ? m.qh : m.eh, with_p ? m.ql : m.el,
-        with_p ? m.ph : m.rh_narrow, with_p ? m.pl : m.rl_narrow, m.w, m.w, ts, with_p ? 2 * TNSLAB : TNSLAB,
-        with_p ? 2 * TNSLAB : TNSLAB, info);
+    trail_tc_kernel<BN, 2><<<static_cast<unsigned>(std::min(ts.n_tiles, num_sms())), T_THREADS, Cfg::SMEM, stream>>>(
+        m.eh, m.el, rh, rl, with_p ? m.qh : m.eh, with_p ? m.ql : m.el, with_p ? m.ph : rh, with_p ? m.pl : rl, m.w, m.w,
+        ts, with_p ? 2 * TNSLAB : TNSLAB, with_p ? 2 * TNSLAB : TNSLAB, info);
     KQ_LAUNCH_CHECK("trail_tc_kernel");
     return KQ_OK;
+}
+}  // namespace
+
+kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, int64_t i0, int64_t cb, int64_t ce,
+                   bool with_p, bool narrow, int* info, cudaStream_t stream) {
+    // Persistent: at most one CTA per SM, each walking the tiles t, t + grid, ... (column
+    // tile fastest, so the CTAs running together share row and column operands in L2). A
+    // range either is a whole number of tiles or ends at d_in (the TMA copies clip the last
+    // tile there).
+    (void)W;
+    narrow = narrow && !with_p;
+    const int bn = narrow ? 64 : 128;
+    if ((ce - cb) % bn != 0 && ce != d_in) {
+        set_error("trailing update: column range [%lld, %lld) is not whole tiles", (long long)cb, (long long)ce);
+        return KQ_ERR_INVALID_ARG;
+    }
+    if (narrow) return launch_trail<64>(m, m.rh64, m.rl64, d_out, i0, cb, ce, false, info, stream);
+    return launch_trail<128>(m, m.rh_narrow, m.rl_narrow, d_out, i0, cb, ce, with_p, info, stream);
 }
 
 // ------------------------------------------------------------ Cholesky step updates

@@ -49,6 +49,7 @@ kq_status make_f32_map(CUtensorMap* m, const float* base, int64_t rows, int64_t 
 struct TrailMaps {
     CUtensorMap eh, el;                  // E_hi, E_lo [d_out x d_in], 128-row boxes
     CUtensorMap rh_narrow, rl_narrow;    // Lt_hi, Lt_lo [d_in x d_in], 128-row boxes
+    CUtensorMap rh64, rl64;              // the same with 64-row boxes (64-column tiles)
     CUtensorMap w;                       // W [d_out x d_in], 128-row boxes (read and written)
     CUtensorMap qh, ql, ph, pl;          // with P: (-Wpre)_hi, _lo [d_out x d_in], Pt_hi, Pt_lo [d_in x d_in]
     kq_status init(const float* E_hi, const float* E_lo, const float* Lt_hi, const float* Lt_lo, int64_t d_out,
@@ -77,9 +78,10 @@ kq_status chol_update_tc(const CholTcMaps& m, int set, int nbk, int a_j0, int a_
 kq_status split_tf32(const float* src, int64_t n, float* hi, float* lo, cudaStream_t stream);
 
 // W[:, cb:ce] -= E[:, i0:i0+128] R[i0:i0+128, cb:ce] (R[k][c] = Lt[c][k]) on tensor cores,
-// and with_p: also -= Q[:, i0:i0+128] P[i0:i0+128, cb:ce] (P[k][c] = Pt[c][k]); [cb, ce) must
-// be whole 128-column tiles or end at d_in. W is the one set_w was given.
+// and with_p: also -= Q[:, i0:i0+128] P[i0:i0+128, cb:ce] (P[k][c] = Pt[c][k]). Tiles are
+// 128 x 64 when narrow (GPTQ mode only; 129 KB of shared memory per CTA), else 128 x 128
+// (193 KB); [cb, ce) must be whole tiles or end at d_in. W is the one set_w was given.
 kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, int64_t i0, int64_t cb, int64_t ce,
-                   bool with_p, int* info, cudaStream_t stream);
+                   bool with_p, bool narrow, int* info, cudaStream_t stream);
 
 }  // namespace kq

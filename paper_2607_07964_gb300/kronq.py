@@ -44,6 +44,7 @@ def lib() -> ctypes.CDLL:
             "kq_launch_count": ([], ctypes.c_uint64),
             "kq_check": ([P, I, P, P], I),
             "kq_selftest_timeout": ([P, I64, P], I),
+            "kq_selftest_div": ([P, P, I64, P, P], I),
             "kq_accum_factor": ([P, I64, I64, I64, P, I, P, P, P], I),
             "kq_compute_scales": ([P, I64, I64, P, P, P, P, P], I),
             "kq_compute_scales_diag": ([P, I64, I64, P, P, P, P, P], I),
@@ -136,6 +137,15 @@ def kq_selftest_timeout(info, limit_us: int, stream=None) -> None:
     """A kernel whose bounded wait runs out (nothing arrives); *info gets -KQ_ERR_TIMEOUT."""
     _need(info, "info", torch.int32)
     _ok(lib().kq_selftest_timeout(_ptr(info), int(limit_us), _stream(stream)), "kq_selftest_timeout")
+
+
+def kq_selftest_div(a, b, mismatches, stream=None) -> None:
+    """mismatches (+)= the count of a[i] / b[i] where the sweep's division differs from IEEE
+    round-to-nearest division in any bit; a, b fp32 of one shape, mismatches one int64."""
+    _need(a, "a", torch.float32)
+    _need(b, "b", torch.float32, tuple(a.shape))
+    _need(mismatches, "mismatches", torch.int64, (1,))
+    _ok(lib().kq_selftest_div(_ptr(a), _ptr(b), a.numel(), _ptr(mismatches), _stream(stream)), "kq_selftest_div")
 
 
 def kq_accum_factor(A, H, accumulate: bool = False, trace=None, info=None, stream=None) -> None:

@@ -432,6 +432,49 @@ def test_diag_variants_match_matrix_variants():
     assert torch.equal(t1, t2)
 
 
+# ------------------------------------------------------------ sweep division
+def _bits_to_f32(u):
+    return u.to(torch.int32).view(torch.float32)
+
+
+@pytest.mark.parametrize("domain", ["all_normal", "sweep_range", "near_binade", "special"])
+def test_sweep_division_matches_ieee_division(domain):
+    """The sweep's division (reciprocal plus two Markstein corrections, with a fallback to the
+    IEEE division outside the range where the theorem holds) equals round-to-nearest IEEE
+    division bit for bit."""
+    g = torch.Generator(device=DEV).manual_seed({"all_normal": 1, "sweep_range": 2, "near_binade": 3, "special": 4}[domain])
+    n = 1 << 24
+
+    def rand_bits(exp_lo, exp_hi, mant=None):
+        sign = torch.randint(0, 2, (n,), device=DEV, generator=g, dtype=torch.int64) << 31
+        e = torch.randint(exp_lo, exp_hi + 1, (n,), device=DEV, generator=g, dtype=torch.int64) << 23
+        m = mant if mant is not None else torch.randint(0, 1 << 23, (n,), device=DEV, generator=g, dtype=torch.int64)
+        u = (sign | e | m) & 0xFFFFFFFF
+        return _bits_to_f32(torch.where(u >= 2**31, u - 2**32, u))
+
+    if domain == "all_normal":
+        a, b = rand_bits(1, 254), rand_bits(1, 254)
+    elif domain == "sweep_range":     # weights / scales and errors / diagonal entries
+        a = (torch.rand(n, device=DEV, generator=g) - 0.5) * 2.0 ** torch.randint(-12, 4, (n,), device=DEV, generator=g)
+        b = torch.rand(n, device=DEV, generator=g) * 2.0 ** torch.randint(-12, 6, (n,), device=DEV, generator=g) + 1e-30
+    elif domain == "near_binade":     # significands near 2 on both sides: q0 furthest from a / b
+        hi = (1 << 23) - torch.randint(1, 1 << 12, (n,), device=DEV, generator=g, dtype=torch.int64)
+        a = rand_bits(100, 150, hi)
+        b = rand_bits(100, 150, torch.randint(0, 1 << 12, (n,), device=DEV, generator=g, dtype=torch.int64))
+    else:                             # zeros, subnormals, range edges, infinities, NaN
+        vals = torch.tensor([0.0, -0.0, 1e-45, -1e-45, 1e-40, 2.0 ** -60, 2.0 ** -61, 2.0 ** 60, 2.0 ** 61,
+                             3.0e38, float("inf"), -float("inf"), float("nan"), 1.0, -1.0, 1.5], device=DEV)
+        idx_a = torch.randint(0, len(vals), (n,), device=DEV, generator=g)
+        idx_b = torch.randint(0, len(vals), (n,), device=DEV, generator=g)
+        a = torch.where(torch.rand(n, device=DEV, generator=g) < 0.5, vals[idx_a], rand_bits(1, 254))
+        b = torch.where(torch.rand(n, device=DEV, generator=g) < 0.5, vals[idx_b], rand_bits(1, 254))
+    a, b = a.float().contiguous(), b.float().contiguous()
+    bad = torch.zeros(1, dtype=torch.int64, device=DEV)
+    K().kq_selftest_div(a, b, bad)
+    torch.cuda.synchronize()
+    assert int(bad.item()) == 0
+
+
 # ------------------------------------------------------------ failure detection
 def test_bounded_wait_reports_timeout_and_context_survives():
     """A wait that nothing satisfies (no GPU fault, no hang): the kernel gives up after its
