@@ -64,22 +64,28 @@ __device__ __forceinline__ void record_error(int* info, int code) {
 // Dev. 34(1), 1990): when y is within half an ulp of 1/b and q within one ulp of a/b, the
 // residual a - b q is exact under an fma and RN(q + (a - b q) y) = RN(a / b). q0 = RN(a y)
 // can be 1.5 ulp off, so one correction brings it within one ulp and a second one rounds
-// correctly. Every intermediate must stay normal: callers pass y = 0 for a divisor outside
-// [2^-60, 2^60] (div_recip), and a dividend outside that range (zero, subnormal, inf, NaN
-// included) also takes __fdiv_rn. Two dependent fma pairs replace the division on the
-// sequential chain of the OBS sweep; the reciprocal is computed once per divisor.
+// correctly; a = +-0 returns q0 (its sign is right). The theorem needs every intermediate
+// normal: div_recip gives y = 0 for a divisor outside [2^-60, 2^60], and div_rn_fast_ok
+// tells whether (a, y) is inside the range where div_rn_fast is exact; div_rn falls back to
+// __fdiv_rn outside it. The OBS sweep runs div_rn_fast (two dependent fma pairs on its
+// sequential chain, the reciprocal computed once per divisor) and redoes a row group with
+// __fdiv_rn when div_rn_fast_ok failed anywhere in it.
 __device__ __forceinline__ float div_recip(float b) {
     const float ab = fabsf(b);
     return (ab >= 0x1p-60f && ab <= 0x1p60f) ? __frcp_rn(b) : 0.0f;
 }
-__device__ __forceinline__ float div_rn(float a, float b, float y) {
+__device__ __forceinline__ bool div_rn_fast_ok(float a, float y) {
     const float aa = fabsf(a);
-    if (y != 0.0f && aa >= 0x1p-60f && aa <= 0x1p60f) {
-        const float q0 = __fmul_rn(a, y);
-        const float q1 = __fmaf_rn(__fmaf_rn(-q0, b, a), y, q0);
-        return __fmaf_rn(__fmaf_rn(-q1, b, a), y, q1);
-    }
-    return __fdiv_rn(a, b);
+    return y != 0.0f && (a == 0.0f || (aa >= 0x1p-60f && aa <= 0x1p60f));
+}
+__device__ __forceinline__ float div_rn_fast(float a, float b, float y) {
+    const float q0 = __fmul_rn(a, y);
+    const float q1 = __fmaf_rn(__fmaf_rn(-q0, b, a), y, q0);
+    const float q2 = __fmaf_rn(__fmaf_rn(-q1, b, a), y, q1);
+    return a == 0.0f ? q0 : q2;
+}
+__device__ __forceinline__ float div_rn(float a, float b, float y) {
+    return div_rn_fast_ok(a, y) ? div_rn_fast(a, b, y) : __fdiv_rn(a, b);
 }
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {

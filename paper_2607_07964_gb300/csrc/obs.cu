@@ -23,6 +23,8 @@
 //   colloss_kernel   col_loss[j] = sum over rows of E_j^2, fixed order (sumsq.cuh)
 #include <math.h>
 
+#include <type_traits>
+
 #include "kq_common.cuh"
 #include "tile_gemm.cuh"
 #include "sumsq.cuh"
@@ -268,6 +270,10 @@ __global__ void __launch_bounds__(HASP ? OBS_THREADS_P : OBS_THREADS, HASP ? 1 :
     }
     cp_async_wait<0>();
     __syncthreads();   // every thread reaches it
+    // Reciprocals of the block's diagonal R_jj for the column steps' divisions.
+    __shared__ float rds[BLK];
+    for (int j = threadIdx.x; j < BLK; j += blockDim.x) rds[j] = j < nb ? div_recip(Rs[j * BLK + pos_of(j)]) : 0.0f;
+    __syncthreads();
     for (int64_t rw = rw0; rw < d_out; rw += rstride) {
         const int64_t r = rw + lane / LPR;
         const bool live = r < d_out;
@@ -296,6 +302,12 @@ __global__ void __launch_bounds__(HASP ? OBS_THREADS_P : OBS_THREADS, HASP ? 1 :
             g.scale = live ? gscale[r] : 1.0f;
             g.zero = live ? gzero[r] : 0.0f;
         }
+        const float ys = div_recip(g.scale);
+        // The column steps of this row group; EXACT: IEEE divisions, else div_rn_fast, with
+        // the return value telling whether every operand was inside its exact range.
+        auto sweep = [&](auto exact_tag) -> bool {
+        constexpr bool EXACT = decltype(exact_tag)::value;
+        bool ok = true;
 #pragma unroll 1
         for (int o = 0; o < LPR; ++o) {
             if (CPL * o >= nb) break;   // uniform across the CTA
@@ -311,14 +323,29 @@ __global__ void __launch_bounds__(HASP ? OBS_THREADS_P : OBS_THREADS, HASP ? 1 :
                 if (j < nb) {   // uniform across the CTA
                     const float* rr = Rs + j * BLK;
                     const float dj = rr[4 * slot_of(o, jj >> 2) + (jj & 3)];
+                    const float yd = rds[j];
                     float4 rv[NV];
 #pragma unroll
                     for (int v = 0; v < NV; ++v) rv[v] = *reinterpret_cast<const float4*>(rr + 4 * slot_of(lp, v));
                     const float wj = __shfl_sync(0xffffffffu, w[jj], gbase | o);
-                    float qq = __fadd_rn(rintf(__fdiv_rn(wj, g.scale)), g.zero);
+                    float q0;
+                    if constexpr (EXACT) {
+                        q0 = __fdiv_rn(wj, g.scale);
+                    } else {
+                        q0 = div_rn_fast(wj, g.scale, ys);
+                        ok = ok & div_rn_fast_ok(wj, ys);
+                    }
+                    float qq = __fadd_rn(rintf(q0), g.zero);
                     qq = fminf(fmaxf(qq, 0.0f), maxq);
                     const float what = __fmul_rn(g.scale, __fsub_rn(qq, g.zero));
-                    const float err = __fdiv_rn(__fsub_rn(wj, what), dj);
+                    const float dif = __fsub_rn(wj, what);
+                    float err;
+                    if constexpr (EXACT) {
+                        err = __fdiv_rn(dif, dj);
+                    } else {
+                        err = div_rn_fast(dif, dj, yd);
+                        ok = ok & div_rn_fast_ok(dif, yd);
+                    }
                     e[jj] = err;
                     cq[jj >> 2] |= static_cast<uint32_t>(qq) << (8 * (jj & 3));
                     if (pre_q && live && lp == o) pre_q[r * d_in + i0 + j] = wj;
@@ -415,6 +442,17 @@ __global__ void __launch_bounds__(HASP ? OBS_THREADS_P : OBS_THREADS, HASP ? 1 :
                         }
                 }
             }
+        }
+        return ok;
+        };
+        if (!__all_sync(0xffffffffu, sweep(std::false_type{}))) {
+            // an operand outside the fast division's range in this warp's rows: the row
+            // group again from its start, with IEEE divisions (same outputs overwritten)
+            if (fused)
+                load_cols<VEC, false>(W, r, d_out, d_in, i0, cb, nb, w);
+            else
+                load_cols<VEC>(W, r, d_out, d_in, i0, cb, nb, w);
+            sweep(std::true_type{});
         }
     }
 }

@@ -250,6 +250,26 @@ def test_sweep_bit_exact(d_out, d_in, bits, group):
     assert np.allclose(g["col_loss"], want_loss, rtol=1e-6, atol=0)
 
 
+@pytest.mark.parametrize("group", [0, 128])
+def test_sweep_bit_exact_extreme_rows(group):
+    """Rows whose values leave the range of the sweep's fast division (tiny and huge rows,
+    exact zeros, subnormals, a zero row) take the IEEE-division redo: still bit-exact."""
+    Wp, Lt = _sweep_inputs(64, 384, seed=11)
+    Wp = Wp.copy()
+    Wp[3] *= np.float32(1e-25)      # grid scale below 2^-60
+    Wp[11] *= np.float32(1e25)      # grid scale above 2^60
+    Wp[7, ::5] = 0.0
+    Wp[7, 1::7] = np.float32(1e-40)
+    Wp[20] = 0.0
+    Wp[21, 130:140] = np.float32(-1e-41)
+    g = _gpu_sweep(Wp, Lt, 4, group)
+    c = obs_sweep_fp32(Wp, Lt, 4, group, 128, want_pre_q=True)
+    assert np.array_equal(g["codes"], c["codes"])
+    assert np.array_equal(g["scale"], c["scale"])
+    assert np.array_equal(g["zero"], c["zero"].astype(np.int32))
+    assert np.array_equal(g["pre_q"], c["pre_q"])
+
+
 def _tie_distance(pre_q, scale_row_groups, group, r, j):
     """|frac(w / scale) - 1/2| of the oracle's value that column j of row r quantizes."""
     g = 0 if group == 0 else j // group
