@@ -168,7 +168,11 @@ KQ_API kq_status kq_accum_drift(const uint16_t* Xt, const uint16_t* X, int64_t T
  *   use the values already in out, so the sides may come from two calls (X side first).
  *
  * kq_rotate_in (input side, length d_in, sign_v = sigma_V):
- *   dir = KQ_FWD: W <- (W S_X) V^T, and if H_X != NULL: H_X <- V S_X^-1 H_X S_X^-1 V^T.
+ *   dir = KQ_FWD: W <- (W S_X) V^T, and if H_X != NULL: H_X <- V S_X^-1 H_X S_X^-1 V^T
+ *   (H_X any square matrix, e.g. the drift statistic D). dir = KQ_FWD_SYM: the same for a
+ *   symmetric H_X, which lets the two-sided transform skip its last transposition: the
+ *   result is the transpose of KQ_FWD's up to rounding (both equal the exact V M V^T to
+ *   fp32 rounding). The same holds for kq_rotate_out's H_G.
  *   dir = KQ_INV: W <- (W V) S_X^-1 (undoes the forward map; H_X untouched).
  * kq_rotate_out (output side, length d_out, sign_u = sigma_U):
  *   dir = KQ_FWD: W <- U (S_G W), and if H_G != NULL: H_G <- U S_G^-1 H_G S_G^-1 U^T.
@@ -197,6 +201,7 @@ KQ_API kq_status kq_biip_stats(const float* W, int64_t d_out, int64_t d_in, cons
 
 #define KQ_FWD 0
 #define KQ_INV 1
+#define KQ_FWD_SYM 2   /* KQ_FWD for a symmetric H_X / H_G (see kq_rotate_in) */
 KQ_API kq_status kq_compute_scales(const float* W, int64_t d_out, int64_t d_in, const float* H_X,
                             const float* H_G, float* s_x, float* s_g, kq_stream_t stream);
 KQ_API kq_status kq_traces(const float* H_X, const float* s_x, int64_t d_in, const float* H_G,

@@ -91,6 +91,168 @@ __global__ void __launch_bounds__(256, HAS28 ? 2 : 4) rht_rows_kernel(float* __r
     }
 }
 
+// ------------------------------------------------------- row transform in registers
+// For n = 2^LG (LG in [9, 14]): T = n / 16 threads per row, 16 values each. Phase q
+// transforms the index bits in rr_mask(LG, q); thread t holds the 16 elements that differ in
+// those bits (value k at the bits of the mask, t spread over the other bits in order).
+// Phase 0 is the thread's 16 contiguous elements, read from global memory with the
+// pre-factor; between phases the values move through shared memory (padded one float in 32:
+// at most four-way bank conflicts, two for n = 4096); the last phase covers the top bits, so
+// consecutive threads write consecutive elements, straight to global memory with the
+// post-factor and 1/sqrt(n). When LG is not a multiple of 4, one phase transforms the few
+// remaining bits and carries some already transformed low bits. Each CTA walks rows
+// r = blockIdx.x, + gridDim.x, ..., loading the next row into registers first.
+__host__ __device__ constexpr int rr_phases(int LG) { return LG / 4 + (LG % 4 ? 1 : 0); }
+__host__ __device__ constexpr uint32_t rr_mask(int LG, int q) {
+    const int nf = LG / 4, rem = LG % 4;
+    if (rem == 0 || q < nf - 1) return 0xFu << (4 * q);
+    const int p = 4 * (nf - 1);
+    if (q == nf - 1) return (((1u << rem) - 1u) << p) | ((1u << (4 - rem)) - 1u);
+    return 0xFu << (p + rem);
+}
+// The k bits (of a 4-bit k deposited into rr_mask(LG, q)) whose index bits phase q is the
+// first to transform.
+__host__ __device__ constexpr uint32_t rr_new_kbits(int LG, int q) {
+    uint32_t before = 0;
+    for (int i = 0; i < q; ++i) before |= rr_mask(LG, i);
+    const uint32_t m = rr_mask(LG, q);
+    uint32_t kb = 0;
+    for (int i = 0, b = 0; i < 32; ++i)
+        if ((m >> i) & 1u) {
+            if (!((before >> i) & 1u)) kb |= 1u << b;
+            ++b;
+        }
+    return kb;
+}
+
+// The low bits of v scattered into the set bits of MASK, in order.
+template <uint32_t MASK>
+__device__ __forceinline__ int deposit_bits(int v) {
+    int out = 0, b = 0;
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+        if ((MASK >> i) & 1u) {
+            out |= ((v >> b) & 1) << i;
+            ++b;
+        }
+    return out;
+}
+
+template <uint32_t KB>
+__device__ __forceinline__ void fwht_kbits(float (&x)[16]) {
+#pragma unroll
+    for (int b = 0; b < 4; ++b)
+        if ((KB >> b) & 1u)
+#pragma unroll
+            for (int i = 0; i < 16; ++i)
+                if ((i & (1 << b)) == 0) {
+                    const float a = x[i], c = x[i | (1 << b)];
+                    x[i] = a + c;
+                    x[i | (1 << b)] = a - c;
+                }
+}
+
+__device__ __forceinline__ int pad32(int j) { return j + (j >> 5); }
+
+// Values of phase Q - 1 to shared memory, those of phase Q back, and phase Q's butterflies.
+template <int LG, int Q>
+__device__ __forceinline__ void rr_transpose(float (&x)[16], float* buf, int t) {
+    constexpr uint32_t N1 = (1u << LG) - 1u;
+    constexpr uint32_t MW = rr_mask(LG, Q - 1), MR = rr_mask(LG, Q);
+    const int tw = deposit_bits<N1 & ~MW>(t), tr = deposit_bits<N1 & ~MR>(t);
+    __syncthreads();   // the previous reads of buf are done
+#pragma unroll
+    for (int k = 0; k < 16; ++k) buf[pad32(tw | deposit_bits<MW>(k))] = x[k];
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < 16; ++k) x[k] = buf[pad32(tr | deposit_bits<MR>(k))];
+    fwht_kbits<rr_new_kbits(LG, Q)>(x);
+}
+
+template <int LG, bool POST>
+__global__ void __launch_bounds__((1 << LG) / 16) rht_rows_reg_kernel(float* __restrict__ M, int64_t rows,
+                                                                      int pre_mode, int post_mode,
+                                                                      const int8_t* __restrict__ sign,
+                                                                      const float* __restrict__ s, float inv_sqrt_n) {
+    constexpr int N = 1 << LG, T = N / 16, NPH = rr_phases(LG);
+    constexpr uint32_t ML = rr_mask(LG, NPH - 1);
+    static_assert(rr_mask(LG, 0) == 0xFu, "phase 0 is the thread's 16 contiguous elements");
+    static_assert(ML >> (LG - 4) == 0xFu, "the last phase covers the top four bits");
+    extern __shared__ __align__(16) float sm_rr[];
+    float* fpre = sm_rr;            // [N]
+    float* fpost = sm_rr + N;       // [N], times 1/sqrt(n)
+    float* buf = sm_rr + 2 * N;     // [N + N / 32]
+    const int t = threadIdx.x;
+    for (int j = t; j < N; j += T) {
+        fpre[j] = factor(pre_mode, sign, s, j);
+        fpost[j] = factor(post_mode, sign, s, j) * inv_sqrt_n;
+    }
+    auto load = [&](int64_t row, float (&v)[16]) {
+        const float4* src = reinterpret_cast<const float4*>(M + row * N + 16 * t);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const float4 a = src[q];
+            v[4 * q] = a.x;
+            v[4 * q + 1] = a.y;
+            v[4 * q + 2] = a.z;
+            v[4 * q + 3] = a.w;
+        }
+    };
+    float x[16], nx[16];
+    int64_t r = blockIdx.x;
+    if (r < rows) load(r, x);
+    __syncthreads();   // factors ready
+    const int tl = deposit_bits<((1u << LG) - 1u) & ~ML>(t);
+    for (; r < rows; r += gridDim.x) {
+        if (r + gridDim.x < rows) load(r + gridDim.x, nx);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const float4 f = reinterpret_cast<const float4*>(fpre + 16 * t)[q];
+            x[4 * q] *= f.x;
+            x[4 * q + 1] *= f.y;
+            x[4 * q + 2] *= f.z;
+            x[4 * q + 3] *= f.w;
+        }
+        fwht_kbits<0xFu>(x);
+        rr_transpose<LG, 1>(x, buf, t);
+        if constexpr (NPH > 2) rr_transpose<LG, 2>(x, buf, t);
+        if constexpr (NPH > 3) rr_transpose<LG, 3>(x, buf, t);
+        float* dst = M + r * N;
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+            const int j = tl | deposit_bits<ML>(k);
+            dst[j] = POST ? x[k] * fpost[j] : x[k] * inv_sqrt_n;
+        }
+#pragma unroll
+        for (int k = 0; k < 16; ++k) x[k] = nx[k];
+    }
+}
+
+// M [n x n] <- M^T in place: the CTA at (bj, bi) of an nt x nt grid of 64 x 64 tiles swaps
+// tiles (bi, bj) and (bj, bi) through shared memory when bi <= bj (a diagonal tile is
+// transposed alone); the CTAs below the diagonal have nothing to do. Each of the 256
+// threads has 16 loads of each tile in flight before the barrier.
+constexpr int TT = 64;
+__global__ void __launch_bounds__(256) transpose_sq_kernel(float* __restrict__ M, int64_t n) {
+    __shared__ float a[TT][TT + 1], b[TT][TT + 1];
+    const int64_t bi = blockIdx.y, bj = blockIdx.x;
+    if (bi > bj) return;
+    const int tx = threadIdx.x & 63, ty = threadIdx.x >> 6;   // 64 x 4
+    for (int yy = ty; yy < TT; yy += 4) {
+        const int64_t r1 = bi * TT + yy, c1 = bj * TT + tx;
+        a[yy][tx] = (r1 < n && c1 < n) ? M[r1 * n + c1] : 0.0f;
+        const int64_t r2 = bj * TT + yy, c2 = bi * TT + tx;
+        if (bi != bj) b[yy][tx] = (r2 < n && c2 < n) ? M[r2 * n + c2] : 0.0f;
+    }
+    __syncthreads();
+    for (int yy = ty; yy < TT; yy += 4) {
+        const int64_t r1 = bj * TT + yy, c1 = bi * TT + tx;   // tile (bj, bi) <- a^T
+        if (r1 < n && c1 < n) M[r1 * n + c1] = a[tx][yy];
+        const int64_t r2 = bi * TT + yy, c2 = bj * TT + tx;   // tile (bi, bj) <- b^T
+        if (bi != bj && r2 < n && c2 < n) M[r2 * n + c2] = b[tx][yy];
+    }
+}
+
 // --------------------------------------------------------------- column transform
 // One radix stage along the row index of M [n x ncols]: for every group base = hi*R*S + lo
 // (lo < S) and CW-column strip, rows base + i*S (i < R) are transformed along i by H_R
@@ -450,10 +612,51 @@ int log2i(int64_t x) {
     return k;
 }
 
+template <int LG>
+kq_status launch_rows_reg(float* M, int64_t rows, int pre, int post, const int8_t* sign, const float* s,
+                          cudaStream_t stream) {
+    constexpr int N = 1 << LG, T = N / 16;
+    constexpr size_t smem = (3 * static_cast<size_t>(N) + N / 32) * sizeof(float);
+    static bool attr = false;
+    if (!attr) {
+        KQ_CUDA(cudaFuncSetAttribute(rht_rows_reg_kernel<LG, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     static_cast<int>(smem)));
+        KQ_CUDA(cudaFuncSetAttribute(rht_rows_reg_kernel<LG, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     static_cast<int>(smem)));
+        attr = true;
+    }
+    // as many CTAs as fit on an SM by shared memory and threads, each walking rows
+    const int64_t per_sm = std::max<int64_t>(1, std::min<int64_t>(static_cast<int64_t>((227 * 1024) / smem), 2048 / T));
+    const int64_t grid = std::min<int64_t>(rows, static_cast<int64_t>(num_sms()) * per_sm);
+    const float isn = static_cast<float>(1.0 / sqrt(static_cast<double>(N)));
+    if (post == F_NONE)
+        rht_rows_reg_kernel<LG, false><<<static_cast<unsigned>(grid), T, smem, stream>>>(M, rows, pre, post, sign, s, isn);
+    else
+        rht_rows_reg_kernel<LG, true><<<static_cast<unsigned>(grid), T, smem, stream>>>(M, rows, pre, post, sign, s, isn);
+    KQ_LAUNCH_CHECK("rht_rows_reg_kernel");
+    return KQ_OK;
+}
+
+// n a power of two from 512 to 16384 and M 16-byte aligned: the register row transform.
+bool rows_reg_ok(const float* M, int64_t n) {
+    return n >= 512 && n <= 16384 && (n & (n - 1)) == 0 && (reinterpret_cast<uintptr_t>(M) & 15u) == 0;
+}
+
 kq_status rows_transform(float* M, int64_t rows, int64_t n, int pre, int post, const int8_t* sign,
                          const float* s, cudaStream_t stream) {
     HadamardPlan p;
     if (!plan_of(n, &p)) return KQ_ERR_UNSUPPORTED;
+    if (rows > 0 && rows_reg_ok(M, n)) {
+        switch (log2i(n)) {
+            case 9: return launch_rows_reg<9>(M, rows, pre, post, sign, s, stream);
+            case 10: return launch_rows_reg<10>(M, rows, pre, post, sign, s, stream);
+            case 11: return launch_rows_reg<11>(M, rows, pre, post, sign, s, stream);
+            case 12: return launch_rows_reg<12>(M, rows, pre, post, sign, s, stream);
+            case 13: return launch_rows_reg<13>(M, rows, pre, post, sign, s, stream);
+            case 14: return launch_rows_reg<14>(M, rows, pre, post, sign, s, stream);
+            default: break;
+        }
+    }
     constexpr size_t kMaxSmem = 227 * 1024;
     const size_t row_bytes = static_cast<size_t>(n) * sizeof(float);
     const int dbl = 2 * row_bytes <= kMaxSmem ? 1 : 0;
@@ -530,6 +733,26 @@ kq_status cols_transform(float* M, int64_t n, int64_t ncols, int pre, int post, 
                 M, static_cast<int>(n), ncols, R[st], S[st], log2i(CW), pm, qm, sign, s, ps);
         KQ_LAUNCH_CHECK("rht_cols_kernel");
     }
+    return KQ_OK;
+}
+
+// M <- R M R^T for M [n x n], R = H_n diag(pre) / sqrt(n) (pre from the factor mode). With
+// the register row transform: B = M R^T (rows), B^T = R M^T, its rows give R M^T R^T, and a
+// last transpose gives R M R^T -- four streaming passes instead of a row pass and two
+// column passes; for a symmetric M (sym) R M^T R^T is already R M R^T up to rounding and the
+// last transpose is left out. Otherwise the row and column transforms.
+kq_status two_sided_transform(float* M, int64_t n, int pre, const int8_t* sign, const float* s, bool sym,
+                              cudaStream_t stream) {
+    kq_status st = rows_transform(M, n, n, pre, F_NONE, sign, s, stream);
+    if (st != KQ_OK) return st;
+    if (!rows_reg_ok(M, n)) return cols_transform(M, n, n, pre, F_NONE, sign, s, stream);
+    const dim3 tg(static_cast<unsigned>(cdiv(n, TT)), static_cast<unsigned>(cdiv(n, TT)));
+    transpose_sq_kernel<<<tg, 256, 0, stream>>>(M, n);
+    KQ_LAUNCH_CHECK("transpose_sq_kernel");
+    st = rows_transform(M, n, n, pre, F_NONE, sign, s, stream);
+    if (st != KQ_OK || sym) return st;
+    transpose_sq_kernel<<<tg, 256, 0, stream>>>(M, n);
+    KQ_LAUNCH_CHECK("transpose_sq_kernel");
     return KQ_OK;
 }
 
@@ -636,6 +859,8 @@ extern "C" kq_status kq_rotate_in(float* W, int64_t d_out, int64_t d_in, float* 
                                   const int8_t* sign_v, int dir, kq_stream_t stream_) {
     cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
     HadamardPlan p;
+    const bool sym = dir == KQ_FWD_SYM;
+    if (sym) dir = KQ_FWD;
     if ((!W && !(H_X && dir == KQ_FWD)) || !sign_v || d_in < 1 || (W && d_out < 1) ||
         (dir != KQ_FWD && dir != KQ_INV)) {
         set_error("kq_rotate_in: invalid arguments");
@@ -654,9 +879,7 @@ extern "C" kq_status kq_rotate_in(float* W, int64_t d_out, int64_t d_in, float* 
         }
         if (H_X) {
             // H_X <- V S_X^-1 H_X S_X^-1 V^T: both sides scaled by sigma / s, then H_n twice.
-            st = rows_transform(H_X, d_in, d_in, s_x ? F_SDIV : F_SIGN, F_NONE, sign_v, s_x, stream);
-            if (st != KQ_OK) return st;
-            st = cols_transform(H_X, d_in, d_in, s_x ? F_SDIV : F_SIGN, F_NONE, sign_v, s_x, stream);
+            st = two_sided_transform(H_X, d_in, s_x ? F_SDIV : F_SIGN, sign_v, s_x, sym, stream);
             if (st != KQ_OK) return st;
         }
     } else {
@@ -671,6 +894,8 @@ extern "C" kq_status kq_rotate_out(float* W, int64_t d_out, int64_t d_in, float*
                                    const int8_t* sign_u, int dir, kq_stream_t stream_) {
     cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
     HadamardPlan p;
+    const bool sym = dir == KQ_FWD_SYM;
+    if (sym) dir = KQ_FWD;
     if ((!W && !(H_G && dir == KQ_FWD)) || !sign_u || d_out < 1 || (W && d_in < 1) ||
         (dir != KQ_FWD && dir != KQ_INV)) {
         set_error("kq_rotate_out: invalid arguments");
@@ -688,9 +913,7 @@ extern "C" kq_status kq_rotate_out(float* W, int64_t d_out, int64_t d_in, float*
             if (st != KQ_OK) return st;
         }
         if (H_G) {
-            st = rows_transform(H_G, d_out, d_out, s_g ? F_SDIV : F_SIGN, F_NONE, sign_u, s_g, stream);
-            if (st != KQ_OK) return st;
-            st = cols_transform(H_G, d_out, d_out, s_g ? F_SDIV : F_SIGN, F_NONE, sign_u, s_g, stream);
+            st = two_sided_transform(H_G, d_out, s_g ? F_SDIV : F_SIGN, sign_u, s_g, sym, stream);
             if (st != KQ_OK) return st;
         }
     } else {

@@ -15,7 +15,7 @@ LIB_PATH = os.path.join(_HERE, "libkronq.so")
 
 KQ_OK, KQ_ERR_INVALID_ARG, KQ_ERR_UNSUPPORTED, KQ_ERR_NOT_PD = 0, 1, 2, 3
 KQ_ERR_CUDA, KQ_ERR_TIMEOUT, KQ_ERR_WORKSPACE = 4, 5, 6
-KQ_FWD, KQ_INV = 0, 1
+KQ_FWD, KQ_INV, KQ_FWD_SYM = 0, 1, 2
 KQ_TRAIL_FP32, KQ_TRAIL_3XTF32 = 0, 1
 KQ_SYRK_CHUNK_TOKENS = 512
 

@@ -142,11 +142,11 @@ class LayerPipeline:
         mark()
         with torch.cuda.stream(s):
             self.Wp.copy_(W)
-        kq.kq_rotate_in(self.Wp, self.HX, self.s_x, sign_v, kq.KQ_FWD, stream=s)         # Eq. (biip), V side
+        kq.kq_rotate_in(self.Wp, self.HX, self.s_x, sign_v, kq.KQ_FWD_SYM, stream=s)         # Eq. (biip), V side
         if Xt is not None:
             kq.kq_rotate_in(None, self.D, self.s_x, sign_v, kq.KQ_FWD, stream=s)         # D' = V S^-1 D S^-1 V^T
         kq.kq_rotate_out(self.Wp, None, self.s_g, sign_u, kq.KQ_FWD, stream=s)           # U side
-        kq.kq_rotate_out(None, self.HG, self.s_g, sign_u, kq.KQ_FWD, stream=s)           # H_G, then released
+        kq.kq_rotate_out(None, self.HG, self.s_g, sign_u, kq.KQ_FWD_SYM, stream=s)           # H_G, then released
         mark()
         kq.kq_chol_inv(self.HX, self.damp, self.Lt, self.info[1:2], self.ws_chol, stream=s)  # Alg. 2
         mark()
@@ -182,7 +182,7 @@ class LayerPipeline:
         e_tx.record(s)
         with torch.cuda.stream(s):
             self.Wp.copy_(W)
-        kq.kq_rotate_in(self.Wp, self.HX, self.s_x, sign_v, kq.KQ_FWD, stream=s)
+        kq.kq_rotate_in(self.Wp, self.HX, self.s_x, sign_v, kq.KQ_FWD_SYM, stream=s)
         e_rin.record(s)
         kq.kq_chol_inv(self.HX, self.damp, self.Lt, self.info[1:2], self.ws_chol, stream=s)
         # The low-priority stream starts once the input-side rotation is done: its long
@@ -201,7 +201,7 @@ class LayerPipeline:
         s2.wait_event(e_rin)
         kq.kq_rotate_out(self.Wp, None, self.s_g, sign_u, kq.KQ_FWD, stream=s2)
         e_side.record(s2)
-        kq.kq_rotate_out(None, self.HG, self.s_g, sign_u, kq.KQ_FWD, stream=s2)
+        kq.kq_rotate_out(None, self.HG, self.s_g, sign_u, kq.KQ_FWD_SYM, stream=s2)
         e_hg.record(s2)
         if Xt is not None:
             s.wait_event(e_d)
@@ -236,7 +236,7 @@ class LayerPipeline:
         e_tx.record(main)
         with torch.cuda.stream(main):
             self.Wp.copy_(W)
-        kq.kq_rotate_in(self.Wp, self.HX, self.s_x, sign_v, kq.KQ_FWD, stream=main)
+        kq.kq_rotate_in(self.Wp, self.HX, self.s_x, sign_v, kq.KQ_FWD_SYM, stream=main)
         e_rin.record(main)
         kq.kq_chol_inv(self.HX, self.damp, self.Lt, self.info[1:2], self.ws_chol, stream=main)
         with torch.cuda.stream(side):
@@ -248,7 +248,7 @@ class LayerPipeline:
         side.wait_event(e_rin)
         kq.kq_rotate_out(self.Wp, None, self.s_g, sign_u, kq.KQ_FWD, stream=side)
         e_side.record(side)
-        kq.kq_rotate_out(None, self.HG, self.s_g, sign_u, kq.KQ_FWD, stream=side)
+        kq.kq_rotate_out(None, self.HG, self.s_g, sign_u, kq.KQ_FWD_SYM, stream=side)
         e_hg.record(side)
         main.wait_event(e_side)
         kq.kq_obs_quantize(self.Wp, self.Lt, self.bits, self.group, self.block, self.codes, self.scale,

@@ -104,8 +104,9 @@ def _layer64(cfg):
     return L, HX, HG
 
 
-@pytest.mark.parametrize("d_out,d_in", [(256, 256), (64, 896), (896, 128), (128, 1)])
-def test_scales_traces_rotations(d_out, d_in):
+@pytest.mark.parametrize("d_out,d_in,sym", [(256, 256, False), (64, 896, False), (896, 128, False), (128, 1, False),
+                                            (512, 1024, False), (512, 1024, True), (2048, 512, True)])
+def test_scales_traces_rotations(d_out, d_in, sym):
     cfg = kqsynth.CONFIGS["tiny256"].replace(d_out=d_out, d_in=d_in, T=2048, n_outliers=min(4, d_in))
     L, HX, HG = _layer64(cfg)
     W = L["W"]
@@ -123,8 +124,9 @@ def test_scales_traces_rotations(d_out, d_in):
         assert abs(t[k] - want[name]) <= 1e-5 * abs(want[name]), name
     su, sv = dev(L["sign_u"], torch.int8), dev(L["sign_v"], torch.int8)
     Wp = Wd.clone()
-    K().kq_rotate_in(Wp, HXd, sx, sv, K().KQ_FWD)
-    K().kq_rotate_out(Wp, HGd, sg, su, K().KQ_FWD)
+    fwd = K().KQ_FWD_SYM if sym else K().KQ_FWD
+    K().kq_rotate_in(Wp, HXd, sx, sv, fwd)
+    K().kq_rotate_out(Wp, HGd, sg, su, fwd)
     assert rel_fro(host(Wp), b["W"]) <= 1e-5
     assert rel_fro(host(HXd), b["HX"]) <= 1e-5
     assert rel_fro(host(HGd), b["HG"]) <= 1e-5
@@ -134,7 +136,7 @@ def test_scales_traces_rotations(d_out, d_in):
     assert rel_fro(host(Wp), W) <= 1e-5
 
 
-@pytest.mark.parametrize("n", [2, 32, 1024, 4096, 28, 28 * 64, 28 * 1024, 32768])
+@pytest.mark.parametrize("n", [2, 32, 512, 1024, 2048, 4096, 8192, 16384, 28, 28 * 64, 28 * 1024, 32768])
 def test_rht_matches_dense_hadamard(n):
     """Pure rotation (no scales) of a few rows against the oracle's dense V."""
     rng = np.random.default_rng(n)
