@@ -238,11 +238,19 @@ __global__ void __launch_bounds__(256) transpose_sq_kernel(float* __restrict__ M
     const int64_t bi = blockIdx.y, bj = blockIdx.x;
     if (bi > bj) return;
     const int tx = threadIdx.x & 63, ty = threadIdx.x >> 6;   // 64 x 4
-    for (int yy = ty; yy < TT; yy += 4) {
+    float ra[TT / 4], rb[TT / 4];   // all loads in flight before the shared-memory stores
+#pragma unroll
+    for (int q = 0; q < TT / 4; ++q) {
+        const int yy = ty + 4 * q;
         const int64_t r1 = bi * TT + yy, c1 = bj * TT + tx;
-        a[yy][tx] = (r1 < n && c1 < n) ? M[r1 * n + c1] : 0.0f;
+        ra[q] = (r1 < n && c1 < n) ? M[r1 * n + c1] : 0.0f;
         const int64_t r2 = bj * TT + yy, c2 = bi * TT + tx;
-        if (bi != bj) b[yy][tx] = (r2 < n && c2 < n) ? M[r2 * n + c2] : 0.0f;
+        rb[q] = (bi != bj && r2 < n && c2 < n) ? M[r2 * n + c2] : 0.0f;
+    }
+#pragma unroll
+    for (int q = 0; q < TT / 4; ++q) {
+        a[ty + 4 * q][tx] = ra[q];
+        b[ty + 4 * q][tx] = rb[q];
     }
     __syncthreads();
     for (int yy = ty; yy < TT; yy += 4) {
