@@ -46,8 +46,11 @@ def parse():
     ap.add_argument("--no-graph", action="store_true", help="launch kernels directly instead of replaying a CUDA graph")
     ap.add_argument("--x-chunk-tokens", type=int, default=0,
                     help="token chunk of the H_X accumulation (0: one call)")
-    ap.add_argument("--g-chunk-tokens", type=int, default=32768,
-                    help="token chunk of the H_G accumulation (0: one call)")
+    ap.add_argument("--g-chunk-tokens", type=int, default=0,
+                    help="token chunk of the H_G accumulation with device-resident inputs (0: one call)")
+    ap.add_argument("--e2e-g-chunk-tokens", type=int, default=32768,
+                    help="token chunk of the H_G accumulation on the host path, where each chunk starts "
+                         "as soon as its copy has landed (0: one call)")
     ap.add_argument("--trailing", default="3xtf32", choices=["fp32", "3xtf32"],
                     help="sweep trailing update: fp32-ordered SIMT (bit-exact) or 3xTF32 tensor cores")
     ap.add_argument("--block", default=None, choices=sorted(kqsynth.BLOCKS),
@@ -423,6 +426,10 @@ def run_ours(args):
         Gh = inp["G"].cpu().pin_memory()
         Wh = inp["W"].cpu().pin_memory()
         suh, svh = inp["sign_u"].cpu().pin_memory(), inp["sign_v"].cpu().pin_memory()
+        if args.e2e_g_chunk_tokens != args.g_chunk_tokens:
+            p = LayerPipeline(cfg.d_out, cfg.d_in, cfg.bits, cfg.group, cfg.block, cfg.damp, device=dev,
+                              x_chunk_tokens=args.x_chunk_tokens, g_chunk_tokens=args.e2e_g_chunk_tokens,
+                              trailing=args.trailing, alpha=args.drift, drift_chunk_tokens=args.drift_chunk_tokens)
         ch = torch.empty(p.codes.shape, dtype=p.codes.dtype).pin_memory()
         sh = torch.empty(p.scale.shape, dtype=p.scale.dtype).pin_memory()
         zh = torch.empty(p.zero.shape, dtype=p.zero.dtype).pin_memory()
@@ -451,7 +458,8 @@ def run_ours(args):
                "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
                "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
                "dtype": "bf16 products, f32 accumulate/arithmetic", "data": "synthetic",
-               "config": config_dict(cfg, args.x_chunk_tokens, args.g_chunk_tokens, args.trailing, args.drift),
+               "config": dict(config_dict(cfg, args.x_chunk_tokens, args.g_chunk_tokens, args.trailing, args.drift),
+                              e2e_factor_chunk_tokens={"X": args.x_chunk_tokens, "G": args.e2e_g_chunk_tokens}),
                "stages_ms": stage_ms, "tflops": tflops,
                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
                "launch_mode": "cuda graph replay (one graph per layer, two streams)" if graph is not None
