@@ -78,10 +78,11 @@ class LayerPipeline:
         self.side = torch.cuda.Stream(device=device, priority=lo) if overlap else None
         self.copy = None
         self._ev = [torch.cuda.Event() for _ in range(8)]
-        # when the low-priority stream may start: after H_X ("factor") or after the
-        # input-side rotation ("rotate"); measured on q_proj: GPTQ mode 7.11 ms ("rotate")
-        # against 7.18, with the drift correction 13.76 ms ("factor") against 13.89
-        self.side_after = "rotate" if alpha is None else "factor"
+        # when the low-priority stream may start: at once ("start": H_G's tiles fill the
+        # SMs H_X's last wave leaves idle), after H_X ("factor") or after the input-side
+        # rotation ("rotate"); measured on q_proj: GPTQ mode 6.17 ms ("start") against 6.22
+        # ("rotate"), with the drift correction 13.76 ms ("factor") against 13.89 ("rotate")
+        self.side_after = "start" if alpha is None else "factor"
 
     def _chunks(self, which: str, T: int) -> list[tuple[int, int]]:
         c = self.chunk_tokens[which]
@@ -185,9 +186,10 @@ class LayerPipeline:
         kq.kq_rotate_in(self.Wp, self.HX, self.s_x, sign_v, kq.KQ_FWD_SYM, stream=s)
         e_rin.record(s)
         kq.kq_chol_inv(self.HX, self.damp, self.Lt, self.info[1:2], self.ws_chol, stream=s)
-        # The low-priority stream starts once the input-side rotation is done: its long
-        # tensor-core tiles would otherwise hold the SMs the memory-bound rotation needs.
-        s2.wait_event(e_rin if self.side_after == "rotate" else e_fx)
+        # When the low-priority stream starts (side_after): its long tensor-core tiles hold
+        # SMs the rotation and the Cholesky then wait for.
+        if self.side_after != "start":
+            s2.wait_event(e_rin if self.side_after == "rotate" else e_fx)
         if Xt is not None:
             if xt_ready is not None:
                 s2.wait_event(xt_ready)
