@@ -78,11 +78,11 @@ class LayerPipeline:
         self.side = torch.cuda.Stream(device=device, priority=lo) if overlap else None
         self.copy = None
         self._ev = [torch.cuda.Event() for _ in range(8)]
-        # when the low-priority stream may start: at once ("start": H_G's tiles fill the
-        # SMs H_X's last wave leaves idle), after H_X ("factor") or after the input-side
-        # rotation ("rotate"); measured on q_proj: GPTQ mode 6.17 ms ("start") against 6.22
-        # ("rotate"), with the drift correction 13.76 ms ("factor") against 13.89 ("rotate")
-        self.side_after = "start" if alpha is None else "factor"
+        # when the low-priority stream may start: at once ("start"), after H_X ("factor") or
+        # after the input-side rotation ("rotate"); measured on q_proj, runs alternated:
+        # GPTQ mode 6.28 ms ("rotate") against 6.47 ("start"), with the drift correction
+        # 13.76 ms ("factor") against 13.89 ("rotate")
+        self.side_after = "rotate" if alpha is None else "factor"
 
     def _chunks(self, which: str, T: int) -> list[tuple[int, int]]:
         c = self.chunk_tokens[which]
