@@ -92,83 +92,11 @@ __global__ void __launch_bounds__(256, HAS28 ? 2 : 4) rht_rows_kernel(float* __r
 }
 
 // ------------------------------------------------------- row transform in registers
-// For n = 2^LG (LG in [9, 14]): T = n / 16 threads per row, 16 values each. Phase q
-// transforms the index bits in rr_mask(LG, q); thread t holds the 16 elements that differ in
-// those bits (value k at the bits of the mask, t spread over the other bits in order).
-// Phase 0 is the thread's 16 contiguous elements, read from global memory with the
-// pre-factor; between phases the values move through shared memory (padded one float in 32:
-// at most four-way bank conflicts, two for n = 4096); the last phase covers the top bits, so
-// consecutive threads write consecutive elements, straight to global memory with the
-// post-factor and 1/sqrt(n). When LG is not a multiple of 4, one phase transforms the few
-// remaining bits and carries some already transformed low bits. Each CTA walks rows
+// For n = 2^LG (LG in [9, 14]), the register transform of rht.cuh per row: phase 0 reads
+// the thread's 16 contiguous elements from global memory with the pre-factor (a per-CTA
+// table), the last phase writes straight to global memory (consecutive threads,
+// consecutive elements) with the post-factor and 1/sqrt(n). Each CTA walks rows
 // r = blockIdx.x, + gridDim.x, ..., loading the next row into registers first.
-__host__ __device__ constexpr int rr_phases(int LG) { return LG / 4 + (LG % 4 ? 1 : 0); }
-__host__ __device__ constexpr uint32_t rr_mask(int LG, int q) {
-    const int nf = LG / 4, rem = LG % 4;
-    if (rem == 0 || q < nf - 1) return 0xFu << (4 * q);
-    const int p = 4 * (nf - 1);
-    if (q == nf - 1) return (((1u << rem) - 1u) << p) | ((1u << (4 - rem)) - 1u);
-    return 0xFu << (p + rem);
-}
-// The k bits (of a 4-bit k deposited into rr_mask(LG, q)) whose index bits phase q is the
-// first to transform.
-__host__ __device__ constexpr uint32_t rr_new_kbits(int LG, int q) {
-    uint32_t before = 0;
-    for (int i = 0; i < q; ++i) before |= rr_mask(LG, i);
-    const uint32_t m = rr_mask(LG, q);
-    uint32_t kb = 0;
-    for (int i = 0, b = 0; i < 32; ++i)
-        if ((m >> i) & 1u) {
-            if (!((before >> i) & 1u)) kb |= 1u << b;
-            ++b;
-        }
-    return kb;
-}
-
-// The low bits of v scattered into the set bits of MASK, in order.
-template <uint32_t MASK>
-__device__ __forceinline__ int deposit_bits(int v) {
-    int out = 0, b = 0;
-#pragma unroll
-    for (int i = 0; i < 32; ++i)
-        if ((MASK >> i) & 1u) {
-            out |= ((v >> b) & 1) << i;
-            ++b;
-        }
-    return out;
-}
-
-template <uint32_t KB>
-__device__ __forceinline__ void fwht_kbits(float (&x)[16]) {
-#pragma unroll
-    for (int b = 0; b < 4; ++b)
-        if ((KB >> b) & 1u)
-#pragma unroll
-            for (int i = 0; i < 16; ++i)
-                if ((i & (1 << b)) == 0) {
-                    const float a = x[i], c = x[i | (1 << b)];
-                    x[i] = a + c;
-                    x[i | (1 << b)] = a - c;
-                }
-}
-
-__device__ __forceinline__ int pad32(int j) { return j + (j >> 5); }
-
-// Values of phase Q - 1 to shared memory, those of phase Q back, and phase Q's butterflies.
-template <int LG, int Q>
-__device__ __forceinline__ void rr_transpose(float (&x)[16], float* buf, int t) {
-    constexpr uint32_t N1 = (1u << LG) - 1u;
-    constexpr uint32_t MW = rr_mask(LG, Q - 1), MR = rr_mask(LG, Q);
-    const int tw = deposit_bits<N1 & ~MW>(t), tr = deposit_bits<N1 & ~MR>(t);
-    __syncthreads();   // the previous reads of buf are done
-#pragma unroll
-    for (int k = 0; k < 16; ++k) buf[pad32(tw | deposit_bits<MW>(k))] = x[k];
-    __syncthreads();
-#pragma unroll
-    for (int k = 0; k < 16; ++k) x[k] = buf[pad32(tr | deposit_bits<MR>(k))];
-    fwht_kbits<rr_new_kbits(LG, Q)>(x);
-}
-
 template <int LG, bool POST>
 __global__ void __launch_bounds__((1 << LG) / 16) rht_rows_reg_kernel(float* __restrict__ M, int64_t rows,
                                                                       int pre_mode, int post_mode,

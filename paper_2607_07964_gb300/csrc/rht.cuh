@@ -192,5 +192,120 @@ __device__ __forceinline__ void block_rht_inplace(float* v, int n, int lgP, bool
     }
 }
 
+// ---------------------------------------------------------------------------------------
+// Walsh-Hadamard transform of n = 2^LG values held in registers, 16 per thread (n / 16
+// threads, LG in [9, 14]). Phase q transforms the index bits in rr_mask(LG, q); thread t
+// holds the 16 elements that differ in those bits (value k at the bits of the mask, t
+// spread over the other bits in order). Phase 0 is the thread's 16 contiguous elements;
+// between phases the values move through shared memory (padded one float in 32: at most
+// four-way bank conflicts, two for n = 4096); the last phase covers the top four bits, so
+// consecutive threads hold consecutive elements. When LG is not a multiple of 4, one phase
+// transforms the few remaining bits and carries some already transformed low bits.
+__host__ __device__ constexpr int rr_phases(int LG) { return LG / 4 + (LG % 4 ? 1 : 0); }
+__host__ __device__ constexpr uint32_t rr_mask(int LG, int q) {
+    const int nf = LG / 4, rem = LG % 4;
+    if (rem == 0 || q < nf - 1) return 0xFu << (4 * q);
+    const int p = 4 * (nf - 1);
+    if (q == nf - 1) return (((1u << rem) - 1u) << p) | ((1u << (4 - rem)) - 1u);
+    return 0xFu << (p + rem);
+}
+// The k bits (of a 4-bit k deposited into rr_mask(LG, q)) whose index bits phase q is the
+// first to transform.
+__host__ __device__ constexpr uint32_t rr_new_kbits(int LG, int q) {
+    uint32_t before = 0;
+    for (int i = 0; i < q; ++i) before |= rr_mask(LG, i);
+    const uint32_t m = rr_mask(LG, q);
+    uint32_t kb = 0;
+    for (int i = 0, b = 0; i < 32; ++i)
+        if ((m >> i) & 1u) {
+            if (!((before >> i) & 1u)) kb |= 1u << b;
+            ++b;
+        }
+    return kb;
+}
+
+// The low bits of v scattered into the set bits of MASK, in order.
+template <uint32_t MASK>
+__device__ __forceinline__ int deposit_bits(int v) {
+    int out = 0, b = 0;
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+        if ((MASK >> i) & 1u) {
+            out |= ((v >> b) & 1) << i;
+            ++b;
+        }
+    return out;
+}
+
+template <uint32_t KB>
+__device__ __forceinline__ void fwht_kbits(float (&x)[16]) {
+#pragma unroll
+    for (int b = 0; b < 4; ++b)
+        if ((KB >> b) & 1u)
+#pragma unroll
+            for (int i = 0; i < 16; ++i)
+                if ((i & (1 << b)) == 0) {
+                    const float a = x[i], c = x[i | (1 << b)];
+                    x[i] = a + c;
+                    x[i | (1 << b)] = a - c;
+                }
+}
+
+__device__ __forceinline__ int pad32(int j) { return j + (j >> 5); }
+
+// Values of phase Q - 1 to shared memory, those of phase Q back, and phase Q's butterflies.
+// Every thread of the CTA calls it (two barriers); threads with act false hold no values.
+template <int LG, int Q>
+__device__ __forceinline__ void rr_transpose(float (&x)[16], float* buf, int t, bool act = true) {
+    constexpr uint32_t N1 = (1u << LG) - 1u;
+    constexpr uint32_t MW = rr_mask(LG, Q - 1), MR = rr_mask(LG, Q);
+    const int tw = deposit_bits<N1 & ~MW>(t), tr = deposit_bits<N1 & ~MR>(t);
+    __syncthreads();   // the previous reads of buf are done
+    if (act) {
+#pragma unroll
+        for (int k = 0; k < 16; ++k) buf[pad32(tw | deposit_bits<MW>(k))] = x[k];
+    }
+    __syncthreads();
+    if (act) {
+#pragma unroll
+        for (int k = 0; k < 16; ++k) x[k] = buf[pad32(tr | deposit_bits<MR>(k))];
+        fwht_kbits<rr_new_kbits(LG, Q)>(x);
+    }
+}
+
+// v (shared, n = 2^LG floats, n / 16 <= blockDim.x) <- scale * H_n v in place, by the first
+// n / 16 threads (16 values each, the phases above); buf: n + n / 32 floats of shared scratch.
+// Every thread of the CTA calls it; it starts and ends with a barrier.
+template <int LG>
+__device__ __forceinline__ void reg_fwht_smem(float* v, float* buf, float scale) {
+    constexpr int T = (1 << LG) / 16, NPH = rr_phases(LG);
+    constexpr uint32_t ML = rr_mask(LG, NPH - 1);
+    const int t = threadIdx.x;
+    const bool act = t < T;
+    float x[16];
+    __syncthreads();   // v complete
+    if (act) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const float4 a = reinterpret_cast<const float4*>(v + 16 * t)[q];
+            x[4 * q] = a.x;
+            x[4 * q + 1] = a.y;
+            x[4 * q + 2] = a.z;
+            x[4 * q + 3] = a.w;
+        }
+        fwht_kbits<0xFu>(x);
+    }
+    rr_transpose<LG, 1>(x, buf, t, act);
+    if constexpr (NPH > 2) rr_transpose<LG, 2>(x, buf, t, act);
+    if constexpr (NPH > 3) rr_transpose<LG, 3>(x, buf, t, act);
+    if (act) {
+        const int tl = deposit_bits<((1u << LG) - 1u) & ~ML>(t);
+#pragma unroll
+        for (int k = 0; k < 16; ++k) v[tl | deposit_bits<ML>(k)] = x[k] * scale;   // v was read before the barriers
+    }
+    __syncthreads();
+}
+
+
 }  // namespace
 }  // namespace kq
