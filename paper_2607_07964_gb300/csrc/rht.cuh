@@ -273,39 +273,6 @@ __device__ __forceinline__ void rr_transpose(float (&x)[16], float* buf, int t, 
     }
 }
 
-// v (shared, n = 2^LG floats, n / 16 <= blockDim.x) <- scale * H_n v in place, by the first
-// n / 16 threads (16 values each, the phases above); buf: n + n / 32 floats of shared scratch.
-// Every thread of the CTA calls it; it starts and ends with a barrier.
-template <int LG>
-__device__ __forceinline__ void reg_fwht_smem(float* v, float* buf, float scale) {
-    constexpr int T = (1 << LG) / 16, NPH = rr_phases(LG);
-    constexpr uint32_t ML = rr_mask(LG, NPH - 1);
-    const int t = threadIdx.x;
-    const bool act = t < T;
-    float x[16];
-    __syncthreads();   // v complete
-    if (act) {
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const float4 a = reinterpret_cast<const float4*>(v + 16 * t)[q];
-            x[4 * q] = a.x;
-            x[4 * q + 1] = a.y;
-            x[4 * q + 2] = a.z;
-            x[4 * q + 3] = a.w;
-        }
-        fwht_kbits<0xFu>(x);
-    }
-    rr_transpose<LG, 1>(x, buf, t, act);
-    if constexpr (NPH > 2) rr_transpose<LG, 2>(x, buf, t, act);
-    if constexpr (NPH > 3) rr_transpose<LG, 3>(x, buf, t, act);
-    if (act) {
-        const int tl = deposit_bits<((1u << LG) - 1u) & ~ML>(t);
-#pragma unroll
-        for (int k = 0; k < 16; ++k) v[tl | deposit_bits<ML>(k)] = x[k] * scale;   // v was read before the barriers
-    }
-    __syncthreads();
-}
-
 
 }  // namespace
 }  // namespace kq
