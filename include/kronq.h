@@ -66,6 +66,20 @@ KQ_API int kq_version(void);
 KQ_API uint64_t kq_launch_count(void);
 
 /*
+ * Graph helpers (runtime plumbing, no counterpart in the paper). kq_graph_instantiate: an
+ *   executable graph from a captured graph (cudaGraph_t passed as a pointer), with
+ *   use_node_priority != 0 honouring the priority each kernel node was captured with (the
+ *   capturing stream's): without it every node takes the priority of the stream the graph
+ *   is launched into, and a two-stream schedule loses its ordering between the critical
+ *   path and the side work. *exec receives the cudaGraphExec_t; the caller keeps the graph
+ *   alive while exec is used and destroys exec with kq_graph_exec_destroy.
+ *   kq_graph_launch: one launch of exec on the stream. CUDA errors give KQ_ERR_CUDA.
+ */
+KQ_API kq_status kq_graph_instantiate(void* graph, int use_node_priority, void** exec);
+KQ_API kq_status kq_graph_launch(void* exec, kq_stream_t stream);
+KQ_API kq_status kq_graph_exec_destroy(void* exec);
+
+/*
  * Synchronize `stream`, then read the device error word `info` (may be NULL) and map it:
  * 0 -> KQ_OK, > 0 -> KQ_ERR_NOT_PD (the value is the 1-based index of the first
  * non-positive pivot), < 0 -> the status -info. Resets *info to 0 when `reset` != 0.

@@ -161,6 +161,32 @@ extern "C" int kq_version(void) { return 100; }
 
 extern "C" uint64_t kq_launch_count(void) { return kq::g_launches.load(std::memory_order_relaxed); }
 
+extern "C" kq_status kq_graph_instantiate(void* graph, int use_node_priority, void** exec) {
+    if (!graph || !exec) {
+        kq::set_error("kq_graph_instantiate: invalid arguments");
+        return KQ_ERR_INVALID_ARG;
+    }
+    cudaGraphExec_t e = nullptr;
+    const unsigned long long flags = use_node_priority ? cudaGraphInstantiateFlagUseNodePriority : 0ull;
+    KQ_CUDA(cudaGraphInstantiateWithFlags(&e, static_cast<cudaGraph_t>(graph), flags));
+    *exec = e;
+    return KQ_OK;
+}
+
+extern "C" kq_status kq_graph_launch(void* exec, kq_stream_t stream) {
+    if (!exec) {
+        kq::set_error("kq_graph_launch: invalid arguments");
+        return KQ_ERR_INVALID_ARG;
+    }
+    KQ_CUDA(cudaGraphLaunch(static_cast<cudaGraphExec_t>(exec), reinterpret_cast<cudaStream_t>(stream)));
+    return KQ_OK;
+}
+
+extern "C" kq_status kq_graph_exec_destroy(void* exec) {
+    if (exec) KQ_CUDA(cudaGraphExecDestroy(static_cast<cudaGraphExec_t>(exec)));
+    return KQ_OK;
+}
+
 extern "C" kq_status kq_check(int* info, int reset, int* pivot_out, kq_stream_t stream_) {
     cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
     KQ_CUDA(cudaStreamSynchronize(stream));

@@ -709,7 +709,7 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
     // but the far update shares the SMs with the block kernel.
     const bool fuse = narrow;
     auto trailing = [&](int64_t i0, int kb, int64_t cb, int64_t ce, cudaStream_t st) -> kq_status {
-        if (tc) return trail_tc(maps, W, d_out, d_in, i0, cb, ce, hp, narrow, info, st);
+        if (tc) return trail_tc(maps, W, d_out, d_in, i0, cb, ce, hp, narrow, kb, info, st);
         dim3 grid(static_cast<unsigned>(cdiv(ce - cb, GT)), static_cast<unsigned>(cdiv(d_out, GT)));
         if (vec)
             trailing_kernel<true><<<grid, G_THREADS, G_SMEM, st>>>(W, o.E, Lt, d_out, d_in, i0, kb, cb, ce, o.Q, Pt);
@@ -718,15 +718,9 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
         KQ_LAUNCH_CHECK("trailing_kernel");
         return KQ_OK;
     };
-    for (int64_t i0 = 0; i0 < d_in; i0 += BLK) {
-        const int64_t b = i0 / BLK;
-        const int kb = static_cast<int>(std::min<int64_t>(BLK, d_in - i0));
+    auto block_launch = [&](int64_t b, const float* rq) {
+        const int64_t i0 = b * BLK;
         const float* rp = o.Rp + b * BLK * BLK;
-        const float* rq = fuse && b > 0 ? o.Rq + (b - 1) * BLK * BLK : nullptr;
-        if (fuse && far_pending[b & 1]) {   // the far update of block b - 2
-            KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[b & 1], 0));
-            far_pending[b & 1] = false;
-        }
         if (hp)
             obs_block_kernel<true, true><<<static_cast<unsigned>(row_ctas), OBS_THREADS_P, 2 * BLK * BLK * 4, stream>>>(
                 W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q, o.Eh, o.El,
@@ -739,37 +733,89 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
             obs_block_kernel<false, false><<<static_cast<unsigned>(row_ctas), OBS_THREADS, BLK * BLK * 4, stream>>>(
                 W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q, o.Eh, o.El,
                 nullptr, nullptr, nullptr, nullptr, rq);
-        KQ_LAUNCH_CHECK("obs_block_kernel");
-        const int64_t nb0 = i0 + kb;                                // next block column
-        if (nb0 >= d_in) break;
-        const int64_t nb1 = std::min<int64_t>(d_in, nb0 + BLK);    // columns beyond it: [nb1, d_in)
-        const bool fork = side && nb1 < d_in;
-        if (fork) KQ_CUDA(cudaEventRecord(side->ev[0], stream));           // E of this block ready
-        kq_status st;
-        if (!fuse) {
-            if (forked) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));  // previous far update done
-            st = trailing(i0, kb, nb0, nb1, stream);
-            if (st != KQ_OK) return st;
-        }
-        if (nb1 < d_in) {
+    };
+    if (fuse && tc) {
+        // Pairs of blocks (2s, 2s + 1). Block 2s + 1 applies block 2s's update of its columns
+        // itself; after the pair, its update (K = 256, still applied 128 of K at a time) of
+        // the next pair's columns runs on the caller's stream just before the next pair,
+        // and that of the columns beyond on the side stream beside the next pair. The
+        // next-pair update waits for the side update of the pair before (it wrote the same
+        // columns); the side updates alternate two events.
+        bool rest_pending[2] = {false, false};
+        for (int64_t b = 0; b < nblk; ++b) {
+            const int64_t i0 = b * BLK;
+            const int64_t pr = b / 2;
+            kq_status st;
+            if ((b & 1) == 0 && b >= 2) {
+                if (rest_pending[pr & 1]) {   // the side update of pair pr - 2
+                    KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[pr & 1], 0));
+                    rest_pending[pr & 1] = false;
+                }
+                st = trailing(i0 - 2 * BLK, 2 * BLK, i0, std::min<int64_t>(d_in, i0 + 2 * BLK), stream);
+                if (st != KQ_OK) return st;
+            }
+            block_launch(b, (b & 1) ? o.Rq + (b - 1) * BLK * BLK : nullptr);
+            KQ_LAUNCH_CHECK("obs_block_kernel");
+            if ((b & 1) == 0) continue;
+            const int64_t nb2 = std::min<int64_t>(d_in, i0 + 3 * BLK);   // beyond the next pair
+            if (nb2 >= d_in) continue;
             cudaStream_t fs = stream;
-            if (fork) {
+            if (side) {
+                KQ_CUDA(cudaEventRecord(side->ev[0], stream));   // E of the pair ready
                 KQ_CUDA(cudaStreamWaitEvent(side->s, side->ev[0], 0));
                 fs = side->s;
             }
-            st = trailing(i0, kb, nb1, d_in, fs);
+            st = trailing(i0 - BLK, 2 * BLK, nb2, d_in, fs);
             if (st != KQ_OK) return st;
-            if (fork) {
-                KQ_CUDA(cudaEventRecord(fuse ? side->ev2[b & 1] : side->ev[1], side->s));
-                if (fuse)
-                    far_pending[b & 1] = true;
-                else
-                    forked = true;
+            if (side) {
+                KQ_CUDA(cudaEventRecord(side->ev2[pr & 1], side->s));
+                rest_pending[pr & 1] = true;
             }
         }
+        for (int q = 0; q < 2; ++q)
+            if (rest_pending[q]) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[q], 0));
+    } else {
+        for (int64_t i0 = 0; i0 < d_in; i0 += BLK) {
+            const int64_t b = i0 / BLK;
+            const int kb = static_cast<int>(std::min<int64_t>(BLK, d_in - i0));
+            const float* rq = fuse && b > 0 ? o.Rq + (b - 1) * BLK * BLK : nullptr;
+            if (fuse && far_pending[b & 1]) {   // the far update of block b - 2
+                KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[b & 1], 0));
+                far_pending[b & 1] = false;
+            }
+            block_launch(b, rq);
+            KQ_LAUNCH_CHECK("obs_block_kernel");
+            const int64_t nb0 = i0 + kb;                                // next block column
+            if (nb0 >= d_in) break;
+            const int64_t nb1 = std::min<int64_t>(d_in, nb0 + BLK);    // columns beyond it: [nb1, d_in)
+            const bool fork = side && nb1 < d_in;
+            if (fork) KQ_CUDA(cudaEventRecord(side->ev[0], stream));           // E of this block ready
+            kq_status st;
+            if (!fuse) {
+                if (forked) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));  // previous far update done
+                st = trailing(i0, kb, nb0, nb1, stream);
+                if (st != KQ_OK) return st;
+            }
+            if (nb1 < d_in) {
+                cudaStream_t fs = stream;
+                if (fork) {
+                    KQ_CUDA(cudaStreamWaitEvent(side->s, side->ev[0], 0));
+                    fs = side->s;
+                }
+                st = trailing(i0, kb, nb1, d_in, fs);
+                if (st != KQ_OK) return st;
+                if (fork) {
+                    KQ_CUDA(cudaEventRecord(fuse ? side->ev2[b & 1] : side->ev[1], side->s));
+                    if (fuse)
+                        far_pending[b & 1] = true;
+                    else
+                        forked = true;
+                }
+            }
+        }
+        for (int q = 0; q < 2; ++q)
+            if (far_pending[q]) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[q], 0));
     }
-    for (int q = 0; q < 2; ++q)
-        if (far_pending[q]) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[q], 0));
     if (forked) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));
     if (col_loss) {
         colloss_kernel<<<static_cast<unsigned>(cdiv(d_in, CS_X)), dim3(CS_X, CS_Y), 0, stream>>>(o.E, d_out, d_in, col_loss);

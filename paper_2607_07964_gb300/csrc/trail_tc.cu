@@ -53,7 +53,8 @@ __device__ __forceinline__ bool wait_quiet(uint64_t* bar, uint32_t parity) {
 
 // Which output tiles a launch updates, and from which operand maps.
 //   mode 0 (the sweep): a row x column grid over W[:, cb:], K slabs at columns i0 + 32 s of
-//     the first pair (E with R) and, for slabs >= 4, of the second pair (-Wpre with P).
+//     the first pair (E with R) and, for slabs >= pslab, at i0 + 32 (s - pslab) of the second
+//     pair (-Wpre with P).
 //   mode 1 (a Cholesky update, see chol.cu): first the A region -- lower tiles (i, j) with
 //     j in [a_j0, a_j1) and i >= j, output A, B operand from the split C rows j -- then the
 //     B region -- tiles (i, j) with i in [b_i0, b_i1), j < b_j1, output Z, B operand from the
@@ -62,7 +63,7 @@ __device__ __forceinline__ bool wait_quiet(uint64_t* bar, uint32_t parity) {
 struct TileSet {
     int mode;
     int n_tiles;
-    int n_col_tiles, cb, i0;                          // mode 0
+    int n_col_tiles, cb, i0, pslab;                   // mode 0
     int nbk, a_j0, a_j1, n_a, b_i0, b_i1, b_j1, kx;   // mode 1
 };
 
@@ -188,9 +189,9 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
                     uint8_t* base = smem + st * C::STAGE;
                     // slabs 0..3: E and R; slabs 4..7 (with P): -Wpre and P. Cholesky tiles
                     // with j <= k take B from the second pair.
-                    const bool second = ts.mode == 0 && s >= TNSLAB;
+                    const bool second = ts.mode == 0 && s >= ts.pslab;
                     const bool bsec = second || alt;
-                    const int x = xk + (second ? s - TNSLAB : s) * TBK;
+                    const int x = xk + (second ? s - ts.pslab : s) * TBK;
                     tma_load_2d(base, second ? &mQh : &mEh, &full[st], x, r0);
                     tma_load_2d(base + A_SLAB, second ? &mQl : &mEl, &full[st], x, r0);
                     tma_load_2d(base + 2 * A_SLAB, bsec ? &mPh : &mRh, &full[st], x, c0);
@@ -407,7 +408,7 @@ kq_status TrailMaps::set_w(float* W, int64_t d_out, int64_t d_in) {
 namespace {
 template <int BN>
 kq_status launch_trail(const TrailMaps& m, const CUtensorMap& rh, const CUtensorMap& rl, int64_t d_out, int64_t i0,
-                       int64_t cb, int64_t ce, bool with_p, int* info, cudaStream_t stream) {
+                       int64_t cb, int64_t ce, bool with_p, int kslabs, int* info, cudaStream_t stream) {
     using Cfg = TrailCfg<BN, 2>;
     static bool attr = false;
     if (!attr) {
@@ -424,16 +425,19 @@ kq_status launch_trail(const TrailMaps& m, const CUtensorMap& rh, const CUtensor
     ts.n_col_tiles = n_col;
     ts.cb = static_cast<int>(cb);
     ts.i0 = static_cast<int>(i0);
+    ts.pslab = with_p ? kslabs : 1 << 30;
+    // the accumulator goes into W every 128 of K (one block's update at a time, as the
+    // per-block schedule does); with P after the E and P halves of one block together
     trail_tc_kernel<BN, 2><<<static_cast<unsigned>(std::min(ts.n_tiles, num_sms())), T_THREADS, Cfg::SMEM, stream>>>(
         m.eh, m.el, rh, rl, with_p ? m.qh : m.eh, with_p ? m.ql : m.el, with_p ? m.ph : rh, with_p ? m.pl : rl, m.w, m.w,
-        ts, with_p ? 2 * TNSLAB : TNSLAB, with_p ? 2 * TNSLAB : TNSLAB, info);
+        ts, with_p ? 2 * kslabs : kslabs, with_p ? 2 * kslabs : TNSLAB, info);
     KQ_LAUNCH_CHECK("trail_tc_kernel");
     return KQ_OK;
 }
 }  // namespace
 
 kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, int64_t i0, int64_t cb, int64_t ce,
-                   bool with_p, bool narrow, int* info, cudaStream_t stream) {
+                   bool with_p, bool narrow, int kb, int* info, cudaStream_t stream) {
     // Persistent: at most one CTA per SM, each walking the tiles t, t + grid, ... (column
     // tile fastest, so the CTAs running together share row and column operands in L2). A
     // range either is a whole number of tiles or ends at d_in (the TMA copies clip the last
@@ -445,8 +449,12 @@ kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, in
         set_error("trailing update: column range [%lld, %lld) is not whole tiles", (long long)cb, (long long)ce);
         return KQ_ERR_INVALID_ARG;
     }
-    if (narrow) return launch_trail<64>(m, m.rh64, m.rl64, d_out, i0, cb, ce, false, info, stream);
-    return launch_trail<128>(m, m.rh_narrow, m.rl_narrow, d_out, i0, cb, ce, with_p, info, stream);
+    if ((kb != 128 && kb != 256) || (with_p && kb != 128)) {
+        set_error("trailing update: K must be 128 or (GPTQ mode) 256, got %d", kb);
+        return KQ_ERR_INVALID_ARG;
+    }
+    if (narrow) return launch_trail<64>(m, m.rh64, m.rl64, d_out, i0, cb, ce, false, kb / TBK, info, stream);
+    return launch_trail<128>(m, m.rh_narrow, m.rl_narrow, d_out, i0, cb, ce, with_p, kb / TBK, info, stream);
 }
 
 // ------------------------------------------------------------ Cholesky step updates

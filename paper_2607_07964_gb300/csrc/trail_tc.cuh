@@ -77,11 +77,12 @@ kq_status chol_update_tc(const CholTcMaps& m, int set, int nbk, int a_j0, int a_
 // hi = src rounded to tf32, lo = src - hi (n elements).
 kq_status split_tf32(const float* src, int64_t n, float* hi, float* lo, cudaStream_t stream);
 
-// W[:, cb:ce] -= E[:, i0:i0+128] R[i0:i0+128, cb:ce] (R[k][c] = Lt[c][k]) on tensor cores,
-// and with_p: also -= Q[:, i0:i0+128] P[i0:i0+128, cb:ce] (P[k][c] = Pt[c][k]). Tiles are
-// 128 x 64 when narrow (GPTQ mode only; 129 KB of shared memory per CTA), else 128 x 128
-// (193 KB); [cb, ce) must be whole tiles or end at d_in. W is the one set_w was given.
+// W[:, cb:ce] -= E[:, i0:i0+kb] R[i0:i0+kb, cb:ce] (R[k][c] = Lt[c][k]) on tensor cores,
+// and with_p: also -= Q[:, i0:i0+kb] P[i0:i0+kb, cb:ce] (P[k][c] = Pt[c][k]). kb = 128, or
+// 256 in GPTQ mode (two blocks' updates in one launch, still applied 128 of K at a time).
+// Tiles are 128 x 64 when narrow (GPTQ mode only; 129 KB of shared memory per CTA), else
+// 128 x 128 (193 KB); [cb, ce) must be whole tiles or end at d_in. W is the one set_w was given.
 kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, int64_t i0, int64_t cb, int64_t ce,
-                   bool with_p, bool narrow, int* info, cudaStream_t stream);
+                   bool with_p, bool narrow, int kb, int* info, cudaStream_t stream);
 
 }  // namespace kq

@@ -42,6 +42,9 @@ def lib() -> ctypes.CDLL:
             "kq_status_name": ([I], ctypes.c_char_p),
             "kq_version": ([], I),
             "kq_launch_count": ([], ctypes.c_uint64),
+            "kq_graph_instantiate": ([P, I, P], I),
+            "kq_graph_launch": ([P, P], I),
+            "kq_graph_exec_destroy": ([P], I),
             "kq_check": ([P, I, P, P], I),
             "kq_selftest_timeout": ([P, I64, P], I),
             "kq_selftest_div": ([P, P, I64, P, P], I),
@@ -137,6 +140,23 @@ def kq_selftest_timeout(info, limit_us: int, stream=None) -> None:
     """A kernel whose bounded wait runs out (nothing arrives); *info gets -KQ_ERR_TIMEOUT."""
     _need(info, "info", torch.int32)
     _ok(lib().kq_selftest_timeout(_ptr(info), int(limit_us), _stream(stream)), "kq_selftest_timeout")
+
+
+def kq_graph_instantiate(graph: int, use_node_priority: bool = True) -> int:
+    """cudaGraphExec_t (as an int) for the cudaGraph_t `graph`, honouring the captured
+    per-node priorities when use_node_priority."""
+    ex = ctypes.c_void_p()
+    _ok(lib().kq_graph_instantiate(ctypes.c_void_p(graph), int(use_node_priority), ctypes.byref(ex)),
+        "kq_graph_instantiate")
+    return int(ex.value)
+
+
+def kq_graph_launch(exec_: int, stream=None) -> None:
+    _ok(lib().kq_graph_launch(ctypes.c_void_p(exec_), _stream(stream)), "kq_graph_launch")
+
+
+def kq_graph_exec_destroy(exec_: int) -> None:
+    _ok(lib().kq_graph_exec_destroy(ctypes.c_void_p(exec_)), "kq_graph_exec_destroy")
 
 
 def kq_selftest_div(a, b, mismatches, stream=None) -> None:

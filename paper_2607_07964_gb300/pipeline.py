@@ -15,6 +15,23 @@ STAGES = ("factor_x", "factor_g", "scales_traces", "rotate", "chol", "sweep")
 STAGES_DRIFT = ("factor_x", "drift", "factor_g", "scales_traces", "rotate", "chol", "p", "sweep")
 
 
+class PriorityGraph:
+    """A captured torch graph (keep_graph=True) instantiated by the library with its
+    per-node priorities; replay() launches it on the current stream."""
+
+    def __init__(self, g):
+        self.g = g   # keeps the captured graph and its memory pool alive
+        self.exec = kq.kq_graph_instantiate(g.raw_cuda_graph(), True)
+
+    def replay(self) -> None:
+        kq.kq_graph_launch(self.exec, torch.cuda.current_stream())
+
+    def __del__(self):
+        if getattr(self, "exec", None):
+            kq.kq_graph_exec_destroy(self.exec)
+            self.exec = None
+
+
 class LayerPipeline:
     """Device buffers for one layer shape and the stage sequence that fills them."""
 
@@ -262,15 +279,25 @@ class LayerPipeline:
 
     def capture(self, X, G, W, sign_u, sign_v, Xt=None) -> tuple:
         """Record one layer (both streams) as a CUDA graph on these fixed buffers. Returns
-        (graph, kernels per replay). Run run() once first so one-time set-up is done."""
+        (graph, kernels per replay); graph.replay() launches it on the current stream. Run
+        run() once first so one-time set-up is done. The graph is instantiated with the
+        priorities its kernels were captured with (critical path above side work), where
+        this PyTorch exposes the captured graph."""
         from . import kronq as _kq
         torch.cuda.synchronize()
-        g = torch.cuda.CUDAGraph()
+        try:
+            g = torch.cuda.CUDAGraph(keep_graph=True)
+        except TypeError:
+            g = None
+        plain = g is None
+        if plain:
+            g = torch.cuda.CUDAGraph()
         cap = torch.cuda.Stream(device=self.HX.device)
         n0 = _kq.launch_count()
         with torch.cuda.graph(g, stream=cap):
             self.run(X, G, W, sign_u, sign_v, stream=cap, Xt=Xt)
-        return g, _kq.launch_count() - n0
+        n = _kq.launch_count() - n0
+        return (g if plain else PriorityGraph(g)), n
 
     def check(self, stream=None) -> None:
         """Raise if a kernel reported a device-side error (timeout, non-PD pivot)."""
