@@ -388,6 +388,30 @@ def test_pipeline_overlap_matches_serial():
         assert np.array_equal(out[0][k], out[1][k]), k
 
 
+def test_pipeline_graph_replay_matches_direct_run():
+    """The layer captured as a CUDA graph and instantiated with its node priorities
+    (kq_graph_instantiate) gives the same bits as the direct two-stream run."""
+    from paper_2607_07964_gb300.pipeline import LayerPipeline, PriorityGraph
+    cfg = kqsynth.CONFIGS["tiny256"].replace(d_out=512, d_in=1024, bits=4, group=128, T=4096, w_bf16=True)
+    L = kqsynth.layer(cfg)
+    X, G, W = bf16_dev(L["X"]), bf16_dev(L["G"]), dev(L["W"])
+    su, sv = dev(L["sign_u"], torch.int8), dev(L["sign_v"], torch.int8)
+    p = LayerPipeline(cfg.d_out, cfg.d_in, cfg.bits, cfg.group, cfg.block, cfg.damp)
+    p.run(X, G, W, su, sv)
+    p.check()
+    want = {k: host(getattr(p, k)) for k in ("codes", "scale", "zero", "Lt", "traces", "col_loss")}
+    g, n = p.capture(X, G, W, su, sv)
+    assert isinstance(g, PriorityGraph) and n > 0
+    p.codes.zero_()
+    p.Lt.zero_()
+    for _ in range(2):
+        g.replay()
+    torch.cuda.synchronize()
+    p.check()
+    for k, v in want.items():
+        assert np.array_equal(host(getattr(p, k)), v), k
+
+
 @pytest.mark.parametrize("overlap", [True, False])
 def test_pipeline_host_path_matches_device_path(overlap):
     """run_host (host buffers, chunked copies overlapped with the factor accumulation)
