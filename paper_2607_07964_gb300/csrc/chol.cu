@@ -40,6 +40,17 @@
 namespace kq {
 namespace {
 
+// D (+)= A B for one m16n8k8 tf32 tile: A 16 x 8 (a0 (g, t), a1 (g + 8, t), a2 (g, t + 4),
+// a3 (g + 8, t + 4)), B 8 x 8 (b0 (t, g), b1 (t + 4, g)), D 16 x 8 (d0 (g, 2t), d1 (g, 2t + 1),
+// d2 (g + 8, 2t), d3 (g + 8, 2t + 1)); g = lane / 4, t = lane % 4. Operands are fp32 bit
+// patterns (the tensor core reads their tf32 part).
+__device__ __forceinline__ void mma_tf32(float (&d)[4], const uint32_t (&a)[4], const uint32_t (&b)[2]) {
+    asm volatile("mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+                 "{%0, %1, %2, %3};"
+                 : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+                 : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+
 constexpr int NB = 128;
 
 constexpr int SPB = 8;                          // blocks per super-panel
@@ -395,6 +406,12 @@ constexpr size_t STRIP_SMEM = smax(smax(Strip<128, 32, true>::SMEM, Strip<32, 12
 // B + c ld + k, col_j = tx + 16 j; BNL = true: B(k, c) at B + k ld + c, col_j = CN tx + j.
 // All global reads finish before the function returns (the output may alias an input
 // row or column strip of this CTA).
+// The products run on the tensor cores: mma.sync m16n8k8 in tf32 with the 3xTF32 split
+// (A_lo B_hi + A_hi B_lo + A_hi B_hi, fp32 accumulation), each of the 8 warps owning a
+// 16 x 32 block of the BM x BNc output (BM BNc = 8 x 512 for the three strip shapes); the
+// fragments are read from the padded shared-memory operands (row stride SLD = 132: the 32
+// lanes of a fragment load hit 32 banks), and the results go back through shared memory
+// into the layout above.
 template <int BM, int BNc, bool BNL>
 __device__ __forceinline__ void strip_gemm(const float* __restrict__ A, const float* __restrict__ B, int64_t ld,
                                            float (&acc)[BM / 16][BNc / 16], float* sm) {
@@ -423,10 +440,17 @@ __device__ __forceinline__ void strip_gemm(const float* __restrict__ A, const fl
         }
         cp_async_commit();
     }
+    const int lane = tid & 31, wid = tid >> 5, g = lane >> 2, t4 = lane & 3;
+    constexpr int WC = BNc / 32;                 // warp columns of 32
+    static_assert((BM / 16) * WC == G_THREADS / 32, "8 warps of 16 x 32");
+    const int wr = wid / WC, wc = wid % WC;
+    float c[4][4];
 #pragma unroll
-    for (int i = 0; i < RM; ++i)
+    for (int nt = 0; nt < 4; ++nt)
 #pragma unroll
-        for (int j = 0; j < CN; ++j) acc[i][j] = 0.0f;
+        for (int e = 0; e < 4; ++e) c[nt][e] = 0.0f;
+    const float* arow0 = As + (16 * wr + g) * SLD;
+    const float* arow1 = arow0 + 8 * SLD;
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
         if (h == 0)
@@ -435,58 +459,47 @@ __device__ __forceinline__ void strip_gemm(const float* __restrict__ A, const fl
             cp_async_wait<0>();
         __syncthreads();
 #pragma unroll 2
-        for (int k4 = h * (SK / 8); k4 < (h + 1) * (SK / 8); ++k4) {
-            float4 a[RM];
+        for (int ks = h * (SK / 2); ks < (h + 1) * (SK / 2); ks += 8) {
+            const float a[4] = {arow0[ks + t4], arow1[ks + t4], arow0[ks + t4 + 4], arow1[ks + t4 + 4]};
+            uint32_t ah[4], al[4];
 #pragma unroll
-            for (int i = 0; i < RM; ++i) a[i] = *reinterpret_cast<const float4*>(As + (ty + 16 * i) * SLD + 4 * k4);
-            if (!BNL) {
+            for (int e = 0; e < 4; ++e) {
+                const float hi = tf32_hi(a[e]);
+                ah[e] = __float_as_uint(hi);
+                al[e] = __float_as_uint(a[e] - hi);
+            }
 #pragma unroll
-                for (int j = 0; j < CN; ++j) {
-                    const float4 b = *reinterpret_cast<const float4*>(Bs + (tx + 16 * j) * SLD + 4 * k4);
-#pragma unroll
-                    for (int i = 0; i < RM; ++i) {
-                        acc[i][j] = fmaf(a[i].x, b.x, acc[i][j]);
-                        acc[i][j] = fmaf(a[i].y, b.y, acc[i][j]);
-                        acc[i][j] = fmaf(a[i].z, b.z, acc[i][j]);
-                        acc[i][j] = fmaf(a[i].w, b.w, acc[i][j]);
-                    }
-                }
-            } else {
-#pragma unroll
-                for (int kk = 0; kk < 4; ++kk) {
-                    const float* brow = Bs + (4 * k4 + kk) * BLD + CN * tx;
-                    float bv[CN];
-                    if constexpr (CN % 4 == 0) {
-#pragma unroll
-                        for (int j4 = 0; j4 < CN / 4; ++j4) {
-                            const float4 t = *reinterpret_cast<const float4*>(brow + 4 * j4);
-                            bv[4 * j4] = t.x;
-                            bv[4 * j4 + 1] = t.y;
-                            bv[4 * j4 + 2] = t.z;
-                            bv[4 * j4 + 3] = t.w;
-                        }
-                    } else {
-                        static_assert(CN == 2, "strip width");
-                        const float2 t = *reinterpret_cast<const float2*>(brow);
-                        bv[0] = t.x;
-                        bv[1] = t.y;
-                    }
-#pragma unroll
-                    for (int i = 0; i < RM; ++i) {
-                        const float av = kk == 0 ? a[i].x : kk == 1 ? a[i].y : kk == 2 ? a[i].z : a[i].w;
-#pragma unroll
-                        for (int j = 0; j < CN; ++j) acc[i][j] = fmaf(av, bv[j], acc[i][j]);
-                    }
-                }
+            for (int nt = 0; nt < 4; ++nt) {
+                const int n = 32 * wc + 8 * nt + g;
+                const float b0 = BNL ? Bs[(ks + t4) * BLD + n] : Bs[n * SLD + ks + t4];
+                const float b1 = BNL ? Bs[(ks + t4 + 4) * BLD + n] : Bs[n * SLD + ks + t4 + 4];
+                const float bh0 = tf32_hi(b0), bh1 = tf32_hi(b1);
+                const uint32_t bh[2] = {__float_as_uint(bh0), __float_as_uint(bh1)};
+                const uint32_t bl[2] = {__float_as_uint(b0 - bh0), __float_as_uint(b1 - bh1)};
+                mma_tf32(c[nt], al, bh);
+                mma_tf32(c[nt], ah, bl);
+                mma_tf32(c[nt], ah, bh);
             }
         }
     }
+    __syncthreads();   // every warp is done with As and Bs
+    constexpr int CLD = BNc + 4;
+    float* Cs = sm;    // [BM][CLD], within As and Bs
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt) {
+        const int r = 16 * wr + g, col = 32 * wc + 8 * nt + 2 * t4;
+        Cs[r * CLD + col] = c[nt][0];
+        Cs[r * CLD + col + 1] = c[nt][1];
+        Cs[(r + 8) * CLD + col] = c[nt][2];
+        Cs[(r + 8) * CLD + col + 1] = c[nt][3];
+    }
+    __syncthreads();
+#pragma unroll
+    for (int i = 0; i < RM; ++i)
+#pragma unroll
+        for (int j = 0; j < CN; ++j) acc[i][j] = Cs[(ty + 16 * i) * CLD + (BNL ? CN * tx + j : tx + 16 * j)];
 }
 
-// --------------------------------------------------------------------- panel
-// CTA (b, s), b < k: column strip s (32 columns) of Z_kb <- C_kk^-1 Z_kb.
-// CTA (b, s), b >= k: row strip s (32 rows) of A_ik <- A_ik C_kk^-T, i = b + 1.
-// Each CTA reads and writes only its own strip, so the in-place update is race-free.
 __global__ void __launch_bounds__(G_THREADS, 2) chol_panel_kernel(Work w, int64_t npad, int k) {
     extern __shared__ __align__(16) float sm[];
     const int b = blockIdx.x, s = blockIdx.y;
