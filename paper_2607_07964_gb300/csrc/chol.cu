@@ -17,7 +17,8 @@
 // block k + 1, on the caller's stream, on the critical path) and the rest (on a library
 // side stream, beside step k + 1's diagonal factorization and panel); step k + 1's own
 // first tiles wait for that rest, which also writes them.
-// The diagonal, panel and first-tile kernels are fp32 SIMT with fused multiply-add. The
+// The diagonal kernel is fp32 SIMT with fused multiply-add; the panel and first-tile
+// kernels multiply on the tensor cores (mma.sync tf32 with the 3xTF32 split). The
 // rest of each update (the bulk of the 2 n^3 / 3 flops) runs on the tensor cores with the
 // 3xTF32 split (trail_tc.cu, Cholesky mode): chol_split_kernel writes the tf32 hi / lo of
 // the panel C_{.k} and of Z_{k.} transposed (the K-major operands), then the persistent
