@@ -41,17 +41,6 @@
 namespace kq {
 namespace {
 
-// D (+)= A B for one m16n8k8 tf32 tile: A 16 x 8 (a0 (g, t), a1 (g + 8, t), a2 (g, t + 4),
-// a3 (g + 8, t + 4)), B 8 x 8 (b0 (t, g), b1 (t + 4, g)), D 16 x 8 (d0 (g, 2t), d1 (g, 2t + 1),
-// d2 (g + 8, 2t), d3 (g + 8, 2t + 1)); g = lane / 4, t = lane % 4. Operands are fp32 bit
-// patterns (the tensor core reads their tf32 part).
-__device__ __forceinline__ void mma_tf32(float (&d)[4], const uint32_t (&a)[4], const uint32_t (&b)[2]) {
-    asm volatile("mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
-                 "{%0, %1, %2, %3};"
-                 : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-                 : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
-}
-
 constexpr int NB = 128;
 
 constexpr int SPB = 8;                          // blocks per super-panel

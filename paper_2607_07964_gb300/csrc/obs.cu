@@ -109,6 +109,9 @@ constexpr int OBS_ROWS = 32;                // rows per CTA
 constexpr int OBS_THREADS = OBS_ROWS * LPR; // 256 or 512
 // With P the CTA holds both diagonal blocks (R and P, 128 KB): one CTA per SM, alone.
 constexpr int OBS_ROWS_P = 32;
+// Dynamic shared memory of the block kernel with the tensor-core fused update: R's block
+// and 32 rows of E_prev (padded), 80.5 KB -- still beside a 129 KB far-update CTA.
+constexpr int OBS_SMEM_MMA = (BLK * BLK + 32 * (BLK + 4)) * 4;
 constexpr int OBS_THREADS_P = OBS_ROWS_P * LPR;
 
 // Packed layout of one diagonal block of R: row j holds R[i0 + j][i0 + c] at pos(c). The
@@ -135,6 +138,72 @@ __global__ void pack_r_kernel(const float* __restrict__ Lt, int64_t n, float* __
         const int j = j0 + r, c = c0 + threadIdx.x;
         out[j * BLK + pos_of(c)] = t[threadIdx.x][r];
     }
+}
+
+// Rq[b][c][k ^ (4 (c & 7))] = R[i0 + k][i1 + c] = Lt[i1 + c][i0 + k] (0 outside the matrix),
+// i0 = b BLK, i1 = i0 + BLK: the block of R right of diagonal block b, column-major with
+// the k index swizzled within 32-float groups, for the tensor-core form of the fused update
+// (its fragment loads then hit 32 banks). Block (32, 8), one 32 x 32 tile per CTA; Lt rows
+// are contiguous in k, so no transpose.
+__global__ void pack_rq_mma_kernel(const float* __restrict__ Lt, int64_t n, float* __restrict__ Rq) {
+    const int64_t i0 = static_cast<int64_t>(blockIdx.z) * BLK, i1 = i0 + BLK;
+    const int k0 = blockIdx.x * 32, c0 = blockIdx.y * 32;
+    float* out = Rq + static_cast<int64_t>(blockIdx.z) * BLK * BLK;
+    for (int r = threadIdx.y; r < 32; r += 8) {
+        const int c = c0 + r, k = k0 + threadIdx.x;
+        const int64_t lr = i1 + c, lc = i0 + k;
+        out[c * BLK + (k ^ (4 * (c & 7)))] = (lr < n && lc < n) ? Lt[lr * n + lc] : 0.0f;
+    }
+}
+
+// The previous block's lazy update of this block column for the CTA's 32 rows on the tensor
+// cores (mma.sync m16n8k8 tf32, 3xTF32 split): C = E_prev R_prev,this with E_prev staged in
+// Es ([32][BLK + 4]) and R_prev,this in Rs (pack_rq_mma_kernel's layout); 8 warps of 16 x 32.
+// C is left in Es (same layout) after a barrier.
+__device__ __forceinline__ void prev_block_update_mma(float* Es, const float* Rs) {
+    constexpr int ESLD = BLK + 4;
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, g = lane >> 2, t4 = lane & 3;
+    const int wr = wid >> 2, wc = wid & 3;
+    float c[4][4];
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) c[nt][e] = 0.0f;
+    const float* a0p = Es + (16 * wr + g) * ESLD;
+    const float* a1p = a0p + 8 * ESLD;
+#pragma unroll 2
+    for (int ks = 0; ks < BLK; ks += 8) {
+        const float a[4] = {a0p[ks + t4], a1p[ks + t4], a0p[ks + t4 + 4], a1p[ks + t4 + 4]};
+        uint32_t ah[4], al[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float hi = tf32_hi(a[e]);
+            ah[e] = __float_as_uint(hi);
+            al[e] = __float_as_uint(a[e] - hi);
+        }
+#pragma unroll
+        for (int nt = 0; nt < 4; ++nt) {
+            const int col = 32 * wc + 8 * nt + g;   // col & 7 == g
+            const float b0 = Rs[col * BLK + ((ks + t4) ^ (4 * g))];
+            const float b1 = Rs[col * BLK + ((ks + t4 + 4) ^ (4 * g))];
+            const float bh0 = tf32_hi(b0), bh1 = tf32_hi(b1);
+            const uint32_t bh[2] = {__float_as_uint(bh0), __float_as_uint(bh1)};
+            const uint32_t bl[2] = {__float_as_uint(b0 - bh0), __float_as_uint(b1 - bh1)};
+            mma_tf32(c[nt], al, bh);
+            mma_tf32(c[nt], ah, bl);
+            mma_tf32(c[nt], ah, bh);
+        }
+    }
+    __syncthreads();   // every warp is done with Es
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt) {
+        const int r = 16 * wr + g, col = 32 * wc + 8 * nt + 2 * t4;
+        Es[r * ESLD + col] = c[nt][0];
+        Es[r * ESLD + col + 1] = c[nt][1];
+        Es[(r + 8) * ESLD + col] = c[nt][2];
+        Es[(r + 8) * ESLD + col + 1] = c[nt][3];
+    }
+    __syncthreads();
 }
 
 __device__ __forceinline__ float group_min(float v) {
@@ -226,7 +295,7 @@ __global__ void __launch_bounds__(HASP ? OBS_THREADS_P : OBS_THREADS, HASP ? 1 :
     uint8_t* __restrict__ codes, float* __restrict__ scale, int32_t* __restrict__ zero,
     float* __restrict__ E, float* __restrict__ pre_q, float* __restrict__ Eh, float* __restrict__ El,
     const float* __restrict__ Pp, float* __restrict__ Q, float* __restrict__ Qh, float* __restrict__ Ql,
-    const float* __restrict__ Rq) {
+    const float* __restrict__ Rq, int fused_mma) {
     extern __shared__ __align__(16) float Rs[];   // [BLK][BLK], packed (pack_r_kernel); then P's
     float* Ps = Rs + BLK * BLK;
     const bool fused = !HASP && Rq != nullptr;
@@ -252,13 +321,35 @@ __global__ void __launch_bounds__(HASP ? OBS_THREADS_P : OBS_THREADS, HASP ? 1 :
         // plain loads; then the diagonal block replaces R_prev,this in shared memory.
         cp_async_wait<0>();
         __syncthreads();
-        for (int64_t rw = rw0; rw < d_out; rw += rstride) {
-            const int64_t r = rw + lane / LPR;
-            float ep[CPL];
-            load_cols<VEC>(E, r, d_out, d_in, i0 - BLK, cb, BLK, ep);
+        if (VEC && fused_mma && rstride >= d_out) {
+            // tensor-core form (one row group per CTA: its 32 rows from blockIdx.x * 32)
+            constexpr int ESLD = BLK + 4;
+            float* Es = Rs + BLK * BLK;
+            const int64_t row0 = static_cast<int64_t>(blockIdx.x) * warps * RPW;
+            for (int q = threadIdx.x; q < 32 * (BLK / 4); q += blockDim.x) {
+                const int rr = q / (BLK / 4), c4 = q % (BLK / 4);
+                const bool lv = row0 + rr < d_out;
+                cp_async16(Es + rr * ESLD + 4 * c4, lv ? E + (row0 + rr) * d_in + (i0 - BLK) + 4 * c4 : E, lv ? 16 : 0);
+            }
+            cp_async_commit();
+            cp_async_wait<0>();
+            __syncthreads();
+            prev_block_update_mma(Es, Rs);
+            const int64_t r = rw0 + lane / LPR;
+            const float* cu = Es + (r - row0) * ESLD + cb;
             load_cols<VEC>(W, r, d_out, d_in, i0, cb, nb, w);
-            prev_block_update(Rs, ep, lp, gbase, w);
+#pragma unroll
+            for (int t = 0; t < CPL; ++t) w[t] = __fsub_rn(w[t], cu[t]);
             store_cols<VEC>(W, r, d_out, d_in, i0, cb, nb, w);
+        } else {
+            for (int64_t rw = rw0; rw < d_out; rw += rstride) {
+                const int64_t r = rw + lane / LPR;
+                float ep[CPL];
+                load_cols<VEC>(E, r, d_out, d_in, i0 - BLK, cb, BLK, ep);
+                load_cols<VEC>(W, r, d_out, d_in, i0, cb, nb, w);
+                prev_block_update(Rs, ep, lp, gbase, w);
+                store_cols<VEC>(W, r, d_out, d_in, i0, cb, nb, w);
+            }
         }
         __syncthreads();
         for (int e = threadIdx.x; e < BLK * BLK / 4; e += blockDim.x) cp_async16(Rs + 4 * e, Rp + 4 * e, 16);
@@ -636,7 +727,7 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
     static bool attr = false;
     if (!attr) {
         KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     BLK * BLK * 4));
+                                     OBS_SMEM_MMA));
         KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      BLK * BLK * 4));
         // Whole shared memory on the SM, so that a CTA fits beside a far-update CTA.
@@ -669,12 +760,24 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
                                                                                 zero, o.gscale, o.gzero);
         KQ_LAUNCH_CHECK("rowgrid_kernel");
     }
+    const bool vec = (d_in % 4 == 0) && (reinterpret_cast<uintptr_t>(Lt) % 16 == 0);
+    const bool bvec = (d_in % 16 == 0) && (reinterpret_cast<uintptr_t>(W) % 16 == 0) &&
+                      (reinterpret_cast<uintptr_t>(codes) % 16 == 0);
     const int64_t nblk = cdiv(d_in, BLK);
     const int64_t row_ctas = hp ? std::min<int64_t>(cdiv(d_out, OBS_ROWS_P), static_cast<int64_t>(num_sms()))
                                 : std::min<int64_t>(cdiv(d_out, OBS_ROWS), 2 * static_cast<int64_t>(num_sms()));
     pack_r_kernel<<<dim3(BLK / 32, BLK / 32, static_cast<unsigned>(nblk)), dim3(32, 8), 0, stream>>>(Lt, d_in, o.Rp, 0);
     KQ_LAUNCH_CHECK("pack_r_kernel");
-    if (!hp && nblk > 1 && row_ctas <= static_cast<int64_t>(num_sms()) && d_out * d_in <= (int64_t{24} << 20)) {
+    // the blocks of R right of the diagonal ones, for the fused update: the tensor-core
+    // form's layout in the 3xTF32 mode, the block kernel's own otherwise
+    const bool fuse_ok = !hp && nblk > 1 && row_ctas <= static_cast<int64_t>(num_sms()) &&
+                         d_out * d_in <= (int64_t{24} << 20);
+    const bool mma_fused = fuse_ok && tc && bvec;
+    if (fuse_ok && mma_fused) {
+        pack_rq_mma_kernel<<<dim3(BLK / 32, BLK / 32, static_cast<unsigned>(nblk - 1)), dim3(32, 8), 0, stream>>>(
+            Lt, d_in, o.Rq);
+        KQ_LAUNCH_CHECK("pack_rq_mma_kernel");
+    } else if (fuse_ok) {
         pack_r_kernel<<<dim3(BLK / 32, BLK / 32, static_cast<unsigned>(nblk - 1)), dim3(32, 8), 0, stream>>>(Lt, d_in,
                                                                                                           o.Rq, 1);
         KQ_LAUNCH_CHECK("pack_r_kernel");
@@ -683,9 +786,6 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
         pack_r_kernel<<<dim3(BLK / 32, BLK / 32, static_cast<unsigned>(nblk)), dim3(32, 8), 0, stream>>>(Pt, d_in, o.Pp, 0);
         KQ_LAUNCH_CHECK("pack_r_kernel");
     }
-    const bool vec = (d_in % 4 == 0) && (reinterpret_cast<uintptr_t>(Lt) % 16 == 0);
-    const bool bvec = (d_in % 16 == 0) && (reinterpret_cast<uintptr_t>(W) % 16 == 0) &&
-                      (reinterpret_cast<uintptr_t>(codes) % 16 == 0);
     // GPTQ mode: block b's kernel first applies the previous block's update of its own
     // columns (E_{b-1} R_{b-1,b}, fused), and the update of the columns beyond block b + 1
     // runs on a library side stream beside block b + 1, whose CTAs share the SMs with it.
@@ -694,8 +794,8 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
     // block column b + 1 runs on the caller's stream (the next block kernel waits for it),
     // the columns beyond on the side stream beside block b + 1.
     // Every column receives the block updates in block order either way. The fused update
-    // is fp32 in the trailing update's order in both modes (the far ones are 3xTF32 in the
-    // tensor-core mode).
+    // is fp32 in the trailing update's order in the fp32 mode, and on the tensor cores
+    // (mma.sync, 3xTF32) in the 3xTF32 mode, like the far updates there.
     SideStream* side = nblk > 2 ? side_stream(stream) : nullptr;
     bool forked = false;
     bool far_pending[2] = {false, false};
@@ -724,15 +824,16 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
         if (hp)
             obs_block_kernel<true, true><<<static_cast<unsigned>(row_ctas), OBS_THREADS_P, 2 * BLK * BLK * 4, stream>>>(
                 W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q, o.Eh, o.El,
-                o.Pp + b * BLK * BLK, o.Q, o.Qh, o.Ql, nullptr);
+                o.Pp + b * BLK * BLK, o.Q, o.Qh, o.Ql, nullptr, 0);
         else if (bvec)
-            obs_block_kernel<true, false><<<static_cast<unsigned>(row_ctas), OBS_THREADS, BLK * BLK * 4, stream>>>(
+            obs_block_kernel<true, false><<<static_cast<unsigned>(row_ctas), OBS_THREADS, mma_fused ? OBS_SMEM_MMA : BLK * BLK * 4,
+                                             stream>>>(
                 W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q, o.Eh, o.El,
-                nullptr, nullptr, nullptr, nullptr, rq);
+                nullptr, nullptr, nullptr, nullptr, rq, mma_fused ? 1 : 0);
         else
             obs_block_kernel<false, false><<<static_cast<unsigned>(row_ctas), OBS_THREADS, BLK * BLK * 4, stream>>>(
                 W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q, o.Eh, o.El,
-                nullptr, nullptr, nullptr, nullptr, rq);
+                nullptr, nullptr, nullptr, nullptr, rq, 0);
     };
     if (fuse && tc) {
         // Pairs of blocks (2s, 2s + 1). Block 2s + 1 applies block 2s's update of its columns
