@@ -660,29 +660,17 @@ def run_infer(args):
             wbytes += packed.numel() * 4 + L["scale"].numel() * 4 + L["zero"].numel() * 4
             layers.append(L)
     stream = torch.cuda.current_stream()
-    # A block's decode step in dependency order: q, k, v read the same input (concurrent), then
-    # o, then gate and up (concurrent), then down.
-    phases = [["q", "k", "v"], ["o"], ["gate", "up"], ["down"]]
-    names = [name for name, _, _, _ in spec]
-    lanes = [torch.cuda.Stream(device=dev) for _ in range(3)]
+    # A block's decode step in dependency order, one stream: q, k, v, o, gate, up, down. Each
+    # call's kernels launch as programmatic dependents of the ones before, so every layer's
+    # weights head for L2 while the previous layer finishes.
 
     def call(L, s):
         kq.kq_infer(L["packed"], L["scale"], L["zero"], L["d_out"], L["d_in"], bits, 128, L["s_x"], L["s_g"],
                     L["su"], L["sv"], L["x"], L["y"], L["ws"], stream=s)
 
     def step(s):
-        for blk in range(nb):
-            for ph in phases:
-                if len(ph) == 1:
-                    call(layers[blk * len(names) + names.index(ph[0])], s)
-                    continue
-                ev = torch.cuda.Event()
-                ev.record(s)
-                for i, name in enumerate(ph):
-                    lanes[i].wait_event(ev)
-                    call(layers[blk * len(names) + names.index(name)], lanes[i])
-                for i in range(len(ph)):
-                    s.wait_stream(lanes[i])
+        for L in layers:
+            call(L, s)
 
     for _ in range(args.warmup):
         step(stream)
@@ -715,10 +703,10 @@ def run_infer(args):
                "vs_baseline": None, "dtype": "f32 arithmetic on packed integer codes", "data": "synthetic",
                "config": {"workload": f"Llama-3-8B linear sublayers x {nb} blocks, {bits}-bit codes "
                                       f"({'4-bit lanes' if bits == 3 else 'packed'}), group 128, B = {B}; per block "
-                                      f"q|k|v concurrent, o, gate|up concurrent, down",
+                                      f"q, k, v, o, gate, up, down in order on one stream",
                           "blocks": nb, "bits": bits, "tokens": B,
                           "l2": f"{wbytes / 1e9:.2f} GB of packed weights per step, larger than L2; no flush"},
-               "roofline": {"kernel": "kq_infer (Hadamard in, dequant_gemv_kernel, Hadamard out) over all sublayers",
+               "roofline": {"kernel": "kq_infer (infer_stream_kernel + infer_out_kernel) over all sublayers",
                             "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm,
                             "traffic": None, "peak_source": f"{peak_src} HBM copy",
                             "bytes_per_step": wbytes},

@@ -90,6 +90,12 @@ __device__ __forceinline__ void mix28_rows(const float (&x)[28], Out& out, std::
     (out(R, pm_sum28<kH28.m[R]>(x)), ...);
 }
 
+// Rows BASE .. BASE + sizeof...(R) - 1 of y = H_28 x.
+template <int BASE, typename Out, int... R>
+__device__ __forceinline__ void mix28_rows_at(const float (&x)[28], Out& out, std::integer_sequence<int, R...>) {
+    (out(BASE + R, pm_sum28<kH28.m[BASE + R]>(x)), ...);
+}
+
 template <typename Out>
 __device__ __forceinline__ void mix28(const float (&x)[28], Out out) {
     mix28_rows(x, out, std::make_integer_sequence<int, 28>{});

@@ -65,7 +65,8 @@ def test_pack_roundtrip(bits):
 
 @pytest.mark.parametrize("d_out,d_in,bits,group,B", [
     (256, 256, 4, 0, 1), (512, 896, 3, 128, 3), (1024, 4096, 2, 128, 1), (448, 1024, 8, 128, 8),
-    (224, 512, 4, 128, 5), (4096, 4096, 4, 128, 2)])
+    (224, 512, 4, 128, 5), (4096, 4096, 4, 128, 2), (14336, 512, 4, 128, 1), (512, 4096, 4, 128, 1),
+    (2048, 1024, 3, 128, 1)])
 def test_infer_matches_dense_reverted_layer(d_out, d_in, bits, group, B):
     codes, scale, zero, s_x, s_g, su, sv = _layer(d_out, d_in, bits, group, d_in + bits)
     x = np.random.default_rng(B).standard_normal((B, d_in)).astype(np.float32)
@@ -80,3 +81,49 @@ def test_infer_matches_dense_reverted_layer(d_out, d_in, bits, group, B):
     got = y.cpu().numpy().astype(np.float64)
     for b in range(B):
         assert np.linalg.norm(got[b] - want[b]) <= 1e-5 * np.linalg.norm(want[b]), b
+
+
+@pytest.mark.parametrize("bits,B", [(4, 1), (2, 2)])
+def test_infer_chain_on_one_stream(bits, B):
+    """Three layers back to back on one stream, each reading the previous one's output: the
+    launches overlap their predecessors (programmatic dependent launch), so this checks that
+    x is read only after the layer before has written it. Each layer matches the oracle on
+    the input it was given; a CUDA graph of the chain reproduces the direct run bit for bit."""
+    d = 1024
+    layers = [_layer(d, d, bits, 128, 100 + i) for i in range(3)]
+    dev = []
+    for codes, scale, zero, s_x, s_g, su, sv in layers:
+        packed = torch.empty(K().kq_packed_codes_bytes(d, d, bits) // 4, dtype=torch.int32, device=DEV)
+        K().kq_pack_codes(_dev(codes), bits, packed)
+        dev.append((packed, _dev(scale), _dev(zero), _dev(s_x), _dev(s_g), _dev(su), _dev(sv)))
+    x0 = _dev(np.random.default_rng(7).standard_normal((B, d)).astype(np.float32))
+    ys = [torch.full((B, d), float("nan"), device=DEV) for _ in range(3)]
+    wss = [torch.empty(K().kq_infer_workspace(B, d, d), dtype=torch.uint8, device=DEV) for _ in range(3)]
+
+    def chain(s):
+        inp = x0
+        for i in range(3):
+            p, sc, z, sx, sg, su, sv = dev[i]
+            K().kq_infer(p, sc, z, d, d, bits, 128, sx, sg, su, sv, inp, ys[i], wss[i], stream=s)
+            inp = ys[i]
+
+    torch.cuda.synchronize()
+    chain(torch.cuda.current_stream())
+    torch.cuda.synchronize()
+    got = [y.cpu().numpy().astype(np.float64) for y in ys]
+    inp = x0.cpu().numpy()
+    for i, (codes, scale, zero, s_x, s_g, su, sv) in enumerate(layers):
+        want = ref.infer(codes, scale, zero, 128, s_x, s_g, su, sv, inp)
+        for b in range(B):
+            assert np.linalg.norm(got[i][b] - want[b]) <= 1e-5 * np.linalg.norm(want[b]), (i, b)
+        inp = got[i].astype(np.float32)
+    for y in ys:
+        y.fill_(float("nan"))
+    g = torch.cuda.CUDAGraph()
+    cap = torch.cuda.Stream()
+    with torch.cuda.graph(g, stream=cap):
+        chain(cap)
+    g.replay()
+    torch.cuda.synchronize()
+    for i in range(3):
+        assert np.array_equal(ys[i].cpu().numpy().astype(np.float64), got[i]), i
