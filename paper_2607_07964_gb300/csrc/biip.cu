@@ -553,14 +553,14 @@ kq_status launch_rows_reg(float* M, int64_t rows, int pre, int post, const int8_
                           cudaStream_t stream) {
     constexpr int N = 1 << LG, T = N / 16;
     constexpr size_t smem = (3 * static_cast<size_t>(N) + N / 32) * sizeof(float);
-    static bool attr = false;
-    if (!attr) {
+    static std::atomic<uint64_t> attr{0};
+    KQ_TRY(once_per_device(attr, [&]() -> kq_status {
         KQ_CUDA(cudaFuncSetAttribute(rht_rows_reg_kernel<LG, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(smem)));
         KQ_CUDA(cudaFuncSetAttribute(rht_rows_reg_kernel<LG, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(smem)));
-        attr = true;
-    }
+        return KQ_OK;
+    }));
     // as many CTAs as fit on an SM by shared memory and threads, each walking rows
     const int64_t per_sm = std::max<int64_t>(1, std::min<int64_t>(static_cast<int64_t>((227 * 1024) / smem), 2048 / T));
     const int64_t grid = std::min<int64_t>(rows, static_cast<int64_t>(num_sms()) * per_sm);
@@ -597,14 +597,14 @@ kq_status rows_transform(float* M, int64_t rows, int64_t n, int pre, int post, c
     const size_t row_bytes = static_cast<size_t>(n) * sizeof(float);
     const int dbl = 2 * row_bytes <= kMaxSmem ? 1 : 0;
     const size_t smem = (dbl ? 2 : 1) * row_bytes;
-    static bool attr = false;
-    if (!attr) {
+    static std::atomic<uint64_t> attr{0};
+    KQ_TRY(once_per_device(attr, [&]() -> kq_status {
         KQ_CUDA(cudaFuncSetAttribute(rht_rows_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(kMaxSmem)));
         KQ_CUDA(cudaFuncSetAttribute(rht_rows_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(kMaxSmem)));
-        attr = true;
-    }
+        return KQ_OK;
+    }));
     const int threads = n >= 512 ? 256 : 128;
     // as many CTAs as fit on an SM by shared memory (at most 8), each walking rows
     const int64_t per_sm = std::max<int64_t>(1, std::min<int64_t>(8, static_cast<int64_t>(kMaxSmem / smem)));
@@ -641,14 +641,14 @@ kq_status cols_transform(float* M, int64_t n, int64_t ncols, int pre, int post, 
         done += kb;
     }
     if (p.has28) { R[ns] = 28; S[ns] = p.P; ++ns; }
-    static bool attr = false;
-    if (!attr) {
+    static std::atomic<uint64_t> attr{0};
+    KQ_TRY(once_per_device(attr, [&]() -> kq_status {
         KQ_CUDA(cudaFuncSetAttribute(rht_cols_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      128 * 1024));
         KQ_CUDA(cudaFuncSetAttribute(rht_cols_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      128 * 1024));
-        attr = true;
-    }
+        return KQ_OK;
+    }));
     const float post_scale = static_cast<float>(1.0 / sqrt(static_cast<double>(n)));
     if (ns == 0) {   // n == 1: only the factors apply
         R[0] = 1; S[0] = 1; ns = 1;

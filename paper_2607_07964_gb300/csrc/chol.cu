@@ -662,16 +662,16 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
         kq_status st = maps.init(w.A, w.Z, npad, width, nsets, w.split);
         if (st != KQ_OK) return st;
     }
-    static bool attr = false;
-    if (!attr) {
+    static std::atomic<uint64_t> attr{0};
+    KQ_TRY(once_per_device(attr, [&]() -> kq_status {
         KQ_CUDA(cudaFuncSetAttribute(chol_diag_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(DIAG_SMEM)));
         KQ_CUDA(cudaFuncSetAttribute(chol_panel_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(STRIP_SMEM)));
         KQ_CUDA(cudaFuncSetAttribute(chol_next_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(STRIP_SMEM)));
-        attr = true;
-    }
+        return KQ_OK;
+    }));
     diag_sum_kernel<<<1, 1024, 0, stream>>>(H, n, w.dsum);
     KQ_LAUNCH_CHECK("diag_sum_kernel");
     const int64_t total = npad * npad;

@@ -282,12 +282,12 @@ extern "C" kq_status kq_gptaq_p(const float* Dp, const float* Lt, int64_t n, flo
     float* Rl = reinterpret_cast<float*>(w8 + 3 * mb);
     float* Ah = reinterpret_cast<float*>(w8 + 4 * mb);   // A1 = (D' L) o M_U, split
     float* Al = reinterpret_cast<float*>(w8 + 5 * mb);
-    static bool attr = false;
-    if (!attr) {
+    static std::atomic<uint64_t> attr{0};
+    KQ_TRY(once_per_device(attr, [&]() -> kq_status {
         KQ_CUDA(cudaFuncSetAttribute(gptaq_gemm_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, P_SMEM));
         KQ_CUDA(cudaFuncSetAttribute(gptaq_gemm_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, P_SMEM));
-        attr = true;
-    }
+        return KQ_OK;
+    }));
     const int64_t N = cdiv(n, PBM);
     const int64_t ntiles = N * (N + 1) / 2;
     kq_status st = split_tf32(Dp, n * n, X0, X1, stream);

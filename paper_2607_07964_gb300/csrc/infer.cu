@@ -748,12 +748,12 @@ kq_status launch_out_reg(int64_t B, cudaStream_t st, const float* yp, int d_out,
                          float* y) {
     constexpr int P = 1 << LG, NT = (H28 ? 28 : 1) * P / 16;
     const size_t smem = static_cast<size_t>(H28 ? 28 : 1) * (P + P / 32) * sizeof(float);
-    static bool attr = false;
-    if (!attr) {
+    static std::atomic<uint64_t> attr{0};
+    KQ_TRY(once_per_device(attr, [&]() -> kq_status {
         KQ_CUDA(cudaFuncSetAttribute(infer_out_reg_kernel<LG, H28>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(smem)));
-        attr = true;
-    }
+        return KQ_OK;
+    }));
     KQ_CUDA(launch_dependent(infer_out_reg_kernel<LG, H28>, dim3(static_cast<unsigned>(B)), dim3(NT), smem, st, 1u, yp,
                              d_out, s_g, su, y));
     KQ_LAUNCH_CHECK("infer_out_reg_kernel");
@@ -794,12 +794,12 @@ kq_status launch_stream_b(const StreamPlan& sp, cudaStream_t st, const uint32_t*
                           const int32_t* zero, int d_out, int d_in, int ng, int grouped, const float* s_x,
                           const float* s_g, const int8_t* su, const int8_t* sv, int lgi, int h28i, int lgo, int h28o,
                           const float* x, float* yp, float* y) {
-    static bool attr = false;
-    if (!attr) {
+    static std::atomic<uint64_t> attr{0};
+    KQ_TRY(once_per_device(attr, [&]() -> kq_status {
         KQ_CUDA(cudaFuncSetAttribute(infer_stream_kernel<PB, B>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(kStreamSmemMax)));
-        attr = true;
-    }
+        return KQ_OK;
+    }));
     KQ_CUDA(launch_dependent(infer_stream_kernel<PB, B>, dim3(sp.grid), dim3(IS_WARPS * 32), sp.smem, st, 1u, packed, scale,
                              zero, d_out, d_in, ng, grouped, s_x, sv, lgi, h28i, x, yp, sp.qps, sp.nslot, sp.part_slot,
                              sp.slot_bytes, sp.xp));

@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "../../include/kronq.h"
 
 namespace kq {
@@ -30,6 +32,29 @@ void count_launch();
     } while (0)
 
 inline int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+// Returns from the enclosing function when a kq_status expression is not KQ_OK.
+#define KQ_TRY(expr)                                                    \
+    do {                                                                \
+        const kq_status _s = (expr);                                    \
+        if (_s != KQ_OK) return _s;                                     \
+    } while (0)
+
+// Runs the set-up f (returning kq_status) once for each device it is called with current:
+// kernel attributes such as the dynamic shared-memory limit belong to the device they were
+// set on, so a process that drives several GPUs sets them on each. A failed set-up is
+// tried again on the next call; two threads may both run it (it only repeats idempotent
+// settings).
+template <typename F>
+inline kq_status once_per_device(std::atomic<uint64_t>& done, F&& f) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return f();
+    const uint64_t bit = uint64_t{1} << dev;
+    if (done.load(std::memory_order_acquire) & bit) return KQ_OK;
+    const kq_status s = f();
+    if (s == KQ_OK) done.fetch_or(bit, std::memory_order_acq_rel);
+    return s;
+}
 
 // Number of SMs of the current device (cached per device).
 int num_sms();

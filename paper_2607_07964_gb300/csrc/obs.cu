@@ -724,8 +724,8 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
                   ws_bytes_of(d_out, d_in, mode, hp));
         return KQ_ERR_WORKSPACE;
     }
-    static bool attr = false;
-    if (!attr) {
+    static std::atomic<uint64_t> attr{0};
+    KQ_TRY(once_per_device(attr, [&]() -> kq_status {
         KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      OBS_SMEM_MMA));
         KQ_CUDA(cudaFuncSetAttribute(obs_block_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -741,8 +741,8 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
                                      static_cast<int>(G_SMEM)));
         KQ_CUDA(cudaFuncSetAttribute(trailing_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(G_SMEM)));
-        attr = true;
-    }
+        return KQ_OK;
+    }));
     ObsWs o = carve(ws, d_out, d_in, mode, hp);
     TrailMaps maps;
     if (tc) {

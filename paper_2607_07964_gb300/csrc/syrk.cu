@@ -421,12 +421,12 @@ extern "C" kq_status kq_accum_factor(const uint16_t* A, int64_t T, int64_t d, in
         CUtensorMap tmap;
         kq_status st = make_bf16_map(&tmap, A, d, T, lda, "kq_accum_factor");
         if (st != KQ_OK) return st;
-        static bool attr_set = false;
-        if (!attr_set) {
+        static std::atomic<uint64_t> attr_set{0};
+        KQ_TRY(once_per_device(attr_set, [&]() -> kq_status {
             KQ_CUDA(cudaFuncSetAttribute(syrk_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          SMEM_BYTES));
-            attr_set = true;
-        }
+            return KQ_OK;
+        }));
         const int n_row = static_cast<int>(cdiv(d, BM));
         const int n_col = static_cast<int>(cdiv(d, BN));
         int64_t tiles = 0;
@@ -478,11 +478,11 @@ extern "C" kq_status kq_accum_drift(const uint16_t* Xt, const uint16_t* X, int64
     }
     uint16_t* hi = static_cast<uint16_t*>(ws);
     uint16_t* lo = hi + Tc * d;
-    static bool attr_set = false;
-    if (!attr_set) {
+    static std::atomic<uint64_t> attr_set{0};
+    KQ_TRY(once_per_device(attr_set, [&]() -> kq_status {
         KQ_CUDA(cudaFuncSetAttribute(drift_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES));
-        attr_set = true;
-    }
+        return KQ_OK;
+    }));
     const int n_row = static_cast<int>(cdiv(d, BM));
     const int n_col = static_cast<int>(cdiv(d, BN));
     const int chunk_stages = KQ_SYRK_CHUNK_TOKENS / BK;

@@ -410,13 +410,13 @@ template <int BN>
 kq_status launch_trail(const TrailMaps& m, const CUtensorMap& rh, const CUtensorMap& rl, int64_t d_out, int64_t i0,
                        int64_t cb, int64_t ce, bool with_p, int kslabs, int* info, cudaStream_t stream) {
     using Cfg = TrailCfg<BN, 2>;
-    static bool attr = false;
-    if (!attr) {
+    static std::atomic<uint64_t> attr{0};
+    KQ_TRY(once_per_device(attr, [&]() -> kq_status {
         KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<BN, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
         KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<BN, 2>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                      cudaSharedmemCarveoutMaxShared));
-        attr = true;
-    }
+        return KQ_OK;
+    }));
     const int n_row = static_cast<int>(cdiv(d_out, TBM));
     const int n_col = static_cast<int>(cdiv(ce - cb, BN));
     TileSet ts{};
@@ -474,11 +474,11 @@ kq_status CholTcMaps::init(float* A, float* Z, int64_t npad, int width, int nset
 kq_status chol_update_tc(const CholTcMaps& m, int set, int nbk, int a_j0, int a_j1, int b_i0, int b_i1, int b_j1,
                          int kx, int nslab, int* info, cudaStream_t stream) {
     using Cfg = TrailCfg<128, 2>;
-    static bool attr = false;
-    if (!attr) {
+    static std::atomic<uint64_t> attr{0};
+    KQ_TRY(once_per_device(attr, [&]() -> kq_status {
         KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<128, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
-        attr = true;
-    }
+        return KQ_OK;
+    }));
     TileSet ts{};
     ts.mode = 1;
     ts.nbk = nbk;
