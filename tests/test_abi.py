@@ -117,3 +117,20 @@ def test_host_side_argument_errors(lib):
     assert lib.kq_infer(*args) == K.KQ_ERR_UNSUPPORTED
     assert lib.kq_pack_codes(fake, 4, 200, 4, fake, None) == K.KQ_ERR_UNSUPPORTED
     assert K.kq_packed_codes_bytes(4, 256, 3) == 4 * 256 // 2 and K.kq_packed_codes_bytes(4, 256, 5) == 0
+
+
+def test_no_cpu_fallback(monkeypatch):
+    """The binding has no CPU path: host tensors are refused before any call, and a missing
+    library makes every call raise instead of computing something else."""
+    import torch
+    from paper_2607_07964_gb300 import kronq as K
+    A = torch.zeros((64, 8), dtype=torch.bfloat16)
+    H = torch.zeros((8, 8), dtype=torch.float32)
+    with pytest.raises(ValueError, match="CUDA tensor"):
+        K.kq_accum_factor(A, H)
+    monkeypatch.setattr(K, "_lib", None)
+    monkeypatch.setattr(K, "LIB_PATH", os.path.join(ROOT, "no_such_dir", "libkronq.so"))
+    with pytest.raises(RuntimeError, match="missing"):
+        K.lib()
+    with pytest.raises(RuntimeError, match="missing"):
+        K.kq_chol_inv_workspace(256)
