@@ -797,7 +797,11 @@ extern "C" kq_status kq_chol_inv_noalloc(const float* H, int64_t n, float damp_r
         if (!g_noalloc_ptr[dev]) {
             void* p = nullptr;
             const cudaError_t e = cudaGetSymbolAddress(&p, g_chol_scratch);
-            if (e != cudaSuccess || !p) return cuda_status(e, "cudaGetSymbolAddress(g_chol_scratch)");
+            if (e != cudaSuccess) return cuda_status(e, "cudaGetSymbolAddress(g_chol_scratch)");
+            if (!p) {
+                set_error("kq_chol_inv_noalloc: cudaGetSymbolAddress(g_chol_scratch) gave a null address");
+                return KQ_ERR_CUDA;
+            }
             g_noalloc_ptr[dev] = p;
         }
         ws = g_noalloc_ptr[dev];
