@@ -269,7 +269,9 @@ KQ_API kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, float* L
  *   device allocation, or a latency-bound loop where a cudaMalloc would synchronize the
  *   device. The paper has no counterpart; this is a convenience of this library.
  *   Scratch comes from a fixed array in device memory that the library owns:
- *   2 * KQ_CHOL_NOALLOC_MAX_N^2 * 4 + 256 bytes (8 MiB), held by every device that loads
+ *   KQ_CHOL_NOALLOC_SCRATCH_BYTES = (2 N^2 + 4 N 128) * 4 + 256 bytes with
+ *   N = KQ_CHOL_NOALLOC_MAX_N (the padded matrix and its inverse factor, plus one set of
+ *   four N x 128 tf32 split panels): 10 MiB + 256 bytes, held by every device that loads
  *   the library until the process exits. n > KQ_CHOL_NOALLOC_MAX_N is rejected with
  *   KQ_ERR_WORKSPACE and a message; no allocation is ever made.
  *   The first call on each device looks up the array's device address (cudaGetSymbolAddress,
@@ -279,6 +281,7 @@ KQ_API kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, float* L
  *   on different streams, or from different host threads -- race: serialize them.
  */
 #define KQ_CHOL_NOALLOC_MAX_N 1024
+#define KQ_CHOL_NOALLOC_SCRATCH_BYTES ((2ull * 1024 * 1024 + 4ull * 1024 * 128) * 4 + 256)
 KQ_API kq_status kq_chol_inv_noalloc(const float* H, int64_t n, float damp_rel, float* Lt, int* info,
                                      kq_stream_t stream);
 
@@ -367,6 +370,9 @@ KQ_API kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, const fl
  *   All arithmetic fp32 (codes are exact as floats; per group scale (sum q x' - zero sum x')).
  *   ws: kq_infer_workspace(B, d_in, d_out) bytes, 256-byte aligned. packed, x, y, s_x, s_g
  *   16-byte aligned, the signs 4-byte aligned, d_out % 4 == 0; s_x, s_g required (not NULL). d_in and d_out need Hadamard constructions (2^k or 28 * 2^k).
+ *   info: optional device error word (see kq_check). The weight stream waits on its copies
+ *   with a time limit; a wait that runs out records -KQ_ERR_TIMEOUT there and leaves that
+ *   part of y as NaN.
  * ---------------------------------------------------------------------------------- */
 KQ_API size_t kq_packed_codes_bytes(int64_t d_out, int64_t d_in, int bits);
 KQ_API kq_status kq_pack_codes(const uint8_t* codes, int64_t d_out, int64_t d_in, int bits, uint32_t* packed,
@@ -375,7 +381,7 @@ KQ_API size_t kq_infer_workspace(int64_t B, int64_t d_in, int64_t d_out);
 KQ_API kq_status kq_infer(const uint32_t* packed, const float* scale, const int32_t* zero, int64_t d_out,
                           int64_t d_in, int bits, int group, const float* s_x, const float* s_g,
                           const int8_t* sign_u, const int8_t* sign_v, const float* x, int64_t B, float* y,
-                          void* ws, size_t ws_bytes, kq_stream_t stream);
+                          int* info, void* ws, size_t ws_bytes, kq_stream_t stream);
 
 /* ------------------------------------------------------------------------------------
  * Check-only calls (not part of the timed path).

@@ -42,7 +42,7 @@ from __future__ import annotations
 import numpy as np
 
 __all__ = [
-    "accum_factor", "factor_entries", "factor_diag", "biip_scales_from_diag", "sylvester", "paley28", "hadamard_matrix", "rht_matrix",
+    "accum_factor", "biip_scales_from_diag", "sylvester", "paley28", "hadamard_matrix", "rht_matrix",
     "biip_scales", "biip", "damp", "inverse_cholesky_upper", "lower_factor",
     "quant_params", "quantize", "obs_sweep", "dequant", "revert", "proxy_loss",
     "traces", "pipeline", "drift_factor", "gptaq_p", "objective", "allocate_bits", "block_scores",
@@ -58,32 +58,6 @@ def accum_factor(A: np.ndarray) -> np.ndarray:
     """H = A^T A for A [T, d] with tokens as rows, in float64 (a library matmul)."""
     A = np.asarray(A, dtype=np.float64)
     return A.T @ A
-
-
-def factor_entries(A, pairs) -> np.ndarray:
-    """Selected entries H[i, j] = sum_t A[t, i] A[t, j] of the factor, each a float64 dot
-    product over all tokens (for checking very large factors entry by entry)."""
-    out = np.empty(len(pairs))
-    cache = {}
-
-    def col(j):
-        if j not in cache:
-            cache[j] = np.asarray(A[:, j], dtype=np.float64)
-        return cache[j]
-
-    for k, (i, j) in enumerate(pairs):
-        out[k] = float(np.dot(col(i), col(j)))
-    return out
-
-
-def factor_diag(A, chunk: int = 8192) -> np.ndarray:
-    """diag(A^T A) = per-channel sums of squares in float64, over row chunks."""
-    A = np.asarray(A)
-    acc = np.zeros(A.shape[1])
-    for t0 in range(0, A.shape[0], chunk):
-        blk = np.asarray(A[t0:t0 + chunk], dtype=np.float64)
-        acc += np.einsum("ij,ij->j", blk, blk)
-    return acc
 
 
 def drift_factor(Xt, X) -> np.ndarray:

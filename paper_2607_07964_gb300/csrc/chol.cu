@@ -773,6 +773,8 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
 namespace {
 constexpr size_t kNoallocBytes = kq::ws_bytes_for(KQ_CHOL_NOALLOC_MAX_N);
 static __device__ __align__(256) unsigned char g_chol_scratch[kNoallocBytes];
+static_assert(kNoallocBytes == KQ_CHOL_NOALLOC_SCRATCH_BYTES,
+              "the documented size of the allocation-free scratch array must match the one it has");
 std::mutex g_noalloc_mu;
 void* g_noalloc_ptr[64] = {};
 }  // namespace

@@ -246,11 +246,12 @@ __global__ void __launch_bounds__(IS_WARPS * 32, stream_ctas_per_sm(B)) infer_st
     const uint32_t* __restrict__ packed, const float* __restrict__ scale, const int32_t* __restrict__ zero, int d_out,
     int d_in, int ng, int grouped, const float* __restrict__ s_x, const int8_t* __restrict__ sign_v, int lg_in,
     int has28_in, const float* __restrict__ x, float* __restrict__ yp, int qps, int nslot, int part_slot,
-    int slot_bytes, int xp) {
+    int slot_bytes, int xp, int* info) {
     extern __shared__ __align__(128) uint8_t ism[];
     __shared__ uint64_t full[IS_SLOTS];
     __shared__ int done[IS_SLOTS];
     __shared__ int abort_flag;
+    __shared__ int issued_hi;   // stages whose copies have been issued: [0, issued_hi)
     constexpr int CPW = 32 / PB;   // codes per word
     constexpr int CPC = 4 * CPW;   // codes per 16-byte chunk
     constexpr int NS = byte_words<PB>();
@@ -275,6 +276,7 @@ __global__ void __launch_bounds__(IS_WARPS * 32, stream_ctas_per_sm(B)) infer_st
         for (int k = 0; k < nslot; ++k) mbar_init(&full[k], 1);
         fence_mbar_init();
         abort_flag = 0;
+        issued_hi = 0;
     }
     if (threadIdx.x < IS_SLOTS) done[threadIdx.x] = 0;
     // the weights do not depend on the preceding kernel: ask L2 for them now
@@ -315,6 +317,7 @@ __global__ void __launch_bounds__(IS_WARPS * 32, stream_ctas_per_sm(B)) infer_st
         const int64_t r0 = static_cast<int64_t>(q0) * 4;
         const uint32_t cb = static_cast<uint32_t>(nq * 4 * rowbytes), sb = static_cast<uint32_t>(nq * 4 * ng * 4);
         uint8_t* dst = slots + static_cast<int64_t>(k) * slot_bytes;
+        atomicMax(&issued_hi, t + 1);
         mbar_arrive_expect_tx(&full[k], cb + 2 * sb);
         bulk_g2s(dst, pk + r0 * rowbytes, cb, &full[k]);
         bulk_g2s(dst + codes_bytes, scale + r0 * ng, sb, &full[k]);
@@ -518,9 +521,19 @@ __global__ void __launch_bounds__(IS_WARPS * 32, stream_ctas_per_sm(B)) infer_st
             }
         }
     }
-    // a wait that gave up (the copies never landed): leave y' as NaN for this CTA's rows
+    // A wait that gave up (the copies never landed): report KQ_ERR_TIMEOUT in the device
+    // error word, give the latest stage issued into each slot one more bounded wait, so that
+    // no copy still in flight lands in shared memory after the CTA has exited, and leave y'
+    // as NaN for this CTA's rows.
     __syncthreads();
     if (abort_flag) {
+        if (threadIdx.x == 0) {
+            record_error(info, -KQ_ERR_TIMEOUT);
+            for (int t = max(0, issued_hi - nslot); t < issued_hi; ++t) {
+                int quiet = 0;
+                mbar_wait(&full[t % nslot], static_cast<uint32_t>((t / nslot) & 1), &quiet);
+            }
+        }
         for (int e = threadIdx.x; e < (qb - qa) * 4 * B; e += blockDim.x) {
             const int rl = e / B, b = e - rl * B;
             yp[static_cast<int64_t>(b) * d_out + static_cast<int64_t>(qa) * 4 + rl] = __int_as_float(0x7fc00000);
@@ -793,7 +806,7 @@ template <int PB, int B>
 kq_status launch_stream_b(const StreamPlan& sp, cudaStream_t st, const uint32_t* packed, const float* scale,
                           const int32_t* zero, int d_out, int d_in, int ng, int grouped, const float* s_x,
                           const float* s_g, const int8_t* su, const int8_t* sv, int lgi, int h28i, int lgo, int h28o,
-                          const float* x, float* yp, float* y) {
+                          const float* x, float* yp, float* y, int* info) {
     static std::atomic<uint64_t> attr{0};
     KQ_TRY(once_per_device(attr, [&]() -> kq_status {
         KQ_CUDA(cudaFuncSetAttribute(infer_stream_kernel<PB, B>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -802,7 +815,7 @@ kq_status launch_stream_b(const StreamPlan& sp, cudaStream_t st, const uint32_t*
     }));
     KQ_CUDA(launch_dependent(infer_stream_kernel<PB, B>, dim3(sp.grid), dim3(IS_WARPS * 32), sp.smem, st, 1u, packed, scale,
                              zero, d_out, d_in, ng, grouped, s_x, sv, lgi, h28i, x, yp, sp.qps, sp.nslot, sp.part_slot,
-                             sp.slot_bytes, sp.xp));
+                             sp.slot_bytes, sp.xp, info));
     KQ_LAUNCH_CHECK("infer_stream_kernel");
     return launch_out(B, st, yp, d_out, s_g, su, lgo, h28o, y);
 }
@@ -811,10 +824,10 @@ template <int PB>
 kq_status launch_stream(int64_t B, const StreamPlan& sp, cudaStream_t st, const uint32_t* packed, const float* scale,
                         const int32_t* zero, int d_out, int d_in, int ng, int grouped, const float* s_x,
                         const float* s_g, const int8_t* su, const int8_t* sv, int lgi, int h28i, int lgo, int h28o,
-                        const float* x, float* yp, float* y) {
+                        const float* x, float* yp, float* y, int* info) {
 #define KQ_STREAM_CASE(NB) \
     case NB:               \
-        return launch_stream_b<PB, NB>(sp, st, packed, scale, zero, d_out, d_in, ng, grouped, s_x, s_g, su, sv, lgi, h28i, lgo, h28o, x, yp, y);
+        return launch_stream_b<PB, NB>(sp, st, packed, scale, zero, d_out, d_in, ng, grouped, s_x, s_g, su, sv, lgi, h28i, lgo, h28o, x, yp, y, info);
     switch (B) {
         KQ_STREAM_CASE(1)
         KQ_STREAM_CASE(2)
@@ -911,7 +924,7 @@ extern "C" size_t kq_infer_workspace(int64_t B, int64_t d_in, int64_t d_out) {
 extern "C" kq_status kq_infer(const uint32_t* packed, const float* scale, const int32_t* zero, int64_t d_out,
                               int64_t d_in, int bits, int group, const float* s_x, const float* s_g,
                               const int8_t* sign_u, const int8_t* sign_v, const float* x, int64_t B, float* y,
-                              void* ws, size_t ws_bytes, kq_stream_t stream_) {
+                              int* info, void* ws, size_t ws_bytes, kq_stream_t stream_) {
     cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
     if (!packed || !scale || !zero || !s_x || !s_g || !sign_u || !sign_v || !x || !y || d_out < 1 || d_in < 1 || B < 1 ||
         B > KQ_INFER_MAX_B) {
@@ -948,12 +961,12 @@ extern "C" kq_status kq_infer(const uint32_t* packed, const float* scale, const 
         const int di = static_cast<int>(d_in), dn = static_cast<int>(d_out), gr = group ? 1 : 0;
         if (pb == 2)
             return launch_stream<2>(B, sp, stream, packed, scale, zero, dn, di, ng, gr, s_x, s_g, sign_u, sign_v, lgi, h28i,
-                                    lgo, h28o, x, yp, y);
+                                    lgo, h28o, x, yp, y, info);
         if (pb == 4)
             return launch_stream<4>(B, sp, stream, packed, scale, zero, dn, di, ng, gr, s_x, s_g, sign_u, sign_v, lgi, h28i,
-                                    lgo, h28o, x, yp, y);
+                                    lgo, h28o, x, yp, y, info);
         return launch_stream<8>(B, sp, stream, packed, scale, zero, dn, di, ng, gr, s_x, s_g, sign_u, sign_v, lgi, h28i,
-                                lgo, h28o, x, yp, y);
+                                lgo, h28o, x, yp, y, info);
     }
     // x' = V S_X^-1 x
     KQ_CUDA(cudaMemcpyAsync(xt, x, static_cast<size_t>(B) * d_in * sizeof(float), cudaMemcpyDeviceToDevice, stream));

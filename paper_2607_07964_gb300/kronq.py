@@ -70,7 +70,7 @@ def lib() -> ctypes.CDLL:
             "kq_packed_codes_bytes": ([I64, I64, I], SZ),
             "kq_pack_codes": ([P, I64, I64, I, P, P], I),
             "kq_infer_workspace": ([I64, I64, I64], SZ),
-            "kq_infer": ([P, P, P, I64, I64, I, I, P, P, P, P, P, I64, P, P, SZ, P], I),
+            "kq_infer": ([P, P, P, I64, I64, I, I, P, P, P, P, P, I64, P, P, P, SZ, P], I),
             "kq_gptaq_p_workspace": ([I64], SZ),
             "kq_gptaq_p": ([P, P, I64, F, P, P, P, SZ, P], I),
             "kq_dequant_revert": ([P, P, P, I64, I64, I, P, P, P, P, P, P], I),
@@ -408,9 +408,10 @@ def kq_infer_workspace(B: int, d_in: int, d_out: int) -> int:
 
 
 def kq_infer(packed, scale, zero, d_out: int, d_in: int, bits: int, group: int, s_x, s_g, sign_u, sign_v, x, y,
-             ws, stream=None) -> None:
+             ws, stream=None, info=None) -> None:
     """y [B, d_out] = W^ x for x [B, d_in]: the reverted quantized layer applied with online
-    Hadamard transforms (Algorithm 2's revert, Sec. 3.2)."""
+    Hadamard transforms (Algorithm 2's revert, Sec. 3.2). info: optional int32 device word
+    for a timed-out weight stream (read with kq_check)."""
     B = x.shape[0]
     _need(packed, "packed", torch.int32)
     _need(scale, "scale", torch.float32)
@@ -422,9 +423,10 @@ def kq_infer(packed, scale, zero, d_out: int, d_in: int, bits: int, group: int, 
     _need(x, "x", torch.float32, (B, d_in))
     _need(y, "y", torch.float32, (B, d_out))
     _need(ws, "ws", torch.uint8)
+    _need(info, "info", torch.int32)
     _ok(lib().kq_infer(_ptr(packed), _ptr(scale), _ptr(zero), d_out, d_in, bits, group, _ptr(s_x), _ptr(s_g),
-                       _ptr(sign_u), _ptr(sign_v), _ptr(x), B, _ptr(y), _ptr(ws), 0 if ws is None else ws.numel(),
-                       _stream(stream)), "kq_infer")
+                       _ptr(sign_u), _ptr(sign_v), _ptr(x), B, _ptr(y), _ptr(info), _ptr(ws),
+                       0 if ws is None else ws.numel(), _stream(stream)), "kq_infer")
 
 
 def kq_dequant_revert(codes, scale, zero, group: int, s_x, s_g, sign_u, sign_v, W_hat, stream=None):

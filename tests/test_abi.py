@@ -109,7 +109,7 @@ def test_host_side_argument_errors(lib):
     assert lib.kq_gptaq_p(fake, fake, 6, 0.25, fake, None, fake, 1 << 20, None) == K.KQ_ERR_UNSUPPORTED
     assert lib.kq_gptaq_p(fake, fake, 8, 0.25, fake, None, fake, 16, None) == K.KQ_ERR_WORKSPACE
     # inference: B in 1..8, bits in {2, 3, 4, 8}, d_in a multiple of 128
-    args = [fake, fake, fake, 64, 256, 4, 128, fake, fake, fake, fake, fake, 9, fake, fake, 1 << 20, None]
+    args = [fake, fake, fake, 64, 256, 4, 128, fake, fake, fake, fake, fake, 9, fake, None, fake, 1 << 20, None]
     assert lib.kq_infer(*args) == K.KQ_ERR_INVALID_ARG
     args[12], args[5] = 1, 5
     assert lib.kq_infer(*args) == K.KQ_ERR_UNSUPPORTED

@@ -75,9 +75,11 @@ def test_infer_matches_dense_reverted_layer(d_out, d_in, bits, group, B):
     K().kq_pack_codes(_dev(codes), bits, packed)
     y = torch.full((B, d_out), float("nan"), device=DEV)
     ws = torch.empty(K().kq_infer_workspace(B, d_in, d_out), dtype=torch.uint8, device=DEV)
+    info = torch.zeros(1, dtype=torch.int32, device=DEV)
     K().kq_infer(packed, _dev(scale), _dev(zero), d_out, d_in, bits, group, _dev(s_x), _dev(s_g),
-                 _dev(su), _dev(sv), _dev(x), y, ws)
+                 _dev(su), _dev(sv), _dev(x), y, ws, info=info)
     torch.cuda.synchronize()
+    assert K().kq_check(info)[0] == K().KQ_OK
     got = y.cpu().numpy().astype(np.float64)
     for b in range(B):
         assert np.linalg.norm(got[b] - want[b]) <= 1e-5 * np.linalg.norm(want[b]), b

@@ -17,12 +17,6 @@ import kqsynth
 pytestmark = pytest.mark.gpu
 
 
-def _rel_fro(a, b):
-    a = np.asarray(a, np.float64)
-    b = np.asarray(b, np.float64)
-    return float(np.linalg.norm(a - b) / np.linalg.norm(b))
-
-
 def test_chol_inv_noalloc_matches_workspace_entry_point():
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
@@ -49,10 +43,10 @@ def test_chol_inv_noalloc_matches_workspace_entry_point():
         assert st == K.KQ_OK, K.last_error()
         assert K.kq_check(info_a)[0] == K.KQ_OK
         assert K.kq_check(info_b)[0] == K.KQ_OK
-        a = Lt_a.cpu().numpy()
-        b = Lt_b.cpu().numpy()
-        assert np.all(np.isfinite(b))
-        assert _rel_fro(b, a) <= 1e-5
+        # the same kernels on the same stream with the same scratch layout: the same bits,
+        # so any byte read from the previous call's contents would show
+        assert torch.isfinite(Lt_b).all()
+        assert torch.equal(Lt_a, Lt_b)
 
 
 def test_chol_inv_noalloc_rejects_oversize():
