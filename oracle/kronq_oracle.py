@@ -43,8 +43,8 @@ import numpy as np
 
 __all__ = [
     "accum_factor", "biip_scales_from_diag", "sylvester", "paley28", "hadamard_matrix", "rht_matrix",
-    "biip_scales", "biip", "damp", "inverse_cholesky_upper", "lower_factor",
-    "quant_params", "quantize", "obs_sweep", "dequant", "revert", "proxy_loss",
+    "biip_scales", "biip", "damp", "inverse_cholesky_upper", "lower_factor", "lower_factor_reversed",
+    "quant_params", "quantize", "quantize_f32", "teacher_forced", "obs_sweep", "dequant", "revert", "proxy_loss",
     "traces", "pipeline", "drift_factor", "gptaq_p", "objective", "allocate_bits", "block_scores",
     "block_pipeline", "infer", "biip_scales_exp", "norm_cv", "rho", "prop2_bound",
 ]
@@ -230,6 +230,29 @@ def lower_factor(Hd: np.ndarray) -> np.ndarray:
     return inverse_cholesky_upper(Hd).T
 
 
+def lower_factor_reversed(Hd: np.ndarray, panel: int = 2048) -> np.ndarray:
+    """The same L (H^-1 = L L^T, L lower with a positive diagonal, which is unique) by the
+    cheaper route for large n: the Cholesky factor C of the reversed matrix J H J (J the
+    exchange matrix) gives H = (J C J)(J C J)^T with J C J upper, so H^-1 = R^T R for
+    R = (J C J)^-1, and L = R^T = J C^-T J. Library Cholesky (LAPACK dpotrf), then C^-1 one
+    panel of columns at a time by triangular solves (BLAS dtrsm) on the rows at and below
+    the panel (C^-1 is lower triangular): about 2 n^3 / 3 flops instead of the textbook
+    route's ~3 n^3."""
+    from scipy.linalg import blas, lapack
+    n = np.asarray(Hd).shape[0]
+    A = np.asfortranarray(np.asarray(Hd, dtype=np.float64)[::-1, ::-1])
+    C, info = lapack.dpotrf(A, lower=1, clean=1, overwrite_a=1)
+    if info != 0:
+        raise np.linalg.LinAlgError(f"dpotrf failed ({info})")
+    Ci = np.zeros((n, n), order="F")
+    for j0 in range(0, n, panel):
+        j1 = min(n, j0 + panel)
+        rhs = np.zeros((n - j0, j1 - j0), order="F")
+        rhs[np.arange(j1 - j0), np.arange(j1 - j0)] = 1.0
+        Ci[j0:, j0:j1] = blas.dtrsm(1.0, np.asfortranarray(C[j0:, j0:]), rhs, lower=1, overwrite_b=1)
+    return np.ascontiguousarray(Ci.T[::-1, ::-1])
+
+
 def gptaq_p(Dp: np.ndarray, L: np.ndarray, alpha: float) -> np.ndarray:
     """The GPTAQ correction of Proposition 1 and Algorithm 2:
     P = alpha ((D' L) o M_U) L^T, with D' the rescaled, rotated drift statistic, L the
@@ -312,6 +335,84 @@ def obs_sweep(Wp: np.ndarray, R: np.ndarray, bits: int, group: int, block: int, 
             if P is not None:
                 W[:, e:] += pre_q[:, i:e] @ P[i:e, e:]
     return {"codes": codes, "scale": scale, "zero": zero, "E": E, "pre_q": pre_q}
+
+
+def quantize_f32(w, scale, zero, bits):
+    """The column step's rounding in float32, as Algorithm 2 runs in a float32 sweep:
+    q = clamp(rint(w / scale) + zero, 0, 2^b - 1) with w / scale one correctly rounded
+    float32 division and rint half to even (not rint(w / scale + zero): the two differ at
+    ties when zero is odd)."""
+    w = np.asarray(w, np.float32)
+    scale = np.asarray(scale, np.float32)
+    zero = np.asarray(zero, np.float32)
+    q = np.rint(w / scale) + zero
+    return np.clip(q, np.float32(0), np.float32(2 ** bits - 1)).astype(np.uint8)
+
+
+def _strict_lower64(M) -> np.ndarray:
+    """float64 copy of M with the diagonal and everything above it zeroed (row slabs, so
+    that a large M needs no index arrays)."""
+    out = np.array(M, dtype=np.float64)
+    for i0 in range(0, out.shape[0], 1024):
+        out[i0:i0 + 1024] = np.tril(out[i0:i0 + 1024], i0 - 1)
+    return out
+
+
+def teacher_forced(Wp, Lt, pre_q, codes, scale, zero, bits: int, group: int, block: int = 128, Pt=None) -> dict:
+    """Algorithm 2 replayed on another sweep's own decisions (teacher forcing), for rows of
+    a layer given that sweep's outputs: its pre-quantization values pre_q, codes and grids
+    (float32), the rotated weights W' it started from and Lt = R^T (and Pt = P^T with the
+    GPTAQ correction).
+
+    Each column step fixes the error from the column's own value and code,
+        E_j = (w_j - scale (q_j - zero)) / R_jj           (float32, as the sweep computes it),
+    and every later column then sees the same compensation Algorithm 2 applies (Eq.
+    obs_update, with the lazy block updates summed out):
+        w_j = W'_j - sum_{k < j} E_k R_kj (+ sum_{k < j} w_k P_kj),
+    evaluated here in float64 from those errors. A sweep that computes what Algorithm 2
+    states quantizes, at column j, a value within its float32 rounding of w_j, and its code
+    is exactly the float32 quantization of its own value. Returned:
+      E         the errors (float32),
+      pre_q     w_j in float64,
+      codes     quantize_f32 of the given pre_q on the given grid (what the codes must be),
+      absum     |W'_j| + sum_{k < j} |E_k R_kj| (+ |w_k P_kj|): the scale of w_j's rounding,
+      block_start (group = block) the columns' float64 values at their block's start,
+                W'_c - sum_{k < block start} E_k R_kc (+ P terms), from which the group grid
+                is drawn (Sec. 5.1 grids, group statistics at the block start).
+    Rows are independent given R, so any subset of rows can be passed."""
+    Wp = np.asarray(Wp, np.float64)
+    m, n = Wp.shape
+    pq32 = np.asarray(pre_q, np.float32)
+    sc = np.asarray(scale, np.float32)
+    zr = np.asarray(zero, np.float32)
+    ng = sc.shape[1]
+    gidx = np.zeros(n, np.int64) if group == 0 else np.arange(n) // group
+    s_col = sc[:, gidx] if ng > 1 else np.repeat(sc, n, axis=1)
+    z_col = zr[:, gidx] if ng > 1 else np.repeat(zr, n, axis=1)
+    q = np.asarray(codes, np.float32)
+    diag = np.ascontiguousarray(np.diagonal(np.asarray(Lt, np.float32)))
+    what = s_col * (q - z_col)
+    E = (pq32 - what) / diag[None, :]
+    Ls = _strict_lower64(Lt)                                # R_kj (k < j) at Ls[j, k]
+    E64 = E.astype(np.float64)
+    comp = E64 @ Ls.T                                       # sum_{k < j} E_k R_kj
+    absum = np.abs(Wp) + np.abs(E64) @ np.abs(Ls).T
+    if Pt is not None:
+        Ps = _strict_lower64(Pt)                            # P_kj (k < j) at Ps[j, k]
+        comp -= pq32.astype(np.float64) @ Ps.T
+        absum += np.abs(pq32.astype(np.float64)) @ np.abs(Ps).T
+    out = {"E": E, "pre_q": Wp - comp, "codes": quantize_f32(pq32, s_col, z_col, bits), "absum": absum}
+    if group:
+        # add back the in-block part of the compensation: the values at the block's start
+        bs = out["pre_q"].copy()
+        for i in range(0, n, block):
+            e = min(i + block, n)
+            blk = Ls[i:e, i:e]
+            bs[:, i:e] += E64[:, i:e] @ blk.T
+            if Pt is not None:
+                bs[:, i:e] -= pq32[:, i:e].astype(np.float64) @ Ps[i:e, i:e].T
+        out["block_start"] = bs
+    return out
 
 
 def dequant(codes, scale, zero, group: int) -> np.ndarray:

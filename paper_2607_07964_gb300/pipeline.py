@@ -38,7 +38,8 @@ class LayerPipeline:
     def __init__(self, d_out: int, d_in: int, bits: int, group: int, block: int = 128,
                  damp: float = 0.01, device: str = "cuda", want_col_loss: bool = True,
                  overlap: bool = True, x_chunk_tokens: int = 0, g_chunk_tokens: int = 32768,
-                 trailing: str = "3xtf32", alpha: float | None = None, drift_chunk_tokens: int = 0):
+                 trailing: str = "3xtf32", alpha: float | None = None, drift_chunk_tokens: int = 0,
+                 debug_outputs: bool = False):
         self.d_out, self.d_in, self.bits, self.group, self.block, self.damp = d_out, d_in, bits, group, block, damp
         # GPTAQ drift correction (Prop. 1, Alg. 2) with scaling alpha; None = GPTQ mode
         self.alpha = alpha
@@ -66,6 +67,10 @@ class LayerPipeline:
         self.ws_obs = torch.empty((kq.kq_obs_quantize_workspace(d_out, d_in, block, self.trail_mode,
                                                                 alpha is not None),),
                                   dtype=torch.uint8, device=device)
+        # debug outputs (checks only): the rotated W' as the sweep receives it, and the
+        # sweep's pre-quantization value of every weight (kq_obs_quantize's pre_q)
+        self.Wp_in = torch.empty((d_out, d_in), **f32) if debug_outputs else None
+        self.pre_q = torch.empty((d_out, d_in), **f32) if debug_outputs else None
         if alpha is not None:
             self.D = torch.empty((d_in, d_in), **f32)      # drift statistic, then D'
             self.Pt = torch.empty((d_in, d_in), **f32)
@@ -171,10 +176,17 @@ class LayerPipeline:
         if Xt is not None:
             kq.kq_gptaq_p(self.D, self.Lt, self.alpha, self.Pt, self.ws_p, info=self.info[1:2], stream=s)  # P
             mark()
-        kq.kq_obs_quantize(self.Wp, self.Lt, self.bits, self.group, self.block, self.codes, self.scale,
-                           self.zero, self.col_loss, None, self.ws_obs, stream=s, mode=self.trail_mode,
-                           info=self.info[3:4], Pt=self.Pt if Xt is not None else None)   # Alg. 2 sweep
+        self._sweep(s, Xt is not None)                                                   # Alg. 2 sweep
         mark()
+
+    def _sweep(self, stream, with_p: bool) -> None:
+        """Algorithm 2's sweep on W' (destroyed) with L; the debug copies first if asked."""
+        if self.Wp_in is not None:
+            with torch.cuda.stream(stream):
+                self.Wp_in.copy_(self.Wp)
+        kq.kq_obs_quantize(self.Wp, self.Lt, self.bits, self.group, self.block, self.codes, self.scale,
+                           self.zero, self.col_loss, self.pre_q, self.ws_obs, stream=stream, mode=self.trail_mode,
+                           info=self.info[3:4], Pt=self.Pt if with_p else None)
 
     def _run_overlapped(self, X, G, W, sign_u, sign_v, caller, x_ready=None, g_ready=None, w_ready=None,
                         Xt=None, xt_ready=None) -> None:
@@ -226,9 +238,7 @@ class LayerPipeline:
             s.wait_event(e_d)
             kq.kq_gptaq_p(self.D, self.Lt, self.alpha, self.Pt, self.ws_p, info=self.info[1:2], stream=s)
         s.wait_event(e_side)
-        kq.kq_obs_quantize(self.Wp, self.Lt, self.bits, self.group, self.block, self.codes, self.scale,
-                           self.zero, self.col_loss, None, self.ws_obs, stream=s, mode=self.trail_mode,
-                           info=self.info[3:4], Pt=self.Pt if Xt is not None else None)
+        self._sweep(s, Xt is not None)
         e_out.record(s)
         caller.wait_event(e_out)
         caller.wait_event(e_hg)
@@ -270,9 +280,7 @@ class LayerPipeline:
         kq.kq_rotate_out(None, self.HG, self.s_g, sign_u, kq.KQ_FWD_SYM, stream=side)
         e_hg.record(side)
         main.wait_event(e_side)
-        kq.kq_obs_quantize(self.Wp, self.Lt, self.bits, self.group, self.block, self.codes, self.scale,
-                           self.zero, self.col_loss, None, self.ws_obs, stream=main, mode=self.trail_mode,
-                           info=self.info[3:4])
+        self._sweep(main, False)
         e_out.record(main)
         s.wait_event(e_out)
         s.wait_event(e_hg)

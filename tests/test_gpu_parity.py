@@ -272,34 +272,49 @@ def test_sweep_bit_exact_extreme_rows(group):
     assert np.array_equal(g["pre_q"], c["pre_q"])
 
 
-def _tie_distance(pre_q, scale_row_groups, group, r, j):
-    """|frac(w / scale) - 1/2| of the oracle's value that column j of row r quantizes."""
-    g = 0 if group == 0 else j // group
-    x = np.float64(pre_q[r, j]) / np.float64(scale_row_groups[r, g])
-    return abs((x - np.floor(x)) - 0.5)
+def _synthetic_lt(n, seed):
+    """A lower-triangular L = R^T with a positive diagonal, drawn directly (no n^3 factorization
+    for the large shapes): the sweep is defined for any such factor. Off-diagonal entries
+    N(0, 0.3^2 / n), diagonal 0.5 + U(0, 1)."""
+    rng = np.random.default_rng(seed)
+    Lt = np.tril(rng.standard_normal((n, n), dtype=np.float32) * np.float32(0.3 / np.sqrt(n)), -1)
+    Lt[np.arange(n), np.arange(n)] = (0.5 + rng.random(n)).astype(np.float32)
+    return Lt
 
 
+# (5120, 1024): more row CTAs than SMs; (1024, 24704): d_out d_in above 24M with one CTA
+# per SM: both take the sweep's schedule for large layers (128 x 128 update tiles, block
+# kernel not fused), the one the 8B MLP and 70B layers run.
 @pytest.mark.parametrize("d_out,d_in,bits,group", [
-    (256, 256, 4, 128), (300, 1024, 4, 128), (512, 896, 3, 128), (128, 1536, 2, 0), (200, 640, 8, 128)])
+    (256, 256, 4, 128), (300, 1024, 4, 128), (512, 896, 3, 128), (128, 1536, 2, 0), (200, 640, 8, 128),
+    (5120, 1024, 3, 128), (5120, 1024, 2, 0), (1024, 24704, 2, 128)])
 def test_sweep_tensor_core_trailing(d_out, d_in, bits, group):
-    """3xTF32 trailing update: codes equal the fp32-ordered definition except where a value
-    sits on a rounding tie (and the rest of that row); at most 0.1 % of codes differ."""
-    Wp, Lt = _sweep_inputs(d_out, d_in, seed=d_in + 7 * bits)
+    """3xTF32 trailing update: teacher forced on every row (codes = quant(GPU pre_q) bit for
+    bit; pre_q within float32 rounding of Algorithm 2 from the GPU's own errors; grids from
+    the block-start values), and against the fp32-ordered definition at most 0.1 % of codes
+    differ, each row's first difference at a rounding tie."""
+    from sweep_checks import check_against_fp32_sweep, check_teacher_forced
+    if d_in > 4096:
+        Wp = (np.random.default_rng(d_in).standard_normal((d_out, d_in)) * 0.05).astype(np.float32)
+        Lt = _synthetic_lt(d_in, seed=bits)
+    else:
+        Wp, Lt = _sweep_inputs(d_out, d_in, seed=d_in + 7 * bits)
     g = _gpu_sweep(Wp, Lt, bits, group, mode=K().KQ_TRAIL_3XTF32)
-    c = obs_sweep_fp32(Wp, Lt, bits, group, 128, want_pre_q=True)
-    mis = g["codes"] != c["codes"]
-    assert mis.mean() <= 1e-3, mis.mean()
-    for r in np.where(mis.any(axis=1))[0]:
-        j = int(np.argmax(mis[r]))
-        assert _tie_distance(c["pre_q"], c["scale"], group, r, j) <= 1e-4, (r, j)
-    same = ~mis.any(axis=1)
-    assert np.allclose(g["scale"][same], c["scale"][same], rtol=1e-4, atol=0)
-    # pre-quantization values follow the fp32 definition to the update's rounding level,
+    big = d_out * d_in > (8 << 20)
+    rng = np.random.default_rng(3)
+    tf_rows = np.sort(rng.choice(d_out, 256, replace=False)) if big else None
+    check_teacher_forced(Wp, Lt, g, bits, group, 128, rows=tf_rows)
+    fp_rows = np.sort(rng.choice(d_out, 32, replace=False)) if big or d_out > 1024 else None
+    c, mis = check_against_fp32_sweep(Wp, Lt, g, bits, group, 128, rows=fp_rows)
+    # rows without a flipped code follow the fp32 definition to the update's rounding level,
     # measured in quantization steps (what decides a code)
+    sel = slice(None) if fp_rows is None else fp_rows
+    same = ~mis.any(axis=1)
     ng = c["scale"].shape[1]
-    step = np.repeat(c["scale"], 1 if ng == 1 else 128, axis=1)[:, :d_in] if ng > 1 else c["scale"]
-    dev_steps = np.abs(g["pre_q"] - c["pre_q"]) / step
+    step = np.repeat(c["scale"], 128, axis=1)[:, :d_in] if ng > 1 else c["scale"]
+    dev_steps = np.abs(g["pre_q"][sel] - c["pre_q"]) / step
     assert np.max(dev_steps[same]) <= 1e-4, np.max(dev_steps[same])
+    assert np.allclose(g["scale"][sel][same], c["scale"][same], rtol=1e-4, atol=0)
 
 
 def test_pipeline_tensor_core_trailing_proxy_loss():

@@ -228,6 +228,18 @@ def test_inverse_cholesky_routes_agree():
     assert np.array_equal(ref.lower_factor(H), R.T)
 
 
+@pytest.mark.parametrize("n", [12, 300])
+def test_inverse_cholesky_reversed_route_is_the_textbook_factor(n):
+    """The LAPACK reverse-order route used for the largest layers' checks gives the textbook
+    factor (the lower Cholesky-type factor of H^-1 with a positive diagonal is unique)."""
+    H = ref.damp(kqsynth.random_spd(n, seed=n), 0.01)
+    L = ref.lower_factor(H)
+    Lr = ref.lower_factor_reversed(H)
+    assert np.array_equal(np.triu(Lr, 1), np.zeros_like(Lr)) and np.all(np.diag(Lr) > 0)
+    assert np.allclose(Lr, L, rtol=1e-9, atol=1e-12 * np.abs(L).max())
+    assert np.allclose(Lr @ Lr.T @ H, np.eye(n), atol=1e-8)
+
+
 def test_obs_row_is_inverse_of_remaining_block():
     """Eq. (obs_update): R[p, p:]/R[p, p] = [H_F^-1]_{p, :}/[H_F^-1]_{pp}, F = {p, .., n-1}."""
     H = ref.damp(kqsynth.random_spd(10, seed=9), 0.01)
@@ -400,6 +412,79 @@ def test_fp32_sweep_row_subset():
     part = obs_sweep_fp32(W, Lt, 3, 16, 16, rows=rows)
     assert np.array_equal(part["codes"], full["codes"][rows])
     assert np.array_equal(part["E"], full["E"][rows])
+
+
+# ------------------------------------------------------------- teacher-forced replay
+def _tf_problem(n=96, m=30, seed=21, with_p=False):
+    H = ref.damp(kqsynth.random_spd(n, seed=seed), 0.01)
+    Lt = ref.lower_factor(H).astype(np.float32)
+    W = (_rng(seed + 1).standard_normal((m, n)) * 0.02).astype(np.float32)
+    Pt = None
+    if with_p:
+        X, Xt, _, _, _, _ = _drift_problem(seed + 2, T=4 * n, n=n)
+        P = ref.gptaq_p(ref.drift_factor(Xt, X), Lt.astype(np.float64), 0.25)
+        Pt = np.ascontiguousarray(P.T.astype(np.float32))
+    return W, Lt, Pt
+
+
+@pytest.mark.parametrize("group,with_p", [(0, False), (32, False), (32, True)])
+def test_teacher_forced_replays_the_fp32_sweep(group, with_p):
+    """Fed the fp32-ordered sweep's own decisions, the replay returns that sweep's errors
+    bit for bit and its codes exactly, puts its pre-quantization values within float32
+    rounding of the exact compensation, and draws its group grids from the block-start
+    values."""
+    W, Lt, Pt = _tf_problem(with_p=with_p)
+    c = obs_sweep_fp32(W, Lt, 3, group, 32, want_pre_q=True, Pt=Pt)
+    tf = ref.teacher_forced(W, Lt, c["pre_q"], c["codes"], c["scale"], c["zero"], 3, group, 32, Pt=Pt)
+    assert np.array_equal(tf["E"], c["E"])
+    assert np.array_equal(tf["codes"], c["codes"])
+    dev = np.abs(tf["pre_q"] - c["pre_q"]) / tf["absum"]
+    assert dev.max() <= 2e-6, dev.max()
+    if group:
+        for g in range(W.shape[1] // group):
+            s, _ = ref.quant_params(tf["block_start"][:, g * group:(g + 1) * group], 3)
+            assert np.allclose(s, c["scale"][:, g], rtol=1e-5, atol=0)
+    else:
+        assert "block_start" not in tf
+
+
+def test_teacher_forced_catches_planted_errors():
+    """Sweeps with a planted mistake fail the replay: one block's lazy update dropped, the
+    compensation's sign flipped, one code off by one."""
+    W, Lt, _ = _tf_problem()
+    group, block = 32, 32
+    good = obs_sweep_fp32(W, Lt, 3, group, block, want_pre_q=True)
+
+    def worst(run):
+        tf = ref.teacher_forced(W, Lt, run["pre_q"], run["codes"], run["scale"], run["zero"], 3, group, block)
+        return float(np.max(np.abs(tf["pre_q"] - run["pre_q"]) / tf["absum"])), tf
+
+    assert worst(good)[0] <= 2e-6
+    dropped = Lt.copy()
+    dropped[64:, 32:64] = 0.0          # R[32:64, 64:] = 0: block 1 never updates the later blocks
+    assert worst(obs_sweep_fp32(W, dropped, 3, group, block, want_pre_q=True))[0] > 1e-3
+    flipped = Lt.copy()
+    off = np.tril(np.ones_like(Lt, dtype=bool), -1)
+    flipped[off] = -flipped[off]       # every compensation with the wrong sign
+    assert worst(obs_sweep_fp32(W, flipped, 3, group, block, want_pre_q=True))[0] > 1e-3
+    codes = good["codes"].copy()
+    codes[3, 40] = codes[3, 40] + 1 if codes[3, 40] < 7 else codes[3, 40] - 1
+    _, tf = worst(dict(good, codes=codes))
+    assert not np.array_equal(tf["codes"], codes)
+
+
+def test_gpu_sweep_checks_accept_the_definition_and_reject_a_planted_error():
+    """The fast-mode checks the GPU tests apply (tests/sweep_checks.py) pass on the
+    fp32-ordered sweep itself and fail on a sweep that drops one block's lazy update."""
+    from sweep_checks import check_fast_sweep
+    W, Lt, _ = _tf_problem(n=256, m=40)
+    good = obs_sweep_fp32(W, Lt, 3, 128, 128, want_pre_q=True)
+    check_fast_sweep(W, Lt, good, 3, 128, 128)
+    dropped = Lt.copy()
+    dropped[128:, :128] *= np.float32(0.5)    # half of block 0's update of block 1
+    bad = obs_sweep_fp32(W, dropped, 3, 128, 128, want_pre_q=True)
+    with pytest.raises(AssertionError):
+        check_fast_sweep(W, Lt, bad, 3, 128, 128)
 
 
 # ---------------------------------------------------------------- GPTAQ drift correction
