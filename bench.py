@@ -2,7 +2,7 @@
 """Benchmark: one synthetic Llama-shaped linear layer through the KronQ per-layer path
 (factors -> BiIP rescale + RHT -> damped inverse Cholesky -> OBS sweep) per step.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--config q_proj_8b] [--impl ours|reference]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--config down_70b] [--impl ours|reference]
 
 Prints one JSON line. `value` is milliseconds per linear layer for the whole job (lower is
 better). Under torchrun each rank quantizes its own layer (the path has no cross-layer
@@ -28,6 +28,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 import kqsynth  # noqa: E402
+import numpy as np  # noqa: E402
 
 METRIC = "ms per linear layer (factors+rotate+chol+OBS sweep)"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}
@@ -39,7 +40,11 @@ def parse():
     ap.add_argument("--steps", type=int, default=None,
                     help="timed steps (default: 100 for a layer or decode, 10 for a block, 3 for the oracle arm)")
     ap.add_argument("--warmup", type=int, default=3)
-    ap.add_argument("--config", default="q_proj_8b", choices=sorted(kqsynth.CONFIGS))
+    ap.add_argument("--config", default="down_70b", choices=sorted(kqsynth.CONFIGS),
+                    help="layer workload (default: the largest, Llama-3-70B down_proj 8192 x 28672)")
+    ap.add_argument("--secondary", default="q_proj_8b",
+                    help="a second layer shape measured in the same run and reported under 'secondary' "
+                         "('' for none)")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -48,6 +53,9 @@ def parse():
                     help="token chunk of the H_X accumulation (0: one call)")
     ap.add_argument("--g-chunk-tokens", type=int, default=0,
                     help="token chunk of the H_G accumulation with device-resident inputs (0: one call)")
+    ap.add_argument("--e2e-x-chunk-tokens", type=int, default=None,
+                    help="token chunk of the H_X accumulation on the host path, each chunk started as soon as "
+                         "its copy has landed (default: 32768 when X is larger than 4 GiB, else one call)")
     ap.add_argument("--e2e-g-chunk-tokens", type=int, default=32768,
                     help="token chunk of the H_G accumulation on the host path, where each chunk starts "
                          "as soon as its copy has landed (0: one call)")
@@ -74,8 +82,10 @@ def parse():
                          "X + 0.1 sigma z); default: GPTQ mode")
     args = ap.parse_args()
     if args.steps is None:
-        # a timed region of at least ~0.5 s, so that the clock record has samples inside it
-        args.steps = 3 if args.impl == "reference" else 10 if args.block else 100
+        # a timed region of several seconds, so that the clock record has samples inside it
+        # (a down_70b layer takes ~0.4 s, a q_proj layer ~6 ms)
+        big = kqsynth.CONFIGS[args.config].d_in * kqsynth.CONFIGS[args.config].d_out > (64 << 20)
+        args.steps = 3 if args.impl == "reference" else 10 if args.block else 20 if big else 100
     return args
 
 
@@ -206,71 +216,101 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------- CPU oracle timing
-def oracle_sample_ms(cfg, repeats: int = 1, T_s: int = 4096, f: int = 2, rows_s: int = 128, alpha=None) -> dict:
-    """Time the oracle on a bounded sample of the workload and extrapolate each stage to
-    the full layer by its cost model: the factors run on T_s of the T tokens at full width
-    (linear in tokens); BiIP, Cholesky and the fp32-ordered sweep run on a layer shrunk by
-    f in both dimensions (dense products and Cholesky cubic in the size; the sweep
-    proportional to rows x d_in^2, run on rows_s rows)."""
+# Bounded samples of the oracle, per stage: the factors on T_s and 2 T_s of the T tokens at
+# full width (a line in the tokens), the BiIP dense products and the textbook inverse
+# Cholesky on the layer shrunk by f in both dimensions (cubic in the size), the fp32-ordered
+# sweep on rows_s rows of that shrunk layer (proportional to rows x d_in^2). f = 1 runs
+# BiIP and the Cholesky at full size.
+ORACLE_SAMPLES = {
+    "large": dict(T_s=1024, f=4, rows_s=64),
+    "medium": dict(T_s=512, f=8, rows_s=64),
+    "small": dict(T_s=256, f=16, rows_s=32),
+}
+
+
+def _shrink(cfg, f: int) -> int:
+    """The largest of f, f/2, ... (down to 1) that leaves both dimensions >= 256 and keeps
+    the Hadamard sizes (2^k or 28 * 2^k) whole."""
+    while f > 1 and (min(cfg.d_in, cfg.d_out) // f < 256 or cfg.d_in % f or cfg.d_out % f):
+        f //= 2
+    return max(f, 1)
+
+
+def _oracle_stages(cfg, T_s: int, f: int, rows_s: int, alpha=None) -> dict:
+    """One timed pass of every stage on its sample, each extrapolated to the full layer (ms)."""
     from oracle import kronq_oracle as ref
     import oracle
 
     T_s = min(cfg.T, T_s)
-    if min(cfg.d_in, cfg.d_out) < 256 * f:
-        f = 1
+    f = _shrink(cfg, f)
     sub = cfg.replace(d_out=cfg.d_out // f, d_in=cfg.d_in // f, T=T_s)
     rows_s = min(sub.d_out, rows_s)
-    L = kqsynth.layer(cfg.replace(T=T_s))
-    Ls = kqsynth.layer(sub)
+    L = {"X": kqsynth.activations(cfg, 2 * T_s), "G": kqsynth.gradients(cfg, 2 * T_s)}
+    Ls = kqsynth.layer(sub) if f > 1 else dict(L, W=kqsynth.weights(cfg), **dict(zip(("sign_u", "sign_v"),
+                                                                                   kqsynth.signs(cfg))))
     drift = alpha is not None
+    per = {}
+    # the factors on T_s and on 2 T_s tokens: a d x d result costs the same at any T (its
+    # allocation and write), so the full layer is the two-point line through both times
+    tf = []
+    for Tk in (T_s, 2 * T_s):
+        t0 = time.perf_counter()
+        ref.accum_factor(L["X"][:Tk])
+        ref.accum_factor(L["G"][:Tk])
+        tf.append(time.perf_counter() - t0)
+    per["factors"] = tf[1] + (cfg.T - 2 * T_s) * (tf[1] - tf[0]) / T_s
+    Ds = None
     if drift:
         Xt = kqsynth.fp_activations(cfg, L["X"])
-        Xts = kqsynth.fp_activations(sub, Ls["X"])
-    stage = {"factors": [], "biip": [], "chol": [], "sweep": []}
+        t1 = time.perf_counter()
+        ref.drift_factor(Xt, L["X"])
+        per["drift"] = (time.perf_counter() - t1) * cfg.T / T_s
+        Ds = ref.drift_factor(kqsynth.fp_activations(sub, Ls["X"]), Ls["X"])
+    HXs, HGs = ref.accum_factor(Ls["X"]), ref.accum_factor(Ls["G"])
+    t1 = time.perf_counter()
+    b = ref.biip(Ls["W"], HXs, HGs, Ls["sign_u"], Ls["sign_v"], Ds)
+    t2 = time.perf_counter()
+    per["biip"] = (t2 - t1) * f ** 3
+    R = ref.inverse_cholesky_upper(ref.damp(b["HX"], cfg.damp))
+    t3 = time.perf_counter()
+    per["chol"] = (t3 - t2) * f ** 3
+    Pt = None
     if drift:
-        stage.update({"drift": [], "p": []})
-    for _ in range(repeats):
-        t0 = time.perf_counter()
-        HX = ref.accum_factor(L["X"])
-        HG = ref.accum_factor(L["G"])
-        t1 = time.perf_counter()
-        stage["factors"].append((t1 - t0) * cfg.T / T_s)
-        Ds = None
-        if drift:
-            t1 = time.perf_counter()
-            ref.drift_factor(Xt, L["X"])
-            stage["drift"].append((time.perf_counter() - t1) * cfg.T / T_s)
-            Ds = ref.drift_factor(Xts, Ls["X"])
-        HXs, HGs = ref.accum_factor(Ls["X"]), ref.accum_factor(Ls["G"])
-        t1 = time.perf_counter()
-        b = ref.biip(Ls["W"], HXs, HGs, Ls["sign_u"], Ls["sign_v"], Ds)
-        t2 = time.perf_counter()
-        stage["biip"].append((t2 - t1) * f ** 3)
-        R = ref.inverse_cholesky_upper(ref.damp(b["HX"], cfg.damp))
-        t3 = time.perf_counter()
-        stage["chol"].append((t3 - t2) * f ** 3)
-        Pt = None
-        if drift:
-            P = ref.gptaq_p(b["D"], R.T, alpha)
-            t3b = time.perf_counter()
-            stage["p"].append((t3b - t3) * f ** 3)
-            Pt = P.T.astype("float32")
-        Wp = b["W"][:rows_s].astype("float32")
-        Lt = R.T.astype("float32")
-        t4 = time.perf_counter()
-        oracle.obs_sweep_fp32(Wp, Lt, cfg.bits, cfg.group, cfg.block, Pt=Pt)
-        t5 = time.perf_counter()
-        stage["sweep"].append((t5 - t4) * (cfg.d_out / rows_s) * f ** 2)
-        del HX, HG, HXs, HGs, b, R
-    per = {k: 1e3 * statistics.mean(v) for k, v in stage.items()}
-    return {"value": sum(per.values()), "unit": "ms", "cores": os.cpu_count(), "kind": "oracle",
-            "stages_ms": per,
-            "sample": (f"factors on {T_s} of {cfg.T} tokens at full width (x{cfg.T / T_s:g}); BiIP dense "
-                       f"products, Cholesky and fp32-ordered sweep ({rows_s} rows) on the "
-                       f"{sub.d_out}x{sub.d_in} layer (x{f}^3, x{f}^3, x{f}^2*{cfg.d_out / rows_s:g}); "
-                       f"{repeats} repeat(s), mean" + ("; drift statistic on the same tokens as the "
-                                                        "factors, P on the shrunk layer (x" + str(f) + "^3)"
-                                                        if drift else ""))}
+        P = ref.gptaq_p(b["D"], R.T, alpha)
+        per["p"] = (time.perf_counter() - t3) * f ** 3
+        Pt = P.T.astype("float32")
+    Wp = np.ascontiguousarray(b["W"][:rows_s]).astype("float32")
+    Lt = R.T.astype("float32")
+    t4 = time.perf_counter()
+    oracle.obs_sweep_fp32(Wp, Lt, cfg.bits, cfg.group, cfg.block, Pt=Pt)
+    per["sweep"] = (time.perf_counter() - t4) * (cfg.d_out / rows_s) * f ** 2
+    return {"stages_ms": {k: 1e3 * v for k, v in per.items()}, "T_s": T_s, "f": f, "rows_s": rows_s}
+
+
+def oracle_sample_ms(cfg, preset: str = "large", alpha=None, check: bool = True) -> dict:
+    """The oracle's time for the layer from the `preset` sample, and (check) the same
+    estimate from a sample half as large (half the tokens, twice the shrink, half the
+    rows), stage by stage, with their ratio: the cost models hold where the two agree."""
+    kw = ORACLE_SAMPLES[preset]
+    main = _oracle_stages(cfg, kw["T_s"], kw["f"], kw["rows_s"], alpha)
+    per = main["stages_ms"]
+    out = {"value": sum(per.values()), "unit": "ms", "cores": os.cpu_count(), "kind": "oracle",
+           "stages_ms": per, "preset": preset,
+           "sample": (f"factors on {main['T_s']} and {2 * main['T_s']} of {cfg.T} tokens at full width (two-point "
+                      f"line to {cfg.T}); "
+                      f"BiIP dense products and textbook inverse Cholesky on the {cfg.d_out // main['f']}x"
+                      f"{cfg.d_in // main['f']} layer (x{main['f']}^3); fp32-ordered sweep on {main['rows_s']} rows "
+                      f"of it (x{main['f']}^2*{cfg.d_out / main['rows_s']:g})"
+                      + ("; drift statistic on the factors' tokens, P on the shrunk layer" if alpha is not None
+                         else ""))}
+    if check:
+        # half the tokens and twice the shrink; the same rows (the fp32 sweep runs rows in
+        # parallel, so fewer rows than a few per core would change the cost per row)
+        half = _oracle_stages(cfg, max(1, kw["T_s"] // 2), 2 * kw["f"], kw["rows_s"], alpha)
+        out["check"] = {"sample": f"T_s {half['T_s']}, shrink {half['f']}, {half['rows_s']} rows",
+                        "stages_ms": half["stages_ms"],
+                        "ratio": {k: per[k] / half["stages_ms"][k] for k in per if half["stages_ms"][k] > 0}}
+    return out
 
 
 # --------------------------------------------------------------------- distributed
@@ -295,6 +335,14 @@ def max_over_ranks(v: float, ws: int, device: str = "cpu") -> float:
     return float(t.item())
 
 
+def reference_preset(steps: int, warmup: int) -> str:
+    """The oracle sample per step of the reference arm: the same sample as our line's
+    cpu_baseline ("large") when the run has few steps, smaller ones when many steps would
+    otherwise run past a few minutes."""
+    n = steps + warmup
+    return "large" if n <= 6 else "medium" if n <= 16 else "small"
+
+
 def run_reference(args):
     ws, rank, _ = dist_setup("gloo")
     cfg = kqsynth.CONFIGS[args.config]
@@ -302,25 +350,163 @@ def run_reference(args):
         cfg = cfg.replace(T=args.tokens)
     if rank != 0:
         return
-    small = dict(T_s=2048, f=4, rows_s=64, alpha=args.drift)
+    preset = reference_preset(args.steps, args.warmup)
     for _ in range(args.warmup):
-        oracle_sample_ms(cfg, **small)
-    vals, last = [], None
+        oracle_sample_ms(cfg, preset, args.drift, check=False)
+    vals, first = [], None
     t0 = time.perf_counter()
-    for _ in range(args.steps):
-        last = oracle_sample_ms(cfg, **small)
-        vals.append(last["value"])
+    for k in range(args.steps):
+        r = oracle_sample_ms(cfg, preset, args.drift, check=(k == 0))
+        first = first or r
+        vals.append(r["value"])
     wall = time.perf_counter() - t0
     v = statistics.mean(vals)
+    cpu = dict(first, value=v, steps_ms=vals)
     out = {"impl": "reference", "metric": metric_of(args.drift), "value": v, "unit": "ms", "n_gpus": args.gpus,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": v, "higher_is_better": False,
            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
            "config": config_dict(cfg, args.x_chunk_tokens, args.g_chunk_tokens, args.trailing, args.drift),
-           "cpu_baseline": {"value": v, "unit": "ms", "cores": last["cores"], "kind": "oracle",
-                            "sample": last["sample"], "stages_ms": last["stages_ms"]},
+           "cpu_baseline": cpu,
            "e2e": {"value": v, "unit": "ms", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+           "timing": "each step times the oracle on a bounded sample of the layer and extrapolates every "
+                     "stage to the full layer by its cost model (see cpu_baseline.sample and .check)",
            "wall_s": wall}
     print(json.dumps(out), flush=True)
+
+
+def tf32_peak(peaks: dict) -> tuple[float, str]:
+    """Dense tf32 tensor peak: the measured bf16 burst times the nominal tf32 : bf16 ratio
+    (1.1 : 2.25 PFLOP/s dense)."""
+    bf16 = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+    return bf16 * 1.1 / 2.25, "measured bf16 dense burst x 1.1/2.25 (nominal tf32 : bf16)"
+
+
+def rotation_bytes(cfg) -> dict:
+    """Bytes of the rotation stage: algorithmic (each two-sided transform of an fp32 matrix
+    read and written once: H_X' 8 d_in^2, H_G' 8 d_out^2, W' 8 d_out d_in) and moved by this
+    implementation (H_X and H_G: row pass, transpose, row pass; W: copy into the work
+    buffer, row pass, column pass)."""
+    hx, hg, w = 4 * cfg.d_in ** 2, 4 * cfg.d_out ** 2, 4 * cfg.d_out * cfg.d_in
+    return {"algorithmic": 2 * (hx + hg + w), "moved": 2 * 3 * (hx + hg) + 2 * 3 * w}
+
+
+def fractions(cfg, stage_ms: dict, peaks: dict, peak_src: str) -> dict:
+    """Per-stage throughput against the roofline that bounds it: the SYRKs against the bf16
+    tensor peak, the Cholesky and the sweep's trailing update against the tf32 peak
+    (algorithmic flops, and executed: the 3xTF32 split runs three tf32 products per
+    multiply-add), the rotations against HBM bandwidth."""
+    bf16 = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+    tf32, tf32_src = tf32_peak(peaks)
+    fl = algorithmic_flops(cfg)
+    out = {"peaks": {"bf16_tflops": bf16, "tf32_tflops": tf32, "hbm_gbs": hbm,
+                     "source": f"{peak_src}; tf32 = {tf32_src}"}}
+    for k in ("factor_x", "factor_g"):
+        t = fl[k] / stage_ms[k] / 1e9
+        out[k] = {"tflops": t, "frac_bf16": t / bf16}
+    for k, name in (("chol", "chol"), ("sweep", "sweep_trailing")):
+        t = fl[k] / stage_ms[k] / 1e9
+        out[name] = {"tflops_algorithmic": t, "frac_tf32_algorithmic": t / tf32,
+                     "tflops_executed_3xtf32": 3 * t, "frac_tf32_executed": 3 * t / tf32}
+    rb = rotation_bytes(cfg)
+    ga, gm = rb["algorithmic"] / stage_ms["rotate"] / 1e6, rb["moved"] / stage_ms["rotate"] / 1e6
+    out["rotate"] = {"gbs_algorithmic": ga, "frac_hbm_algorithmic": ga / hbm, "gbs_moved": gm,
+                     "frac_hbm_moved": gm / hbm, "bytes_algorithmic": rb["algorithmic"], "bytes_moved": rb["moved"]}
+    return out
+
+
+def h2d_link_probe(dev, nbytes: int = 1 << 31, reps: int = 3) -> dict:
+    """Host-to-device bandwidth from pinned memory: the same bytes copied on one stream, and
+    split evenly over 2 and 4 streams running at once (best of `reps`, CUDA events)."""
+    import torch
+
+    host = torch.empty(nbytes, dtype=torch.uint8).pin_memory()
+    devb = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    out = {}
+    for ns in (1, 2, 4):
+        streams = [torch.cuda.Stream(device=dev) for _ in range(ns)]
+        per = nbytes // ns
+        best = float("inf")
+        for _ in range(reps):
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            cur = torch.cuda.current_stream()
+            e0.record(cur)
+            for k, st in enumerate(streams):
+                st.wait_event(e0)
+                with torch.cuda.stream(st):
+                    devb[k * per:(k + 1) * per].copy_(host[k * per:(k + 1) * per], non_blocking=True)
+            for st in streams:
+                cur.wait_stream(st)
+            e1.record(cur)
+            torch.cuda.synchronize()
+            best = min(best, e0.elapsed_time(e1))
+        out[f"{ns}_streams"] = nbytes / best / 1e6
+    del host, devb
+    return {"bytes": nbytes, "gbs": out}
+
+
+def measure_layer(cfg, args, dev, ws, steps, stream, barrier, sample_clocks: bool = True):
+    """Warm-up, then `steps` timed graph replays (or direct runs) of one layer, then a
+    serialized pass with per-stage events. Returns the timings and the pipeline."""
+    import torch
+
+    from paper_2607_07964_gb300 import kronq as kq
+    from paper_2607_07964_gb300.pipeline import LayerPipeline
+
+    inp = kqsynth.device_layer(cfg, device=dev)
+    drift = args.drift is not None
+    Xt = kqsynth.device_fp_activations(cfg, inp["X"]) if drift else None
+    p = LayerPipeline(cfg.d_out, cfg.d_in, cfg.bits, cfg.group, cfg.block, cfg.damp, device=dev,
+                      x_chunk_tokens=args.x_chunk_tokens, g_chunk_tokens=args.g_chunk_tokens,
+                      trailing=args.trailing, alpha=args.drift, drift_chunk_tokens=args.drift_chunk_tokens)
+    run_args = (inp["X"], inp["G"], inp["W"], inp["sign_u"], inp["sign_v"])
+    for _ in range(args.warmup):
+        p.run(*run_args, stream=stream, Xt=Xt)
+    p.check(stream)
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    props = torch.cuda.get_device_properties(dev)
+    sampler = ClockSampler(getattr(props, "pci_bus_id", None))
+    barrier()
+    torch.cuda.synchronize()
+    graph = None
+    per_step = 0
+    if not args.no_graph:
+        graph, per_step = p.capture(*run_args, Xt=Xt)
+        for _ in range(2):
+            graph.replay()
+        torch.cuda.synchronize()
+        barrier()
+    if sample_clocks:
+        sampler.start()
+    n0 = kq.launch_count()
+    t_start.record(stream)
+    for _ in range(steps):
+        if graph is not None:
+            graph.replay()
+        else:
+            p.run(*run_args, stream=stream, Xt=Xt)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    launches = per_step * steps if graph is not None else kq.launch_count() - n0
+    clocks = sampler.stop() if sample_clocks else None
+    p.check(stream)
+    total_ms = max_over_ranks(t_start.elapsed_time(t_end), ws, dev)
+    del graph
+    # Per-stage times come from a second, serialized pass (each stage alone on the stream,
+    # bracketed by events); the headline value above overlaps stages.
+    n_ser = max(1, min(steps, 10))
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(len(p.stages) + 1)] for _ in range(n_ser)]
+    torch.cuda.synchronize()
+    for k in range(n_ser):
+        p.run(*run_args, stream=stream, events=evs[k], Xt=Xt)
+    torch.cuda.synchronize()
+    p.check(stream)
+    stage_ms = {name: statistics.mean(evs[k][i].elapsed_time(evs[k][i + 1]) for k in range(n_ser))
+                for i, name in enumerate(p.stages)}
+    return {"total_ms": total_ms, "stage_ms": stage_ms, "launches": launches, "clocks": clocks,
+            "graph": not args.no_graph, "pipeline": p, "inputs": inp, "Xt": Xt}
 
 
 def run_ours(args):
@@ -329,7 +515,6 @@ def run_ours(args):
     from paper_2607_07964_gb300 import build as kbuild
     ws, rank, local = dist_setup("nccl")
     kbuild.build()
-    from paper_2607_07964_gb300 import kronq as kq
     from paper_2607_07964_gb300.pipeline import LayerPipeline
 
     torch.cuda.set_device(local)
@@ -337,60 +522,18 @@ def run_ours(args):
     cfg = kqsynth.CONFIGS[args.config].replace(seed=rank)
     if args.tokens > 0:
         cfg = cfg.replace(T=args.tokens)
-    inp = kqsynth.device_layer(cfg, device=dev)
     drift = args.drift is not None
-    Xt = kqsynth.device_fp_activations(cfg, inp["X"]) if drift else None
-    p = LayerPipeline(cfg.d_out, cfg.d_in, cfg.bits, cfg.group, cfg.block, cfg.damp, device=dev,
-                      x_chunk_tokens=args.x_chunk_tokens, g_chunk_tokens=args.g_chunk_tokens,
-                      trailing=args.trailing, alpha=args.drift, drift_chunk_tokens=args.drift_chunk_tokens)
-    STAGES = p.stages
     stream = torch.cuda.current_stream()
 
     def barrier():
         if ws > 1:
             torch.distributed.barrier()
 
-    for _ in range(args.warmup):
-        p.run(inp["X"], inp["G"], inp["W"], inp["sign_u"], inp["sign_v"], stream=stream, Xt=Xt)
-    p.check(stream)
-
-    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    sampler = ClockSampler(torch.cuda.get_device_properties(local).pci_bus_id if hasattr(
-        torch.cuda.get_device_properties(local), "pci_bus_id") else None)
-    barrier()
-    torch.cuda.synchronize()
-    graph = None
-    if not args.no_graph:
-        graph, per_step = p.capture(inp["X"], inp["G"], inp["W"], inp["sign_u"], inp["sign_v"], Xt=Xt)
-        for _ in range(2):
-            graph.replay()
-        torch.cuda.synchronize()
-        barrier()
-    sampler.start()
-    n0 = kq.launch_count()
-    t_start.record(stream)
-    for k in range(args.steps):
-        if graph is not None:
-            graph.replay()
-        else:
-            p.run(inp["X"], inp["G"], inp["W"], inp["sign_u"], inp["sign_v"], stream=stream, Xt=Xt)
-    t_end.record(stream)
-    torch.cuda.synchronize()
-    barrier()
-    launches = per_step * args.steps if graph is not None else kq.launch_count() - n0
-    clocks = sampler.stop()
-    p.check(stream)
-    total_ms = max_over_ranks(t_start.elapsed_time(t_end), ws, dev)
-    # Per-stage times and the SYRK roofline come from a second, serialized pass (each stage
-    # alone on the stream, bracketed by events); the headline value above overlaps stages.
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(len(STAGES) + 1)] for _ in range(args.steps)]
-    torch.cuda.synchronize()
-    for k in range(args.steps):
-        p.run(inp["X"], inp["G"], inp["W"], inp["sign_u"], inp["sign_v"], stream=stream, events=evs[k], Xt=Xt)
-    torch.cuda.synchronize()
-    p.check(stream)
-    stage_ms = {name: statistics.mean(evs[k][i].elapsed_time(evs[k][i + 1]) for k in range(args.steps))
-                for i, name in enumerate(STAGES)}
+    steps = args.steps
+    m = measure_layer(cfg, args, dev, ws, steps, stream, barrier)
+    p, inp, Xt = m["pipeline"], m["inputs"], m["Xt"]
+    stage_ms, total_ms, launches, clocks = m["stage_ms"], m["total_ms"], m["launches"], m["clocks"]
+    used_graph = m["graph"]
     fl = algorithmic_flops(cfg, drift)
     tflops = {"factor_x": fl["factor_x"] / stage_ms["factor_x"] / 1e9,
               "factor_g": fl["factor_g"] / stage_ms["factor_g"] / 1e9,
@@ -407,8 +550,9 @@ def run_ours(args):
     traffic = syrk_traffic(cfg, cfg.T // n_launch)
     roofline = {"kernel": "syrk_tc_kernel (H_X = X^T X)", "bound": "tensor", "achieved": achieved,
                 "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak, "traffic": traffic,
-                "peak_source": f"{peak_src} bf16 dense burst",
-                "algorithmic_flops_per_launch": fl["factor_x"] / n_launch, "launches_per_factor": n_launch}
+                "peak_source": f"{peak_src} bf16 dense burst (of measured)",
+                "algorithmic_flops_per_launch": fl["factor_x"] / n_launch, "launches_per_factor": n_launch,
+                "timing": "CUDA events around the H_X stage of the serialized pass (one launch, on its stream)"}
     if drift:
         # the drift stage (one split pass + one drift_tc_kernel launch with K = 2 T): algorithmic
         # flops of (X~ - X)^T X over the stage time; the split pair executes twice as many
@@ -426,9 +570,13 @@ def run_ours(args):
         Gh = inp["G"].cpu().pin_memory()
         Wh = inp["W"].cpu().pin_memory()
         suh, svh = inp["sign_u"].cpu().pin_memory(), inp["sign_v"].cpu().pin_memory()
-        if args.e2e_g_chunk_tokens != args.g_chunk_tokens:
+        e2e_x = args.e2e_x_chunk_tokens
+        if e2e_x is None:
+            e2e_x = 32768 if cfg.T * cfg.d_in * 2 > (4 << 30) else args.x_chunk_tokens
+        link = h2d_link_probe(dev)
+        if args.e2e_g_chunk_tokens != args.g_chunk_tokens or e2e_x != args.x_chunk_tokens:
             p = LayerPipeline(cfg.d_out, cfg.d_in, cfg.bits, cfg.group, cfg.block, cfg.damp, device=dev,
-                              x_chunk_tokens=args.x_chunk_tokens, g_chunk_tokens=args.e2e_g_chunk_tokens,
+                              x_chunk_tokens=e2e_x, g_chunk_tokens=args.e2e_g_chunk_tokens,
                               trailing=args.trailing, alpha=args.drift, drift_chunk_tokens=args.drift_chunk_tokens)
         ch = torch.empty(p.codes.shape, dtype=p.codes.dtype).pin_memory()
         sh = torch.empty(p.scale.shape, dtype=p.scale.dtype).pin_memory()
@@ -440,31 +588,46 @@ def run_ours(args):
         torch.cuda.synchronize()
         e0.record(stream)
         nin = nout = 0
-        for _ in range(args.steps):
+        e_steps = max(1, min(steps, 20))
+        for _ in range(e_steps):
             nin, nout = p.run_host(Xh, Gh, Wh, suh, svh, ch, sh, zh, stream=stream, Xt_h=Xth)
         e1.record(stream)
         torch.cuda.synchronize()
         barrier()
         e_ms = max_over_ranks(e0.elapsed_time(e1), ws, dev)
-        e2e = {"value": e_ms / (ws * args.steps), "unit": "ms", "h2d_bytes_per_step": nin,
-               "d2h_bytes_per_step": nout}
+        e2e = {"value": e_ms / (ws * e_steps), "unit": "ms", "h2d_bytes_per_step": nin,
+               "d2h_bytes_per_step": nout, "steps": e_steps,
+               "factor_chunk_tokens": {"X": e2e_x, "G": args.e2e_g_chunk_tokens}, "h2d_link": link,
+               "bound_ms": max(total_ms / steps, nin / (max(link["gbs"].values()) * 1e6))}
+        del Xh, Xth, Gh, Wh
+    del p, inp, Xt, m
+    torch.cuda.empty_cache()
+
+    secondary = None
+    if args.secondary and args.secondary != args.config and not drift and args.tokens == 0:
+        scfg = kqsynth.CONFIGS[args.secondary].replace(seed=rank)
+        ms = measure_layer(scfg, args, dev, ws, 50, stream, barrier, sample_clocks=False)
+        secondary = {"workload": workload_name(scfg), "value": ms["total_ms"] / (ws * 50), "unit": "ms",
+                     "steps": 50, "stages_ms": ms["stage_ms"], "gpu_launches": ms["launches"],
+                     "fractions": fractions(scfg, ms["stage_ms"], peaks, peak_src)}
+        del ms
+        torch.cuda.empty_cache()
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        cpu = oracle_sample_ms(cfg, repeats=2, alpha=args.drift)
+        cpu = oracle_sample_ms(cfg, "large", alpha=args.drift)
 
     if rank == 0:
-        out = {"metric": metric_of(args.drift), "value": total_ms / (ws * args.steps), "unit": "ms", "n_gpus": ws,
-               "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
+        out = {"metric": metric_of(args.drift), "value": total_ms / (ws * steps), "unit": "ms", "n_gpus": ws,
+               "steps": steps, "warmup": args.warmup, "ms_per_step": total_ms / steps,
                "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
                "dtype": "bf16 products, f32 accumulate/arithmetic", "data": "synthetic",
-               "config": dict(config_dict(cfg, args.x_chunk_tokens, args.g_chunk_tokens, args.trailing, args.drift),
-                              e2e_factor_chunk_tokens={"X": args.x_chunk_tokens, "G": args.e2e_g_chunk_tokens}),
-               "stages_ms": stage_ms, "tflops": tflops,
+               "config": config_dict(cfg, args.x_chunk_tokens, args.g_chunk_tokens, args.trailing, args.drift),
+               "stages_ms": stage_ms, "tflops": tflops, "fractions": fractions(cfg, stage_ms, peaks, peak_src),
                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
-               "launch_mode": "cuda graph replay (one graph per layer, two streams)" if graph is not None
+               "launch_mode": "cuda graph replay (one graph per layer, two streams)" if used_graph
                else "direct launches (two streams)",
-               "clocks": clocks}
+               "clocks": clocks, "secondary": secondary}
         print(json.dumps(out), flush=True)
     if ws > 1:
         torch.distributed.destroy_process_group()
@@ -494,12 +657,12 @@ def oracle_block_ms(bc, small: bool = False) -> dict:
     """The oracle's time for a block: the layer estimate of oracle_sample_ms per sublayer,
     minus the H_X accumulations the shared inputs do not repeat."""
     spec = kqsynth.block_spec(bc)
-    kw = dict(T_s=2048, f=4, rows_s=64) if small else {}
+    preset = "medium" if small else "large"
     total, seen, parts = 0.0, set(), {}
     for name, grp, d_out, d_in in spec:
         c = kqsynth.LayerConfig(name, d_out, d_in, bc.T, bc.low_bits, bc.group, bc.n_outliers, bc.g_sigma,
                                 block=bc.block, damp=bc.damp)
-        r = oracle_sample_ms(c, **kw)
+        r = oracle_sample_ms(c, preset, check=False)
         v = r["value"]
         if grp in seen:   # H_X of a shared input is accumulated once: drop this layer's X share
             v -= r["stages_ms"]["factors"] * d_in * d_in / (d_in * d_in + d_out * d_out)

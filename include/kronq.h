@@ -53,7 +53,8 @@ typedef enum kq_status {
     KQ_ERR_NOT_PD = 3,       /* non-positive pivot in kq_chol_inv (reported through `info`) */
     KQ_ERR_CUDA = 4,         /* a CUDA runtime/driver call failed */
     KQ_ERR_TIMEOUT = 5,      /* a kernel gave up a bounded wait (reported through `info`) */
-    KQ_ERR_WORKSPACE = 6     /* ws is NULL or smaller than the *_workspace() size */
+    KQ_ERR_WORKSPACE = 6,    /* ws is NULL or smaller than the *_workspace() size */
+    KQ_ERR_NONFINITE = 7     /* a NaN or infinity reached the quantizer (kq_obs_quantize, `info`) */
 } kq_status;
 
 /* Text of the last host-side error of the calling thread ("" when none). */
@@ -96,6 +97,25 @@ KQ_API kq_status kq_check(int* info, int reset, int* pivot_out, kq_stream_t stre
  *   returns an error status and leaves the context usable.
  */
 KQ_API kq_status kq_selftest_timeout(int* info, int64_t limit_us, kq_stream_t stream);
+
+/*
+ * Debug build (no counterpart in the paper). libkronq_debug.so is the same library compiled
+ * with -DKQ_DEBUG: before their global-memory stores the kernels check each index against
+ * the size of the buffer it belongs to, and a failed check skips the store and records the
+ * source line (first failure per source file) instead of faulting. A stand-in for a memory
+ * checker on machines where none may run.
+ * kq_debug_build: 1 for the debug build, 0 otherwise.
+ * kq_debug_status: synchronizes the device, then *unit = the first source file (0 api,
+ *   1 syrk, 2 biip, 3 chol, 4 obs, 5 trail_tc, 6 gptaq, 7 infer, 8 check) whose checks
+ *   failed and *line = its first failing line, or *unit = -1 and *line = 0 when none did
+ *   (always so in the normal build); reset clears the recorded lines.
+ * kq_selftest_bounds: writes buf[i] = i for i = 0 .. n under a check against n; buf must
+ *   hold n + 1 floats, so every write stays inside it in either build. The debug build skips
+ *   index n and records it (the check itself is what this exercises).
+ */
+KQ_API int kq_debug_build(void);
+KQ_API kq_status kq_debug_status(int* unit, int* line, int reset);
+KQ_API kq_status kq_selftest_bounds(float* buf, int64_t n, kq_stream_t stream);
 
 /*
  * kq_selftest_div: a diagnostic with no counterpart in the paper. The OBS sweep (Sec. 2.1
@@ -339,7 +359,9 @@ KQ_API kq_status kq_gptaq_p(const float* Dp, const float* Lt, int64_t n, float a
  *     Needs d_in % 4 == 0 and a 16-byte aligned W.
  *   Requirements: 1 <= bits <= 8, block == 128, group in {0, block}; with P also
  *   d_in % 16 == 0 and W, codes, Pt 16-byte aligned.
- *   info (nullable, device int): -KQ_ERR_TIMEOUT if a tensor-core pipeline wait gave up.
+ *   info (nullable, device int): -KQ_ERR_TIMEOUT if a tensor-core pipeline wait gave up;
+ *   -KQ_ERR_NONFINITE if a value about to be quantized was NaN or infinite (a non-finite W',
+ *   for example from a NaN weight; that row's codes and grids are then meaningless).
  *   ws: kq_obs_quantize_workspace(d_out, d_in, block, mode, with_p) bytes (with_p = 1 when
  *   Pt will be passed), 256-byte aligned.
  * ---------------------------------------------------------------------------------- */

@@ -108,9 +108,14 @@ class BlockQuantizer:
         return bits, sc
 
     def check(self) -> None:
+        """Raise the first device-side error of the block; every word is read and cleared."""
         torch.cuda.synchronize()
         st, raw = kq.kq_check(self.info, reset=True)
-        if st != kq.KQ_OK:
-            raise kq.KronqError(st, "block", f"device word {raw}")
+        first = None if st == kq.KQ_OK else kq.KronqError(st, "block", f"device word {raw}")
         for p in self.pipes.values():
-            p.check()
+            try:
+                p.check()
+            except kq.KronqError as e:
+                first = first or e
+        if first is not None:
+            raise first

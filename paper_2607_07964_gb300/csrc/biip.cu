@@ -149,10 +149,86 @@ __global__ void __launch_bounds__((1 << LG) / 16) rht_rows_reg_kernel(float* __r
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
             const int j = tl | deposit_bits<ML>(k);
-            dst[j] = POST ? x[k] * fpost[j] : x[k] * inv_sqrt_n;
+            if (KQ_IN_RANGE(r * N + j, rows * N)) dst[j] = POST ? x[k] * fpost[j] : x[k] * inv_sqrt_n;
         }
 #pragma unroll
         for (int k = 0; k < 16; ++k) x[k] = nx[k];
+    }
+}
+
+// ------------------------------------------- row transform in registers, n = 28 * 2^LG
+// For n = 28 P (P = 2^LG, LG in [9, 10]: 14336 and 28672) with index j = a P + b (b
+// fastest): every chunk a of P contiguous elements takes the Walsh-Hadamard transform H_P,
+// then every column b takes the 28-point mix across the chunks. Seven groups of P / 16
+// threads; group g transforms chunks g, g + 7, g + 14, g + 21 one after another with the
+// four-bit register phases of rht.cuh (each group with its own exchange buffer) and leaves
+// them in a shared-memory copy of the row; then each thread mixes whole columns b
+// (mix28_paley) and writes the 28 results straight to global memory, consecutive threads
+// at consecutive b. While chunk c of a row is transformed, chunk c of the CTA's next row is
+// already on its way into the register slot the current chunk left, so the whole next row
+// is in flight during the mixes. One CTA per SM (the row copy is 112 KB at n = 28672).
+template <int LG, bool POST>
+__global__ void __launch_bounds__(7 * (1 << LG) / 16, 1) rht_rows28_reg_kernel(float* __restrict__ M, int64_t rows,
+                                                                             int pre_mode, int post_mode,
+                                                                             const int8_t* __restrict__ sign,
+                                                                             const float* __restrict__ s,
+                                                                             float inv_sqrt_n) {
+    constexpr int P = 1 << LG, N = 28 * P, TG = P / 16, T = 7 * TG, NPH = rr_phases(LG);
+    constexpr uint32_t ML = rr_mask(LG, NPH - 1);
+    static_assert(NPH == 3, "three register phases for P = 512 and 1024");
+    extern __shared__ __align__(16) float sm28[];
+    float* v = sm28;                                         // [N]
+    const int t = threadIdx.x, g = t / TG, tl = t - g * TG;
+    float* buf = sm28 + N + g * (P + P / 32);                // this group's exchange buffer
+    auto load = [&](int64_t row, int c, float (&x)[16]) {
+        const float4* src = reinterpret_cast<const float4*>(M + row * N + (g + 7 * c) * P + 16 * tl);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const float4 a = src[q];
+            x[4 * q] = a.x;
+            x[4 * q + 1] = a.y;
+            x[4 * q + 2] = a.z;
+            x[4 * q + 3] = a.w;
+        }
+    };
+    float cur[4][16];
+    int64_t r = blockIdx.x;
+    if (r < rows) {
+#pragma unroll
+        for (int c = 0; c < 4; ++c) load(r, c, cur[c]);
+    }
+    const int tw = deposit_bits<(P - 1) & ~ML>(tl);
+    for (; r < rows; r += gridDim.x) {
+        const bool more = r + gridDim.x < rows;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            float x[16];
+#pragma unroll
+            for (int k = 0; k < 16; ++k) x[k] = cur[c][k];
+            if (more) load(r + gridDim.x, c, cur[c]);
+            const int a = g + 7 * c;
+#pragma unroll
+            for (int k = 0; k < 16; ++k) x[k] *= factor(pre_mode, sign, s, a * P + 16 * tl + k);
+            fwht_kbits<0xFu>(x);
+            rr_transpose<LG, 1>(x, buf, tl);
+            rr_transpose<LG, 2>(x, buf, tl);
+#pragma unroll
+            for (int k = 0; k < 16; ++k)
+                if (KQ_IN_RANGE(a * P + (tw | deposit_bits<ML>(k)), N)) v[a * P + (tw | deposit_bits<ML>(k))] = x[k];
+        }
+        __syncthreads();
+        float* dst = M + r * N;
+        for (int b = t; b < P; b += T) {
+            float y[28];
+#pragma unroll
+            for (int a = 0; a < 28; ++a) y[a] = v[a * P + b];
+            mix28_paley(y, [&](int a, float val) {
+                const int j = a * P + b;
+                if (KQ_IN_RANGE(r * N + j, rows * N))
+                    dst[j] = POST ? val * (factor(post_mode, sign, s, j) * inv_sqrt_n) : val * inv_sqrt_n;
+            });
+        }
+        __syncthreads();   // v is rewritten by the next row
     }
 }
 
@@ -183,9 +259,9 @@ __global__ void __launch_bounds__(256) transpose_sq_kernel(float* __restrict__ M
     __syncthreads();
     for (int yy = ty; yy < TT; yy += 4) {
         const int64_t r1 = bj * TT + yy, c1 = bi * TT + tx;   // tile (bj, bi) <- a^T
-        if (r1 < n && c1 < n) M[r1 * n + c1] = a[tx][yy];
+        if (r1 < n && c1 < n && KQ_IN_RANGE(r1 * n + c1, n * n)) M[r1 * n + c1] = a[tx][yy];
         const int64_t r2 = bi * TT + yy, c2 = bj * TT + tx;   // tile (bi, bj) <- b^T
-        if (bi != bj && r2 < n && c2 < n) M[r2 * n + c2] = b[tx][yy];
+        if (bi != bj && r2 < n && c2 < n && KQ_IN_RANGE(r2 * n + c2, n * n)) M[r2 * n + c2] = b[tx][yy];
     }
 }
 
@@ -247,13 +323,17 @@ __global__ void __launch_bounds__(256, IS28 ? 2 : 4) rht_cols_kernel(float* __re
             if (vec && cw == CW) {
                 for (int e = threadIdx.x; e < (28 * CW) >> 2; e += blockDim.x) {
                     const int i = (4 * e) >> lgCW, c = (4 * e) & (CW - 1);
-                    *reinterpret_cast<float4*>(M + (base + static_cast<int64_t>(i) * S) * ncols + c0 + c) =
-                        *reinterpret_cast<const float4*>(v + 4 * e);
+                    if (KQ_IN_RANGE((base + static_cast<int64_t>(i) * S) * ncols + c0 + c + 3,
+                                    static_cast<int64_t>(n) * ncols))
+                        *reinterpret_cast<float4*>(M + (base + static_cast<int64_t>(i) * S) * ncols + c0 + c) =
+                            *reinterpret_cast<const float4*>(v + 4 * e);
                 }
             } else {
                 for (int e = threadIdx.x; e < 28 * CW; e += blockDim.x) {
                     const int i = e >> lgCW, c = e & (CW - 1);
-                    if (c < cw) M[(base + static_cast<int64_t>(i) * S) * ncols + c0 + c] = v[e];
+                    if (c < cw && KQ_IN_RANGE((base + static_cast<int64_t>(i) * S) * ncols + c0 + c,
+                                              static_cast<int64_t>(n) * ncols))
+                        M[(base + static_cast<int64_t>(i) * S) * ncols + c0 + c] = v[e];
                 }
             }
         } else {
@@ -276,10 +356,9 @@ __global__ void __launch_bounds__(256, IS28 ? 2 : 4) rht_cols_kernel(float* __re
                     for (int q = 0; q < 8; ++q)
                         if (q < rr) {
                             if (last) {
-                                if (c < cw) {
-                                    const int64_t r = base + static_cast<int64_t>(bi + q * h) * S;
+                                const int64_t r = base + static_cast<int64_t>(bi + q * h) * S;
+                                if (c < cw && KQ_IN_RANGE(r * ncols + c0 + c, static_cast<int64_t>(n) * ncols))
                                     M[r * ncols + c0 + c] = x[q] * (factor(post_mode, sign, s, r) * post_scale);
-                                }
                             } else {
                                 v[((bi + q * h) << lgCW) + c] = x[q];
                             }
@@ -573,15 +652,46 @@ kq_status launch_rows_reg(float* M, int64_t rows, int pre, int post, const int8_
     return KQ_OK;
 }
 
-// n a power of two from 512 to 16384 and M 16-byte aligned: the register row transform.
+template <int LG>
+kq_status launch_rows28_reg(float* M, int64_t rows, int pre, int post, const int8_t* sign, const float* s,
+                            cudaStream_t stream) {
+    constexpr int P = 1 << LG, T = 7 * P / 16;
+    constexpr size_t smem = (28 * static_cast<size_t>(P) + 7 * (P + P / 32)) * sizeof(float);
+    static std::atomic<uint64_t> attr{0};
+    KQ_TRY(once_per_device(attr, [&]() -> kq_status {
+        KQ_CUDA(cudaFuncSetAttribute(rht_rows28_reg_kernel<LG, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     static_cast<int>(smem)));
+        KQ_CUDA(cudaFuncSetAttribute(rht_rows28_reg_kernel<LG, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     static_cast<int>(smem)));
+        return KQ_OK;
+    }));
+    const int64_t per_sm = std::max<int64_t>(1, std::min<int64_t>(static_cast<int64_t>((227 * 1024) / smem), 2048 / T));
+    const int64_t grid = std::min<int64_t>(rows, static_cast<int64_t>(num_sms()) * per_sm);
+    const float isn = static_cast<float>(1.0 / sqrt(static_cast<double>(28 * P)));
+    if (post == F_NONE)
+        rht_rows28_reg_kernel<LG, false><<<static_cast<unsigned>(grid), T, smem, stream>>>(M, rows, pre, post, sign, s, isn);
+    else
+        rht_rows28_reg_kernel<LG, true><<<static_cast<unsigned>(grid), T, smem, stream>>>(M, rows, pre, post, sign, s, isn);
+    KQ_LAUNCH_CHECK("rht_rows28_reg_kernel");
+    return KQ_OK;
+}
+
+// M 16-byte aligned and n a power of two from 512 to 16384, or 28 * 512 / 28 * 1024: a
+// register row transform.
 bool rows_reg_ok(const float* M, int64_t n) {
-    return n >= 512 && n <= 16384 && (n & (n - 1)) == 0 && (reinterpret_cast<uintptr_t>(M) & 15u) == 0;
+    if ((reinterpret_cast<uintptr_t>(M) & 15u) != 0) return false;
+    if (n == 28 * 512 || n == 28 * 1024) return true;
+    return n >= 512 && n <= 16384 && (n & (n - 1)) == 0;
 }
 
 kq_status rows_transform(float* M, int64_t rows, int64_t n, int pre, int post, const int8_t* sign,
                          const float* s, cudaStream_t stream) {
     HadamardPlan p;
     if (!plan_of(n, &p)) return KQ_ERR_UNSUPPORTED;
+    if (rows > 0 && rows_reg_ok(M, n) && p.has28) {
+        if (p.P == 512) return launch_rows28_reg<9>(M, rows, pre, post, sign, s, stream);
+        return launch_rows28_reg<10>(M, rows, pre, post, sign, s, stream);
+    }
     if (rows > 0 && rows_reg_ok(M, n)) {
         switch (log2i(n)) {
             case 9: return launch_rows_reg<9>(M, rows, pre, post, sign, s, stream);
@@ -693,6 +803,8 @@ kq_status two_sided_transform(float* M, int64_t n, int pre, const int8_t* sign, 
 }
 
 }  // namespace
+
+KQ_DEBUG_UNIT(biip)
 }  // namespace kq
 
 using namespace kq;

@@ -101,6 +101,8 @@ __global__ void sum_kernel(const double* __restrict__ partial, int n, double* ou
 constexpr int DOT_BLOCKS = 256;
 
 }  // namespace
+
+KQ_DEBUG_UNIT(check)
 }  // namespace kq
 
 using namespace kq;

@@ -93,8 +93,10 @@ __global__ void prep_kernel(const float* __restrict__ H, int64_t n, int64_t npad
         } else {
             v = (i == j) ? 1.0f : 0.0f;
         }
-        A[e] = v;
-        Z[e] = 0.0f;
+        if (KQ_IN_RANGE(e, total)) {
+            A[e] = v;
+            Z[e] = 0.0f;
+        }
     }
 }
 
@@ -368,7 +370,8 @@ __global__ void __launch_bounds__(DIAG_THREADS) chol_diag_kernel(Work w, int64_t
                 const int kk = k0 + c;
                 o[c] = kk < i ? -m[r][c] * idv[kk] * si : (kk == i ? si : 0.0f);
             }
-            *reinterpret_cast<float4*>(w.Z + (off + i) * npad + off + k0) = make_float4(o[0], o[1], o[2], o[3]);
+            if (KQ_IN_RANGE((off + i) * npad + off + k0 + 3, npad * npad))
+                *reinterpret_cast<float4*>(w.Z + (off + i) * npad + off + k0) = make_float4(o[0], o[1], o[2], o[3]);
         }
     }
 }
@@ -502,7 +505,8 @@ __global__ void __launch_bounds__(G_THREADS, 2) chol_panel_kernel(Work w, int64_
         strip_gemm<128, 32, true>(cinv, out, npad, acc, sm);
 #pragma unroll
         for (int i = 0; i < 8; ++i)
-            *reinterpret_cast<float2*>(out + (ty + 16 * i) * npad + 2 * tx) = make_float2(acc[i][0], acc[i][1]);
+            if (KQ_IN_RANGE((out - w.Z) + (ty + 16 * i) * npad + 2 * tx + 1, npad * npad))
+                *reinterpret_cast<float2*>(out + (ty + 16 * i) * npad + 2 * tx) = make_float2(acc[i][0], acc[i][1]);
     } else {
         float* out = w.A + (static_cast<int64_t>(b + 1) * NB + 32 * s) * npad + off;
         float acc[2][8];
@@ -510,7 +514,9 @@ __global__ void __launch_bounds__(G_THREADS, 2) chol_panel_kernel(Work w, int64_
 #pragma unroll
         for (int i = 0; i < 2; ++i)
 #pragma unroll
-            for (int j = 0; j < 8; ++j) out[(ty + 16 * i) * npad + tx + 16 * j] = acc[i][j];
+            for (int j = 0; j < 8; ++j)
+                if (KQ_IN_RANGE((out - w.A) + (ty + 16 * i) * npad + tx + 16 * j, npad * npad))
+                    out[(ty + 16 * i) * npad + tx + 16 * j] = acc[i][j];
     }
 }
 
@@ -533,7 +539,9 @@ __device__ __forceinline__ void update_quad(const Work& w, int64_t npad, int k, 
 #pragma unroll
         for (int a = 0; a < 4; ++a)
 #pragma unroll
-            for (int c = 0; c < 4; ++c) out[(ty + 16 * a) * npad + tx + 16 * c] = o[a][c] - acc[a][c];
+            for (int c = 0; c < 4; ++c)
+                if (KQ_IN_RANGE((out - w.A) + (ty + 16 * a) * npad + tx + 16 * c, npad * npad))
+                    out[(ty + 16 * a) * npad + tx + 16 * c] = o[a][c] - acc[a][c];
     } else {
         strip_gemm<64, 64, true>(cik, w.Z + ko * npad + c0, npad, acc, sm);
         float* out = w.Z + r0 * npad + c0;
@@ -542,8 +550,9 @@ __device__ __forceinline__ void update_quad(const Work& w, int64_t npad, int k, 
         for (int a = 0; a < 4; ++a) o[a] = *reinterpret_cast<const float4*>(out + (ty + 16 * a) * npad + 4 * tx);
 #pragma unroll
         for (int a = 0; a < 4; ++a)
-            *reinterpret_cast<float4*>(out + (ty + 16 * a) * npad + 4 * tx) =
-                make_float4(o[a].x - acc[a][0], o[a].y - acc[a][1], o[a].z - acc[a][2], o[a].w - acc[a][3]);
+            if (KQ_IN_RANGE((out - w.Z) + (ty + 16 * a) * npad + 4 * tx + 3, npad * npad))
+                *reinterpret_cast<float4*>(out + (ty + 16 * a) * npad + 4 * tx) =
+                    make_float4(o[a].x - acc[a][0], o[a].y - acc[a][1], o[a].z - acc[a][2], o[a].w - acc[a][3]);
     }
 }
 
@@ -577,6 +586,7 @@ __global__ void chol_split_kernel(const float* __restrict__ A, const float* __re
         for (int r = threadIdx.y; r < 32; r += 8) {
             const float x = A[(r0 + r) * npad + ko + c0 + threadIdx.x];
             const float h = tf32_hi(x);
+            if (!KQ_IN_RANGE((r0 + r) * width + col + c0 + threadIdx.x, npad * width)) continue;
             Ch[(r0 + r) * width + col + c0 + threadIdx.x] = h;
             Cl[(r0 + r) * width + col + c0 + threadIdx.x] = x - h;
         }
@@ -590,6 +600,7 @@ __global__ void chol_split_kernel(const float* __restrict__ A, const float* __re
         for (int r = threadIdx.y; r < 32; r += 8) {
             const float x = t[threadIdx.x][r];   // Z[ko + kc0 + threadIdx.x][q0 + r]
             const float h = tf32_hi(x);
+            if (!KQ_IN_RANGE((q0 + r) * width + col + kc0 + threadIdx.x, npad * width)) continue;
             Zh[(q0 + r) * width + col + kc0 + threadIdx.x] = h;
             Zl[(q0 + r) * width + col + kc0 + threadIdx.x] = x - h;
         }
@@ -599,6 +610,7 @@ __global__ void chol_split_kernel(const float* __restrict__ A, const float* __re
     const int64_t q0 = ko + NB + (b / (NB / 32)) * 32, kc0 = (b % (NB / 32)) * 32;
     if (q0 < zero_to)
         for (int r = threadIdx.y; r < 32; r += 8) {
+            if (!KQ_IN_RANGE((q0 + r) * width + col + kc0 + threadIdx.x, npad * width)) continue;
             Zh[(q0 + r) * width + col + kc0 + threadIdx.x] = 0.0f;
             Zl[(q0 + r) * width + col + kc0 + threadIdx.x] = 0.0f;
         }
@@ -620,11 +632,13 @@ __global__ void finish_kernel(const float* __restrict__ Z, int64_t n, int64_t np
     __syncthreads();
     for (int r = threadIdx.y; r < 32; r += blockDim.y) {
         const int64_t i = i0 + r, j = j0 + threadIdx.x;
-        if (i < n && j < n) Lt[i * n + j] = t[threadIdx.x][r];
+        if (i < n && j < n && KQ_IN_RANGE(i * n + j, n * n)) Lt[i * n + j] = t[threadIdx.x][r];
     }
 }
 
 }  // namespace
+
+KQ_DEBUG_UNIT(chol)
 }  // namespace kq
 
 using namespace kq;

@@ -250,6 +250,8 @@ __global__ void split_transpose_kernel(const float* __restrict__ L, int64_t n, f
 inline size_t mat_bytes(int64_t n) { return (static_cast<size_t>(n) * n * sizeof(float) + 255) & ~static_cast<size_t>(255); }
 
 }  // namespace
+
+KQ_DEBUG_UNIT(gptaq)
 }  // namespace kq
 
 using namespace kq;

@@ -512,7 +512,9 @@ __global__ void __launch_bounds__(IS_WARPS * 32, stream_ctas_per_sm(B)) infer_st
                 const int rl = e / B, b = e - rl * B;
                 float a = 0.0f;
                 for (int s2 = 0; s2 < S; ++s2) a += pp[(rl * S + s2) * B + b];
-                yp[static_cast<int64_t>(b) * d_out + static_cast<int64_t>(q0) * 4 + rl] = a;
+                if (KQ_IN_RANGE(static_cast<int64_t>(b) * d_out + static_cast<int64_t>(q0) * 4 + rl,
+                                static_cast<int64_t>(B) * d_out))
+                    yp[static_cast<int64_t>(b) * d_out + static_cast<int64_t>(q0) * 4 + rl] = a;
             }
             __syncwarp();
             if (lane == 0 && t + nslot < nst) {
@@ -886,6 +888,8 @@ kq_status launch_gemv(int64_t B, dim3 grid, cudaStream_t st, const uint32_t* pac
 inline size_t al256(size_t b) { return (b + 255) & ~static_cast<size_t>(255); }
 
 }  // namespace
+
+KQ_DEBUG_UNIT(infer)
 }  // namespace kq
 
 using namespace kq;

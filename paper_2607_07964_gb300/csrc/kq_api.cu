@@ -153,6 +153,7 @@ extern "C" const char* kq_status_name(int s) {
         case KQ_ERR_CUDA: return "KQ_ERR_CUDA";
         case KQ_ERR_TIMEOUT: return "KQ_ERR_TIMEOUT";
         case KQ_ERR_WORKSPACE: return "KQ_ERR_WORKSPACE";
+        case KQ_ERR_NONFINITE: return "KQ_ERR_NONFINITE";
         default: return "KQ_ERR_UNKNOWN";
     }
 }
@@ -203,4 +204,71 @@ extern "C" kq_status kq_check(int* info, int reset, int* pivot_out, kq_stream_t 
     }
     kq::set_error("kernel reported %s", kq_status_name(-v));
     return static_cast<kq_status>(-v);
+}
+
+// ------------------------------------------------------------------ debug build
+namespace kq {
+namespace {
+// buf[i] = i for i in [0, n] under a bounds check against n: buf holds n + 1 floats, so the
+// last write stays inside it in every build; the debug build's check skips it and records
+// this line.
+__global__ void selftest_bounds_kernel(float* __restrict__ buf, int64_t n) {
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i <= n;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x)
+        if (KQ_IN_RANGE(i, n)) buf[i] = static_cast<float>(i);
+}
+}  // namespace
+
+KQ_DEBUG_UNIT(api)
+int debug_read_syrk(int);
+int debug_read_biip(int);
+int debug_read_chol(int);
+int debug_read_obs(int);
+int debug_read_trail_tc(int);
+int debug_read_gptaq(int);
+int debug_read_infer(int);
+int debug_read_check(int);
+}  // namespace kq
+
+extern "C" int kq_debug_build(void) {
+#ifdef KQ_DEBUG
+    return 1;
+#else
+    return 0;
+#endif
+}
+
+extern "C" kq_status kq_debug_status(int* unit, int* line, int reset) {
+    using Reader = int (*)(int);
+    static const Reader readers[] = {kq::debug_read_api,      kq::debug_read_syrk,  kq::debug_read_biip,
+                                     kq::debug_read_chol,     kq::debug_read_obs,   kq::debug_read_trail_tc,
+                                     kq::debug_read_gptaq,    kq::debug_read_infer, kq::debug_read_check};
+    KQ_CUDA(cudaDeviceSynchronize());
+    int u = -1, l = 0;
+    for (int k = 0; k < static_cast<int>(sizeof(readers) / sizeof(readers[0])); ++k) {
+        const int v = readers[k](reset);
+        if (v < 0) {
+            kq::set_error("kq_debug_status: cannot read the debug word of unit %d", k);
+            return KQ_ERR_CUDA;
+        }
+        if (v > 0 && u < 0) {
+            u = k;
+            l = v;
+        }
+    }
+    if (unit) *unit = u;
+    if (line) *line = l;
+    return KQ_OK;
+}
+
+extern "C" kq_status kq_selftest_bounds(float* buf, int64_t n, kq_stream_t stream_) {
+    if (!buf || n < 1) {
+        kq::set_error("kq_selftest_bounds: buf must hold n + 1 floats, n >= 1");
+        return KQ_ERR_INVALID_ARG;
+    }
+    const int64_t blocks = std::min<int64_t>(kq::cdiv(n + 1, 256), 1024);
+    kq::selftest_bounds_kernel<<<static_cast<unsigned>(blocks), 256, 0, reinterpret_cast<cudaStream_t>(stream_)>>>(
+        buf, n);
+    KQ_LAUNCH_CHECK("selftest_bounds_kernel");
+    return KQ_OK;
 }

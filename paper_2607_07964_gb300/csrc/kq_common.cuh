@@ -77,6 +77,40 @@ struct SideStream {
 };
 SideStream* side_stream(cudaStream_t caller);
 
+// ------------------------------------------------------------------ debug bounds checks
+// In the debug build (libkronq_debug.so, compiled with -DKQ_DEBUG), KQ_IN_RANGE(i, n) checks
+// 0 <= i < n for an index into a buffer of n elements before the kernel accesses it: a
+// failed check records the source line in this translation unit's debug word (the first
+// failure wins) and the guarded access is skipped, so a wrong index shows up as a status
+// (kq_debug_status) instead of a fault. In the normal build it is `true` and costs
+// nothing. Each .cu file ends with KQ_DEBUG_UNIT(name), which defines the host function
+// that reads and clears that file's word.
+#ifdef KQ_DEBUG
+namespace {
+__device__ int g_kq_debug_line;
+}
+__device__ __forceinline__ bool debug_in_range(long long i, long long n, int line) {
+    if (i >= 0 && i < n) return true;
+    atomicCAS(&g_kq_debug_line, 0, line);
+    return false;
+}
+#define KQ_IN_RANGE(i, n) (::kq::debug_in_range(static_cast<long long>(i), static_cast<long long>(n), __LINE__))
+#define KQ_DEBUG_UNIT(name)                                                                    \
+    int debug_read_##name(int reset) {                                                         \
+        int v = 0;                                                                             \
+        if (cudaMemcpyFromSymbol(&v, g_kq_debug_line, sizeof(int)) != cudaSuccess) return -1;  \
+        if (reset && v) {                                                                      \
+            const int z = 0;                                                                   \
+            if (cudaMemcpyToSymbol(g_kq_debug_line, &z, sizeof(int)) != cudaSuccess) return -1; \
+        }                                                                                      \
+        return v;                                                                              \
+    }
+#else
+#define KQ_IN_RANGE(i, n) true
+#define KQ_DEBUG_UNIT(name) \
+    int debug_read_##name(int) { return 0; }
+#endif
+
 // ------------------------------------------------------------------------- device side
 // Device error words: info == 0 ok; > 0 a 1-based pivot index (Cholesky); < 0 minus a
 // kq_status recorded by a kernel (for example -KQ_ERR_TIMEOUT).

@@ -23,6 +23,7 @@
 //   colloss_kernel   col_loss[j] = sum over rows of E_j^2, fixed order (sumsq.cuh)
 #include <math.h>
 
+#include <cstdlib>
 #include <type_traits>
 
 #include "kq_common.cuh"
@@ -34,6 +35,17 @@ namespace kq {
 namespace {
 
 constexpr int BLK = 128;          // block size B (Algorithm 2); the only supported value
+constexpr int SPB = 8;            // blocks per super-panel of the two-level lazy update
+
+// Column width of the long (super-panel) update tiles: 256, or 128 when the environment
+// variable KQ_TRAIL_TILE_N says so (a tuning switch; both give the same sums per tile).
+int long_tile_n() {
+    static const int n = [] {
+        const char* e = std::getenv("KQ_TRAIL_TILE_N");
+        return (e && std::atoi(e) == 128) ? 128 : 256;
+    }();
+    return n;
+}
 
 struct Grid {
     float scale, zero;
@@ -77,7 +89,7 @@ __global__ void rowgrid_kernel(const float* __restrict__ W, int64_t d_out, int64
     mn = warp_min(mn);
     mx = warp_max(mx);
     const Grid g = make_grid(mn, mx, static_cast<float>((1 << bits) - 1));
-    if (lane == 0) {
+    if (lane == 0 && KQ_IN_RANGE(r, d_out)) {
         scale[r] = g.scale;
         zero[r] = static_cast<int32_t>(g.zero);
         gscale[r] = g.scale;
@@ -136,7 +148,7 @@ __global__ void pack_r_kernel(const float* __restrict__ Lt, int64_t n, float* __
     float* out = Rp + static_cast<int64_t>(blockIdx.z) * BLK * BLK;
     for (int r = threadIdx.y; r < 32; r += 8) {
         const int j = j0 + r, c = c0 + threadIdx.x;
-        out[j * BLK + pos_of(c)] = t[threadIdx.x][r];
+        if (KQ_IN_RANGE(j * BLK + pos_of(c), BLK * BLK)) out[j * BLK + pos_of(c)] = t[threadIdx.x][r];
     }
 }
 
@@ -152,7 +164,8 @@ __global__ void pack_rq_mma_kernel(const float* __restrict__ Lt, int64_t n, floa
     for (int r = threadIdx.y; r < 32; r += 8) {
         const int c = c0 + r, k = k0 + threadIdx.x;
         const int64_t lr = i1 + c, lc = i0 + k;
-        out[c * BLK + (k ^ (4 * (c & 7)))] = (lr < n && lc < n) ? Lt[lr * n + lc] : 0.0f;
+        if (KQ_IN_RANGE(c * BLK + (k ^ (4 * (c & 7))), BLK * BLK))
+            out[c * BLK + (k ^ (4 * (c & 7)))] = (lr < n && lc < n) ? Lt[lr * n + lc] : 0.0f;
     }
 }
 
@@ -242,7 +255,7 @@ __device__ __forceinline__ void load_cols(const float* __restrict__ W, int64_t r
 template <bool VEC>
 __device__ __forceinline__ void store_cols(float* W, int64_t r, int64_t d_out, int64_t d_in, int64_t i0, int cb,
                                            int nb, const float (&w)[CPL]) {
-    if (r >= d_out) return;
+    if (r >= d_out || !KQ_IN_RANGE(r * d_in + i0 + cb + min(CPL, nb - cb) - 1, d_out * d_in)) return;
     float* dst = W + r * d_in + i0 + cb;
     if (VEC && cb + CPL <= nb) {
 #pragma unroll
@@ -295,7 +308,7 @@ __global__ void __launch_bounds__(HASP ? OBS_THREADS_P : OBS_THREADS, HASP ? 1 :
     uint8_t* __restrict__ codes, float* __restrict__ scale, int32_t* __restrict__ zero,
     float* __restrict__ E, float* __restrict__ pre_q, float* __restrict__ Eh, float* __restrict__ El,
     const float* __restrict__ Pp, float* __restrict__ Q, float* __restrict__ Qh, float* __restrict__ Ql,
-    const float* __restrict__ Rq, int fused_mma) {
+    const float* __restrict__ Rq, int fused_mma, int* info) {
     extern __shared__ __align__(16) float Rs[];   // [BLK][BLK], packed (pack_r_kernel); then P's
     float* Ps = Rs + BLK * BLK;
     const bool fused = !HASP && Rq != nullptr;
@@ -384,7 +397,7 @@ __global__ void __launch_bounds__(HASP ? OBS_THREADS_P : OBS_THREADS, HASP ? 1 :
                     mx = fmaxf(mx, w[t]);
                 }
             g = make_grid(group_min(mn), group_max(mx), maxq);
-            if (live && lp == 0) {
+            if (live && lp == 0 && KQ_IN_RANGE(r * ngroups + i0 / group, d_out * ngroups)) {
                 const int64_t gi = r * ngroups + i0 / group;
                 scale[gi] = g.scale;
                 zero[gi] = static_cast<int32_t>(g.zero);
@@ -394,6 +407,7 @@ __global__ void __launch_bounds__(HASP ? OBS_THREADS_P : OBS_THREADS, HASP ? 1 :
             g.zero = live ? gzero[r] : 0.0f;
         }
         const float ys = div_recip(g.scale);
+        bool finite = true;   // every value quantized in this row group was finite
         // The column steps of this row group; EXACT: IEEE divisions, else div_rn_fast, with
         // the return value telling whether every operand was inside its exact range.
         auto sweep = [&](auto exact_tag) -> bool {
@@ -419,6 +433,7 @@ __global__ void __launch_bounds__(HASP ? OBS_THREADS_P : OBS_THREADS, HASP ? 1 :
 #pragma unroll
                     for (int v = 0; v < NV; ++v) rv[v] = *reinterpret_cast<const float4*>(rr + 4 * slot_of(lp, v));
                     const float wj = __shfl_sync(0xffffffffu, w[jj], gbase | o);
+                    finite = finite & (fabsf(wj) <= 3.402823466e38f);
                     float q0;
                     if constexpr (EXACT) {
                         q0 = __fdiv_rn(wj, g.scale);
@@ -439,7 +454,8 @@ __global__ void __launch_bounds__(HASP ? OBS_THREADS_P : OBS_THREADS, HASP ? 1 :
                     }
                     e[jj] = err;
                     cq[jj >> 2] |= static_cast<uint32_t>(qq) << (8 * (jj & 3));
-                    if (pre_q && live && lp == o) pre_q[r * d_in + i0 + j] = wj;
+                    if (pre_q && live && lp == o && KQ_IN_RANGE(r * d_in + i0 + j, d_out * d_in))
+                        pre_q[r * d_in + i0 + j] = wj;
                     if constexpr (HASP) {
                         wq[jj] = wj;
                         const float* pr = Ps + j * BLK;
@@ -466,7 +482,7 @@ __global__ void __launch_bounds__(HASP ? OBS_THREADS_P : OBS_THREADS, HASP ? 1 :
                     wq[jj] = 0.0f;
                 }
             }
-            if (live && lp == o) {
+            if (live && lp == o && KQ_IN_RANGE(r * d_in + i0 + min(CPL * o + CPL, nb) - 1, d_out * d_in)) {
                 const int64_t ob = r * d_in + i0 + CPL * o;
                 if (VEC && CPL * o + CPL <= nb) {
 #pragma unroll
@@ -545,6 +561,7 @@ __global__ void __launch_bounds__(HASP ? OBS_THREADS_P : OBS_THREADS, HASP ? 1 :
                 load_cols<VEC>(W, r, d_out, d_in, i0, cb, nb, w);
             sweep(std::true_type{});
         }
+        if (!__all_sync(0xffffffffu, finite) && lane == 0) record_error(info, -KQ_ERR_NONFINITE);
     }
 }
 
@@ -583,7 +600,8 @@ __global__ void __launch_bounds__(G_THREADS, 2) trailing_kernel(float* __restric
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
                 const int rr = gt_row(ty, 4 * h + i), cc = gt_col<false>(tx, j);
-                if (rr < arows && cc < bcols) W[(r0 + rr) * d_in + c0 + cc] = __fsub_rn(wv[i][j], acc[4 * h + i][j]);
+                if (rr < arows && cc < bcols && KQ_IN_RANGE((r0 + rr) * d_in + c0 + cc, d_out * d_in))
+                    W[(r0 + rr) * d_in + c0 + cc] = __fsub_rn(wv[i][j], acc[4 * h + i][j]);
             }
     }
 }
@@ -594,7 +612,7 @@ __global__ void colloss_kernel(const float* __restrict__ E, int64_t d_out, int64
                                float* __restrict__ col_loss) {
     const int64_t j = static_cast<int64_t>(blockIdx.x) * CS_X + threadIdx.x;
     const double a = col_sumsq(E, d_out, d_in, j);
-    if (threadIdx.y == 0 && j < d_in) col_loss[j] = static_cast<float>(a);
+    if (threadIdx.y == 0 && j < d_in && KQ_IN_RANGE(j, d_in)) col_loss[j] = static_cast<float>(a);
 }
 
 struct ObsWs {
@@ -681,6 +699,8 @@ ObsWs carve(void* ws, int64_t d_out, int64_t d_in, int mode, bool with_p) {
 }
 
 }  // namespace
+
+KQ_DEBUG_UNIT(obs)
 }  // namespace kq
 
 using namespace kq;
@@ -824,18 +844,83 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
         if (hp)
             obs_block_kernel<true, true><<<static_cast<unsigned>(row_ctas), OBS_THREADS_P, 2 * BLK * BLK * 4, stream>>>(
                 W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q, o.Eh, o.El,
-                o.Pp + b * BLK * BLK, o.Q, o.Qh, o.Ql, nullptr, 0);
+                o.Pp + b * BLK * BLK, o.Q, o.Qh, o.Ql, nullptr, 0, info);
         else if (bvec)
             obs_block_kernel<true, false><<<static_cast<unsigned>(row_ctas), OBS_THREADS, mma_fused ? OBS_SMEM_MMA : BLK * BLK * 4,
                                              stream>>>(
                 W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q, o.Eh, o.El,
-                nullptr, nullptr, nullptr, nullptr, rq, mma_fused ? 1 : 0);
+                nullptr, nullptr, nullptr, nullptr, rq, mma_fused ? 1 : 0, info);
         else
             obs_block_kernel<false, false><<<static_cast<unsigned>(row_ctas), OBS_THREADS, BLK * BLK * 4, stream>>>(
                 W, d_out, d_in, rp, i0, bits, group, o.gscale, o.gzero, codes, scale, zero, o.E, pre_q, o.Eh, o.El,
-                nullptr, nullptr, nullptr, nullptr, rq, 0);
+                nullptr, nullptr, nullptr, nullptr, rq, 0, info);
     };
-    if (fuse && tc) {
+    // Two levels for the large layers on the tensor cores (super-panels of SPB blocks, the
+    // GPTQ lazy update grouped once more): inside a super-panel each block updates the next
+    // block column on the caller's stream and the rest of the super-panel's columns on the
+    // side stream (K = 128); after a super-panel's last block one update with the whole
+    // super-panel's K covers every column beyond it -- the next super-panel's columns on the
+    // caller's stream, the rest on the second side stream beside the next super-panel's
+    // blocks -- so each W tile beyond is read and written once per super-panel instead of
+    // once per block. Every column still receives the block updates in block order (the
+    // long update drains its accumulator into W one block's K at a time).
+    const bool two_level = tc && !hp && !fuse && nblk > SPB;
+    if (two_level) {
+        constexpr int64_t SPW = static_cast<int64_t>(SPB) * BLK;
+        const int bn = long_tile_n();
+        bool in_pending = false;    // the in-panel update of the previous block (side stream)
+        bool far_pending = false;   // the far update of the previous super-panel (second side stream)
+        cudaStream_t s_in = side ? side->s : stream;
+        cudaStream_t s_far = side ? side->s2 : stream;
+        for (int64_t b = 0; b < nblk; ++b) {
+            const int64_t i0 = b * BLK;
+            block_launch(b, nullptr);
+            KQ_LAUNCH_CHECK("obs_block_kernel");
+            const int64_t nb0 = i0 + BLK;                               // next block column
+            if (nb0 >= d_in) break;
+            const int64_t sp0 = (b / SPB) * SPW;                         // this super-panel
+            const int64_t spe = std::min(d_in, sp0 + SPW);
+            if (side) KQ_CUDA(cudaEventRecord(side->ev[0], stream));     // E of this block ready
+            kq_status st;
+            if (nb0 < spe) {
+                if (in_pending) {   // it wrote the next block column too
+                    KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));
+                    in_pending = false;
+                }
+                const int64_t nb1 = std::min(spe, nb0 + BLK);
+                st = trailing(i0, BLK, nb0, nb1, stream);
+                if (st != KQ_OK) return st;
+                if (nb1 < spe) {
+                    if (side) KQ_CUDA(cudaStreamWaitEvent(s_in, side->ev[0], 0));
+                    st = trailing(i0, BLK, nb1, spe, s_in);
+                    if (st != KQ_OK) return st;
+                    if (side) {
+                        KQ_CUDA(cudaEventRecord(side->ev[1], s_in));
+                        in_pending = true;
+                    }
+                }
+            } else {
+                const int64_t sp1 = std::min(d_in, spe + SPW);           // the next super-panel's end
+                if (far_pending) {   // the previous super-panel's far update wrote these columns
+                    KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[0], 0));
+                    far_pending = false;
+                }
+                st = trail_tc_long(maps, d_out, d_in, sp0, static_cast<int>(spe - sp0), spe, sp1, bn, info, stream);
+                if (st != KQ_OK) return st;
+                if (sp1 < d_in) {
+                    if (side) KQ_CUDA(cudaStreamWaitEvent(s_far, side->ev[0], 0));
+                    st = trail_tc_long(maps, d_out, d_in, sp0, static_cast<int>(spe - sp0), sp1, d_in, bn, info, s_far);
+                    if (st != KQ_OK) return st;
+                    if (side) {
+                        KQ_CUDA(cudaEventRecord(side->ev2[0], s_far));
+                        far_pending = true;
+                    }
+                }
+            }
+        }
+        if (in_pending) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));
+        if (far_pending) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[0], 0));
+    } else if (fuse && tc) {
         // Pairs of blocks (2s, 2s + 1). Block 2s + 1 applies block 2s's update of its columns
         // itself; after the pair, its update (K = 256, still applied 128 of K at a time) of
         // the next pair's columns runs on the caller's stream just before the next pair,

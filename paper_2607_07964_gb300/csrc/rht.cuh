@@ -198,6 +198,54 @@ __device__ __forceinline__ void block_rht_inplace(float* v, int n, int lgP, bool
     }
 }
 
+// y = H_28 x by the block structure of Paley's construction: with s_a = x_2a + x_2a+1 and
+// d_a = x_2a - x_2a+1 (a < 14), every nonzero entry c of the conference matrix C contributes
+// c [[1, 1], [1, -1]], i.e. c s_a to y_2r and c d_a to y_2r+1, and the zero diagonal entry
+// [[1, -1], [-1, -1]], i.e. d_r to y_2r and -s_r to y_2r+1. So y_2r = (C s)_r + d_r and
+// y_2r+1 = (C d)_r - s_r: 390 additions instead of the 756 of the dense +-1 sums. The
+// signs of C come from the same constexpr table (row masks of H_28: the sign of entry
+// (2r, 2a) is c for a != r). out(r, y_r) receives every output.
+template <int R, uint32_t M>
+__device__ __forceinline__ float conf_row_sum(const float (&v)[14]) {
+    float acc = 0.0f;
+#pragma unroll
+    for (int a = 0; a < 14; ++a)
+        if (a != R) acc = ((M >> (2 * a)) & 1u) ? acc - v[a] : acc + v[a];
+    return acc;
+}
+template <typename Out, int... R>
+__device__ __forceinline__ void mix28_paley_rows(const float (&sv)[14], const float (&dv)[14], Out& out,
+                                                 std::integer_sequence<int, R...>) {
+    ((out(2 * R, conf_row_sum<R, kH28.m[2 * R]>(sv) + dv[R]),
+      out(2 * R + 1, conf_row_sum<R, kH28.m[2 * R]>(dv) - sv[R])),
+     ...);
+}
+template <typename Out>
+__device__ __forceinline__ void mix28_paley(const float (&x)[28], Out out) {
+    float sv[14], dv[14];
+#pragma unroll
+    for (int a = 0; a < 14; ++a) {
+        sv[a] = x[2 * a] + x[2 * a + 1];
+        dv[a] = x[2 * a] - x[2 * a + 1];
+    }
+    mix28_paley_rows(sv, dv, out, std::make_integer_sequence<int, 14>{});
+}
+// The block structure above, checked on the table at compile time.
+constexpr bool h28_has_paley_blocks() {
+    for (int r = 0; r < 14; ++r)
+        for (int a = 0; a < 14; ++a) {
+            const int e00 = h28_entry(2 * r, 2 * a), e01 = h28_entry(2 * r, 2 * a + 1);
+            const int e10 = h28_entry(2 * r + 1, 2 * a), e11 = h28_entry(2 * r + 1, 2 * a + 1);
+            if (a == r) {
+                if (e00 != 1 || e01 != -1 || e10 != -1 || e11 != -1) return false;
+            } else if (e01 != e00 || e10 != e00 || e11 != -e00) {
+                return false;
+            }
+        }
+    return true;
+}
+static_assert(h28_has_paley_blocks(), "H_28 must have the 2 x 2 block structure mix28_paley relies on");
+
 // ---------------------------------------------------------------------------------------
 // Walsh-Hadamard transform of n = 2^LG values held in registers, 16 per thread (n / 16
 // threads, LG in [9, 14]). Phase q transforms the index bits in rr_mask(LG, q); thread t

@@ -19,6 +19,7 @@
 //   * every mbarrier wait is bounded (kq::mbar_wait); a timeout is reported as
 //     -KQ_ERR_TIMEOUT in *info and the CTA drains its own copies and MMAs before exit.
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 
 #include "kq_common.cuh"
@@ -42,16 +43,97 @@ constexpr uint32_t TMEM_COLS = 512;
 constexpr uint32_t LBO = BOX_BYTES;   // next 64 features
 constexpr uint32_t SBO = 1024;        // next 8 tokens
 
-__device__ __forceinline__ void tile_of(int bid, int n_row_tiles, int* ti, int* tj) {
-    int j = 0;
-    for (;;) {
-        int cnt = n_row_tiles - 2 * j;
-        if (bid < cnt) break;
-        bid -= cnt;
-        ++j;
+// Tile order of the lower triangle (tile (i, j) needs i >= 2 j): bands of BAND column tiles,
+// each band row by row, BAND tiles per row once past the diagonal. The CTAs resident at
+// one time (about one per SM) then cover ~19 row panels x 8 column panels, i.e. ~4.5k of
+// the d features, instead of one column panel and ~150 row panels (~20k features): every
+// resident set streams all T tokens of its features from HBM, so this is what keeps a
+// large factor (d = 14336, 28672) from re-reading X several times over.
+constexpr int BAND = 8;
+// Tiles of a band's first r rows past its start (row k of the band holds min(w, k / 2 + 1)).
+__host__ __device__ constexpr int band_tiles(int r, int w) {
+    return r <= 2 * w ? (r / 2) * (r / 2 + 1) + (r & 1) * (r / 2 + 1) : w * (w + 1) + (r - 2 * w) * w;
+}
+__device__ __forceinline__ void tile_of(int bid, int n_row_tiles, int n_col_tiles, int* ti, int* tj) {
+    for (int j0 = 0; j0 < n_col_tiles; j0 += BAND) {
+        const int w = min(BAND, n_col_tiles - j0);
+        const int rows = n_row_tiles - 2 * j0;
+        const int cnt = band_tiles(rows, w);
+        if (bid >= cnt) {
+            bid -= cnt;
+            continue;
+        }
+        int k = 0;
+        if (bid >= w * (w + 1) && rows > 2 * w) {   // past the triangle: w tiles a row
+            k = 2 * w + (bid - w * (w + 1)) / w;
+            bid = (bid - w * (w + 1)) % w;
+        } else {
+            while (bid >= min(w, k / 2 + 1)) bid -= min(w, k++ / 2 + 1);
+        }
+        *ti = 2 * j0 + k;
+        *tj = j0 + bid;
+        return;
     }
-    *tj = j;
-    *ti = 2 * j + bid;
+    *ti = 0;   // not reached for bid < the number of lower tiles
+    *tj = 0;
+}
+
+// Pairs of row tiles (2m, 2m + 1) hold the same lower-triangle columns (j <= m), so a
+// cluster of two CTAs takes one pair and the column panel j they share: each CTA loads half
+// of the panel's operand boxes and multicasts them to both, halving the L2 reads of the
+// larger operand. Pairs in the same banded order as the tiles (BAND columns a band, one row
+// pair after another).
+__device__ __forceinline__ void pair_of(int pid, int n_row_pairs, int n_col_tiles, int* m, int* tj) {
+    for (int j0 = 0; j0 < n_col_tiles; j0 += BAND) {
+        const int w = min(BAND, n_col_tiles - j0);
+        const int rows = n_row_pairs - j0;
+        const int tri = w * (w + 1) / 2;
+        const int cnt = rows <= w ? rows * (rows + 1) / 2 : tri + (rows - w) * w;
+        if (pid >= cnt) {
+            pid -= cnt;
+            continue;
+        }
+        int k = 0;
+        if (pid >= tri && rows > w) {   // past the triangle: w pairs a row pair
+            k = w + (pid - tri) / w;
+            pid = (pid - tri) % w;
+        } else {
+            while (pid >= min(w, k + 1)) pid -= min(w, k++ + 1);
+        }
+        *m = j0 + k;
+        *tj = j0 + pid;
+        return;
+    }
+    *m = 0;   // not reached for pid < the number of pairs
+    *tj = 0;
+}
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// TMA load of one box into the same shared-memory offset of every CTA in `mask`, each
+// CTA's mbarrier at the offset of `bar` receiving the bytes it got.
+__device__ __forceinline__ void tma_load_2d_mc(void* dst, const CUtensorMap* m, uint64_t* bar, int x, int y,
+                                               uint16_t mask) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
+        " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(m)), "r"(smem_u32(bar)), "r"(x), "r"(y), "h"(mask)
+        : "memory");
+}
+// Arrive once on `bar` (same offset) in every CTA of `mask` when this thread's issued MMAs
+// have completed.
+__device__ __forceinline__ void tc_commit_mc(uint64_t* bar, uint16_t mask) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+            smem_u32(bar)),
+        "h"(mask)
+        : "memory");
 }
 
 __device__ __forceinline__ bool wait_noabort(uint64_t* bar, uint32_t parity) {
@@ -64,7 +146,7 @@ __device__ __forceinline__ bool wait_noabort(uint64_t* bar, uint32_t parity) {
 //     operand box comes from map a0.
 //   CROSS = true: D (+)= (A_hi + A_lo)^T B over all tiles, no symmetry: the K loop runs over
 //     the T tokens of the pair (a0 = A_hi, b) and then over the pair (a1 = A_lo, b).
-template <bool CROSS>
+template <bool CROSS, bool PAIR = false>
 __device__ __forceinline__ void gram_tc_body(const CUtensorMap* a0, const CUtensorMap* a1,
                                              const CUtensorMap* bmap, float* __restrict__ H, int d,
                                              int T, int n_row_tiles, int chunk_stages, int accumulate,
@@ -83,11 +165,16 @@ __device__ __forceinline__ void gram_tc_body(const CUtensorMap* a0, const CUtens
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     int ti, tj;
+    const uint32_t rank = PAIR ? cluster_rank() : 0u;
     if (CROSS) {
         ti = static_cast<int>(blockIdx.x) % n_row_tiles;
         tj = static_cast<int>(blockIdx.x) / n_row_tiles;
+    } else if (PAIR) {
+        int m;
+        pair_of(static_cast<int>(blockIdx.x >> 1), n_row_tiles / 2, (d + BN - 1) / BN, &m, &tj);
+        ti = 2 * m + static_cast<int>(rank);
     } else {
-        tile_of(blockIdx.x, n_row_tiles, &ti, &tj);
+        tile_of(blockIdx.x, n_row_tiles, (d + BN - 1) / BN, &ti, &tj);
     }
     const int i0 = ti * BM;
     const int j0 = tj * BN;
@@ -98,7 +185,7 @@ __device__ __forceinline__ void gram_tc_body(const CUtensorMap* a0, const CUtens
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&full[s], 1);
-            mbar_init(&empty[s], 1);
+            mbar_init(&empty[s], PAIR ? 2 : 1);   // with a pair: both CTAs' MMAs release a stage
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&tfull[b], 1);
@@ -112,6 +199,8 @@ __device__ __forceinline__ void gram_tc_body(const CUtensorMap* a0, const CUtens
         tmem_alloc(tmem_slot, TMEM_COLS);
         tmem_relinquish();
     }
+    // the partner's barriers must be initialized before any copy or arrive reaches them
+    if (PAIR) cluster_sync_all();
     if (warp == 0 && lane == 0) {
         tma_prefetch_desc(a0);
         if (CROSS) {
@@ -141,9 +230,15 @@ __device__ __forceinline__ void gram_tc_body(const CUtensorMap* a0, const CUtens
                 const CUtensorMap* bm = CROSS ? bmap : a0;
                 tma_load_2d(a, am, &full[s], i0, y);
                 tma_load_2d(a + BOX_BYTES, am, &full[s], i0 + 64, y);
+                if (PAIR) {   // this CTA's half of the column panel, into both CTAs
 #pragma unroll
-                for (int q = 0; q < 4; ++q)
-                    tma_load_2d(b + q * BOX_BYTES, bm, &full[s], j0 + 64 * q, y);
+                    for (int q = 2 * static_cast<int>(rank); q < 2 * static_cast<int>(rank) + 2; ++q)
+                        tma_load_2d_mc(b + q * BOX_BYTES, bm, &full[s], j0 + 64 * q, y, 0x3);
+                } else {
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+                        tma_load_2d(b + q * BOX_BYTES, bm, &full[s], j0 + 64 * q, y);
+                }
                 issued = k + 1;
             }
             // Drain: every issued load must have landed before the CTA may exit.
@@ -178,7 +273,10 @@ __device__ __forceinline__ void gram_tc_body(const CUtensorMap* a0, const CUtens
                         const uint64_t bd = smem_desc_sw128(b + k16 * 2048, LBO, SBO);
                         tc_mma_f16(dt, ad, bd, idesc, (kk > 0 || k16 > 0) ? 1u : 0u);
                     }
-                    tc_commit(&empty[s]);
+                    if (PAIR)
+                        tc_commit_mc(&empty[s], 0x3);   // the stage is free once both CTAs are done
+                    else
+                        tc_commit(&empty[s]);
                 }
                 if (ok) tc_commit(&tfull[buf]);
             }
@@ -249,7 +347,8 @@ __device__ __forceinline__ void gram_tc_body(const CUtensorMap* a0, const CUtens
 #pragma unroll
                     for (int m = 0; m < 4; ++m) {
                         const int col = cbase + lane + 32 * m;
-                        if (rr < d && col < d && (CROSS || col <= rr)) {
+                        if (rr < d && col < d && (CROSS || col <= rr) &&
+                            KQ_IN_RANGE(static_cast<int64_t>(rr) * d + col, static_cast<int64_t>(d) * d)) {
                             const float v = st[(r8 + u) * SLD + lane + 32 * m] + old[u][m];
                             H[static_cast<int64_t>(rr) * d + col] = v;
                             st[(r8 + u) * SLD + lane + 32 * m] = v;
@@ -262,13 +361,16 @@ __device__ __forceinline__ void gram_tc_body(const CUtensorMap* a0, const CUtens
 #pragma unroll 4
                 for (int i = 0; i < 128; ++i) {
                     const int col = cbase + i;
-                    if (col < d && col < row) H[static_cast<int64_t>(col) * d + row] = st[lane * SLD + i];
+                    if (col < d && col < row && KQ_IN_RANGE(static_cast<int64_t>(col) * d + row, static_cast<int64_t>(d) * d))
+                        H[static_cast<int64_t>(col) * d + row] = st[lane * SLD + i];
                 }
             }
         }
     }
 
     __syncthreads();
+    // neither CTA of a pair leaves while the other may still send it copies or arrivals
+    if (PAIR) cluster_sync_all();
     if (*abort_flag && threadIdx.x == 0) record_error(info, -KQ_ERR_TIMEOUT);
     if (warp == 1) {
         tc_fence_after();
@@ -280,6 +382,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 syrk_tc_kernel(const __grid_constant__ CUtensorMap tmap, float* __restrict__ H, int d, int T,
                int n_row_tiles, int chunk_stages, int accumulate, int* info) {
     gram_tc_body<false>(&tmap, &tmap, &tmap, H, d, T, n_row_tiles, chunk_stages, accumulate, info);
+}
+
+// The same with clusters of two CTAs sharing their column panel (pair_of); grid = 2 x pairs.
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
+syrk_tc_pair_kernel(const __grid_constant__ CUtensorMap tmap, float* __restrict__ H, int d, int T,
+                    int n_row_tiles, int chunk_stages, int accumulate, int* info) {
+    gram_tc_body<false, true>(&tmap, &tmap, &tmap, H, d, T, n_row_tiles, chunk_stages, accumulate, info);
 }
 
 __global__ void __launch_bounds__(NUM_THREADS, 1)
@@ -391,6 +500,16 @@ kq_status make_bf16_map(CUtensorMap* m, const uint16_t* base, int64_t d, int64_t
     return KQ_OK;
 }
 
+// Clusters of two for the SYRK unless the environment variable KQ_SYRK_PAIRS is 0 (a
+// switch for comparing the two launch forms; both compute the same sums per tile).
+bool syrk_pairs_enabled() {
+    static const bool on = [] {
+        const char* e = std::getenv("KQ_SYRK_PAIRS");
+        return !(e && e[0] == '0');
+    }();
+    return on;
+}
+
 }  // namespace
 
 kq_status launch_trace(const float* H, int64_t n, double* out, cudaStream_t stream) {
@@ -399,6 +518,7 @@ kq_status launch_trace(const float* H, int64_t n, double* out, cudaStream_t stre
     return KQ_OK;
 }
 
+KQ_DEBUG_UNIT(syrk)
 }  // namespace kq
 
 extern "C" kq_status kq_accum_factor(const uint16_t* A, int64_t T, int64_t d, int64_t lda,
@@ -425,6 +545,8 @@ extern "C" kq_status kq_accum_factor(const uint16_t* A, int64_t T, int64_t d, in
         KQ_TRY(once_per_device(attr_set, [&]() -> kq_status {
             KQ_CUDA(cudaFuncSetAttribute(syrk_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          SMEM_BYTES));
+            KQ_CUDA(cudaFuncSetAttribute(syrk_tc_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         SMEM_BYTES));
             return KQ_OK;
         }));
         const int n_row = static_cast<int>(cdiv(d, BM));
@@ -432,9 +554,16 @@ extern "C" kq_status kq_accum_factor(const uint16_t* A, int64_t T, int64_t d, in
         int64_t tiles = 0;
         for (int j = 0; j < n_col; ++j) tiles += (n_row - 2 * j > 0) ? n_row - 2 * j : 0;
         const int chunk_stages = KQ_SYRK_CHUNK_TOKENS / BK;
-        syrk_tc_kernel<<<static_cast<unsigned>(tiles), NUM_THREADS, SMEM_BYTES, stream>>>(
-            tmap, H, static_cast<int>(d), static_cast<int>(T), n_row, chunk_stages, accumulate, info);
-        KQ_LAUNCH_CHECK("syrk_tc_kernel");
+        if (n_row % 2 == 0 && syrk_pairs_enabled()) {
+            // every row tile has its partner (2m, 2m + 1): clusters of two share the column panel
+            syrk_tc_pair_kernel<<<static_cast<unsigned>(tiles), NUM_THREADS, SMEM_BYTES, stream>>>(
+                tmap, H, static_cast<int>(d), static_cast<int>(T), n_row, chunk_stages, accumulate, info);
+            KQ_LAUNCH_CHECK("syrk_tc_pair_kernel");
+        } else {
+            syrk_tc_kernel<<<static_cast<unsigned>(tiles), NUM_THREADS, SMEM_BYTES, stream>>>(
+                tmap, H, static_cast<int>(d), static_cast<int>(T), n_row, chunk_stages, accumulate, info);
+            KQ_LAUNCH_CHECK("syrk_tc_kernel");
+        }
     }
     if (trace) return launch_trace(H, d, trace, stream);
     return KQ_OK;

@@ -36,14 +36,21 @@ constexpr int TNSLAB = TK / TBK;         // 4
 constexpr int T_THREADS = 320;           // 10 warps: TMA, MMA, 8 epilogue
 constexpr int A_SLAB = TBM * TBK * 4;    // 16 KB
 
-template <int BN, int STAGES>
+// RED = false: the tile of W comes in by TMA, the epilogue subtracts the accumulator from
+// it in shared memory and a TMA store writes it back. RED = true: W never enters shared
+// memory; the epilogue stages -accumulator one 128 x 32 box at a time (one staging box per
+// column half) and a TMA reduce-add applies it to W in global memory, which leaves room for
+// a deeper operand ring or wider tiles.
+template <int BN, int STAGES, bool RED = false>
 struct TrailCfg {
     static constexpr int B_SLAB = BN * TBK * 4;                    // 16 KB for BN = 128
     static constexpr int STAGE = 2 * A_SLAB + 2 * B_SLAB;          // hi + lo of both
-    static constexpr int WTILE = TBM * BN * 4;                     // the tile of W (64 KB)
+    static constexpr int WBOX = TBM * 32 * 4;                      // one 128 x 32 box of W (16 KB)
+    static constexpr int WTILE = RED ? 2 * WBOX : TBM * BN * 4;    // staging boxes, or the tile of W
     static constexpr int SMEM = STAGES * STAGE + WTILE + 1024 + 256;
     static_assert(2 * BN <= 512, "two accumulators must fit in TMEM");
-    static_assert(BN % 32 == 0, "W moves in 32-column boxes");
+    static_assert(BN % 64 == 0, "W moves in 32-column boxes, two column halves");
+    static_assert(SMEM <= 232448, "dynamic shared memory above the per-CTA limit");
 };
 
 __device__ __forceinline__ bool wait_quiet(uint64_t* bar, uint32_t parity) {
@@ -63,7 +70,7 @@ __device__ __forceinline__ bool wait_quiet(uint64_t* bar, uint32_t parity) {
 struct TileSet {
     int mode;
     int n_tiles;
-    int n_col_tiles, cb, i0, pslab;                   // mode 0
+    int n_col_tiles, cb, i0, pslab, ce;               // mode 0 (ce: end of the column range)
     int nbk, a_j0, a_j1, n_a, b_i0, b_i1, b_j1, kx;   // mode 1
 };
 
@@ -93,7 +100,7 @@ __device__ __forceinline__ void tile_at(const TileSet& ts, int t, int bn, int* r
     *alt = true;
 }
 
-template <int BN, int TSTAGES>
+template <int BN, int TSTAGES, bool RED>
 __global__ void __launch_bounds__(T_THREADS, 1)
 trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__ CUtensorMap mEl,
                 const __grid_constant__ CUtensorMap mRh, const __grid_constant__ CUtensorMap mRl,
@@ -103,8 +110,8 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
                 int nslab, int drain, int* info) {
     const int n_tiles = ts.n_tiles;
     const int xk = ts.mode == 0 ? ts.i0 : ts.kx;
-    using C = TrailCfg<BN, TSTAGES>;
-    constexpr int WBOX = TBM * 32 * 4;     // one 128-row x 32-column box of W (16 KB)
+    using C = TrailCfg<BN, TSTAGES, RED>;
+    constexpr int WBOX = C::WBOX;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -172,12 +179,16 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
                 bool alt;
                 tile_at(ts, t, BN, &r0, &c0, &alt);
                 const CUtensorMap* wm = alt ? &mW2 : &mW;
-                // the tile of W, once the previous tile has been stored from the buffer
-                if (!mbar_wait(wfree, (static_cast<uint32_t>(li) & 1u) ^ 1u, abort_flag)) break;
-                mbar_arrive_expect_tx(wfull, C::WTILE);
+                if constexpr (!RED) {
+                    // the tile of W, once the previous tile has been stored from the buffer
+                    if (!mbar_wait(wfree, (static_cast<uint32_t>(li) & 1u) ^ 1u, abort_flag)) break;
+                    mbar_arrive_expect_tx(wfull, C::WTILE);
 #pragma unroll
-                for (int j = 0; j < BN / 32; ++j) tma_load_2d(wtile + j * WBOX, wm, wfull, c0 + 32 * j, r0);
-                w_issued = li + 1;
+                    for (int j = 0; j < BN / 32; ++j) tma_load_2d(wtile + j * WBOX, wm, wfull, c0 + 32 * j, r0);
+                    w_issued = li + 1;
+                } else {
+                    (void)wm;
+                }
                 for (int s = 0; s < nslab; ++s, ++k) {
                     const int st = k % TSTAGES;
                     const uint32_t u = static_cast<uint32_t>(k / TSTAGES);
@@ -255,12 +266,67 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
         // memory as 128-byte swizzled rows (16-byte chunk c of row r at c ^ (r & 7)), so the
         // float4 accesses of 8 consecutive rows hit distinct banks.
         constexpr int HALF = BN / 2;
+        constexpr int PIECES = HALF / 32;       // 32-column boxes per half
         const int q = warp & 3;                 // TMEM lane quadrant this warp may access
         const int h = (warp - 2) >> 2;          // which half of the columns
         const int r = q * 32 + lane;            // row within the tile
+        const bool issuer = RED && (warp == 2 + 4 * h) && lane == 0;
         int li = 0, cc = 0;
         bool ok = true;
         for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++li) {
+            if constexpr (RED) {
+                int r0, c0;
+                bool alt;
+                tile_at(ts, t, BN, &r0, &c0, &alt);
+                const CUtensorMap* wm = alt ? &mW2 : &mW;
+                uint8_t* stg = wtile + h * WBOX;
+                for (int s0 = 0; s0 < nslab; s0 += drain, ++cc) {
+                    const int buf = cc & 1;
+                    ok = mbar_wait(&tfull[buf], (static_cast<uint32_t>(cc) >> 1) & 1u, abort_flag);
+                    ok = __all_sync(0xffffffffu, ok) && !*abort_flag;
+                    // every warp of this half leaves together (the named barriers below)
+                    ok = named_bar_all(1 + h, 128, ok);
+                    if (!ok) break;
+                    tc_fence_after();
+                    const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) +
+                                           static_cast<uint32_t>(buf * BN + h * HALF);
+#pragma unroll 1
+                    for (int p = 0; p < PIECES; ++p) {
+                        const int x = c0 + h * HALF + 32 * p;
+                        float v[32];
+                        tmem_ld32(taddr + static_cast<uint32_t>(p * 32), v);
+                        tc_wait_ld();
+                        if (p == PIECES - 1) {   // the accumulator may be reused
+                            tc_fence_before();
+                            __syncwarp();
+                            if (lane == 0) mbar_arrive(&tempty[buf]);
+                        }
+                        if (x >= ts.ce) continue;   // a box wholly past the range (same for the half)
+                        // -acc as one 128 x 32 box, 128-byte swizzled like the tensor map
+                        float4* rowp = reinterpret_cast<float4*>(stg + r * 128);
+#pragma unroll
+                        for (int c = 0; c < 8; ++c)
+                            rowp[c ^ (r & 7)] = make_float4(-v[4 * c], -v[4 * c + 1], -v[4 * c + 2], -v[4 * c + 3]);
+                        fence_proxy_async();
+                        named_bar_sync(1 + h, 128);
+                        if (issuer) {
+                            // the same box of the previous chunk must have landed first, so
+                            // that every element takes its block updates in order (a half
+                            // cut short by the range end commits fewer boxes a chunk: wait
+                            // for all of them)
+                            if (c0 + h * HALF + HALF <= ts.ce)
+                                bulk_wait_le<PIECES - 1>();
+                            else
+                                bulk_wait_le<0>();
+                            tma_reduce_add_2d(wm, stg, x, r0);
+                            bulk_commit();
+                            bulk_wait_read0();
+                        }
+                        named_bar_sync(1 + h, 128);   // the staging box is free again
+                    }
+                }
+                continue;
+            }
             ok = mbar_wait(wfull, static_cast<uint32_t>(li) & 1u, abort_flag);
             ok = __all_sync(0xffffffffu, ok) && !*abort_flag;
             if (!ok) break;
@@ -309,7 +375,7 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
                 }
             }
         }
-        if (warp == 2 && lane == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+        if ((warp == 2 || (RED && warp == 6)) && lane == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
     }
 
     tc_fence_before();
@@ -327,6 +393,7 @@ __global__ void split_tf32_kernel(const float* __restrict__ src, int64_t n, floa
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const float x = src[i];
         const float h = tf32_hi(x);
+        if (!KQ_IN_RANGE(i, n)) continue;
         hi[i] = h;
         lo[i] = x - h;
     }
@@ -388,6 +455,8 @@ kq_status TrailMaps::init(const float* E_hi, const float* E_lo, const float* Lt_
     if ((st = make_f32_map(&rl_narrow, Lt_lo, d_in, d_in, 128)) != KQ_OK) return st;
     if ((st = make_f32_map(&rh64, Lt_hi, d_in, d_in, 64)) != KQ_OK) return st;
     if ((st = make_f32_map(&rl64, Lt_lo, d_in, d_in, 64)) != KQ_OK) return st;
+    if ((st = make_f32_map(&rh256, Lt_hi, d_in, d_in, 256)) != KQ_OK) return st;
+    if ((st = make_f32_map(&rl256, Lt_lo, d_in, d_in, 256)) != KQ_OK) return st;
     return KQ_OK;
 }
 
@@ -409,11 +478,11 @@ namespace {
 template <int BN>
 kq_status launch_trail(const TrailMaps& m, const CUtensorMap& rh, const CUtensorMap& rl, int64_t d_out, int64_t i0,
                        int64_t cb, int64_t ce, bool with_p, int kslabs, int* info, cudaStream_t stream) {
-    using Cfg = TrailCfg<BN, 2>;
+    using Cfg = TrailCfg<BN, 2, false>;
     static std::atomic<uint64_t> attr{0};
     KQ_TRY(once_per_device(attr, [&]() -> kq_status {
-        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<BN, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
-        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<BN, 2>, cudaFuncAttributePreferredSharedMemoryCarveout,
+        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<BN, 2, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
+        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<BN, 2, false>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                      cudaSharedmemCarveoutMaxShared));
         return KQ_OK;
     }));
@@ -426,9 +495,10 @@ kq_status launch_trail(const TrailMaps& m, const CUtensorMap& rh, const CUtensor
     ts.cb = static_cast<int>(cb);
     ts.i0 = static_cast<int>(i0);
     ts.pslab = with_p ? kslabs : 1 << 30;
+    ts.ce = static_cast<int>(ce);
     // the accumulator goes into W every 128 of K (one block's update at a time, as the
     // per-block schedule does); with P after the E and P halves of one block together
-    trail_tc_kernel<BN, 2><<<static_cast<unsigned>(std::min(ts.n_tiles, num_sms())), T_THREADS, Cfg::SMEM, stream>>>(
+    trail_tc_kernel<BN, 2, false><<<static_cast<unsigned>(std::min(ts.n_tiles, num_sms())), T_THREADS, Cfg::SMEM, stream>>>(
         m.eh, m.el, rh, rl, with_p ? m.qh : m.eh, with_p ? m.ql : m.el, with_p ? m.ph : rh, with_p ? m.pl : rl, m.w, m.w,
         ts, with_p ? 2 * kslabs : kslabs, with_p ? 2 * kslabs : TNSLAB, info);
     KQ_LAUNCH_CHECK("trail_tc_kernel");
@@ -457,6 +527,54 @@ kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, in
     return launch_trail<128>(m, m.rh_narrow, m.rl_narrow, d_out, i0, cb, ce, with_p, kb / TBK, info, stream);
 }
 
+namespace {
+template <int BN, int STAGES>
+kq_status launch_trail_red(const TrailMaps& m, const CUtensorMap& rh, const CUtensorMap& rl, int64_t d_out,
+                           int64_t i0, int kb, int64_t cb, int64_t ce, int* info, cudaStream_t stream) {
+    using Cfg = TrailCfg<BN, STAGES, true>;
+    static std::atomic<uint64_t> attr{0};
+    KQ_TRY(once_per_device(attr, [&]() -> kq_status {
+        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<BN, STAGES, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     Cfg::SMEM));
+        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<BN, STAGES, true>,
+                                     cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared));
+        return KQ_OK;
+    }));
+    const int n_row = static_cast<int>(cdiv(d_out, TBM));
+    const int n_col = static_cast<int>(cdiv(ce - cb, BN));
+    TileSet ts{};
+    ts.mode = 0;
+    ts.n_tiles = n_row * n_col;
+    ts.n_col_tiles = n_col;
+    ts.cb = static_cast<int>(cb);
+    ts.i0 = static_cast<int>(i0);
+    ts.pslab = 1 << 30;
+    ts.ce = static_cast<int>(ce);
+    const int nslab = static_cast<int>(cdiv(kb, TBK));
+    trail_tc_kernel<BN, STAGES, true><<<static_cast<unsigned>(std::min(ts.n_tiles, num_sms())), T_THREADS, Cfg::SMEM,
+                                        stream>>>(m.eh, m.el, rh, rl, m.eh, m.el, rh, rl, m.w, m.w, ts, nslab, TNSLAB,
+                                                  info);
+    KQ_LAUNCH_CHECK("trail_tc_kernel");
+    return KQ_OK;
+}
+}  // namespace
+
+kq_status trail_tc_long(const TrailMaps& m, int64_t d_out, int64_t d_in, int64_t i0, int kb, int64_t cb, int64_t ce,
+                        int bn, int* info, cudaStream_t stream) {
+    if (kb < 1 || kb > 1024 || i0 + kb > d_in || (kb % TK != 0 && i0 + kb != d_in)) {
+        set_error("trailing update: K = %d from column %lld is not whole blocks of the super-panel", kb, (long long)i0);
+        return KQ_ERR_INVALID_ARG;
+    }
+    if ((bn != 128 && bn != 256) || ((ce - cb) % bn != 0 && ce != d_in)) {
+        set_error("trailing update: column range [%lld, %lld) is not whole %d-column tiles", (long long)cb,
+                  (long long)ce, bn);
+        return KQ_ERR_INVALID_ARG;
+    }
+    if (ce <= cb) return KQ_OK;
+    if (bn == 256) return launch_trail_red<256, 2>(m, m.rh256, m.rl256, d_out, i0, kb, cb, ce, info, stream);
+    return launch_trail_red<128, 3>(m, m.rh_narrow, m.rl_narrow, d_out, i0, kb, cb, ce, info, stream);
+}
+
 // ------------------------------------------------------------ Cholesky step updates
 kq_status CholTcMaps::init(float* A, float* Z, int64_t npad, int width, int nsets, float* const* split) {
     kq_status st;
@@ -473,10 +591,15 @@ kq_status CholTcMaps::init(float* A, float* Z, int64_t npad, int width, int nset
 
 kq_status chol_update_tc(const CholTcMaps& m, int set, int nbk, int a_j0, int a_j1, int b_i0, int b_i1, int b_j1,
                          int kx, int nslab, int* info, cudaStream_t stream) {
-    using Cfg = TrailCfg<128, 2>;
+    // 128 x 128 tiles, three-stage operand ring, the tiles of A and Z updated by TMA
+    // reduce-adds (no shared-memory copy of the tile)
+    using Cfg = TrailCfg<128, 3, true>;
     static std::atomic<uint64_t> attr{0};
     KQ_TRY(once_per_device(attr, [&]() -> kq_status {
-        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<128, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
+        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<128, 3, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     Cfg::SMEM));
+        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<128, 3, true>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                     cudaSharedmemCarveoutMaxShared));
         return KQ_OK;
     }));
     TileSet ts{};
@@ -489,13 +612,16 @@ kq_status chol_update_tc(const CholTcMaps& m, int set, int nbk, int a_j0, int a_
     ts.b_i1 = b_i1;
     ts.b_j1 = b_j1;
     ts.kx = kx;
+    ts.ce = 1 << 30;   // every tile lies inside the padded matrices
     ts.n_tiles = ts.n_a + ((b_i1 > b_i0 && b_j1 > 0) ? (b_i1 - b_i0) * b_j1 : 0);
     if (ts.n_tiles == 0) return KQ_OK;
-    trail_tc_kernel<128, 2><<<static_cast<unsigned>(std::min(ts.n_tiles, num_sms())), T_THREADS, Cfg::SMEM, stream>>>(
+    trail_tc_kernel<128, 3, true><<<static_cast<unsigned>(std::min(ts.n_tiles, num_sms())), T_THREADS, Cfg::SMEM, stream>>>(
         m.ch[set], m.cl[set], m.ch[set], m.cl[set], m.ch[set], m.cl[set], m.zh[set], m.zl[set], m.a, m.z, ts, nslab,
         TNSLAB, info);
     KQ_LAUNCH_CHECK("trail_tc_kernel");
     return KQ_OK;
 }
 
+
+KQ_DEBUG_UNIT(trail_tc)
 }  // namespace kq

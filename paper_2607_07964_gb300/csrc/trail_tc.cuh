@@ -29,6 +29,35 @@ __device__ __forceinline__ void tma_store_2d(const CUtensorMap* m, const void* s
                  "r"(smem_u32(src)), "r"(x), "r"(y)
                  : "memory");
 }
+// W[y:y+128, x:x+32] += the box in shared memory (element type and swizzle from the map;
+// rows and columns outside the matrix are skipped).
+__device__ __forceinline__ void tma_reduce_add_2d(const CUtensorMap* m, const void* src, int x, int y) {
+    asm volatile("cp.reduce.async.bulk.tensor.2d.global.shared::cta.add.tile.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                     reinterpret_cast<uint64_t>(m)),
+                 "r"(smem_u32(src)), "r"(x), "r"(y)
+                 : "memory");
+}
+// Wait until at most N of this thread's bulk groups are still pending (their writes done).
+template <int N>
+__device__ __forceinline__ void bulk_wait_le() { asm volatile("cp.async.bulk.wait_group %0;" ::"n"(N) : "memory"); }
+// Barrier `id` over n threads (whole warps; the non-.aligned form, so a warp may reach it
+// after a branch taken by some of its lanes).
+__device__ __forceinline__ void named_bar_sync(int id, int n) {
+    asm volatile("barrier.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+// The same barrier, returning whether p held in every participating thread.
+__device__ __forceinline__ bool named_bar_all(int id, int n, bool p) {
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred a, b;\n\t"
+        "setp.ne.u32 a, %1, 0;\n\t"
+        "barrier.red.and.pred b, %2, %3, a;\n\t"
+        "selp.u32 %0, 1, 0, b;\n\t}"
+        : "=r"(r)
+        : "r"(static_cast<uint32_t>(p)), "r"(id), "r"(n)
+        : "memory");
+    return r != 0;
+}
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
 __device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
@@ -61,6 +90,7 @@ struct TrailMaps {
     CUtensorMap eh, el;                  // E_hi, E_lo [d_out x d_in], 128-row boxes
     CUtensorMap rh_narrow, rl_narrow;    // Lt_hi, Lt_lo [d_in x d_in], 128-row boxes
     CUtensorMap rh64, rl64;              // the same with 64-row boxes (64-column tiles)
+    CUtensorMap rh256, rl256;            // the same with 256-row boxes (256-column tiles)
     CUtensorMap w;                       // W [d_out x d_in], 128-row boxes (read and written)
     CUtensorMap qh, ql, ph, pl;          // with P: (-Wpre)_hi, _lo [d_out x d_in], Pt_hi, Pt_lo [d_in x d_in]
     kq_status init(const float* E_hi, const float* E_lo, const float* Lt_hi, const float* Lt_lo, int64_t d_out,
@@ -95,5 +125,13 @@ kq_status split_tf32(const float* src, int64_t n, float* hi, float* lo, cudaStre
 // 128 x 128 (193 KB); [cb, ce) must be whole tiles or end at d_in. W is the one set_w was given.
 kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, int64_t i0, int64_t cb, int64_t ce,
                    bool with_p, bool narrow, int kb, int* info, cudaStream_t stream);
+
+// The same update for K = kb <= 1024 (the blocks of one super-panel, GPTQ mode), still
+// applied to W 128 of K at a time in block order, through TMA reduce-adds instead of a
+// shared-memory copy of the W tile: 128 x 256 tiles (bn = 256, two-stage operand ring) or
+// 128 x 128 (bn = 128, three stages). [cb, ce) whole tiles or ending at d_in; kb whole
+// blocks unless the super-panel ends at d_in.
+kq_status trail_tc_long(const TrailMaps& m, int64_t d_out, int64_t d_in, int64_t i0, int kb, int64_t cb, int64_t ce,
+                        int bn, int* info, cudaStream_t stream);
 
 }  // namespace kq

@@ -11,10 +11,12 @@ import os
 import torch
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_HERE, "libkronq.so")
+# KQ_DEBUG=1 selects the debug build (bounds checks before the kernels' stores; see
+# kq_debug_status), built with `python -m paper_2607_07964_gb300.build --debug`
+LIB_PATH = os.path.join(_HERE, "libkronq_debug.so" if os.environ.get("KQ_DEBUG") == "1" else "libkronq.so")
 
 KQ_OK, KQ_ERR_INVALID_ARG, KQ_ERR_UNSUPPORTED, KQ_ERR_NOT_PD = 0, 1, 2, 3
-KQ_ERR_CUDA, KQ_ERR_TIMEOUT, KQ_ERR_WORKSPACE = 4, 5, 6
+KQ_ERR_CUDA, KQ_ERR_TIMEOUT, KQ_ERR_WORKSPACE, KQ_ERR_NONFINITE = 4, 5, 6, 7
 KQ_FWD, KQ_INV, KQ_FWD_SYM = 0, 1, 2
 KQ_TRAIL_FP32, KQ_TRAIL_3XTF32 = 0, 1
 KQ_SYRK_CHUNK_TOKENS = 512
@@ -47,6 +49,9 @@ def lib() -> ctypes.CDLL:
             "kq_graph_exec_destroy": ([P], I),
             "kq_check": ([P, I, P, P], I),
             "kq_selftest_timeout": ([P, I64, P], I),
+            "kq_debug_build": ([], I),
+            "kq_debug_status": ([P, P, I], I),
+            "kq_selftest_bounds": ([P, I64, P], I),
             "kq_selftest_div": ([P, P, I64, P, P], I),
             "kq_accum_factor": ([P, I64, I64, I64, P, I, P, P, P], I),
             "kq_compute_scales": ([P, I64, I64, P, P, P, P, P], I),
@@ -134,6 +139,26 @@ def kq_check(info=None, reset: bool = True, stream=None) -> tuple[int, int]:
     raw = ctypes.c_int(0)
     st = lib().kq_check(_ptr(info), int(reset), ctypes.byref(raw), _stream(stream))
     return st, raw.value
+
+
+def kq_debug_build() -> bool:
+    return bool(lib().kq_debug_build())
+
+
+DEBUG_UNITS = ("api", "syrk", "biip", "chol", "obs", "trail_tc", "gptaq", "infer", "check")
+
+
+def kq_debug_status(reset: bool = True) -> tuple[str | None, int]:
+    """(source file, line) of the first failed bounds check of the debug build, or (None, 0)."""
+    unit, line = ctypes.c_int(-1), ctypes.c_int(0)
+    _ok(lib().kq_debug_status(ctypes.byref(unit), ctypes.byref(line), int(reset)), "kq_debug_status")
+    return (DEBUG_UNITS[unit.value] if unit.value >= 0 else None), line.value
+
+
+def kq_selftest_bounds(buf, n: int, stream=None) -> None:
+    """buf: n + 1 float32 on the device; writes buf[i] = i for i <= n under a check against n."""
+    _need(buf, "buf", torch.float32, (n + 1,))
+    _ok(lib().kq_selftest_bounds(_ptr(buf), int(n), _stream(stream)), "kq_selftest_bounds")
 
 
 def kq_selftest_timeout(info, limit_us: int, stream=None) -> None:

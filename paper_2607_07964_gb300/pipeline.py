@@ -148,9 +148,14 @@ class LayerPipeline:
         marks = iter(range(len(self.stages) + 1))
 
         def mark():
+            # stage boundary: an event (if asked) and an NVTX range named after the stage
             i = next(marks)
             if events is not None:
                 events[i].record(s)
+            if i > 0:
+                torch.cuda.nvtx.range_pop()
+            if i < len(self.stages):
+                torch.cuda.nvtx.range_push(f"kronq.{self.stages[i]}")
 
         mark()
         self._factor("X", X, self.HX, self.trace_x, self.info[0:1], s)                           # Alg. 1: H_X
@@ -198,6 +203,13 @@ class LayerPipeline:
         low-priority stream, and P on the high-priority one after the Cholesky.
         Events order the shared buffers; x_ready / g_ready / w_ready / xt_ready are the host
         path's copy events."""
+        torch.cuda.nvtx.range_push("kronq.layer")
+        try:
+            self._enqueue_overlapped(X, G, W, sign_u, sign_v, caller, x_ready, g_ready, w_ready, Xt, xt_ready)
+        finally:
+            torch.cuda.nvtx.range_pop()
+
+    def _enqueue_overlapped(self, X, G, W, sign_u, sign_v, caller, x_ready, g_ready, w_ready, Xt, xt_ready) -> None:
         s, s2 = self.main, self.side
         e_in, e_fx, e_tx, e_rin, e_side, e_out, e_hg, e_d = self._ev
         e_in.record(caller)
@@ -312,8 +324,9 @@ class LayerPipeline:
         if self.side is not None:
             self.side.synchronize()
             self.main.synchronize()
-        for k in range(4):
-            st, raw = kq.kq_check(self.info[k:k + 1], reset=True, stream=stream)
+        # read (and clear) every word first, so that no stale report survives the raise
+        found = [kq.kq_check(self.info[k:k + 1], reset=True, stream=stream) for k in range(4)]
+        for st, raw in found:
             if st != kq.KQ_OK:
                 raise kq.KronqError(st, "pipeline", f"device word {raw}")
 

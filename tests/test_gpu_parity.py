@@ -136,7 +136,7 @@ def test_scales_traces_rotations(d_out, d_in, sym):
     assert rel_fro(host(Wp), W) <= 1e-5
 
 
-@pytest.mark.parametrize("n", [2, 32, 512, 1024, 2048, 4096, 8192, 16384, 28, 28 * 64, 28 * 1024, 32768])
+@pytest.mark.parametrize("n", [2, 32, 512, 1024, 2048, 4096, 8192, 16384, 28, 28 * 64, 28 * 512, 28 * 1024, 32768])
 def test_rht_matches_dense_hadamard(n):
     """Pure rotation (no scales) of a few rows against the oracle's dense V."""
     rng = np.random.default_rng(n)
@@ -153,6 +153,29 @@ def test_rht_matches_dense_hadamard(n):
     # column direction on a [n x 3] matrix equals the row direction on its transpose
     Wc = dev(np.ascontiguousarray(W.T))
     K().kq_rotate_out(Wc, None, None, dev(sign, torch.int8), K().KQ_FWD)
+    assert rel_fro(host(Wc).T, got) <= 1e-6
+
+
+@pytest.mark.parametrize("n", [28 * 512, 28 * 1024])
+def test_rht_rows_many_rows_28(n):
+    """The register row transform for n = 28 * 2^k over more rows than CTAs (each CTA walks
+    several rows, the next one loaded while the current one is transformed), with the
+    input-side scales: sampled output columns against rows of V S^-1 built from the
+    definition, and the whole result against the column transform of the transpose."""
+    rng = np.random.default_rng(n + 1)
+    rows = 2 * 152 + 37
+    W = rng.standard_normal((rows, n)).astype(np.float32)
+    sign = np.where(rng.random(n) < 0.5, -1, 1).astype(np.int8)
+    s = np.exp(0.3 * rng.standard_normal(n)).astype(np.float32)
+    Wd = dev(W)
+    K().kq_rotate_in(Wd, None, dev(s), dev(sign, torch.int8), K().KQ_FWD)
+    got = host(Wd)
+    cols = np.unique(rng.integers(0, n, 24))
+    V = ref.rht_rows(n, sign, cols)                       # rows of H diag(sign) / sqrt(n)
+    want = (W.astype(np.float64) * s[None, :].astype(np.float64)) @ V.T
+    assert rel_fro(got[:, cols], want) <= 1e-5
+    Wc = dev(np.ascontiguousarray(W.T))
+    K().kq_rotate_out(Wc, None, dev(s), dev(sign, torch.int8), K().KQ_FWD)
     assert rel_fro(host(Wc).T, got) <= 1e-6
 
 
@@ -283,11 +306,13 @@ def _synthetic_lt(n, seed):
 
 
 # (5120, 1024): more row CTAs than SMs; (1024, 24704): d_out d_in above 24M with one CTA
-# per SM: both take the sweep's schedule for large layers (128 x 128 update tiles, block
-# kernel not fused), the one the 8B MLP and 70B layers run.
+# per SM: both take the sweep's schedule for large layers (block kernel not fused), the one
+# the 8B MLP and 70B layers run; with more than 8 blocks (2304, 1156, 24704) the two-level
+# lazy update (super-panels of 8 blocks, one long update of the columns beyond each), 1156
+# ending in a ragged super-panel of one block and 4 columns.
 @pytest.mark.parametrize("d_out,d_in,bits,group", [
     (256, 256, 4, 128), (300, 1024, 4, 128), (512, 896, 3, 128), (128, 1536, 2, 0), (200, 640, 8, 128),
-    (5120, 1024, 3, 128), (5120, 1024, 2, 0), (1024, 24704, 2, 128)])
+    (5120, 1024, 3, 128), (5120, 1024, 2, 0), (5120, 2304, 4, 0), (5120, 1156, 3, 128), (1024, 24704, 2, 128)])
 def test_sweep_tensor_core_trailing(d_out, d_in, bits, group):
     """3xTF32 trailing update: teacher forced on every row (codes = quant(GPU pre_q) bit for
     bit; pre_q within float32 rounding of Algorithm 2 from the GPU's own errors; grids from
