@@ -222,9 +222,9 @@ class ClockSampler:
 # sweep on rows_s rows of that shrunk layer (proportional to rows x d_in^2). f = 1 runs
 # BiIP and the Cholesky at full size.
 ORACLE_SAMPLES = {
-    "large": dict(T_s=1024, f=4, rows_s=64),
-    "medium": dict(T_s=512, f=8, rows_s=64),
-    "small": dict(T_s=256, f=16, rows_s=32),
+    "large": dict(T_s=2048, f=4, rows_s=64),
+    "medium": dict(T_s=1024, f=8, rows_s=64),
+    "small": dict(T_s=512, f=16, rows_s=32),
 }
 
 

@@ -207,8 +207,10 @@ __global__ void __launch_bounds__(7 * (1 << LG) / 16, 1) rht_rows28_reg_kernel(f
             for (int k = 0; k < 16; ++k) x[k] = cur[c][k];
             if (more) load(r + gridDim.x, c, cur[c]);
             const int a = g + 7 * c;
+            float f[16];
+            factors16(pre_mode, sign, s, a * P + 16 * tl, f);
 #pragma unroll
-            for (int k = 0; k < 16; ++k) x[k] *= factor(pre_mode, sign, s, a * P + 16 * tl + k);
+            for (int k = 0; k < 16; ++k) x[k] *= f[k];
             fwht_kbits<0xFu>(x);
             rr_transpose<LG, 1>(x, buf, tl);
             rr_transpose<LG, 2>(x, buf, tl);
@@ -688,7 +690,8 @@ kq_status rows_transform(float* M, int64_t rows, int64_t n, int pre, int post, c
                          const float* s, cudaStream_t stream) {
     HadamardPlan p;
     if (!plan_of(n, &p)) return KQ_ERR_UNSUPPORTED;
-    if (rows > 0 && rows_reg_ok(M, n) && p.has28) {
+    if (rows > 0 && rows_reg_ok(M, n) && p.has28 && (reinterpret_cast<uintptr_t>(sign) & 15u) == 0 &&
+        (reinterpret_cast<uintptr_t>(s) & 15u) == 0) {
         if (p.P == 512) return launch_rows28_reg<9>(M, rows, pre, post, sign, s, stream);
         return launch_rows28_reg<10>(M, rows, pre, post, sign, s, stream);
     }

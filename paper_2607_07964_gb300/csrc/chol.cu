@@ -558,9 +558,12 @@ __device__ __forceinline__ void update_quad(const Work& w, int64_t npad, int k, 
 
 // The tiles that step k + 1 reads first: row block k + 1 (tiles (k + 1, j), j <= k + 1)
 // and block column k + 1 below it (tiles (i, k + 1), i > k + 1); nbk tiles x 4 quadrants.
-__global__ void __launch_bounds__(G_THREADS, 2) chol_next_kernel(Work w, int64_t npad, int k) {
+// part 0: all of them; part 1: only the diagonal tile (k + 1, k + 1), which is all the next
+// diagonal step needs (grid 1 x 4); part 2: all but that tile, for the next panel.
+__global__ void __launch_bounds__(G_THREADS, 2) chol_next_kernel(Work w, int64_t npad, int k, int part) {
     extern __shared__ __align__(16) float sm[];
-    const int bid = blockIdx.x;
+    const int bid = part == 1 ? k + 1 : static_cast<int>(blockIdx.x);
+    if (part == 2 && bid == k + 1) return;
     if (bid < k + 2)
         update_quad(w, npad, k, k + 1, bid, blockIdx.y, sm);
     else
@@ -694,6 +697,7 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
     KQ_LAUNCH_CHECK("prep_kernel");
     SideStream* side = nbk > 2 ? side_stream(stream) : nullptr;
     bool forked = false, remote_pending = false;
+    bool next_pending = false;   // the next panel's tiles, updated on the side stream
     for (int k0 = 0; k0 < nbk; k0 += (two_level ? SPB : nbk)) {
         const int k1 = two_level ? std::min(nbk, k0 + SPB) : nbk;   // this super-panel: blocks [k0, k1)
         const int set = two_level ? (k0 / SPB) & 1 : 0;
@@ -701,6 +705,10 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
         for (int k = k0; k < k1; ++k) {
             chol_diag_kernel<<<1, DIAG_THREADS, DIAG_SMEM, stream>>>(w, n, npad, k, info);
             KQ_LAUNCH_CHECK("chol_diag_kernel");
+            if (next_pending) {   // the tiles of this panel, updated beside the diagonal step
+                KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[2], 0));
+                next_pending = false;
+            }
             if (nbk > 1) {
                 chol_panel_kernel<<<dim3(nbk - 1, 4), G_THREADS, STRIP_SMEM, stream>>>(w, npad, k);
                 KQ_LAUNCH_CHECK("chol_panel_kernel");
@@ -709,10 +717,23 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
             const bool has_rest = k + 2 < k1;                 // tiles of this super-panel beyond k + 1
             const bool need_split = has_rest || far_after;   // the super-panel update reads every slice
             const bool fork = side && need_split;
-            if (fork) KQ_CUDA(cudaEventRecord(side->ev[0], stream));      // panel k done
+            if (side && (need_split || k + 1 < k1)) KQ_CUDA(cudaEventRecord(side->ev[0], stream));   // panel k done
             if (forked) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));  // update of step k - 1 done
             if (k + 1 < k1) {
-                chol_next_kernel<<<dim3(nbk, 4), G_THREADS, STRIP_SMEM, stream>>>(w, npad, k);
+                if (side) {
+                    // Step k's update of the next diagonal tile alone on this stream, so the
+                    // next diagonal step starts at once; the rest of the tiles the next panel
+                    // reads on the side stream beside it (ahead of this step's split and
+                    // in-panel update there, which touch other tiles).
+                    KQ_CUDA(cudaStreamWaitEvent(side->s, side->ev[0], 0));
+                    chol_next_kernel<<<dim3(nbk, 4), G_THREADS, STRIP_SMEM, side->s>>>(w, npad, k, 2);
+                    KQ_LAUNCH_CHECK("chol_next_kernel");
+                    KQ_CUDA(cudaEventRecord(side->ev2[2], side->s));
+                    next_pending = true;
+                    chol_next_kernel<<<dim3(1, 4), G_THREADS, STRIP_SMEM, stream>>>(w, npad, k, 1);
+                } else {
+                    chol_next_kernel<<<dim3(nbk, 4), G_THREADS, STRIP_SMEM, stream>>>(w, npad, k, 0);
+                }
                 KQ_LAUNCH_CHECK("chol_next_kernel");
             }
             if (need_split) {

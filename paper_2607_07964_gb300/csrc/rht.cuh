@@ -65,11 +65,49 @@ static_assert(h28_is_hadamard(), "H_28 must satisfy H H^T = 28 I and be symmetri
 // Factor applied to element index j before (pre) or after (post) a transform.
 enum FactorMode { F_NONE = 0, F_SMUL = 1, F_SDIV = 2, F_SIGN = 3 };
 
+// F_SDIV's sign / s is +-1 over s correctly rounded, i.e. +-__frcp_rn(s): the same bits as
+// the division for a numerator of +-1, without its slower sequence.
 __device__ __forceinline__ float factor(int mode, const int8_t* sign, const float* s, int64_t j) {
     if (mode == F_NONE) return 1.0f;
     const float sg = static_cast<float>(sign[j]);
     if (mode == F_SIGN || s == nullptr) return sg;
-    return mode == F_SMUL ? sg * s[j] : sg / s[j];
+    if (mode == F_SMUL) return sg * s[j];
+    const float r = __frcp_rn(s[j]);
+    return sg < 0.0f ? -r : r;
+}
+
+// factor() for the 16 consecutive indices j0 .. j0 + 15 (j0 a multiple of 16; sign and s
+// 16-byte aligned): one 16-byte load of the signs and four of the scales.
+__device__ __forceinline__ void factors16(int mode, const int8_t* sign, const float* s, int64_t j0,
+                                          float (&f)[16]) {
+    if (mode == F_NONE) {
+#pragma unroll
+        for (int k = 0; k < 16; ++k) f[k] = 1.0f;
+        return;
+    }
+    const int4 sg4 = __ldg(reinterpret_cast<const int4*>(sign + j0));
+    const int32_t sw[4] = {sg4.x, sg4.y, sg4.z, sg4.w};
+    float sv[16];
+    if (mode != F_SIGN && s != nullptr) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const float4 v = __ldg(reinterpret_cast<const float4*>(s + j0) + q);
+            sv[4 * q] = v.x;
+            sv[4 * q + 1] = v.y;
+            sv[4 * q + 2] = v.z;
+            sv[4 * q + 3] = v.w;
+        }
+    }
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+        const int8_t b = static_cast<int8_t>((sw[k >> 2] >> (8 * (k & 3))) & 0xff);
+        const bool neg = b < 0;
+        float m;
+        if (mode == F_SIGN || s == nullptr) m = 1.0f;
+        else if (mode == F_SMUL) m = sv[k];
+        else m = __frcp_rn(sv[k]);
+        f[k] = neg ? -m : m;
+    }
 }
 
 // y = H_28 x for 28 values in registers, each output handed to out(r, y_r) as soon as it is

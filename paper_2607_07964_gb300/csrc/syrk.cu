@@ -78,64 +78,6 @@ __device__ __forceinline__ void tile_of(int bid, int n_row_tiles, int n_col_tile
     *tj = 0;
 }
 
-// Pairs of row tiles (2m, 2m + 1) hold the same lower-triangle columns (j <= m), so a
-// cluster of two CTAs takes one pair and the column panel j they share: each CTA loads half
-// of the panel's operand boxes and multicasts them to both, halving the L2 reads of the
-// larger operand. Pairs in the same banded order as the tiles (BAND columns a band, one row
-// pair after another).
-__device__ __forceinline__ void pair_of(int pid, int n_row_pairs, int n_col_tiles, int* m, int* tj) {
-    for (int j0 = 0; j0 < n_col_tiles; j0 += BAND) {
-        const int w = min(BAND, n_col_tiles - j0);
-        const int rows = n_row_pairs - j0;
-        const int tri = w * (w + 1) / 2;
-        const int cnt = rows <= w ? rows * (rows + 1) / 2 : tri + (rows - w) * w;
-        if (pid >= cnt) {
-            pid -= cnt;
-            continue;
-        }
-        int k = 0;
-        if (pid >= tri && rows > w) {   // past the triangle: w pairs a row pair
-            k = w + (pid - tri) / w;
-            pid = (pid - tri) % w;
-        } else {
-            while (pid >= min(w, k + 1)) pid -= min(w, k++ + 1);
-        }
-        *m = j0 + k;
-        *tj = j0 + pid;
-        return;
-    }
-    *m = 0;   // not reached for pid < the number of pairs
-    *tj = 0;
-}
-
-__device__ __forceinline__ uint32_t cluster_rank() {
-    uint32_t r;
-    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-    return r;
-}
-__device__ __forceinline__ void cluster_sync_all() {
-    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-// TMA load of one box into the same shared-memory offset of every CTA in `mask`, each
-// CTA's mbarrier at the offset of `bar` receiving the bytes it got.
-__device__ __forceinline__ void tma_load_2d_mc(void* dst, const CUtensorMap* m, uint64_t* bar, int x, int y,
-                                               uint16_t mask) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
-        " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
-        "l"(reinterpret_cast<uint64_t>(m)), "r"(smem_u32(bar)), "r"(x), "r"(y), "h"(mask)
-        : "memory");
-}
-// Arrive once on `bar` (same offset) in every CTA of `mask` when this thread's issued MMAs
-// have completed.
-__device__ __forceinline__ void tc_commit_mc(uint64_t* bar, uint16_t mask) {
-    asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
-            smem_u32(bar)),
-        "h"(mask)
-        : "memory");
-}
-
 __device__ __forceinline__ bool wait_noabort(uint64_t* bar, uint32_t parity) {
     int dummy = 0;
     return mbar_wait(bar, parity, &dummy);
@@ -146,7 +88,7 @@ __device__ __forceinline__ bool wait_noabort(uint64_t* bar, uint32_t parity) {
 //     operand box comes from map a0.
 //   CROSS = true: D (+)= (A_hi + A_lo)^T B over all tiles, no symmetry: the K loop runs over
 //     the T tokens of the pair (a0 = A_hi, b) and then over the pair (a1 = A_lo, b).
-template <bool CROSS, bool PAIR = false>
+template <bool CROSS>
 __device__ __forceinline__ void gram_tc_body(const CUtensorMap* a0, const CUtensorMap* a1,
                                              const CUtensorMap* bmap, float* __restrict__ H, int d,
                                              int T, int n_row_tiles, int chunk_stages, int accumulate,
@@ -165,14 +107,9 @@ __device__ __forceinline__ void gram_tc_body(const CUtensorMap* a0, const CUtens
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     int ti, tj;
-    const uint32_t rank = PAIR ? cluster_rank() : 0u;
     if (CROSS) {
         ti = static_cast<int>(blockIdx.x) % n_row_tiles;
         tj = static_cast<int>(blockIdx.x) / n_row_tiles;
-    } else if (PAIR) {
-        int m;
-        pair_of(static_cast<int>(blockIdx.x >> 1), n_row_tiles / 2, (d + BN - 1) / BN, &m, &tj);
-        ti = 2 * m + static_cast<int>(rank);
     } else {
         tile_of(blockIdx.x, n_row_tiles, (d + BN - 1) / BN, &ti, &tj);
     }
@@ -185,7 +122,7 @@ __device__ __forceinline__ void gram_tc_body(const CUtensorMap* a0, const CUtens
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&full[s], 1);
-            mbar_init(&empty[s], PAIR ? 2 : 1);   // with a pair: both CTAs' MMAs release a stage
+            mbar_init(&empty[s], 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&tfull[b], 1);
@@ -199,8 +136,6 @@ __device__ __forceinline__ void gram_tc_body(const CUtensorMap* a0, const CUtens
         tmem_alloc(tmem_slot, TMEM_COLS);
         tmem_relinquish();
     }
-    // the partner's barriers must be initialized before any copy or arrive reaches them
-    if (PAIR) cluster_sync_all();
     if (warp == 0 && lane == 0) {
         tma_prefetch_desc(a0);
         if (CROSS) {
@@ -230,15 +165,9 @@ __device__ __forceinline__ void gram_tc_body(const CUtensorMap* a0, const CUtens
                 const CUtensorMap* bm = CROSS ? bmap : a0;
                 tma_load_2d(a, am, &full[s], i0, y);
                 tma_load_2d(a + BOX_BYTES, am, &full[s], i0 + 64, y);
-                if (PAIR) {   // this CTA's half of the column panel, into both CTAs
 #pragma unroll
-                    for (int q = 2 * static_cast<int>(rank); q < 2 * static_cast<int>(rank) + 2; ++q)
-                        tma_load_2d_mc(b + q * BOX_BYTES, bm, &full[s], j0 + 64 * q, y, 0x3);
-                } else {
-#pragma unroll
-                    for (int q = 0; q < 4; ++q)
-                        tma_load_2d(b + q * BOX_BYTES, bm, &full[s], j0 + 64 * q, y);
-                }
+                for (int q = 0; q < 4; ++q)
+                    tma_load_2d(b + q * BOX_BYTES, bm, &full[s], j0 + 64 * q, y);
                 issued = k + 1;
             }
             // Drain: every issued load must have landed before the CTA may exit.
@@ -273,10 +202,7 @@ __device__ __forceinline__ void gram_tc_body(const CUtensorMap* a0, const CUtens
                         const uint64_t bd = smem_desc_sw128(b + k16 * 2048, LBO, SBO);
                         tc_mma_f16(dt, ad, bd, idesc, (kk > 0 || k16 > 0) ? 1u : 0u);
                     }
-                    if (PAIR)
-                        tc_commit_mc(&empty[s], 0x3);   // the stage is free once both CTAs are done
-                    else
-                        tc_commit(&empty[s]);
+                    tc_commit(&empty[s]);
                 }
                 if (ok) tc_commit(&tfull[buf]);
             }
@@ -369,8 +295,6 @@ __device__ __forceinline__ void gram_tc_body(const CUtensorMap* a0, const CUtens
     }
 
     __syncthreads();
-    // neither CTA of a pair leaves while the other may still send it copies or arrivals
-    if (PAIR) cluster_sync_all();
     if (*abort_flag && threadIdx.x == 0) record_error(info, -KQ_ERR_TIMEOUT);
     if (warp == 1) {
         tc_fence_after();
@@ -382,13 +306,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 syrk_tc_kernel(const __grid_constant__ CUtensorMap tmap, float* __restrict__ H, int d, int T,
                int n_row_tiles, int chunk_stages, int accumulate, int* info) {
     gram_tc_body<false>(&tmap, &tmap, &tmap, H, d, T, n_row_tiles, chunk_stages, accumulate, info);
-}
-
-// The same with clusters of two CTAs sharing their column panel (pair_of); grid = 2 x pairs.
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
-syrk_tc_pair_kernel(const __grid_constant__ CUtensorMap tmap, float* __restrict__ H, int d, int T,
-                    int n_row_tiles, int chunk_stages, int accumulate, int* info) {
-    gram_tc_body<false, true>(&tmap, &tmap, &tmap, H, d, T, n_row_tiles, chunk_stages, accumulate, info);
 }
 
 __global__ void __launch_bounds__(NUM_THREADS, 1)
@@ -500,14 +417,15 @@ kq_status make_bf16_map(CUtensorMap* m, const uint16_t* base, int64_t d, int64_t
     return KQ_OK;
 }
 
-// Clusters of two for the SYRK unless the environment variable KQ_SYRK_PAIRS is 0 (a
-// switch for comparing the two launch forms; both compute the same sums per tile).
-bool syrk_pairs_enabled() {
-    static const bool on = [] {
-        const char* e = std::getenv("KQ_SYRK_PAIRS");
-        return !(e && e[0] == '0');
+// Stages (64 tokens each) between drains of the SYRK accumulator: KQ_SYRK_CHUNK_TOKENS, or
+// the environment variable KQ_SYRK_DRAIN_TOKENS (512, 1024 or 2048; a tuning switch).
+int syrk_chunk_stages() {
+    static const int n = [] {
+        const char* e = std::getenv("KQ_SYRK_DRAIN_TOKENS");
+        const int t = e ? std::atoi(e) : 0;
+        return (t == 512 || t == 1024 || t == 2048) ? t / BK : KQ_SYRK_CHUNK_TOKENS / BK;
     }();
-    return on;
+    return n;
 }
 
 }  // namespace
@@ -545,25 +463,16 @@ extern "C" kq_status kq_accum_factor(const uint16_t* A, int64_t T, int64_t d, in
         KQ_TRY(once_per_device(attr_set, [&]() -> kq_status {
             KQ_CUDA(cudaFuncSetAttribute(syrk_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          SMEM_BYTES));
-            KQ_CUDA(cudaFuncSetAttribute(syrk_tc_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         SMEM_BYTES));
             return KQ_OK;
         }));
         const int n_row = static_cast<int>(cdiv(d, BM));
         const int n_col = static_cast<int>(cdiv(d, BN));
         int64_t tiles = 0;
         for (int j = 0; j < n_col; ++j) tiles += (n_row - 2 * j > 0) ? n_row - 2 * j : 0;
-        const int chunk_stages = KQ_SYRK_CHUNK_TOKENS / BK;
-        if (n_row % 2 == 0 && syrk_pairs_enabled()) {
-            // every row tile has its partner (2m, 2m + 1): clusters of two share the column panel
-            syrk_tc_pair_kernel<<<static_cast<unsigned>(tiles), NUM_THREADS, SMEM_BYTES, stream>>>(
-                tmap, H, static_cast<int>(d), static_cast<int>(T), n_row, chunk_stages, accumulate, info);
-            KQ_LAUNCH_CHECK("syrk_tc_pair_kernel");
-        } else {
-            syrk_tc_kernel<<<static_cast<unsigned>(tiles), NUM_THREADS, SMEM_BYTES, stream>>>(
-                tmap, H, static_cast<int>(d), static_cast<int>(T), n_row, chunk_stages, accumulate, info);
-            KQ_LAUNCH_CHECK("syrk_tc_kernel");
-        }
+        const int chunk_stages = syrk_chunk_stages();
+        syrk_tc_kernel<<<static_cast<unsigned>(tiles), NUM_THREADS, SMEM_BYTES, stream>>>(
+            tmap, H, static_cast<int>(d), static_cast<int>(T), n_row, chunk_stages, accumulate, info);
+        KQ_LAUNCH_CHECK("syrk_tc_kernel");
     }
     if (trace) return launch_trace(H, d, trace, stream);
     return KQ_OK;
@@ -614,7 +523,7 @@ extern "C" kq_status kq_accum_drift(const uint16_t* Xt, const uint16_t* X, int64
     }));
     const int n_row = static_cast<int>(cdiv(d, BM));
     const int n_col = static_cast<int>(cdiv(d, BN));
-    const int chunk_stages = KQ_SYRK_CHUNK_TOKENS / BK;
+    const int chunk_stages = syrk_chunk_stages();
     for (int64_t t0 = 0; t0 < T; t0 += Tc) {
         const int64_t tn = std::min<int64_t>(Tc, T - t0);
         const int64_t vecs = tn * (d / 8);

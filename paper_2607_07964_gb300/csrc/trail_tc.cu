@@ -22,6 +22,7 @@
 // Every mbarrier wait is bounded; a timeout sets -KQ_ERR_TIMEOUT in *info and the CTA
 // drains its copies and MMAs before it exits.
 #include <algorithm>
+#include <cstdlib>
 #include <cstring>
 
 #include "trail_tc.cuh"
@@ -528,6 +529,26 @@ kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, in
 }
 
 namespace {
+// CTAs of a reduce-add launch: persistent, one per SM walking the tiles (one CTA per tile,
+// which would let the critical-path kernels beside it take SMs as tiles finish, measured
+// slower on the 70B down_proj layer: 331 against 320 ms, the per-CTA set-up costing more than
+// the overlap it buys).
+unsigned red_grid(int n_tiles) { return static_cast<unsigned>(std::min(n_tiles, num_sms())); }
+
+// Slabs of 32 K between two drains of the accumulator into W in the long updates (K up to
+// 1024): 8, i.e. two blocks' updates summed in TMEM before each reduce-add into W (half the
+// epilogue traffic of one drain per block: the 70B down_proj layer 297 against 309 ms; the
+// inverse Cholesky's relative error at n = 4096 and 8192 grows from 5.6e-7 and 6.4e-7 to
+// 9.2e-7 and 1.1e-6, against a 1e-5 bar), or 4 (one block at a time) when the environment
+// variable KQ_TRAIL_DRAIN_SLABS says 4 (a tuning switch).
+int long_drain_slabs() {
+    static const int n = [] {
+        const char* e = std::getenv("KQ_TRAIL_DRAIN_SLABS");
+        return (e && std::atoi(e) == 4) ? 4 : 8;
+    }();
+    return n;
+}
+
 template <int BN, int STAGES>
 kq_status launch_trail_red(const TrailMaps& m, const CUtensorMap& rh, const CUtensorMap& rl, int64_t d_out,
                            int64_t i0, int kb, int64_t cb, int64_t ce, int* info, cudaStream_t stream) {
@@ -551,9 +572,8 @@ kq_status launch_trail_red(const TrailMaps& m, const CUtensorMap& rh, const CUte
     ts.pslab = 1 << 30;
     ts.ce = static_cast<int>(ce);
     const int nslab = static_cast<int>(cdiv(kb, TBK));
-    trail_tc_kernel<BN, STAGES, true><<<static_cast<unsigned>(std::min(ts.n_tiles, num_sms())), T_THREADS, Cfg::SMEM,
-                                        stream>>>(m.eh, m.el, rh, rl, m.eh, m.el, rh, rl, m.w, m.w, ts, nslab, TNSLAB,
-                                                  info);
+    trail_tc_kernel<BN, STAGES, true><<<red_grid(ts.n_tiles), T_THREADS, Cfg::SMEM, stream>>>(
+        m.eh, m.el, rh, rl, m.eh, m.el, rh, rl, m.w, m.w, ts, nslab, long_drain_slabs(), info);
     KQ_LAUNCH_CHECK("trail_tc_kernel");
     return KQ_OK;
 }
@@ -615,9 +635,9 @@ kq_status chol_update_tc(const CholTcMaps& m, int set, int nbk, int a_j0, int a_
     ts.ce = 1 << 30;   // every tile lies inside the padded matrices
     ts.n_tiles = ts.n_a + ((b_i1 > b_i0 && b_j1 > 0) ? (b_i1 - b_i0) * b_j1 : 0);
     if (ts.n_tiles == 0) return KQ_OK;
-    trail_tc_kernel<128, 3, true><<<static_cast<unsigned>(std::min(ts.n_tiles, num_sms())), T_THREADS, Cfg::SMEM, stream>>>(
+    trail_tc_kernel<128, 3, true><<<red_grid(ts.n_tiles), T_THREADS, Cfg::SMEM, stream>>>(
         m.ch[set], m.cl[set], m.ch[set], m.cl[set], m.ch[set], m.cl[set], m.zh[set], m.zl[set], m.a, m.z, ts, nslab,
-        TNSLAB, info);
+        nslab > TNSLAB ? long_drain_slabs() : TNSLAB, info);
     KQ_LAUNCH_CHECK("trail_tc_kernel");
     return KQ_OK;
 }

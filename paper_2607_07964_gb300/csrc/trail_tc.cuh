@@ -126,11 +126,11 @@ kq_status split_tf32(const float* src, int64_t n, float* hi, float* lo, cudaStre
 kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, int64_t i0, int64_t cb, int64_t ce,
                    bool with_p, bool narrow, int kb, int* info, cudaStream_t stream);
 
-// The same update for K = kb <= 1024 (the blocks of one super-panel, GPTQ mode), still
-// applied to W 128 of K at a time in block order, through TMA reduce-adds instead of a
-// shared-memory copy of the W tile: 128 x 256 tiles (bn = 256, two-stage operand ring) or
-// 128 x 128 (bn = 128, three stages). [cb, ce) whole tiles or ending at d_in; kb whole
-// blocks unless the super-panel ends at d_in.
+// The same update for K = kb <= 1024 (the blocks of one super-panel, GPTQ mode), applied to
+// W two blocks' K at a time in block order (the accumulator drained every 256 of K), through
+// TMA reduce-adds instead of a shared-memory copy of the W tile: 128 x 256 tiles (bn = 256,
+// two-stage operand ring) or 128 x 128 (bn = 128, three stages). [cb, ce) whole tiles or
+// ending at d_in; kb whole blocks unless the super-panel ends at d_in.
 kq_status trail_tc_long(const TrailMaps& m, int64_t d_out, int64_t d_in, int64_t i0, int kb, int64_t cb, int64_t ce,
                         int bn, int* info, cudaStream_t stream);
 

@@ -8,8 +8,13 @@ another (equally valid) path. It is judged in two ways:
     values are within float32 rounding (2e-5 of |W'_j| + sum_k |E_k R_kj|) of what
     Algorithm 2 computes from the GPU's own earlier errors; its group grids come from the
     block-start values that the same replay gives;
-  * against the fp32-ordered oracle sweep: at most 0.1 % of codes differ, and the first
-    difference in each row sits within 1e-4 quantization steps of a rounding tie.
+  * against the fp32-ordered oracle sweep: the first difference in each row sits within 1e-4
+    quantization steps of a rounding tie, and such first differences are at most 0.1 % of
+    the codes compared up to them. After a row's first difference its error feedback takes
+    the other (equally valid) path, so later codes of that row differ too; how many depends
+    on where the tie falls and on the row length (a flip near the start of a 28672-wide row
+    makes most of that row differ), which is why the rate is taken over the independent
+    disagreements and the rest of the row is held to the teacher-forced check instead.
 """
 import numpy as np
 
@@ -51,18 +56,26 @@ def check_teacher_forced(Wp, Lt, g, bits, group, block=128, Pt=None, rows=None):
 
 
 def check_against_fp32_sweep(Wp, Lt, g, bits, group, block=128, Pt=None, rows=None, max_rate=1e-3):
-    """<= max_rate of codes differ from the fp32-ordered sweep on the given rows, and each
-    row's first difference is at a rounding tie of the oracle's value."""
+    """Each row's first difference from the fp32-ordered sweep is at a rounding tie of the
+    oracle's value, and first differences are <= max_rate of the codes compared up to them
+    (module docstring). Returns the oracle's sweep and the mismatch mask."""
     sel = slice(None) if rows is None else np.asarray(rows)
     c = obs_sweep_fp32(Wp, Lt, bits, group, block, rows=rows, want_pre_q=True, Pt=Pt)
     codes = g["codes"][sel]
     mis = codes != c["codes"]
-    assert mis.mean() <= max_rate, mis.mean()
-    for r in np.where(mis.any(axis=1))[0]:
+    n = codes.shape[1]
+    firsts, compared = 0, 0
+    for r in range(codes.shape[0]):
+        if not mis[r].any():
+            compared += n
+            continue
         j = int(np.argmax(mis[r]))
+        firsts += 1
+        compared += j + 1
         gi = 0 if group == 0 else j // group
         x = np.float64(c["pre_q"][r, j]) / np.float64(c["scale"][r, gi])
         assert abs((x - np.floor(x)) - 0.5) <= 1e-4, (r, j)
+    assert firsts <= max_rate * compared, (firsts, compared, float(mis.mean()))
     return c, mis
 
 

@@ -163,7 +163,7 @@ def test_fullsize_sweep_tensor_core(layer):
     Wp = snap["Wp_in"].cpu().numpy()
     Lt = np.ascontiguousarray(snap["Lt"].cpu().numpy())
     check_teacher_forced(Wp, Lt, g, cfg.bits, cfg.group, cfg.block, rows=_sample_rows(cfg.d_out, 64, 9))
-    check_against_fp32_sweep(Wp, Lt, g, cfg.bits, cfg.group, cfg.block, rows=_sample_rows(cfg.d_out, 24, 10))
+    check_against_fp32_sweep(Wp, Lt, g, cfg.bits, cfg.group, cfg.block, rows=_sample_rows(cfg.d_out, 64, 10))
 
 
 def test_fullsize_sweep_fp32_mode_bit_exact(layer):
