@@ -71,7 +71,7 @@ __device__ __forceinline__ bool wait_quiet(uint64_t* bar, uint32_t parity) {
 struct TileSet {
     int mode;
     int n_tiles;
-    int n_col_tiles, cb, i0, pslab, ce;               // mode 0 (ce: end of the column range)
+    int n_col_tiles, cb, i0, pslab, ce, rows;         // mode 0 (ce: end of the column range; rows of W)
     int nbk, a_j0, a_j1, n_a, b_i0, b_i1, b_j1, kx;   // mode 1
 };
 
@@ -388,6 +388,386 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
     }
 }
 
+// ------------------------------------------------------------ two-CTA tiles (cta_group::2)
+// A cluster of two CTAs on two SMs computes one 256 x 256 tile. CTA r holds rows
+// [128 r, 128 r + 128) of the tile's A operand and rows [128 r, 128 r + 128) of its B
+// operand (the tile's columns 128 r ..); one tcgen05.mma with M = 256, issued by CTA 0,
+// reads both CTAs' operand slabs and writes each CTA's 128 rows of the accumulator into
+// that CTA's tensor memory. Each SM then stages and reads 128 x k of B per k slab instead
+// of 256 x k: per 32-k slab and SM 64 KB of TMA writes and 96 KB of operand reads for
+// 1536 MMA cycles, against 96 + 144 KB for the same cycles in the one-CTA 128 x 256 tile,
+// whose loop is bound by the 128 bytes per cycle of shared memory. Only the reduce-add
+// epilogue (W never enters shared memory).
+//
+// Synchronization: every CTA loads its own slabs with TMA, the transaction bytes of both
+// landing on CTA 0's `full` barrier (the cta_group::2 form of the copy may signal the peer's
+// barrier); CTA 0's MMA commits arrive on `empty`, `tfull` and `mma_done` of both CTAs
+// (multicast); both CTAs' epilogue warps arrive on CTA 0's `tempty` (16 arrivals). Every
+// wait is bounded as in the one-CTA kernel; both CTAs leave through one cluster barrier.
+constexpr int PBN = 256;                        // tile columns (N of the pair's MMA)
+constexpr int PSTAGES = 3;
+constexpr int P_SLAB = TBM * TBK * 4;           // 16 KB: 128 rows x 32 k
+constexpr int P_STAGE = 4 * P_SLAB;             // A hi, A lo, B hi, B lo of this CTA
+constexpr int P_WBOX = TBM * 32 * 4;            // one 128 x 32 staging box
+constexpr int P_SMEM = PSTAGES * P_STAGE + 2 * P_WBOX + 1024 + 256;
+static_assert(P_SMEM <= 232448, "dynamic shared memory above the per-CTA limit");
+
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+// Address of the same shared variable in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
+    uint32_t d;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(d) : "r"(addr), "r"(rank));
+    return d;
+}
+__device__ __forceinline__ void cluster_barrier() {
+    asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait_cl(uint64_t* bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Bounded wait (as mbar_wait) with cluster scope, for barriers the peer CTA arrives on.
+__device__ __forceinline__ bool mbar_wait_cl(uint64_t* bar, uint32_t parity, volatile int* abort) {
+    if (mbar_try_wait_cl(bar, parity)) return true;
+    const uint64_t t0 = global_timer_ns();
+    for (uint32_t it = 0; it < kWaitLimitIters; ++it) {
+        if (mbar_try_wait_cl(bar, parity)) return true;
+        if (*abort) return false;
+        if ((it & 255u) == 255u && global_timer_ns() - t0 > kWaitLimitNs) break;
+    }
+    *abort = 1;
+    return false;
+}
+// TMA load into this CTA's shared memory whose transaction bytes land on the mbarrier at
+// cluster address `bar` (this CTA's or the peer's).
+__device__ __forceinline__ void tma_load_2d_pair(void* dst, const CUtensorMap* m, uint32_t bar, int x, int y) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(m)), "r"(bar), "r"(x), "r"(y)
+        : "memory");
+}
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t* dst_smem, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst_smem)),
+                 "r"(ncols)
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish_pair() {
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_mma_tf32_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                                 uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+// Arrive once on `bar` (same offset) in both CTAs of the pair when the pair's MMAs issued
+// so far have completed.
+__device__ __forceinline__ void tc_commit_pair(uint64_t* bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+            smem_u32(bar)),
+        "h"(static_cast<uint16_t>(3))
+        : "memory");
+}
+
+// Pair tile t as seen by CTA `rank`: the rows of the A operand it loads (ra; also the rows
+// it writes), the rows of the B operand it loads (rb), the tile's first column (co), whether
+// B and the output come from the second pair of maps, and which of its two 128-column
+// halves it writes.
+//   mode 0: tiles of 256 rows x 256 columns over W[:, cb:ce], column tiles inner.
+//   mode 1: the A region in column-block pairs (a_j0 + 2 p, + 1), each with its row-block
+//     pairs from the diagonal down (the strictly upper block of a diagonal tile is not
+//     written), then the B region in (row pair, column pair) order.
+struct PairTile {
+    int ra, rb, co;
+    bool alt;
+    bool wr0, wr1;
+};
+
+__device__ __forceinline__ PairTile pair_tile_at(const TileSet& ts, int t, int rank) {
+    PairTile p;
+    if (ts.mode == 0) {
+        const int r0 = (t / ts.n_col_tiles) * 2 * TBM;
+        const int c0 = ts.cb + (t % ts.n_col_tiles) * PBN;
+        p.ra = r0 + TBM * rank;
+        p.rb = c0 + TBM * rank;
+        p.co = c0;
+        p.alt = false;
+        p.wr0 = p.ra < ts.rows && c0 < ts.ce;
+        p.wr1 = p.ra < ts.rows && c0 + TBM < ts.ce;
+        return p;
+    }
+    if (t < ts.n_a) {
+        int jp = ts.a_j0;
+        while (t >= (ts.nbk - jp + 1) / 2) {
+            t -= (ts.nbk - jp + 1) / 2;
+            jp += 2;
+        }
+        const int i = jp + 2 * t + rank;
+        p.ra = i * TBM;
+        p.rb = (jp + rank) * TBM;
+        p.co = jp * TBM;
+        p.alt = false;
+        p.wr0 = i < ts.nbk;
+        p.wr1 = i < ts.nbk && jp + 1 < ts.a_j1 && jp + 1 <= i;
+        return p;
+    }
+    t -= ts.n_a;
+    const int ncp = (ts.b_j1 + 1) / 2;
+    const int i = ts.b_i0 + 2 * (t / ncp) + rank;
+    const int j0 = 2 * (t % ncp);
+    p.ra = i * TBM;
+    p.rb = (j0 + rank) * TBM;
+    p.co = j0 * TBM;
+    p.alt = true;
+    p.wr0 = i < ts.b_i1;
+    p.wr1 = i < ts.b_i1 && j0 + 1 < ts.b_j1;
+    return p;
+}
+
+// mA*: the A operand (E, or the split C panel), K slabs at columns xk + 32 s; mB*: the B
+// operand (R, or the split C panel); mB2*: the second B operand (mode 1: the split Z^T
+// rows); mW / mW2: the output for B / B2. Grid: two CTAs per cluster, the clusters walking
+// the tiles (persistent).
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(T_THREADS, 1)
+trail_pair_kernel(const __grid_constant__ CUtensorMap mAh, const __grid_constant__ CUtensorMap mAl,
+                  const __grid_constant__ CUtensorMap mBh, const __grid_constant__ CUtensorMap mBl,
+                  const __grid_constant__ CUtensorMap mB2h, const __grid_constant__ CUtensorMap mB2l,
+                  const __grid_constant__ CUtensorMap mW, const __grid_constant__ CUtensorMap mW2, TileSet ts,
+                  int nslab, int drain, int* info) {
+    const int n_tiles = ts.n_tiles;
+    const int xk = ts.mode == 0 ? ts.i0 : ts.kx;
+    const uint32_t rank = cluster_ctarank();
+    const int pair = static_cast<int>(blockIdx.x >> 1);
+    const int npairs = static_cast<int>(gridDim.x >> 1);
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    uint8_t* wtile = smem + PSTAGES * P_STAGE;    // two staging boxes (one per column half)
+    uint64_t* full = reinterpret_cast<uint64_t*>(wtile + 2 * P_WBOX);
+    uint64_t* empty = full + PSTAGES;
+    uint64_t* tfull = empty + PSTAGES;
+    uint64_t* tempty = tfull + 2;
+    uint64_t* mma_done = tempty + 2;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < PSTAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&tfull[b], 1);
+            mbar_init(&tempty[b], 16);   // 8 epilogue warps in each CTA
+        }
+        mbar_init(mma_done, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc_pair(tmem_slot, 2 * PBN);
+        tmem_relinquish_pair();
+    }
+    if (warp == 0 && lane == 0) {
+        tma_prefetch_desc(&mAh);
+        tma_prefetch_desc(&mAl);
+        tma_prefetch_desc(&mBh);
+        tma_prefetch_desc(&mBl);
+        if (ts.mode == 1) {
+            tma_prefetch_desc(&mB2h);
+            tma_prefetch_desc(&mB2l);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    cluster_barrier();   // both CTAs' barriers initialized before any remote arrival
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    const uint32_t full0 = mapa_shared(smem_u32(full), 0);       // CTA 0's full[0]
+    const uint32_t tempty0 = mapa_shared(smem_u32(tempty), 0);   // CTA 0's tempty[0]
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer (both CTAs)
+        if (lane == 0) {
+            int k = 0;
+            bool ok = true;
+            for (int t = pair; t < n_tiles && ok; t += npairs) {
+                const PairTile pt = pair_tile_at(ts, t, static_cast<int>(rank));
+                const CUtensorMap* bh = pt.alt ? &mB2h : &mBh;
+                const CUtensorMap* bl = pt.alt ? &mB2l : &mBl;
+                for (int s = 0; s < nslab; ++s, ++k) {
+                    const int st = k % PSTAGES;
+                    const uint32_t u = static_cast<uint32_t>(k / PSTAGES);
+                    if (!mbar_wait(&empty[st], (u & 1u) ^ 1u, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    if (rank == 0) mbar_arrive_expect_tx(&full[st], 2 * P_STAGE);
+                    uint8_t* base = smem + st * P_STAGE;
+                    const uint32_t bar = full0 + static_cast<uint32_t>(st * 8);
+                    const int x = xk + s * TBK;
+                    tma_load_2d_pair(base, &mAh, bar, x, pt.ra);
+                    tma_load_2d_pair(base + P_SLAB, &mAl, bar, x, pt.ra);
+                    tma_load_2d_pair(base + 2 * P_SLAB, bh, bar, x, pt.rb);
+                    tma_load_2d_pair(base + 3 * P_SLAB, bl, bar, x, pt.rb);
+                }
+            }
+            // the last slabs consumed by the pair's MMAs (so this CTA's loads have landed)
+            for (int j = (k > PSTAGES ? k - PSTAGES : 0); j < k; ++j)
+                wait_quiet(&empty[j % PSTAGES], static_cast<uint32_t>(j / PSTAGES) & 1u);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer (CTA 0)
+        if (lane == 0) {
+            if (rank == 0) {
+                constexpr uint32_t idesc = idesc_tf32_k_major(2 * TBM, PBN);
+                int k = 0, cc = 0;
+                bool ok = true;
+                for (int t = pair; t < n_tiles && ok; t += npairs) {
+                    for (int s0 = 0; s0 < nslab && ok; s0 += drain, ++cc) {
+                        const int buf = cc & 1;
+                        if (!mbar_wait_cl(&tempty[buf], ((static_cast<uint32_t>(cc) >> 1) & 1u) ^ 1u, abort_flag)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t dt = tmem + static_cast<uint32_t>(buf * PBN);
+                        const int s1 = min(nslab, s0 + drain);
+                        for (int s = s0; s < s1; ++s, ++k) {
+                            const int st = k % PSTAGES;
+                            if (!mbar_wait(&full[st], static_cast<uint32_t>(k / PSTAGES) & 1u, abort_flag)) {
+                                ok = false;
+                                break;
+                            }
+                            tc_fence_after();
+                            const uint32_t a_hi = smem_u32(smem + st * P_STAGE);
+                            const uint32_t a_lo = a_hi + P_SLAB;
+                            const uint32_t b_hi = a_hi + 2 * P_SLAB;
+                            const uint32_t b_lo = a_hi + 3 * P_SLAB;
+#pragma unroll
+                            for (int kk = 0; kk < TBK / 8; ++kk) {
+                                const uint32_t ko = static_cast<uint32_t>(kk * 32);
+                                const uint64_t dah = smem_desc_sw128(a_hi + ko, 16, 1024);
+                                const uint64_t dal = smem_desc_sw128(a_lo + ko, 16, 1024);
+                                const uint64_t dbh = smem_desc_sw128(b_hi + ko, 16, 1024);
+                                const uint64_t dbl = smem_desc_sw128(b_lo + ko, 16, 1024);
+                                tc_mma_tf32_pair(dt, dal, dbh, idesc, (s > s0 || kk > 0) ? 1u : 0u);
+                                tc_mma_tf32_pair(dt, dah, dbl, idesc, 1u);
+                                tc_mma_tf32_pair(dt, dah, dbh, idesc, 1u);
+                            }
+                            tc_commit_pair(&empty[st]);
+                        }
+                        if (ok) tc_commit_pair(&tfull[buf]);
+                    }
+                }
+                tc_commit_pair(mma_done);
+            }
+            wait_quiet(mma_done, 0);
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue (8 warps, both CTAs)
+        // As in the one-CTA reduce-add epilogue: thread = one row of this CTA's 128 rows;
+        // warps 2-5 take columns [0, 128) of the tile, warps 6-9 columns [128, 256).
+        constexpr int HALF = PBN / 2;
+        constexpr int PIECES = HALF / 32;
+        const int q = warp & 3;
+        const int h = (warp - 2) >> 2;
+        const int r = q * 32 + lane;
+        const bool issuer = (warp == 2 + 4 * h) && lane == 0;
+        uint8_t* stg = wtile + h * P_WBOX;
+        int cc = 0;
+        bool ok = true;
+        for (int t = pair; t < n_tiles && ok; t += npairs) {
+            const PairTile pt = pair_tile_at(ts, t, static_cast<int>(rank));
+            const CUtensorMap* wm = pt.alt ? &mW2 : &mW;
+            const int xh = pt.co + h * HALF;
+            const bool wrh = h ? pt.wr1 : pt.wr0;
+            const bool whole = wrh && (ts.mode == 1 || xh + HALF <= ts.ce);
+            for (int s0 = 0; s0 < nslab; s0 += drain, ++cc) {
+                const int buf = cc & 1;
+                ok = mbar_wait(&tfull[buf], (static_cast<uint32_t>(cc) >> 1) & 1u, abort_flag);
+                ok = __all_sync(0xffffffffu, ok) && !*abort_flag;
+                ok = named_bar_all(1 + h, 128, ok);
+                if (!ok) break;
+                tc_fence_after();
+                const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) +
+                                       static_cast<uint32_t>(buf * PBN + h * HALF);
+#pragma unroll 1
+                for (int p = 0; p < PIECES; ++p) {
+                    const int x = xh + 32 * p;
+                    float v[32];
+                    tmem_ld32(taddr + static_cast<uint32_t>(p * 32), v);
+                    tc_wait_ld();
+                    if (p == PIECES - 1) {   // the accumulator may be reused
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive_remote(tempty0 + static_cast<uint32_t>(buf * 8));
+                    }
+                    if (!wrh || (ts.mode == 0 && x >= ts.ce)) continue;   // same for the whole half
+                    float4* rowp = reinterpret_cast<float4*>(stg + r * 128);
+#pragma unroll
+                    for (int c = 0; c < 8; ++c)
+                        rowp[c ^ (r & 7)] = make_float4(-v[4 * c], -v[4 * c + 1], -v[4 * c + 2], -v[4 * c + 3]);
+                    fence_proxy_async();
+                    named_bar_sync(1 + h, 128);
+                    if (issuer) {
+                        // the same box of the previous chunk lands first (block order per element)
+                        if (whole)
+                            bulk_wait_le<PIECES - 1>();
+                        else
+                            bulk_wait_le<0>();
+                        tma_reduce_add_2d(wm, stg, x, pt.ra);
+                        bulk_commit();
+                        bulk_wait_read0();
+                    }
+                    named_bar_sync(1 + h, 128);
+                }
+            }
+        }
+        if ((warp == 2 || warp == 6) && lane == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (*abort_flag && threadIdx.x == 0) {
+        record_error(info, -KQ_ERR_TIMEOUT);
+        // copies this CTA issued toward the peer's barriers have had time to land
+        const uint64_t t0 = global_timer_ns();
+        while (global_timer_ns() - t0 < 1000000ull) {
+        }
+    }
+    cluster_barrier();   // neither CTA leaves while the other may still signal it
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc_pair(tmem, 2 * PBN);
+    }
+}
+
 __global__ void split_tf32_kernel(const float* __restrict__ src, int64_t n, float* __restrict__ hi,
                                   float* __restrict__ lo) {
     for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
@@ -549,6 +929,43 @@ int long_drain_slabs() {
     return n;
 }
 
+// Whether the K > 128 updates run on the two-CTA kernel: yes unless the environment
+// variable KQ_TRAIL_PAIR says 0 (a tuning switch).
+bool pair_enabled() {
+    static const bool on = [] {
+        const char* e = std::getenv("KQ_TRAIL_PAIR");
+        return !(e && std::atoi(e) == 0);
+    }();
+    return on;
+}
+
+kq_status launch_pair(const CUtensorMap& ah, const CUtensorMap& al, const CUtensorMap& bh, const CUtensorMap& bl,
+                      const CUtensorMap& b2h, const CUtensorMap& b2l, const CUtensorMap& w, const CUtensorMap& w2,
+                      const TileSet& ts, int nslab, int drain, int* info, cudaStream_t stream) {
+    static std::atomic<uint64_t> attr{0};
+    static std::atomic<int> clusters{0};
+    KQ_TRY(once_per_device(attr, [&]() -> kq_status {
+        KQ_CUDA(cudaFuncSetAttribute(trail_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, P_SMEM));
+        KQ_CUDA(cudaFuncSetAttribute(trail_pair_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                     cudaSharedmemCarveoutMaxShared));
+        // clusters resident at once (pairs of SMs that can both take a CTA)
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(static_cast<unsigned>(2 * num_sms()));
+        cfg.blockDim = dim3(T_THREADS);
+        cfg.dynamicSmemBytes = P_SMEM;
+        int c = 0;
+        KQ_CUDA(cudaOccupancyMaxActiveClusters(&c, trail_pair_kernel, &cfg));
+        clusters.store(c > 0 ? c : num_sms() / 2);
+        return KQ_OK;
+    }));
+    if (ts.n_tiles == 0) return KQ_OK;
+    const int nc = std::min(ts.n_tiles, clusters.load());
+    trail_pair_kernel<<<static_cast<unsigned>(2 * nc), T_THREADS, P_SMEM, stream>>>(ah, al, bh, bl, b2h, b2l, w, w2,
+                                                                                    ts, nslab, drain, info);
+    KQ_LAUNCH_CHECK("trail_pair_kernel");
+    return KQ_OK;
+}
+
 template <int BN, int STAGES>
 kq_status launch_trail_red(const TrailMaps& m, const CUtensorMap& rh, const CUtensorMap& rl, int64_t d_out,
                            int64_t i0, int kb, int64_t cb, int64_t ce, int* info, cudaStream_t stream) {
@@ -591,6 +1008,19 @@ kq_status trail_tc_long(const TrailMaps& m, int64_t d_out, int64_t d_in, int64_t
         return KQ_ERR_INVALID_ARG;
     }
     if (ce <= cb) return KQ_OK;
+    if (bn == 256 && pair_enabled()) {
+        TileSet ts{};
+        ts.mode = 0;
+        ts.n_col_tiles = static_cast<int>(cdiv(ce - cb, PBN));
+        ts.n_tiles = static_cast<int>(cdiv(d_out, 2 * TBM)) * ts.n_col_tiles;
+        ts.cb = static_cast<int>(cb);
+        ts.i0 = static_cast<int>(i0);
+        ts.pslab = 1 << 30;
+        ts.ce = static_cast<int>(ce);
+        ts.rows = static_cast<int>(d_out);
+        return launch_pair(m.eh, m.el, m.rh_narrow, m.rl_narrow, m.rh_narrow, m.rl_narrow, m.w, m.w, ts,
+                           static_cast<int>(cdiv(kb, TBK)), long_drain_slabs(), info, stream);
+    }
     if (bn == 256) return launch_trail_red<256, 2>(m, m.rh256, m.rl256, d_out, i0, kb, cb, ce, info, stream);
     return launch_trail_red<128, 3>(m, m.rh_narrow, m.rl_narrow, d_out, i0, kb, cb, ce, info, stream);
 }
@@ -611,6 +1041,23 @@ kq_status CholTcMaps::init(float* A, float* Z, int64_t npad, int width, int nset
 
 kq_status chol_update_tc(const CholTcMaps& m, int set, int nbk, int a_j0, int a_j1, int b_i0, int b_i1, int b_j1,
                          int kx, int nslab, int* info, cudaStream_t stream) {
+    if (nslab > TNSLAB && pair_enabled()) {
+        // a super-panel's update (K > 128): 256 x 256 tiles on CTA pairs
+        TileSet ts{};
+        ts.mode = 1;
+        ts.nbk = nbk;
+        ts.a_j0 = a_j0;
+        ts.a_j1 = a_j1;
+        for (int jp = a_j0; jp < a_j1; jp += 2) ts.n_a += (nbk - jp + 1) / 2;
+        ts.b_i0 = b_i0;
+        ts.b_i1 = b_i1;
+        ts.b_j1 = b_j1;
+        ts.kx = kx;
+        ts.ce = 1 << 30;
+        ts.n_tiles = ts.n_a + ((b_i1 > b_i0 && b_j1 > 0) ? ((b_i1 - b_i0 + 1) / 2) * ((b_j1 + 1) / 2) : 0);
+        return launch_pair(m.ch[set], m.cl[set], m.ch[set], m.cl[set], m.zh[set], m.zl[set], m.a, m.z, ts, nslab,
+                           long_drain_slabs(), info, stream);
+    }
     // 128 x 128 tiles, three-stage operand ring, the tiles of A and Z updated by TMA
     // reduce-adds (no shared-memory copy of the tile)
     using Cfg = TrailCfg<128, 3, true>;

@@ -111,7 +111,9 @@ struct CholTcMaps {
 
 // A Cholesky update on the tensor cores (3xTF32): A_ij -= C_i. C_j.^T for the lower tiles with
 // j in [a_j0, a_j1), i >= j, and Z_ij -= C_i. Z_.j for i in [b_i0, b_i1), j < b_j1, where the
-// dot runs over the nslab * 32 split columns starting at kx of split set `set`.
+// dot runs over the nslab * 32 split columns starting at kx of split set `set`. One block's K
+// (nslab = 4): 128 x 128 tiles on single CTAs; more (a super-panel's update): 256 x 256 tiles
+// of 128 x 128 blocks on pairs of CTAs (unless KQ_TRAIL_PAIR=0).
 kq_status chol_update_tc(const CholTcMaps& m, int set, int nbk, int a_j0, int a_j1, int b_i0, int b_i1, int b_j1,
                          int kx, int nslab, int* info, cudaStream_t stream);
 
@@ -128,9 +130,11 @@ kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, in
 
 // The same update for K = kb <= 1024 (the blocks of one super-panel, GPTQ mode), applied to
 // W two blocks' K at a time in block order (the accumulator drained every 256 of K), through
-// TMA reduce-adds instead of a shared-memory copy of the W tile: 128 x 256 tiles (bn = 256,
-// two-stage operand ring) or 128 x 128 (bn = 128, three stages). [cb, ce) whole tiles or
-// ending at d_in; kb whole blocks unless the super-panel ends at d_in.
+// TMA reduce-adds instead of a shared-memory copy of the W tile. bn = 256: 256 x 256 tiles
+// on pairs of CTAs (cta_group::2, three-stage ring per CTA; with KQ_TRAIL_PAIR=0 in the
+// environment, 128 x 256 tiles on single CTAs, two stages); bn = 128: 128 x 128 tiles, three
+// stages. [cb, ce) whole tiles or ending at d_in; kb whole blocks unless the super-panel
+// ends at d_in.
 kq_status trail_tc_long(const TrailMaps& m, int64_t d_out, int64_t d_in, int64_t i0, int kb, int64_t cb, int64_t ce,
                         int bn, int* info, cudaStream_t stream);
 
