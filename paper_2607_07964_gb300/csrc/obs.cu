@@ -417,7 +417,8 @@ __global__ void __launch_bounds__(HASP ? OBS_THREADS_P : OBS_THREADS, HASP ? 1 :
         for (int o = 0; o < LPR; ++o) {
             if (CPL * o >= nb) break;   // uniform across the CTA
             float e[CPL];
-            float wq[HASP ? CPL : 1];
+            float wq[HASP ? CPL : 1];   // the values before quantization (with P only)
+            (void)wq;
             uint32_t cq[NV];
 #pragma unroll
             for (int v = 0; v < NV; ++v) cq[v] = 0u;
