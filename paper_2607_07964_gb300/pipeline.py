@@ -110,6 +110,12 @@ class LayerPipeline:
         c = self.chunk_tokens[which]
         c = c if c > 0 else max(T, 1)
         ch = [(t0, min(T, t0 + c)) for t0 in range(0, max(T, 1), c)]
+        if which == "X" and self.chunk_tokens["X"] > 0 and len(ch) > 1:
+            # the first chunk in four: on the host path the accumulation of H_X starts once a
+            # quarter chunk has arrived (the later chunks arrive faster than they are summed)
+            t0, t1 = ch.pop(0)
+            q = max(1, -(-(t1 - t0) // 4))
+            ch = [(a, min(t1, a + q)) for a in range(t0, t1, q)] + ch
         if which == "G" and self.chunk_tokens["G"] > 0 and len(ch) > 1:
             # the last chunk in four: after G's last bytes arrive on the host path, only a
             # quarter chunk of accumulation stands before S_G, U and the sweep
@@ -335,9 +341,9 @@ class LayerPipeline:
         layer's inputs to the device, run the four stages, copy codes and grids back.
         Enqueued on `stream`; the caller synchronizes. Returns (bytes in, bytes out).
 
-        The copies run on their own stream in the order W, signs, X chunks, G chunks, and
-        each chunk's factor accumulation starts as soon as that chunk has arrived, so the
-        host link (the bound at these sizes) overlaps the factor, rescale, rotation and
+        The copies run on their own stream in the order X chunks, W, signs, G chunks (W is
+        first needed after H_X), and each chunk's factor accumulation starts as soon as that
+        chunk has arrived, so the host link overlaps the factor, rescale, rotation and
         Cholesky work; without the two-stream schedule the copies simply precede the run."""
         self._need_xt(Xt_h)
         s = torch.cuda.current_stream() if stream is None else stream
@@ -371,10 +377,6 @@ class LayerPipeline:
             e0.record(s)
             cs.wait_event(e0)
             with torch.cuda.stream(cs):
-                for k, h in (("W", W_h), ("su", su_h), ("sv", sv_h)):
-                    st[k].copy_(h, non_blocking=True)
-                w_ready = torch.cuda.Event()
-                w_ready.record(cs)
                 ready = {}
                 for k, h in (("X", X_h), ("G", G_h)):
                     ready[k] = []
@@ -383,10 +385,15 @@ class LayerPipeline:
                         ev = torch.cuda.Event()
                         ev.record(cs)
                         ready[k].append(ev)
-                    if k == "X" and Xt_h is not None:   # X~ right after X: the drift needs both
-                        st["Xt"].copy_(Xt_h, non_blocking=True)
-                        xt_ready = torch.cuda.Event()
-                        xt_ready.record(cs)
+                    if k == "X":
+                        if Xt_h is not None:   # X~ right after X: the drift needs both
+                            st["Xt"].copy_(Xt_h, non_blocking=True)
+                            xt_ready = torch.cuda.Event()
+                            xt_ready.record(cs)
+                        for kk, hh in (("W", W_h), ("su", su_h), ("sv", sv_h)):
+                            st[kk].copy_(hh, non_blocking=True)
+                        w_ready = torch.cuda.Event()
+                        w_ready.record(cs)
             self._run_overlapped(st["X"], st["G"], st["W"], st["su"], st["sv"], s, x_ready=ready["X"],
                                  g_ready=ready["G"], w_ready=w_ready, Xt=st.get("Xt"),
                                  xt_ready=xt_ready if Xt_h is not None else None)
