@@ -100,6 +100,34 @@ __global__ void prep_kernel(const float* __restrict__ H, int64_t n, int64_t npad
     }
 }
 
+// The same with 16-byte accesses (n % 4 == 0, H 16-byte aligned): four columns per
+// thread and step, H's row read as reversed float4 quads.
+__global__ void prep4_kernel(const float* __restrict__ H, int64_t n, int64_t npad, float damp_rel,
+                             const double* __restrict__ dsum, float* __restrict__ A, float* __restrict__ Z) {
+    const float delta = static_cast<float>(static_cast<double>(damp_rel) * (*dsum / static_cast<double>(n)));
+    const int64_t nq = npad / 4, total = npad * nq;
+    for (int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < total;
+         e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t i = e / nq, j = 4 * (e - i * nq);
+        float v[4];
+        if (i < n && j < n) {   // the whole quad (n % 4 == 0): A[i][j + t] = H[n-1-i][n-1-j-t]
+            const float4 h = *reinterpret_cast<const float4*>(H + (n - 1 - i) * n + (n - 4 - j));
+            v[0] = h.w;
+            v[1] = h.z;
+            v[2] = h.y;
+            v[3] = h.x;
+            if (i >= j && i < j + 4) v[i - j] += delta;
+        } else {
+#pragma unroll
+            for (int t = 0; t < 4; ++t) v[t] = (i == j + t) ? 1.0f : 0.0f;
+        }
+        if (KQ_IN_RANGE(4 * e + 3, npad * npad)) {
+            reinterpret_cast<float4*>(A)[e] = make_float4(v[0], v[1], v[2], v[3]);
+            reinterpret_cast<float4*>(Z)[e] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+        }
+    }
+}
+
 // ---------------------------------------------------------------- diag block
 // Factor A_kk = C C^T and invert C on one CTA, as an L D L^T sweep that builds L^-1 in
 // place (Gauss-Jordan on the lower triangle), four columns per barrier.
@@ -639,6 +667,42 @@ __global__ void finish_kernel(const float* __restrict__ Z, int64_t n, int64_t np
     }
 }
 
+// The same with 64 x 64 tiles and 16-byte accesses (n % 4 == 0, Lt 16-byte aligned): the
+// tile of Lt at (i0, j0) reads rows a = n-1-j of Z over columns n-1-i, a quad at a time
+// (reversed into shared memory), and writes quads of Lt's rows; tiles wholly above the
+// diagonal only write zeros.
+__global__ void __launch_bounds__(256) finish4_kernel(const float* __restrict__ Z, int64_t n, int64_t npad,
+                                                      float* __restrict__ Lt) {
+    __shared__ float t[64][65];   // t[jj][ii] = Lt[i0 + ii][j0 + jj]
+    const int64_t i0 = static_cast<int64_t>(blockIdx.y) * 64, j0 = static_cast<int64_t>(blockIdx.x) * 64;
+    const int q = threadIdx.x & 15, r0 = threadIdx.x >> 4;   // 16 quads x 16 rows per pass
+    const bool above = j0 > i0 + 63;
+    if (!above) {
+        for (int jj = r0; jj < 64; jj += 16) {
+            const int64_t j = j0 + jj;
+            // Z row n-1-j, columns n-64-i0 + 4q .. +3, i.e. ii = 63-4q-u for u = 0..3
+            const int64_t c = n - 64 - i0 + 4 * q;
+            float4 z = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+            if (j < n && c >= 0) z = *reinterpret_cast<const float4*>(Z + (n - 1 - j) * npad + c);
+            const float zv[4] = {z.x, z.y, z.z, z.w};
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int ii = 63 - 4 * q - u;
+                const int64_t i = i0 + ii;
+                t[jj][ii] = (j < n && i < n && j <= i) ? zv[u] : 0.0f;
+            }
+        }
+    }
+    __syncthreads();
+    for (int ii = r0; ii < 64; ii += 16) {
+        const int64_t i = i0 + ii, j = j0 + 4 * q;
+        if (i >= n || j >= n) continue;   // whole quads (n % 4 == 0)
+        float4 v = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+        if (!above) v = make_float4(t[4 * q][ii], t[4 * q + 1][ii], t[4 * q + 2][ii], t[4 * q + 3][ii]);
+        if (KQ_IN_RANGE(i * n + j + 3, n * n)) *reinterpret_cast<float4*>(Lt + i * n + j) = v;
+    }
+}
+
 }  // namespace
 
 KQ_DEBUG_UNIT(chol)
@@ -692,9 +756,15 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
     diag_sum_kernel<<<1, 1024, 0, stream>>>(H, n, w.dsum);
     KQ_LAUNCH_CHECK("diag_sum_kernel");
     const int64_t total = npad * npad;
-    const int64_t pgrid = std::min<int64_t>(cdiv(total, 256), static_cast<int64_t>(num_sms()) * 32);
-    prep_kernel<<<static_cast<unsigned>(pgrid), 256, 0, stream>>>(H, n, npad, damp_rel, w.dsum, w.A, w.Z);
-    KQ_LAUNCH_CHECK("prep_kernel");
+    if (n % 4 == 0 && (reinterpret_cast<uintptr_t>(H) & 15u) == 0) {
+        const int64_t g4 = std::min<int64_t>(cdiv(total / 4, 256), static_cast<int64_t>(num_sms()) * 32);
+        prep4_kernel<<<static_cast<unsigned>(g4), 256, 0, stream>>>(H, n, npad, damp_rel, w.dsum, w.A, w.Z);
+        KQ_LAUNCH_CHECK("prep4_kernel");
+    } else {
+        const int64_t pgrid = std::min<int64_t>(cdiv(total, 256), static_cast<int64_t>(num_sms()) * 32);
+        prep_kernel<<<static_cast<unsigned>(pgrid), 256, 0, stream>>>(H, n, npad, damp_rel, w.dsum, w.A, w.Z);
+        KQ_LAUNCH_CHECK("prep_kernel");
+    }
     SideStream* side = nbk > 2 ? side_stream(stream) : nullptr;
     bool forked = false, remote_pending = false;
     bool next_pending = false;   // the next panel's tiles, updated on the side stream
@@ -791,9 +861,15 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
     }
     if (forked) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));
     if (remote_pending) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[1], 0));
-    finish_kernel<<<dim3(static_cast<unsigned>(cdiv(n, 32)), static_cast<unsigned>(cdiv(n, 32))),
-                    dim3(32, 8), 0, stream>>>(w.Z, n, npad, Lt);
-    KQ_LAUNCH_CHECK("finish_kernel");
+    if (n % 4 == 0 && (reinterpret_cast<uintptr_t>(Lt) & 15u) == 0) {
+        finish4_kernel<<<dim3(static_cast<unsigned>(cdiv(n, 64)), static_cast<unsigned>(cdiv(n, 64))), 256, 0,
+                         stream>>>(w.Z, n, npad, Lt);
+        KQ_LAUNCH_CHECK("finish4_kernel");
+    } else {
+        finish_kernel<<<dim3(static_cast<unsigned>(cdiv(n, 32)), static_cast<unsigned>(cdiv(n, 32))),
+                        dim3(32, 8), 0, stream>>>(w.Z, n, npad, Lt);
+        KQ_LAUNCH_CHECK("finish_kernel");
+    }
     return KQ_OK;
 }
 

@@ -203,9 +203,11 @@ def test_chol_inv_parity(d_in, T):
     assert rel_fro(got, Lref) <= 1e-5
 
 
-@pytest.mark.parametrize("n", [200, 300])
+@pytest.mark.parametrize("n", [200, 300, 203, 1154])
 def test_chol_inv_ragged(n):
-    """n not a multiple of the 128 block: padded with an identity block internally."""
+    """n not a multiple of the 128 block: padded with an identity block internally (n % 4
+    != 0 also takes the scalar reversal kernels instead of the quad ones; 1154 has two
+    levels of super-panels)."""
     H = kqsynth.random_spd(n, seed=n, cond_decay=1.0).astype(np.float32)
     Lref = ref.lower_factor(ref.damp(H.astype(np.float64), 0.01))
     Lt = torch.empty((n, n), device=DEV)
@@ -213,7 +215,26 @@ def test_chol_inv_ragged(n):
     ws = torch.empty(K().kq_chol_inv_workspace(n), dtype=torch.uint8, device=DEV)
     K().kq_chol_inv(dev(H), 0.01, Lt, info, ws)
     assert K().kq_check(info)[0] == 0
-    assert rel_fro(host(Lt), Lref) <= 1e-5
+    got = host(Lt)
+    assert np.array_equal(np.triu(got, 1), np.zeros_like(got))
+    assert rel_fro(got, Lref) <= 1e-5
+
+
+def test_chol_inv_unaligned_buffers():
+    """H and Lt at 4-byte offsets (no 16-byte alignment): the scalar reversal kernels, the
+    same result as aligned buffers bit for bit."""
+    n = 256
+    H = kqsynth.random_spd(n, seed=7, cond_decay=1.0).astype(np.float32)
+    ws = torch.empty(K().kq_chol_inv_workspace(n), dtype=torch.uint8, device=DEV)
+    info = torch.zeros(1, dtype=torch.int32, device=DEV)
+    Lt = torch.empty((n, n), device=DEV)
+    K().kq_chol_inv(dev(H), 0.01, Lt, info, ws)
+    Hbuf = torch.empty(n * n + 1, device=DEV)
+    Hbuf[1:] = dev(H).reshape(-1)
+    Lbuf = torch.empty(n * n + 1, device=DEV)
+    K().kq_chol_inv(Hbuf[1:].view(n, n), 0.01, Lbuf[1:].view(n, n), info, ws)
+    assert K().kq_check(info)[0] == 0
+    assert torch.equal(Lbuf[1:].view(n, n), Lt)
 
 
 def test_chol_inv_not_pd_reports_pivot():
