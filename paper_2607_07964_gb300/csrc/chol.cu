@@ -116,7 +116,9 @@ __global__ void prep4_kernel(const float* __restrict__ H, int64_t n, int64_t npa
             v[1] = h.z;
             v[2] = h.y;
             v[3] = h.x;
-            if (i >= j && i < j + 4) v[i - j] += delta;
+#pragma unroll
+            for (int t = 0; t < 4; ++t)
+                if (i == j + t) v[t] += delta;
         } else {
 #pragma unroll
             for (int t = 0; t < 4; ++t) v[t] = (i == j + t) ? 1.0f : 0.0f;
