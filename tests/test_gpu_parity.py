@@ -203,11 +203,12 @@ def test_chol_inv_parity(d_in, T):
     assert rel_fro(got, Lref) <= 1e-5
 
 
-@pytest.mark.parametrize("n", [200, 300, 203, 1154])
+@pytest.mark.parametrize("n", [200, 300, 203, 1154, 1300])
 def test_chol_inv_ragged(n):
     """n not a multiple of the 128 block: padded with an identity block internally (n % 4
-    != 0 also takes the scalar reversal kernels instead of the quad ones; 1154 has two
-    levels of super-panels)."""
+    != 0 also takes the scalar reversal kernels instead of the quad ones; 1154 and 1300
+    have two levels of super-panels, 1300's second one three blocks wide, so its update
+    on CTA pairs ends in a pair with one column block past the range)."""
     H = kqsynth.random_spd(n, seed=n, cond_decay=1.0).astype(np.float32)
     Lref = ref.lower_factor(ref.damp(H.astype(np.float64), 0.01))
     Lt = torch.empty((n, n), device=DEV)
