@@ -401,9 +401,11 @@ def fractions(cfg, stage_ms: dict, peaks: dict, peak_src: str) -> dict:
     fl = algorithmic_flops(cfg)
     out = {"peaks": {"bf16_tflops": bf16, "tf32_tflops": tf32, "hbm_gbs": hbm,
                      "source": f"{peak_src}; tf32 = {tf32_src}"}}
+    bf16_s = float(peaks.get("bf16_tflops_sustained", bf16))
+    out["peaks"]["bf16_tflops_sustained"] = bf16_s
     for k in ("factor_x", "factor_g"):
         t = fl[k] / stage_ms[k] / 1e9
-        out[k] = {"tflops": t, "frac_bf16": t / bf16}
+        out[k] = {"tflops": t, "frac_bf16": t / bf16, "frac_bf16_sustained": t / bf16_s}
     for k, name in (("chol", "chol"), ("sweep", "sweep_trailing")):
         t = fl[k] / stage_ms[k] / 1e9
         out[name] = {"tflops_algorithmic": t, "frac_tf32_algorithmic": t / tf32,
@@ -543,14 +545,22 @@ def run_ours(args):
         tflops["drift"] = fl["drift"] / stage_ms["drift"] / 1e9
         tflops["p"] = fl["p"] / stage_ms["p"] / 1e9
     peaks, peak_src = measured_peaks()
-    peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+    burst = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+    sustained = float(peaks.get("bf16_tflops_sustained", burst))
     # factor_x is one SYRK launch per token chunk: flops per launch / mean launch time.
     n_launch = len(p._chunks("X", cfg.T))
     achieved = tflops["factor_x"]
     traffic = syrk_traffic(cfg, cfg.T // n_launch)
+    # A launch of tens of milliseconds inside back-to-back layer steps runs under the power
+    # cap: its peak is the sustained figure; a short launch is compared with the burst one.
+    long_launch = stage_ms["factor_x"] / n_launch >= 10.0
+    peak = sustained if long_launch else burst
     roofline = {"kernel": "syrk_tc_kernel (H_X = X^T X)", "bound": "tensor", "achieved": achieved,
                 "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak, "traffic": traffic,
-                "peak_source": f"{peak_src} bf16 dense burst (of measured)",
+                "peak_source": (f"{peak_src} bf16 dense sustained (of measured: the launch lasts "
+                                f"{stage_ms['factor_x'] / n_launch:.0f} ms inside back-to-back layer steps)"
+                                if long_launch else f"{peak_src} bf16 dense burst (of measured)"),
+                "frac_of_burst": achieved / burst, "frac_of_sustained": achieved / sustained,
                 "algorithmic_flops_per_launch": fl["factor_x"] / n_launch, "launches_per_factor": n_launch,
                 "timing": "CUDA events around the H_X stage of the serialized pass (one launch, on its stream)"}
     if drift:
@@ -558,10 +568,10 @@ def run_ours(args):
         # flops of (X~ - X)^T X over the stage time; the split pair executes twice as many
         a = tflops["drift"]
         roofline = {"kernel": "drift stage (drift_split_kernel + drift_tc_kernel, D = (X~ - X)^T X)",
-                    "bound": "tensor", "achieved": a, "peak": peak, "unit": "TFLOP/s", "frac": a / peak,
+                    "bound": "tensor", "achieved": a, "peak": burst, "unit": "TFLOP/s", "frac": a / burst,
                     "traffic": None, "peak_source": f"{peak_src} bf16 dense burst",
                     "algorithmic_flops_per_launch": fl["drift"], "executed_flops_per_launch": 2 * fl["drift"],
-                    "executed_frac": 2 * a / peak, "syrk_h_x": roofline}
+                    "executed_frac": 2 * a / burst, "syrk_h_x": roofline}
 
     e2e = None
     if not args.no_e2e:
