@@ -159,54 +159,43 @@ __global__ void __launch_bounds__((1 << LG) / 16) rht_rows_reg_kernel(float* __r
 // ------------------------------------------- row transform in registers, n = 28 * 2^LG
 // For n = 28 P (P = 2^LG, LG in [9, 10]: 14336 and 28672) with index j = a P + b (b
 // fastest): every chunk a of P contiguous elements takes the Walsh-Hadamard transform H_P,
-// then every column b takes the 28-point mix across the chunks. Seven groups of P / 16
-// threads; group g transforms chunks g, g + 7, g + 14, g + 21 one after another with the
-// four-bit register phases of rht.cuh (each group with its own exchange buffer) and leaves
-// them in a shared-memory copy of the row; then each thread mixes whole columns b
-// (mix28_paley) and writes the 28 results straight to global memory, consecutive threads
-// at consecutive b. While chunk c of a row is transformed, chunk c of the CTA's next row is
-// already on its way into the register slot the current chunk left, so the whole next row
-// is in flight during the mixes. One CTA per SM (the row copy is 112 KB at n = 28672).
+// then every column b takes the 28-point mix across the chunks. Fourteen groups of P / 16
+// threads; group g transforms chunks g and g + 14 one after the other with the four-bit
+// register phases of rht.cuh (each group with its own exchange buffer) and leaves them in
+// a shared-memory copy of the row; then each thread mixes whole columns b (mix28_paley)
+// and writes the 28 results straight to global memory, consecutive threads at consecutive
+// b. At n = 28672 the 112 KB row copy leaves one CTA (28 warps) per SM, at 14336 two; the
+// warps of the other groups keep loads in flight while one group waits on its chunk.
+// (Seven groups of four chunks each, with the next row prefetched into registers,
+// measured 14.6-14.8 against 13.3 ms for the rotation stage of the 70B down_proj layer.)
 template <int LG, bool POST>
-__global__ void __launch_bounds__(7 * (1 << LG) / 16, 1) rht_rows28_reg_kernel(float* __restrict__ M, int64_t rows,
-                                                                             int pre_mode, int post_mode,
-                                                                             const int8_t* __restrict__ sign,
-                                                                             const float* __restrict__ s,
-                                                                             float inv_sqrt_n) {
-    constexpr int P = 1 << LG, N = 28 * P, TG = P / 16, T = 7 * TG, NPH = rr_phases(LG);
+__global__ void __launch_bounds__(14 * (1 << LG) / 16, 1) rht_rows28_reg_kernel(float* __restrict__ M, int64_t rows,
+                                                                              int pre_mode, int post_mode,
+                                                                              const int8_t* __restrict__ sign,
+                                                                              const float* __restrict__ s,
+                                                                              float inv_sqrt_n) {
+    constexpr int G = 14, P = 1 << LG, N = 28 * P, TG = P / 16, T = G * TG, NPH = rr_phases(LG), CPG = 28 / G;
     constexpr uint32_t ML = rr_mask(LG, NPH - 1);
     static_assert(NPH == 3, "three register phases for P = 512 and 1024");
     extern __shared__ __align__(16) float sm28[];
     float* v = sm28;                                         // [N]
     const int t = threadIdx.x, g = t / TG, tl = t - g * TG;
     float* buf = sm28 + N + g * (P + P / 32);                // this group's exchange buffer
-    auto load = [&](int64_t row, int c, float (&x)[16]) {
-        const float4* src = reinterpret_cast<const float4*>(M + row * N + (g + 7 * c) * P + 16 * tl);
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const float4 a = src[q];
-            x[4 * q] = a.x;
-            x[4 * q + 1] = a.y;
-            x[4 * q + 2] = a.z;
-            x[4 * q + 3] = a.w;
-        }
-    };
-    float cur[4][16];
-    int64_t r = blockIdx.x;
-    if (r < rows) {
-#pragma unroll
-        for (int c = 0; c < 4; ++c) load(r, c, cur[c]);
-    }
     const int tw = deposit_bits<(P - 1) & ~ML>(tl);
-    for (; r < rows; r += gridDim.x) {
-        const bool more = r + gridDim.x < rows;
+    for (int64_t r = blockIdx.x; r < rows; r += gridDim.x) {
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
+        for (int c = 0; c < CPG; ++c) {
+            const int a = g + G * c;
             float x[16];
+            const float4* src = reinterpret_cast<const float4*>(M + r * N + a * P + 16 * tl);
 #pragma unroll
-            for (int k = 0; k < 16; ++k) x[k] = cur[c][k];
-            if (more) load(r + gridDim.x, c, cur[c]);
-            const int a = g + 7 * c;
+            for (int q = 0; q < 4; ++q) {
+                const float4 w4 = src[q];
+                x[4 * q] = w4.x;
+                x[4 * q + 1] = w4.y;
+                x[4 * q + 2] = w4.z;
+                x[4 * q + 3] = w4.w;
+            }
             float f[16];
             factors16(pre_mode, sign, s, a * P + 16 * tl, f);
 #pragma unroll
@@ -657,8 +646,8 @@ kq_status launch_rows_reg(float* M, int64_t rows, int pre, int post, const int8_
 template <int LG>
 kq_status launch_rows28_reg(float* M, int64_t rows, int pre, int post, const int8_t* sign, const float* s,
                             cudaStream_t stream) {
-    constexpr int P = 1 << LG, T = 7 * P / 16;
-    constexpr size_t smem = (28 * static_cast<size_t>(P) + 7 * (P + P / 32)) * sizeof(float);
+    constexpr int P = 1 << LG, T = 14 * P / 16;
+    constexpr size_t smem = (28 * static_cast<size_t>(P) + 14 * (P + P / 32)) * sizeof(float);
     static std::atomic<uint64_t> attr{0};
     KQ_TRY(once_per_device(attr, [&]() -> kq_status {
         KQ_CUDA(cudaFuncSetAttribute(rht_rows28_reg_kernel<LG, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
