@@ -164,12 +164,14 @@ __global__ void __launch_bounds__((1 << LG) / 16) rht_rows_reg_kernel(float* __r
 // register phases of rht.cuh (each group with its own exchange buffer) and leaves them in
 // a shared-memory copy of the row; then each thread mixes whole columns b (mix28_paley)
 // and writes the 28 results straight to global memory, consecutive threads at consecutive
-// b. At n = 28672 the 112 KB row copy leaves one CTA (28 warps) per SM, at 14336 two; the
+// b. At n = 28672 the 112 KB row copy leaves one CTA (28 warps) per SM, at 14336 two (the
+// launch bound holds the registers to what two CTAs of 14 warps can share: down_8b's
+// rotation stage 2.89 -> 2.42 ms against one CTA per SM); the
 // warps of the other groups keep loads in flight while one group waits on its chunk.
 // (Seven groups of four chunks each, with the next row prefetched into registers,
 // measured 14.6-14.8 against 13.3 ms for the rotation stage of the 70B down_proj layer.)
 template <int LG, bool POST>
-__global__ void __launch_bounds__(14 * (1 << LG) / 16, 1) rht_rows28_reg_kernel(float* __restrict__ M, int64_t rows,
+__global__ void __launch_bounds__(14 * (1 << LG) / 16, LG == 9 ? 2 : 1) rht_rows28_reg_kernel(float* __restrict__ M, int64_t rows,
                                                                               int pre_mode, int post_mode,
                                                                               const int8_t* __restrict__ sign,
                                                                               const float* __restrict__ s,
