@@ -37,16 +37,6 @@ namespace {
 constexpr int BLK = 128;          // block size B (Algorithm 2); the only supported value
 constexpr int SPB = 8;            // blocks per super-panel of the two-level lazy update
 
-// Column width of the long (super-panel) update tiles: 256, or 128 when the environment
-// variable KQ_TRAIL_TILE_N says so (a tuning switch; both give the same sums per tile).
-int long_tile_n() {
-    static const int n = [] {
-        const char* e = std::getenv("KQ_TRAIL_TILE_N");
-        return (e && std::atoi(e) == 128) ? 128 : 256;
-    }();
-    return n;
-}
-
 struct Grid {
     float scale, zero;
 };
@@ -868,7 +858,6 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
     const bool two_level = tc && !hp && !fuse && nblk > SPB;
     if (two_level) {
         constexpr int64_t SPW = static_cast<int64_t>(SPB) * BLK;
-        const int bn = long_tile_n();
         bool in_pending = false;    // the in-panel update of the previous block (side stream)
         bool far_pending = false;   // the far update of the previous super-panel (second side stream)
         cudaStream_t s_in = side ? side->s : stream;
@@ -906,11 +895,11 @@ extern "C" kq_status kq_obs_quantize(float* W, int64_t d_out, int64_t d_in, cons
                     KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[0], 0));
                     far_pending = false;
                 }
-                st = trail_tc_long(maps, d_out, d_in, sp0, static_cast<int>(spe - sp0), spe, sp1, bn, info, stream);
+                st = trail_tc_long(maps, d_out, d_in, sp0, static_cast<int>(spe - sp0), spe, sp1, info, stream);
                 if (st != KQ_OK) return st;
                 if (sp1 < d_in) {
                     if (side) KQ_CUDA(cudaStreamWaitEvent(s_far, side->ev[0], 0));
-                    st = trail_tc_long(maps, d_out, d_in, sp0, static_cast<int>(spe - sp0), sp1, d_in, bn, info, s_far);
+                    st = trail_tc_long(maps, d_out, d_in, sp0, static_cast<int>(spe - sp0), sp1, d_in, info, s_far);
                     if (st != KQ_OK) return st;
                     if (side) {
                         KQ_CUDA(cudaEventRecord(side->ev2[0], s_far));

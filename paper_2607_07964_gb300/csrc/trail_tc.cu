@@ -767,8 +767,6 @@ kq_status TrailMaps::init(const float* E_hi, const float* E_lo, const float* Lt_
     if ((st = make_f32_map(&rl_narrow, Lt_lo, d_in, d_in, 128)) != KQ_OK) return st;
     if ((st = make_f32_map(&rh64, Lt_hi, d_in, d_in, 64)) != KQ_OK) return st;
     if ((st = make_f32_map(&rl64, Lt_lo, d_in, d_in, 64)) != KQ_OK) return st;
-    if ((st = make_f32_map(&rh256, Lt_hi, d_in, d_in, 256)) != KQ_OK) return st;
-    if ((st = make_f32_map(&rl256, Lt_lo, d_in, d_in, 256)) != KQ_OK) return st;
     return KQ_OK;
 }
 
@@ -860,16 +858,6 @@ int long_drain_slabs() {
     return n;
 }
 
-// Whether the K > 128 updates run on the two-CTA kernel: yes unless the environment
-// variable KQ_TRAIL_PAIR says 0 (a tuning switch).
-bool pair_enabled() {
-    static const bool on = [] {
-        const char* e = std::getenv("KQ_TRAIL_PAIR");
-        return !(e && std::atoi(e) == 0);
-    }();
-    return on;
-}
-
 // Persistent: as many clusters as can be resident at once walk the tiles. One cluster per
 // tile (so that finished clusters hand their SMs to the critical-path kernels of the
 // higher-priority stream) measured slower on the 70B down_proj layer: Cholesky 84.5 against
@@ -901,63 +889,31 @@ kq_status launch_pair(const CUtensorMap& ah, const CUtensorMap& al, const CUtens
     return KQ_OK;
 }
 
-template <int BN, int STAGES>
-kq_status launch_trail_red(const TrailMaps& m, const CUtensorMap& rh, const CUtensorMap& rl, int64_t d_out,
-                           int64_t i0, int kb, int64_t cb, int64_t ce, int* info, cudaStream_t stream) {
-    using Cfg = TrailCfg<BN, STAGES, true>;
-    static std::atomic<uint64_t> attr{0};
-    KQ_TRY(once_per_device(attr, [&]() -> kq_status {
-        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<BN, STAGES, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     Cfg::SMEM));
-        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<BN, STAGES, true>,
-                                     cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared));
-        return KQ_OK;
-    }));
-    const int n_row = static_cast<int>(cdiv(d_out, TBM));
-    const int n_col = static_cast<int>(cdiv(ce - cb, BN));
-    TileSet ts{};
-    ts.mode = 0;
-    ts.n_tiles = n_row * n_col;
-    ts.n_col_tiles = n_col;
-    ts.cb = static_cast<int>(cb);
-    ts.i0 = static_cast<int>(i0);
-    ts.pslab = 1 << 30;
-    ts.ce = static_cast<int>(ce);
-    const int nslab = static_cast<int>(cdiv(kb, TBK));
-    trail_tc_kernel<BN, STAGES, true><<<red_grid(ts.n_tiles), T_THREADS, Cfg::SMEM, stream>>>(
-        m.eh, m.el, rh, rl, m.eh, m.el, rh, rl, m.w, m.w, ts, nslab, long_drain_slabs(), info);
-    KQ_LAUNCH_CHECK("trail_tc_kernel");
-    return KQ_OK;
-}
 }  // namespace
 
 kq_status trail_tc_long(const TrailMaps& m, int64_t d_out, int64_t d_in, int64_t i0, int kb, int64_t cb, int64_t ce,
-                        int bn, int* info, cudaStream_t stream) {
+                        int* info, cudaStream_t stream) {
     if (kb < 1 || kb > 1024 || i0 + kb > d_in || (kb % TK != 0 && i0 + kb != d_in)) {
         set_error("trailing update: K = %d from column %lld is not whole blocks of the super-panel", kb, (long long)i0);
         return KQ_ERR_INVALID_ARG;
     }
-    if ((bn != 128 && bn != 256) || ((ce - cb) % bn != 0 && ce != d_in)) {
+    if ((ce - cb) % PBN != 0 && ce != d_in) {
         set_error("trailing update: column range [%lld, %lld) is not whole %d-column tiles", (long long)cb,
-                  (long long)ce, bn);
+                  (long long)ce, PBN);
         return KQ_ERR_INVALID_ARG;
     }
     if (ce <= cb) return KQ_OK;
-    if (bn == 256 && pair_enabled()) {
-        TileSet ts{};
-        ts.mode = 0;
-        ts.n_col_tiles = static_cast<int>(cdiv(ce - cb, PBN));
-        ts.n_tiles = static_cast<int>(cdiv(d_out, 2 * TBM)) * ts.n_col_tiles;
-        ts.cb = static_cast<int>(cb);
-        ts.i0 = static_cast<int>(i0);
-        ts.pslab = 1 << 30;
-        ts.ce = static_cast<int>(ce);
-        ts.rows = static_cast<int>(d_out);
-        return launch_pair(m.eh, m.el, m.rh_narrow, m.rl_narrow, m.rh_narrow, m.rl_narrow, m.w, m.w, ts,
-                           static_cast<int>(cdiv(kb, TBK)), long_drain_slabs(), info, stream);
-    }
-    if (bn == 256) return launch_trail_red<256, 2>(m, m.rh256, m.rl256, d_out, i0, kb, cb, ce, info, stream);
-    return launch_trail_red<128, 3>(m, m.rh_narrow, m.rl_narrow, d_out, i0, kb, cb, ce, info, stream);
+    TileSet ts{};
+    ts.mode = 0;
+    ts.n_col_tiles = static_cast<int>(cdiv(ce - cb, PBN));
+    ts.n_tiles = static_cast<int>(cdiv(d_out, 2 * TBM)) * ts.n_col_tiles;
+    ts.cb = static_cast<int>(cb);
+    ts.i0 = static_cast<int>(i0);
+    ts.pslab = 1 << 30;
+    ts.ce = static_cast<int>(ce);
+    ts.rows = static_cast<int>(d_out);
+    return launch_pair(m.eh, m.el, m.rh_narrow, m.rl_narrow, m.rh_narrow, m.rl_narrow, m.w, m.w, ts,
+                       static_cast<int>(cdiv(kb, TBK)), long_drain_slabs(), info, stream);
 }
 
 // ------------------------------------------------------------ Cholesky step updates
@@ -976,7 +932,7 @@ kq_status CholTcMaps::init(float* A, float* Z, int64_t npad, int width, int nset
 
 kq_status chol_update_tc(const CholTcMaps& m, int set, int nbk, int a_j0, int a_j1, int b_i0, int b_i1, int b_j1,
                          int kx, int nslab, int* info, cudaStream_t stream) {
-    if (nslab > TNSLAB && pair_enabled()) {
+    if (nslab > TNSLAB) {
         // a super-panel's update (K > 128): 256 x 256 tiles on CTA pairs
         TileSet ts{};
         ts.mode = 1;

@@ -90,7 +90,6 @@ struct TrailMaps {
     CUtensorMap eh, el;                  // E_hi, E_lo [d_out x d_in], 128-row boxes
     CUtensorMap rh_narrow, rl_narrow;    // Lt_hi, Lt_lo [d_in x d_in], 128-row boxes
     CUtensorMap rh64, rl64;              // the same with 64-row boxes (64-column tiles)
-    CUtensorMap rh256, rl256;            // the same with 256-row boxes (256-column tiles)
     CUtensorMap w;                       // W [d_out x d_in], 128-row boxes (read and written)
     CUtensorMap qh, ql, ph, pl;          // with P: (-Wpre)_hi, _lo [d_out x d_in], Pt_hi, Pt_lo [d_in x d_in]
     kq_status init(const float* E_hi, const float* E_lo, const float* Lt_hi, const float* Lt_lo, int64_t d_out,
@@ -113,7 +112,7 @@ struct CholTcMaps {
 // j in [a_j0, a_j1), i >= j, and Z_ij -= C_i. Z_.j for i in [b_i0, b_i1), j < b_j1, where the
 // dot runs over the nslab * 32 split columns starting at kx of split set `set`. One block's K
 // (nslab = 4): 128 x 128 tiles on single CTAs; more (a super-panel's update): 256 x 256 tiles
-// of 128 x 128 blocks on pairs of CTAs (unless KQ_TRAIL_PAIR=0).
+// of 128 x 128 blocks on pairs of CTAs.
 kq_status chol_update_tc(const CholTcMaps& m, int set, int nbk, int a_j0, int a_j1, int b_i0, int b_i1, int b_j1,
                          int kx, int nslab, int* info, cudaStream_t stream);
 
@@ -130,12 +129,10 @@ kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, in
 
 // The same update for K = kb <= 1024 (the blocks of one super-panel, GPTQ mode), applied to
 // W two blocks' K at a time in block order (the accumulator drained every 256 of K), through
-// TMA reduce-adds instead of a shared-memory copy of the W tile. bn = 256: 256 x 256 tiles
-// on pairs of CTAs (cta_group::2, three-stage ring per CTA; with KQ_TRAIL_PAIR=0 in the
-// environment, 128 x 256 tiles on single CTAs, two stages); bn = 128: 128 x 128 tiles, three
-// stages. [cb, ce) whole tiles or ending at d_in; kb whole blocks unless the super-panel
-// ends at d_in.
+// TMA reduce-adds instead of a shared-memory copy of the W tile, on 256 x 256 tiles spread
+// over pairs of CTAs (cta_group::2, a three-stage ring per CTA). [cb, ce) whole 256-column
+// tiles or ending at d_in; kb whole blocks unless the super-panel ends at d_in.
 kq_status trail_tc_long(const TrailMaps& m, int64_t d_out, int64_t d_in, int64_t i0, int kb, int64_t cb, int64_t ce,
-                        int bn, int* info, cudaStream_t stream);
+                        int* info, cudaStream_t stream);
 
 }  // namespace kq
