@@ -182,7 +182,7 @@ __global__ void __launch_bounds__(14 * (1 << LG) / 16, LG == 9 ? 2 : 1) rht_rows
     extern __shared__ __align__(16) float sm28[];
     float* v = sm28;                                         // [N]
     const int t = threadIdx.x, g = t / TG, tl = t - g * TG;
-    float* buf = sm28 + N + g * (P + P / 32);                // this group's exchange buffer
+    float* buf = sm28 + N + g * P;                           // this group's exchange buffer
     const int tw = deposit_bits<(P - 1) & ~ML>(tl);
     for (int64_t r = blockIdx.x; r < rows; r += gridDim.x) {
 #pragma unroll
@@ -203,8 +203,8 @@ __global__ void __launch_bounds__(14 * (1 << LG) / 16, LG == 9 ? 2 : 1) rht_rows
 #pragma unroll
             for (int k = 0; k < 16; ++k) x[k] *= f[k];
             fwht_kbits<0xFu>(x);
-            rr_transpose<LG, 1>(x, buf, tl);
-            rr_transpose<LG, 2>(x, buf, tl);
+            rr_transpose<LG, 1, true>(x, buf, tl);
+            rr_transpose<LG, 2, true>(x, buf, tl);
 #pragma unroll
             for (int k = 0; k < 16; ++k)
                 if (KQ_IN_RANGE(a * P + (tw | deposit_bits<ML>(k)), N)) v[a * P + (tw | deposit_bits<ML>(k))] = x[k];
@@ -649,7 +649,7 @@ template <int LG>
 kq_status launch_rows28_reg(float* M, int64_t rows, int pre, int post, const int8_t* sign, const float* s,
                             cudaStream_t stream) {
     constexpr int P = 1 << LG, T = 14 * P / 16;
-    constexpr size_t smem = (28 * static_cast<size_t>(P) + 14 * (P + P / 32)) * sizeof(float);
+    constexpr size_t smem = (28 * static_cast<size_t>(P) + 14 * static_cast<size_t>(P)) * sizeof(float);
     static std::atomic<uint64_t> attr{0};
     KQ_TRY(once_per_device(attr, [&]() -> kq_status {
         KQ_CUDA(cudaFuncSetAttribute(rht_rows28_reg_kernel<LG, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,

@@ -345,22 +345,48 @@ __device__ __forceinline__ void fwht_kbits(float (&x)[16]) {
 
 __device__ __forceinline__ int pad32(int j) { return j + (j >> 5); }
 
+// Exchange-buffer addresses without padding for LG = 9 and 10 (P = 512, 1024): element j
+// goes to j with the row bits r = j >> 5 XORed into its bank bits through a GF(2)-linear
+// map chosen so that, for each of the four access patterns of the two exchanges (a warp's 32
+// threads vary index bits {4..8}, {2, 3, 6, 7, 8} or {0..4} for LG = 10; {4..8}, {3, 5..8} or
+// {0..4} for LG = 9), the 32 addresses fall in 32 distinct banks. A permutation of [0, P)
+// within each 32-float row, so the buffer needs no padding.
+template <int LG>
+__device__ __forceinline__ int swz_bank(int j) {
+    static_assert(LG == 9 || LG == 10, "exchange swizzle for P = 512 and 1024");
+    const int r = j >> 5;
+    int m;
+    if constexpr (LG == 10)
+        m = ((r & 1) << 3) | ((r >> 1) & 1) | (((r >> 2) & 1) << 1) | (((r >> 3) & 1) * 0x14);
+    else
+        m = (r & 7) | (((r >> 3) & 1) * 0x18);
+    return j ^ m;
+}
+
 // Values of phase Q - 1 to shared memory, those of phase Q back, and phase Q's butterflies.
 // Every thread of the CTA calls it (two barriers); threads with act false hold no values.
-template <int LG, int Q>
+// SWZ: the buffer holds P floats addressed through swz_bank (LG = 9, 10), else P + P / 32
+// padded one float in 32.
+template <int LG, int Q, bool SWZ = false>
 __device__ __forceinline__ void rr_transpose(float (&x)[16], float* buf, int t, bool act = true) {
     constexpr uint32_t N1 = (1u << LG) - 1u;
     constexpr uint32_t MW = rr_mask(LG, Q - 1), MR = rr_mask(LG, Q);
     const int tw = deposit_bits<N1 & ~MW>(t), tr = deposit_bits<N1 & ~MR>(t);
+    auto at = [](int j) {
+        if constexpr (SWZ)
+            return swz_bank<LG>(j);
+        else
+            return pad32(j);
+    };
     __syncthreads();   // the previous reads of buf are done
     if (act) {
 #pragma unroll
-        for (int k = 0; k < 16; ++k) buf[pad32(tw | deposit_bits<MW>(k))] = x[k];
+        for (int k = 0; k < 16; ++k) buf[at(tw | deposit_bits<MW>(k))] = x[k];
     }
     __syncthreads();
     if (act) {
 #pragma unroll
-        for (int k = 0; k < 16; ++k) x[k] = buf[pad32(tr | deposit_bits<MR>(k))];
+        for (int k = 0; k < 16; ++k) x[k] = buf[at(tr | deposit_bits<MR>(k))];
         fwht_kbits<rr_new_kbits(LG, Q)>(x);
     }
 }
