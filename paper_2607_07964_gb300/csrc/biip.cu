@@ -258,116 +258,94 @@ __global__ void __launch_bounds__(256) transpose_sq_kernel(float* __restrict__ M
     }
 }
 
-// --------------------------------------------------------------- column transform
-// One radix stage along the row index of M [n x ncols]: for every group base = hi*R*S + lo
-// (lo < S) and CW-column strip, rows base + i*S (i < R) are transformed along i by H_R
-// (R a power of two, as radix-8 passes) or H_28 (R == 28). Shared memory [R][CW], CW a
-// power of two, filled with cp.async; the last pass writes straight to global memory.
-template <bool IS28>
-__global__ void __launch_bounds__(256, IS28 ? 2 : 4) rht_cols_kernel(float* __restrict__ M, int n, int64_t ncols, int R, int S,
-                                int lgCW, int pre_mode, int post_mode, const int8_t* __restrict__ sign,
-                                const float* __restrict__ s, float post_scale) {
-    extern __shared__ __align__(16) float v[];
-    const int CW = 1 << lgCW;
-    const int64_t nstrips = (ncols + CW - 1) >> lgCW;
+// ------------------------------------------------- column transform in registers
+// One radix stage along the row index of M [n x ncols] with the whole radix in registers:
+// a work item is a group of R rows (base + i S, i < R) and a strip of columns; the TPC =
+// max(1, R / 32) consecutive lanes of a column each hold V = R / TPC of its values (lane u:
+// rows u V .. u V + V - 1), transform them (butterflies for R = 2^k, the cross-lane stages
+// by shuffles; the 28-point mix for R = 28) and store them back. Consecutive columns sit in
+// consecutive lane groups, so every row load of a warp is 32 / TPC contiguous floats. The
+// group's pre- and post-factors are staged once in shared memory. No shared-memory round
+// trips between radix-2 stages (a tiled shared-memory version with radix-8 sub-stages moved
+// each element through shared memory several times per pass: 2.35 against ~4 TB/s).
+template <int V>
+__device__ __forceinline__ void fwht_regs(float (&x)[V]) {
+#pragma unroll
+    for (int h = 1; h < V; h <<= 1)
+#pragma unroll
+        for (int i = 0; i < V; i += 2 * h)
+#pragma unroll
+            for (int j = i; j < i + h; ++j) {
+                const float a = x[j], b = x[j + h];
+                x[j] = a + b;
+                x[j + h] = a - b;
+            }
+}
+
+template <int R>
+__global__ void __launch_bounds__(128) rht_cols_reg_kernel(float* __restrict__ M, int n, int64_t ncols, int S,
+                                                           int pre_mode, int post_mode,
+                                                           const int8_t* __restrict__ sign,
+                                                           const float* __restrict__ s, float post_scale) {
+    constexpr int TPC = R > 32 ? R / 32 : 1, V = R / TPC, CPB = 128 / TPC;   // columns per CTA
+    __shared__ float pf[R], qf[R];
+    const int u = threadIdx.x % TPC, cl = threadIdx.x / TPC;
     const int64_t ngroups = n / R;
-    int lgR = 0;
-    while ((1 << lgR) < R) ++lgR;
-    const bool vec = (ncols & 3) == 0 && (reinterpret_cast<uintptr_t>(M) & 15u) == 0;
+    const int64_t nstrips = (ncols + CPB - 1) / CPB;
     for (int64_t w = blockIdx.x; w < ngroups * nstrips; w += gridDim.x) {
-        const int64_t g = w / nstrips;
-        const int64_t c0 = (w - g * nstrips) << lgCW;
+        const int64_t g = w / nstrips, c0 = (w - g * nstrips) * CPB;
         const int64_t base = (g / S) * static_cast<int64_t>(R) * S + (g % S);
-        const int cw = static_cast<int>(min(static_cast<int64_t>(CW), ncols - c0));
-        if (vec) {
-            for (int e = threadIdx.x; e < (R * CW) >> 2; e += blockDim.x) {
-                const int i = (4 * e) >> lgCW, c = (4 * e) & (CW - 1);
-                const int64_t r = base + static_cast<int64_t>(i) * S;
-                const int valid = max(0, min(4, cw - c));
-                cp_async16(v + 4 * e, valid ? static_cast<const void*>(M + r * ncols + c0 + c) : static_cast<const void*>(M),
-                           4 * valid);
-            }
-            cp_async_commit();
-            cp_async_wait<0>();
-        } else {
-            for (int e = threadIdx.x; e < R * CW; e += blockDim.x) {
-                const int i = e >> lgCW, c = e & (CW - 1);
-                v[e] = c < cw ? M[(base + static_cast<int64_t>(i) * S) * ncols + c0 + c] : 0.0f;
-            }
+        __syncthreads();   // the previous item's factors are no longer read
+        for (int i = threadIdx.x; i < R; i += blockDim.x) {
+            const int64_t r = base + static_cast<int64_t>(i) * S;
+            pf[i] = factor(pre_mode, sign, s, r);
+            qf[i] = factor(post_mode, sign, s, r) * post_scale;
         }
         __syncthreads();
-        if (IS28) {
-            // the 28 rows' pre- and post-factors, once per work item
-            float* pf = v + 28 * CW;
-            if (threadIdx.x < 28) {
-                const int64_t r = base + static_cast<int64_t>(threadIdx.x) * S;
-                pf[threadIdx.x] = factor(pre_mode, sign, s, r);
-                pf[28 + threadIdx.x] = factor(post_mode, sign, s, r) * post_scale;
-            }
-            __syncthreads();
-            // mix in place (each thread owns its columns), then store the tile row by row
-            for (int c = threadIdx.x; c < CW; c += blockDim.x) {
-                float x[28];
+        const int64_t c = c0 + cl;
+        const bool act = c < ncols;   // whole lane groups agree (a column's lanes share c)
+        const int64_t step = static_cast<int64_t>(S) * ncols;
+        float* col = M + (base + static_cast<int64_t>(u) * V * S) * ncols + (act ? c : 0);
+        float x[V];
 #pragma unroll
-                for (int a = 0; a < 28; ++a) x[a] = v[a * CW + c] * pf[a];
-                mix28(x, [&](int a, float y) { v[a * CW + c] = y * pf[28 + a]; });
-            }
-            __syncthreads();
-            if (vec && cw == CW) {
-                for (int e = threadIdx.x; e < (28 * CW) >> 2; e += blockDim.x) {
-                    const int i = (4 * e) >> lgCW, c = (4 * e) & (CW - 1);
-                    if (KQ_IN_RANGE((base + static_cast<int64_t>(i) * S) * ncols + c0 + c + 3,
-                                    static_cast<int64_t>(n) * ncols))
-                        *reinterpret_cast<float4*>(M + (base + static_cast<int64_t>(i) * S) * ncols + c0 + c) =
-                            *reinterpret_cast<const float4*>(v + 4 * e);
-                }
-            } else {
-                for (int e = threadIdx.x; e < 28 * CW; e += blockDim.x) {
-                    const int i = e >> lgCW, c = e & (CW - 1);
-                    if (c < cw && KQ_IN_RANGE((base + static_cast<int64_t>(i) * S) * ncols + c0 + c,
-                                              static_cast<int64_t>(n) * ncols))
-                        M[(base + static_cast<int64_t>(i) * S) * ncols + c0 + c] = v[e];
-                }
-            }
+        for (int i = 0; i < V; ++i) x[i] = act ? col[i * step] * pf[u * V + i] : 0.0f;
+        if constexpr (R == 28) {
+            float y[28];
+            mix28_paley(x, [&](int a, float v) { y[a] = v; });
+#pragma unroll
+            for (int i = 0; i < 28; ++i) x[i] = y[i];
         } else {
-            for (int lgh = 0; lgh < lgR;) {
-                const int lgr = min(3, lgR - lgh);
-                const int h = 1 << lgh, rr = 1 << lgr;
-                const bool first = lgh == 0, last = lgh + lgr == lgR;
-                for (int gg = threadIdx.x; gg < ((R >> lgr) << lgCW); gg += blockDim.x) {
-                    const int c = gg & (CW - 1), gi = gg >> lgCW;
-                    const int bi = ((gi >> lgh) << (lgh + lgr)) | (gi & (h - 1));
-                    float x[8];
+            fwht_regs<V>(x);
 #pragma unroll
-                    for (int q = 0; q < 8; ++q)
-                        if (q < rr) {
-                            x[q] = v[((bi + q * h) << lgCW) + c];
-                            if (first) x[q] *= factor(pre_mode, sign, s, base + static_cast<int64_t>(bi + q * h) * S);
-                        }
-                    fwht_reg_r(x, rr);
+            for (int m = 1; m < TPC; m <<= 1) {   // the stages across the column's lanes
+                const bool hi = (u & m) != 0;
 #pragma unroll
-                    for (int q = 0; q < 8; ++q)
-                        if (q < rr) {
-                            if (last) {
-                                const int64_t r = base + static_cast<int64_t>(bi + q * h) * S;
-                                if (c < cw && KQ_IN_RANGE(r * ncols + c0 + c, static_cast<int64_t>(n) * ncols))
-                                    M[r * ncols + c0 + c] = x[q] * (factor(post_mode, sign, s, r) * post_scale);
-                            } else {
-                                v[((bi + q * h) << lgCW) + c] = x[q];
-                            }
-                        }
+                for (int i = 0; i < V; ++i) {
+                    const float o = __shfl_xor_sync(0xffffffffu, x[i], m);
+                    x[i] = hi ? o - x[i] : x[i] + o;
                 }
-                __syncthreads();
-                lgh += lgr;
-            }
-            if (lgR == 0) {   // R == 1: only the factors apply
-                for (int c = threadIdx.x; c < cw; c += blockDim.x)
-                    M[base * ncols + c0 + c] = v[c] * factor(pre_mode, sign, s, base) * (factor(post_mode, sign, s, base) * post_scale);
             }
         }
-        __syncthreads();
+        if (act) {
+#pragma unroll
+            for (int i = 0; i < V; ++i)
+                if (KQ_IN_RANGE((col - M) + i * step, static_cast<int64_t>(n) * ncols))
+                    col[i * step] = x[i] * qf[u * V + i];
+        }
     }
 }
+
+template <int R>
+kq_status launch_cols_reg(float* M, int64_t n, int64_t ncols, int S, int pm, int qm, const int8_t* sign,
+                          const float* s, float ps, cudaStream_t stream) {
+    const int64_t items = (n / R) * cdiv(ncols, 128 / (R > 32 ? R / 32 : 1));
+    const int64_t grid = std::min<int64_t>(items, static_cast<int64_t>(num_sms()) * 16);
+    rht_cols_reg_kernel<R><<<static_cast<unsigned>(grid), 128, 0, stream>>>(M, static_cast<int>(n), ncols, S, pm, qm,
+                                                                         sign, s, ps);
+    KQ_LAUNCH_CHECK("rht_cols_reg_kernel");
+    return KQ_OK;
+}
+
 
 // ------------------------------------------------------------------------ scales
 __device__ __forceinline__ float quarter_root_ratio(float h, double a) {
@@ -730,50 +708,41 @@ kq_status cols_transform(float* M, int64_t n, int64_t ncols, int pre, int post, 
                          const float* s, cudaStream_t stream) {
     HadamardPlan p;
     if (!plan_of(n, &p)) return KQ_ERR_UNSUPPORTED;
-    // Radix stages: (R, S) pairs applied in order; S = product of earlier radices.
-    // Radix at most 128 per stage, tiles of at most 64 KB ([64 x 256] or [128 x 128]), which
-    // leaves room for three CTAs per SM, so one CTA's loads overlap another's butterflies (a
-    // single 512- or 1024-row stage, one CTA per SM, ran below 0.7 TB/s). n = 8192 thus takes
-    // two passes (64 x 128) rather than three (16 x 16 x 32): the 70B down_proj layer's
-    // rotation stage 14.2 -> 12.8 ms.
+    // Radix stages: (R, S) pairs applied in order; S = product of earlier radices. Radix at
+    // most 128 (values of a column spread over up to four lanes), as even as possible: n =
+    // 8192 in two passes (64 x 128), each reading and writing M once.
     int R[4], S[4], ns = 0;
     const int kp = log2i(p.P);
     const int nst = (kp + 6) / 7;
     for (int st = 0, done = 0; st < nst; ++st) {
-        const int kb = (kp - done) / (nst - st);   // as even as possible
+        const int kb = (kp - done) / (nst - st);
         R[ns] = 1 << kb;
         S[ns] = 1 << done;
         ++ns;
         done += kb;
     }
     if (p.has28) { R[ns] = 28; S[ns] = p.P; ++ns; }
-    static std::atomic<uint64_t> attr{0};
-    KQ_TRY(once_per_device(attr, [&]() -> kq_status {
-        KQ_CUDA(cudaFuncSetAttribute(rht_cols_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     128 * 1024));
-        KQ_CUDA(cudaFuncSetAttribute(rht_cols_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     128 * 1024));
-        return KQ_OK;
-    }));
-    const float post_scale = static_cast<float>(1.0 / sqrt(static_cast<double>(n)));
     if (ns == 0) {   // n == 1: only the factors apply
         R[0] = 1; S[0] = 1; ns = 1;
     }
+    const float post_scale = static_cast<float>(1.0 / sqrt(static_cast<double>(n)));
     for (int st = 0; st < ns; ++st) {
-        int CW = (R[st] == 128 ? 16384 : 32768) / R[st];
-        CW = CW < 32 ? 32 : (CW > 256 ? 256 : CW);
-        const size_t smem = (static_cast<size_t>(R[st]) * CW + (R[st] == 28 ? 56 : 0)) * sizeof(float);
-        const int64_t items = (n / R[st]) * cdiv(ncols, CW);
-        const int64_t grid = std::min<int64_t>(items, static_cast<int64_t>(num_sms()) * 16);
         const int pm = st == 0 ? pre : F_NONE, qm = st == ns - 1 ? post : F_NONE;
         const float ps = st == ns - 1 ? post_scale : 1.0f;
-        if (R[st] == 28)
-            rht_cols_kernel<true><<<static_cast<unsigned>(grid), 256, smem, stream>>>(
-                M, static_cast<int>(n), ncols, R[st], S[st], log2i(CW), pm, qm, sign, s, ps);
-        else
-            rht_cols_kernel<false><<<static_cast<unsigned>(grid), 256, smem, stream>>>(
-                M, static_cast<int>(n), ncols, R[st], S[st], log2i(CW), pm, qm, sign, s, ps);
-        KQ_LAUNCH_CHECK("rht_cols_kernel");
+        kq_status rs = KQ_ERR_UNSUPPORTED;
+        switch (R[st]) {
+            case 1: rs = launch_cols_reg<1>(M, n, ncols, S[st], pm, qm, sign, s, ps, stream); break;
+            case 2: rs = launch_cols_reg<2>(M, n, ncols, S[st], pm, qm, sign, s, ps, stream); break;
+            case 4: rs = launch_cols_reg<4>(M, n, ncols, S[st], pm, qm, sign, s, ps, stream); break;
+            case 8: rs = launch_cols_reg<8>(M, n, ncols, S[st], pm, qm, sign, s, ps, stream); break;
+            case 16: rs = launch_cols_reg<16>(M, n, ncols, S[st], pm, qm, sign, s, ps, stream); break;
+            case 32: rs = launch_cols_reg<32>(M, n, ncols, S[st], pm, qm, sign, s, ps, stream); break;
+            case 64: rs = launch_cols_reg<64>(M, n, ncols, S[st], pm, qm, sign, s, ps, stream); break;
+            case 128: rs = launch_cols_reg<128>(M, n, ncols, S[st], pm, qm, sign, s, ps, stream); break;
+            case 28: rs = launch_cols_reg<28>(M, n, ncols, S[st], pm, qm, sign, s, ps, stream); break;
+            default: break;
+        }
+        if (rs != KQ_OK) return rs;
     }
     return KQ_OK;
 }
