@@ -34,6 +34,8 @@
 // super-panel's split does not overwrite the operands the previous remote update reads.
 #include <math.h>
 
+#include <cstdlib>
+
 #include "kq_common.cuh"
 #include "tile_gemm.cuh"
 #include "trail_tc.cuh"
@@ -523,9 +525,9 @@ __device__ __forceinline__ void strip_gemm(const float* __restrict__ A, const fl
         for (int j = 0; j < CN; ++j) acc[i][j] = Cs[(ty + 16 * i) * CLD + (BNL ? CN * tx + j : tx + 16 * j)];
 }
 
-__global__ void __launch_bounds__(G_THREADS, 2) chol_panel_kernel(Work w, int64_t npad, int k) {
+__global__ void __launch_bounds__(G_THREADS, 2) chol_panel_kernel(Work w, int64_t npad, int k, int b0) {
     extern __shared__ __align__(16) float sm[];
-    const int b = blockIdx.x, s = blockIdx.y;
+    const int b = static_cast<int>(blockIdx.x) + b0, s = blockIdx.y;
     const int64_t off = static_cast<int64_t>(k) * NB;
     const float* cinv = w.Z + off * npad + off;
     const int ty = threadIdx.x >> 4, tx = threadIdx.x & 15;
@@ -586,13 +588,14 @@ __device__ __forceinline__ void update_quad(const Work& w, int64_t npad, int k, 
     }
 }
 
-// The tiles that step k + 1 reads first: row block k + 1 (tiles (k + 1, j), j <= k + 1)
-// and block column k + 1 below it (tiles (i, k + 1), i > k + 1); nbk tiles x 4 quadrants.
-// part 0: all of them; part 1: only the diagonal tile (k + 1, k + 1), which is all the next
-// diagonal step needs (grid 1 x 4); part 2: all but that tile, for the next panel.
-__global__ void __launch_bounds__(G_THREADS, 2) chol_next_kernel(Work w, int64_t npad, int k, int part) {
+// The tiles that step k + 1 reads first: row block k + 1 (tiles (k + 1, j), b0 <= j <= k + 1)
+// and block column k + 1 below it (tiles (i, k + 1), k + 1 < i < b0 + gridDim.x); one tile
+// x 4 quadrants per block index from b0. part 0: all of them; part 1: only the diagonal
+// tile (k + 1, k + 1), which is all the next diagonal step needs (grid 1 x 4); part 2: all
+// but that tile, for the next panel.
+__global__ void __launch_bounds__(G_THREADS, 2) chol_next_kernel(Work w, int64_t npad, int k, int part, int b0) {
     extern __shared__ __align__(16) float sm[];
-    const int bid = part == 1 ? k + 1 : static_cast<int>(blockIdx.x);
+    const int bid = part == 1 ? k + 1 : static_cast<int>(blockIdx.x) + b0;
     if (part == 2 && bid == k + 1) return;
     if (bid < k + 2)
         update_quad(w, npad, k, k + 1, bid, blockIdx.y, sm);
@@ -600,53 +603,124 @@ __global__ void __launch_bounds__(G_THREADS, 2) chol_next_kernel(Work w, int64_t
         update_quad(w, npad, k, bid, k + 1, blockIdx.y, sm);
 }
 
-// Operands of step k's tensor-core updates, tf32 hi / lo, into columns [col, col + NB) of
-// the [npad x width] split buffers: Ch/Cl rows r >= (k + 1) NB hold C[r][k NB + c] (column
-// block k of A); Zh/Zl rows q < (k + 1) NB hold Z[k NB + c][q] (row block k of Z, transposed
-// through a 32 x 33 tile) and rows q in [(k + 1) NB, zero_to) are zero (Z_kj = 0 for j > k).
-// Block (32, 8); one 32 x 32 tile per CTA.
-__global__ void chol_split_kernel(const float* __restrict__ A, const float* __restrict__ Z, int64_t npad, int k,
-                                  int width, int col, int64_t zero_to, float* __restrict__ Ch, float* __restrict__ Cl,
-                                  float* __restrict__ Zh, float* __restrict__ Zl) {
-    __shared__ float t[32][33];
-    const int64_t ko = static_cast<int64_t>(k) * NB;
-    const int64_t crow0 = static_cast<int64_t>(k + 1) * NB;
-    const int64_t nct = (npad - crow0) / 32 * (NB / 32);
-    const int64_t nzt = (ko + NB) / 32 * (NB / 32);
-    int64_t b = blockIdx.x;
-    if (b < nct) {
-        const int64_t r0 = crow0 + (b / (NB / 32)) * 32, c0 = (b % (NB / 32)) * 32;
-        for (int r = threadIdx.y; r < 32; r += 8) {
-            const float x = A[(r0 + r) * npad + ko + c0 + threadIdx.x];
-            const float h = tf32_hi(x);
-            if (!KQ_IN_RANGE((r0 + r) * width + col + c0 + threadIdx.x, npad * width)) continue;
-            Ch[(r0 + r) * width + col + c0 + threadIdx.x] = h;
-            Cl[(r0 + r) * width + col + c0 + threadIdx.x] = x - h;
+// The rest of step k's update inside the blocks [k0, k1): the lower tiles (i, j) of A with
+// k + 2 <= j <= i < k1, then the tiles (i, j) of B with k + 2 <= i < k1, k0 <= j <= k;
+// one tile x 4 quadrants per block index.
+__global__ void __launch_bounds__(G_THREADS, 2) chol_rest_kernel(Work w, int64_t npad, int k, int k0, int k1) {
+    extern __shared__ __align__(16) float sm[];
+    const int m = k1 - k - 2;
+    int t = static_cast<int>(blockIdx.x), i, j;
+    if (t < m * (m + 1) / 2) {
+        j = k + 2;
+        while (t >= k1 - j) {
+            t -= k1 - j;
+            ++j;
         }
-        return;
+        i = j + t;
+    } else {
+        t -= m * (m + 1) / 2;
+        const int nzc = k - k0 + 1;
+        i = k + 2 + t / nzc;
+        j = k0 + t % nzc;
     }
-    b -= nct;
-    if (b < nzt) {
-        const int64_t kc0 = (b % (NB / 32)) * 32, q0 = (b / (NB / 32)) * 32;
-        for (int r = threadIdx.y; r < 32; r += 8) t[r][threadIdx.x] = Z[(ko + kc0 + r) * npad + q0 + threadIdx.x];
+    update_quad(w, npad, k, i, j, blockIdx.y, sm);
+}
+
+// hi / lo = tf32 split of sign * src over a [rows x cols] block of a row-major matrix
+// (leading dimension lds; rows and cols multiples of 64), written as [rows x cols] (trans = 0)
+// or transposed, [cols x rows] (trans = 1), with leading dimension ldd; zero_src: the block
+// of src is set to 0 after it is read. src_n / dst_n: elements addressable from src / hi.
+// Block (32, 8) walking 64 x 64 tiles (persistent grid): each thread has its 16 loads of a
+// tile in flight before the stores; the transposed tile goes through shared memory.
+constexpr int SPLIT_T = 64;
+__global__ void __launch_bounds__(256) split_block_kernel(float* __restrict__ src, int64_t lds, int64_t rows,
+                                                          int64_t cols, float* __restrict__ hi,
+                                                          float* __restrict__ lo, int64_t ldd, int trans, float sign,
+                                                          int zero_src, int64_t src_n, int64_t dst_n) {
+    __shared__ float t[SPLIT_T][SPLIT_T + 1];
+    const int64_t nct = cols / SPLIT_T, ntiles = (rows / SPLIT_T) * nct;
+    const int tx = threadIdx.x, ty = threadIdx.y;
+    for (int64_t b = blockIdx.x; b < ntiles; b += gridDim.x) {
+        const int64_t r0 = (b / nct) * SPLIT_T, c0 = (b % nct) * SPLIT_T;
+        float v[8][2];
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int64_t si = (r0 + ty + 8 * i) * lds + c0 + 32 * h + tx;
+                v[i][h] = KQ_IN_RANGE(si, src_n) ? src[si] : 0.0f;
+            }
+        if (zero_src) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int64_t si = (r0 + ty + 8 * i) * lds + c0 + 32 * h + tx;
+                    if (KQ_IN_RANGE(si, src_n)) src[si] = 0.0f;
+                }
+        }
+        if (!trans) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int64_t di = (r0 + ty + 8 * i) * ldd + c0 + 32 * h + tx;
+                    if (!KQ_IN_RANGE(di, dst_n)) continue;
+                    const float x = sign * v[i][h];
+                    const float hv = tf32_hi(x);
+                    hi[di] = hv;
+                    lo[di] = x - hv;
+                }
+            continue;
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+#pragma unroll
+            for (int h = 0; h < 2; ++h) t[ty + 8 * i][32 * h + tx] = v[i][h];
         __syncthreads();
-        for (int r = threadIdx.y; r < 32; r += 8) {
-            const float x = t[threadIdx.x][r];   // Z[ko + kc0 + threadIdx.x][q0 + r]
-            const float h = tf32_hi(x);
-            if (!KQ_IN_RANGE((q0 + r) * width + col + kc0 + threadIdx.x, npad * width)) continue;
-            Zh[(q0 + r) * width + col + kc0 + threadIdx.x] = h;
-            Zl[(q0 + r) * width + col + kc0 + threadIdx.x] = x - h;
-        }
-        return;
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int c = ty + 8 * i, r = 32 * h + tx;   // src[r0 + r][c0 + c]
+                const int64_t di = (c0 + c) * ldd + r0 + r;
+                if (!KQ_IN_RANGE(di, dst_n)) continue;
+                const float x = sign * t[r][c];
+                const float hv = tf32_hi(x);
+                hi[di] = hv;
+                lo[di] = x - hv;
+            }
+        __syncthreads();
     }
-    b -= nzt;
-    const int64_t q0 = ko + NB + (b / (NB / 32)) * 32, kc0 = (b % (NB / 32)) * 32;
-    if (q0 < zero_to)
-        for (int r = threadIdx.y; r < 32; r += 8) {
-            if (!KQ_IN_RANGE((q0 + r) * width + col + kc0 + threadIdx.x, npad * width)) continue;
-            Zh[(q0 + r) * width + col + kc0 + threadIdx.x] = 0.0f;
-            Zl[(q0 + r) * width + col + kc0 + threadIdx.x] = 0.0f;
-        }
+}
+
+kq_status split_block(float* src, int64_t lds, int64_t rows, int64_t cols, float* hi, float* lo, int64_t ldd,
+                      int trans, float sign, int zero_src, int64_t src_n, int64_t dst_n, cudaStream_t stream) {
+    if (rows <= 0 || cols <= 0) return KQ_OK;
+    if (rows % SPLIT_T || cols % SPLIT_T) {
+        set_error("kq_chol_inv: split block %lld x %lld is not whole %d x %d tiles", (long long)rows,
+                  (long long)cols, SPLIT_T, SPLIT_T);
+        return KQ_ERR_INVALID_ARG;
+    }
+    const int64_t tiles = (rows / SPLIT_T) * (cols / SPLIT_T);
+    const int64_t grid = std::min<int64_t>(tiles, static_cast<int64_t>(num_sms()) * 8);
+    split_block_kernel<<<static_cast<unsigned>(grid), dim3(32, 8), 0, stream>>>(src, lds, rows, cols, hi, lo, ldd,
+                                                                                trans, sign, zero_src, src_n, dst_n);
+    KQ_LAUNCH_CHECK("split_block_kernel");
+    return KQ_OK;
+}
+
+// SMs left to the next super-panel's steps while the update of the tiles beyond the
+// next super-panel runs beside them (its grid is that many SMs short of all resident
+// clusters): KQ_CHOL_FREE_SMS, an even number below the SM count, else FAR_FREE_SMS.
+constexpr int FAR_FREE_SMS = 16;
+int far_free_sms() {
+    static const int v = [] {
+        const char* e = std::getenv("KQ_CHOL_FREE_SMS");
+        const int x = e ? std::atoi(e) : FAR_FREE_SMS;
+        return (x >= 0 && x % 2 == 0 && x < num_sms()) ? x : FAR_FREE_SMS;
+    }();
+    return v;
 }
 
 // -------------------------------------------------------------------- finish
@@ -741,7 +815,7 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
     for (int q = 0; q < 4 * nsets; ++q, sp += npad * width) w.split[q] = sp;
     w.dsum = reinterpret_cast<double*>(sp);
     CholTcMaps maps;
-    if (nbk > 2) {
+    if (two_level) {
         kq_status st = maps.init(w.A, w.Z, npad, width, nsets, w.split);
         if (st != KQ_OK) return st;
     }
@@ -752,6 +826,8 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
         KQ_CUDA(cudaFuncSetAttribute(chol_panel_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(STRIP_SMEM)));
         KQ_CUDA(cudaFuncSetAttribute(chol_next_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     static_cast<int>(STRIP_SMEM)));
+        KQ_CUDA(cudaFuncSetAttribute(chol_rest_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(STRIP_SMEM)));
         return KQ_OK;
     }));
@@ -770,10 +846,13 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
     SideStream* side = nbk > 2 ? side_stream(stream) : nullptr;
     bool forked = false, remote_pending = false;
     bool next_pending = false;   // the next panel's tiles, updated on the side stream
+    const int free_sms = far_free_sms();
     for (int k0 = 0; k0 < nbk; k0 += (two_level ? SPB : nbk)) {
         const int k1 = two_level ? std::min(nbk, k0 + SPB) : nbk;   // this super-panel: blocks [k0, k1)
         const int set = two_level ? (k0 / SPB) & 1 : 0;
         const bool far_after = two_level && k1 < nbk;
+        // The steps of the super-panel inside its own blocks: A's lower tiles in rows and
+        // columns [k0, k1) and B's tiles in rows and columns [k0, k1).
         for (int k = k0; k < k1; ++k) {
             chol_diag_kernel<<<1, DIAG_THREADS, DIAG_SMEM, stream>>>(w, n, npad, k, info);
             KQ_LAUNCH_CHECK("chol_diag_kernel");
@@ -781,87 +860,100 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
                 KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[2], 0));
                 next_pending = false;
             }
-            if (nbk > 1) {
-                chol_panel_kernel<<<dim3(nbk - 1, 4), G_THREADS, STRIP_SMEM, stream>>>(w, npad, k);
+            if (k1 - 1 - k0 > 0) {
+                chol_panel_kernel<<<dim3(k1 - 1 - k0, 4), G_THREADS, STRIP_SMEM, stream>>>(w, npad, k, k0);
                 KQ_LAUNCH_CHECK("chol_panel_kernel");
             }
-            if (k + 1 >= nbk) break;
-            const bool has_rest = k + 2 < k1;                 // tiles of this super-panel beyond k + 1
-            const bool need_split = has_rest || far_after;   // the super-panel update reads every slice
-            const bool fork = side && need_split;
-            if (side && (need_split || k + 1 < k1)) KQ_CUDA(cudaEventRecord(side->ev[0], stream));   // panel k done
-            if (forked) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));  // update of step k - 1 done
-            if (k + 1 < k1) {
-                if (side) {
-                    // Step k's update of the next diagonal tile alone on this stream, so the
-                    // next diagonal step starts at once; the rest of the tiles the next panel
-                    // reads on the side stream beside it (ahead of this step's split and
-                    // in-panel update there, which touch other tiles).
-                    KQ_CUDA(cudaStreamWaitEvent(side->s, side->ev[0], 0));
-                    chol_next_kernel<<<dim3(nbk, 4), G_THREADS, STRIP_SMEM, side->s>>>(w, npad, k, 2);
-                    KQ_LAUNCH_CHECK("chol_next_kernel");
-                    KQ_CUDA(cudaEventRecord(side->ev2[2], side->s));
-                    next_pending = true;
-                    chol_next_kernel<<<dim3(1, 4), G_THREADS, STRIP_SMEM, stream>>>(w, npad, k, 1);
-                } else {
-                    chol_next_kernel<<<dim3(nbk, 4), G_THREADS, STRIP_SMEM, stream>>>(w, npad, k, 0);
-                }
+            if (k + 1 >= k1) break;
+            const bool has_rest = k + 2 < k1;   // tiles of this super-panel beyond k + 1
+            if (side) KQ_CUDA(cudaEventRecord(side->ev[0], stream));       // panel k done
+            if (forked) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));   // rest of step k - 1 done
+            if (side) {
+                // Step k's update of the next diagonal tile alone on this stream, so the next
+                // diagonal step starts at once; the other tiles the next panel reads, then the
+                // rest of the step's update (other tiles), on the side stream beside it.
+                KQ_CUDA(cudaStreamWaitEvent(side->s, side->ev[0], 0));
+                chol_next_kernel<<<dim3(k1 - k0, 4), G_THREADS, STRIP_SMEM, side->s>>>(w, npad, k, 2, k0);
                 KQ_LAUNCH_CHECK("chol_next_kernel");
+                KQ_CUDA(cudaEventRecord(side->ev2[2], side->s));
+                next_pending = true;
+                chol_next_kernel<<<dim3(1, 4), G_THREADS, STRIP_SMEM, stream>>>(w, npad, k, 1, k0);
+            } else {
+                chol_next_kernel<<<dim3(k1 - k0, 4), G_THREADS, STRIP_SMEM, stream>>>(w, npad, k, 0, k0);
             }
-            if (need_split) {
-                cudaStream_t rs = stream;
-                if (fork) {
-                    KQ_CUDA(cudaStreamWaitEvent(side->s, side->ev[0], 0));
-                    rs = side->s;
-                }
-                const int col = two_level ? (k - k0) * NB : 0;
-                const int64_t zero_to = far_after ? static_cast<int64_t>(k1) * NB : 0;
-                const int64_t tiles = (npad - static_cast<int64_t>(k + 1) * NB) / 32 * (NB / 32) +
-                                      static_cast<int64_t>(k + 1) * NB / 32 * (NB / 32) +
-                                      std::max<int64_t>(0, zero_to - static_cast<int64_t>(k + 1) * NB) / 32 * (NB / 32);
-                float* const* sp4 = w.split + 4 * set;
-                chol_split_kernel<<<static_cast<unsigned>(tiles), dim3(32, 8), 0, rs>>>(
-                    w.A, w.Z, npad, k, width, col, zero_to, sp4[0], sp4[1], sp4[2], sp4[3]);
-                KQ_LAUNCH_CHECK("chol_split_kernel");
-                if (has_rest) {
-                    // A: block columns [k + 2, k1), all rows below; Z: block rows [k + 2, k1), j <= k
-                    kq_status st = chol_update_tc(maps, set, nbk, k + 2, k1, k + 2, k1, k + 1, col, NB / 32, info, rs);
-                    if (st != KQ_OK) return st;
-                }
-                if (fork) {
+            KQ_LAUNCH_CHECK("chol_next_kernel");
+            if (has_rest) {
+                const int m = k1 - k - 2;
+                const unsigned tiles = static_cast<unsigned>(m * (m + 1) / 2 + m * (k - k0 + 1));
+                chol_rest_kernel<<<dim3(tiles, 4), G_THREADS, STRIP_SMEM, side ? side->s : stream>>>(w, npad, k, k0, k1);
+                KQ_LAUNCH_CHECK("chol_rest_kernel");
+                if (side) {
                     KQ_CUDA(cudaEventRecord(side->ev[1], side->s));
                     forked = true;
                 }
             }
         }
+        if (!two_level) continue;
+        if (forked) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));
+        if (next_pending) {
+            KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[2], 0));
+            next_pending = false;
+        }
+        // the previous super-panel's update of the tiles beyond its successor's diagonal block
+        if (remote_pending) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[1], 0));
+        // The super-panel's blocks of C below it and of Z left of it, from its diagonal block
+        // of Z (= C_SS^-1, lower triangular), as two products on the tensor cores:
+        //   C_DS = A'_DS C_SS^-T = A'_DS Z_SS^T,   Z_SP = C_SS^-1 B'_SP = Z_SS B'_SP,
+        // A' and B' as the earlier super-panels' updates left them (D: the rows below the
+        // super-panel, P: the columns left of it). Operands in split set `set`: -A'_DS in the
+        // C slices' rows of D, Z_SS in the Z slices' rows of S, -B'_SP transposed in the Z
+        // slices' rows of P; the output blocks are cleared as their operands are read.
+        const int64_t sw = static_cast<int64_t>(k1 - k0) * NB;
+        const int64_t s0 = static_cast<int64_t>(k0) * NB, s1 = static_cast<int64_t>(k1) * NB;
+        float* const* sp4 = w.split + 4 * set;
+        const int64_t nsplit = npad * width;
+        float* a_ds = w.A + s1 * npad + s0;
+        float* z_sp = w.Z + s0 * npad;
+        KQ_TRY(split_block(a_ds, npad, npad - s1, sw, sp4[0] + s1 * width, sp4[1] + s1 * width, width, 0, -1.0f, 1,
+                           npad * npad - (s1 * npad + s0), nsplit - s1 * width, stream));
+        KQ_TRY(split_block(z_sp + s0, npad, sw, sw, sp4[2] + s0 * width, sp4[3] + s0 * width, width, 0, 1.0f, 0,
+                           npad * npad - (s0 * npad + s0), nsplit - s0 * width, stream));
+        KQ_TRY(split_block(z_sp, npad, sw, s0, sp4[2], sp4[3], width, 1, -1.0f, 1, npad * npad - s0 * npad, nsplit,
+                           stream));
+        KQ_TRY(chol_gemm_tc(a_ds, npad, npad - s1, sw, sp4[0] + s1 * width, sp4[1] + s1 * width,
+                            sp4[2] + s0 * width, sp4[3] + s0 * width, width, static_cast<int>(sw), 1, info, stream));
+        KQ_TRY(chol_gemm_tc(z_sp, npad, sw, s0, sp4[2] + s0 * width, sp4[3] + s0 * width, sp4[2], sp4[3], width,
+                            static_cast<int>(sw), 2, info, stream));
         if (!far_after) continue;
-        // The super-panel's update of every tile beyond it, K = (k1 - k0) NB: the next
-        // super-panel's block columns and rows first, on the caller's stream, then the rest on
-        // the second library stream beside the next super-panel (which touches none of it).
+        // Operands of the update of every tile beyond the super-panel (K = its width): C_DS
+        // in the C slices' rows of D, Z_S. (columns left of the super-panel's end) transposed
+        // in the Z slices' rows.
+        KQ_TRY(split_block(a_ds, npad, npad - s1, sw, sp4[0] + s1 * width, sp4[1] + s1 * width, width, 0, 1.0f, 0,
+                           npad * npad - (s1 * npad + s0), nsplit - s1 * width, stream));
+        KQ_TRY(split_block(z_sp, npad, sw, s1, sp4[2], sp4[3], width, 1, 1.0f, 0, npad * npad - s0 * npad, nsplit,
+                           stream));
+        // The update of the tiles beyond: the next super-panel's diagonal block first, on the
+        // caller's stream (all the next super-panel's steps read), then every other tile --
+        // A's block columns from k1 below row block k2, A beyond, Z's rows from k1 left of
+        // column block k1 -- on the second library stream, beside the next super-panel's
+        // steps, on all SMs but free_sms (the products after those steps wait for it).
         const int k2 = std::min(nbk, k1 + SPB);
         const int nslab = (k1 - k0) * NB / 32;
+        if (side) KQ_CUDA(cudaEventRecord(side->ev2[0], stream));   // this super-panel's operands
+        KQ_TRY(chol_update_tc(maps, set, nbk, k1, k2, 0, 0, 0, 0, nslab, info, stream, 0, 0, k2));
+        cudaStream_t rs = stream;
         if (side) {
-            KQ_CUDA(cudaEventRecord(side->ev2[0], side->s));                 // this super-panel's splits
-            KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[0], 0));
-            if (remote_pending) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[1], 0));   // previous remote part
+            KQ_CUDA(cudaStreamWaitEvent(side->s2, side->ev2[0], 0));
+            rs = side->s2;
         }
-        kq_status st = chol_update_tc(maps, set, nbk, k1, k2, k1, k2, k1, 0, nslab, info, stream);
-        if (st != KQ_OK) return st;
-        if (k2 < nbk) {
-            cudaStream_t rs = stream;
-            if (side) {
-                KQ_CUDA(cudaStreamWaitEvent(side->s2, side->ev2[0], 0));
-                rs = side->s2;
-            }
-            st = chol_update_tc(maps, set, nbk, k2, nbk, k2, nbk, k1, 0, nslab, info, rs);
-            if (st != KQ_OK) return st;
-            if (side) {
-                KQ_CUDA(cudaEventRecord(side->ev2[1], side->s2));
-                remote_pending = true;
-            }
+        KQ_TRY(chol_update_tc(maps, set, nbk, k1, nbk, k1, nbk, k1, 0, nslab, info, rs, side ? free_sms : 0, k2, nbk));
+        if (side) {
+            KQ_CUDA(cudaEventRecord(side->ev2[1], side->s2));
+            remote_pending = true;
         }
     }
     if (forked) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev[1], 0));
+    if (next_pending) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[2], 0));
     if (remote_pending) KQ_CUDA(cudaStreamWaitEvent(stream, side->ev2[1], 0));
     if (n % 4 == 0 && (reinterpret_cast<uintptr_t>(Lt) & 15u) == 0) {
         finish4_kernel<<<dim3(static_cast<unsigned>(cdiv(n, 64)), static_cast<unsigned>(cdiv(n, 64))), 256, 0,

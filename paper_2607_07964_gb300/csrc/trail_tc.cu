@@ -73,6 +73,8 @@ struct TileSet {
     int n_tiles;
     int n_col_tiles, cb, i0, pslab, ce, rows;         // mode 0 (ce: end of the column range; rows of W)
     int nbk, a_j0, a_j1, n_a, b_i0, b_i1, b_j1, kx;   // mode 1
+    int a_r0, a_r1;   // pair kernel, mode 1: A-region rows [max(j, a_r0), a_r1) of column block j
+    int ktri;   // pair kernel, mode 0: 0, or a triangular operand bounds K per tile (see below)
 };
 
 // Tile t: top-left corner (row r0, column c0) and whether it takes the second B pair and
@@ -436,6 +438,15 @@ struct PairTile {
     bool wr0, wr1;
 };
 
+// K slabs of pair tile t: nslab, or in mode 0 with ktri set, only the slabs up to the end
+// of the tile's 256 columns (ktri = 1: B rows c vanish beyond column c of K) or of its 256
+// rows (ktri = 2: A rows r vanish beyond column r of K). The same for both CTAs of a pair.
+__device__ __forceinline__ int pair_tile_nslab(const TileSet& ts, int t, int nslab) {
+    if (ts.mode != 0 || ts.ktri == 0) return nslab;
+    const int key = ts.ktri == 1 ? ts.cb + (t % ts.n_col_tiles) * PBN : (t / ts.n_col_tiles) * 2 * TBM;
+    return min(nslab, (key + PBN) / TBK);
+}
+
 __device__ __forceinline__ PairTile pair_tile_at(const TileSet& ts, int t, int rank) {
     PairTile p;
     if (ts.mode == 0) {
@@ -451,17 +462,17 @@ __device__ __forceinline__ PairTile pair_tile_at(const TileSet& ts, int t, int r
     }
     if (t < ts.n_a) {
         int jp = ts.a_j0;
-        while (t >= (ts.nbk - jp + 1) / 2) {
-            t -= (ts.nbk - jp + 1) / 2;
+        while (t >= (ts.a_r1 - max(jp, ts.a_r0) + 1) / 2) {
+            t -= (ts.a_r1 - max(jp, ts.a_r0) + 1) / 2;
             jp += 2;
         }
-        const int i = jp + 2 * t + rank;
+        const int i = max(jp, ts.a_r0) + 2 * t + rank;
         p.ra = i * TBM;
         p.rb = (jp + rank) * TBM;
         p.co = jp * TBM;
         p.alt = false;
-        p.wr0 = i < ts.nbk;
-        p.wr1 = i < ts.nbk && jp + 1 < ts.a_j1 && jp + 1 <= i;
+        p.wr0 = i < ts.a_r1;
+        p.wr1 = i < ts.a_r1 && jp + 1 < ts.a_j1 && jp + 1 <= i;
         return p;
     }
     t -= ts.n_a;
@@ -551,7 +562,8 @@ trail_pair_kernel(const __grid_constant__ CUtensorMap mAh, const __grid_constant
                 const PairTile pt = pair_tile_at(ts, t, static_cast<int>(rank));
                 const CUtensorMap* bh = pt.alt ? &mB2h : &mBh;
                 const CUtensorMap* bl = pt.alt ? &mB2l : &mBl;
-                for (int s = 0; s < nslab; ++s, ++k) {
+                const int ns = pair_tile_nslab(ts, t, nslab);
+                for (int s = 0; s < ns; ++s, ++k) {
                     const int st = k % PSTAGES;
                     const uint32_t u = static_cast<uint32_t>(k / PSTAGES);
                     if (!mbar_wait(&empty[st], (u & 1u) ^ 1u, abort_flag)) {
@@ -580,7 +592,8 @@ trail_pair_kernel(const __grid_constant__ CUtensorMap mAh, const __grid_constant
                 int k = 0, cc = 0;
                 bool ok = true;
                 for (int t = pair; t < n_tiles && ok; t += npairs) {
-                    for (int s0 = 0; s0 < nslab && ok; s0 += drain, ++cc) {
+                    const int ns = pair_tile_nslab(ts, t, nslab);
+                    for (int s0 = 0; s0 < ns && ok; s0 += drain, ++cc) {
                         const int buf = cc & 1;
                         if (!mbar_wait_cl(&tempty[buf], ((static_cast<uint32_t>(cc) >> 1) & 1u) ^ 1u, abort_flag)) {
                             ok = false;
@@ -588,7 +601,7 @@ trail_pair_kernel(const __grid_constant__ CUtensorMap mAh, const __grid_constant
                         }
                         tc_fence_after();
                         const uint32_t dt = tmem + static_cast<uint32_t>(buf * PBN);
-                        const int s1 = min(nslab, s0 + drain);
+                        const int s1 = min(ns, s0 + drain);
                         for (int s = s0; s < s1; ++s, ++k) {
                             const int st = k % PSTAGES;
                             if (!mbar_wait(&full[st], static_cast<uint32_t>(k / PSTAGES) & 1u, abort_flag)) {
@@ -639,7 +652,8 @@ trail_pair_kernel(const __grid_constant__ CUtensorMap mAh, const __grid_constant
             const int xh = pt.co + h * HALF;
             const bool wrh = h ? pt.wr1 : pt.wr0;
             const bool whole = wrh && (ts.mode == 1 || xh + HALF <= ts.ce);
-            for (int s0 = 0; s0 < nslab; s0 += drain, ++cc) {
+            const int ns = pair_tile_nslab(ts, t, nslab);
+            for (int s0 = 0; s0 < ns; s0 += drain, ++cc) {
                 const int buf = cc & 1;
                 ok = mbar_wait(&tfull[buf], (static_cast<uint32_t>(cc) >> 1) & 1u, abort_flag);
                 ok = __all_sync(0xffffffffu, ok) && !*abort_flag;
@@ -731,6 +745,10 @@ EncodeTiledFn encode_tiled() {
 }  // namespace
 
 kq_status make_f32_map(CUtensorMap* m, const float* base, int64_t rows, int64_t cols, int box_rows) {
+    return make_f32_map_ld(m, base, rows, cols, cols, box_rows);
+}
+
+kq_status make_f32_map_ld(CUtensorMap* m, const float* base, int64_t rows, int64_t cols, int64_t ld, int box_rows) {
     EncodeTiledFn enc = encode_tiled();
     if (!enc) {
         set_error("trailing update: cuTensorMapEncodeTiled is unavailable");
@@ -738,7 +756,7 @@ kq_status make_f32_map(CUtensorMap* m, const float* base, int64_t rows, int64_t 
     }
     std::memset(m, 0, sizeof(*m));
     cuuint64_t gdim[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
-    cuuint64_t gstride[1] = {static_cast<cuuint64_t>(cols) * 4};
+    cuuint64_t gstride[1] = {static_cast<cuuint64_t>(ld) * 4};
     cuuint32_t box[2] = {static_cast<cuuint32_t>(TBK), static_cast<cuuint32_t>(box_rows)};
     cuuint32_t estride[2] = {1, 1};
     CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(base), gdim, gstride, box, estride,
@@ -864,7 +882,7 @@ int long_drain_slabs() {
 // 74.6 ms, sweep 37.9 against 34.2 ms.
 kq_status launch_pair(const CUtensorMap& ah, const CUtensorMap& al, const CUtensorMap& bh, const CUtensorMap& bl,
                       const CUtensorMap& b2h, const CUtensorMap& b2l, const CUtensorMap& w, const CUtensorMap& w2,
-                      const TileSet& ts, int nslab, int drain, int* info, cudaStream_t stream) {
+                      const TileSet& ts, int nslab, int drain, int* info, cudaStream_t stream, int free_sms = 0) {
     static std::atomic<uint64_t> attr{0};
     static std::atomic<int> clusters{0};
     KQ_TRY(once_per_device(attr, [&]() -> kq_status {
@@ -882,7 +900,7 @@ kq_status launch_pair(const CUtensorMap& ah, const CUtensorMap& al, const CUtens
         return KQ_OK;
     }));
     if (ts.n_tiles == 0) return KQ_OK;
-    const int nc = std::min(ts.n_tiles, clusters.load());
+    const int nc = std::min(ts.n_tiles, std::max(1, clusters.load() - free_sms / 2));
     trail_pair_kernel<<<static_cast<unsigned>(2 * nc), T_THREADS, P_SMEM, stream>>>(ah, al, bh, bl, b2h, b2l, w, w2,
                                                                                     ts, nslab, drain, info);
     KQ_LAUNCH_CHECK("trail_pair_kernel");
@@ -930,8 +948,38 @@ kq_status CholTcMaps::init(float* A, float* Z, int64_t npad, int width, int nset
     return KQ_OK;
 }
 
+kq_status chol_gemm_tc(float* out, int64_t ld_out, int64_t rows, int64_t cols, const float* a_hi, const float* a_lo,
+                       const float* b_hi, const float* b_lo, int64_t ld_ab, int k, int ktri, int* info,
+                       cudaStream_t stream) {
+    if (rows < 1 || cols < 1) return KQ_OK;
+    if (k < TBK || k % TBK != 0 || k > ld_ab || cols % PBN != 0 || ktri < 0 || ktri > 2) {
+        set_error("Cholesky GEMM: K = %d, %lld columns (whole %d-column tiles, K in 32-column slabs)", k,
+                  (long long)cols, PBN);
+        return KQ_ERR_INVALID_ARG;
+    }
+    CUtensorMap ah, al, bh, bl, w;
+    kq_status st;
+    if ((st = make_f32_map_ld(&ah, a_hi, rows, k, ld_ab, TBM)) != KQ_OK) return st;
+    if ((st = make_f32_map_ld(&al, a_lo, rows, k, ld_ab, TBM)) != KQ_OK) return st;
+    if ((st = make_f32_map_ld(&bh, b_hi, cols, k, ld_ab, TBM)) != KQ_OK) return st;
+    if ((st = make_f32_map_ld(&bl, b_lo, cols, k, ld_ab, TBM)) != KQ_OK) return st;
+    if ((st = make_f32_map_ld(&w, out, rows, cols, ld_out, TBM)) != KQ_OK) return st;
+    TileSet ts{};
+    ts.mode = 0;
+    ts.n_col_tiles = static_cast<int>(cols / PBN);
+    ts.n_tiles = static_cast<int>(cdiv(rows, 2 * TBM)) * ts.n_col_tiles;
+    ts.cb = 0;
+    ts.i0 = 0;
+    ts.pslab = 1 << 30;
+    ts.ce = static_cast<int>(cols);
+    ts.rows = static_cast<int>(rows);
+    ts.ktri = ktri;
+    return launch_pair(ah, al, bh, bl, bh, bl, w, w, ts, k / TBK, long_drain_slabs(), info, stream);
+}
+
 kq_status chol_update_tc(const CholTcMaps& m, int set, int nbk, int a_j0, int a_j1, int b_i0, int b_i1, int b_j1,
-                         int kx, int nslab, int* info, cudaStream_t stream) {
+                         int kx, int nslab, int* info, cudaStream_t stream, int free_sms, int a_r0, int a_r1) {
+    if (a_r1 < 0) a_r1 = nbk;
     if (nslab > TNSLAB) {
         // a super-panel's update (K > 128): 256 x 256 tiles on CTA pairs
         TileSet ts{};
@@ -939,7 +987,9 @@ kq_status chol_update_tc(const CholTcMaps& m, int set, int nbk, int a_j0, int a_
         ts.nbk = nbk;
         ts.a_j0 = a_j0;
         ts.a_j1 = a_j1;
-        for (int jp = a_j0; jp < a_j1; jp += 2) ts.n_a += (nbk - jp + 1) / 2;
+        ts.a_r0 = a_r0;
+        ts.a_r1 = a_r1;
+        for (int jp = a_j0; jp < a_j1; jp += 2) ts.n_a += std::max(0, (a_r1 - std::max(jp, a_r0) + 1) / 2);
         ts.b_i0 = b_i0;
         ts.b_i1 = b_i1;
         ts.b_j1 = b_j1;
@@ -947,7 +997,7 @@ kq_status chol_update_tc(const CholTcMaps& m, int set, int nbk, int a_j0, int a_
         ts.ce = 1 << 30;
         ts.n_tiles = ts.n_a + ((b_i1 > b_i0 && b_j1 > 0) ? ((b_i1 - b_i0 + 1) / 2) * ((b_j1 + 1) / 2) : 0);
         return launch_pair(m.ch[set], m.cl[set], m.ch[set], m.cl[set], m.zh[set], m.zl[set], m.a, m.z, ts, nslab,
-                           long_drain_slabs(), info, stream);
+                           long_drain_slabs(), info, stream, free_sms);
     }
     // 128 x 128 tiles, three-stage operand ring, the tiles of A and Z updated by TMA
     // reduce-adds (no shared-memory copy of the tile)

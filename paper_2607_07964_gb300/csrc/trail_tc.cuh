@@ -84,6 +84,8 @@ __device__ __forceinline__ void tc_mma_tf32(uint32_t d_tmem, uint64_t adesc, uin
 // 2-D fp32 tensor map over a row-major [rows x cols] matrix: box = box_rows x 32 columns,
 // 128-byte swizzle (a 32-float row is one swizzle atom), zero fill outside the matrix.
 kq_status make_f32_map(CUtensorMap* m, const float* base, int64_t rows, int64_t cols, int box_rows);
+// The same over a [rows x cols] block of a row-major matrix with leading dimension ld.
+kq_status make_f32_map_ld(CUtensorMap* m, const float* base, int64_t rows, int64_t cols, int64_t ld, int box_rows);
 
 // Tensor maps over the split error block and the split L, encoded once per sweep.
 struct TrailMaps {
@@ -114,7 +116,17 @@ struct CholTcMaps {
 // (nslab = 4): 128 x 128 tiles on single CTAs; more (a super-panel's update): 256 x 256 tiles
 // of 128 x 128 blocks on pairs of CTAs.
 kq_status chol_update_tc(const CholTcMaps& m, int set, int nbk, int a_j0, int a_j1, int b_i0, int b_i1, int b_j1,
-                         int kx, int nslab, int* info, cudaStream_t stream);
+                         int kx, int nslab, int* info, cudaStream_t stream, int free_sms = 0, int a_r0 = 0,
+                         int a_r1 = -1);
+
+// out[r][c] -= sum over x < k of a[r][x] b[c][x] for r < rows, c < cols (3xTF32 from the
+// tf32 hi / lo of a and b, row-major with leading dimension ld_ab; out with ld_out), on
+// 256 x 256 tiles over pairs of CTAs. cols a multiple of 256, k of 32. ktri = 1: b is lower
+// triangular (b[c][x] = 0 for x > c), so a tile of columns [c0, c0 + 256) runs K up to
+// c0 + 256; ktri = 2: a is (a[r][x] = 0 for x > r), K up to the tile's last row + 1.
+kq_status chol_gemm_tc(float* out, int64_t ld_out, int64_t rows, int64_t cols, const float* a_hi, const float* a_lo,
+                       const float* b_hi, const float* b_lo, int64_t ld_ab, int k, int ktri, int* info,
+                       cudaStream_t stream);
 
 // hi = src rounded to tf32, lo = src - hi (n elements).
 kq_status split_tf32(const float* src, int64_t n, float* hi, float* lo, cudaStream_t stream);
