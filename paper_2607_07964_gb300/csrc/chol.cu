@@ -908,45 +908,54 @@ extern "C" kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, floa
         // super-panel, P: the columns left of it). Operands in split set `set`: -A'_DS in the
         // C slices' rows of D, Z_SS in the Z slices' rows of S, -B'_SP transposed in the Z
         // slices' rows of P; the output blocks are cleared as their operands are read.
+        // C_DS and the next diagonal block's update are on the caller's stream (the next
+        // super-panel's steps wait for them); Z_SP, the Z operands of the update of the tiles
+        // beyond and that update on the second library stream, beside the next steps.
         const int64_t sw = static_cast<int64_t>(k1 - k0) * NB;
         const int64_t s0 = static_cast<int64_t>(k0) * NB, s1 = static_cast<int64_t>(k1) * NB;
         float* const* sp4 = w.split + 4 * set;
         const int64_t nsplit = npad * width;
         float* a_ds = w.A + s1 * npad + s0;
         float* z_sp = w.Z + s0 * npad;
-        KQ_TRY(split_block(a_ds, npad, npad - s1, sw, sp4[0] + s1 * width, sp4[1] + s1 * width, width, 0, -1.0f, 1,
-                           npad * npad - (s1 * npad + s0), nsplit - s1 * width, stream));
+        cudaStream_t rs = side ? side->s2 : stream;
         KQ_TRY(split_block(z_sp + s0, npad, sw, sw, sp4[2] + s0 * width, sp4[3] + s0 * width, width, 0, 1.0f, 0,
                            npad * npad - (s0 * npad + s0), nsplit - s0 * width, stream));
-        KQ_TRY(split_block(z_sp, npad, sw, s0, sp4[2], sp4[3], width, 1, -1.0f, 1, npad * npad - s0 * npad, nsplit,
-                           stream));
-        KQ_TRY(chol_gemm_tc(a_ds, npad, npad - s1, sw, sp4[0] + s1 * width, sp4[1] + s1 * width,
-                            sp4[2] + s0 * width, sp4[3] + s0 * width, width, static_cast<int>(sw), 1, info, stream));
-        KQ_TRY(chol_gemm_tc(z_sp, npad, sw, s0, sp4[2] + s0 * width, sp4[3] + s0 * width, sp4[2], sp4[3], width,
-                            static_cast<int>(sw), 2, info, stream));
-        if (!far_after) continue;
-        // Operands of the update of every tile beyond the super-panel (K = its width): C_DS
-        // in the C slices' rows of D, Z_S. (columns left of the super-panel's end) transposed
-        // in the Z slices' rows.
-        KQ_TRY(split_block(a_ds, npad, npad - s1, sw, sp4[0] + s1 * width, sp4[1] + s1 * width, width, 0, 1.0f, 0,
-                           npad * npad - (s1 * npad + s0), nsplit - s1 * width, stream));
-        KQ_TRY(split_block(z_sp, npad, sw, s1, sp4[2], sp4[3], width, 1, 1.0f, 0, npad * npad - s0 * npad, nsplit,
-                           stream));
-        // The update of the tiles beyond: the next super-panel's diagonal block first, on the
-        // caller's stream (all the next super-panel's steps read), then every other tile --
-        // A's block columns from k1 below row block k2, A beyond, Z's rows from k1 left of
-        // column block k1 -- on the second library stream, beside the next super-panel's
-        // steps, on all SMs but free_sms (the products after those steps wait for it).
-        const int k2 = std::min(nbk, k1 + SPB);
-        const int nslab = (k1 - k0) * NB / 32;
-        if (side) KQ_CUDA(cudaEventRecord(side->ev2[0], stream));   // this super-panel's operands
-        KQ_TRY(chol_update_tc(maps, set, nbk, k1, k2, 0, 0, 0, 0, nslab, info, stream, 0, 0, k2));
-        cudaStream_t rs = stream;
         if (side) {
+            KQ_CUDA(cudaEventRecord(side->ev2[0], stream));   // Z_SS split; the earlier updates done
             KQ_CUDA(cudaStreamWaitEvent(side->s2, side->ev2[0], 0));
-            rs = side->s2;
         }
-        KQ_TRY(chol_update_tc(maps, set, nbk, k1, nbk, k1, nbk, k1, 0, nslab, info, rs, side ? free_sms : 0, k2, nbk));
+        KQ_TRY(split_block(z_sp, npad, sw, s0, sp4[2], sp4[3], width, 1, -1.0f, 1, npad * npad - s0 * npad, nsplit,
+                           rs));
+        KQ_TRY(chol_gemm_tc(z_sp, npad, sw, s0, sp4[2] + s0 * width, sp4[3] + s0 * width, sp4[2], sp4[3], width,
+                            static_cast<int>(sw), 2, info, rs));
+        if (far_after) {
+            KQ_TRY(split_block(a_ds, npad, npad - s1, sw, sp4[0] + s1 * width, sp4[1] + s1 * width, width, 0, -1.0f,
+                               1, npad * npad - (s1 * npad + s0), nsplit - s1 * width, stream));
+            KQ_TRY(chol_gemm_tc(a_ds, npad, npad - s1, sw, sp4[0] + s1 * width, sp4[1] + s1 * width,
+                                sp4[2] + s0 * width, sp4[3] + s0 * width, width, static_cast<int>(sw), 1, info,
+                                stream));
+            // operands of the update of every tile beyond the super-panel (K = its width):
+            // C_DS in the C slices' rows of D ...
+            KQ_TRY(split_block(a_ds, npad, npad - s1, sw, sp4[0] + s1 * width, sp4[1] + s1 * width, width, 0, 1.0f,
+                               0, npad * npad - (s1 * npad + s0), nsplit - s1 * width, stream));
+            if (side) {
+                KQ_CUDA(cudaEventRecord(side->ev2[3], stream));   // C_DS split; Z_SS no longer read here
+                KQ_CUDA(cudaStreamWaitEvent(side->s2, side->ev2[3], 0));
+            }
+            // ... and Z_S. (the columns left of the super-panel's end) transposed in the Z
+            // slices' rows, over Z_SS's split once both products have read it
+            KQ_TRY(split_block(z_sp, npad, sw, s1, sp4[2], sp4[3], width, 1, 1.0f, 0, npad * npad - s0 * npad, nsplit,
+                               rs));
+            // The update of the tiles beyond: the next super-panel's diagonal block on the
+            // caller's stream (all the next super-panel's steps read it), every other tile --
+            // A's block columns from k1 below row block k2, A beyond, Z's rows from k1 left of
+            // column block k1 -- on the second library stream on all SMs but free_sms.
+            const int k2 = std::min(nbk, k1 + SPB);
+            const int nslab = (k1 - k0) * NB / 32;
+            KQ_TRY(chol_update_tc(maps, set, nbk, k1, k2, 0, 0, 0, 0, nslab, info, stream, 0, 0, k2));
+            KQ_TRY(chol_update_tc(maps, set, nbk, k1, nbk, k1, nbk, k1, 0, nslab, info, rs, side ? free_sms : 0, k2,
+                                  nbk));
+        }
         if (side) {
             KQ_CUDA(cudaEventRecord(side->ev2[1], side->s2));
             remote_pending = true;

@@ -76,7 +76,8 @@ SideStream* side_stream(cudaStream_t caller) {
         cudaEventCreateWithFlags(&e.side.ev[1], cudaEventDisableTiming) != cudaSuccess ||
         cudaEventCreateWithFlags(&e.side.ev2[0], cudaEventDisableTiming) != cudaSuccess ||
         cudaEventCreateWithFlags(&e.side.ev2[1], cudaEventDisableTiming) != cudaSuccess ||
-        cudaEventCreateWithFlags(&e.side.ev2[2], cudaEventDisableTiming) != cudaSuccess) {
+        cudaEventCreateWithFlags(&e.side.ev2[2], cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&e.side.ev2[3], cudaEventDisableTiming) != cudaSuccess) {
         cudaGetLastError();
         e.side.s = nullptr;
     }

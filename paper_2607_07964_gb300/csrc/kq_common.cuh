@@ -72,7 +72,7 @@ struct SideStream {
     cudaStream_t s;
     cudaEvent_t ev[2];
     cudaStream_t s2;        // a second side stream (same priority) for long-running work
-    cudaEvent_t ev2[3];
+    cudaEvent_t ev2[4];
     bool tried;
 };
 SideStream* side_stream(cudaStream_t caller);

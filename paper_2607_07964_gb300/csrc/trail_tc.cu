@@ -37,17 +37,14 @@ constexpr int TNSLAB = TK / TBK;         // 4
 constexpr int T_THREADS = 320;           // 10 warps: TMA, MMA, 8 epilogue
 constexpr int A_SLAB = TBM * TBK * 4;    // 16 KB
 
-// RED = false: the tile of W comes in by TMA, the epilogue subtracts the accumulator from
-// it in shared memory and a TMA store writes it back. RED = true: W never enters shared
-// memory; the epilogue stages -accumulator one 128 x 32 box at a time (one staging box per
-// column half) and a TMA reduce-add applies it to W in global memory, which leaves room for
-// a deeper operand ring or wider tiles.
-template <int BN, int STAGES, bool RED = false>
+// One-CTA tiles: the tile of W comes in by TMA, the epilogue subtracts the accumulator
+// from it in shared memory and a TMA store writes it back.
+template <int BN, int STAGES>
 struct TrailCfg {
     static constexpr int B_SLAB = BN * TBK * 4;                    // 16 KB for BN = 128
     static constexpr int STAGE = 2 * A_SLAB + 2 * B_SLAB;          // hi + lo of both
     static constexpr int WBOX = TBM * 32 * 4;                      // one 128 x 32 box of W (16 KB)
-    static constexpr int WTILE = RED ? 2 * WBOX : TBM * BN * 4;    // staging boxes, or the tile of W
+    static constexpr int WTILE = TBM * BN * 4;                     // the tile of W
     static constexpr int SMEM = STAGES * STAGE + WTILE + 1024 + 256;
     static_assert(2 * BN <= 512, "two accumulators must fit in TMEM");
     static_assert(BN % 64 == 0, "W moves in 32-column boxes, two column halves");
@@ -60,14 +57,14 @@ __device__ __forceinline__ bool wait_quiet(uint64_t* bar, uint32_t parity) {
 }
 
 // Which output tiles a launch updates, and from which operand maps.
-//   mode 0 (the sweep): a row x column grid over W[:, cb:], K slabs at columns i0 + 32 s of
-//     the first pair (E with R) and, for slabs >= pslab, at i0 + 32 (s - pslab) of the second
-//     pair (-Wpre with P).
-//   mode 1 (a Cholesky update, see chol.cu): first the A region -- lower tiles (i, j) with
-//     j in [a_j0, a_j1) and i >= j, output A, B operand from the split C rows j -- then the
-//     B region -- tiles (i, j) with i in [b_i0, b_i1), j < b_j1, output Z, B operand from the
-//     split transposed Z rows j. The A operand is the split C rows i; K slabs at columns
-//     kx + 32 s of the split buffers.
+//   mode 0 (the sweep; the Cholesky's products on CTA pairs): a row x column grid over
+//     W[:, cb:], K slabs at columns i0 + 32 s of the first pair (E with R) and, for slabs
+//     >= pslab (one-CTA kernel), at i0 + 32 (s - pslab) of the second pair (-Wpre with P).
+//   mode 1 (a Cholesky update on CTA pairs, see chol.cu): first the A region -- lower tiles
+//     (i, j) with j in [a_j0, a_j1) and max(j, a_r0) <= i < a_r1, output A, B operand from
+//     the split C rows j -- then the B region -- tiles (i, j) with i in [b_i0, b_i1),
+//     j < b_j1, output Z, B operand from the split transposed Z rows j. The A operand is the
+//     split C rows i; K slabs at columns kx + 32 s of the split buffers.
 struct TileSet {
     int mode;
     int n_tiles;
@@ -77,43 +74,22 @@ struct TileSet {
     int ktri;   // pair kernel, mode 0: 0, or a triangular operand bounds K per tile (see below)
 };
 
-// Tile t: top-left corner (row r0, column c0) and whether it takes the second B pair and
-// the second W map.
-__device__ __forceinline__ void tile_at(const TileSet& ts, int t, int bn, int* r0, int* c0, bool* alt) {
-    if (ts.mode == 0) {
-        *r0 = (t / ts.n_col_tiles) * TBM;
-        *c0 = ts.cb + (t % ts.n_col_tiles) * bn;
-        *alt = false;
-        return;
-    }
-    if (t < ts.n_a) {
-        int j = ts.a_j0;
-        while (t >= ts.nbk - j) {
-            t -= ts.nbk - j;
-            ++j;
-        }
-        *r0 = (j + t) * TBM;
-        *c0 = j * TBM;
-        *alt = false;
-        return;
-    }
-    t -= ts.n_a;
-    *r0 = (ts.b_i0 + t / ts.b_j1) * TBM;
-    *c0 = (t % ts.b_j1) * TBM;
-    *alt = true;
+// Tile t of the one-CTA kernel (mode 0): top-left corner (row r0, column c0).
+__device__ __forceinline__ void tile_at(const TileSet& ts, int t, int bn, int* r0, int* c0) {
+    *r0 = (t / ts.n_col_tiles) * TBM;
+    *c0 = ts.cb + (t % ts.n_col_tiles) * bn;
 }
 
-template <int BN, int TSTAGES, bool RED>
+template <int BN, int TSTAGES>
 __global__ void __launch_bounds__(T_THREADS, 1)
 trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__ CUtensorMap mEl,
                 const __grid_constant__ CUtensorMap mRh, const __grid_constant__ CUtensorMap mRl,
                 const __grid_constant__ CUtensorMap mQh, const __grid_constant__ CUtensorMap mQl,
                 const __grid_constant__ CUtensorMap mPh, const __grid_constant__ CUtensorMap mPl,
-                const __grid_constant__ CUtensorMap mW, const __grid_constant__ CUtensorMap mW2, TileSet ts,
-                int nslab, int drain, int* info) {
+                const __grid_constant__ CUtensorMap mW, TileSet ts, int nslab, int drain, int* info) {
     const int n_tiles = ts.n_tiles;
-    const int xk = ts.mode == 0 ? ts.i0 : ts.kx;
-    using C = TrailCfg<BN, TSTAGES, RED>;
+    const int xk = ts.i0;
+    using C = TrailCfg<BN, TSTAGES>;
     constexpr int WBOX = C::WBOX;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -159,8 +135,7 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
         tma_prefetch_desc(&mRh);
         tma_prefetch_desc(&mRl);
         tma_prefetch_desc(&mW);
-        if (ts.mode == 1) tma_prefetch_desc(&mW2);
-        if (nslab > TNSLAB || ts.mode == 1) {
+        if (nslab > TNSLAB) {
             tma_prefetch_desc(&mQh);
             tma_prefetch_desc(&mQl);
             tma_prefetch_desc(&mPh);
@@ -179,19 +154,13 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
             bool ok = true;
             for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++li) {
                 int r0, c0;
-                bool alt;
-                tile_at(ts, t, BN, &r0, &c0, &alt);
-                const CUtensorMap* wm = alt ? &mW2 : &mW;
-                if constexpr (!RED) {
-                    // the tile of W, once the previous tile has been stored from the buffer
-                    if (!mbar_wait(wfree, (static_cast<uint32_t>(li) & 1u) ^ 1u, abort_flag)) break;
-                    mbar_arrive_expect_tx(wfull, C::WTILE);
+                tile_at(ts, t, BN, &r0, &c0);
+                // the tile of W, once the previous tile has been stored from the buffer
+                if (!mbar_wait(wfree, (static_cast<uint32_t>(li) & 1u) ^ 1u, abort_flag)) break;
+                mbar_arrive_expect_tx(wfull, C::WTILE);
 #pragma unroll
-                    for (int j = 0; j < BN / 32; ++j) tma_load_2d(wtile + j * WBOX, wm, wfull, c0 + 32 * j, r0);
-                    w_issued = li + 1;
-                } else {
-                    (void)wm;
-                }
+                for (int j = 0; j < BN / 32; ++j) tma_load_2d(wtile + j * WBOX, &mW, wfull, c0 + 32 * j, r0);
+                w_issued = li + 1;
                 for (int s = 0; s < nslab; ++s, ++k) {
                     const int st = k % TSTAGES;
                     const uint32_t u = static_cast<uint32_t>(k / TSTAGES);
@@ -201,15 +170,13 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
                     }
                     mbar_arrive_expect_tx(&full[st], C::STAGE);
                     uint8_t* base = smem + st * C::STAGE;
-                    // slabs 0..3: E and R; slabs 4..7 (with P): -Wpre and P. Cholesky tiles
-                    // with j <= k take B from the second pair.
-                    const bool second = ts.mode == 0 && s >= ts.pslab;
-                    const bool bsec = second || alt;
+                    // slabs 0..3: E and R; slabs 4..7 (with P): -Wpre and P
+                    const bool second = s >= ts.pslab;
                     const int x = xk + (second ? s - ts.pslab : s) * TBK;
                     tma_load_2d(base, second ? &mQh : &mEh, &full[st], x, r0);
                     tma_load_2d(base + A_SLAB, second ? &mQl : &mEl, &full[st], x, r0);
-                    tma_load_2d(base + 2 * A_SLAB, bsec ? &mPh : &mRh, &full[st], x, c0);
-                    tma_load_2d(base + 2 * A_SLAB + C::B_SLAB, bsec ? &mPl : &mRl, &full[st], x, c0);
+                    tma_load_2d(base + 2 * A_SLAB, second ? &mPh : &mRh, &full[st], x, c0);
+                    tma_load_2d(base + 2 * A_SLAB + C::B_SLAB, second ? &mPl : &mRl, &full[st], x, c0);
                 }
             }
             // every issued load must land before the CTA exits
@@ -269,67 +236,12 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
         // memory as 128-byte swizzled rows (16-byte chunk c of row r at c ^ (r & 7)), so the
         // float4 accesses of 8 consecutive rows hit distinct banks.
         constexpr int HALF = BN / 2;
-        constexpr int PIECES = HALF / 32;       // 32-column boxes per half
         const int q = warp & 3;                 // TMEM lane quadrant this warp may access
         const int h = (warp - 2) >> 2;          // which half of the columns
         const int r = q * 32 + lane;            // row within the tile
-        const bool issuer = RED && (warp == 2 + 4 * h) && lane == 0;
         int li = 0, cc = 0;
         bool ok = true;
         for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++li) {
-            if constexpr (RED) {
-                int r0, c0;
-                bool alt;
-                tile_at(ts, t, BN, &r0, &c0, &alt);
-                const CUtensorMap* wm = alt ? &mW2 : &mW;
-                uint8_t* stg = wtile + h * WBOX;
-                for (int s0 = 0; s0 < nslab; s0 += drain, ++cc) {
-                    const int buf = cc & 1;
-                    ok = mbar_wait(&tfull[buf], (static_cast<uint32_t>(cc) >> 1) & 1u, abort_flag);
-                    ok = __all_sync(0xffffffffu, ok) && !*abort_flag;
-                    // every warp of this half leaves together (the named barriers below)
-                    ok = named_bar_all(1 + h, 128, ok);
-                    if (!ok) break;
-                    tc_fence_after();
-                    const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) +
-                                           static_cast<uint32_t>(buf * BN + h * HALF);
-#pragma unroll 1
-                    for (int p = 0; p < PIECES; ++p) {
-                        const int x = c0 + h * HALF + 32 * p;
-                        float v[32];
-                        tmem_ld32(taddr + static_cast<uint32_t>(p * 32), v);
-                        tc_wait_ld();
-                        if (p == PIECES - 1) {   // the accumulator may be reused
-                            tc_fence_before();
-                            __syncwarp();
-                            if (lane == 0) mbar_arrive(&tempty[buf]);
-                        }
-                        if (x >= ts.ce) continue;   // a box wholly past the range (same for the half)
-                        // -acc as one 128 x 32 box, 128-byte swizzled like the tensor map
-                        float4* rowp = reinterpret_cast<float4*>(stg + r * 128);
-#pragma unroll
-                        for (int c = 0; c < 8; ++c)
-                            rowp[c ^ (r & 7)] = make_float4(-v[4 * c], -v[4 * c + 1], -v[4 * c + 2], -v[4 * c + 3]);
-                        fence_proxy_async();
-                        named_bar_sync(1 + h, 128);
-                        if (issuer) {
-                            // the same box of the previous chunk must have landed first, so
-                            // that every element takes its block updates in order (a half
-                            // cut short by the range end commits fewer boxes a chunk: wait
-                            // for all of them)
-                            if (c0 + h * HALF + HALF <= ts.ce)
-                                bulk_wait_le<PIECES - 1>();
-                            else
-                                bulk_wait_le<0>();
-                            tma_reduce_add_2d(wm, stg, x, r0);
-                            bulk_commit();
-                            bulk_wait_read0();
-                        }
-                        named_bar_sync(1 + h, 128);   // the staging box is free again
-                    }
-                }
-                continue;
-            }
             ok = mbar_wait(wfull, static_cast<uint32_t>(li) & 1u, abort_flag);
             ok = __all_sync(0xffffffffu, ok) && !*abort_flag;
             if (!ok) break;
@@ -367,18 +279,16 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
                 // store the tile once every warp has updated it, then free the buffer
                 if (mbar_wait(wdone, static_cast<uint32_t>(li) & 1u, abort_flag)) {
                     int r0, c0;
-                    bool alt;
-                    tile_at(ts, t, BN, &r0, &c0, &alt);
-                    const CUtensorMap* wm = alt ? &mW2 : &mW;
+                    tile_at(ts, t, BN, &r0, &c0);
 #pragma unroll
-                    for (int j = 0; j < BN / 32; ++j) tma_store_2d(wm, wtile + j * WBOX, c0 + 32 * j, r0);
+                    for (int j = 0; j < BN / 32; ++j) tma_store_2d(&mW, wtile + j * WBOX, c0 + 32 * j, r0);
                     bulk_commit();
                     bulk_wait_read0();
                     mbar_arrive(wfree);
                 }
             }
         }
-        if ((warp == 2 || (RED && warp == 6)) && lane == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+        if (warp == 2 && lane == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
     }
 
     tc_fence_before();
@@ -397,9 +307,10 @@ trail_tc_kernel(const __grid_constant__ CUtensorMap mEh, const __grid_constant__
 // reads both CTAs' operand slabs and writes each CTA's 128 rows of the accumulator into
 // that CTA's tensor memory. Each SM then stages and reads 128 x k of B per k slab instead
 // of 256 x k: per 32-k slab and SM 64 KB of TMA writes and 96 KB of operand reads for
-// 1536 MMA cycles, against 96 + 144 KB for the same cycles in the one-CTA 128 x 256 tile,
-// whose loop is bound by the 128 bytes per cycle of shared memory. Only the reduce-add
-// epilogue (W never enters shared memory).
+// 1536 MMA cycles, against 96 + 144 KB for the same cycles in a one-CTA 128 x 256 tile,
+// whose loop is bound by the 128 bytes per cycle of shared memory. W never enters shared
+// memory: the epilogue stages -accumulator one 128 x 32 box at a time (one staging box per
+// column half) and a TMA reduce-add applies it to W in global memory.
 //
 // Synchronization: every CTA loads its own slabs with TMA, the transaction bytes of both
 // landing on CTA 0's `full` barrier (the cta_group::2 form of the copy may signal the peer's
@@ -635,8 +546,10 @@ trail_pair_kernel(const __grid_constant__ CUtensorMap mAh, const __grid_constant
         }
     } else {
         // ------------------------------------------------------------ epilogue (8 warps, both CTAs)
-        // As in the one-CTA reduce-add epilogue: thread = one row of this CTA's 128 rows;
-        // warps 2-5 take columns [0, 128) of the tile, warps 6-9 columns [128, 256).
+        // Thread = one row of this CTA's 128 rows (TMEM lane); warps 2-5 take columns
+        // [0, 128) of the tile, warps 6-9 columns [128, 256). Each drained chunk goes to W
+        // box by box, the same box of the previous chunk landing first (block order per
+        // element).
         constexpr int HALF = PBN / 2;
         constexpr int PIECES = HALF / 32;
         const int q = warp & 3;
@@ -806,11 +719,11 @@ namespace {
 template <int BN>
 kq_status launch_trail(const TrailMaps& m, const CUtensorMap& rh, const CUtensorMap& rl, int64_t d_out, int64_t i0,
                        int64_t cb, int64_t ce, bool with_p, int kslabs, int* info, cudaStream_t stream) {
-    using Cfg = TrailCfg<BN, 2, false>;
+    using Cfg = TrailCfg<BN, 2>;
     static std::atomic<uint64_t> attr{0};
     KQ_TRY(once_per_device(attr, [&]() -> kq_status {
-        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<BN, 2, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
-        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<BN, 2, false>, cudaFuncAttributePreferredSharedMemoryCarveout,
+        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<BN, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
+        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<BN, 2>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                      cudaSharedmemCarveoutMaxShared));
         return KQ_OK;
     }));
@@ -826,9 +739,9 @@ kq_status launch_trail(const TrailMaps& m, const CUtensorMap& rh, const CUtensor
     ts.ce = static_cast<int>(ce);
     // the accumulator goes into W every 128 of K (one block's update at a time, as the
     // per-block schedule does); with P after the E and P halves of one block together
-    trail_tc_kernel<BN, 2, false><<<static_cast<unsigned>(std::min(ts.n_tiles, num_sms())), T_THREADS, Cfg::SMEM, stream>>>(
-        m.eh, m.el, rh, rl, with_p ? m.qh : m.eh, with_p ? m.ql : m.el, with_p ? m.ph : rh, with_p ? m.pl : rl, m.w, m.w,
-        ts, with_p ? 2 * kslabs : kslabs, with_p ? 2 * kslabs : TNSLAB, info);
+    trail_tc_kernel<BN, 2><<<static_cast<unsigned>(std::min(ts.n_tiles, num_sms())), T_THREADS, Cfg::SMEM, stream>>>(
+        m.eh, m.el, rh, rl, with_p ? m.qh : m.eh, with_p ? m.ql : m.el, with_p ? m.ph : rh, with_p ? m.pl : rl, m.w, ts,
+        with_p ? 2 * kslabs : kslabs, with_p ? 2 * kslabs : TNSLAB, info);
     KQ_LAUNCH_CHECK("trail_tc_kernel");
     return KQ_OK;
 }
@@ -856,12 +769,6 @@ kq_status trail_tc(const TrailMaps& m, float* W, int64_t d_out, int64_t d_in, in
 }
 
 namespace {
-// CTAs of a reduce-add launch: persistent, one per SM walking the tiles (one CTA per tile,
-// which would let the critical-path kernels beside it take SMs as tiles finish, measured
-// slower on the 70B down_proj layer: 331 against 320 ms, the per-CTA set-up costing more than
-// the overlap it buys).
-unsigned red_grid(int n_tiles) { return static_cast<unsigned>(std::min(n_tiles, num_sms())); }
-
 // Slabs of 32 K between two drains of the accumulator into W in the long updates (K up to
 // 1024): 8, i.e. two blocks' updates summed in TMEM before each reduce-add into W (half the
 // epilogue traffic of one drain per block: the 70B down_proj layer 297 against 309 ms; the
@@ -979,55 +886,24 @@ kq_status chol_gemm_tc(float* out, int64_t ld_out, int64_t rows, int64_t cols, c
 
 kq_status chol_update_tc(const CholTcMaps& m, int set, int nbk, int a_j0, int a_j1, int b_i0, int b_i1, int b_j1,
                          int kx, int nslab, int* info, cudaStream_t stream, int free_sms, int a_r0, int a_r1) {
+    // 256 x 256 tiles on CTA pairs
     if (a_r1 < 0) a_r1 = nbk;
-    if (nslab > TNSLAB) {
-        // a super-panel's update (K > 128): 256 x 256 tiles on CTA pairs
-        TileSet ts{};
-        ts.mode = 1;
-        ts.nbk = nbk;
-        ts.a_j0 = a_j0;
-        ts.a_j1 = a_j1;
-        ts.a_r0 = a_r0;
-        ts.a_r1 = a_r1;
-        for (int jp = a_j0; jp < a_j1; jp += 2) ts.n_a += std::max(0, (a_r1 - std::max(jp, a_r0) + 1) / 2);
-        ts.b_i0 = b_i0;
-        ts.b_i1 = b_i1;
-        ts.b_j1 = b_j1;
-        ts.kx = kx;
-        ts.ce = 1 << 30;
-        ts.n_tiles = ts.n_a + ((b_i1 > b_i0 && b_j1 > 0) ? ((b_i1 - b_i0 + 1) / 2) * ((b_j1 + 1) / 2) : 0);
-        return launch_pair(m.ch[set], m.cl[set], m.ch[set], m.cl[set], m.zh[set], m.zl[set], m.a, m.z, ts, nslab,
-                           long_drain_slabs(), info, stream, free_sms);
-    }
-    // 128 x 128 tiles, three-stage operand ring, the tiles of A and Z updated by TMA
-    // reduce-adds (no shared-memory copy of the tile)
-    using Cfg = TrailCfg<128, 3, true>;
-    static std::atomic<uint64_t> attr{0};
-    KQ_TRY(once_per_device(attr, [&]() -> kq_status {
-        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<128, 3, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     Cfg::SMEM));
-        KQ_CUDA(cudaFuncSetAttribute(trail_tc_kernel<128, 3, true>, cudaFuncAttributePreferredSharedMemoryCarveout,
-                                     cudaSharedmemCarveoutMaxShared));
-        return KQ_OK;
-    }));
     TileSet ts{};
     ts.mode = 1;
     ts.nbk = nbk;
     ts.a_j0 = a_j0;
     ts.a_j1 = a_j1;
-    for (int j = a_j0; j < a_j1; ++j) ts.n_a += nbk - j;
+    ts.a_r0 = a_r0;
+    ts.a_r1 = a_r1;
+    for (int jp = a_j0; jp < a_j1; jp += 2) ts.n_a += std::max(0, (a_r1 - std::max(jp, a_r0) + 1) / 2);
     ts.b_i0 = b_i0;
     ts.b_i1 = b_i1;
     ts.b_j1 = b_j1;
     ts.kx = kx;
-    ts.ce = 1 << 30;   // every tile lies inside the padded matrices
-    ts.n_tiles = ts.n_a + ((b_i1 > b_i0 && b_j1 > 0) ? (b_i1 - b_i0) * b_j1 : 0);
-    if (ts.n_tiles == 0) return KQ_OK;
-    trail_tc_kernel<128, 3, true><<<red_grid(ts.n_tiles), T_THREADS, Cfg::SMEM, stream>>>(
-        m.ch[set], m.cl[set], m.ch[set], m.cl[set], m.ch[set], m.cl[set], m.zh[set], m.zl[set], m.a, m.z, ts, nslab,
-        nslab > TNSLAB ? long_drain_slabs() : TNSLAB, info);
-    KQ_LAUNCH_CHECK("trail_tc_kernel");
-    return KQ_OK;
+    ts.ce = 1 << 30;
+    ts.n_tiles = ts.n_a + ((b_i1 > b_i0 && b_j1 > 0) ? ((b_i1 - b_i0 + 1) / 2) * ((b_j1 + 1) / 2) : 0);
+    return launch_pair(m.ch[set], m.cl[set], m.ch[set], m.cl[set], m.zh[set], m.zl[set], m.a, m.z, ts, nslab,
+                       long_drain_slabs(), info, stream, free_sms);
 }
 
 

@@ -111,10 +111,10 @@ struct CholTcMaps {
 };
 
 // A Cholesky update on the tensor cores (3xTF32): A_ij -= C_i. C_j.^T for the lower tiles with
-// j in [a_j0, a_j1), i >= j, and Z_ij -= C_i. Z_.j for i in [b_i0, b_i1), j < b_j1, where the
-// dot runs over the nslab * 32 split columns starting at kx of split set `set`. One block's K
-// (nslab = 4): 128 x 128 tiles on single CTAs; more (a super-panel's update): 256 x 256 tiles
-// of 128 x 128 blocks on pairs of CTAs.
+// j in [a_j0, a_j1) and max(j, a_r0) <= i < a_r1 (a_r1 < 0: nbk), and Z_ij -= C_i. Z_.j for
+// i in [b_i0, b_i1), j < b_j1, where the dot runs over the nslab * 32 split columns starting
+// at kx of split set `set`: 256 x 256 tiles of 128 x 128 blocks on pairs of CTAs, on all
+// resident clusters but free_sms / 2.
 kq_status chol_update_tc(const CholTcMaps& m, int set, int nbk, int a_j0, int a_j1, int b_i0, int b_i1, int b_j1,
                          int kx, int nslab, int* info, cudaStream_t stream, int free_sms = 0, int a_r0 = 0,
                          int a_r1 = -1);
