@@ -349,6 +349,15 @@ struct PairTile {
     bool wr0, wr1;
 };
 
+// Tile of cluster `pair` in round rd of the persistent walk: the rounds alternate direction
+// (boustrophedon), so a cluster that took one of the first tiles of a round takes one of the
+// last of the next. Tiles whose cost grows along the order (the K bound of ktri) then even
+// out per cluster, which the plain stride (with the cluster count a multiple of the column
+// tiles, every tile of a cluster in one column) does not.
+__device__ __forceinline__ int round_tile(int rd, int pair, int npairs) {
+    return rd * npairs + ((rd & 1) ? npairs - 1 - pair : pair);
+}
+
 // K slabs of pair tile t: nslab, or in mode 0 with ktri set, only the slabs up to the end
 // of the tile's 256 columns (ktri = 1: B rows c vanish beyond column c of K) or of its 256
 // rows (ktri = 2: A rows r vanish beyond column r of K). The same for both CTAs of a pair.
@@ -469,7 +478,9 @@ trail_pair_kernel(const __grid_constant__ CUtensorMap mAh, const __grid_constant
         if (lane == 0) {
             int k = 0;
             bool ok = true;
-            for (int t = pair; t < n_tiles && ok; t += npairs) {
+            for (int rd = 0; rd * npairs < n_tiles && ok; ++rd) {
+                const int t = round_tile(rd, pair, npairs);
+                if (t >= n_tiles) continue;
                 const PairTile pt = pair_tile_at(ts, t, static_cast<int>(rank));
                 const CUtensorMap* bh = pt.alt ? &mB2h : &mBh;
                 const CUtensorMap* bl = pt.alt ? &mB2l : &mBl;
@@ -502,7 +513,9 @@ trail_pair_kernel(const __grid_constant__ CUtensorMap mAh, const __grid_constant
                 constexpr uint32_t idesc = idesc_tf32_k_major(2 * TBM, PBN);
                 int k = 0, cc = 0;
                 bool ok = true;
-                for (int t = pair; t < n_tiles && ok; t += npairs) {
+                for (int rd = 0; rd * npairs < n_tiles && ok; ++rd) {
+                    const int t = round_tile(rd, pair, npairs);
+                    if (t >= n_tiles) continue;
                     const int ns = pair_tile_nslab(ts, t, nslab);
                     for (int s0 = 0; s0 < ns && ok; s0 += drain, ++cc) {
                         const int buf = cc & 1;
@@ -559,7 +572,9 @@ trail_pair_kernel(const __grid_constant__ CUtensorMap mAh, const __grid_constant
         uint8_t* stg = wtile + h * P_WBOX;
         int cc = 0;
         bool ok = true;
-        for (int t = pair; t < n_tiles && ok; t += npairs) {
+        for (int rd = 0; rd * npairs < n_tiles && ok; ++rd) {
+            const int t = round_tile(rd, pair, npairs);
+            if (t >= n_tiles) continue;
             const PairTile pt = pair_tile_at(ts, t, static_cast<int>(rank));
             const CUtensorMap* wm = pt.alt ? &mW2 : &mW;
             const int xh = pt.co + h * HALF;
