@@ -270,9 +270,11 @@ KQ_API kq_status kq_rotate_out(float* W, int64_t d_out, int64_t d_in, float* H_G
  *   and positive diagonal; the strict upper triangle of Lt is written with zeros. R = L^T
  *   is the upper factor whose row j drives the OBS update of column j. Computed as the
  *   Cholesky factorization of the index-reversed matrix with its triangular inverse formed in
- *   the same sweep (2 n^3 / 3 flops): fp32 on the diagonal blocks and panels, the trailing
- *   updates on the tensor cores with the 3xTF32 split (fp32-accurate products, fp32 sums),
- *   grouped into K = 1024 updates beyond each 1024-column super-panel when n > 1024.
+ *   the same sweep (2 n^3 / 3 flops): fp32 on the diagonal blocks, the products on the tensor
+ *   cores with the 3xTF32 split (fp32-accurate products, fp32 sums). When n > 1024 the
+ *   128-column steps of each 1024-column super-panel stay inside its diagonal block, its
+ *   panel below and its rows of the inverse to the left come from two products with that
+ *   block's inverse, and the tiles beyond take one K = 1024 update per super-panel.
  *   On a non-positive pivot, *info (required for that report) receives the 1-based index
  *   (in H's own indexing) of the failing pivot; Lt is then undefined. The caller may retry
  *   with a larger damp_rel.
@@ -289,9 +291,8 @@ KQ_API kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, float* L
  *   device allocation, or a latency-bound loop where a cudaMalloc would synchronize the
  *   device. The paper has no counterpart; this is a convenience of this library.
  *   Scratch comes from a fixed array in device memory that the library owns:
- *   KQ_CHOL_NOALLOC_SCRATCH_BYTES = (2 N^2 + 4 N 128) * 4 + 256 bytes with
- *   N = KQ_CHOL_NOALLOC_MAX_N (the padded matrix and its inverse factor, plus one set of
- *   four N x 128 tf32 split panels): 10 MiB + 256 bytes, held by every device that loads
+ *   KQ_CHOL_NOALLOC_SCRATCH_BYTES = 2 N^2 * 4 + 256 bytes with N = KQ_CHOL_NOALLOC_MAX_N
+ *   (the padded matrix and its inverse factor): 8 MiB + 256 bytes, held by every device that loads
  *   the library until the process exits. n > KQ_CHOL_NOALLOC_MAX_N is rejected with
  *   KQ_ERR_WORKSPACE and a message; no allocation is ever made.
  *   The first call on each device looks up the array's device address (cudaGetSymbolAddress,
@@ -301,7 +302,7 @@ KQ_API kq_status kq_chol_inv(const float* H, int64_t n, float damp_rel, float* L
  *   on different streams, or from different host threads -- race: serialize them.
  */
 #define KQ_CHOL_NOALLOC_MAX_N 1024
-#define KQ_CHOL_NOALLOC_SCRATCH_BYTES ((2ull * 1024 * 1024 + 4ull * 1024 * 128) * 4 + 256)
+#define KQ_CHOL_NOALLOC_SCRATCH_BYTES ((2ull * 1024 * 1024) * 4 + 256)
 KQ_API kq_status kq_chol_inv_noalloc(const float* H, int64_t n, float damp_rel, float* Lt, int* info,
                                      kq_stream_t stream);
 

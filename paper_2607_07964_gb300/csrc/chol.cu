@@ -56,10 +56,11 @@ struct Work {
 
 inline size_t npad_of(int64_t n) { return static_cast<size_t>(cdiv(n, NB) * NB); }
 
-// Split panel width and number of sets: one 128-column slice when one super-panel covers
-// the matrix, else two sets of a super-panel's width.
-constexpr size_t split_width(size_t np) { return np / NB > static_cast<size_t>(SPB) ? static_cast<size_t>(SPB) * NB : NB; }
-constexpr size_t split_sets(size_t np) { return np / NB > static_cast<size_t>(SPB) ? 2 : 1; }
+// Split operand width and number of sets: two sets of a super-panel's width when the matrix
+// takes more than one super-panel; none otherwise (the one-level schedule multiplies on the
+// strip kernels, which split their operands as they load them).
+constexpr size_t split_width(size_t) { return static_cast<size_t>(SPB) * NB; }
+constexpr size_t split_sets(size_t np) { return np / NB > static_cast<size_t>(SPB) ? 2 : 0; }
 constexpr size_t ws_bytes_for(size_t np) {
     return (2 * np * np + split_sets(np) * 4 * np * split_width(np)) * sizeof(float) + 256;
 }
