@@ -14,24 +14,27 @@
 // where B (stored in Z's blocks) is the right-hand side I of C Z = I after the earlier
 // steps' eliminations. The matrix is padded to a multiple of nb with an identity block.
 // Look-ahead: the update is split into the tiles step k + 1 reads first (row and column
-// block k + 1, on the caller's stream, on the critical path) and the rest (on a library
-// side stream, beside step k + 1's diagonal factorization and panel); step k + 1's own
-// first tiles wait for that rest, which also writes them.
-// The diagonal kernel is fp32 SIMT with fused multiply-add; the panel and first-tile
-// kernels multiply on the tensor cores (mma.sync tf32 with the 3xTF32 split). The
-// rest of each update (the bulk of the 2 n^3 / 3 flops) runs on the tensor cores with the
-// 3xTF32 split (trail_tc.cu, Cholesky mode): chol_split_kernel writes the tf32 hi / lo of
-// the panel C_{.k} and of Z_{k.} transposed (the K-major operands), then the persistent
-// tensor-core kernel updates the tiles in place (TMA load, subtract, TMA store).
-// Two levels when n > 8 NB: steps are grouped in super-panels of 8 blocks. Inside a
-// super-panel the per-step update touches only its block columns (all rows below) and its
-// block rows of Z; the tiles beyond get the whole super-panel's update at once (K = 8 NB):
-// first the next super-panel's columns and rows (on the caller's stream: the next steps
-// read them), the remaining ones on a second library stream beside the next super-panel.
-// The trailing matrix is then read and written once per super-panel rather than once per
-// step (at n = 28672, ~90 GB of HBM traffic instead of ~700 GB), and the K = 1024 products
-// keep the tensor cores busy. The split sets alternate between super-panels, so a
-// super-panel's split does not overwrite the operands the previous remote update reads.
+// block k + 1; the next diagonal tile alone on the caller's stream, the rest on a library
+// side stream) and the rest of the step's tiles (side stream, beside step k + 1's diagonal
+// factorization and panel). The diagonal kernel is fp32 SIMT with fused multiply-add; the
+// panel and the tile updates multiply on the tensor cores (mma.sync tf32 with the 3xTF32
+// split, operands split as they are loaded).
+// Two levels when n > 8 NB: steps are grouped in super-panels S of 8 blocks (D: the rows
+// below S, P: the columns left of it). The steps of S touch only S's diagonal block (A's
+// lower tiles and B's tiles in rows and columns S), so they stay small kernels. S's panel
+// below and its rows of Z to the left then follow from the inverse of its diagonal block,
+// Z_SS = C_SS^-1, which those steps built: with A' and B' as the earlier super-panels left
+// them, A'_DS = C_DS C_SS^T (the Schur complement's block) and C_SS Z_SP = B'_SP (forward
+// substitution), so C_DS = A'_DS Z_SS^T and Z_SP = Z_SS B'_SP, two K = 8 NB products on the
+// tensor cores (3xTF32, trail_tc.cu's two-CTA kernel, each tile's K bounded by the
+// triangle of Z_SS). Every tile beyond S then takes the whole super-panel's update at once
+// (K = 8 NB): the next super-panel's diagonal block first, on the caller's stream (the next
+// steps read only it), every other tile on a second library stream beside the next
+// super-panel's steps, leaving them a few SMs. The products and the update read tf32 hi / lo
+// splits of their operands (split_block_kernel); the split sets alternate between
+// super-panels, so a super-panel's splits do not overwrite the operands the previous
+// super-panel's update reads. The trailing matrix is read and written once per super-panel
+// rather than once per step (at n = 28672, ~90 GB of HBM traffic instead of ~700 GB).
 #include <math.h>
 
 #include <cstdlib>
