@@ -798,10 +798,11 @@ int long_drain_slabs() {
     return n;
 }
 
-// Persistent: as many clusters as can be resident at once walk the tiles. One cluster per
-// tile (so that finished clusters hand their SMs to the critical-path kernels of the
-// higher-priority stream) measured slower on the 70B down_proj layer: Cholesky 84.5 against
-// 74.6 ms, sweep 37.9 against 34.2 ms.
+// Persistent: as many clusters as can be resident at once walk the tiles, less free_sms / 2
+// (SMs left to kernels that run beside the launch, such as the next super-panel's steps of
+// the inverse Cholesky). One cluster per tile (so that finished clusters hand their SMs to
+// the critical-path kernels of the higher-priority stream) measured slower on the 70B
+// down_proj layer: Cholesky 84.5 against 74.6 ms, sweep 37.9 against 34.2 ms.
 kq_status launch_pair(const CUtensorMap& ah, const CUtensorMap& al, const CUtensorMap& bh, const CUtensorMap& bl,
                       const CUtensorMap& b2h, const CUtensorMap& b2l, const CUtensorMap& w, const CUtensorMap& w2,
                       const TileSet& ts, int nslab, int drain, int* info, cudaStream_t stream, int free_sms = 0) {
