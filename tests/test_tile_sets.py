@@ -44,7 +44,7 @@ def pair_mode1_blocks(nbk, a_j0, a_j1, a_r0, a_r1, b_i0, b_i1, b_j1):
     return out
 
 
-@pytest.mark.parametrize("nbk", [10, 11, 17, 32, 64, 224, 225])
+@pytest.mark.parametrize("nbk", [9, 10, 11, 12, 17, 32, 64, 224, 225])
 def test_far_update_parts_cover_every_block_once(nbk):
     """The next diagonal block's part (caller's stream) and the rest (second stream) of a
     super-panel's update write the lower blocks of A right of the super-panel and the blocks
@@ -175,7 +175,7 @@ def blocked_inverse_cholesky(H, nb, spb):
     return Z[:n, :n].T[::-1, ::-1]                            # L[i][j] = Z[n-1-j][n-1-i]
 
 
-@pytest.mark.parametrize("n,nb,spb", [(7, 4, 3), (24, 4, 3), (50, 4, 3), (100, 4, 8), (37, 4, 2), (200, 8, 4)])
+@pytest.mark.parametrize("n,nb,spb", [(7, 4, 3), (24, 4, 3), (50, 4, 3), (100, 4, 8), (36, 4, 8), (37, 4, 2), (200, 8, 4)])
 def test_blocked_schedule_gives_the_inverse_factor(n, nb, spb):
     rng = np.random.default_rng(n)
     X = rng.standard_normal((3 * n, n))
