@@ -236,6 +236,13 @@ def _shrink(cfg, f: int) -> int:
     return max(f, 1)
 
 
+def two_point_tokens(t1: float, t2: float, T_s: int, T: int) -> float:
+    """Time for T tokens from times t1, t2 on T_s and 2 T_s tokens: the line through both,
+    or t2 scaled by T / (2 T_s) when t2 <= t1 (no usable slope)."""
+    slope = (t2 - t1) / T_s
+    return t2 + (T - 2 * T_s) * slope if slope > 0 else t2 * T / (2 * T_s)
+
+
 def _oracle_stages(cfg, T_s: int, f: int, rows_s: int, alpha=None) -> dict:
     """One timed pass of every stage on its sample, each extrapolated to the full layer (ms)."""
     from oracle import kronq_oracle as ref
@@ -250,15 +257,19 @@ def _oracle_stages(cfg, T_s: int, f: int, rows_s: int, alpha=None) -> dict:
                                                                                    kqsynth.signs(cfg))))
     drift = alpha is not None
     per = {}
-    # the factors on T_s and on 2 T_s tokens: a d x d result costs the same at any T (its
-    # allocation and write), so the full layer is the two-point line through both times
+    # the factors on T_s and on 2 T_s tokens, after an untimed call that starts the library's
+    # threads: a d x d result costs the same at any T (its allocation and write), so the
+    # full layer is the two-point line through both times. Where the second time is not the
+    # larger (the fixed part varied between the calls by more than the tokens' part), the
+    # line has no usable slope and the larger sample is scaled in proportion to the tokens.
+    ref.accum_factor(L["G"][:min(64, T_s)])
     tf = []
     for Tk in (T_s, 2 * T_s):
         t0 = time.perf_counter()
         ref.accum_factor(L["X"][:Tk])
         ref.accum_factor(L["G"][:Tk])
         tf.append(time.perf_counter() - t0)
-    per["factors"] = tf[1] + (cfg.T - 2 * T_s) * (tf[1] - tf[0]) / T_s
+    per["factors"] = two_point_tokens(tf[0], tf[1], T_s, cfg.T)
     Ds = None
     if drift:
         Xt = kqsynth.fp_activations(cfg, L["X"])
